@@ -1,0 +1,162 @@
+"""ctypes front end of the fp64 CPU oracle (``oracle.cpp``).
+
+TEST INFRASTRUCTURE ONLY: imported by ``tests/``, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py``, never by the product package.  It shares no code
+with the CUDA library; the only common dependency is the seeded input generator
+(``synth``), which holds no attention arithmetic.
+
+Arrays are numpy: Q [B, Hq, Sq, D], K/V [B, Hkv, Skv, D] as uint16 bfloat16 bit
+patterns, results in float64.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.cpp")
+_LIB_DIR = os.path.join(_HERE, "_build")
+_LIB = os.path.join(_LIB_DIR, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+_u16p = np.ctypeslib.ndpointer(dtype=np.uint16, flags="C_CONTIGUOUS")
+_f64p = np.ctypeslib.ndpointer(dtype=np.float64, flags="C_CONTIGUOUS")
+
+
+def build(force: bool = False) -> str:
+    """Compile ``oracle.cpp`` into ``_build/liboracle.so`` (plain g++, no fast-math)."""
+    os.makedirs(_LIB_DIR, exist_ok=True)
+    stale = (not os.path.exists(_LIB)) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC)
+    if force or stale:
+        tmp = _LIB + f".tmp{os.getpid()}"
+        cmd = ["g++", "-O2", "-std=c++17", "-shared", "-fPIC", "-pthread", "-o", tmp, _SRC]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _bind(path: str):
+    """Open a compiled oracle library and declare its C signatures."""
+    lib = ctypes.CDLL(path)
+    i32, i64, dbl = ctypes.c_int, ctypes.c_int64, ctypes.c_double
+    vp = ctypes.c_void_p
+    lib.oracle_attention.argtypes = [_u16p, _u16p, _u16p, i32, i32, i32, i32, i32, i32,
+                                     i32, dbl, vp, vp, i64, _f64p, _f64p, i32]
+    lib.oracle_attention.restype = i32
+    lib.oracle_decode_split_merge.argtypes = [_u16p, _u16p, _u16p, i32, i32, i32, i32, i32,
+                                              dbl, vp, i32, i32, vp, vp, _f64p, _f64p, i32]
+    lib.oracle_decode_split_merge.restype = i32
+    lib.oracle_attention_naive.argtypes = [_u16p, _u16p, _u16p, i32, i32, i32, i32, i32,
+                                           i32, i32, dbl, _f64p, _f64p]
+    lib.oracle_attention_naive.restype = i32
+    lib.oracle_decode_chunk.argtypes = [i64, i32, i32]
+    lib.oracle_decode_chunk.restype = i64
+    return lib
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            _lib = _bind(build())
+    return _lib
+
+
+def _shapes(q, k, v):
+    if q.ndim != 4 or k.ndim != 4 or v.shape != k.shape:
+        raise ValueError("expected Q [B,Hq,Sq,D] and K/V [B,Hkv,Skv,D]")
+    B, Hq, Sq, D = q.shape
+    Bk, Hkv, Skv, Dk = k.shape
+    if Bk != B or Dk != D:
+        raise ValueError("batch or head-dim mismatch between Q and K/V")
+    return B, Hq, Hkv, Sq, Skv, D
+
+
+def _u16(a):
+    return np.ascontiguousarray(a, dtype=np.uint16)
+
+
+def attention(q, k, v, *, causal=False, scale=None, seqlens_k=None, rows=None, nthreads=0):
+    """Attention by definition in fp64.
+
+    ``rows`` optionally lists flat row indices ``(b*Hq + h)*Sq + i``; the result then
+    holds only those rows.  Returns ``(o, lse)``: o [B,Hq,Sq,D] (or [nrows, D]) and
+    lse [B,Hq,Sq] (or [nrows]).
+    """
+    q, k, v = _u16(q), _u16(k), _u16(v)
+    B, Hq, Hkv, Sq, Skv, D = _shapes(q, k, v)
+    if scale is None:
+        scale = 1.0 / np.sqrt(D)
+    sl = None if seqlens_k is None else np.ascontiguousarray(seqlens_k, dtype=np.int32)
+    if rows is None:
+        nrows = B * Hq * Sq
+        rp = None
+    else:
+        rows = np.ascontiguousarray(rows, dtype=np.int64)
+        nrows = rows.size
+        rp = rows.ctypes.data
+    o = np.zeros((max(nrows, 1), D), dtype=np.float64)
+    lse = np.zeros(max(nrows, 1), dtype=np.float64)
+    rc = _load().oracle_attention(q, k, v, B, Hq, Hkv, Sq, Skv, D, int(bool(causal)), float(scale),
+                                  None if sl is None else sl.ctypes.data, rp, nrows, o, lse,
+                                  int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle_attention rejected its arguments")
+    o, lse = o[:nrows], lse[:nrows]
+    if rows is None:
+        return o.reshape(B, Hq, Sq, D), lse.reshape(B, Hq, Sq)
+    return o, lse
+
+
+def decode_chunk(length: int, num_splits: int, chunk_align: int = 64) -> int:
+    """Chunk length of the Flash Decode split rule (see ``oracle.cpp``)."""
+    return int(_load().oracle_decode_chunk(int(length), int(num_splits), int(chunk_align)))
+
+
+def decode_split_merge(q, k, v, *, num_splits, scale=None, seqlens_k=None, chunk_align=64,
+                       nthreads=0):
+    """Flash Decode in fp64: per-split partials then the log-sum-exp merge.
+
+    q [B,Hq,1,D].  Returns ``(o [B,Hq,D], lse [B,Hq], o_part [B,Hq,S,D], lse_part [B,Hq,S])``.
+    """
+    q, k, v = _u16(q), _u16(k), _u16(v)
+    B, Hq, Hkv, Sq, Skv, D = _shapes(q, k, v)
+    if Sq != 1:
+        raise ValueError("decode takes Sq == 1")
+    if scale is None:
+        scale = 1.0 / np.sqrt(D)
+    sl = None if seqlens_k is None else np.ascontiguousarray(seqlens_k, dtype=np.int32)
+    o = np.zeros((B * Hq, D), dtype=np.float64)
+    lse = np.zeros(max(B * Hq, 1), dtype=np.float64)
+    o_part = np.zeros((B * Hq * num_splits, D), dtype=np.float64)
+    lse_part = np.zeros(max(B * Hq * num_splits, 1), dtype=np.float64)
+    rc = _load().oracle_decode_split_merge(q, k, v, B, Hq, Hkv, Skv, D, float(scale),
+                                           None if sl is None else sl.ctypes.data,
+                                           int(num_splits), int(chunk_align),
+                                           o_part.ctypes.data, lse_part.ctypes.data, o, lse,
+                                           int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle_decode_split_merge rejected its arguments")
+    return (o.reshape(B, Hq, D), lse[:B * Hq].reshape(B, Hq),
+            o_part.reshape(B, Hq, num_splits, D), lse_part[:B * Hq * num_splits].reshape(B, Hq, num_splits))
+
+
+def attention_naive(q, k, v, *, causal=False, scale=None):
+    """Long-double naive attention (no max subtraction); tiny inputs only."""
+    q, k, v = _u16(q), _u16(k), _u16(v)
+    B, Hq, Hkv, Sq, Skv, D = _shapes(q, k, v)
+    if scale is None:
+        scale = 1.0 / np.sqrt(D)
+    o = np.zeros((max(B * Hq * Sq, 1), D), dtype=np.float64)
+    lse = np.zeros(max(B * Hq * Sq, 1), dtype=np.float64)
+    rc = _load().oracle_attention_naive(q, k, v, B, Hq, Hkv, Sq, Skv, D, int(bool(causal)),
+                                        float(scale), o, lse)
+    if rc != 0:
+        raise ValueError("oracle_attention_naive rejected its arguments")
+    n = B * Hq * Sq
+    return o[:n].reshape(B, Hq, Sq, D), lse[:n].reshape(B, Hq, Sq)
