@@ -1,0 +1,128 @@
+/*
+ * loom_attn.h -- C ABI of the GB300 (sm_103a) fused-attention library.
+ *
+ * The library computes scaled-dot-product attention
+ *
+ *     O = softmax(scale * Q K^T [+ causal mask]) V,   LSE = ln sum_j exp(scale * q . k_j)
+ *
+ * in the two forms the Loom paper evaluates: Flash Attention prefill (Sec. 3.2.2:
+ * "matrix multiplication, softmax, and value aggregation" fused in one kernel) and
+ * Flash Decode (Sec. 2.6 Flash Decode example and Sec. 3.2.3: the sequence axis is
+ * split across cores, each split runs a local softmax loop, and the partial results
+ * are gathered, globally softmaxed and finally scaled).
+ *
+ * Conventions shared by every entry point:
+ *   - Tensors are dense, contiguous, row-major device buffers:
+ *       Q, O   [B, Hq,  Sq,  D]  bfloat16
+ *       K, V   [B, Hkv, Skv, D]  bfloat16
+ *       LSE    [B, Hq,  Sq]      float32 (natural log)
+ *   - Grouped-query attention: query head h reads kv head h / (Hq / Hkv).
+ *   - Causal masking is bottom-right aligned: query i sees key j iff j <= i + (Skv - Sq).
+ *   - D must be 64 or 128; scale must be finite and > 0.
+ *   - Every device pointer must be 16-byte aligned.
+ *   - All calls are asynchronous on `stream` (a cudaStream_t passed as void*; NULL is
+ *     the legacy default stream).  The caller owns every buffer, including the decode
+ *     workspace; the library allocates no device memory.
+ *   - Argument errors are reported synchronously by the return value and nothing is
+ *     launched.  Launch failures return LOOM_ERR_CUDA.  A kernel that gives up on a
+ *     bounded internal wait sets a device error word, which loom_attn_check_error
+ *     reports as LOOM_ERR_TIMEOUT.
+ */
+#ifndef LOOM_ATTN_H_
+#define LOOM_ATTN_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  LOOM_OK = 0,
+  LOOM_ERR_INVALID_ARG = 1, /* null pointer, non-positive size, Hq % Hkv != 0, bad scale, ... */
+  LOOM_ERR_UNSUPPORTED = 2, /* D not in {64, 128}, too many splits, ... */
+  LOOM_ERR_MISALIGNED = 3,  /* a pointer is not 16-byte aligned */
+  LOOM_ERR_WORKSPACE = 4,   /* decode workspace missing or too small */
+  LOOM_ERR_CUDA = 5,        /* a CUDA runtime/driver call or kernel launch failed */
+  LOOM_ERR_TIMEOUT = 6      /* a kernel abandoned a bounded wait (reported by check_error) */
+} loom_status;
+
+/*
+ * Flash Attention forward (prefill), paper Sec. 3.2.2.
+ *   q      [B, Hq, Sq, D]  bf16, read
+ *   k, v   [B, Hkv, Skv, D] bf16, read
+ *   o      [B, Hq, Sq, D]  bf16, written
+ *   lse    [B, Hq, Sq]     fp32, written; may be NULL
+ *   causal 0 or 1 (bottom-right aligned; causal requires Sq <= Skv)
+ * Errors: INVALID_ARG (null q/k/v/o, any size <= 0, Hq % Hkv, causal with Sq > Skv,
+ * scale not finite or <= 0), UNSUPPORTED (D), MISALIGNED, CUDA.
+ */
+loom_status loom_attn_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B,
+                          int Hq, int Hkv, int Sq, int Skv, int D, int causal, float scale,
+                          void* stream);
+
+/*
+ * Number of KV splits the decode path uses for this problem when the caller passes
+ * num_splits = 0: the analytic model's choice (one wave of split CTAs over the GPU's
+ * SMs, Sec. 2.6 Eq. 8-9 restated for GB300).  Returns 0 on invalid sizes.
+ * Skv is the KV-cache capacity (the longest possible sequence).
+ */
+int loom_attn_decode_num_splits(int B, int Hq, int Hkv, int Skv, int D);
+
+/*
+ * Device workspace (bytes) that loom_attn_decode needs: the per-split partial outputs
+ * O_i [B, Hq, splits, D] fp32 and log-sum-exps lse_i [B, Hq, splits] fp32.  num_splits
+ * = 0 means the model's choice.  Returns 0 on invalid sizes.
+ */
+size_t loom_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int Skv, int D, int num_splits);
+
+/*
+ * Flash Decode (Sq = 1), paper Sec. 2.6 (Flash Decode HEG) and Sec. 3.2.3.
+ *   q          [B, Hq, 1, D]      bf16, read
+ *   k_cache,
+ *   v_cache    [B, Hkv, Skv, D]   bf16, read (Skv = cache capacity)
+ *   seqlens_k  [B] int32 on the device: valid length of each sequence, 0..Skv; NULL means
+ *              every sequence has Skv keys.  Lengths outside [0, Skv] are clamped.
+ *   o          [B, Hq, 1, D]      bf16, written
+ *   lse        [B, Hq]            fp32, written; may be NULL
+ *   workspace  device scratch of at least loom_attn_decode_workspace_bytes(...) bytes;
+ *              its contents on entry do not matter and are overwritten.
+ *   num_splits 0 = analytic model, otherwise 1..1024 splits of each sequence.
+ * Split i of sequence b covers keys [i*C, min((i+1)*C, len_b)), C = ceil(len_b/splits)
+ * rounded up to a multiple of 64; empty splits contribute nothing.  A sequence of
+ * length 0 yields O = 0 and LSE = -inf.
+ * Errors: INVALID_ARG, UNSUPPORTED, MISALIGNED, WORKSPACE, CUDA.
+ */
+loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_cache,
+                             const int32_t* seqlens_k, void* o, float* lse, void* workspace,
+                             size_t workspace_bytes, int B, int Hq, int Hkv, int Skv, int D,
+                             float scale, int num_splits, void* stream);
+
+/*
+ * Synchronises `stream`, then reads and clears the current device's error word.
+ * Returns LOOM_OK, LOOM_ERR_TIMEOUT if a kernel abandoned a bounded wait since the last
+ * check, or LOOM_ERR_CUDA if the synchronisation itself failed.
+ */
+loom_status loom_attn_check_error(void* stream);
+
+/* Static, human-readable name of a status code. */
+const char* loom_status_string(loom_status status);
+
+/*
+ * Test hooks (not needed for normal use).
+ * loom_debug_set_timeout_ns: upper bound, in nanoseconds of %globaltimer, on every
+ *   internal wait of the kernels (default 2e9).  0 restores the default.
+ * loom_debug_inject: 0 = off; 1 = the decode split kernel's loader skips the copy of
+ *   its second stage; 2 = the prefill kernel's loader skips its second K tile.  The
+ *   waits on the skipped data then expire, the kernel unwinds and the next
+ *   loom_attn_check_error returns LOOM_ERR_TIMEOUT.  Host-side switch; no fault.
+ */
+void loom_debug_set_timeout_ns(uint64_t ns);
+void loom_debug_inject(int mode);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LOOM_ATTN_H_ */

@@ -1,0 +1,219 @@
+"""GB300 fused attention (prefill + Flash Decode): thin Python binding of ``libloomattn.so``.
+
+Every function here only marshals arguments (tensor data pointers, sizes, the current
+CUDA stream) into the C ABI declared in ``include/loom_attn.h``; all computation runs
+in the library's CUDA kernels.  There is no fallback: if the compiled library is
+missing, every call raises.
+
+Two layers:
+
+* ``capi()`` returns the ``ctypes.CDLL`` with argument types declared -- the raw C ABI,
+  taking integer device pointers.
+* Functions with the C names (``loom_attn_fwd``, ``loom_attn_decode``, ...) that take
+  torch tensors, check their dtype/device/layout, and raise ``LoomError`` on a non-OK
+  status.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+__all__ = [
+    "LoomError", "capi", "library_path", "STATUS",
+    "loom_attn_fwd", "loom_attn_decode", "loom_attn_decode_workspace_bytes",
+    "loom_attn_decode_num_splits", "loom_attn_check_error", "loom_status_string",
+    "loom_debug_set_timeout_ns", "loom_debug_inject",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "libloomattn.so")
+_lock = threading.Lock()
+_lib = None
+
+STATUS = {
+    0: "LOOM_OK", 1: "LOOM_ERR_INVALID_ARG", 2: "LOOM_ERR_UNSUPPORTED", 3: "LOOM_ERR_MISALIGNED",
+    4: "LOOM_ERR_WORKSPACE", 5: "LOOM_ERR_CUDA", 6: "LOOM_ERR_TIMEOUT",
+}
+
+
+class LoomError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS.get(status, status)}")
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def capi() -> ctypes.CDLL:
+    """The compiled library with its C signatures declared (raises if it is missing)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(_LIB_PATH):
+                raise RuntimeError(
+                    f"{_LIB_PATH} is missing: build it with paper_2609_29219_gb300.build.build() "
+                    "(there is no fallback implementation)")
+            lib = ctypes.CDLL(_LIB_PATH)
+            vp, i32, f32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+            lib.loom_attn_fwd.argtypes = [vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, vp]
+            lib.loom_attn_fwd.restype = i32
+            lib.loom_attn_decode_num_splits.argtypes = [i32, i32, i32, i32, i32]
+            lib.loom_attn_decode_num_splits.restype = i32
+            lib.loom_attn_decode_workspace_bytes.argtypes = [i32, i32, i32, i32, i32, i32]
+            lib.loom_attn_decode_workspace_bytes.restype = sz
+            lib.loom_attn_decode.argtypes = [vp, vp, vp, vp, vp, vp, vp, sz, i32, i32, i32, i32, i32,
+                                             f32, i32, vp]
+            lib.loom_attn_decode.restype = i32
+            lib.loom_attn_check_error.argtypes = [vp]
+            lib.loom_attn_check_error.restype = i32
+            lib.loom_status_string.argtypes = [i32]
+            lib.loom_status_string.restype = ctypes.c_char_p
+            lib.loom_debug_set_timeout_ns.argtypes = [ctypes.c_uint64]
+            lib.loom_debug_set_timeout_ns.restype = None
+            lib.loom_debug_inject.argtypes = [i32]
+            lib.loom_debug_inject.restype = None
+            _lib = lib
+    return _lib
+
+
+# ------------------------------------------------------------------ marshalling helpers
+def _torch():
+    import torch
+    return torch
+
+
+def _dev_ptr(t, name, dtype=None, ndim=None):
+    torch = _torch()
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims, got shape {tuple(t.shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _stream_ptr(stream, device):
+    torch = _torch()
+    if stream is None:
+        stream = torch.cuda.current_stream(device)
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        raise LoomError(status, where)
+
+
+# ------------------------------------------------------------------ C-ABI functions
+def loom_attn_fwd(q, k, v, o=None, lse=None, *, causal=False, scale=None, stream=None,
+                  return_lse=False):
+    """Prefill attention.  q [B,Hq,Sq,D], k/v [B,Hkv,Skv,D] bf16 CUDA tensors.
+
+    Writes ``o`` ([B,Hq,Sq,D] bf16, allocated if None) and, if given (or
+    ``return_lse``), ``lse`` ([B,Hq,Sq] fp32).  Returns ``o`` or ``(o, lse)``.
+    """
+    torch = _torch()
+    bf16 = torch.bfloat16
+    qp = _dev_ptr(q, "q", bf16, 4)
+    kp = _dev_ptr(k, "k", bf16, 4)
+    vp_ = _dev_ptr(v, "v", bf16, 4)
+    B, Hq, Sq, D = q.shape
+    Bk, Hkv, Skv, Dk = k.shape
+    if tuple(v.shape) != tuple(k.shape) or Bk != B or Dk != D:
+        raise ValueError("q/k/v shapes disagree")
+    if o is None:
+        o = torch.empty_like(q)
+    if tuple(o.shape) != tuple(q.shape):
+        raise ValueError("o must have q's shape")
+    op = _dev_ptr(o, "o", bf16, 4)
+    if lse is None and return_lse:
+        lse = torch.empty((B, Hq, Sq), dtype=torch.float32, device=q.device)
+    lp = None
+    if lse is not None:
+        if tuple(lse.shape) != (B, Hq, Sq):
+            raise ValueError("lse must be [B, Hq, Sq]")
+        lp = _dev_ptr(lse, "lse", torch.float32)
+    if scale is None:
+        scale = D ** -0.5
+    st = capi().loom_attn_fwd(qp, kp, vp_, op, lp, B, Hq, Hkv, Sq, Skv, D, int(bool(causal)),
+                              float(scale), _stream_ptr(stream, q.device))
+    _check(st, "loom_attn_fwd")
+    return (o, lse) if (return_lse or lse is not None) else o
+
+
+def loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D) -> int:
+    return int(capi().loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D))
+
+
+def loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, num_splits=0) -> int:
+    return int(capi().loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, num_splits))
+
+
+def loom_attn_decode(q, k_cache, v_cache, seqlens_k=None, o=None, lse=None, workspace=None, *,
+                     scale=None, num_splits=0, stream=None, return_lse=False):
+    """Flash Decode.  q [B,Hq,1,D], k_cache/v_cache [B,Hkv,Skv,D] bf16, seqlens_k [B] int32.
+
+    ``workspace`` is a CUDA uint8 tensor of at least ``loom_attn_decode_workspace_bytes``
+    bytes (allocated here if None).  Returns ``o`` or ``(o, lse)``.
+    """
+    torch = _torch()
+    bf16 = torch.bfloat16
+    qp = _dev_ptr(q, "q", bf16, 4)
+    kp = _dev_ptr(k_cache, "k_cache", bf16, 4)
+    vp_ = _dev_ptr(v_cache, "v_cache", bf16, 4)
+    B, Hq, Sq, D = q.shape
+    Bk, Hkv, Skv, Dk = k_cache.shape
+    if Sq != 1 or tuple(v_cache.shape) != tuple(k_cache.shape) or Bk != B or Dk != D:
+        raise ValueError("decode takes q [B,Hq,1,D] and k/v caches [B,Hkv,Skv,D]")
+    sp = None
+    if seqlens_k is not None:
+        if tuple(seqlens_k.shape) != (B,):
+            raise ValueError("seqlens_k must be [B]")
+        sp = _dev_ptr(seqlens_k, "seqlens_k", torch.int32)
+    if o is None:
+        o = torch.empty_like(q)
+    op = _dev_ptr(o, "o", bf16, 4)
+    if lse is None and return_lse:
+        lse = torch.empty((B, Hq), dtype=torch.float32, device=q.device)
+    lp = None
+    if lse is not None:
+        if lse.numel() != B * Hq:
+            raise ValueError("lse must hold B*Hq values")
+        lp = _dev_ptr(lse, "lse", torch.float32)
+    need = loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, num_splits)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=q.device)
+    wp = _dev_ptr(workspace, "workspace")
+    if scale is None:
+        scale = D ** -0.5
+    st = capi().loom_attn_decode(qp, kp, vp_, sp, op, lp, wp, workspace.numel() * workspace.element_size(),
+                                 B, Hq, Hkv, Skv, D, float(scale), int(num_splits),
+                                 _stream_ptr(stream, q.device))
+    _check(st, "loom_attn_decode")
+    return (o, lse) if (return_lse or lse is not None) else o
+
+
+def loom_attn_check_error(stream=None, device=None):
+    """Synchronise and raise ``LoomError`` if a kernel abandoned a bounded wait."""
+    st = capi().loom_attn_check_error(_stream_ptr(stream, device))
+    _check(st, "loom_attn_check_error")
+
+
+def loom_status_string(status: int) -> str:
+    return capi().loom_status_string(int(status)).decode()
+
+
+def loom_debug_set_timeout_ns(ns: int):
+    capi().loom_debug_set_timeout_ns(int(ns))
+
+
+def loom_debug_inject(mode: int):
+    capi().loom_debug_inject(int(mode))

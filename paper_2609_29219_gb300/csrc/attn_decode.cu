@@ -1,0 +1,454 @@
+// Flash Decode for GB300: split-KV partial attention + log-sum-exp merge.
+//
+// Paper: Sec. 2.6 (the Flash Decode HEG is a sequential composition of a local
+// softmax loop, a gather of partial results, a global softmax and a final scaling) and
+// Sec. 3.2.3 (the sequence axis, the reduction axis, is split across cores).
+//
+// Kernel 1, decode_split_kernel -- one CTA per (split, kv head, head group, batch):
+//   * a loader warp streams the split's K and V rows with 1-D bulk copies
+//     (cp.async.bulk, 16 KB per tile) into an NSTAGE-deep shared-memory ring guarded by
+//     full/empty mbarriers, so that 2 CTAs x 3 stages x 32 KB are in flight per SM;
+//   * 8 compute warps each take T/8 tokens of every stage; they read K rows with
+//     128-bit shared loads, form the scores of all GT query heads of the kv head at
+//     once (fp32 FMA), reduce them across lanes with a transposing butterfly, run an
+//     online softmax in base 2 with a lazily rescaled running max, and accumulate P.V;
+//   * the 8 warps' states are merged in shared memory into the split's normalised
+//     partial O_i (fp32) and lse_i (natural log) in the workspace.
+// Kernel 2, decode_merge_kernel -- one CTA per (batch, query head): L = max_i lse_i,
+//   w_i = exp(lse_i - L), O = sum w_i O_i / sum w_i -> bf16, lse = L + ln sum w_i.
+//   It is launched with programmatic dependent launch so its launch overlaps the
+//   split kernel's tail.
+#include <cuda_bf16.h>
+
+#include <cmath>
+
+#include "kernels.h"
+#include "model.h"
+#include "ptx.cuh"
+
+namespace loom {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+// Lazy rescaling: the running max of a head is only moved when the new tile max
+// exceeds it by more than this many base-2 units; P stays <= 2^8, exact in fp32.
+constexpr float kRescaleThreshold = 8.0f;
+
+// Stage constants: the analytic model's choice for this head dimension.
+template <int D>
+struct DecodeCfg {
+  static constexpr model::DecodeStagePlan kPlan = model::decode_stage_plan(D);
+  static_assert(kPlan.feasible, "no feasible decode stage plan");
+  static constexpr int T = kPlan.tokens;           // tokens per stage
+  static constexpr int NSTAGE = kPlan.stages;
+  static constexpr int CTAS_PER_SM = kPlan.ctas_per_sm;
+  static constexpr int NCW = 8;                    // compute warps
+  static constexpr int THREADS = (NCW + 1) * 32;   // + loader warp
+  static constexpr int TW = T / NCW;               // tokens per warp per stage
+  static constexpr int KL = D / 8;                 // lanes per K row (8 dims = 16 B each)
+  static constexpr int TPR = 32 / KL;              // tokens per 128-bit load round
+  static constexpr int KROUNDS = TW / TPR;
+  static constexpr int VD = D / 32;                // dims per lane in the P.V phase
+  static constexpr uint32_t TILE_BYTES = T * D * 2;
+  static constexpr uint32_t STAGE_BYTES = 2 * TILE_BYTES;
+  static constexpr uint32_t RING_BYTES = NSTAGE * STAGE_BYTES;
+  static_assert(TW % TPR == 0, "whole 128-bit load rounds per warp");
+};
+
+template <int D, int GT>
+struct DecodeSmem {
+  using C = DecodeCfg<D>;
+  // ring first (16-byte aligned bulk-copy destinations), then the small arrays
+  static constexpr uint32_t P_OFF = C::RING_BYTES;                      // [NCW][TW][GT] f32
+  static constexpr uint32_t ALPHA_OFF = P_OFF + C::NCW * C::TW * GT * 4;  // [NCW][GT] f32
+  static constexpr uint32_t WM_OFF = ALPHA_OFF + C::NCW * GT * 4;       // [NCW][GT] f32
+  static constexpr uint32_t WL_OFF = WM_OFF + C::NCW * GT * 4;          // [NCW][GT] f32
+  static constexpr uint32_t BAR_OFF = ((WL_OFF + C::NCW * GT * 4) + 7) / 8 * 8;
+  static constexpr uint32_t ABORT_OFF = BAR_OFF + 2 * C::NSTAGE * 8;
+  static constexpr uint32_t BYTES = ABORT_OFF + 16;
+  // the cross-warp merge reuses the ring: [NCW][GT][D] f32
+  static_assert(C::NCW * GT * D * 4 <= C::RING_BYTES, "merge buffer must fit in the ring");
+};
+
+// Sum over the KL lanes of a K row of the GT per-head partial dot products.  Each
+// butterfly level halves the number of live values (the "transposing" levels) until
+// one is left, so lane l ends up holding the full sum for head head_of_lane(l).
+template <int KL, int GT>
+__device__ __forceinline__ float transpose_reduce(float (&acc)[GT], int lane) {
+  static_assert(GT <= KL, "more heads than lanes per row");
+#pragma unroll
+  for (int off = KL / 2, n = GT; off >= 1; off >>= 1) {
+    if (n > 1) {
+      const int half = n >> 1;
+      const bool upper = (lane & off) != 0;
+#pragma unroll
+      for (int i = 0; i < GT / 2; ++i) {
+        if (i < half) {
+          const float send = upper ? acc[i] : acc[i + half];
+          const float keep = upper ? acc[i + half] : acc[i];
+          acc[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+        }
+      }
+      n = half;
+    } else {
+      acc[0] += __shfl_xor_sync(0xffffffffu, acc[0], off);
+    }
+  }
+  return acc[0];
+}
+
+template <int KL, int GT>
+__device__ __forceinline__ int head_of_lane(int lane) {
+  int h = 0;
+#pragma unroll
+  for (int off = KL / 2, n = GT; off >= 1 && n > 1; off >>= 1, n >>= 1)
+    if (lane & off) h += n >> 1;
+  return h;
+}
+
+template <int D, int GT>
+__global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_SM)
+    decode_split_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
+                        const __nv_bfloat16* __restrict__ v, const int32_t* __restrict__ seqlens,
+                        float* __restrict__ o_part, float* __restrict__ lse_part, int Hq, int Hkv,
+                        int Skv, int splits, int n_groups, float c, KernelCtl ctl) {
+  using C = DecodeCfg<D>;
+  using L = DecodeSmem<D, GT>;
+  extern __shared__ __align__(128) uint8_t smem[];
+
+  // Let the merge grid launch as soon as every split CTA is resident.
+  asm volatile("griddepcontrol.launch_dependents;");
+
+  const int split = blockIdx.x;
+  const int hk = blockIdx.y / n_groups, grp = blockIdx.y % n_groups;
+  const int b = blockIdx.z;
+  const int G = Hq / Hkv;
+  const int h0 = hk * G + grp * GT;
+  const int nh = min(GT, G - grp * GT);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  int len = seqlens ? seqlens[b] : Skv;
+  len = max(0, min(len, Skv));
+  int chunk = (len + splits - 1) / splits;
+  chunk = (chunk + kDecodeChunkAlign - 1) / kDecodeChunkAlign * kDecodeChunkAlign;
+  const int t_begin = min(split * chunk, len);
+  const int t_end = min(t_begin + chunk, len);
+  const size_t row0 = (static_cast<size_t>(b) * Hq + h0) * splits + split;  // head h0's partial
+
+  if (t_begin >= t_end) {  // empty split: contributes nothing to the merge
+    for (int i = threadIdx.x; i < nh * D; i += blockDim.x)
+      o_part[(row0 + static_cast<size_t>(i / D) * splits) * D + i % D] = 0.f;
+    if (threadIdx.x < nh) lse_part[row0 + static_cast<size_t>(threadIdx.x) * splits] = -INFINITY;
+    return;
+  }
+  const int n_stages = (t_end - t_begin + C::T - 1) / C::T;
+
+  const uint32_t s_base = smem_u32(smem);
+  const uint32_t bar_full = s_base + L::BAR_OFF;
+  const uint32_t bar_empty = bar_full + C::NSTAGE * 8;
+  Abort ab{reinterpret_cast<volatile int*>(smem + L::ABORT_OFF)};
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSTAGE; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, C::NCW);
+    }
+    *ab.flag = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+
+  const size_t kv_row0 = (static_cast<size_t>(b) * Hkv + hk) * Skv;
+
+  if (warp == C::NCW) {
+    // ------------------------------------------------------------ loader warp
+    if (lane == 0) {
+      int issued = 0, skipped = -1;
+      for (int it = 0; it < n_stages; ++it) {
+        const int slot = it % C::NSTAGE, round = it / C::NSTAGE;
+        if (!mbar_wait(bar_empty + 8 * slot, (round & 1) ^ 1, ctl, ab)) break;
+        const int tok0 = t_begin + it * C::T;
+        const uint32_t bytes = static_cast<uint32_t>(min(C::T, t_end - tok0)) * D * 2;
+        issued = it + 1;
+        if (ctl.inject == 1 && it == 1) {  // test hook: never fill this stage
+          skipped = it;
+          continue;
+        }
+        const uint32_t dst = s_base + slot * C::STAGE_BYTES;
+        mbar_expect_tx(bar_full + 8 * slot, 2 * bytes);
+        bulk_g2s(dst, k + (kv_row0 + tok0) * D, bytes, bar_full + 8 * slot);
+        bulk_g2s(dst + C::TILE_BYTES, v + (kv_row0 + tok0) * D, bytes, bar_full + 8 * slot);
+      }
+      // Drain: never leave the CTA with copies still landing in its shared memory.
+      Abort no_abort{reinterpret_cast<volatile int*>(smem + L::ABORT_OFF + 4)};
+      *no_abort.flag = 0;
+      for (int it = max(0, issued - C::NSTAGE); it < issued; ++it) {
+        if (it == skipped) continue;
+        mbar_wait(bar_full + 8 * (it % C::NSTAGE), (it / C::NSTAGE) & 1, ctl, no_abort);
+      }
+    }
+    return;
+  }
+
+  // -------------------------------------------------------------- compute warps
+  const int kl = lane % C::KL;   // 16-byte column of the K row this lane reads
+  const int tg = lane / C::KL;   // token within a load round
+  const int hl = head_of_lane<C::KL, GT>(lane);
+  const bool primary = ((lane % C::KL) & (C::KL / GT - 1)) == 0;  // one lane per (token, head)
+
+  // q of the GT heads, pre-multiplied by scale*log2(e) so scores come out in base 2
+  float qf[GT][8];
+#pragma unroll
+  for (int h = 0; h < GT; ++h) {
+    if (h < nh) {
+      const uint4 raw = *reinterpret_cast<const uint4*>(
+          q + (static_cast<size_t>(b) * Hq + h0 + h) * D + kl * 8);
+      const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        qf[h][2 * i] = bf16lo(w[i]) * c;
+        qf[h][2 * i + 1] = bf16hi(w[i]) * c;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) qf[h][i] = 0.f;
+    }
+  }
+
+  float m_run = -INFINITY, l_run = 0.f;
+  float acc_o[GT][C::VD];
+#pragma unroll
+  for (int h = 0; h < GT; ++h)
+#pragma unroll
+    for (int d = 0; d < C::VD; ++d) acc_o[h][d] = 0.f;
+
+  float* ps = reinterpret_cast<float*>(smem + L::P_OFF) + warp * C::TW * GT;
+  float* alpha_s = reinterpret_cast<float*>(smem + L::ALPHA_OFF) + warp * GT;
+
+  for (int it = 0; it < n_stages; ++it) {
+    const int slot = it % C::NSTAGE;
+    if (!mbar_wait_warp(bar_full + 8 * slot, (it / C::NSTAGE) & 1, ctl, ab)) break;
+    const int ntok = min(C::T, t_end - (t_begin + it * C::T));
+    const uint8_t* ks = smem + slot * C::STAGE_BYTES;
+    const uint8_t* vs = ks + C::TILE_BYTES;
+
+    // scores of this warp's TW tokens, in base-2 units
+    float sc[C::KROUNDS];
+#pragma unroll
+    for (int r = 0; r < C::KROUNDS; ++r) {
+      const int tl = warp * C::TW + r * C::TPR + tg;
+      const uint4 raw = *reinterpret_cast<const uint4*>(ks + tl * (D * 2) + kl * 16);
+      const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+      float kf[8];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        kf[2 * i] = bf16lo(w[i]);
+        kf[2 * i + 1] = bf16hi(w[i]);
+      }
+      float acc[GT];
+#pragma unroll
+      for (int h = 0; h < GT; ++h) {
+        float s = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) s = fmaf(qf[h][i], kf[i], s);
+        acc[h] = s;
+      }
+      const float s = transpose_reduce<C::KL, GT>(acc, lane);
+      sc[r] = (tl < ntok) ? s : -INFINITY;
+    }
+
+    // online softmax (per head, over this warp's tokens)
+    float mx = sc[0];
+#pragma unroll
+    for (int r = 1; r < C::KROUNDS; ++r) mx = fmaxf(mx, sc[r]);
+#pragma unroll
+    for (int off = C::KL; off < 32; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    const float m_new = fmaxf(m_run, mx);
+    const bool need = m_new > m_run + kRescaleThreshold;
+    const float alpha = need ? ex2(m_run - m_new) : 1.f;
+    if (need) m_run = m_new;
+    const float ms = (m_run == -INFINITY) ? 0.f : m_run;
+    float psum = 0.f;
+    __syncwarp();
+#pragma unroll
+    for (int r = 0; r < C::KROUNDS; ++r) {
+      const float p = ex2(sc[r] - ms);
+      psum += p;
+      if (primary) ps[(r * C::TPR + tg) * GT + hl] = p;
+    }
+    l_run = l_run * alpha + psum;
+    if (primary && tg == 0) alpha_s[hl] = alpha;
+    __syncwarp();
+
+    if (__any_sync(0xffffffffu, need)) {
+#pragma unroll
+      for (int h = 0; h < GT; ++h) {
+        const float a = alpha_s[h];
+#pragma unroll
+        for (int d = 0; d < C::VD; ++d) acc_o[h][d] *= a;
+      }
+    }
+
+    // P.V over this warp's tokens; lane owns dims [lane*VD, lane*VD + VD)
+    const int nmine = min(C::TW, ntok - warp * C::TW);
+#pragma unroll 4
+    for (int tt = 0; tt < nmine; ++tt) {
+      const int tl = warp * C::TW + tt;
+      float vf[C::VD];
+      if constexpr (C::VD == 4) {
+        const uint2 raw = *reinterpret_cast<const uint2*>(vs + tl * (D * 2) + lane * 8);
+        vf[0] = bf16lo(raw.x);
+        vf[1] = bf16hi(raw.x);
+        vf[2] = bf16lo(raw.y);
+        vf[3] = bf16hi(raw.y);
+      } else {
+        const uint32_t raw = *reinterpret_cast<const uint32_t*>(vs + tl * (D * 2) + lane * 4);
+        vf[0] = bf16lo(raw);
+        vf[1] = bf16hi(raw);
+      }
+      float pv[GT];
+      if constexpr (GT % 4 == 0) {
+#pragma unroll
+        for (int h = 0; h < GT; h += 4) {
+          const float4 p4 = *reinterpret_cast<const float4*>(ps + tt * GT + h);
+          pv[h] = p4.x;
+          pv[h + 1] = p4.y;
+          pv[h + 2] = p4.z;
+          pv[h + 3] = p4.w;
+        }
+      } else {
+#pragma unroll
+        for (int h = 0; h < GT; ++h) pv[h] = ps[tt * GT + h];
+      }
+#pragma unroll
+      for (int h = 0; h < GT; ++h)
+#pragma unroll
+        for (int d = 0; d < C::VD; ++d) acc_o[h][d] = fmaf(pv[h], vf[d], acc_o[h][d]);
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar_empty + 8 * slot);
+  }
+
+  // ---------------------------------------------------------------- merge the 8 warps
+#pragma unroll
+  for (int off = C::KL; off < 32; off <<= 1) l_run += __shfl_xor_sync(0xffffffffu, l_run, off);
+  asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");  // ring no longer read
+  float* wm = reinterpret_cast<float*>(smem + L::WM_OFF);
+  float* wl = reinterpret_cast<float*>(smem + L::WL_OFF);
+  float* wo = reinterpret_cast<float*>(smem);  // [NCW][GT][D], reuses the ring
+  if (primary && tg == 0) {
+    wm[warp * GT + hl] = m_run;
+    wl[warp * GT + hl] = l_run;
+  }
+#pragma unroll
+  for (int h = 0; h < GT; ++h)
+#pragma unroll
+    for (int d = 0; d < C::VD; ++d) wo[(warp * GT + h) * D + lane * C::VD + d] = acc_o[h][d];
+  asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");
+
+  for (int idx = threadIdx.x; idx < nh * D; idx += C::NCW * 32) {
+    const int h = idx / D, d = idx % D;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < C::NCW; ++w) M = fmaxf(M, wm[w * GT + h]);
+    float lsum = 0.f, osum = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < C::NCW; ++w) {
+        const float a = ex2(wm[w * GT + h] - M);  // 0 for warps that saw no key
+        lsum = fmaf(a, wl[w * GT + h], lsum);
+        osum = fmaf(a, wo[(w * GT + h) * D + d], osum);
+      }
+    }
+    const size_t row = row0 + static_cast<size_t>(h) * splits;
+    const bool any = lsum > 0.f;
+    o_part[row * D + d] = any ? osum / lsum : 0.f;
+    if (d == 0) lse_part[row] = any ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(D) decode_merge_kernel(const float* __restrict__ o_part,
+                                                         const float* __restrict__ lse_part,
+                                                         __nv_bfloat16* __restrict__ o,
+                                                         float* __restrict__ lse, int splits) {
+  // Wait until the split kernel's partials are complete and visible.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const int bh = blockIdx.x, d = threadIdx.x;
+  const float* lp = lse_part + static_cast<size_t>(bh) * splits;
+  float M = -INFINITY;
+  for (int i = 0; i < splits; ++i) M = fmaxf(M, lp[i]);
+  float W = 0.f, acc = 0.f;
+  if (M != -INFINITY) {
+    const float* op = o_part + static_cast<size_t>(bh) * splits * D + d;
+    for (int i = 0; i < splits; ++i) {
+      const float w = ex2((lp[i] - M) * kLog2e);
+      W += w;
+      acc = fmaf(w, op[static_cast<size_t>(i) * D], acc);
+    }
+  }
+  const bool any = W > 0.f;
+  o[static_cast<size_t>(bh) * D + d] = __float2bfloat16_rn(any ? acc / W : 0.f);
+  if (lse && d == 0) lse[bh] = any ? M + log2f(W) * kLn2 : -INFINITY;
+}
+
+template <int D, int GT>
+cudaError_t launch_split(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  using C = DecodeCfg<D>;
+  constexpr uint32_t smem = DecodeSmem<D, GT>::BYTES;
+  static unsigned long long configured = 0;  // one bit per device
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (!(configured & (1ull << (dev & 63)))) {
+    cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D, GT>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    configured |= 1ull << (dev & 63);
+  }
+  const int G = a.Hq / a.Hkv;
+  const int n_groups = (G + GT - 1) / GT;
+  dim3 grid(a.splits, a.Hkv * n_groups, a.B);
+  decode_split_kernel<D, GT><<<grid, C::THREADS, smem, stream>>>(
+      static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.k),
+      static_cast<const __nv_bfloat16*>(a.v), a.seqlens, a.o_part, a.lse_part, a.Hq, a.Hkv, a.Skv,
+      a.splits, n_groups, a.scale * kLog2e, ctl);
+  return cudaGetLastError();
+}
+
+template <int D>
+cudaError_t launch_merge(const DecodeArgs& a, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.B * a.Hq);
+  cfg.blockDim = dim3(D);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decode_merge_kernel<D>, static_cast<const float*>(a.o_part),
+                            static_cast<const float*>(a.lse_part),
+                            static_cast<__nv_bfloat16*>(a.o), a.lse, a.splits);
+}
+
+template <int D>
+cudaError_t launch_decode_d(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  const int G = a.Hq / a.Hkv;
+  cudaError_t e;
+  if (G >= 8) e = launch_split<D, 8>(a, ctl, stream);
+  else if (G >= 4) e = launch_split<D, 4>(a, ctl, stream);
+  else if (G >= 2) e = launch_split<D, 2>(a, ctl, stream);
+  else e = launch_split<D, 1>(a, ctl, stream);
+  if (e != cudaSuccess) return e;
+  return launch_merge<D>(a, stream);
+}
+
+}  // namespace
+
+cudaError_t launch_decode(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  if (a.D == 128) return launch_decode_d<128>(a, ctl, stream);
+  return launch_decode_d<64>(a, ctl, stream);
+}
+
+}  // namespace loom

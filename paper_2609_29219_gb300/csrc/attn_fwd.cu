@@ -1,0 +1,438 @@
+// Flash Attention prefill for GB300 (sm_103a): TMA + mbarrier ring, tcgen05 MMAs with
+// TMEM accumulators, warp-specialised loader / MMA / softmax roles.
+//
+// Paper: Sec. 3.2.2 evaluates Flash Attention as fused "matrix multiplication, softmax,
+// and value aggregation"; the pipelining of its load, compute and store stages through
+// counted circular buffers is the virtual-buffer protocol of Sec. 2.3, and the tile and
+// stage constants come from the latency model of Sec. 2.6 (Eq. 6-9, see model.cpp).
+//
+// One CTA owns NQT = 2 query tiles of BM = 128 rows (tile 0 and tile 1) of one
+// (batch, query head) and walks the key/value sequence in tiles of BN = 128 rows:
+//
+//   warp 8 (loader, 1 thread)   Q0, Q1 once; then K_0, V_0, K_1, V_1, ... into an
+//                               NSLOT-deep ring of 128B-swizzled shared-memory slots
+//   warp 9 (MMA, 1 thread)      S_t = Q_t K_j^T          (SS MMA, fp32 in TMEM)
+//                               O_t += P_t V_j           (TS MMA: P read from TMEM)
+//                               issue order S0 S1 | PV0 S0' | PV1 S1' | ... so the
+//                               tensor pipe works on one tile while the other tile's
+//                               softmax runs
+//   warps 0-3 / 4-7 (softmax)   one thread per query row of tile 0 / tile 1: read the
+//                               S row from TMEM, mask, online softmax in base 2 with a
+//                               lazily moved running max, write P (bf16) back over S,
+//                               rescale O in TMEM on the rare max jumps, and finally
+//                               normalise O, store it (bf16) and the log-sum-exp.
+//
+// TMEM (512 columns): [0,128) S0/P0 | [128,256) S1/P1 | [256,256+D) O0 | [256+D, 256+2D) O1.
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include <cmath>
+#include <mutex>
+
+#include "kernels.h"
+#include "model.h"
+#include "ptx.cuh"
+
+namespace loom {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kRescaleThreshold = 8.0f;  // base-2 units; P <= 2^8 between rescales
+
+// Tile and stage constants: the analytic model's argmin for this head dimension.
+template <int D>
+struct FwdCfg {
+  static constexpr model::FwdPlan kPlan = model::fwd_plan(D);
+  static_assert(kPlan.feasible, "no feasible prefill schedule");
+  static constexpr int BM = kPlan.bm;         // rows per query tile (= TMEM lanes)
+  static constexpr int NQT = kPlan.q_tiles;   // query tiles per CTA
+  static constexpr int BN = kPlan.bn;         // keys per KV tile
+  static constexpr int NSLOT = kPlan.kv_slots;  // K/V ring slots
+  static_assert(BM == 128 && NQT == 2, "warp roles assume two 128-row query tiles");
+  static_assert(BN % 64 == 0 && BN <= 128, "softmax holds one S row of <= 128 fp32 in registers");
+  static_assert(kPlan.b_lm == 1 && NSLOT >= 4, "the loader runs ahead of the MMA by >= one tile");
+  static constexpr int THREADS = 320;               // 8 softmax warps + loader + MMA
+  static constexpr int BOX_COLS = 64;               // 128-byte swizzle atom = 64 bf16
+  static constexpr int NBOX = D / BOX_COLS;         // TMA boxes per row of a tile
+  static constexpr uint32_t Q_BOX_BYTES = BM * 128;
+  static constexpr uint32_t Q_TILE_BYTES = NBOX * Q_BOX_BYTES;
+  static constexpr uint32_t KV_BOX_BYTES = BN * 128;
+  static constexpr uint32_t SLOT_BYTES = NBOX * KV_BOX_BYTES;
+  static constexpr uint32_t Q_OFF = 0;
+  static constexpr uint32_t RING_OFF = NQT * Q_TILE_BYTES;
+  static constexpr uint32_t BAR_OFF = RING_OFF + NSLOT * SLOT_BYTES;
+  // barriers: q_full, full[NSLOT], empty[NSLOT], s_full[2], p_full[2], o_full[2], drain
+  static constexpr int NBAR = 1 + 2 * NSLOT + 7;
+  static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
+  static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
+  static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;  // + alignment slack
+  static constexpr uint32_t TMEM_COLS = 512;
+  static constexpr uint32_t S_COL = 0;        // + t * BN
+  static constexpr uint32_t O_COL = 2 * BN;   // + t * D
+  static_assert(BYTES <= 227 * 1024, "shared memory budget");
+  static_assert(O_COL + NQT * D <= TMEM_COLS, "TMEM budget");
+};
+
+struct FwdParams {
+  __nv_bfloat16* o;
+  float* lse;
+  int Hq, Hkv, Sq, Skv;
+  int n_pairs;   // query-tile pairs per (b, h)
+  int causal;
+  int heavy_first;
+  float c;       // scale * log2(e)
+  KernelCtl ctl;
+};
+
+template <int D>
+__global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
+    attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                    const __grid_constant__ CUtensorMap tm_v, const FwdParams p) {
+  using C = FwdCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  // 1024-byte alignment for the 128B-swizzled tiles
+  const uint32_t raw_base = smem_u32(smem_raw);
+  const uint32_t sbase = (raw_base + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (sbase - raw_base);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int BH = gridDim.x / p.n_pairs;
+  int pair, bh;
+  if (p.heavy_first) {  // causal: the longest (bottom) tile pairs of every head go first
+    pair = p.n_pairs - 1 - static_cast<int>(blockIdx.x) / BH;
+    bh = static_cast<int>(blockIdx.x) % BH;
+  } else {              // consecutive CTAs share K/V of one head in L2
+    pair = static_cast<int>(blockIdx.x) % p.n_pairs;
+    bh = static_cast<int>(blockIdx.x) / p.n_pairs;
+  }
+  const int h = bh % p.Hq, b = bh / p.Hq;
+  const int hk = h / (p.Hq / p.Hkv);
+  const int kv_z = b * p.Hkv + hk;
+  const int q0 = pair * (C::NQT * C::BM);
+  const int off = p.Skv - p.Sq;  // bottom-right causal offset
+  int n_kv = p.Skv;
+  if (p.causal) n_kv = min(p.Skv, q0 + C::NQT * C::BM + off);
+  const int n_tiles = (n_kv + C::BN - 1) / C::BN;
+
+  const uint32_t bar_q = sbase + C::BAR_OFF;
+  const uint32_t bar_full = bar_q + 8;
+  const uint32_t bar_empty = bar_full + 8 * C::NSLOT;
+  const uint32_t bar_s = bar_empty + 8 * C::NSLOT;  // [2]
+  const uint32_t bar_p = bar_s + 16;                 // [2]
+  const uint32_t bar_o = bar_p + 16;                 // [2]
+  const uint32_t bar_drain = bar_o + 16;
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::TMEM_PTR_OFF);
+  Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
+
+  if (threadIdx.x == 0) {
+    mbar_init(bar_q, 1);
+    for (int s = 0; s < C::NSLOT; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, 1);
+    }
+    for (int t = 0; t < 2; ++t) {
+      mbar_init(bar_s + 8 * t, 1);
+      mbar_init(bar_p + 8 * t, C::BM);
+      mbar_init(bar_o + 8 * t, 1);
+    }
+    mbar_init(bar_drain, 1);
+    *ab.flag = 0;
+    *(ab.flag + 1) = 0;
+    fence_barrier_init();
+  }
+  if (warp == 9) tmem_alloc(smem_u32(tmem_ptr), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_ptr;
+
+  if (warp == 8) {
+    // ------------------------------------------------------------------ loader
+    if (lane == 0) {
+      prefetch_tensormap(&tm_q);
+      prefetch_tensormap(&tm_k);
+      prefetch_tensormap(&tm_v);
+      const int q_z = b * p.Hq + h;
+      mbar_expect_tx(bar_q, C::NQT * C::Q_TILE_BYTES);
+      for (int t = 0; t < C::NQT; ++t)
+        for (int x = 0; x < C::NBOX; ++x)
+          tma_load_3d(sbase + C::Q_OFF + t * C::Q_TILE_BYTES + x * C::Q_BOX_BYTES, &tm_q,
+                      x * C::BOX_COLS, q0 + t * C::BM, q_z, bar_q);
+      int issued = 0, skipped = -1;
+      for (int pos = 0; pos < 2 * n_tiles; ++pos) {  // K_0, V_0, K_1, V_1, ...
+        const int slot = pos % C::NSLOT, round = pos / C::NSLOT;
+        if (!mbar_wait(bar_empty + 8 * slot, (round & 1) ^ 1, p.ctl, ab)) break;
+        issued = pos + 1;
+        if (p.ctl.inject == 2 && pos == 2) {  // test hook: never load K_1
+          skipped = pos;
+          continue;
+        }
+        const CUtensorMap* map = (pos & 1) ? &tm_v : &tm_k;
+        const int row = (pos >> 1) * C::BN;
+        mbar_expect_tx(bar_full + 8 * slot, C::SLOT_BYTES);
+        for (int x = 0; x < C::NBOX; ++x)
+          tma_load_3d(sbase + C::RING_OFF + slot * C::SLOT_BYTES + x * C::KV_BOX_BYTES, map,
+                      x * C::BOX_COLS, row, kv_z, bar_full + 8 * slot);
+      }
+      // drain copies still in flight before the CTA may exit
+      Abort no_abort{ab.flag + 1};
+      mbar_wait(bar_q, 0, p.ctl, no_abort);
+      for (int pos = max(0, issued - C::NSLOT); pos < issued; ++pos)
+        if (pos != skipped)
+          mbar_wait(bar_full + 8 * (pos % C::NSLOT), (pos / C::NSLOT) & 1, p.ctl, no_abort);
+    }
+  } else if (warp == 9) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16(C::BM, C::BN, 0, 0);  // Q, K both K-major
+      constexpr uint32_t idesc_pv = idesc_bf16(C::BM, D, 0, 1);     // P from TMEM, V MN-major
+      auto slot_addr = [&](int pos) { return sbase + C::RING_OFF + (pos % C::NSLOT) * C::SLOT_BYTES; };
+      auto wait_slot = [&](int pos) {
+        return mbar_wait(bar_full + 8 * (pos % C::NSLOT), (pos / C::NSLOT) & 1, p.ctl, ab);
+      };
+      auto issue_s = [&](int t, int kpos) {
+        const uint32_t qa = sbase + C::Q_OFF + t * C::Q_TILE_BYTES;
+        const uint32_t ka = slot_addr(kpos);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t koff = (kk / 4) * C::Q_BOX_BYTES + (kk % 4) * 32;
+          const uint32_t kvoff = (kk / 4) * C::KV_BOX_BYTES + (kk % 4) * 32;
+          mma_ss(tmem + C::S_COL + t * C::BN, sdesc_sw128(qa + koff, 16, 1024),
+                 sdesc_sw128(ka + kvoff, 16, 1024), idesc_s, kk > 0);
+        }
+      };
+      auto issue_pv = [&](int t, int vpos, bool acc) {
+        const uint32_t va = slot_addr(vpos);
+#pragma unroll
+        for (int kk = 0; kk < C::BN / 16; ++kk)
+          mma_ts(tmem + C::O_COL + t * D, tmem + C::S_COL + t * C::BN + kk * 8,
+                 sdesc_sw128(va + kk * 16 * 128, C::KV_BOX_BYTES, 1024), idesc_pv,
+                 (acc || kk > 0) ? 1u : 0u);
+      };
+      bool ok = mbar_wait(bar_q, 0, p.ctl, ab) && wait_slot(0);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, 0);
+        tc_commit(bar_s);
+        issue_s(1, 0);
+        tc_commit(bar_s + 8);
+        tc_commit(bar_empty + 8 * (0 % C::NSLOT));
+      }
+      for (int j = 0; ok && j < n_tiles; ++j) {
+        const int vpos = 2 * j + 1, kpos = 2 * j + 2;
+        const bool more = j + 1 < n_tiles;
+        ok = wait_slot(vpos) && mbar_wait(bar_p, j & 1, p.ctl, ab);
+        if (!ok) break;
+        tc_fence_after();
+        issue_pv(0, vpos, j > 0);
+        tc_commit(bar_o);
+        if (more) {
+          if (!(ok = wait_slot(kpos))) break;
+          tc_fence_after();
+          issue_s(0, kpos);
+          tc_commit(bar_s);
+        }
+        if (!(ok = mbar_wait(bar_p + 8, j & 1, p.ctl, ab))) break;
+        tc_fence_after();
+        issue_pv(1, vpos, j > 0);
+        tc_commit(bar_o + 8);
+        tc_commit(bar_empty + 8 * (vpos % C::NSLOT));
+        if (more) {
+          issue_s(1, kpos);
+          tc_commit(bar_s + 8);
+          tc_commit(bar_empty + 8 * (kpos % C::NSLOT));
+        }
+      }
+      // wait for every MMA issued above before TMEM may be released
+      Abort no_abort{ab.flag + 1};
+      tc_commit(bar_drain);
+      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+    }
+  } else {
+    // ------------------------------------------------------------------ softmax
+    const int t = warp >> 2;                        // query tile of this warpgroup
+    const int row_in_tile = (warp & 3) * 32 + lane;  // == TMEM lane
+    const int row = q0 + t * C::BM + row_in_tile;
+    const uint32_t lane_addr = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t s_tm = tmem + lane_addr + C::S_COL + t * C::BN;
+    const uint32_t o_tm = tmem + lane_addr + C::O_COL + t * D;
+    const uint32_t my_bar_s = bar_s + 8 * t, my_bar_p = bar_p + 8 * t, my_bar_o = bar_o + 8 * t;
+    const int limit = p.causal ? min(p.Skv, row + off + 1) : p.Skv;  // keys [0, limit) visible
+    const float c = p.c;
+
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < n_tiles; ++j) {
+      if (!(ok = mbar_wait_warp(my_bar_s, j & 1, p.ctl, ab))) break;
+      tc_fence_after();
+      uint32_t s[C::BN];
+#pragma unroll
+      for (int ch = 0; ch < C::BN / 32; ++ch) tmem_ld32(s_tm + ch * 32, s + ch * 32);
+      tmem_wait_ld();
+#pragma unroll
+      for (int ch = 0; ch < C::BN / 32; ++ch) reg_fence32(s + ch * 32);
+      const int kbase = j * C::BN;
+      if (kbase + C::BN > limit) {
+#pragma unroll
+        for (int i = 0; i < C::BN; ++i)
+          if (kbase + i >= limit) s[i] = __float_as_uint(-INFINITY);
+      }
+      float mx = __uint_as_float(s[0]);
+#pragma unroll
+      for (int i = 1; i < C::BN; ++i) mx = fmaxf(mx, __uint_as_float(s[i]));
+      const float m_new = fmaxf(m_run, mx * c);
+      const bool need = m_new > m_run + kRescaleThreshold;
+      const float alpha = need ? ex2(m_run - m_new) : 1.f;
+      if (need) m_run = m_new;
+      if (j > 0 && __any_sync(0xffffffffu, need)) {
+        // O_t must hold P_{j-1} V_{j-1} before it is rescaled
+        if (!(ok = mbar_wait_warp(my_bar_o, (j - 1) & 1, p.ctl, ab))) break;
+        tc_fence_after();
+#pragma unroll 1
+        for (int ch = 0; ch < D / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld32(o_tm + ch * 32, r);
+          tmem_wait_ld();
+          reg_fence32(r);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+          tmem_st32(o_tm + ch * 32, r);
+        }
+        tmem_wait_st();
+      }
+      const float ms = (m_run == -INFINITY) ? 0.f : m_run;
+      float rs = 0.f;
+      uint32_t pk[C::BN / 2];
+#pragma unroll
+      for (int i = 0; i < C::BN / 2; ++i) {
+        const float p0 = ex2(fmaf(__uint_as_float(s[2 * i]), c, -ms));
+        const float p1 = ex2(fmaf(__uint_as_float(s[2 * i + 1]), c, -ms));
+        rs += p0 + p1;
+        pk[i] = pack_bf16x2(p0, p1);
+      }
+#pragma unroll
+      for (int ch = 0; ch < C::BN / 64; ++ch) tmem_st32(s_tm + ch * 32, pk + ch * 32);
+      tmem_wait_st();
+      l_run = l_run * alpha + rs;
+      tc_fence_before();
+      mbar_arrive(my_bar_p);
+    }
+
+    // epilogue: O / l -> bf16 rows, LSE
+    if (ok && n_tiles > 0) ok = mbar_wait_warp(my_bar_o, (n_tiles - 1) & 1, p.ctl, ab);
+    if (ok) {
+      tc_fence_after();
+      const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
+      const bool store = row < p.Sq;
+      __nv_bfloat16* orow =
+          p.o + ((static_cast<size_t>(b) * p.Hq + h) * p.Sq + (store ? row : 0)) * D;
+#pragma unroll 1
+      for (int ch = 0; ch < D / 32; ++ch) {
+        uint32_t r[32];
+        tmem_ld32(o_tm + ch * 32, r);
+        tmem_wait_ld();
+        reg_fence32(r);
+        uint32_t w[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          w[i] = pack_bf16x2(__uint_as_float(r[2 * i]) * inv_l, __uint_as_float(r[2 * i + 1]) * inv_l);
+        if (store) {
+          uint4* dst = reinterpret_cast<uint4*>(orow + ch * 32);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) dst[i] = make_uint4(w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+        }
+      }
+      if (store && p.lse)
+        p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.Sq + row] =
+            l_run > 0.f ? (m_run + log2f(l_run)) * kLn2 : -INFINITY;
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------- host side
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult qres;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &qres) == cudaSuccess &&
+        qres == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+// 3-D view [planes, rows, D] of a [B, H, S, D] bf16 tensor with a 64 x box_rows box.
+bool make_map(CUtensorMap* map, const void* base, int D, int rows, int planes, int box_rows) {
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(rows),
+                        static_cast<cuuint64_t>(planes)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2,
+                           static_cast<cuuint64_t>(D) * 2 * static_cast<cuuint64_t>(rows)};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(box_rows), 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D>
+cudaError_t launch_fwd_d(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  using C = FwdCfg<D>;
+  CUtensorMap mq, mk, mv;
+  if (!make_map(&mq, a.q, D, a.Sq, a.B * a.Hq, C::BM) ||
+      !make_map(&mk, a.k, D, a.Skv, a.B * a.Hkv, C::BN) ||
+      !make_map(&mv, a.v, D, a.Skv, a.B * a.Hkv, C::BN))
+    return cudaErrorInvalidValue;
+  static unsigned long long configured = 0;  // one bit per device
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (!(configured & (1ull << (dev & 63)))) {
+    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         C::BYTES);
+    if (e != cudaSuccess) return e;
+    configured |= 1ull << (dev & 63);
+  }
+  FwdParams p;
+  p.o = static_cast<__nv_bfloat16*>(a.o);
+  p.lse = a.lse;
+  p.Hq = a.Hq;
+  p.Hkv = a.Hkv;
+  p.Sq = a.Sq;
+  p.Skv = a.Skv;
+  p.n_pairs = (a.Sq + C::NQT * C::BM - 1) / (C::NQT * C::BM);
+  p.causal = a.causal;
+  p.heavy_first = a.causal;
+  p.c = a.scale * kLog2e;
+  p.ctl = ctl;
+  const long long grid = static_cast<long long>(p.n_pairs) * a.B * a.Hq;
+  if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  attn_fwd_kernel<D><<<static_cast<unsigned>(grid), C::THREADS, C::BYTES, stream>>>(mq, mk, mv, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_fwd(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  if (a.D == 128) return launch_fwd_d<128>(a, ctl, stream);
+  return launch_fwd_d<64>(a, ctl, stream);
+}
+
+}  // namespace loom

@@ -1,0 +1,165 @@
+// C ABI of the library (declared in include/loom_attn.h): argument validation, the
+// device error word, the analytic model hook for the decode split count, and dispatch
+// to the kernels.  No device memory is allocated here: the error word is a
+// file-scope __device__ variable whose address is looked up once per device.
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "../../include/loom_attn.h"
+#include "kernels.h"
+#include "model.h"
+
+namespace loom {
+namespace {
+
+__device__ uint32_t g_error_word = 0;
+
+constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // 2 s
+uint64_t g_timeout_ns = kDefaultTimeoutNs;
+int g_inject = 0;
+
+constexpr int kMaxDevices = 64;
+uint32_t* g_err_ptr[kMaxDevices] = {};
+std::mutex g_err_mutex;
+
+// Device address of the error word on the current device (looked up once per device).
+uint32_t* error_word_ptr() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(g_err_mutex);
+  if (!g_err_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
+    g_err_ptr[dev] = static_cast<uint32_t*>(p);
+  }
+  return g_err_ptr[dev];
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int current_sm_count() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return sms;
+}
+
+bool make_ctl(KernelCtl* ctl) {
+  ctl->err = error_word_ptr();
+  ctl->timeout_ns = g_timeout_ns;
+  ctl->inject = g_inject;
+  return ctl->err != nullptr;
+}
+
+}  // namespace
+}  // namespace loom
+
+using namespace loom;
+
+extern "C" {
+
+const char* loom_status_string(loom_status s) {
+  switch (s) {
+    case LOOM_OK: return "LOOM_OK";
+    case LOOM_ERR_INVALID_ARG: return "LOOM_ERR_INVALID_ARG";
+    case LOOM_ERR_UNSUPPORTED: return "LOOM_ERR_UNSUPPORTED";
+    case LOOM_ERR_MISALIGNED: return "LOOM_ERR_MISALIGNED";
+    case LOOM_ERR_WORKSPACE: return "LOOM_ERR_WORKSPACE";
+    case LOOM_ERR_CUDA: return "LOOM_ERR_CUDA";
+    case LOOM_ERR_TIMEOUT: return "LOOM_ERR_TIMEOUT";
+  }
+  return "LOOM_ERR_UNKNOWN";
+}
+
+loom_status loom_attn_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B,
+                          int Hq, int Hkv, int Sq, int Skv, int D, int causal, float scale,
+                          void* stream) {
+  if (!q || !k || !v || !o) return LOOM_ERR_INVALID_ARG;
+  if (B <= 0 || Hq <= 0 || Hkv <= 0 || Sq <= 0 || Skv <= 0 || D <= 0) return LOOM_ERR_INVALID_ARG;
+  if (Hq % Hkv != 0) return LOOM_ERR_INVALID_ARG;
+  if (causal != 0 && causal != 1) return LOOM_ERR_INVALID_ARG;
+  if (causal && Sq > Skv) return LOOM_ERR_INVALID_ARG;
+  if (!std::isfinite(scale) || scale <= 0.f) return LOOM_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return LOOM_ERR_UNSUPPORTED;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o)) return LOOM_ERR_MISALIGNED;
+  if (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)) return LOOM_ERR_MISALIGNED;
+  // TMA views use 32-bit coordinates: rows and planes must fit
+  if (static_cast<long long>(B) * Hq > 0x7fffffff || static_cast<long long>(B) * Hkv > 0x7fffffff)
+    return LOOM_ERR_UNSUPPORTED;
+  KernelCtl ctl;
+  if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
+  FwdArgs a{q, k, v, o, lse, B, Hq, Hkv, Sq, Skv, D, causal, scale};
+  return launch_fwd(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
+                                                                               : LOOM_ERR_CUDA;
+}
+
+int loom_attn_decode_num_splits(int B, int Hq, int Hkv, int Skv, int D) {
+  if (B <= 0 || Hq <= 0 || Hkv <= 0 || Skv <= 0 || Hq % Hkv != 0) return 0;
+  if (D != 64 && D != 128) return 0;
+  int sms = current_sm_count();
+  if (sms <= 0) sms = model::kGb300.num_sms;
+  return model::choose_decode_splits(B, Hq, Hkv, Skv, D, sms).splits;
+}
+
+size_t loom_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int Skv, int D, int num_splits) {
+  if (num_splits == 0) num_splits = loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D);
+  if (num_splits <= 0 || num_splits > kMaxDecodeSplits) return 0;
+  if (B <= 0 || Hq <= 0 || (D != 64 && D != 128)) return 0;
+  return decode_workspace_bytes(B, Hq, D, num_splits);
+}
+
+loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_cache,
+                             const int32_t* seqlens_k, void* o, float* lse, void* workspace,
+                             size_t workspace_bytes, int B, int Hq, int Hkv, int Skv, int D,
+                             float scale, int num_splits, void* stream) {
+  if (!q || !k_cache || !v_cache || !o) return LOOM_ERR_INVALID_ARG;
+  if (B <= 0 || Hq <= 0 || Hkv <= 0 || Skv <= 0 || D <= 0) return LOOM_ERR_INVALID_ARG;
+  if (Hq % Hkv != 0) return LOOM_ERR_INVALID_ARG;
+  if (!std::isfinite(scale) || scale <= 0.f) return LOOM_ERR_INVALID_ARG;
+  if (num_splits < 0) return LOOM_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return LOOM_ERR_UNSUPPORTED;
+  if (num_splits > kMaxDecodeSplits) return LOOM_ERR_UNSUPPORTED;
+  if (static_cast<long long>(B) * Hq * (num_splits ? num_splits : 1) > 0x7fffffffLL ||
+      static_cast<long long>(B) > 65535)
+    return LOOM_ERR_UNSUPPORTED;
+  if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(o))
+    return LOOM_ERR_MISALIGNED;
+  if ((lse && (reinterpret_cast<uintptr_t>(lse) & 3u)) ||
+      (seqlens_k && (reinterpret_cast<uintptr_t>(seqlens_k) & 3u)))
+    return LOOM_ERR_MISALIGNED;
+  if (num_splits == 0) num_splits = loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D);
+  if (num_splits <= 0) return LOOM_ERR_INVALID_ARG;
+  const size_t need = decode_workspace_bytes(B, Hq, D, num_splits);
+  if (!workspace || workspace_bytes < need) return LOOM_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return LOOM_ERR_MISALIGNED;
+  KernelCtl ctl;
+  if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
+  const size_t rows = static_cast<size_t>(B) * Hq * num_splits;
+  float* o_part = static_cast<float*>(workspace);
+  float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
+                                             (rows * D * sizeof(float) + 255) / 256 * 256);
+  DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D,
+               num_splits, scale};
+  return launch_decode(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
+                                                                                 : LOOM_ERR_CUDA;
+}
+
+loom_status loom_attn_check_error(void* stream) {
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return LOOM_ERR_CUDA;
+  uint32_t* p = error_word_ptr();
+  if (!p) return LOOM_ERR_CUDA;
+  uint32_t word = 0;
+  if (cudaMemcpy(&word, p, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess) return LOOM_ERR_CUDA;
+  if (word) {
+    const uint32_t zero = 0;
+    if (cudaMemcpy(p, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return LOOM_ERR_CUDA;
+  }
+  return (word & kErrTimeout) ? LOOM_ERR_TIMEOUT : LOOM_OK;
+}
+
+void loom_debug_set_timeout_ns(uint64_t ns) { g_timeout_ns = ns ? ns : kDefaultTimeoutNs; }
+
+void loom_debug_inject(int mode) { g_inject = mode; }
+
+}  // extern "C"

@@ -1,0 +1,257 @@
+// Analytic schedule model: the paper's Hierarchical Execution Graph latency model
+// (Sec. 2.6, Eq. 5-7) and its constrained selection (Eq. 8-9), restated for one GB300
+// SM and evaluated by exhaustive enumeration over a small finite domain instead of a
+// CP-SAT solve.  Everything is constexpr: the kernels take their tile and stage
+// constants from `fwd_plan(D)` / `decode_stage_plan(D)` at compile time, and the host
+// picks the decode split count with `choose_decode_splits` at run time.
+//
+// Architecture description (Sec. 2.7): structural numbers are GB300 specifications;
+// throughput numbers are measurements on this GPU type (HBM copy bandwidth and dense
+// bf16 GEMM throughput measured with a STREAM-style copy and a cuBLAS GEMM).  Numbers
+// marked "assumed" are placeholders for per-architecture microbenchmarks.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+namespace loom {
+namespace model {
+
+struct ArchDesc {
+  // structural (specifications)
+  int num_sms;              // streaming multiprocessors
+  int smem_per_sm;          // bytes of shared memory per SM usable by CTAs
+  int smem_per_cta;         // bytes of dynamic shared memory one CTA may opt into
+  int tmem_cols;            // 32-bit TMEM columns per SM (x 128 lanes)
+  int regs_per_sm;          // 32-bit registers per SM
+  // performance (measured / assumed)
+  double sm_ghz;            // SM clock under sustained load (measured median)
+  double hbm_gbs;           // HBM copy bandwidth, GB/s (measured)
+  double mma_tflops;        // dense bf16 tensor throughput of the GPU (measured burst)
+  double l2_smem_gbs_sm;    // L2 -> shared memory bandwidth of one SM, GB/s (assumed)
+  double ex2_per_clk_sm;    // MUFU.EX2 results per clock per SM (assumed)
+  double fp32_per_clk_sm;   // fp32 FMA-pipe lane-ops per clock per SM (specification)
+  double mem_latency_ns;    // loaded HBM latency of a bulk copy (assumed)
+  double sync_ns;           // fixed per-iteration cost of an mbarrier/TMEM round trip (assumed)
+  double launch_ns;         // fixed cost of one dependent kernel launch (assumed)
+};
+
+inline constexpr ArchDesc kGb300 = {
+    152, 228 * 1024, 227 * 1024, 512, 65536,
+    1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0,
+};
+
+// ------------------------------------------------------------------ HEG composition
+// Eq. 6: latency of pipe(l, body, s) under the two-bit pipeline knob (b_lm, b_ms).
+constexpr double heg_pipe(double l, double m, double s, int b_lm, int b_ms) {
+  if (!b_lm && !b_ms) return l + m + s;
+  if (!b_lm && b_ms) return (l + m) > s ? (l + m) : s;
+  if (b_lm && !b_ms) return l > (m + s) ? l : (m + s);
+  double x = l > m ? l : m;
+  return x > s ? x : s;
+}
+// Eq. 7: for(i, g)
+constexpr double heg_for(double trips, double body) { return trips * body; }
+// Eq. 5: g1 ; g2
+constexpr double heg_seq(double a, double b) { return a + b; }
+
+constexpr double dmax(double a, double b) { return a > b ? a : b; }
+constexpr long long cdiv(long long a, long long b) { return (a + b - 1) / b; }
+
+// ------------------------------------------------------------------ prefill
+// Candidate x = (BN keys per tile, KV ring slots), knobs b = (b_lm, b_ms).  Fixed by the
+// kernel structure: BM = 128 query rows per tile (one per TMEM lane) and 2 query tiles
+// per CTA, whose softmax and MMA phases alternate on the tensor pipe.
+struct FwdPlan {
+  int bm, bn, q_tiles, kv_slots, b_lm, b_ms;
+  int smem_bytes, tmem_cols;
+  double t_load_ns, t_mma_ns, t_softmax_ns, t_iter_ns;  // one KV-tile iteration of one CTA
+  bool feasible;
+};
+
+// Primitive latencies of one KV-tile iteration of one CTA (ns).
+constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int bn, int slots, int b_lm, int b_ms) {
+  FwdPlan p{};
+  p.bm = 128;
+  p.q_tiles = 2;
+  p.bn = bn;
+  p.kv_slots = slots;
+  p.b_lm = b_lm;
+  p.b_ms = b_ms;
+  const double clk = a.sm_ghz;  // clocks per ns
+  // load stage: K_j and V_j tiles, mostly L2 hits (the CTAs of a head share them)
+  const double kv_bytes = 2.0 * bn * D * 2;
+  p.t_load_ns = kv_bytes / a.l2_smem_gbs_sm;  // GB/s == bytes/ns
+  // compute leaf: 2 GEMMs (S = Q K^T, O += P V) per query tile on the tensor pipe
+  const double flops = 2.0 * p.q_tiles * (2.0 * p.bm * bn * D);
+  const double f_sm = a.mma_tflops * 1e3 / a.num_sms;  // FLOP/ns per SM
+  p.t_mma_ns = flops / f_sm;
+  // softmax leaf: one ex2 per score on MUFU; ~5 FMA-pipe ops per score (scale/subtract,
+  // max, add, half a pack, mask/compare amortised) -- two tiles share the SM
+  const double scores = 1.0 * p.q_tiles * p.bm * bn;
+  const double t_ex2 = scores / (a.ex2_per_clk_sm * clk);
+  const double t_fma = scores * 5.0 / (a.fp32_per_clk_sm * clk);
+  p.t_softmax_ns = dmax(t_ex2, t_fma);
+  // body: with two query tiles the tensor pipe and the softmax warps overlap; each
+  // iteration still pays one S-ready / P-ready handshake that nothing hides
+  const double body = dmax(p.t_mma_ns, p.t_softmax_ns) + a.sync_ns;
+  // store stage of the iteration is empty (O is stored once per tile)
+  p.t_iter_ns = heg_pipe(p.t_load_ns, body, 0.0, b_lm, b_ms);
+  // resources (Eq. 8 constraints)
+  p.smem_bytes = p.q_tiles * p.bm * D * 2 + slots * bn * D * 2 + 1024 + 256;
+  p.tmem_cols = p.q_tiles * (bn + D);
+  p.feasible = true;
+  if (bn % 16 != 0 || bn < 16 || bn > 256) p.feasible = false;   // MMA N for M = 128
+  if (bn % 32 != 0 || bn > 128) p.feasible = false;              // softmax: <= 128 fp32 regs/row
+  if (D % 64 != 0) p.feasible = false;                            // 128 B swizzle atoms
+  if (p.smem_bytes > a.smem_per_cta) p.feasible = false;          // L1 footprint
+  if (p.tmem_cols > a.tmem_cols) p.feasible = false;
+  if (slots < 2) p.feasible = false;                              // K and V of one tile
+  // an open load boundary needs the next tile's K and V in flight while this tile's
+  // K and V are being read: >= 4 slots, and enough of them to cover the latency
+  if (b_lm && (slots < 4 || (slots / 2 - 1) * body < a.mem_latency_ns * 0.5)) p.feasible = false;
+  if (slots % 2 != 0) p.feasible = false;                         // K/V alternate in the ring
+  return p;
+}
+
+// Eq. 8-9 by enumeration: BN in {32, ..., 256}, slots in {2, ..., 16}, knobs in {0,1}^2.
+// Ties go to fewer slots (less shared memory), then smaller BN.
+constexpr FwdPlan fwd_plan(int D, const ArchDesc& a = kGb300) {
+  FwdPlan best{};
+  best.feasible = false;
+  for (int bn = 32; bn <= 256; bn += 16)
+    for (int slots = 2; slots <= 16; ++slots)
+      for (int b_lm = 0; b_lm <= 1; ++b_lm)
+        for (int b_ms = 0; b_ms <= 1; ++b_ms) {
+          FwdPlan p = fwd_eval(a, D, bn, slots, b_lm, b_ms);
+          if (!p.feasible) continue;
+          // per-key cost: iterations scale with 1 / BN
+          const double cost = p.t_iter_ns / bn;
+          const double best_cost = best.feasible ? best.t_iter_ns / best.bn : 1e300;
+          if (cost < best_cost * (1.0 - 1e-9)) best = p;
+        }
+  return best;
+}
+
+// Modeled time (us) of a whole prefill launch under a plan.
+constexpr double fwd_time_us(const FwdPlan& p, int B, int Hq, int Sq, int Skv, int D, int causal,
+                             const ArchDesc& a = kGb300) {
+  const long long rows_per_cta = 1LL * p.q_tiles * p.bm;
+  const long long pairs = cdiv(Sq, rows_per_cta);
+  const long long ctas = pairs * B * Hq;
+  // average KV tiles per CTA
+  double tiles = 0;
+  for (long long i = 0; i < pairs; ++i) {
+    long long n_kv = Skv;
+    if (causal) {
+      const long long lim = (i + 1) * rows_per_cta + (Skv - Sq);
+      n_kv = lim < Skv ? lim : Skv;
+    }
+    tiles += static_cast<double>(cdiv(n_kv, p.bn));
+  }
+  tiles /= static_cast<double>(pairs);
+  const double t_q = 2.0 * rows_per_cta * D * 2 / a.l2_smem_gbs_sm;
+  const double t_o = 1.0 * rows_per_cta * D * 2 / a.l2_smem_gbs_sm;
+  const double t_cta = heg_seq(heg_seq(t_q, heg_for(tiles, p.t_iter_ns)), t_o);
+  const double waves = static_cast<double>(ctas) / a.num_sms;  // fractional: LPT ordering
+  const double w = waves < 1.0 ? 1.0 : waves;
+  return w * t_cta * 1e-3;
+}
+
+// ------------------------------------------------------------------ decode
+// Stage plan of the split kernel: T keys per stage, NSTAGE ring depth, CTAs per SM.
+struct DecodeStagePlan {
+  int tokens, stages, ctas_per_sm;
+  int smem_bytes;
+  double t_stage_ns;      // one stage of one CTA at its share of HBM bandwidth
+  double bytes_in_flight_sm;
+  bool feasible;
+};
+
+constexpr DecodeStagePlan decode_stage_eval(const ArchDesc& a, int D, int tokens, int stages,
+                                            int ctas_per_sm) {
+  DecodeStagePlan p{};
+  p.tokens = tokens;
+  p.stages = stages;
+  p.ctas_per_sm = ctas_per_sm;
+  const double stage_bytes = 2.0 * tokens * D * 2;
+  p.smem_bytes = static_cast<int>(stages * stage_bytes) + 4096;
+  p.bytes_in_flight_sm = stage_bytes * (stages - 1) * ctas_per_sm;
+  const double bw_cta = a.hbm_gbs / (a.num_sms * ctas_per_sm);  // bytes/ns per CTA
+  const double l = stage_bytes / bw_cta;
+  p.t_stage_ns = heg_pipe(l, 0.0, 0.0, 1, 1);
+  // Little's law: enough bytes in flight per SM to cover the memory latency
+  const double need = a.hbm_gbs / a.num_sms * a.mem_latency_ns;
+  // while the compute warps read one stage, the other stages-1 are in flight
+  p.feasible = p.smem_bytes * ctas_per_sm <= a.smem_per_sm && p.smem_bytes <= a.smem_per_cta &&
+               stage_bytes * (stages - 1) * ctas_per_sm >= need && stages >= 2 &&
+               tokens % 64 == 0 && (tokens / 8) % (256 / D) == 0;
+  return p;
+}
+
+// Smallest footprint that keeps HBM saturated: among feasible (tokens, stages,
+// CTAs/SM), prefer 2 CTAs per SM (latency tolerance of the compute warps), then the
+// smallest ring.
+constexpr DecodeStagePlan decode_stage_plan(int D, const ArchDesc& a = kGb300) {
+  DecodeStagePlan best{};
+  best.feasible = false;
+  for (int ctas = 2; ctas >= 1; --ctas)
+    for (int tokens = 64; tokens <= 256; tokens += 64)
+      for (int stages = 2; stages <= 8; ++stages) {
+        DecodeStagePlan p = decode_stage_eval(a, D, tokens, stages, ctas);
+        if (!p.feasible) continue;
+        if (!best.feasible || p.ctas_per_sm > best.ctas_per_sm ||
+            (p.ctas_per_sm == best.ctas_per_sm && p.smem_bytes < best.smem_bytes))
+          best = p;
+      }
+  return best;
+}
+
+struct DecodeSplitPlan {
+  int splits;
+  double t_us;   // modeled split + merge time
+};
+
+// Number of q heads one split CTA serves (must match the kernel dispatch).
+constexpr int decode_group_tile(int G) { return G >= 8 ? 8 : G >= 4 ? 4 : G >= 2 ? 2 : 1; }
+
+// Eq. 5 for Flash Decode: T = T_split-loop ; T_merge (gather + global softmax + scale).
+// The split loop is Eq. 6-7 with an open load boundary (the ring keeps copies in
+// flight), so a CTA streams its chunk at its share of HBM bandwidth, capped by the
+// bytes it can keep in flight (Little's law); CTAs run in waves of num_sms * CTAs/SM.
+constexpr double decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms,
+                                const ArchDesc& a = kGb300) {
+  const DecodeStagePlan sp = decode_stage_plan(D, a);
+  const int G = Hq / Hkv;
+  const int gt = decode_group_tile(G);
+  const long long units = 1LL * B * Hkv * cdiv(G, gt);
+  const long long ctas = units * splits;
+  const long long slots = 1LL * num_sms * sp.ctas_per_sm;
+  const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
+  const double active = static_cast<double>(ctas < slots ? ctas : slots);
+  const double in_flight_cta = 2.0 * sp.tokens * D * 2 * (sp.stages - 1);
+  double bw_cta = a.hbm_gbs / active;                 // bytes/ns
+  const double cap = in_flight_cta / a.mem_latency_ns;
+  if (bw_cta > cap) bw_cta = cap;
+  const double stages = static_cast<double>(cdiv(chunk, sp.tokens));
+  const double t_cta = heg_seq(a.mem_latency_ns, heg_for(stages, 2.0 * sp.tokens * D * 2 / bw_cta));
+  const double waves = static_cast<double>(cdiv(ctas, slots));
+  const double t_split = waves * t_cta;
+  const double part_bytes = 1.0 * B * Hq * splits * (D + 1) * 4;
+  const double t_merge = a.launch_ns * 0.2 + 2.0 * part_bytes / a.hbm_gbs;
+  return heg_seq(t_split, t_merge) * 1e-3;
+}
+
+constexpr DecodeSplitPlan choose_decode_splits(int B, int Hq, int Hkv, int Skv, int D, int num_sms,
+                                               const ArchDesc& a = kGb300) {
+  DecodeSplitPlan best{1, 1e300};
+  const long long max_splits = cdiv(Skv, 64) < 1024 ? cdiv(Skv, 64) : 1024;
+  for (int s = 1; s <= max_splits; ++s) {
+    const double t = decode_time_us(s, B, Hq, Hkv, Skv, D, num_sms, a);
+    if (t < best.t_us * (1.0 - 1e-9)) best = {s, t};
+  }
+  return best;
+}
+
+}  // namespace model
+}  // namespace loom

@@ -1,0 +1,102 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds for sm_103a,
+loads, exports every function include/loom_attn.h declares, and rejects bad
+arguments before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "loom_attn.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_29219_gb300 import build
+    build.build()
+    import paper_2609_29219_gb300 as loom
+    return loom.capi()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(loom_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("loom_attn_fwd", "loom_attn_decode", "loom_attn_decode_workspace_bytes",
+                     "loom_attn_check_error", "loom_status_string"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, f"not exported: {missing}"
+
+
+def test_status_strings(lib):
+    import paper_2609_29219_gb300 as loom
+    for code, name in loom.STATUS.items():
+        assert loom.loom_status_string(code) == name
+
+
+FAKE = 0x10000  # aligned, never dereferenced: every call below is rejected during validation
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((0, FAKE, FAKE, FAKE, None, 1, 2, 2, 128, 128, 64, 0, 0.125), 1),     # null q
+    ((FAKE, FAKE, FAKE, FAKE, None, 0, 2, 2, 128, 128, 64, 0, 0.125), 1),  # B = 0
+    ((FAKE, FAKE, FAKE, FAKE, None, 1, 3, 2, 128, 128, 64, 0, 0.125), 1),  # Hq % Hkv
+    ((FAKE, FAKE, FAKE, FAKE, None, 1, 2, 2, 256, 128, 64, 1, 0.125), 1),  # causal Sq > Skv
+    ((FAKE, FAKE, FAKE, FAKE, None, 1, 2, 2, 128, 128, 64, 0, float("nan")), 1),
+    ((FAKE, FAKE, FAKE, FAKE, None, 1, 2, 2, 128, 128, 64, 0, 0.0), 1),
+    ((FAKE, FAKE, FAKE, FAKE, None, 1, 2, 2, 128, 128, 64, 2, 0.125), 1),  # causal not 0/1
+    ((FAKE, FAKE, FAKE, FAKE, None, 1, 2, 2, 128, 128, 96, 0, 0.125), 2),  # D unsupported
+    ((FAKE + 8, FAKE, FAKE, FAKE, None, 1, 2, 2, 128, 128, 64, 0, 0.125), 3),  # misaligned
+    ((FAKE, FAKE, FAKE, FAKE, FAKE + 2, 1, 2, 2, 128, 128, 64, 0, 0.125), 3),  # misaligned lse
+])
+def test_fwd_rejects_bad_arguments(lib, args, expect):
+    assert lib.loom_attn_fwd(*args, None) == expect
+
+
+def test_decode_rejects_bad_arguments(lib):
+    ok = (FAKE, FAKE, FAKE, None, FAKE, None, FAKE, 1 << 20, 2, 8, 2, 1024, 128, 0.08, 4, None)
+
+    def call(**kw):
+        names = ["q", "k", "v", "sl", "o", "lse", "ws", "wsb", "B", "Hq", "Hkv", "Skv", "D", "scale",
+                 "splits", "stream"]
+        a = dict(zip(names, ok))
+        a.update(kw)
+        return lib.loom_attn_decode(*[a[n] for n in names])
+
+    assert call(q=0) == 1
+    assert call(Hq=7) == 1
+    assert call(scale=-1.0) == 1
+    assert call(splits=-1) == 1
+    assert call(D=80) == 2
+    assert call(splits=5000) == 2
+    assert call(v=FAKE + 4) == 3
+    assert call(sl=FAKE + 2) == 3
+    assert call(ws=0) == 4
+    assert call(wsb=100) == 4
+
+
+def test_workspace_size_formula(lib):
+    # O_i [B,Hq,S,D] fp32 + lse_i [B,Hq,S] fp32, each padded to 256 bytes
+    B, Hq, D, S = 3, 8, 128, 7
+    rows = B * Hq * S
+    expect = (rows * D * 4 + 255) // 256 * 256 + (rows * 4 + 255) // 256 * 256
+    assert lib.loom_attn_decode_workspace_bytes(B, Hq, 2, 4096, D, S) == expect
+    assert lib.loom_attn_decode_workspace_bytes(B, Hq, 2, 4096, 96, S) == 0
+    assert lib.loom_attn_decode_workspace_bytes(B, Hq, 2, 4096, D, 2000) == 0
+
+
+def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
+    import paper_2609_29219_gb300 as loom
+    monkeypatch.setattr(loom, "_lib", None)
+    monkeypatch.setattr(loom, "_LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="no fallback"):
+        loom.capi()

@@ -1,0 +1,109 @@
+"""GPU parity of the Flash Decode kernels (split + merge, through the C ABI)."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from tests.gpu_util import assert_parity, o_to_f64, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def loom():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2609_29219_gb300 as m
+    return m
+
+
+def _inputs(seed, B, Hq, Hkv, Skv, D):
+    return (synth.bf16_normal(seed, synth.STREAM_Q, (B, Hq, 1, D)),
+            synth.bf16_normal(seed, synth.STREAM_K, (B, Hkv, Skv, D)),
+            synth.bf16_normal(seed, synth.STREAM_V, (B, Hkv, Skv, D)))
+
+
+def _run(loom, q, k, v, lens, num_splits, workspace=None):
+    import torch
+    sl = None if lens is None else torch.from_numpy(np.asarray(lens, np.int32)).cuda()
+    o, lse = loom.loom_attn_decode(to_dev(q), to_dev(k), to_dev(v), sl, num_splits=num_splits,
+                                   workspace=workspace, return_lse=True)
+    loom.loom_attn_check_error()
+    return o, lse
+
+
+def test_batched_decode_config(loom):
+    # B=16, Hq=32, Hkv=8, Skv=8192, lengths U[4096, 8192] (stream 3), D=128, 16 splits
+    B, Hq, Hkv, Skv, D = 16, 32, 8, 8192, 128
+    q, k, v = _inputs(0, B, Hq, Hkv, Skv, D)
+    lens = synth.decode_lengths(0, B, 4096, 8192)
+    o, lse = _run(loom, q, k, v, lens, 16)
+    o_ref, lse_ref = oracle.attention(q, k, v, seqlens_k=lens)
+    assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "batched decode")
+
+
+@pytest.mark.slow
+def test_long_context_decode_config(loom):
+    # B=1, Hq=32, Hkv=8, Skv=131072, D=128, model-chosen splits (>= one wave of CTAs)
+    B, Hq, Hkv, Skv, D = 1, 32, 8, 131072, 128
+    q, k, v = _inputs(0, B, Hq, Hkv, Skv, D)
+    splits = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
+    assert splits * Hkv >= 148
+    o, lse = _run(loom, q, k, v, None, 0)
+    o_ref, lse_ref = oracle.attention(q, k, v)
+    assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "long decode")
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_edge_lengths(loom, D):
+    # empty sequence, single key, chunk-1, chunk+1, full
+    B, Hq, Hkv, Skv = 6, 4, 2, 300
+    q, k, v = _inputs(3, B, Hq, Hkv, Skv, D)
+    lens = np.array([0, 1, 63, 65, 129, 300], np.int32)
+    for splits in (1, 3, 16, 64):
+        o, lse = _run(loom, q, k, v, lens, splits)
+        o_ref, lse_ref = oracle.attention(q, k, v, seqlens_k=lens)
+        assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"D={D} splits={splits}")
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(1, 1), (3, 1), (8, 8), (16, 2), (32, 1), (12, 4)])
+def test_group_sizes(loom, Hq, Hkv):
+    B, Skv, D = 2, 777, 128
+    q, k, v = _inputs(Hq + Hkv, B, Hq, Hkv, Skv, D)
+    for splits in (1, 5):
+        o, lse = _run(loom, q, k, v, None, splits)
+        o_ref, lse_ref = oracle.attention(q, k, v)
+        assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"Hq={Hq} Hkv={Hkv} splits={splits}")
+
+
+def test_partials_match_oracle_split_form(loom):
+    """The workspace holds the per-split partial (O_i, lse_i) of the Flash Decode form."""
+    import torch
+    B, Hq, Hkv, Skv, D, S = 2, 8, 2, 1000, 128, 5
+    q, k, v = _inputs(9, B, Hq, Hkv, Skv, D)
+    lens = np.array([1000, 333], np.int32)
+    nbytes = loom.loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, S)
+    ws = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    o, lse = _run(loom, q, k, v, lens, S, workspace=ws)
+    _, _, o_part_ref, lse_part_ref = oracle.decode_split_merge(q, k, v, num_splits=S, seqlens_k=lens)
+    n = B * Hq * S
+    opart = ws[: n * D * 4].view(torch.float32).cpu().numpy().astype(np.float64).reshape(B, Hq, S, D)
+    off = (n * D * 4 + 255) // 256 * 256
+    lpart = ws[off: off + n * 4].view(torch.float32).cpu().numpy().astype(np.float64).reshape(B, Hq, S)
+    assert_parity(opart, o_part_ref, lpart, lse_part_ref, "partials")
+
+
+def test_workspace_and_argument_errors(loom):
+    import torch
+    B, Hq, Hkv, Skv, D = 1, 4, 2, 256, 128
+    q, k, v = _inputs(1, B, Hq, Hkv, Skv, D)
+    small = torch.empty(16, dtype=torch.uint8, device="cuda")
+    with pytest.raises(loom.LoomError) as e:
+        loom.loom_attn_decode(to_dev(q), to_dev(k), to_dev(v), None, workspace=small, num_splits=4)
+    assert e.value.status == 4
+    with pytest.raises(loom.LoomError) as e:
+        loom.loom_attn_decode(to_dev(q), to_dev(k), to_dev(v), None, num_splits=2000)
+    assert e.value.status == 2
