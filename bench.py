@@ -1,0 +1,503 @@
+"""Benchmark of the fused-attention hot path on GB300.
+
+Default (N=1): the headline workload is Flash Attention prefill, B=4, Hq=Hkv=32,
+Sq=Skv=2048, D=128, non-causal, bf16 inputs i.i.d. N(0,1) from the seeded generator.
+One "step" is one prefill launch over that batch; `value` is TFLOP/s (4*B*H*Sq*Skv*D
+per step).  The same run also measures, each with its own warm-up and timed loop:
+the causal variant, the long-sequence prefills (S=8192, Hq=32/Hkv=8 D=128 and
+Hq=64/Hkv=16 D=64, causal), batched Flash Decode (B=16, Hq=32, Hkv=8, lengths
+U[4096,8192], 16 splits) and long-context Flash Decode (B=1, Hq=32, Hkv=8, Skv=131072,
+model-chosen splits), reported under "workloads" with their own rooflines.
+
+--impl reference times the fp64 CPU oracle (the reference arm) on host cores on a
+bounded sample of the same workload and prints the same metric.
+
+Multi-GPU (torchrun, one rank per GPU): every rank runs an independent replica of the
+workload (the problems are independent; there is no data-path collective), timing is
+bracketed by barriers and the max over ranks is taken; `value` counts all ranks' work.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "attn fwd TFLOP/s & % of BF16 peak; decode KV GB/s & % of HBM BW (1 GB300)"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# ------------------------------------------------------------------ environment
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in ("hbm_gbs", "bf16_tflops", "bf16_tflops_sustained")}, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+class ClockSampler:
+    """Samples nvidia-smi clocks and throttle reasons while a timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.lines = []
+        self.t0 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "100",
+                 "-i", str(self.dev)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.reader = threading.Thread(target=self._read, daemon=True)
+            self.reader.start()
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self):
+        self.t0 = time.time()
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        t1 = time.time()
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=2)
+        except Exception:
+            self.proc.kill()
+        sms, maxes, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for t, line in self.lines:
+            if self.t0 is not None and not (self.t0 - 0.15 <= t <= t1 + 0.15):
+                continue
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sms.append(float(parts[1]))
+                maxes.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sms:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples in timed region"]}
+        return {"sm_mhz": statistics.median(sms), "sm_max_mhz": max(maxes), "samples": len(sms),
+                "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------------ workloads
+def prefill_flops(B, Hq, Sq, Skv, D, causal):
+    """Algorithmic FLOPs: 4*D per visible (query, key) pair (QK^T and PV, 2 FLOP per MAC)."""
+    if not causal:
+        pairs = Sq * Skv
+    else:
+        off = Skv - Sq
+        pairs = sum(min(Skv, i + off + 1) for i in range(Sq))
+    return 4.0 * B * Hq * D * pairs
+
+
+class Prefill:
+    def __init__(self, name, B, Hq, Hkv, S, D, causal, seed=0, sets=2):
+        self.name, self.B, self.Hq, self.Hkv, self.S, self.D, self.causal = name, B, Hq, Hkv, S, D, causal
+        self.seed, self.sets = seed, sets
+        self.flops = prefill_flops(B, Hq, S, S, D, causal)
+        # algorithmic HBM bytes: read Q, K, V once, write O and LSE
+        self.bytes = 2 * (B * Hq * S * D * 2 + B * Hkv * S * D * 2) + B * Hq * S * 4
+        self.unit = "TFLOP/s"
+
+    def describe(self):
+        return (f"prefill B={self.B} Hq={self.Hq} Hkv={self.Hkv} Sq=Skv={self.S} D={self.D} "
+                f"{'causal' if self.causal else 'non-causal'}")
+
+    def host_inputs(self, s):
+        seed = self.seed + s
+        return (synth.bf16_normal(seed, synth.STREAM_Q, (self.B, self.Hq, self.S, self.D)),
+                synth.bf16_normal(seed, synth.STREAM_K, (self.B, self.Hkv, self.S, self.D)),
+                synth.bf16_normal(seed, synth.STREAM_V, (self.B, self.Hkv, self.S, self.D)))
+
+    def setup(self, torch, dev, loom):
+        self.loom = loom
+        self.inp = []
+        for s in range(self.sets):
+            q, k, v = (to_tensor(torch, x, dev) for x in self.host_inputs(s))
+            o = torch.empty_like(q)
+            lse = torch.empty((self.B, self.Hq, self.S), dtype=torch.float32, device=dev)
+            self.inp.append((q, k, v, o, lse))
+
+    def launches_per_step(self):
+        return 1
+
+    def step(self, i, stream):
+        q, k, v, o, lse = self.inp[i % self.sets]
+        self.loom.loom_attn_fwd(q, k, v, o, lse, causal=self.causal, stream=stream)
+
+    def value(self, seconds_per_step):
+        return self.flops / seconds_per_step / 1e12
+
+    # end to end through the public API with host buffers
+    def e2e_setup(self, torch, dev):
+        q, k, v = self.host_inputs(0)
+        pin = lambda a: to_host_tensor(torch, a).pin_memory()
+        self.h_in = [pin(q), pin(k), pin(v)]
+        self.h_o = torch.empty(q.shape, dtype=torch.bfloat16).pin_memory()
+        self.h_lse = torch.empty((self.B, self.Hq, self.S), dtype=torch.float32).pin_memory()
+        self.d_in = [torch.empty(t.shape, dtype=t.dtype, device=dev) for t in self.h_in]
+        self.d_o = torch.empty(q.shape, dtype=torch.bfloat16, device=dev)
+        self.d_lse = torch.empty(self.h_lse.shape, dtype=torch.float32, device=dev)
+        self.h2d = sum(t.numel() * t.element_size() for t in self.h_in)
+        self.d2h = self.h_o.numel() * 2 + self.h_lse.numel() * 4
+
+    def e2e_step(self, stream):
+        for d, h in zip(self.d_in, self.h_in):
+            d.copy_(h, non_blocking=True)
+        self.loom.loom_attn_fwd(*self.d_in, self.d_o, self.d_lse, causal=self.causal, stream=stream)
+        self.h_o.copy_(self.d_o, non_blocking=True)
+        self.h_lse.copy_(self.d_lse, non_blocking=True)
+
+
+class Decode:
+    def __init__(self, name, B, Hq, Hkv, Skv, D, splits, lengths=None, seed=0, sets=2):
+        self.name, self.B, self.Hq, self.Hkv, self.Skv, self.D = name, B, Hq, Hkv, Skv, D
+        self.splits, self.seed, self.sets = splits, seed, sets
+        self.lens = None if lengths is None else np.asarray(lengths, np.int32)
+        total = int(self.lens.sum()) if self.lens is not None else B * Skv
+        # algorithmic bytes: the K and V rows actually needed + q + o + lse
+        self.bytes = 2 * Hkv * total * D * 2 + 2 * B * Hq * D * 2 + B * Hq * 4
+        self.flops = 4.0 * Hq * total * D
+        self.unit = "GB/s"
+
+    def describe(self):
+        ln = "lengths U[4096,8192]" if self.lens is not None else f"Skv={self.Skv}"
+        return (f"decode B={self.B} Hq={self.Hq} Hkv={self.Hkv} Skv_max={self.Skv} D={self.D} {ln} "
+                f"splits={self.splits or 'model'}")
+
+    def host_inputs(self, s):
+        seed = self.seed + s
+        return (synth.bf16_normal(seed, synth.STREAM_Q, (self.B, self.Hq, 1, self.D)),
+                synth.bf16_normal(seed, synth.STREAM_K, (self.B, self.Hkv, self.Skv, self.D)),
+                synth.bf16_normal(seed, synth.STREAM_V, (self.B, self.Hkv, self.Skv, self.D)))
+
+    def setup(self, torch, dev, loom):
+        self.loom = loom
+        self.inp = []
+        self.sl = None if self.lens is None else torch.from_numpy(self.lens).to(dev)
+        nbytes = loom.loom_attn_decode_workspace_bytes(self.B, self.Hq, self.Hkv, self.Skv, self.D, self.splits)
+        self.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        self.used_splits = self.splits or loom.loom_attn_decode_num_splits(self.B, self.Hq, self.Hkv, self.Skv, self.D)
+        for s in range(self.sets):
+            q, k, v = (to_tensor(torch, x, dev) for x in self.host_inputs(s))
+            o = torch.empty_like(q)
+            lse = torch.empty((self.B, self.Hq), dtype=torch.float32, device=dev)
+            self.inp.append((q, k, v, o, lse))
+
+    def launches_per_step(self):
+        return 2
+
+    def step(self, i, stream):
+        q, k, v, o, lse = self.inp[i % self.sets]
+        self.loom.loom_attn_decode(q, k, v, self.sl, o, lse, self.ws, num_splits=self.splits, stream=stream)
+
+    def value(self, seconds_per_step):
+        return self.bytes / seconds_per_step / 1e9
+
+
+def to_tensor(torch, bits, dev):
+    return to_host_tensor(torch, bits).to(dev)
+
+
+def to_host_tensor(torch, bits):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16)
+
+
+# ------------------------------------------------------------------ timing
+def time_steps(torch, wl, steps, warmup, stream, barrier, per_launch_events=True):
+    """Warm up, then time exactly `steps` steps with CUDA events on `stream`."""
+    with torch.cuda.stream(stream):
+        for i in range(warmup):
+            wl.step(i, stream)
+    torch.cuda.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(steps)] if per_launch_events else []
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t_start.record(stream)
+        for i in range(steps):
+            if evs:
+                evs[i][0].record(stream)
+            wl.step(warmup + i, stream)
+            if evs:
+                evs[i][1].record(stream)
+        t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    total_ms = t_start.elapsed_time(t_end)
+    launch_ms = [a.elapsed_time(b) for a, b in evs]
+    return total_ms, launch_ms
+
+
+def measure(torch, wl, steps, warmup, stream, barrier, world, reduce_max, peaks):
+    total_ms, launch_ms = time_steps(torch, wl, steps, warmup, stream, barrier)
+    total_ms = reduce_max(total_ms)
+    ms_per_step = total_ms / steps
+    value = wl.value(ms_per_step * 1e-3) * world
+    avg_launch_ms = statistics.mean(launch_ms) if launch_ms else ms_per_step
+    if wl.unit == "TFLOP/s":
+        achieved = wl.flops / (avg_launch_ms * 1e-3) / 1e12
+        roof = {"bound": "tensor", "achieved": round(achieved, 2), "peak": peaks["bf16_tflops"],
+                "unit": "TFLOP/s", "frac": round(achieved / peaks["bf16_tflops"], 4)}
+    else:
+        achieved = wl.bytes / (avg_launch_ms * 1e-3) / 1e9
+        roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": round(achieved / peaks["hbm_gbs"], 4)}
+    return {"value": round(value, 3), "unit": wl.unit, "ms_per_step": round(ms_per_step, 5),
+            "avg_launch_ms": round(avg_launch_ms, 5), "roofline": roof}
+
+
+def measure_e2e(torch, wl, steps, warmup, stream, barrier, reduce_max, world):
+    wl.e2e_setup(torch, stream.device)
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            wl.e2e_step(stream)
+    torch.cuda.synchronize()
+    barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        a.record(stream)
+        for _ in range(steps):
+            wl.e2e_step(stream)
+        b.record(stream)
+    torch.cuda.synchronize()
+    ms = reduce_max(a.elapsed_time(b)) / steps
+    return {"value": round(wl.value(ms * 1e-3) * world, 3), "unit": wl.unit,
+            "h2d_bytes_per_step": int(wl.h2d), "d2h_bytes_per_step": int(wl.d2h),
+            "ms_per_step": round(ms, 4)}
+
+
+# ------------------------------------------------------------------ CPU oracle leg
+def oracle_sample(wl, budget_s, threads=0):
+    """Time the fp64 oracle on whole (b, h) heads of the prefill workload until the
+    time budget is used; returns (TFLOP/s, heads done, seconds, threads)."""
+    import oracle
+    oracle.build()
+    q, k, v = wl.host_inputs(0)
+    heads_total = wl.B * wl.Hq
+    done, flops, t0 = 0, 0.0, time.perf_counter()
+    per_head = wl.flops / heads_total
+    while done < heads_total and time.perf_counter() - t0 < budget_s:
+        b, h = divmod(done, wl.Hq)
+        rows = (np.arange(wl.S, dtype=np.int64) + (b * wl.Hq + h) * wl.S)
+        oracle.attention(q, k, v, causal=wl.causal, rows=rows, nthreads=threads)
+        done += 1
+        flops += per_head
+    dt = time.perf_counter() - t0
+    return flops / dt / 1e12, done, dt, threads or (os.cpu_count() or 1)
+
+
+# ------------------------------------------------------------------ main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["loom", "reference"], default="loom")
+    ap.add_argument("--quick", action="store_true", help="headline workload only")
+    ap.add_argument("--oracle-seconds", type=float, default=12.0)
+    args = ap.parse_args()
+    world, rank, local = dist_env()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    headline = Prefill("prefill", 4, 32, 32, 2048, 128, causal=False)
+    if args.impl == "reference":
+        return run_reference(args, headline, world, rank)
+
+    import torch
+    import paper_2609_29219_gb300 as loom
+    from paper_2609_29219_gb300 import build as libbuild
+    if not os.path.exists(loom.library_path()):
+        libbuild.build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+        def barrier():
+            dist.barrier()
+
+        def reduce_max(x):
+            t = torch.tensor([float(x)], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            return float(t.item())
+    else:
+        def barrier():
+            pass
+
+        def reduce_max(x):
+            return float(x)
+
+    peaks, peak_src = load_peaks()
+    stream = torch.cuda.Stream(dev)
+
+    # headline: prefill non-causal, with clocks sampled during the timed loop
+    headline.setup(torch, dev, loom)
+    clocks = ClockSampler(local)
+    clocks.start()
+    # a short untimed pass first so the clock sampler starts on a busy GPU
+    time_steps(torch, headline, 20, args.warmup, stream, barrier, per_launch_events=False)
+    clocks.mark()
+    res = measure(torch, headline, args.steps, args.warmup, stream, barrier, world, reduce_max, peaks)
+    clk = clocks.stop()
+    loom.loom_attn_check_error(stream)
+    e2e = measure_e2e(torch, headline, max(5, min(args.steps, 50)), 3, stream, barrier, reduce_max, world)
+    loom.loom_attn_check_error(stream)
+    headline.inp = None
+
+    workloads = {}
+    if not args.quick:
+        lens = synth.decode_lengths(0, 16, 4096, 8192)
+        extra = [
+            Prefill("prefill_causal", 4, 32, 32, 2048, 128, causal=True),
+            Prefill("long_prefill_d128", 1, 32, 8, 8192, 128, causal=True),
+            Prefill("long_prefill_d64", 1, 64, 16, 8192, 64, causal=True),
+            Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
+            Decode("long_decode", 1, 32, 8, 131072, 128, splits=0),
+        ]
+        for wl in extra:
+            wl.setup(torch, dev, loom)
+            r = measure(torch, wl, max(10, args.steps // 2), args.warmup, stream, barrier, world, reduce_max, peaks)
+            loom.loom_attn_check_error(stream)
+            r["workload"] = wl.describe()
+            if isinstance(wl, Decode):
+                r["splits"] = wl.used_splits
+                r["kv_bytes_per_step"] = int(wl.bytes)
+            r["gpu_launches"] = wl.launches_per_step() * max(10, args.steps // 2)
+            workloads[wl.name] = r
+            wl.inp = None
+            torch.cuda.empty_cache()
+
+    cpu = None
+    if rank == 0 and world == 1:
+        tf, heads, dt, thr = oracle_sample(headline, args.oracle_seconds)
+        cpu = {"value": round(tf, 6), "unit": "TFLOP/s", "cores": thr, "kind": "oracle",
+               "sample": f"{heads} of {headline.B * headline.Hq} (b,h) heads x all {headline.S} query rows "
+                         f"of the headline workload, fp64, {dt:.1f} s"}
+
+    if rank == 0:
+        roof = dict(res["roofline"])
+        roof["traffic"] = None
+        roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json bf16 burst)" if peak_src == "measured" else peak_src
+        line = {
+            "metric": METRIC,
+            "value": res["value"],
+            "unit": "TFLOP/s",
+            "n_gpus": world,
+            "steps": args.steps,
+            "warmup": args.warmup,
+            "ms_per_step": res["ms_per_step"],
+            "higher_is_better": True,
+            "scaling": "weak",
+            "vs_baseline": None,
+            "dtype": "bf16",
+            "data": "synthetic (seeded splitmix64/Box-Muller N(0,1) rounded to bf16)",
+            "config": {"workload": headline.describe(), "B": 4, "Hq": 32, "Hkv": 32, "Sq": 2048, "Skv": 2048,
+                       "D": 128, "causal": False, "global_batch": 4 * world, "seq_len": 2048,
+                       "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                       "l2": "inputs larger than L2 (268 MB per step), 2 rotating input sets"},
+            "roofline": roof,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": args.steps * headline.launches_per_step(),
+            "clocks": clk,
+            "workloads": workloads,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_reference(args, wl, world, rank):
+    """Reference arm: the fp64 oracle on host cores; each step is a bounded sample of
+    the headline workload (512 query rows of one (b, h) head, heads rotating)."""
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    q, k, v = wl.host_inputs(0)
+    rows_per_step = 512
+    heads = wl.B * wl.Hq
+    per_row = wl.flops / (heads * wl.S)  # non-causal: every row costs the same
+
+    def step(i):
+        head = i % heads
+        r0 = (i // heads * rows_per_step) % wl.S
+        rows = np.arange(r0, r0 + rows_per_step, dtype=np.int64) % wl.S + head * wl.S
+        oracle.attention(q, k, v, causal=wl.causal, rows=rows)
+
+    for i in range(args.warmup):
+        step(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        step(args.warmup + i)
+    dt = time.perf_counter() - t0
+    ms = dt * 1e3 / args.steps
+    value = rows_per_step * per_row / (ms * 1e-3) / 1e12
+    cores = os.cpu_count() or 1
+    line = {
+        "impl": "reference",
+        "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded splitmix64/Box-Muller N(0,1) rounded to bf16)",
+        "config": {"workload": wl.describe(), "B": 4, "Hq": 32, "Hkv": 32, "Sq": 2048, "Skv": 2048, "D": 128,
+                   "causal": False},
+        "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{rows_per_step} query rows of one (b,h) head per step (fp64 oracle, "
+                                   f"{cores} threads)"},
+        "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()
