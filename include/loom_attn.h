@@ -100,6 +100,29 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
                              float scale, int num_splits, void* stream);
 
 /*
+ * Flash Decode without any allocation and without a workspace argument.  The paper has
+ * no counterpart; this entry point exists for callers that cannot obtain device scratch
+ * memory for a call -- serving engines that reserve all device memory at start-up and
+ * forbid allocation on the request path (cudaMalloc synchronises the whole device and
+ * can fail mid-request), and plug-in hosts that pass a library only the call's tensors.
+ *
+ * Arguments, layouts and results are those of loom_attn_decode.  The per-split partials
+ * live in a scratch array built into the library (LOOM_DECODE_NOALLOC_SCRATCH_BYTES,
+ * 8 MiB), held by every GPU that loads the library until the process exits.  A problem
+ * whose partials need more (loom_attn_decode_workspace_bytes(...) larger than that)
+ * returns LOOM_ERR_WORKSPACE without launching anything.  The first call on a device
+ * looks up the array's device address (cudaGetSymbolAddress, current device); make that
+ * first call before any stream capture.  All calls share the array, which keeps the last
+ * call's contents (nothing in it needs to start at zero); calls whose kernels overlap on
+ * the GPU race on it.  This entry point itself calls no cudaMalloc or cudaFree.
+ */
+#define LOOM_DECODE_NOALLOC_SCRATCH_BYTES ((size_t)8 << 20)
+loom_status loom_attn_decode_noalloc(const void* q, const void* k_cache, const void* v_cache,
+                                     const int32_t* seqlens_k, void* o, float* lse, int B, int Hq,
+                                     int Hkv, int Skv, int D, float scale, int num_splits,
+                                     void* stream);
+
+/*
  * Synchronises `stream`, then reads and clears the current device's error word.
  * Returns LOOM_OK, LOOM_ERR_TIMEOUT if a kernel abandoned a bounded wait since the last
  * check, or LOOM_ERR_CUDA if the synchronisation itself failed.
