@@ -367,28 +367,58 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
   }
 }
 
+// One CTA (D threads) per (batch, query head).  The split log-sum-exps are read in
+// parallel (one per thread), reduced, turned into weights in shared memory, and the
+// partial rows are streamed with 8 independent loads in flight per thread.
 template <int D>
 __global__ void __launch_bounds__(D) decode_merge_kernel(const float* __restrict__ o_part,
                                                          const float* __restrict__ lse_part,
                                                          __nv_bfloat16* __restrict__ o,
                                                          float* __restrict__ lse, int splits) {
+  constexpr int NW = D / 32;
+  __shared__ float w_s[kMaxDecodeSplits];
+  __shared__ float red[NW];
   // Wait until the split kernel's partials are complete and visible.
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  const int bh = blockIdx.x, d = threadIdx.x;
+  const int bh = blockIdx.x, d = threadIdx.x, lane = d & 31, wid = d >> 5;
   const float* lp = lse_part + static_cast<size_t>(bh) * splits;
-  float M = -INFINITY;
-  for (int i = 0; i < splits; ++i) M = fmaxf(M, lp[i]);
-  float W = 0.f, acc = 0.f;
-  if (M != -INFINITY) {
-    const float* op = o_part + static_cast<size_t>(bh) * splits * D + d;
-    for (int i = 0; i < splits; ++i) {
-      const float w = ex2((lp[i] - M) * kLog2e);
-      W += w;
-      acc = fmaf(w, op[static_cast<size_t>(i) * D], acc);
-    }
+
+  float m = -INFINITY;
+  for (int i = d; i < splits; i += D) m = fmaxf(m, lp[i]);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+  if (lane == 0) red[wid] = m;
+  __syncthreads();
+  float M = red[0];
+#pragma unroll
+  for (int w = 1; w < NW; ++w) M = fmaxf(M, red[w]);
+  __syncthreads();
+
+  float ws = 0.f;
+  for (int i = d; i < splits; i += D) {
+    const float w = (M == -INFINITY) ? 0.f : ex2((lp[i] - M) * kLog2e);  // 0 for empty splits
+    w_s[i] = w;
+    ws += w;
   }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) ws += __shfl_xor_sync(0xffffffffu, ws, off);
+  if (lane == 0) red[wid] = ws;
+  __syncthreads();
+  float W = 0.f;
+#pragma unroll
+  for (int w = 0; w < NW; ++w) W += red[w];
+
+  const float* op = o_part + static_cast<size_t>(bh) * splits * D + d;
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  int i = 0;
+  for (; i + 8 <= splits; i += 8) {
+#pragma unroll
+    for (int u = 0; u < 8; ++u) acc[u] = fmaf(w_s[i + u], op[static_cast<size_t>(i + u) * D], acc[u]);
+  }
+  for (; i < splits; ++i) acc[0] = fmaf(w_s[i], op[static_cast<size_t>(i) * D], acc[0]);
+  const float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
   const bool any = W > 0.f;
-  o[static_cast<size_t>(bh) * D + d] = __float2bfloat16_rn(any ? acc / W : 0.f);
+  o[static_cast<size_t>(bh) * D + d] = __float2bfloat16_rn(any ? sum / W : 0.f);
   if (lse && d == 0) lse[bh] = any ? M + log2f(W) * kLn2 : -INFINITY;
 }
 

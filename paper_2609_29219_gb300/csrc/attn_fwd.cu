@@ -111,9 +111,15 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
   const int kv_z = b * p.Hkv + hk;
   const int q0 = pair * (C::NQT * C::BM);
   const int off = p.Skv - p.Sq;  // bottom-right causal offset
-  int n_kv = p.Skv;
-  if (p.causal) n_kv = min(p.Skv, q0 + C::NQT * C::BM + off);
-  const int n_tiles = (n_kv + C::BN - 1) / C::BN;
+  // KV tiles each query tile needs (causal: up to the diagonal of its last row); the
+  // CTA loads the union, i.e. tile 1's range.
+  int n_kv0 = p.Skv, n_kv1 = p.Skv;
+  if (p.causal) {
+    n_kv0 = min(p.Skv, q0 + C::BM + off);
+    n_kv1 = min(p.Skv, q0 + 2 * C::BM + off);
+  }
+  const int n_tiles0 = (n_kv0 + C::BN - 1) / C::BN;
+  const int n_tiles = (n_kv1 + C::BN - 1) / C::BN;
 
   const uint32_t bar_q = sbase + C::BAR_OFF;
   const uint32_t bar_full = bar_q + 8;
@@ -222,16 +228,20 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
       for (int j = 0; ok && j < n_tiles; ++j) {
         const int vpos = 2 * j + 1, kpos = 2 * j + 2;
         const bool more = j + 1 < n_tiles;
-        ok = wait_slot(vpos) && mbar_wait(bar_p, j & 1, p.ctl, ab);
-        if (!ok) break;
-        tc_fence_after();
-        issue_pv(0, vpos, j > 0);
-        tc_commit(bar_o);
+        if (!(ok = wait_slot(vpos))) break;
+        if (j < n_tiles0) {  // query tile 0 stops at its own diagonal
+          if (!(ok = mbar_wait(bar_p, j & 1, p.ctl, ab))) break;
+          tc_fence_after();
+          issue_pv(0, vpos, j > 0);
+          tc_commit(bar_o);
+        }
         if (more) {
           if (!(ok = wait_slot(kpos))) break;
           tc_fence_after();
-          issue_s(0, kpos);
-          tc_commit(bar_s);
+          if (j + 1 < n_tiles0) {
+            issue_s(0, kpos);
+            tc_commit(bar_s);
+          }
         }
         if (!(ok = mbar_wait(bar_p + 8, j & 1, p.ctl, ab))) break;
         tc_fence_after();
@@ -259,11 +269,13 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
     const uint32_t o_tm = tmem + lane_addr + C::O_COL + t * D;
     const uint32_t my_bar_s = bar_s + 8 * t, my_bar_p = bar_p + 8 * t, my_bar_o = bar_o + 8 * t;
     const int limit = p.causal ? min(p.Skv, row + off + 1) : p.Skv;  // keys [0, limit) visible
+    const int my_tiles = t == 0 ? n_tiles0 : n_tiles;
     const float c = p.c;
+    const uint64_t c2 = f2(c, c);
 
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
-    for (int j = 0; j < n_tiles; ++j) {
+    for (int j = 0; j < my_tiles; ++j) {
       if (!(ok = mbar_wait_warp(my_bar_s, j & 1, p.ctl, ab))) break;
       tc_fence_after();
       uint32_t s[C::BN];
@@ -278,17 +290,53 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
         for (int i = 0; i < C::BN; ++i)
           if (kbase + i >= limit) s[i] = __float_as_uint(-INFINITY);
       }
-      float mx = __uint_as_float(s[0]);
+      // row max: 8 independent chains of 3-input max, then a small tree
+      float mx;
+      {
+        float mm[8];
 #pragma unroll
-      for (int i = 1; i < C::BN; ++i) mx = fmaxf(mx, __uint_as_float(s[i]));
+        for (int g = 0; g < 8; ++g) mm[g] = __uint_as_float(s[g]);
+#pragma unroll
+        for (int i = 8; i + 16 <= C::BN; i += 16)
+#pragma unroll
+          for (int g = 0; g < 8; ++g)
+            mm[g] = max3(mm[g], __uint_as_float(s[i + g]), __uint_as_float(s[i + 8 + g]));
+        if constexpr ((C::BN - 8) % 16 != 0) {
+#pragma unroll
+          for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], __uint_as_float(s[C::BN - 8 + g]));
+        }
+        mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
+      }
       const float m_new = fmaxf(m_run, mx * c);
       const bool need = m_new > m_run + kRescaleThreshold;
       const float alpha = need ? ex2(m_run - m_new) : 1.f;
       if (need) m_run = m_new;
+      const float ms = (m_run == -INFINITY) ? 0.f : m_run;
+      const uint64_t nms2 = f2(-ms, -ms);
+      // p = 2^(s*c - m): packed FMA, one MUFU ex2 per score, 4 packed partial sums
+      uint64_t acc[4] = {0, 0, 0, 0};
+      uint32_t pk[C::BN / 2];
+#pragma unroll
+      for (int i = 0; i < C::BN / 2; ++i) {
+        const uint64_t x = fma2(f2(__uint_as_float(s[2 * i]), __uint_as_float(s[2 * i + 1])), c2, nms2);
+        const float p0 = ex2(f2lo(x));
+        const float p1 = ex2(f2hi(x));
+        acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
+        pk[i] = pack_bf16x2(p0, p1);
+      }
+#pragma unroll
+      for (int ch = 0; ch < C::BN / 64; ++ch) tmem_st32(s_tm + ch * 32, pk + ch * 32);
+      const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+      const float rs = f2lo(a01) + f2hi(a01);
+      tmem_wait_st();
+      l_run = l_run * alpha + rs;
+      // O_t must hold P_{j-1} V_{j-1} before it is rescaled, and be rescaled before
+      // P_j V_j is issued (i.e. before the P-ready arrive below).  Done after P is
+      // written so that the S row is no longer live in registers.
       if (j > 0 && __any_sync(0xffffffffu, need)) {
-        // O_t must hold P_{j-1} V_{j-1} before it is rescaled
         if (!(ok = mbar_wait_warp(my_bar_o, (j - 1) & 1, p.ctl, ab))) break;
         tc_fence_after();
+        const uint64_t a2 = f2(alpha, alpha);
 #pragma unroll 1
         for (int ch = 0; ch < D / 32; ++ch) {
           uint32_t r[32];
@@ -296,31 +344,21 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
           tmem_wait_ld();
           reg_fence32(r);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+          for (int i = 0; i < 16; ++i) {
+            const uint64_t x = mul2(f2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1])), a2);
+            r[2 * i] = __float_as_uint(f2lo(x));
+            r[2 * i + 1] = __float_as_uint(f2hi(x));
+          }
           tmem_st32(o_tm + ch * 32, r);
         }
         tmem_wait_st();
       }
-      const float ms = (m_run == -INFINITY) ? 0.f : m_run;
-      float rs = 0.f;
-      uint32_t pk[C::BN / 2];
-#pragma unroll
-      for (int i = 0; i < C::BN / 2; ++i) {
-        const float p0 = ex2(fmaf(__uint_as_float(s[2 * i]), c, -ms));
-        const float p1 = ex2(fmaf(__uint_as_float(s[2 * i + 1]), c, -ms));
-        rs += p0 + p1;
-        pk[i] = pack_bf16x2(p0, p1);
-      }
-#pragma unroll
-      for (int ch = 0; ch < C::BN / 64; ++ch) tmem_st32(s_tm + ch * 32, pk + ch * 32);
-      tmem_wait_st();
-      l_run = l_run * alpha + rs;
       tc_fence_before();
       mbar_arrive(my_bar_p);
     }
 
     // epilogue: O / l -> bf16 rows, LSE
-    if (ok && n_tiles > 0) ok = mbar_wait_warp(my_bar_o, (n_tiles - 1) & 1, p.ctl, ab);
+    if (ok && my_tiles > 0) ok = mbar_wait_warp(my_bar_o, (my_tiles - 1) & 1, p.ctl, ab);
     if (ok) {
       tc_fence_after();
       const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
@@ -334,9 +372,12 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
         tmem_wait_ld();
         reg_fence32(r);
         uint32_t w[16];
+        const uint64_t il2 = f2(inv_l, inv_l);
 #pragma unroll
-        for (int i = 0; i < 16; ++i)
-          w[i] = pack_bf16x2(__uint_as_float(r[2 * i]) * inv_l, __uint_as_float(r[2 * i + 1]) * inv_l);
+        for (int i = 0; i < 16; ++i) {
+          const uint64_t x = mul2(f2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1])), il2);
+          w[i] = pack_bf16x2(f2lo(x), f2hi(x));
+        }
         if (store) {
           uint4* dst = reinterpret_cast<uint4*>(orow + ch * 32);
 #pragma unroll
