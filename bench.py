@@ -62,7 +62,7 @@ class ClockSampler:
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap,clocks.mem")
 
     def __init__(self, device_index: int):
         self.dev = device_index
@@ -85,30 +85,23 @@ class ClockSampler:
         for line in self.proc.stdout:
             self.lines.append((time.time(), line.strip()))
 
-    def mark(self):
-        self.t0 = time.time()
+    def now(self):
+        return time.time()
 
-    def stop(self):
-        if self.proc is None:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        t1 = time.time()
-        time.sleep(0.15)
-        self.proc.terminate()
-        try:
-            self.proc.wait(timeout=2)
-        except Exception:
-            self.proc.kill()
-        sms, maxes, reasons = [], [], set()
+    def window(self, t0, t1):
+        """Median SM/memory clock and throttle reasons seen between t0 and t1."""
+        sms, maxes, mems, reasons = [], [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for t, line in self.lines:
-            if self.t0 is not None and not (self.t0 - 0.15 <= t <= t1 + 0.15):
+        for t, line in list(self.lines):
+            if not (t0 - 0.12 <= t <= t1 + 0.12):
                 continue
             parts = [p.strip() for p in line.split(",")]
-            if len(parts) < 9:
+            if len(parts) < 10:
                 continue
             try:
                 sms.append(float(parts[1]))
                 maxes.append(float(parts[2]))
+                mems.append(float(parts[9]))
             except ValueError:
                 continue
             for name, val in zip(names, parts[5:9]):
@@ -116,8 +109,17 @@ class ClockSampler:
                     reasons.add(name)
         if not sms:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples in timed region"]}
-        return {"sm_mhz": statistics.median(sms), "sm_max_mhz": max(maxes), "samples": len(sms),
-                "reasons": sorted(reasons)}
+        return {"sm_mhz": statistics.median(sms), "sm_max_mhz": max(maxes), "mem_mhz": statistics.median(mems),
+                "samples": len(sms), "reasons": sorted(reasons)}
+
+    def stop(self):
+        if self.proc is None:
+            return
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=2)
+        except Exception:
+            self.proc.kill()
 
 
 # ------------------------------------------------------------------ workloads
@@ -245,11 +247,21 @@ def to_host_tensor(torch, bits):
 
 
 # ------------------------------------------------------------------ timing
+WARMUP_SECONDS = 1.0  # clocks ramp up slowly after host-side idle periods
+
+
 def time_steps(torch, wl, steps, warmup, stream, barrier, per_launch_events=True):
-    """Warm up, then time exactly `steps` steps with CUDA events on `stream`."""
+    """Warm up (at least `warmup` steps and WARMUP_SECONDS of back-to-back work), then
+    time exactly `steps` steps with CUDA events on `stream`."""
+    t0 = time.perf_counter()
+    i = 0
     with torch.cuda.stream(stream):
-        for i in range(warmup):
-            wl.step(i, stream)
+        while i < warmup or time.perf_counter() - t0 < WARMUP_SECONDS:
+            for _ in range(max(1, warmup)):
+                wl.step(i, stream)
+                i += 1
+            stream.synchronize()
+    warmup = i
     torch.cuda.synchronize()
     barrier()
     torch.cuda.synchronize()
@@ -274,8 +286,12 @@ def time_steps(torch, wl, steps, warmup, stream, barrier, per_launch_events=True
     return total_ms, launch_ms
 
 
-def measure(torch, wl, steps, warmup, stream, barrier, world, reduce_max, peaks):
+def measure(torch, wl, steps, warmup, stream, barrier, world, reduce_max, peaks, clocks=None):
+    t_wall0 = time.time()
     total_ms, launch_ms = time_steps(torch, wl, steps, warmup, stream, barrier)
+    t_wall1 = time.time()
+    window = (t_wall1 - total_ms * 1e-3, t_wall1)  # the timed loop ends at the final sync
+    del t_wall0
     total_ms = reduce_max(total_ms)
     ms_per_step = total_ms / steps
     value = wl.value(ms_per_step * 1e-3) * world
@@ -288,8 +304,11 @@ def measure(torch, wl, steps, warmup, stream, barrier, world, reduce_max, peaks)
         achieved = wl.bytes / (avg_launch_ms * 1e-3) / 1e9
         roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": round(achieved / peaks["hbm_gbs"], 4)}
-    return {"value": round(value, 3), "unit": wl.unit, "ms_per_step": round(ms_per_step, 5),
-            "avg_launch_ms": round(avg_launch_ms, 5), "roofline": roof}
+    res = {"value": round(value, 3), "unit": wl.unit, "ms_per_step": round(ms_per_step, 5),
+           "avg_launch_ms": round(avg_launch_ms, 5), "roofline": roof}
+    if clocks is not None:
+        res["clocks"] = clocks.window(*window)
+    return res
 
 
 def measure_e2e(torch, wl, steps, warmup, stream, barrier, reduce_max, world):
@@ -340,7 +359,11 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["loom", "reference"], default="loom")
     ap.add_argument("--quick", action="store_true", help="headline workload only")
+    ap.add_argument("--only", default=None,
+                    help="comma-separated subset (and order) of the extra workloads to run")
     ap.add_argument("--oracle-seconds", type=float, default=12.0)
+    ap.add_argument("--sweep", choices=["decode"], default=None,
+                    help="model-vs-measured sweep of the decode split count (one JSON line per point)")
     args = ap.parse_args()
     world, rank, local = dist_env()
     if args.warmup < 3:
@@ -377,23 +400,22 @@ def main():
 
     peaks, peak_src = load_peaks()
     stream = torch.cuda.Stream(dev)
+    if args.sweep == "decode":
+        return run_decode_sweep(torch, loom, dev, stream, args, peaks)
 
     # headline: prefill non-causal, with clocks sampled during the timed loop
     headline.setup(torch, dev, loom)
     clocks = ClockSampler(local)
     clocks.start()
-    # a short untimed pass first so the clock sampler starts on a busy GPU
-    time_steps(torch, headline, 20, args.warmup, stream, barrier, per_launch_events=False)
-    clocks.mark()
-    res = measure(torch, headline, args.steps, args.warmup, stream, barrier, world, reduce_max, peaks)
-    clk = clocks.stop()
+    res = measure(torch, headline, args.steps, args.warmup, stream, barrier, world, reduce_max, peaks, clocks)
+    clk = res.pop("clocks", None)
     loom.loom_attn_check_error(stream)
     e2e = measure_e2e(torch, headline, max(5, min(args.steps, 50)), 3, stream, barrier, reduce_max, world)
     loom.loom_attn_check_error(stream)
     headline.inp = None
 
     workloads = {}
-    if not args.quick:
+    if not args.quick or args.only:
         lens = synth.decode_lengths(0, 16, 4096, 8192)
         extra = [
             Prefill("prefill_causal", 4, 32, 32, 2048, 128, causal=True),
@@ -402,9 +424,13 @@ def main():
             Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
             Decode("long_decode", 1, 32, 8, 131072, 128, splits=0),
         ]
+        if args.only:
+            by_name = {wl.name: wl for wl in extra}
+            extra = [by_name[n] for n in args.only.split(",") if n]
         for wl in extra:
             wl.setup(torch, dev, loom)
-            r = measure(torch, wl, max(10, args.steps // 2), args.warmup, stream, barrier, world, reduce_max, peaks)
+            r = measure(torch, wl, max(10, args.steps // 2), args.warmup, stream, barrier, world, reduce_max, peaks,
+                        clocks)
             loom.loom_attn_check_error(stream)
             r["workload"] = wl.describe()
             if isinstance(wl, Decode):
@@ -415,6 +441,7 @@ def main():
             wl.inp = None
             torch.cuda.empty_cache()
 
+    clocks.stop()
     cpu = None
     if rank == 0 and world == 1:
         tf, heads, dt, thr = oracle_sample(headline, args.oracle_seconds)
@@ -454,6 +481,33 @@ def main():
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def run_decode_sweep(torch, loom, dev, stream, args, peaks):
+    """Measured vs modeled Flash Decode time over split counts (the model's choice is the
+    point marked "model": true)."""
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    lens = synth.decode_lengths(0, 16, 4096, 8192)
+    cases = [
+        (Decode("long_decode", 1, 32, 8, 131072, 128, splits=0), [8, 16, 19, 24, 32, 38, 48, 57, 64, 76, 96, 114, 152]),
+        (Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens), [1, 2, 3, 4, 6, 8, 12, 16, 19, 24, 32]),
+    ]
+    for wl, splits in cases:
+        wl.setup(torch, dev, loom)
+        chosen = loom.loom_attn_decode_num_splits(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D)
+        for sp in sorted(set(splits + [chosen])):
+            wl.splits = sp
+            nbytes = loom.loom_attn_decode_workspace_bytes(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sp)
+            wl.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+            r = measure(torch, wl, max(10, args.steps // 4), args.warmup, stream, lambda: None, 1, float, peaks)
+            loom.loom_attn_check_error(stream)
+            model_us = loom.loom_model_decode_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sms)
+            print(json.dumps({"sweep": "decode", "workload": wl.describe(), "splits": sp,
+                              "model_choice": sp == chosen, "measured_us": round(r["ms_per_step"] * 1e3, 2),
+                              "model_us": round(model_us, 2), "GB/s": r["value"],
+                              "frac": r["roofline"]["frac"]}), flush=True)
+        wl.inp = None
+        torch.cuda.empty_cache()
 
 
 def run_reference(args, wl, world, rank):

@@ -123,6 +123,28 @@ loom_status loom_attn_decode_noalloc(const void* q, const void* k_cache, const v
                                      void* stream);
 
 /*
+ * Analytic schedule model (paper Sec. 2.6: HEG latency, Eq. 5-7, and the constrained
+ * selection of Eq. 8-9, solved by enumeration) with the GB300 architecture description
+ * of Sec. 2.7.  The kernels are compiled with the plan these functions report.
+ *
+ * loom_model_fwd_plan: the prefill plan for head dimension D (64 or 128): rows per query
+ *   tile, keys per KV tile, query tiles per CTA, K/V ring slots, the pipeline knob
+ *   (b_lm, b_ms) of Eq. 6, shared-memory bytes, TMEM columns, and the modeled latencies
+ *   (ns) of one KV-tile iteration: load stage, MMA leaf, softmax leaf, and the pipe node.
+ *   Returns LOOM_ERR_UNSUPPORTED for other D, LOOM_ERR_INVALID_ARG for a NULL out.
+ * loom_model_fwd_time_us: modeled time of a whole prefill launch (us); < 0 on bad sizes.
+ * loom_model_decode_time_us: modeled split + merge time (us) of Flash Decode with
+ *   `splits` splits on `num_sms` SMs (every sequence Skv keys); < 0 on bad sizes.
+ */
+typedef struct {
+  int bm, bn, q_tiles, kv_slots, b_lm, b_ms, smem_bytes, tmem_cols;
+  double t_load_ns, t_mma_ns, t_softmax_ns, t_iter_ns;
+} loom_fwd_plan;
+loom_status loom_model_fwd_plan(int D, loom_fwd_plan* out);
+double loom_model_fwd_time_us(int B, int Hq, int Sq, int Skv, int D, int causal);
+double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms);
+
+/*
  * Synchronises `stream`, then reads and clears the current device's error word.
  * Returns LOOM_OK, LOOM_ERR_TIMEOUT if a kernel abandoned a bounded wait since the last
  * check, or LOOM_ERR_CUDA if the synchronisation itself failed.

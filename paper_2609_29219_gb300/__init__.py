@@ -23,7 +23,8 @@ __all__ = [
     "LoomError", "capi", "library_path", "STATUS",
     "loom_attn_fwd", "loom_attn_decode", "loom_attn_decode_workspace_bytes",
     "loom_attn_decode_num_splits", "loom_attn_check_error", "loom_status_string",
-    "loom_debug_set_timeout_ns", "loom_debug_inject",
+    "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
+    "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -35,6 +36,16 @@ STATUS = {
     0: "LOOM_OK", 1: "LOOM_ERR_INVALID_ARG", 2: "LOOM_ERR_UNSUPPORTED", 3: "LOOM_ERR_MISALIGNED",
     4: "LOOM_ERR_WORKSPACE", 5: "LOOM_ERR_CUDA", 6: "LOOM_ERR_TIMEOUT",
 }
+
+
+class FwdPlan(ctypes.Structure):
+    """Mirror of ``loom_fwd_plan`` (include/loom_attn.h)."""
+    _fields_ = [(n, ctypes.c_int) for n in ("bm", "bn", "q_tiles", "kv_slots", "b_lm", "b_ms",
+                                             "smem_bytes", "tmem_cols")] + \
+               [(n, ctypes.c_double) for n in ("t_load_ns", "t_mma_ns", "t_softmax_ns", "t_iter_ns")]
+
+    def as_dict(self):
+        return {n: getattr(self, n) for n, _ in self._fields_}
 
 
 class LoomError(RuntimeError):
@@ -75,6 +86,12 @@ def capi() -> ctypes.CDLL:
             lib.loom_debug_set_timeout_ns.restype = None
             lib.loom_debug_inject.argtypes = [i32]
             lib.loom_debug_inject.restype = None
+            lib.loom_model_fwd_plan.argtypes = [i32, ctypes.POINTER(FwdPlan)]
+            lib.loom_model_fwd_plan.restype = i32
+            lib.loom_model_fwd_time_us.argtypes = [i32, i32, i32, i32, i32, i32]
+            lib.loom_model_fwd_time_us.restype = ctypes.c_double
+            lib.loom_model_decode_time_us.argtypes = [i32, i32, i32, i32, i32, i32, i32]
+            lib.loom_model_decode_time_us.restype = ctypes.c_double
             _lib = lib
     return _lib
 
@@ -188,8 +205,8 @@ def loom_attn_decode(q, k_cache, v_cache, seqlens_k=None, o=None, lse=None, work
         if lse.numel() != B * Hq:
             raise ValueError("lse must hold B*Hq values")
         lp = _dev_ptr(lse, "lse", torch.float32)
-    need = loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, num_splits)
     if workspace is None:
+        need = loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, num_splits)
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=q.device)
     wp = _dev_ptr(workspace, "workspace")
     if scale is None:
@@ -217,3 +234,17 @@ def loom_debug_set_timeout_ns(ns: int):
 
 def loom_debug_inject(mode: int):
     capi().loom_debug_inject(int(mode))
+
+
+def loom_model_fwd_plan(D: int) -> dict:
+    plan = FwdPlan()
+    _check(capi().loom_model_fwd_plan(int(D), ctypes.byref(plan)), "loom_model_fwd_plan")
+    return plan.as_dict()
+
+
+def loom_model_fwd_time_us(B, Hq, Sq, Skv, D, causal) -> float:
+    return float(capi().loom_model_fwd_time_us(B, Hq, Sq, Skv, D, int(bool(causal))))
+
+
+def loom_model_decode_time_us(splits, B, Hq, Hkv, Skv, D, num_sms) -> float:
+    return float(capi().loom_model_decode_time_us(splits, B, Hq, Hkv, Skv, D, num_sms))

@@ -5,6 +5,8 @@
 #include <cmath>
 #include <cstdint>
 #include <mutex>
+#include <utility>
+#include <vector>
 
 #include "../../include/loom_attn.h"
 #include "kernels.h"
@@ -44,6 +46,15 @@ int current_sm_count() {
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
   return sms;
 }
+
+struct SplitKey {
+  int B, Hq, Hkv, Skv, D, sms;
+  bool operator==(const SplitKey& o) const {
+    return B == o.B && Hq == o.Hq && Hkv == o.Hkv && Skv == o.Skv && D == o.D && sms == o.sms;
+  }
+};
+std::vector<std::pair<SplitKey, int>> g_split_cache;
+std::mutex g_split_mutex;
 
 bool make_ctl(KernelCtl* ctl) {
   ctl->err = error_word_ptr();
@@ -99,7 +110,18 @@ int loom_attn_decode_num_splits(int B, int Hq, int Hkv, int Skv, int D) {
   if (D != 64 && D != 128) return 0;
   int sms = current_sm_count();
   if (sms <= 0) sms = model::kGb300.num_sms;
-  return model::choose_decode_splits(B, Hq, Hkv, Skv, D, sms).splits;
+  // The enumeration costs ~0.1 ms of host time: remember the answer per problem shape.
+  const SplitKey key{B, Hq, Hkv, Skv, D, sms};
+  {
+    std::lock_guard<std::mutex> lock(g_split_mutex);
+    for (const auto& e : g_split_cache)
+      if (e.first == key) return e.second;
+  }
+  const int splits = model::choose_decode_splits(B, Hq, Hkv, Skv, D, sms).splits;
+  std::lock_guard<std::mutex> lock(g_split_mutex);
+  if (g_split_cache.size() >= 256) g_split_cache.erase(g_split_cache.begin());
+  g_split_cache.emplace_back(key, splits);
+  return splits;
 }
 
 size_t loom_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int Skv, int D, int num_splits) {
@@ -156,6 +178,37 @@ loom_status loom_attn_check_error(void* stream) {
     if (cudaMemcpy(p, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return LOOM_ERR_CUDA;
   }
   return (word & kErrTimeout) ? LOOM_ERR_TIMEOUT : LOOM_OK;
+}
+
+loom_status loom_model_fwd_plan(int D, loom_fwd_plan* out) {
+  if (!out) return LOOM_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return LOOM_ERR_UNSUPPORTED;
+  const model::FwdPlan p = model::fwd_plan(D);
+  out->bm = p.bm;
+  out->bn = p.bn;
+  out->q_tiles = p.q_tiles;
+  out->kv_slots = p.kv_slots;
+  out->b_lm = p.b_lm;
+  out->b_ms = p.b_ms;
+  out->smem_bytes = p.smem_bytes;
+  out->tmem_cols = p.tmem_cols;
+  out->t_load_ns = p.t_load_ns;
+  out->t_mma_ns = p.t_mma_ns;
+  out->t_softmax_ns = p.t_softmax_ns;
+  out->t_iter_ns = p.t_iter_ns;
+  return LOOM_OK;
+}
+
+double loom_model_fwd_time_us(int B, int Hq, int Sq, int Skv, int D, int causal) {
+  if (B <= 0 || Hq <= 0 || Sq <= 0 || Skv <= 0 || (D != 64 && D != 128)) return -1.0;
+  return model::fwd_time_us(model::fwd_plan(D), B, Hq, Sq, Skv, D, causal != 0);
+}
+
+double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms) {
+  if (splits <= 0 || B <= 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv || Skv <= 0 || num_sms <= 0 ||
+      (D != 64 && D != 128))
+    return -1.0;
+  return model::decode_time_us(splits, B, Hq, Hkv, Skv, D, num_sms);
 }
 
 void loom_debug_set_timeout_ns(uint64_t ns) { g_timeout_ns = ns ? ns : kDefaultTimeoutNs; }

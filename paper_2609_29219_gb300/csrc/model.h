@@ -34,11 +34,13 @@ struct ArchDesc {
   double mem_latency_ns;    // loaded HBM latency of a bulk copy (assumed)
   double sync_ns;           // fixed per-iteration cost of an mbarrier/TMEM round trip (assumed)
   double launch_ns;         // fixed cost of one dependent kernel launch (assumed)
+  double decode_cta_gbs;    // KV stream rate of a lone decode split CTA on an SM (measured)
+  double cta_start_ns;      // start-up of a decode split CTA: launch, first copies (measured)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
-    1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0,
+    1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -207,6 +209,11 @@ constexpr DecodeStagePlan decode_stage_plan(int D, const ArchDesc& a = kGb300) {
   return best;
 }
 
+// The stage plans of the two supported head dimensions, evaluated at compile time.
+inline constexpr DecodeStagePlan kDecodeStage64 = decode_stage_plan(64);
+inline constexpr DecodeStagePlan kDecodeStage128 = decode_stage_plan(128);
+constexpr const DecodeStagePlan& decode_stage(int D) { return D == 64 ? kDecodeStage64 : kDecodeStage128; }
+
 struct DecodeSplitPlan {
   int splits;
   double t_us;   // modeled split + merge time
@@ -216,27 +223,30 @@ struct DecodeSplitPlan {
 constexpr int decode_group_tile(int G) { return G >= 8 ? 8 : G >= 4 ? 4 : G >= 2 ? 2 : 1; }
 
 // Eq. 5 for Flash Decode: T = T_split-loop ; T_merge (gather + global softmax + scale).
-// The split loop is Eq. 6-7 with an open load boundary (the ring keeps copies in
-// flight), so a CTA streams its chunk at its share of HBM bandwidth, capped by the
-// bytes it can keep in flight (Little's law); CTAs run in waves of num_sms * CTAs/SM.
+// The split loop is Eq. 6-7 with an open load boundary, evaluated on the busiest SM:
+// it runs ceil(CTAs / SMs) split CTAs in rounds of at most CTAs-per-SM at a time; a
+// round of k CTAs streams at min(the SM's share of HBM / k, the rate one CTA sustains),
+// and each round pays the CTA start-up (launch and first copies).
 constexpr double decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms,
                                 const ArchDesc& a = kGb300) {
-  const DecodeStagePlan sp = decode_stage_plan(D, a);
+  const DecodeStagePlan& sp = decode_stage(D);
   const int G = Hq / Hkv;
   const int gt = decode_group_tile(G);
   const long long units = 1LL * B * Hkv * cdiv(G, gt);
   const long long ctas = units * splits;
-  const long long slots = 1LL * num_sms * sp.ctas_per_sm;
   const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
-  const double active = static_cast<double>(ctas < slots ? ctas : slots);
-  const double in_flight_cta = 2.0 * sp.tokens * D * 2 * (sp.stages - 1);
-  double bw_cta = a.hbm_gbs / active;                 // bytes/ns
-  const double cap = in_flight_cta / a.mem_latency_ns;
-  if (bw_cta > cap) bw_cta = cap;
-  const double stages = static_cast<double>(cdiv(chunk, sp.tokens));
-  const double t_cta = heg_seq(a.mem_latency_ns, heg_for(stages, 2.0 * sp.tokens * D * 2 / bw_cta));
-  const double waves = static_cast<double>(cdiv(ctas, slots));
-  const double t_split = waves * t_cta;
+  const double chunk_bytes = 2.0 * chunk * D * 2;
+  const long long per_sm = cdiv(ctas, num_sms);
+  const double active_sms = static_cast<double>(ctas < num_sms ? ctas : num_sms);
+  const double share = a.hbm_gbs / active_sms;  // bytes/ns for one SM
+  double t_split = 0.0;
+  for (long long left = per_sm; left > 0;) {
+    const long long k = left < sp.ctas_per_sm ? left : sp.ctas_per_sm;
+    left -= k;
+    double bw = share / static_cast<double>(k);
+    if (bw > a.decode_cta_gbs) bw = a.decode_cta_gbs;
+    t_split += heg_seq(a.cta_start_ns, chunk_bytes / bw);
+  }
   const double part_bytes = 1.0 * B * Hq * splits * (D + 1) * 4;
   const double t_merge = a.launch_ns * 0.2 + 2.0 * part_bytes / a.hbm_gbs;
   return heg_seq(t_split, t_merge) * 1e-3;
