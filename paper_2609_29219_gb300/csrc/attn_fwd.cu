@@ -50,7 +50,7 @@ struct FwdCfg {
   static constexpr int BN = kPlan.bn;         // keys per KV tile
   static constexpr int NSLOT = kPlan.kv_slots;  // K/V ring slots
   static_assert(BM == 128 && NQT == 2, "warp roles assume two 128-row query tiles");
-  static_assert(BN % 64 == 0 && BN <= 128, "softmax holds one S row of <= 128 fp32 in registers");
+  static_assert(BN == 128, "softmax holds one S row of 128 fp32 in registers, P leaves in two 64-key halves");
   static_assert(kPlan.b_lm == 1 && NSLOT >= 4, "the loader runs ahead of the MMA by >= one tile");
   static constexpr int THREADS = 320;               // 8 softmax warps + loader + MMA
   static constexpr int BOX_COLS = 64;               // 128-byte swizzle atom = 64 bf16
@@ -62,8 +62,8 @@ struct FwdCfg {
   static constexpr uint32_t Q_OFF = 0;
   static constexpr uint32_t RING_OFF = NQT * Q_TILE_BYTES;
   static constexpr uint32_t BAR_OFF = RING_OFF + NSLOT * SLOT_BYTES;
-  // barriers: q_full, full[NSLOT], empty[NSLOT], s_full[2], p_full[2], o_full[2], drain
-  static constexpr int NBAR = 1 + 2 * NSLOT + 7;
+  // barriers: q_full, q_empty, full[NSLOT], empty[NSLOT], s[2], p[2][2], o[2], o_empty[2], drain
+  static constexpr int NBAR = 2 + 2 * NSLOT + 11;
   static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
   static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
   static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;  // + alignment slack
@@ -79,11 +79,56 @@ struct FwdParams {
   float* lse;
   int Hq, Hkv, Sq, Skv;
   int n_pairs;   // query-tile pairs per (b, h)
+  int n_items;   // n_pairs * B * Hq work items
   int causal;
-  int heavy_first;
   float c;       // scale * log2(e)
   KernelCtl ctl;
 };
+
+// One work item of a persistent CTA: a pair of 128-row query tiles of one (b, h).
+struct Item {
+  int b, h, q_z, kv_z, q0, n_tiles0, n_tiles;
+};
+
+// The r-th item of this CTA (-1 once it has none left).  Causal items are ordered
+// heaviest first and dealt out in a snake order (CTA c takes item c of even rounds and
+// item G-1-c of odd rounds) so that long and short items even out per CTA.
+__device__ __forceinline__ int item_index(const FwdParams& p, int r) {
+  const int G = static_cast<int>(gridDim.x), c = static_cast<int>(blockIdx.x);
+  const long long idx = static_cast<long long>(r) * G + ((p.causal && (r & 1)) ? G - 1 - c : c);
+  return idx < p.n_items ? static_cast<int>(idx) : -1;
+}
+
+template <int D>
+__device__ __forceinline__ Item make_item(const FwdParams& p, int idx) {
+  using C = FwdCfg<D>;
+  const int BH = p.n_items / p.n_pairs;
+  int pair, bh;
+  if (p.causal) {  // the longest (bottom) tile pairs of every head go first
+    pair = p.n_pairs - 1 - idx / BH;
+    bh = idx % BH;
+  } else {         // consecutive items share K/V of one head in L2
+    pair = idx % p.n_pairs;
+    bh = idx / p.n_pairs;
+  }
+  Item it;
+  it.h = bh % p.Hq;
+  it.b = bh / p.Hq;
+  it.q_z = bh;
+  it.kv_z = it.b * p.Hkv + it.h / (p.Hq / p.Hkv);
+  it.q0 = pair * (C::NQT * C::BM);
+  // KV tiles each query tile needs (causal: up to the diagonal of its last row); the
+  // CTA loads the union, i.e. tile 1's range.
+  const int off = p.Skv - p.Sq;  // bottom-right causal offset
+  int n_kv0 = p.Skv, n_kv1 = p.Skv;
+  if (p.causal) {
+    n_kv0 = min(p.Skv, it.q0 + C::BM + off);
+    n_kv1 = min(p.Skv, it.q0 + 2 * C::BM + off);
+  }
+  it.n_tiles0 = (n_kv0 + C::BN - 1) / C::BN;
+  it.n_tiles = (n_kv1 + C::BN - 1) / C::BN;
+  return it;
+}
 
 template <int D>
 __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
@@ -95,52 +140,33 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
   const uint32_t raw_base = smem_u32(smem_raw);
   const uint32_t sbase = (raw_base + 1023u) & ~1023u;
   uint8_t* smem = smem_raw + (sbase - raw_base);
-
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int BH = gridDim.x / p.n_pairs;
-  int pair, bh;
-  if (p.heavy_first) {  // causal: the longest (bottom) tile pairs of every head go first
-    pair = p.n_pairs - 1 - static_cast<int>(blockIdx.x) / BH;
-    bh = static_cast<int>(blockIdx.x) % BH;
-  } else {              // consecutive CTAs share K/V of one head in L2
-    pair = static_cast<int>(blockIdx.x) % p.n_pairs;
-    bh = static_cast<int>(blockIdx.x) / p.n_pairs;
-  }
-  const int h = bh % p.Hq, b = bh / p.Hq;
-  const int hk = h / (p.Hq / p.Hkv);
-  const int kv_z = b * p.Hkv + hk;
-  const int q0 = pair * (C::NQT * C::BM);
-  const int off = p.Skv - p.Sq;  // bottom-right causal offset
-  // KV tiles each query tile needs (causal: up to the diagonal of its last row); the
-  // CTA loads the union, i.e. tile 1's range.
-  int n_kv0 = p.Skv, n_kv1 = p.Skv;
-  if (p.causal) {
-    n_kv0 = min(p.Skv, q0 + C::BM + off);
-    n_kv1 = min(p.Skv, q0 + 2 * C::BM + off);
-  }
-  const int n_tiles0 = (n_kv0 + C::BN - 1) / C::BN;
-  const int n_tiles = (n_kv1 + C::BN - 1) / C::BN;
 
-  const uint32_t bar_q = sbase + C::BAR_OFF;
-  const uint32_t bar_full = bar_q + 8;
+  const uint32_t bar_q = sbase + C::BAR_OFF;       // Q tiles loaded (once per item)
+  const uint32_t bar_qe = bar_q + 8;               // Q tiles no longer read (once per item)
+  const uint32_t bar_full = bar_qe + 8;            // [NSLOT]
   const uint32_t bar_empty = bar_full + 8 * C::NSLOT;
-  const uint32_t bar_s = bar_empty + 8 * C::NSLOT;  // [2]
-  const uint32_t bar_p = bar_s + 16;                 // [2]
-  const uint32_t bar_o = bar_p + 16;                 // [2]
-  const uint32_t bar_drain = bar_o + 16;
+  const uint32_t bar_s = bar_empty + 8 * C::NSLOT;  // [2] S_t ready
+  const uint32_t bar_p = bar_s + 16;                // [2][2] half h of P_t written (h = 0: and O_t rescaled)
+  const uint32_t bar_o = bar_p + 32;                // [2] P_t V_j accumulated into O_t
+  const uint32_t bar_oe = bar_o + 16;               // [2] O_t read out by the epilogue
+  const uint32_t bar_drain = bar_oe + 16;
   uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::TMEM_PTR_OFF);
   Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
 
   if (threadIdx.x == 0) {
     mbar_init(bar_q, 1);
+    mbar_init(bar_qe, 1);
     for (int s = 0; s < C::NSLOT; ++s) {
       mbar_init(bar_full + 8 * s, 1);
       mbar_init(bar_empty + 8 * s, 1);
     }
     for (int t = 0; t < 2; ++t) {
       mbar_init(bar_s + 8 * t, 1);
-      mbar_init(bar_p + 8 * t, C::BM);
+      mbar_init(bar_p + 16 * t, C::BM);
+      mbar_init(bar_p + 16 * t + 8, C::BM);
       mbar_init(bar_o + 8 * t, 1);
+      mbar_init(bar_oe + 8 * t, C::BM);
     }
     mbar_init(bar_drain, 1);
     *ab.flag = 0;
@@ -159,100 +185,126 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
       prefetch_tensormap(&tm_q);
       prefetch_tensormap(&tm_k);
       prefetch_tensormap(&tm_v);
-      const int q_z = b * p.Hq + h;
-      mbar_expect_tx(bar_q, C::NQT * C::Q_TILE_BYTES);
-      for (int t = 0; t < C::NQT; ++t)
-        for (int x = 0; x < C::NBOX; ++x)
-          tma_load_3d(sbase + C::Q_OFF + t * C::Q_TILE_BYTES + x * C::Q_BOX_BYTES, &tm_q,
-                      x * C::BOX_COLS, q0 + t * C::BM, q_z, bar_q);
-      int issued = 0, skipped = -1;
-      for (int pos = 0; pos < 2 * n_tiles; ++pos) {  // K_0, V_0, K_1, V_1, ...
-        const int slot = pos % C::NSLOT, round = pos / C::NSLOT;
-        if (!mbar_wait(bar_empty + 8 * slot, (round & 1) ^ 1, p.ctl, ab)) break;
-        issued = pos + 1;
-        if (p.ctl.inject == 2 && pos == 2) {  // test hook: never load K_1
-          skipped = pos;
-          continue;
+      int pos = 0, issued = 0, skipped = -1, q_issued = 0;
+      bool ok = true;
+      for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+        const Item it = make_item<D>(p, idx);
+        // the previous item's S MMAs must be done with the Q tiles
+        if (r > 0 && !(ok = mbar_wait(bar_qe, (r - 1) & 1, p.ctl, ab))) break;
+        mbar_expect_tx(bar_q, C::NQT * C::Q_TILE_BYTES);
+        for (int t = 0; t < C::NQT; ++t)
+          for (int x = 0; x < C::NBOX; ++x)
+            tma_load_3d(sbase + C::Q_OFF + t * C::Q_TILE_BYTES + x * C::Q_BOX_BYTES, &tm_q,
+                        x * C::BOX_COLS, it.q0 + t * C::BM, it.q_z, bar_q);
+        q_issued = r + 1;
+        for (int jj = 0; jj < 2 * it.n_tiles; ++jj, ++pos) {  // K_0, V_0, K_1, V_1, ...
+          const int slot = pos % C::NSLOT, round = pos / C::NSLOT;
+          if (!(ok = mbar_wait(bar_empty + 8 * slot, (round & 1) ^ 1, p.ctl, ab))) break;
+          issued = pos + 1;
+          if (p.ctl.inject == 2 && pos == 2) {  // test hook: never load this tile
+            skipped = pos;
+            continue;
+          }
+          const CUtensorMap* map = (jj & 1) ? &tm_v : &tm_k;
+          const int row = (jj >> 1) * C::BN;
+          mbar_expect_tx(bar_full + 8 * slot, C::SLOT_BYTES);
+          for (int x = 0; x < C::NBOX; ++x)
+            tma_load_3d(sbase + C::RING_OFF + slot * C::SLOT_BYTES + x * C::KV_BOX_BYTES, map,
+                        x * C::BOX_COLS, row, it.kv_z, bar_full + 8 * slot);
         }
-        const CUtensorMap* map = (pos & 1) ? &tm_v : &tm_k;
-        const int row = (pos >> 1) * C::BN;
-        mbar_expect_tx(bar_full + 8 * slot, C::SLOT_BYTES);
-        for (int x = 0; x < C::NBOX; ++x)
-          tma_load_3d(sbase + C::RING_OFF + slot * C::SLOT_BYTES + x * C::KV_BOX_BYTES, map,
-                      x * C::BOX_COLS, row, kv_z, bar_full + 8 * slot);
       }
       // drain copies still in flight before the CTA may exit
       Abort no_abort{ab.flag + 1};
-      mbar_wait(bar_q, 0, p.ctl, no_abort);
-      for (int pos = max(0, issued - C::NSLOT); pos < issued; ++pos)
-        if (pos != skipped)
-          mbar_wait(bar_full + 8 * (pos % C::NSLOT), (pos / C::NSLOT) & 1, p.ctl, no_abort);
+      if (q_issued > 0) mbar_wait(bar_q, (q_issued - 1) & 1, p.ctl, no_abort);
+      for (int ps = max(0, issued - C::NSLOT); ps < issued; ++ps)
+        if (ps != skipped)
+          mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, no_abort);
     }
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc_s = idesc_bf16(C::BM, C::BN, 0, 0);  // Q, K both K-major
       constexpr uint32_t idesc_pv = idesc_bf16(C::BM, D, 0, 1);     // P from TMEM, V MN-major
-      auto slot_addr = [&](int pos) { return sbase + C::RING_OFF + (pos % C::NSLOT) * C::SLOT_BYTES; };
-      auto wait_slot = [&](int pos) {
-        return mbar_wait(bar_full + 8 * (pos % C::NSLOT), (pos / C::NSLOT) & 1, p.ctl, ab);
+      auto wait_slot = [&](int ps) {
+        return mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, ab);
       };
+      // Base descriptors, built once: Q tile t, and ring slot s read as K (K-major) or V
+      // (MN-major); a slot or box step is a constant added to the start-address field.
+      const uint64_t dq0 = sdesc_sw128(sbase + C::Q_OFF, 16, 1024);
+      const uint64_t dk0 = sdesc_sw128(sbase + C::RING_OFF, 16, 1024);
+      const uint64_t dv0 = sdesc_sw128(sbase + C::RING_OFF, C::KV_BOX_BYTES, 1024);
+      constexpr uint32_t kSlot16 = C::SLOT_BYTES >> 4, kQTile16 = C::Q_TILE_BYTES >> 4;
+      constexpr uint32_t kQBox16 = C::Q_BOX_BYTES >> 4, kKBox16 = C::KV_BOX_BYTES >> 4;
+      // S_t = Q_t K^T over K = D in 64-wide boxes
       auto issue_s = [&](int t, int kpos) {
-        const uint32_t qa = sbase + C::Q_OFF + t * C::Q_TILE_BYTES;
-        const uint32_t ka = slot_addr(kpos);
+        const uint64_t a = dq0 + t * kQTile16;
+        const uint64_t b = dk0 + (kpos % C::NSLOT) * kSlot16;
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t koff = (kk / 4) * C::Q_BOX_BYTES + (kk % 4) * 32;
-          const uint32_t kvoff = (kk / 4) * C::KV_BOX_BYTES + (kk % 4) * 32;
-          mma_ss(tmem + C::S_COL + t * C::BN, sdesc_sw128(qa + koff, 16, 1024),
-                 sdesc_sw128(ka + kvoff, 16, 1024), idesc_s, kk > 0);
-        }
+        for (int x = 0; x < C::NBOX; ++x)
+          mma_ss_k64(tmem + C::S_COL + t * C::BN, a + x * kQBox16, b + x * kKBox16, idesc_s, x > 0);
       };
-      auto issue_pv = [&](int t, int vpos, bool acc) {
-        const uint32_t va = slot_addr(vpos);
-#pragma unroll
-        for (int kk = 0; kk < C::BN / 16; ++kk)
-          mma_ts(tmem + C::O_COL + t * D, tmem + C::S_COL + t * C::BN + kk * 8,
-                 sdesc_sw128(va + kk * 16 * 128, C::KV_BOX_BYTES, 1024), idesc_pv,
-                 (acc || kk > 0) ? 1u : 0u);
+      // O_t += P_t[:, half] V_j[half, :] over K = BN/2 keys
+      auto issue_pv = [&](int t, int vpos, bool acc, int half) {
+        const uint64_t b = dv0 + (vpos % C::NSLOT) * kSlot16 + half * (C::BN / 2) * (128 >> 4);
+        static_assert(C::BN / 2 == 64, "a half of P is one 64-key block of four K-steps");
+        mma_ts_k64(tmem + C::O_COL + t * D, tmem + C::S_COL + t * C::BN + half * (C::BN / 4), b, idesc_pv,
+                   acc ? 1u : 0u);
       };
-      bool ok = mbar_wait(bar_q, 0, p.ctl, ab) && wait_slot(0);
-      if (ok) {
+      int pos = 0, cnt0 = 0, cnt1 = 0;  // ring position of K_0; S/P/O uses so far per tile
+      bool ok = true;
+      for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+        const Item it = make_item<D>(p, idx);
+        const int nt0 = it.n_tiles0, nt = it.n_tiles;
+        if (!(ok = mbar_wait(bar_q, r & 1, p.ctl, ab) && wait_slot(pos))) break;
         tc_fence_after();
-        issue_s(0, 0);
+        issue_s(0, pos);
         tc_commit(bar_s);
-        issue_s(1, 0);
+        issue_s(1, pos);
         tc_commit(bar_s + 8);
-        tc_commit(bar_empty + 8 * (0 % C::NSLOT));
-      }
-      for (int j = 0; ok && j < n_tiles; ++j) {
-        const int vpos = 2 * j + 1, kpos = 2 * j + 2;
-        const bool more = j + 1 < n_tiles;
-        if (!(ok = wait_slot(vpos))) break;
-        if (j < n_tiles0) {  // query tile 0 stops at its own diagonal
-          if (!(ok = mbar_wait(bar_p, j & 1, p.ctl, ab))) break;
+        tc_commit(bar_empty + 8 * (pos % C::NSLOT));
+        if (nt == 1) tc_commit(bar_qe);  // every S of this item issued
+        for (int j = 0; j < nt; ++j) {
+          const int vpos = pos + 2 * j + 1, kpos = pos + 2 * j + 2;
+          const bool more = j + 1 < nt;
+          if (!(ok = wait_slot(vpos))) break;
+          if (j < nt0) {  // query tile 0 stops at its own diagonal
+            if (!(ok = mbar_wait(bar_p, (cnt0 + j) & 1, p.ctl, ab))) break;
+            // O_0 of the previous item must have been read out
+            if (j == 0 && r > 0 && !(ok = mbar_wait(bar_oe, (r - 1) & 1, p.ctl, ab))) break;
+            tc_fence_after();
+            issue_pv(0, vpos, j > 0, 0);
+            if (!(ok = mbar_wait(bar_p + 8, (cnt0 + j) & 1, p.ctl, ab))) break;
+            tc_fence_after();
+            issue_pv(0, vpos, true, 1);
+            tc_commit(bar_o);
+          }
+          if (more) {
+            if (!(ok = wait_slot(kpos))) break;
+            tc_fence_after();
+            if (j + 1 < nt0) {
+              issue_s(0, kpos);
+              tc_commit(bar_s);
+            }
+          }
+          if (!(ok = mbar_wait(bar_p + 16, (cnt1 + j) & 1, p.ctl, ab))) break;
+          if (j == 0 && r > 0 && !(ok = mbar_wait(bar_oe + 8, (r - 1) & 1, p.ctl, ab))) break;
           tc_fence_after();
-          issue_pv(0, vpos, j > 0);
-          tc_commit(bar_o);
-        }
-        if (more) {
-          if (!(ok = wait_slot(kpos))) break;
+          issue_pv(1, vpos, j > 0, 0);
+          if (!(ok = mbar_wait(bar_p + 24, (cnt1 + j) & 1, p.ctl, ab))) break;
           tc_fence_after();
-          if (j + 1 < n_tiles0) {
-            issue_s(0, kpos);
-            tc_commit(bar_s);
+          issue_pv(1, vpos, true, 1);
+          tc_commit(bar_o + 8);
+          tc_commit(bar_empty + 8 * (vpos % C::NSLOT));
+          if (more) {
+            issue_s(1, kpos);
+            tc_commit(bar_s + 8);
+            tc_commit(bar_empty + 8 * (kpos % C::NSLOT));
+            if (j + 2 == nt) tc_commit(bar_qe);  // that was the item's last S
           }
         }
-        if (!(ok = mbar_wait(bar_p + 8, j & 1, p.ctl, ab))) break;
-        tc_fence_after();
-        issue_pv(1, vpos, j > 0);
-        tc_commit(bar_o + 8);
-        tc_commit(bar_empty + 8 * (vpos % C::NSLOT));
-        if (more) {
-          issue_s(1, kpos);
-          tc_commit(bar_s + 8);
-          tc_commit(bar_empty + 8 * (kpos % C::NSLOT));
-        }
+        cnt0 += nt0;
+        cnt1 += nt;
+        pos += 2 * nt;
       }
       // wait for every MMA issued above before TMEM may be released
       Abort no_abort{ab.flag + 1};
@@ -263,119 +315,129 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
     // ------------------------------------------------------------------ softmax
     const int t = warp >> 2;                        // query tile of this warpgroup
     const int row_in_tile = (warp & 3) * 32 + lane;  // == TMEM lane
-    const int row = q0 + t * C::BM + row_in_tile;
     const uint32_t lane_addr = static_cast<uint32_t>((warp & 3) * 32) << 16;
     const uint32_t s_tm = tmem + lane_addr + C::S_COL + t * C::BN;
     const uint32_t o_tm = tmem + lane_addr + C::O_COL + t * D;
-    const uint32_t my_bar_s = bar_s + 8 * t, my_bar_p = bar_p + 8 * t, my_bar_o = bar_o + 8 * t;
-    const int limit = p.causal ? min(p.Skv, row + off + 1) : p.Skv;  // keys [0, limit) visible
-    const int my_tiles = t == 0 ? n_tiles0 : n_tiles;
+    const uint32_t my_bar_s = bar_s + 8 * t, my_bar_p = bar_p + 16 * t, my_bar_o = bar_o + 8 * t;
+    const uint32_t my_bar_oe = bar_oe + 8 * t;
     const float c = p.c;
     const uint64_t c2 = f2(c, c);
+    const int off = p.Skv - p.Sq;
 
-    float m_run = -INFINITY, l_run = 0.f;
+    int cnt = 0;  // S tiles of this query tile processed in earlier items
     bool ok = true;
-    for (int j = 0; j < my_tiles; ++j) {
-      if (!(ok = mbar_wait_warp(my_bar_s, j & 1, p.ctl, ab))) break;
-      tc_fence_after();
-      uint32_t s[C::BN];
-#pragma unroll
-      for (int ch = 0; ch < C::BN / 32; ++ch) tmem_ld32(s_tm + ch * 32, s + ch * 32);
-      tmem_wait_ld();
-#pragma unroll
-      for (int ch = 0; ch < C::BN / 32; ++ch) reg_fence32(s + ch * 32);
-      const int kbase = j * C::BN;
-      if (kbase + C::BN > limit) {
-#pragma unroll
-        for (int i = 0; i < C::BN; ++i)
-          if (kbase + i >= limit) s[i] = __float_as_uint(-INFINITY);
-      }
-      // row max: 8 independent chains of 3-input max, then a small tree
-      float mx;
-      {
-        float mm[8];
-#pragma unroll
-        for (int g = 0; g < 8; ++g) mm[g] = __uint_as_float(s[g]);
-#pragma unroll
-        for (int i = 8; i + 16 <= C::BN; i += 16)
-#pragma unroll
-          for (int g = 0; g < 8; ++g)
-            mm[g] = max3(mm[g], __uint_as_float(s[i + g]), __uint_as_float(s[i + 8 + g]));
-        if constexpr ((C::BN - 8) % 16 != 0) {
-#pragma unroll
-          for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], __uint_as_float(s[C::BN - 8 + g]));
-        }
-        mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
-      }
-      const float m_new = fmaxf(m_run, mx * c);
-      const bool need = m_new > m_run + kRescaleThreshold;
-      const float alpha = need ? ex2(m_run - m_new) : 1.f;
-      if (need) m_run = m_new;
-      const float ms = (m_run == -INFINITY) ? 0.f : m_run;
-      const uint64_t nms2 = f2(-ms, -ms);
-      // p = 2^(s*c - m): packed FMA, one MUFU ex2 per score, 4 packed partial sums
-      uint64_t acc[4] = {0, 0, 0, 0};
-      uint32_t pk[C::BN / 2];
-#pragma unroll
-      for (int i = 0; i < C::BN / 2; ++i) {
-        const uint64_t x = fma2(f2(__uint_as_float(s[2 * i]), __uint_as_float(s[2 * i + 1])), c2, nms2);
-        const float p0 = ex2(f2lo(x));
-        const float p1 = ex2(f2hi(x));
-        acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
-        pk[i] = pack_bf16x2(p0, p1);
-      }
-#pragma unroll
-      for (int ch = 0; ch < C::BN / 64; ++ch) tmem_st32(s_tm + ch * 32, pk + ch * 32);
-      const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
-      const float rs = f2lo(a01) + f2hi(a01);
-      tmem_wait_st();
-      l_run = l_run * alpha + rs;
-      // O_t must hold P_{j-1} V_{j-1} before it is rescaled, and be rescaled before
-      // P_j V_j is issued (i.e. before the P-ready arrive below).  Done after P is
-      // written so that the S row is no longer live in registers.
-      if (j > 0 && __any_sync(0xffffffffu, need)) {
-        if (!(ok = mbar_wait_warp(my_bar_o, (j - 1) & 1, p.ctl, ab))) break;
+    for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+      const Item it = make_item<D>(p, idx);
+      const int row = it.q0 + t * C::BM + row_in_tile;
+      const int limit = p.causal ? min(p.Skv, row + off + 1) : p.Skv;  // keys [0, limit) visible
+      const int my_tiles = t == 0 ? it.n_tiles0 : it.n_tiles;
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int j = 0; j < my_tiles; ++j) {
+        if (!(ok = mbar_wait_warp(my_bar_s, (cnt + j) & 1, p.ctl, ab))) break;
         tc_fence_after();
-        const uint64_t a2 = f2(alpha, alpha);
-#pragma unroll 1
-        for (int ch = 0; ch < D / 32; ++ch) {
-          uint32_t r[32];
-          tmem_ld32(o_tm + ch * 32, r);
-          tmem_wait_ld();
-          reg_fence32(r);
+        uint32_t s[C::BN];
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const uint64_t x = mul2(f2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1])), a2);
-            r[2 * i] = __float_as_uint(f2lo(x));
-            r[2 * i + 1] = __float_as_uint(f2hi(x));
-          }
-          tmem_st32(o_tm + ch * 32, r);
+        for (int ch = 0; ch < C::BN / 32; ++ch) tmem_ld32(s_tm + ch * 32, s + ch * 32);
+        tmem_wait_ld();
+#pragma unroll
+        for (int ch = 0; ch < C::BN / 32; ++ch) reg_fence32(s + ch * 32);
+        const int kbase = j * C::BN;
+        if (kbase + C::BN > limit) {
+#pragma unroll
+          for (int i = 0; i < C::BN; ++i)
+            if (kbase + i >= limit) s[i] = __float_as_uint(-INFINITY);
         }
-        tmem_wait_st();
+        // row max: 8 independent chains of 3-input max, then a small tree
+        float mx;
+        {
+          float mm[8];
+#pragma unroll
+          for (int g = 0; g < 8; ++g) mm[g] = __uint_as_float(s[g]);
+#pragma unroll
+          for (int i = 8; i + 16 <= C::BN; i += 16)
+#pragma unroll
+            for (int g = 0; g < 8; ++g)
+              mm[g] = max3(mm[g], __uint_as_float(s[i + g]), __uint_as_float(s[i + 8 + g]));
+          if constexpr ((C::BN - 8) % 16 != 0) {
+#pragma unroll
+            for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], __uint_as_float(s[C::BN - 8 + g]));
+          }
+          mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
+        }
+        const float m_new = fmaxf(m_run, mx * c);
+        const bool need = m_new > m_run + kRescaleThreshold;
+        const float alpha = need ? ex2(m_run - m_new) : 1.f;
+        if (need) m_run = m_new;
+        const float ms = (m_run == -INFINITY) ? 0.f : m_run;
+        const uint64_t nms2 = f2(-ms, -ms);
+        // p = 2^(s*c - m): packed FMA, one MUFU ex2 per score, 4 packed partial sums.
+        // P goes out in two halves so that P[:, :BN/2] V can run while the second half
+        // of the exponentials is computed.
+        uint64_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          uint32_t pk[C::BN / 4];
+#pragma unroll
+          for (int i = 0; i < C::BN / 4; ++i) {
+            const int e = half * (C::BN / 2) + 2 * i;
+            const uint64_t x = fma2(f2(__uint_as_float(s[e]), __uint_as_float(s[e + 1])), c2, nms2);
+            const float p0 = ex2(f2lo(x));
+            const float p1 = ex2(f2hi(x));
+            acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
+            pk[i] = pack_bf16x2(p0, p1);
+          }
+#pragma unroll
+          for (int ch = 0; ch < C::BN / 128; ++ch)
+            tmem_st32(s_tm + half * (C::BN / 4) + ch * 32, pk + ch * 32);
+          tmem_wait_st();
+          // O_t must hold P_{j-1} V_{j-1} before it is rescaled, and be rescaled before
+          // P_j V_j starts (the first-half arrive below).
+          if (half == 0 && j > 0 && __any_sync(0xffffffffu, need)) {
+            if (!(ok = mbar_wait_warp(my_bar_o, (cnt + j - 1) & 1, p.ctl, ab))) break;
+            tc_fence_after();
+            const uint64_t a2 = f2(alpha, alpha);
+#pragma unroll 1
+            for (int ch = 0; ch < D / 32; ++ch) {
+              uint32_t rr[32];
+              tmem_ld32(o_tm + ch * 32, rr);
+              tmem_wait_ld();
+              reg_fence32(rr);
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                const uint64_t x = mul2(f2(__uint_as_float(rr[2 * i]), __uint_as_float(rr[2 * i + 1])), a2);
+                rr[2 * i] = __float_as_uint(f2lo(x));
+                rr[2 * i + 1] = __float_as_uint(f2hi(x));
+              }
+              tmem_st32(o_tm + ch * 32, rr);
+            }
+            tmem_wait_st();
+          }
+          tc_fence_before();
+          mbar_arrive(my_bar_p + 8 * half);
+        }
+        if (!ok) break;
+        const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+        l_run = l_run * alpha + (f2lo(a01) + f2hi(a01));
       }
-      tc_fence_before();
-      mbar_arrive(my_bar_p);
-    }
+      if (!ok) break;
 
-    // epilogue: O / l -> bf16 rows, LSE
-    if (ok && my_tiles > 0) ok = mbar_wait_warp(my_bar_o, (my_tiles - 1) & 1, p.ctl, ab);
-    if (ok) {
+      // epilogue: O / l -> bf16 rows, LSE; then hand O_t back to the MMA warp
+      if (!(ok = mbar_wait_warp(my_bar_o, (cnt + my_tiles - 1) & 1, p.ctl, ab))) break;
       tc_fence_after();
       const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
       const bool store = row < p.Sq;
-      __nv_bfloat16* orow =
-          p.o + ((static_cast<size_t>(b) * p.Hq + h) * p.Sq + (store ? row : 0)) * D;
+      __nv_bfloat16* orow = p.o + (static_cast<size_t>(it.q_z) * p.Sq + (store ? row : 0)) * D;
+      const uint64_t il2 = f2(inv_l, inv_l);
 #pragma unroll 1
       for (int ch = 0; ch < D / 32; ++ch) {
-        uint32_t r[32];
-        tmem_ld32(o_tm + ch * 32, r);
+        uint32_t rr[32];
+        tmem_ld32(o_tm + ch * 32, rr);
         tmem_wait_ld();
-        reg_fence32(r);
+        reg_fence32(rr);
         uint32_t w[16];
-        const uint64_t il2 = f2(inv_l, inv_l);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const uint64_t x = mul2(f2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1])), il2);
+          const uint64_t x = mul2(f2(__uint_as_float(rr[2 * i]), __uint_as_float(rr[2 * i + 1])), il2);
           w[i] = pack_bf16x2(f2lo(x), f2hi(x));
         }
         if (store) {
@@ -384,9 +446,12 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
           for (int i = 0; i < 4; ++i) dst[i] = make_uint4(w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
         }
       }
+      tc_fence_before();
+      mbar_arrive(my_bar_oe);
       if (store && p.lse)
-        p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.Sq + row] =
+        p.lse[static_cast<size_t>(it.q_z) * p.Sq + row] =
             l_run > 0.f ? (m_run + log2f(l_run)) * kLn2 : -INFINITY;
+      cnt += my_tiles;
     }
   }
 
@@ -460,12 +525,17 @@ cudaError_t launch_fwd_d(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t st
   p.Skv = a.Skv;
   p.n_pairs = (a.Sq + C::NQT * C::BM - 1) / (C::NQT * C::BM);
   p.causal = a.causal;
-  p.heavy_first = a.causal;
   p.c = a.scale * kLog2e;
   p.ctl = ctl;
-  const long long grid = static_cast<long long>(p.n_pairs) * a.B * a.Hq;
-  if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  attn_fwd_kernel<D><<<static_cast<unsigned>(grid), C::THREADS, C::BYTES, stream>>>(mq, mk, mv, p);
+  const long long items = static_cast<long long>(p.n_pairs) * a.B * a.Hq;
+  if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  p.n_items = static_cast<int>(items);
+  // persistent: one CTA per SM (shared memory admits one), each walking its items
+  int sms = 0;
+  cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const int grid = static_cast<int>(items < sms ? items : sms);
+  attn_fwd_kernel<D><<<grid, C::THREADS, C::BYTES, stream>>>(mq, mk, mv, p);
   return cudaGetLastError();
 }
 
