@@ -1,0 +1,313 @@
+// Architecture microbenchmarks for the analytic schedule model (the paper's Sec. 2.7:
+// performance properties of an architecture are characterised once, by isolated
+// microbenchmarks, and reused across operators and shapes).
+//
+// Built as a standalone program (paper_2609_29219_gb300/arch_probe.py builds and runs it)
+// and printing one JSON object:
+//   pipes : ex2.approx / fma.rn.f32 / fma.rn.f32x2 instruction-lanes per clock per SM
+//   mma   : clocks per tcgen05.mma kind::f16 128xNx16 (SS with N = 64, 128, 256; TS N = 128)
+//   mix   : clocks per 128x128x128 GEMM of the prefill kernel's MMA stream (P.V as TS,
+//           S = Q.K^T as SS, two query tiles) alone and under added load: bulk copies,
+//           TMEM loads/stores, commits, fences, random operands, and neighbour warps that
+//           keep the issue ports busy.
+// Every kernel runs one CTA per SM, touches only its own shared memory / TMEM and the
+// buffers allocated below, and bounds every wait.
+#include <cstdint>
+#include <cstdio>
+
+#include "ptx.cuh"
+
+namespace {
+using namespace loom;
+__device__ __forceinline__ float ex2f_(float x){float y; asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x)); return y;}
+template <int MODE>
+__global__ void pipe_kernel(float* out, long long* cyc, int iters) {
+  float v[8];
+  for (int i=0;i<8;i++) v[i] = -1e-3f * (threadIdx.x + i);
+  unsigned long long w[8];
+  for (int i=0;i<8;i++) { float a=v[i], b=v[i]*0.5f; asm("mov.b64 %0, {%1,%2};" : "=l"(w[i]) : "f"(a), "f"(b)); }
+  const unsigned long long m2 = 0x3f0000003f000000ull;  // (0.5, 0.5)
+  __syncthreads();
+  long long t0 = clock64();
+  for (int it = 0; it < iters; ++it) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      if (MODE == 0) v[i] = ex2f_(v[i]) - 1.5f;              // 1 MUFU + 1 FADD
+      if (MODE == 1) v[i] = fmaf(v[i], 0.999f, 1e-7f);       // 1 FFMA
+      if (MODE == 2) asm volatile("fma.rn.f32x2 %0, %0, %1, %1;" : "+l"(w[i]) : "l"(m2));  // 1 FFMA2
+    }
+  }
+  __syncthreads();
+  long long t1 = clock64();
+  float s = 0; for (int i=0;i<8;i++) s += v[i] + __uint_as_float((unsigned)w[i]);
+  out[blockIdx.x * blockDim.x + threadIdx.x] = s;
+  if (threadIdx.x == 0) cyc[blockIdx.x] = t1 - t0;
+}
+template <int MODE>  // 0: SS N=128, 1: TS N=128, 2: SS N=256, 3: SS N=64
+__global__ void __launch_bounds__(128, 1) mma_kernel(long long* out, int iters) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* sm = smem_raw + (base - raw);
+  __shared__ uint64_t bar;
+  __shared__ uint32_t tptr;
+  for (int i = threadIdx.x; i < 65536 / 4; i += blockDim.x) reinterpret_cast<uint32_t*>(sm)[i] = 0;  // A 16K | B 32K | pad
+  const uint32_t bar_a = smem_u32(&bar);
+  if (threadIdx.x == 0) { mbar_init(bar_a, 1); fence_barrier_init(); }
+  if (threadIdx.x < 32) tmem_alloc(smem_u32(&tptr), 512);
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  tc_fence_before(); __syncthreads(); tc_fence_after();
+  const uint32_t tmem = tptr;
+  if (threadIdx.x == 0) {
+    constexpr int N = MODE == 2 ? 256 : MODE == 3 ? 64 : 128;
+    const uint32_t idesc = idesc_bf16(128, N, 0, 0);
+    const uint32_t a = base, b = base + 16384;
+    // warm-up + timed
+    long long t0 = 0;
+    for (int rep = 0; rep < 2; ++rep) {
+      if (rep == 1) t0 = clock64();
+      for (int it = 0; it < iters; ++it) {
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t bd = sdesc_sw128(b + (kk % 4) * 32, 16, 1024);
+          if (MODE == 1) mma_ts(tmem, tmem + 256 + kk * 8, bd, idesc, 1);
+          else mma_ss(tmem, sdesc_sw128(a + (kk % 4) * 32, 16, 1024), bd, idesc, 1);
+        }
+      }
+      tc_commit(bar_a);
+      for (long long spin = 0; spin < (1LL << 26) && !mbar_try_wait(bar_a, rep & 1); ++spin) {}
+    }
+    long long t1 = clock64();
+    out[blockIdx.x] = t1 - t0;
+  }
+  tc_fence_before(); __syncthreads(); tc_fence_after();
+  if (threadIdx.x < 32) tmem_dealloc(tmem, 512);
+}
+// and concurrent tcgen05.ld/st traffic by 8 other warps.  Reports clocks per 128^3 GEMM.
+// smem: Q 2x32K at 0, ring 4x32K at 64K  (total 192K + 1K align)
+template <int MODE>  // bit0: bulk copies; bit1: tcgen05.ld/st traffic; bit2: busy ALU warps; bit3: commit per GEMM
+__global__ void __launch_bounds__(320, 1) mix_kernel(long long* out, const uint8_t* __restrict__ g, int iters) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  __shared__ uint64_t bars[4];
+  __shared__ uint32_t tptr;
+  __shared__ volatile int done;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) { for (int i = 0; i < 4; ++i) mbar_init(smem_u32(&bars[i]), 1); done = 0; fence_barrier_init(); }
+  {
+    uint32_t* w = reinterpret_cast<uint32_t*>(smem_raw + (base - raw));
+    for (int i = threadIdx.x; i < 6 * 32768 / 4; i += blockDim.x) {
+      uint32_t x = (MODE & 16) ? (uint32_t)i * 2654435761u + 12345u : 0u;
+      x ^= x >> 13; x *= 0x5bd1e995u; x ^= x >> 15;
+      // two bf16 values with exponent in [2^-2, 2^1] and random sign/mantissa
+      const uint32_t lo = (x & 0x807Fu) | 0x3E80u | ((x >> 7) & 0x0180u);
+      const uint32_t hi = ((x >> 16) & 0x807Fu) | 0x3E80u | ((x >> 23) & 0x0180u);
+      w[i] = (MODE & 16) ? (lo | (hi << 16)) : 0u;
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 9) tmem_alloc(smem_u32(&tptr), 512);
+  tc_fence_before(); __syncthreads(); tc_fence_after();
+  const uint32_t tmem = tptr;
+  if (warp == 9 && lane == 0) {
+    const uint32_t ids = idesc_bf16(128, 128, 0, 0), idpv = idesc_bf16(128, 128, 0, 1);
+    long long t0 = 0;
+    for (int rep = 0; rep < 2; ++rep) {
+      if (rep == 1) t0 = clock64();
+      if (MODE & 128) {
+        // lean issue: descriptors built once, then a 32-bit add per MMA on the address field
+        const uint64_t dq0 = sdesc_sw128(base, 16, 1024), dq1 = sdesc_sw128(base + 32768, 16, 1024);
+        const uint64_t dk = sdesc_sw128(base + 65536, 16, 1024), dv = sdesc_sw128(base + 65536, 16384, 1024);
+        for (int it = 0; it < iters; ++it) {
+          const uint32_t vs = ((2 * it + 1) % 4) * (32768 >> 4), ks = ((2 * it + 2) % 4) * (32768 >> 4);
+#pragma unroll
+          for (int t = 0; t < 2; ++t) {
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+              mma_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8, dv + vs + kk * (2048 >> 4), idpv, 1);
+            const uint64_t dq = t ? dq1 : dq0;
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+              mma_ss(tmem + t * 128, dq + ((kk / 4) * 16384 + (kk % 4) * 32) / 16,
+                     dk + ks + ((kk / 4) * 16384 + (kk % 4) * 32) / 16, ids, 1);
+          }
+        }
+      } else
+      for (int it = 0; it < iters; ++it) {
+        for (int t = 0; t < 2; ++t) {
+          const uint32_t va = base + 65536 + ((2 * it + 1) % 4) * 32768;
+          if (MODE & 32) tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+            mma_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8, sdesc_sw128(va + kk * 2048, 16384, 1024), idpv, 1);
+          if (MODE & 8) tc_commit(smem_u32(&bars[3]));
+          const uint32_t qa = base + t * 32768, ka = base + 65536 + ((2 * it + 2) % 4) * 32768;
+          if (MODE & 32) tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+            mma_ss(tmem + t * 128, sdesc_sw128(qa + (kk / 4) * 16384 + (kk % 4) * 32, 16, 1024),
+                   sdesc_sw128(ka + (kk / 4) * 16384 + (kk % 4) * 32, 16, 1024), ids, 1);
+          if (MODE & 8) { tc_commit(smem_u32(&bars[3])); tc_commit(smem_u32(&bars[3])); }
+        }
+      }
+      tc_commit(smem_u32(&bars[0]));
+      for (long long spin = 0; spin < (1LL << 26) && !mbar_try_wait(smem_u32(&bars[0]), rep & 1); ++spin) {}
+    }
+    out[blockIdx.x] = clock64() - t0;
+    done = 1;
+  } else if (warp == 8 && lane == 0 && (MODE & 1)) {
+    // bulk copies of 32 KB into the ring slots, back to back, until the MMA stream is done
+    int n = 0;
+    for (long long spin = 0; spin < (1LL << 22) && !done; ++spin) {
+      const uint32_t b = smem_u32(&bars[1 + (n & 1)]);
+      if (n >= 2) for (long long s2 = 0; s2 < (1LL << 24) && !mbar_try_wait(b, ((n >> 1) - 1) & 1); ++s2) {}
+      mbar_expect_tx(b, 32768);
+      bulk_g2s(base + 65536 + (n % 4) * 32768, g + (size_t)(n % 64) * 32768, 32768, b);
+      ++n;
+    }
+    for (int m = (n >= 2 ? n - 2 : 0); m < n; ++m)
+      for (long long s2 = 0; s2 < (1LL << 24) && !mbar_try_wait(smem_u32(&bars[1 + (m & 1)]), (m >> 1) & 1); ++s2) {}
+  } else if (warp < 8 && (MODE & 64)) {
+    // high-ILP issue pressure: 32 independent FMA chains per thread
+    float v[32];
+    for (int i = 0; i < 32; ++i) v[i] = 1e-3f * (lane + i);
+    for (long long spin = 0; spin < (1LL << 22) && !done; ++spin) {
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = fmaf(v[i], 0.999f, 1e-6f);
+    }
+    float acc = 0.f;
+    for (int i = 0; i < 32; ++i) acc += v[i];
+    if (acc == 12345.f) out[0] = 1;
+  } else if (warp < 8 && (MODE & 4)) {
+    // softmax-like issue pressure: FMA + MUFU work, no sleeping
+    float v[8];
+    for (int i = 0; i < 8; ++i) v[i] = -1e-3f * (lane + i);
+    for (long long spin = 0; spin < (1LL << 22) && !done; ++spin) {
+#pragma unroll
+      for (int u = 0; u < 16; ++u)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = ex2(fmaf(v[i], 0.5f, -0.75f)) - 1.5f;
+    }
+    if (v[0] == 12345.f) out[0] = 1;
+  } else if (warp < 8 && (MODE & 2)) {
+    // softmax-like TMEM traffic: read 128 columns of S, write 64 columns of P (other tile's columns)
+    const uint32_t lane_addr = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t s_tm = tmem + lane_addr + (warp >> 2) * 128;
+    for (long long spin = 0; spin < (1LL << 20) && !done; ++spin) {
+      uint32_t r[32];
+      float acc = 0.f;
+      for (int ch = 0; ch < 4; ++ch) { tmem_ld32(s_tm + ch * 32, r); tmem_wait_ld(); reg_fence32(r); acc += __uint_as_float(r[0]); }
+      for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(acc);
+      for (int ch = 0; ch < 2; ++ch) tmem_st32(s_tm + ch * 32, r);
+      tmem_wait_st();
+      __nanosleep(600);
+    }
+  }
+  __syncwarp();
+  tc_fence_before(); __syncthreads(); tc_fence_after();
+  if (warp == 9) tmem_dealloc(tmem, 512);
+}
+
+}  // namespace
+
+#define CHECK(x)                                                           \
+  do {                                                                     \
+    cudaError_t e_ = (x);                                                  \
+    if (e_ != cudaSuccess) {                                               \
+      printf("{\"error\": \"%s at line %d\"}\n", cudaGetErrorString(e_), __LINE__); \
+      return 1;                                                            \
+    }                                                                      \
+  } while (0)
+
+template <typename F>
+static double avg_cycles(F launch, long long* d, long long* h, int sms) {
+  launch();
+  if (cudaDeviceSynchronize() != cudaSuccess) return -1.0;
+  cudaMemcpy(h, d, sizeof(long long) * sms, cudaMemcpyDeviceToHost);
+  double avg = 0;
+  for (int i = 0; i < sms; ++i) avg += static_cast<double>(h[i]);
+  return avg / sms;
+}
+
+int main() {
+  int sms = 0;
+  CHECK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0));
+  long long* d = nullptr;
+  CHECK(cudaMalloc(&d, sizeof(long long) * sms));
+  float* out = nullptr;
+  CHECK(cudaMalloc(&out, sizeof(float) * sms * 1024));
+  uint8_t* g = nullptr;
+  CHECK(cudaMalloc(&g, 64 * 32768));
+  CHECK(cudaMemset(g, 0, 64 * 32768));
+  long long* h = new long long[sms];
+  printf("{\"sms\": %d", sms);
+
+  // pipes: 1024 threads x 4096 iterations x 8 ops per CTA
+  {
+    const double ops = 1024.0 * 4096 * 8;
+    const char* names[3] = {"ex2_per_clk_sm", "ffma_lanes_per_clk_sm", "ffma2_instr_lanes_per_clk_sm"};
+    for (int mode = 0; mode < 3; ++mode) {
+      auto launch = [&] {
+        for (int rep = 0; rep < 2; ++rep) {
+          if (mode == 0) pipe_kernel<0><<<sms, 1024>>>(out, d, 4096);
+          if (mode == 1) pipe_kernel<1><<<sms, 1024>>>(out, d, 4096);
+          if (mode == 2) pipe_kernel<2><<<sms, 1024>>>(out, d, 4096);
+        }
+      };
+      const double cyc = avg_cycles(launch, d, h, sms);
+      if (cyc <= 0) { printf(", \"error\": \"pipe probe failed\"}\n"); return 1; }
+      printf(", \"%s\": %.2f", names[mode], ops / cyc);
+    }
+  }
+  // single-MMA rates
+  {
+    const int smem = 65536 + 2048, iters = 2000;
+    CHECK(cudaFuncSetAttribute(mma_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    CHECK(cudaFuncSetAttribute(mma_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    CHECK(cudaFuncSetAttribute(mma_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    CHECK(cudaFuncSetAttribute(mma_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    const char* names[4] = {"mma_ss_128x128x16_clk", "mma_ts_128x128x16_clk", "mma_ss_128x256x16_clk",
+                            "mma_ss_128x64x16_clk"};
+    for (int mode = 0; mode < 4; ++mode) {
+      auto launch = [&] {
+        if (mode == 0) mma_kernel<0><<<sms, 128, smem>>>(d, iters);
+        if (mode == 1) mma_kernel<1><<<sms, 128, smem>>>(d, iters);
+        if (mode == 2) mma_kernel<2><<<sms, 128, smem>>>(d, iters);
+        if (mode == 3) mma_kernel<3><<<sms, 128, smem>>>(d, iters);
+      };
+      const double cyc = avg_cycles(launch, d, h, sms);
+      if (cyc <= 0) { printf(", \"error\": \"mma probe failed\"}\n"); return 1; }
+      printf(", \"%s\": %.1f", names[mode], cyc / (iters * 8.0));
+    }
+  }
+  // prefill-like MMA stream under load
+  {
+    const int iters = 500, smem = 6 * 32768 + 1024;
+    const int modes[11] = {0, 1, 2, 3, 4, 8, 16, 26, 32, 64, 192};
+    const char* names[11] = {"alone", "bulk_copies", "tmem_ld_st", "copies_and_tmem", "mufu_warps",
+                             "commit_per_gemm", "random_operands", "random_commits_tmem",
+                             "fence_per_gemm", "ilp_fma_warps", "ilp_fma_warps_lean_issue"};
+    printf(", \"mix_clk_per_gemm\": {");
+    for (int i = 0; i < 11; ++i) {
+      auto launch = [&] {
+#define LOOM_MIX(M)                                                                        \
+  if (modes[i] == M) {                                                                     \
+    cudaFuncSetAttribute(mix_kernel<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem); \
+    mix_kernel<M><<<sms, 320, smem>>>(d, g, iters);                                        \
+  }
+        LOOM_MIX(0) LOOM_MIX(1) LOOM_MIX(2) LOOM_MIX(3) LOOM_MIX(4) LOOM_MIX(8) LOOM_MIX(16)
+        LOOM_MIX(26) LOOM_MIX(32) LOOM_MIX(64) LOOM_MIX(192)
+#undef LOOM_MIX
+      };
+      const double cyc = avg_cycles(launch, d, h, sms);
+      if (cyc <= 0) { printf("}, \"error\": \"mix probe failed\"}\n"); return 1; }
+      printf("%s\"%s\": %.1f", i ? ", " : "", names[i], cyc / (iters * 4.0));
+    }
+    printf("}");
+  }
+  printf("}\n");
+  return 0;
+}

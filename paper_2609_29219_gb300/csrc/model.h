@@ -36,11 +36,13 @@ struct ArchDesc {
   double launch_ns;         // fixed cost of one dependent kernel launch (assumed)
   double decode_cta_gbs;    // KV stream rate of a lone decode split CTA on an SM (measured)
   double cta_start_ns;      // start-up of a decode split CTA: launch, first copies (measured)
+  double mma_clk_per_n;     // clocks of one 128xNx16 bf16 MMA per unit of N (measured: 0.5)
+  double mma_min_clk;       // floor on one MMA's clocks (measured: 48 at N = 64)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
-    1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0,
+    1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -84,10 +86,11 @@ constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int bn, int slots, int b_lm
   // load stage: K_j and V_j tiles, mostly L2 hits (the CTAs of a head share them)
   const double kv_bytes = 2.0 * bn * D * 2;
   p.t_load_ns = kv_bytes / a.l2_smem_gbs_sm;  // GB/s == bytes/ns
-  // compute leaf: 2 GEMMs (S = Q K^T, O += P V) per query tile on the tensor pipe
-  const double flops = 2.0 * p.q_tiles * (2.0 * p.bm * bn * D);
-  const double f_sm = a.mma_tflops * 1e3 / a.num_sms;  // FLOP/ns per SM
-  p.t_mma_ns = flops / f_sm;
+  // compute leaf: 2 GEMMs (S = Q K^T with N = BN, O += P V with N = D) per query tile,
+  // K/16 tcgen05 MMAs each, at the measured clocks per 128xNx16 MMA
+  auto mma_clk = [&](int n) { return dmax(a.mma_clk_per_n * n, a.mma_min_clk); };
+  const double clk_s = (D / 16.0) * mma_clk(bn), clk_pv = (bn / 16.0) * mma_clk(D);
+  p.t_mma_ns = p.q_tiles * (clk_s + clk_pv) / clk;
   // softmax leaf: one ex2 per score on MUFU; ~5 FMA-pipe ops per score (scale/subtract,
   // max, add, half a pack, mask/compare amortised) -- two tiles share the SM
   const double scores = 1.0 * p.q_tiles * p.bm * bn;
