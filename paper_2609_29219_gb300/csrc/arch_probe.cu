@@ -168,6 +168,12 @@ __global__ void __launch_bounds__(320, 1) mix_kernel(long long* out, const uint8
     }
     for (int m = (n >= 2 ? n - 2 : 0); m < n; ++m)
       for (long long s2 = 0; s2 < (1LL << 24) && !mbar_try_wait(smem_u32(&bars[1 + (m & 1)]), (m >> 1) & 1); ++s2) {}
+  } else if (warp < 8 && (MODE & 256)) {
+    // neighbours polling an mbarrier phase that never completes, the way waiting
+    // softmax warps do (all lanes in try_wait, warp-wide vote)
+    const uint32_t never = smem_u32(&bars[3]);
+    for (long long spin = 0; spin < (1LL << 24) && !done; ++spin)
+      if (__all_sync(0xffffffffu, mbar_try_wait(never, 0))) break;
   } else if (warp < 8 && (MODE & 64)) {
     // high-ILP issue pressure: 32 independent FMA chains per thread
     float v[32];
@@ -286,12 +292,13 @@ int main() {
   // prefill-like MMA stream under load
   {
     const int iters = 500, smem = 6 * 32768 + 1024;
-    const int modes[11] = {0, 1, 2, 3, 4, 8, 16, 26, 32, 64, 192};
-    const char* names[11] = {"alone", "bulk_copies", "tmem_ld_st", "copies_and_tmem", "mufu_warps",
+    const int modes[12] = {0, 1, 2, 3, 4, 8, 16, 26, 32, 64, 192, 256};
+    const char* names[12] = {"alone", "bulk_copies", "tmem_ld_st", "copies_and_tmem", "mufu_warps",
                              "commit_per_gemm", "random_operands", "random_commits_tmem",
-                             "fence_per_gemm", "ilp_fma_warps", "ilp_fma_warps_lean_issue"};
+                             "fence_per_gemm", "ilp_fma_warps", "ilp_fma_warps_lean_issue",
+                             "polling_warps"};
     printf(", \"mix_clk_per_gemm\": {");
-    for (int i = 0; i < 11; ++i) {
+    for (int i = 0; i < 12; ++i) {
       auto launch = [&] {
 #define LOOM_MIX(M)                                                                        \
   if (modes[i] == M) {                                                                     \
@@ -299,7 +306,7 @@ int main() {
     mix_kernel<M><<<sms, 320, smem>>>(d, g, iters);                                        \
   }
         LOOM_MIX(0) LOOM_MIX(1) LOOM_MIX(2) LOOM_MIX(3) LOOM_MIX(4) LOOM_MIX(8) LOOM_MIX(16)
-        LOOM_MIX(26) LOOM_MIX(32) LOOM_MIX(64) LOOM_MIX(192)
+        LOOM_MIX(26) LOOM_MIX(32) LOOM_MIX(64) LOOM_MIX(192) LOOM_MIX(256)
 #undef LOOM_MIX
       };
       const double cyc = avg_cycles(launch, d, h, sms);

@@ -1,0 +1,92 @@
+"""Failure detection without a GPU fault.
+
+Every mbarrier wait in the kernels is bounded by %globaltimer.  The host-side test hook
+loom_debug_inject makes a kernel's loader skip one copy, so that the waits on it run out;
+the kernel then unwinds (drains the copies it issued, waits for its issued MMAs, frees
+TMEM) and sets the device error word.  These tests check that loom_attn_check_error
+reports LOOM_ERR_TIMEOUT and that the context stays usable: the very next normal call
+matches the oracle and reports no error.
+"""
+import pytest
+
+import oracle
+import synth
+from tests.gpu_util import assert_parity, o_to_f64, to_dev
+
+pytestmark = pytest.mark.gpu
+
+TIMEOUT_NS = 50_000_000  # 50 ms per wait while the hook is on
+
+
+@pytest.fixture(scope="module")
+def loom():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2609_29219_gb300 as m
+    yield m
+    m.loom_debug_inject(0)
+    m.loom_debug_set_timeout_ns(0)
+
+
+def _expect_timeout(loom, call):
+    loom.loom_attn_check_error()  # nothing pending
+    loom.loom_debug_set_timeout_ns(TIMEOUT_NS)
+    try:
+        call()
+        with pytest.raises(loom.LoomError) as e:
+            loom.loom_attn_check_error()
+        assert e.value.status == 6, e.value
+    finally:
+        loom.loom_debug_inject(0)
+        loom.loom_debug_set_timeout_ns(0)
+    loom.loom_attn_check_error()  # the word was cleared
+
+
+def test_decode_skipped_stage_times_out_and_context_survives(loom):
+    B, Hq, Hkv, Skv, D = 1, 4, 1, 2048, 128  # one split of 32 stages, one CTA
+    q = synth.bf16_normal(31, synth.STREAM_Q, (B, Hq, 1, D))
+    k = synth.bf16_normal(31, synth.STREAM_K, (B, Hkv, Skv, D))
+    v = synth.bf16_normal(31, synth.STREAM_V, (B, Hkv, Skv, D))
+    qd, kd, vd = to_dev(q), to_dev(k), to_dev(v)
+
+    def bad():
+        loom.loom_debug_inject(1)
+        loom.loom_attn_decode(qd, kd, vd, None, num_splits=1)
+
+    _expect_timeout(loom, bad)
+    o, lse = loom.loom_attn_decode(qd, kd, vd, None, num_splits=1, return_lse=True)
+    loom.loom_attn_check_error()
+    o_ref, lse_ref = oracle.attention(q, k, v)
+    assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "decode after timeout")
+
+
+def test_prefill_skipped_tile_times_out_and_context_survives(loom):
+    B, H, S, D = 1, 2, 512, 128  # 4 work items, each with 4 KV tiles
+    q = synth.bf16_normal(32, synth.STREAM_Q, (B, H, S, D))
+    k = synth.bf16_normal(32, synth.STREAM_K, (B, H, S, D))
+    v = synth.bf16_normal(32, synth.STREAM_V, (B, H, S, D))
+    qd, kd, vd = to_dev(q), to_dev(k), to_dev(v)
+
+    def bad():
+        loom.loom_debug_inject(2)
+        loom.loom_attn_fwd(qd, kd, vd)
+
+    _expect_timeout(loom, bad)
+    for causal in (False, True):
+        o, lse = loom.loom_attn_fwd(qd, kd, vd, causal=causal, return_lse=True)
+        loom.loom_attn_check_error()
+        o_ref, lse_ref = oracle.attention(q, k, v, causal=causal)
+        assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"prefill after timeout causal={causal}")
+
+
+def test_no_false_timeouts_under_default_limit(loom):
+    # a full-size call with the default 2 s limit never trips the error word
+    B, H, S, D = 4, 32, 2048, 128
+    import torch
+    q = torch.randn(B, H, S, D, device="cuda").to(torch.bfloat16)
+    for causal in (False, True):
+        loom.loom_attn_fwd(q, q, q, causal=causal)
+    loom.loom_attn_check_error()
