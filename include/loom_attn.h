@@ -166,6 +166,14 @@ const char* loom_status_string(loom_status status);
 void loom_debug_set_timeout_ns(uint64_t ns);
 void loom_debug_inject(int mode);
 
+/*
+ * Test hook: force the prefill design instead of the analytic model's choice (used to
+ * measure the alternatives the model ranks).  q_tiles = 2: two query tiles per CTA that
+ * alternate on the tensor pipe; q_tiles = 1: one query tile with S double-buffered in
+ * TMEM; anything else: the model's choice (default).
+ */
+void loom_debug_prefill_design(int q_tiles);
+
 #ifdef __cplusplus
 }
 #endif

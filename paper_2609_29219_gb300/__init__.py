@@ -24,7 +24,7 @@ __all__ = [
     "loom_attn_fwd", "loom_attn_decode", "loom_attn_decode_workspace_bytes",
     "loom_attn_decode_num_splits", "loom_attn_check_error", "loom_status_string",
     "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
-    "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan",
+    "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -86,6 +86,8 @@ def capi() -> ctypes.CDLL:
             lib.loom_debug_set_timeout_ns.restype = None
             lib.loom_debug_inject.argtypes = [i32]
             lib.loom_debug_inject.restype = None
+            lib.loom_debug_prefill_design.argtypes = [i32]
+            lib.loom_debug_prefill_design.restype = None
             lib.loom_model_fwd_plan.argtypes = [i32, ctypes.POINTER(FwdPlan)]
             lib.loom_model_fwd_plan.restype = i32
             lib.loom_model_fwd_time_us.argtypes = [i32, i32, i32, i32, i32, i32]
@@ -234,6 +236,10 @@ def loom_debug_set_timeout_ns(ns: int):
 
 def loom_debug_inject(mode: int):
     capi().loom_debug_inject(int(mode))
+
+
+def loom_debug_prefill_design(q_tiles: int):
+    capi().loom_debug_prefill_design(int(q_tiles))
 
 
 def loom_model_fwd_plan(D: int) -> dict:

@@ -14,6 +14,7 @@
 // buffers allocated below, and bounds every wait.
 #include <cstdint>
 #include <cstdio>
+#include <initializer_list>
 
 #include "ptx.cuh"
 
@@ -217,6 +218,72 @@ __global__ void __launch_bounds__(320, 1) mix_kernel(long long* out, const uint8
   if (warp == 9) tmem_dealloc(tmem, 512);
 }
 
+// The prefill softmax step on register data: per 128-key row, a 3-input max tree, then
+// p = 2^(s*c - m) with a bf16x2 pack and the row sum.  Each iteration perturbs the row
+// so nothing is hoisted.  Reports clocks per row per warp.  Variants of the per-pair work:
+//   0: packed FMA (f32x2), two ex2, packed add into 4 accumulators, pack
+//   1: scalar FMA, two ex2, scalar adds into 4 accumulators, pack
+//   2: like 1 without the row sum (sum delegated elsewhere)
+//   3: scalar FMA and ex2 only (no pack, no sum): MUFU-bound reference
+//   4: variant 0 with every other pair's exponentials on the FMA pipe (exp2_poly)
+//   5: variant 0 with one pair in four on the FMA pipe
+template <int V, int CAP_THREADS = 256>
+__global__ void __launch_bounds__(CAP_THREADS, 1) softmax_row_kernel(long long* cyc, float* sink, int iters) {
+  if (threadIdx.x >= 256) return;  // extra threads only lower the register cap
+  float s[128];
+  for (int i = 0; i < 128; ++i) s[i] = 0.01f * ((threadIdx.x * 7 + i * 13) % 97) - 0.5f;
+  const float c = 0.18f;
+  const uint64_t c2 = f2(c, c);
+  uint32_t keep = 0;
+  float lsum = 0.f;
+  __syncthreads();
+  const long long t0 = clock64();
+  for (int it = 0; it < iters; ++it) {
+    float mm[8];
+#pragma unroll
+    for (int g = 0; g < 8; ++g) mm[g] = s[g];
+#pragma unroll
+    for (int i = 8; i + 16 <= 128; i += 16)
+#pragma unroll
+      for (int g = 0; g < 8; ++g) mm[g] = max3(mm[g], s[i + g], s[i + 8 + g]);
+#pragma unroll
+    for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], s[120 + g]);
+    const float mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
+    const float nm = -mx * c;
+    if constexpr (V == 0 || V == 4 || V == 5) {
+      const uint64_t nms2 = f2(nm, nm);
+      uint64_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+      for (int i = 0; i < 64; ++i) {
+        const uint64_t x = fma2(f2(s[2 * i], s[2 * i + 1]), c2, nms2);
+        const bool poly = (V == 4 && (i & 1)) || (V == 5 && (i & 3) == 3);
+        const float p0 = poly ? exp2_poly(f2lo(x)) : ex2(f2lo(x));
+        const float p1 = poly ? exp2_poly(f2hi(x)) : ex2(f2hi(x));
+        acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
+        keep ^= pack_bf16x2(p0, p1);
+      }
+      const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+      lsum += f2lo(a01) + f2hi(a01);
+    } else {
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int i = 0; i < 64; ++i) {
+        const float p0 = ex2(fmaf(s[2 * i], c, nm)), p1 = ex2(fmaf(s[2 * i + 1], c, nm));
+        if constexpr (V == 1) {
+          acc[i & 3] += p0;
+          acc[(i + 2) & 3] += p1;
+        }
+        if constexpr (V != 3) keep ^= pack_bf16x2(p0, p1);
+        else keep ^= __float_as_uint(p0) ^ __float_as_uint(p1);
+      }
+      lsum += (acc[0] + acc[1]) + (acc[2] + acc[3]);
+    }
+    s[0] += 1e-3f * static_cast<float>(it & 1);  // perturb (static index: stays in registers)
+  }
+  const long long t1 = clock64();
+  if (threadIdx.x == 0) cyc[blockIdx.x] = t1 - t0;
+  sink[blockIdx.x * blockDim.x + threadIdx.x] = lsum + __uint_as_float(keep & 0x3f800000u);
+}
 }  // namespace
 
 #define CHECK(x)                                                           \
@@ -266,6 +333,36 @@ int main() {
       const double cyc = avg_cycles(launch, d, h, sms);
       if (cyc <= 0) { printf(", \"error\": \"pipe probe failed\"}\n"); return 1; }
       printf(", \"%s\": %.2f", names[mode], ops / cyc);
+    }
+  }
+  // softmax row step variants: 4 warps (one per SM sub-partition) and 8 warps (two each)
+  {
+    const int iters = 2000;
+    for (int v = 0; v < 6; ++v)
+      for (int warps : {4, 8}) {
+        auto launch = [&] {
+          if (v == 0) softmax_row_kernel<0><<<sms, warps * 32>>>(d, out, iters);
+          if (v == 1) softmax_row_kernel<1><<<sms, warps * 32>>>(d, out, iters);
+          if (v == 2) softmax_row_kernel<2><<<sms, warps * 32>>>(d, out, iters);
+          if (v == 3) softmax_row_kernel<3><<<sms, warps * 32>>>(d, out, iters);
+          if (v == 4) softmax_row_kernel<4><<<sms, warps * 32>>>(d, out, iters);
+          if (v == 5) softmax_row_kernel<5><<<sms, warps * 32>>>(d, out, iters);
+        };
+        const double cyc = avg_cycles(launch, d, h, sms);
+        if (cyc <= 0) { printf(", \"error\": \"softmax probe failed\"}\n"); return 1; }
+        printf(", \"softmax_row128_v%d_clk_%dwarps\": %.1f", v, warps, cyc / iters);
+      }
+  }
+  // variant 0 compiled under the prefill kernel's register cap (10 warps -> 168 registers)
+  {
+    const int iters = 2000;
+    for (int warps : {4, 8}) {
+      auto launch = [&] { softmax_row_kernel<0, 320><<<sms, 320>>>(d, out, iters); };
+      (void)warps;
+      const double cyc = avg_cycles(launch, d, h, sms);
+      if (cyc <= 0) { printf(", \"error\": \"softmax probe failed\"}\n"); return 1; }
+      printf(", \"softmax_row128_v0_clk_8warps_168regs\": %.1f", cyc / iters);
+      break;
     }
   }
   // single-MMA rates

@@ -43,8 +43,8 @@ constexpr float kRescaleThreshold = 8.0f;  // base-2 units; P <= 2^8 between res
 // Tile and stage constants: the analytic model's argmin for this head dimension.
 template <int D>
 struct FwdCfg {
-  static constexpr model::FwdPlan kPlan = model::fwd_plan(D);
-  static_assert(kPlan.feasible, "no feasible prefill schedule");
+  static constexpr model::FwdPlan kPlan = model::fwd_plan_variant(D, 2);
+  static_assert(kPlan.feasible, "no feasible two-tile prefill schedule");
   static constexpr int BM = kPlan.bm;         // rows per query tile (= TMEM lanes)
   static constexpr int NQT = kPlan.q_tiles;   // query tiles per CTA
   static constexpr int BN = kPlan.bn;         // keys per KV tile
@@ -128,6 +128,139 @@ __device__ __forceinline__ Item make_item(const FwdParams& p, int idx) {
   it.n_tiles0 = (n_kv0 + C::BN - 1) / C::BN;
   it.n_tiles = (n_kv1 + C::BN - 1) / C::BN;
   return it;
+}
+
+// One online-softmax step of one query row (this thread's TMEM lane) over a BN-key
+// tile of S in TMEM at s_tm: wait for S, mask keys >= limit, move the running max
+// lazily, write P = 2^(S*c - m) as bf16 over the first half of the S columns in two
+// halves (arriving on bar_p and bar_p + 8 after each, so that P.V can start on the first
+// half), rescale O at o_tm when the max moved (after waiting for the previous P.V on
+// bar_o with parity par_o), and accumulate the row sum.  Returns false if a wait gave up.
+template <int D, int BN>
+__device__ __forceinline__ bool softmax_step(uint32_t s_tm, uint32_t o_tm, uint32_t bar_s,
+                                             uint32_t par_s, uint32_t bar_p, uint32_t bar_o,
+                                             uint32_t par_o, bool first, int kbase, int limit,
+                                             float c, uint64_t c2, float& m_run, float& l_run,
+                                             const KernelCtl& ctl, const Abort& ab) {
+  if (!mbar_wait_warp(bar_s, par_s, ctl, ab)) return false;
+  tc_fence_after();
+  uint32_t s[BN];
+#pragma unroll
+  for (int ch = 0; ch < BN / 32; ++ch) tmem_ld32(s_tm + ch * 32, s + ch * 32);
+  tmem_wait_ld();
+#pragma unroll
+  for (int ch = 0; ch < BN / 32; ++ch) reg_fence32(s + ch * 32);
+  if (kbase + BN > limit) {
+#pragma unroll
+    for (int i = 0; i < BN; ++i)
+      if (kbase + i >= limit) s[i] = __float_as_uint(-INFINITY);
+  }
+  // row max: 8 independent chains of 3-input max, then a small tree
+  float mx;
+  {
+    float mm[8];
+#pragma unroll
+    for (int g = 0; g < 8; ++g) mm[g] = __uint_as_float(s[g]);
+#pragma unroll
+    for (int i = 8; i + 16 <= BN; i += 16)
+#pragma unroll
+      for (int g = 0; g < 8; ++g)
+        mm[g] = max3(mm[g], __uint_as_float(s[i + g]), __uint_as_float(s[i + 8 + g]));
+    if constexpr ((BN - 8) % 16 != 0) {
+#pragma unroll
+      for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], __uint_as_float(s[BN - 8 + g]));
+    }
+    mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
+  }
+  const float m_new = fmaxf(m_run, mx * c);
+  const bool need = m_new > m_run + kRescaleThreshold;
+  const float alpha = need ? ex2(m_run - m_new) : 1.f;
+  if (need) m_run = m_new;
+  const float ms = (m_run == -INFINITY) ? 0.f : m_run;
+  const uint64_t nms2 = f2(-ms, -ms);
+  // p = 2^(s*c - m): packed FMA, one MUFU ex2 per score, 4 packed partial sums
+  uint64_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+  for (int half = 0; half < 2; ++half) {
+    uint32_t pk[BN / 4];
+#pragma unroll
+    for (int i = 0; i < BN / 4; ++i) {
+      const int e = half * (BN / 2) + 2 * i;
+      const uint64_t x = fma2(f2(__uint_as_float(s[e]), __uint_as_float(s[e + 1])), c2, nms2);
+      const float p0 = ex2(f2lo(x));
+      const float p1 = ex2(f2hi(x));
+      acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
+      pk[i] = pack_bf16x2(p0, p1);
+    }
+#pragma unroll
+    for (int ch = 0; ch < BN / 128; ++ch) tmem_st32(s_tm + half * (BN / 4) + ch * 32, pk + ch * 32);
+    tmem_wait_st();
+    // O must hold the previous P.V before it is rescaled, and be rescaled before this
+    // tile's P.V starts (the first-half arrive below).
+    if (half == 0 && !first && __any_sync(0xffffffffu, need)) {
+      if (!mbar_wait_warp(bar_o, par_o, ctl, ab)) return false;
+      tc_fence_after();
+      const uint64_t a2 = f2(alpha, alpha);
+#pragma unroll 1
+      for (int ch = 0; ch < D / 32; ++ch) {
+        uint32_t rr[32];
+        tmem_ld32(o_tm + ch * 32, rr);
+        tmem_wait_ld();
+        reg_fence32(rr);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const uint64_t x = mul2(f2(__uint_as_float(rr[2 * i]), __uint_as_float(rr[2 * i + 1])), a2);
+          rr[2 * i] = __float_as_uint(f2lo(x));
+          rr[2 * i + 1] = __float_as_uint(f2hi(x));
+        }
+        tmem_st32(o_tm + ch * 32, rr);
+      }
+      tmem_wait_st();
+    }
+    tc_fence_before();
+    mbar_arrive(bar_p + 8 * half);
+  }
+  const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+  l_run = l_run * alpha + (f2lo(a01) + f2hi(a01));
+  return true;
+}
+
+// Epilogue of one query row: wait for the last P.V (bar_o, par_o), read O from TMEM,
+// write O / l as bf16 and the log-sum-exp, then hand the O columns back (bar_oe).
+template <int D>
+__device__ __forceinline__ bool softmax_epilogue(uint32_t o_tm, uint32_t bar_o, uint32_t par_o,
+                                                 uint32_t bar_oe, float m_run, float l_run,
+                                                 int row, int q_z, const FwdParams& p,
+                                                 const Abort& ab) {
+  if (!mbar_wait_warp(bar_o, par_o, p.ctl, ab)) return false;
+  tc_fence_after();
+  const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
+  const bool store = row < p.Sq;
+  __nv_bfloat16* orow = p.o + (static_cast<size_t>(q_z) * p.Sq + (store ? row : 0)) * D;
+  const uint64_t il2 = f2(inv_l, inv_l);
+#pragma unroll 1
+  for (int ch = 0; ch < D / 32; ++ch) {
+    uint32_t rr[32];
+    tmem_ld32(o_tm + ch * 32, rr);
+    tmem_wait_ld();
+    reg_fence32(rr);
+    uint32_t w[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const uint64_t x = mul2(f2(__uint_as_float(rr[2 * i]), __uint_as_float(rr[2 * i + 1])), il2);
+      w[i] = pack_bf16x2(f2lo(x), f2hi(x));
+    }
+    if (store) {
+      uint4* dst = reinterpret_cast<uint4*>(orow + ch * 32);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) dst[i] = make_uint4(w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+    }
+  }
+  tc_fence_before();
+  mbar_arrive(bar_oe);
+  if (store && p.lse)
+    p.lse[static_cast<size_t>(q_z) * p.Sq + row] = l_run > 0.f ? (m_run + log2f(l_run)) * kLn2 : -INFINITY;
+  return true;
 }
 
 template <int D>
@@ -332,125 +465,15 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
       const int limit = p.causal ? min(p.Skv, row + off + 1) : p.Skv;  // keys [0, limit) visible
       const int my_tiles = t == 0 ? it.n_tiles0 : it.n_tiles;
       float m_run = -INFINITY, l_run = 0.f;
-      for (int j = 0; j < my_tiles; ++j) {
-        if (!(ok = mbar_wait_warp(my_bar_s, (cnt + j) & 1, p.ctl, ab))) break;
-        tc_fence_after();
-        uint32_t s[C::BN];
-#pragma unroll
-        for (int ch = 0; ch < C::BN / 32; ++ch) tmem_ld32(s_tm + ch * 32, s + ch * 32);
-        tmem_wait_ld();
-#pragma unroll
-        for (int ch = 0; ch < C::BN / 32; ++ch) reg_fence32(s + ch * 32);
-        const int kbase = j * C::BN;
-        if (kbase + C::BN > limit) {
-#pragma unroll
-          for (int i = 0; i < C::BN; ++i)
-            if (kbase + i >= limit) s[i] = __float_as_uint(-INFINITY);
-        }
-        // row max: 8 independent chains of 3-input max, then a small tree
-        float mx;
-        {
-          float mm[8];
-#pragma unroll
-          for (int g = 0; g < 8; ++g) mm[g] = __uint_as_float(s[g]);
-#pragma unroll
-          for (int i = 8; i + 16 <= C::BN; i += 16)
-#pragma unroll
-            for (int g = 0; g < 8; ++g)
-              mm[g] = max3(mm[g], __uint_as_float(s[i + g]), __uint_as_float(s[i + 8 + g]));
-          if constexpr ((C::BN - 8) % 16 != 0) {
-#pragma unroll
-            for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], __uint_as_float(s[C::BN - 8 + g]));
-          }
-          mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
-        }
-        const float m_new = fmaxf(m_run, mx * c);
-        const bool need = m_new > m_run + kRescaleThreshold;
-        const float alpha = need ? ex2(m_run - m_new) : 1.f;
-        if (need) m_run = m_new;
-        const float ms = (m_run == -INFINITY) ? 0.f : m_run;
-        const uint64_t nms2 = f2(-ms, -ms);
-        // p = 2^(s*c - m): packed FMA, one MUFU ex2 per score, 4 packed partial sums.
-        // P goes out in two halves so that P[:, :BN/2] V can run while the second half
-        // of the exponentials is computed.
-        uint64_t acc[4] = {0, 0, 0, 0};
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          uint32_t pk[C::BN / 4];
-#pragma unroll
-          for (int i = 0; i < C::BN / 4; ++i) {
-            const int e = half * (C::BN / 2) + 2 * i;
-            const uint64_t x = fma2(f2(__uint_as_float(s[e]), __uint_as_float(s[e + 1])), c2, nms2);
-            const float p0 = ex2(f2lo(x));
-            const float p1 = ex2(f2hi(x));
-            acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
-            pk[i] = pack_bf16x2(p0, p1);
-          }
-#pragma unroll
-          for (int ch = 0; ch < C::BN / 128; ++ch)
-            tmem_st32(s_tm + half * (C::BN / 4) + ch * 32, pk + ch * 32);
-          tmem_wait_st();
-          // O_t must hold P_{j-1} V_{j-1} before it is rescaled, and be rescaled before
-          // P_j V_j starts (the first-half arrive below).
-          if (half == 0 && j > 0 && __any_sync(0xffffffffu, need)) {
-            if (!(ok = mbar_wait_warp(my_bar_o, (cnt + j - 1) & 1, p.ctl, ab))) break;
-            tc_fence_after();
-            const uint64_t a2 = f2(alpha, alpha);
-#pragma unroll 1
-            for (int ch = 0; ch < D / 32; ++ch) {
-              uint32_t rr[32];
-              tmem_ld32(o_tm + ch * 32, rr);
-              tmem_wait_ld();
-              reg_fence32(rr);
-#pragma unroll
-              for (int i = 0; i < 16; ++i) {
-                const uint64_t x = mul2(f2(__uint_as_float(rr[2 * i]), __uint_as_float(rr[2 * i + 1])), a2);
-                rr[2 * i] = __float_as_uint(f2lo(x));
-                rr[2 * i + 1] = __float_as_uint(f2hi(x));
-              }
-              tmem_st32(o_tm + ch * 32, rr);
-            }
-            tmem_wait_st();
-          }
-          tc_fence_before();
-          mbar_arrive(my_bar_p + 8 * half);
-        }
-        if (!ok) break;
-        const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
-        l_run = l_run * alpha + (f2lo(a01) + f2hi(a01));
-      }
+      for (int j = 0; ok && j < my_tiles; ++j)
+        ok = softmax_step<D, C::BN>(s_tm, o_tm, my_bar_s, (cnt + j) & 1, my_bar_p, my_bar_o,
+                                    (cnt + j - 1) & 1, j == 0, j * C::BN, limit, c, c2, m_run,
+                                    l_run, p.ctl, ab);
       if (!ok) break;
-
       // epilogue: O / l -> bf16 rows, LSE; then hand O_t back to the MMA warp
-      if (!(ok = mbar_wait_warp(my_bar_o, (cnt + my_tiles - 1) & 1, p.ctl, ab))) break;
-      tc_fence_after();
-      const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
-      const bool store = row < p.Sq;
-      __nv_bfloat16* orow = p.o + (static_cast<size_t>(it.q_z) * p.Sq + (store ? row : 0)) * D;
-      const uint64_t il2 = f2(inv_l, inv_l);
-#pragma unroll 1
-      for (int ch = 0; ch < D / 32; ++ch) {
-        uint32_t rr[32];
-        tmem_ld32(o_tm + ch * 32, rr);
-        tmem_wait_ld();
-        reg_fence32(rr);
-        uint32_t w[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const uint64_t x = mul2(f2(__uint_as_float(rr[2 * i]), __uint_as_float(rr[2 * i + 1])), il2);
-          w[i] = pack_bf16x2(f2lo(x), f2hi(x));
-        }
-        if (store) {
-          uint4* dst = reinterpret_cast<uint4*>(orow + ch * 32);
-#pragma unroll
-          for (int i = 0; i < 4; ++i) dst[i] = make_uint4(w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
-        }
-      }
-      tc_fence_before();
-      mbar_arrive(my_bar_oe);
-      if (store && p.lse)
-        p.lse[static_cast<size_t>(it.q_z) * p.Sq + row] =
-            l_run > 0.f ? (m_run + log2f(l_run)) * kLn2 : -INFINITY;
+      if (!(ok = softmax_epilogue<D>(o_tm, my_bar_o, (cnt + my_tiles - 1) & 1, my_bar_oe, m_run,
+                                     l_run, row, it.q_z, p, ab)))
+        break;
       cnt += my_tiles;
     }
   }
@@ -459,6 +482,274 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
   tc_fence_before();
   __syncthreads();
   if (warp == 9) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------- single-tile variant
+// One 128-row query tile per CTA with S double-buffered in TMEM: while the softmax
+// warpgroup works on S_j in buffer j % 2, the tensor pipe computes S_{j+1} in the other
+// buffer and P_{j-1} V_{j-1}.  In the paper's terms this opens the boundary between the
+// S MMA (load stage of the softmax) and the softmax body of Eq. 6, paid for with a
+// second S buffer of TMEM (the capacity constraint of Eq. 8).
+//
+//   warps 0-3 softmax (thread = query row = TMEM lane), warp 4 loader, warp 5 MMA
+//   TMEM: [0, BN) S/P buffer 0 | [BN, 2BN) S/P buffer 1 | [2BN, 2BN + D) O
+//   ring order per item: K_0, K_1, V_0, K_2, V_1, ..., K_{n-1}, V_{n-2}, V_{n-1}
+template <int D>
+struct Fwd1Cfg {
+  static constexpr model::FwdPlan kPlan = model::fwd_plan_variant(D, 1);
+  static_assert(kPlan.feasible, "no feasible single-tile prefill schedule");
+  static constexpr int BM = 128;
+  static constexpr int BN = kPlan.bn;
+  static constexpr int NSLOT = kPlan.kv_slots;
+  static_assert(kPlan.q_tiles == 1 && kPlan.s_buffers == 2, "single-tile variant");
+  static_assert(BN == 128, "softmax holds one S row of 128 fp32 in registers");
+  static constexpr int THREADS = 192;
+  static constexpr int BOX_COLS = 64;
+  static constexpr int NBOX = D / BOX_COLS;
+  static constexpr uint32_t Q_BOX_BYTES = BM * 128;
+  static constexpr uint32_t Q_TILE_BYTES = NBOX * Q_BOX_BYTES;
+  static constexpr uint32_t KV_BOX_BYTES = BN * 128;
+  static constexpr uint32_t SLOT_BYTES = NBOX * KV_BOX_BYTES;
+  static constexpr uint32_t Q_OFF = 0;
+  static constexpr uint32_t RING_OFF = Q_TILE_BYTES;
+  static constexpr uint32_t BAR_OFF = RING_OFF + NSLOT * SLOT_BYTES;
+  // barriers: q_full, q_empty, full[NSLOT], empty[NSLOT], s[2], p[2][2], o[2], o_empty, drain
+  static constexpr int NBAR = 2 + 2 * NSLOT + 12;
+  static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
+  static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
+  static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;
+  static constexpr uint32_t TMEM_COLS = 512;
+  static constexpr uint32_t S_COL = 0;       // + buffer * BN
+  static constexpr uint32_t O_COL = 2 * BN;
+  static_assert(BYTES <= 227 * 1024, "shared memory budget");
+  static_assert(O_COL + D <= TMEM_COLS, "TMEM budget");
+};
+
+template <int D>
+__device__ __forceinline__ Item make_item1(const FwdParams& p, int idx) {
+  using C = Fwd1Cfg<D>;
+  const int BH = p.n_items / p.n_pairs;  // n_pairs holds the query tiles per (b, h) here
+  int qt, bh;
+  if (p.causal) {
+    qt = p.n_pairs - 1 - idx / BH;
+    bh = idx % BH;
+  } else {
+    qt = idx % p.n_pairs;
+    bh = idx / p.n_pairs;
+  }
+  Item it;
+  it.h = bh % p.Hq;
+  it.b = bh / p.Hq;
+  it.q_z = bh;
+  it.kv_z = it.b * p.Hkv + it.h / (p.Hq / p.Hkv);
+  it.q0 = qt * C::BM;
+  int n_kv = p.Skv;
+  if (p.causal) n_kv = min(p.Skv, it.q0 + C::BM + (p.Skv - p.Sq));
+  it.n_tiles0 = it.n_tiles = (n_kv + C::BN - 1) / C::BN;
+  return it;
+}
+
+// Ring positions of K_j and V_j within an item of n KV tiles (order above).
+__device__ __forceinline__ int ring_pos_k(int j) { return j == 0 ? 0 : 2 * j - 1; }
+__device__ __forceinline__ int ring_pos_v(int j, int n) { return j == n - 1 ? 2 * n - 1 : 2 * j + 2; }
+
+template <int D>
+__global__ void __launch_bounds__(Fwd1Cfg<D>::THREADS, 1)
+    attn_fwd1_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                     const __grid_constant__ CUtensorMap tm_v, const FwdParams p) {
+  using C = Fwd1Cfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_base = smem_u32(smem_raw);
+  const uint32_t sbase = (raw_base + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (sbase - raw_base);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const uint32_t bar_q = sbase + C::BAR_OFF;
+  const uint32_t bar_qe = bar_q + 8;
+  const uint32_t bar_full = bar_qe + 8;               // [NSLOT]
+  const uint32_t bar_empty = bar_full + 8 * C::NSLOT;  // [NSLOT]
+  const uint32_t bar_s = bar_empty + 8 * C::NSLOT;     // [2]    S in buffer b ready
+  const uint32_t bar_p = bar_s + 16;                   // [2][2] half h of P in buffer b written
+  const uint32_t bar_o = bar_p + 32;                   // [2]    P.V of S number g (g % 2 == b) done
+  const uint32_t bar_oe = bar_o + 16;                  // O read out by the epilogue
+  const uint32_t bar_drain = bar_oe + 8;
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::TMEM_PTR_OFF);
+  Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
+
+  if (threadIdx.x == 0) {
+    mbar_init(bar_q, 1);
+    mbar_init(bar_qe, 1);
+    for (int i = 0; i < C::NSLOT; ++i) {
+      mbar_init(bar_full + 8 * i, 1);
+      mbar_init(bar_empty + 8 * i, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(bar_s + 8 * b, 1);
+      mbar_init(bar_p + 16 * b, C::BM);
+      mbar_init(bar_p + 16 * b + 8, C::BM);
+      mbar_init(bar_o + 8 * b, 1);
+    }
+    mbar_init(bar_oe, C::BM);
+    mbar_init(bar_drain, 1);
+    *ab.flag = 0;
+    *(ab.flag + 1) = 0;
+    fence_barrier_init();
+  }
+  if (warp == 5) tmem_alloc(smem_u32(tmem_ptr), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_ptr;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------------ loader
+    if (lane == 0) {
+      prefetch_tensormap(&tm_q);
+      prefetch_tensormap(&tm_k);
+      prefetch_tensormap(&tm_v);
+      int pos = 0, issued = 0, skipped = -1, q_issued = 0;
+      bool ok = true;
+      for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+        const Item it = make_item1<D>(p, idx);
+        const int n = it.n_tiles;
+        if (r > 0 && !(ok = mbar_wait(bar_qe, (r - 1) & 1, p.ctl, ab))) break;
+        mbar_expect_tx(bar_q, C::Q_TILE_BYTES);
+        for (int x = 0; x < C::NBOX; ++x)
+          tma_load_3d(sbase + C::Q_OFF + x * C::Q_BOX_BYTES, &tm_q, x * C::BOX_COLS, it.q0, it.q_z, bar_q);
+        q_issued = r + 1;
+        for (int sq = 0; sq < 2 * n; ++sq, ++pos) {
+          const int slot = pos % C::NSLOT, round = pos / C::NSLOT;
+          if (!(ok = mbar_wait(bar_empty + 8 * slot, (round & 1) ^ 1, p.ctl, ab))) break;
+          issued = pos + 1;
+          if (p.ctl.inject == 2 && pos == 2) {  // test hook: never load this tile
+            skipped = pos;
+            continue;
+          }
+          // sequence index sq -> K_0 | V_{n-1} (last) | K_{(sq+1)/2} (odd) | V_{sq/2-1} (even)
+          const bool is_v = sq != 0 && (sq == 2 * n - 1 || (sq & 1) == 0);
+          const int tile = sq == 0 ? 0 : sq == 2 * n - 1 ? n - 1 : (sq & 1) ? (sq + 1) / 2 : sq / 2 - 1;
+          mbar_expect_tx(bar_full + 8 * slot, C::SLOT_BYTES);
+          for (int x = 0; x < C::NBOX; ++x)
+            tma_load_3d(sbase + C::RING_OFF + slot * C::SLOT_BYTES + x * C::KV_BOX_BYTES,
+                        is_v ? &tm_v : &tm_k, x * C::BOX_COLS, tile * C::BN, it.kv_z, bar_full + 8 * slot);
+        }
+      }
+      Abort no_abort{ab.flag + 1};
+      if (q_issued > 0) mbar_wait(bar_q, (q_issued - 1) & 1, p.ctl, no_abort);
+      for (int ps = max(0, issued - C::NSLOT); ps < issued; ++ps)
+        if (ps != skipped)
+          mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, no_abort);
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16(C::BM, C::BN, 0, 0);
+      constexpr uint32_t idesc_pv = idesc_bf16(C::BM, D, 0, 1);
+      const uint64_t dq = sdesc_sw128(sbase + C::Q_OFF, 16, 1024);
+      const uint64_t dk0 = sdesc_sw128(sbase + C::RING_OFF, 16, 1024);
+      const uint64_t dv0 = sdesc_sw128(sbase + C::RING_OFF, C::KV_BOX_BYTES, 1024);
+      constexpr uint32_t kSlot16 = C::SLOT_BYTES >> 4, kQBox16 = C::Q_BOX_BYTES >> 4;
+      constexpr uint32_t kKBox16 = C::KV_BOX_BYTES >> 4;
+      auto wait_slot = [&](int ps) {
+        return mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, ab);
+      };
+      auto issue_s = [&](int buf, int kpos) {
+        const uint64_t b = dk0 + (kpos % C::NSLOT) * kSlot16;
+#pragma unroll
+        for (int x = 0; x < C::NBOX; ++x)
+          mma_ss_k64(tmem + C::S_COL + buf * C::BN, dq + x * kQBox16, b + x * kKBox16, idesc_s, x > 0);
+      };
+      auto issue_pv = [&](int buf, int vpos, bool acc, int half) {
+        const uint64_t b = dv0 + (vpos % C::NSLOT) * kSlot16 + half * (C::BN / 2) * (128 >> 4);
+        mma_ts_k64(tmem + C::O_COL, tmem + C::S_COL + buf * C::BN + half * (C::BN / 4), b, idesc_pv,
+                   acc ? 1u : 0u);
+      };
+      int pos = 0, g = 0;  // ring position of the item's first tile; S tiles issued so far
+      bool ok = true;
+      for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+        const Item it = make_item1<D>(p, idx);
+        const int n = it.n_tiles;
+        if (!(ok = mbar_wait(bar_q, r & 1, p.ctl, ab))) break;
+        // S_0 and S_1 of the item into the two buffers
+        for (int j = 0; j < 2 && j < n; ++j) {
+          const int kp = pos + ring_pos_k(j);
+          if (!(ok = wait_slot(kp))) break;
+          tc_fence_after();
+          issue_s((g + j) & 1, kp);
+          tc_commit(bar_s + 8 * ((g + j) & 1));
+          tc_commit(bar_empty + 8 * (kp % C::NSLOT));
+        }
+        if (!ok) break;
+        if (n <= 2) tc_commit(bar_qe);  // every S of this item issued
+        for (int j = 0; j < n; ++j) {
+          const int gj = g + j, buf = gj & 1;
+          const int vp = pos + ring_pos_v(j, n);
+          if (!(ok = wait_slot(vp))) break;
+          if (!(ok = mbar_wait(bar_p + 16 * buf, (gj >> 1) & 1, p.ctl, ab))) break;
+          if (j == 0 && r > 0 && !(ok = mbar_wait(bar_oe, (r - 1) & 1, p.ctl, ab))) break;
+          tc_fence_after();
+          issue_pv(buf, vp, j > 0, 0);
+          if (!(ok = mbar_wait(bar_p + 16 * buf + 8, (gj >> 1) & 1, p.ctl, ab))) break;
+          tc_fence_after();
+          issue_pv(buf, vp, true, 1);
+          tc_commit(bar_o + 8 * buf);
+          tc_commit(bar_empty + 8 * (vp % C::NSLOT));
+          if (j + 2 < n) {  // S_{j+2} into the buffer P_j V_j has just been issued from
+            const int kp = pos + ring_pos_k(j + 2);
+            if (!(ok = wait_slot(kp))) break;
+            tc_fence_after();
+            issue_s(buf, kp);
+            tc_commit(bar_s + 8 * buf);
+            tc_commit(bar_empty + 8 * (kp % C::NSLOT));
+            if (j + 3 == n) tc_commit(bar_qe);
+          }
+        }
+        g += n;
+        pos += 2 * n;
+      }
+      Abort no_abort{ab.flag + 1};
+      tc_commit(bar_drain);
+      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+    }
+  } else {
+    // ------------------------------------------------------------------ softmax
+    const uint32_t lane_addr = static_cast<uint32_t>(warp * 32) << 16;
+    const uint32_t s_tm0 = tmem + lane_addr + C::S_COL;
+    const uint32_t o_tm = tmem + lane_addr + C::O_COL;
+    const float c = p.c;
+    const uint64_t c2 = f2(c, c);
+    const int off = p.Skv - p.Sq;
+    int g = 0;  // S tiles processed in earlier items
+    bool ok = true;
+    for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+      const Item it = make_item1<D>(p, idx);
+      const int n = it.n_tiles;
+      const int row = it.q0 + warp * 32 + lane;
+      const int limit = p.causal ? min(p.Skv, row + off + 1) : p.Skv;
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int j = 0; ok && j < n; ++j) {
+        const int gj = g + j, buf = gj & 1;
+        // the previous P.V (S number gj - 1) completes on bar_o[(gj - 1) % 2]
+        ok = softmax_step<D, C::BN>(s_tm0 + buf * C::BN, o_tm, bar_s + 8 * buf, (gj >> 1) & 1,
+                                    bar_p + 16 * buf, bar_o + 8 * ((gj - 1) & 1), ((gj - 1) >> 1) & 1,
+                                    j == 0, j * C::BN, limit, c, c2, m_run, l_run, p.ctl, ab);
+      }
+      if (!ok) break;
+      const int gl = g + n - 1;  // the item's last P.V
+      if (!(ok = softmax_epilogue<D>(o_tm, bar_o + 8 * (gl & 1), (gl >> 1) & 1, bar_oe, m_run, l_run,
+                                     row, it.q_z, p, ab)))
+        break;
+      g += n;
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
@@ -499,20 +790,20 @@ bool make_map(CUtensorMap* map, const void* base, int D, int rows, int planes, i
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int D>
-cudaError_t launch_fwd_d(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
-  using C = FwdCfg<D>;
+// Launch one design: C is its configuration, rows_per_item the query rows of one work
+// item (C::NQT * C::BM).
+template <int D, class C, class Kernel>
+cudaError_t launch_design(Kernel kernel, int rows_per_item, const FwdArgs& a, const KernelCtl& ctl,
+                          cudaStream_t stream, unsigned long long& configured) {
   CUtensorMap mq, mk, mv;
   if (!make_map(&mq, a.q, D, a.Sq, a.B * a.Hq, C::BM) ||
       !make_map(&mk, a.k, D, a.Skv, a.B * a.Hkv, C::BN) ||
       !make_map(&mv, a.v, D, a.Skv, a.B * a.Hkv, C::BN))
     return cudaErrorInvalidValue;
-  static unsigned long long configured = 0;  // one bit per device
   int dev = 0;
   cudaGetDevice(&dev);
   if (!(configured & (1ull << (dev & 63)))) {
-    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         C::BYTES);
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::BYTES);
     if (e != cudaSuccess) return e;
     configured |= 1ull << (dev & 63);
   }
@@ -523,20 +814,31 @@ cudaError_t launch_fwd_d(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t st
   p.Hkv = a.Hkv;
   p.Sq = a.Sq;
   p.Skv = a.Skv;
-  p.n_pairs = (a.Sq + C::NQT * C::BM - 1) / (C::NQT * C::BM);
+  p.n_pairs = (a.Sq + rows_per_item - 1) / rows_per_item;
   p.causal = a.causal;
   p.c = a.scale * kLog2e;
   p.ctl = ctl;
   const long long items = static_cast<long long>(p.n_pairs) * a.B * a.Hq;
   if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   p.n_items = static_cast<int>(items);
-  // persistent: one CTA per SM (shared memory admits one), each walking its items
+  // persistent: one CTA per SM (shared memory / TMEM admit one), each walking its items
   int sms = 0;
   cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
   const int grid = static_cast<int>(items < sms ? items : sms);
-  attn_fwd_kernel<D><<<grid, C::THREADS, C::BYTES, stream>>>(mq, mk, mv, p);
+  kernel<<<grid, C::THREADS, C::BYTES, stream>>>(mq, mk, mv, p);
   return cudaGetLastError();
+}
+
+template <int D>
+cudaError_t launch_fwd_d(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  static unsigned long long configured2 = 0, configured1 = 0;  // one bit per device
+  constexpr int kModelTiles = model::fwd_plan(D).q_tiles;
+  const int q_tiles = a.design ? a.design : kModelTiles;
+  if (q_tiles == 1)
+    return launch_design<D, Fwd1Cfg<D>>(attn_fwd1_kernel<D>, Fwd1Cfg<D>::BM, a, ctl, stream, configured1);
+  return launch_design<D, FwdCfg<D>>(attn_fwd_kernel<D>, FwdCfg<D>::NQT * FwdCfg<D>::BM, a, ctl, stream,
+                                     configured2);
 }
 
 }  // namespace

@@ -20,6 +20,7 @@ __device__ uint32_t g_error_word = 0;
 constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // 2 s
 uint64_t g_timeout_ns = kDefaultTimeoutNs;
 int g_inject = 0;
+int g_prefill_design = 0;
 
 constexpr int kMaxDevices = 64;
 uint32_t* g_err_ptr[kMaxDevices] = {};
@@ -100,7 +101,7 @@ loom_status loom_attn_fwd(const void* q, const void* k, const void* v, void* o, 
     return LOOM_ERR_UNSUPPORTED;
   KernelCtl ctl;
   if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
-  FwdArgs a{q, k, v, o, lse, B, Hq, Hkv, Sq, Skv, D, causal, scale};
+  FwdArgs a{q, k, v, o, lse, B, Hq, Hkv, Sq, Skv, D, causal, scale, g_prefill_design};
   return launch_fwd(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                : LOOM_ERR_CUDA;
 }
@@ -214,5 +215,7 @@ double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, in
 void loom_debug_set_timeout_ns(uint64_t ns) { g_timeout_ns = ns ? ns : kDefaultTimeoutNs; }
 
 void loom_debug_inject(int mode) { g_inject = mode; }
+
+void loom_debug_prefill_design(int q_tiles) { g_prefill_design = (q_tiles == 1 || q_tiles == 2) ? q_tiles : 0; }
 
 }  // extern "C"

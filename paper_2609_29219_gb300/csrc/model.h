@@ -38,11 +38,12 @@ struct ArchDesc {
   double cta_start_ns;      // start-up of a decode split CTA: launch, first copies (measured)
   double mma_clk_per_n;     // clocks of one 128xNx16 bf16 MMA per unit of N (measured: 0.5)
   double mma_min_clk;       // floor on one MMA's clocks (measured: 48 at N = 64)
+  double softmax_clk_per_key;  // softmax of one 128-row tile, clocks per key (measured)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
-    1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0,
+    1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -63,102 +64,118 @@ constexpr double dmax(double a, double b) { return a > b ? a : b; }
 constexpr long long cdiv(long long a, long long b) { return (a + b - 1) / b; }
 
 // ------------------------------------------------------------------ prefill
-// Candidate x = (BN keys per tile, KV ring slots), knobs b = (b_lm, b_ms).  Fixed by the
-// kernel structure: BM = 128 query rows per tile (one per TMEM lane) and 2 query tiles
-// per CTA, whose softmax and MMA phases alternate on the tensor pipe.
+// Candidates: design (q_tiles, s_buffers) x BN keys per tile x KV ring slots x knob
+// b = (b_lm, b_ms).  BM = 128 query rows per tile (one per TMEM lane).  Two designs
+// are implemented:
+//   q_tiles = 2, s_buffers = 1: two query tiles alternate on the tensor pipe; each
+//     tile's chain S -> softmax -> P.V -> next S is serial;
+//   q_tiles = 1, s_buffers = 2: one query tile with S double-buffered in TMEM, i.e.
+//     the boundary between the S MMA and the softmax body is opened (Eq. 6 knob) at the
+//     price of a second S buffer (TMEM capacity, Eq. 8).
 struct FwdPlan {
-  int bm, bn, q_tiles, kv_slots, b_lm, b_ms;
+  int bm, bn, q_tiles, s_buffers, kv_slots, b_lm, b_ms;
   int smem_bytes, tmem_cols;
-  double t_load_ns, t_mma_ns, t_softmax_ns, t_iter_ns;  // one KV-tile iteration of one CTA
+  double t_load_ns, t_mma_ns, t_softmax_ns, t_iter_ns;  // per KV tile, per query tile
   bool feasible;
 };
 
-// Primitive latencies of one KV-tile iteration of one CTA (ns).
-constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int bn, int slots, int b_lm, int b_ms) {
+// Primitive latencies of one KV-tile iteration (per query tile, ns).
+constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int q_tiles, int s_buffers, int bn, int slots,
+                           int b_lm, int b_ms) {
   FwdPlan p{};
   p.bm = 128;
-  p.q_tiles = 2;
+  p.q_tiles = q_tiles;
+  p.s_buffers = s_buffers;
   p.bn = bn;
   p.kv_slots = slots;
   p.b_lm = b_lm;
   p.b_ms = b_ms;
   const double clk = a.sm_ghz;  // clocks per ns
-  // load stage: K_j and V_j tiles, mostly L2 hits (the CTAs of a head share them)
-  const double kv_bytes = 2.0 * bn * D * 2;
-  p.t_load_ns = kv_bytes / a.l2_smem_gbs_sm;  // GB/s == bytes/ns
-  // compute leaf: 2 GEMMs (S = Q K^T with N = BN, O += P V with N = D) per query tile,
-  // K/16 tcgen05 MMAs each, at the measured clocks per 128xNx16 MMA
+  // load stage: K_j and V_j tiles (mostly L2 hits), shared by the CTA's query tiles
+  p.t_load_ns = 2.0 * bn * D * 2 / a.l2_smem_gbs_sm / q_tiles;
+  // compute leaf: S = Q K^T (N = BN) and O += P V (N = D), K/16 MMAs each
   auto mma_clk = [&](int n) { return dmax(a.mma_clk_per_n * n, a.mma_min_clk); };
-  const double clk_s = (D / 16.0) * mma_clk(bn), clk_pv = (bn / 16.0) * mma_clk(D);
-  p.t_mma_ns = p.q_tiles * (clk_s + clk_pv) / clk;
-  // softmax leaf: one ex2 per score on MUFU; ~5 FMA-pipe ops per score (scale/subtract,
-  // max, add, half a pack, mask/compare amortised) -- two tiles share the SM
-  const double scores = 1.0 * p.q_tiles * p.bm * bn;
-  const double t_ex2 = scores / (a.ex2_per_clk_sm * clk);
-  const double t_fma = scores * 5.0 / (a.fp32_per_clk_sm * clk);
-  p.t_softmax_ns = dmax(t_ex2, t_fma);
-  // body: with two query tiles the tensor pipe and the softmax warps overlap; each
-  // iteration still pays one S-ready / P-ready handshake that nothing hides
-  const double body = dmax(p.t_mma_ns, p.t_softmax_ns) + a.sync_ns;
-  // store stage of the iteration is empty (O is stored once per tile)
+  p.t_mma_ns = ((D / 16.0) * mma_clk(bn) + (bn / 16.0) * mma_clk(D)) / clk;
+  // softmax leaf of one query tile (measured clocks per key of a 128-row tile)
+  p.t_softmax_ns = a.softmax_clk_per_key * bn / clk;
+  const double sync = a.sync_ns;
+  double body = 0.0;
+  if (q_tiles == 2) {
+    // two tiles alternate: per pair of tile-iterations the tensor pipe needs 2 * mma,
+    // and each tile's chain (softmax, then its P.V and next S) must fit in the period;
+    // the two softmaxes share the SM's MUFU and issue slots, so they do not overlap
+    body = dmax(2 * p.t_mma_ns, dmax(p.t_softmax_ns + p.t_mma_ns, 2 * p.t_softmax_ns) + 2 * sync) / 2;
+  } else {
+    // S double-buffered: softmax and MMA overlap fully; one handshake per tile
+    body = dmax(p.t_mma_ns, p.t_softmax_ns) + sync;
+  }
   p.t_iter_ns = heg_pipe(p.t_load_ns, body, 0.0, b_lm, b_ms);
   // resources (Eq. 8 constraints)
-  p.smem_bytes = p.q_tiles * p.bm * D * 2 + slots * bn * D * 2 + 1024 + 256;
-  p.tmem_cols = p.q_tiles * (bn + D);
+  p.smem_bytes = q_tiles * p.bm * D * 2 + slots * bn * D * 2 + 1024 + 256;
+  p.tmem_cols = q_tiles * (s_buffers * bn + D);
   p.feasible = true;
+  if (!((q_tiles == 2 && s_buffers == 1) || (q_tiles == 1 && s_buffers == 2))) p.feasible = false;
   if (bn % 16 != 0 || bn < 16 || bn > 256) p.feasible = false;   // MMA N for M = 128
-  if (bn % 32 != 0 || bn > 128) p.feasible = false;              // softmax: <= 128 fp32 regs/row
+  if (bn != 128) p.feasible = false;  // softmax: one S row of 128 fp32 per thread, P in halves
   if (D % 64 != 0) p.feasible = false;                            // 128 B swizzle atoms
   if (p.smem_bytes > a.smem_per_cta) p.feasible = false;          // L1 footprint
   if (p.tmem_cols > a.tmem_cols) p.feasible = false;
-  if (slots < 2) p.feasible = false;                              // K and V of one tile
-  // an open load boundary needs the next tile's K and V in flight while this tile's
-  // K and V are being read: >= 4 slots, and enough of them to cover the latency
-  if (b_lm && (slots < 4 || (slots / 2 - 1) * body < a.mem_latency_ns * 0.5)) p.feasible = false;
-  if (slots % 2 != 0) p.feasible = false;                         // K/V alternate in the ring
+  // an open load boundary needs the loads of the next tiles in flight while the current
+  // ones are read: at least 4 slots, enough of them to cover the memory latency
+  if (slots < 4) p.feasible = false;
+  if (b_lm && (slots / 2 - 1) * body * q_tiles < a.mem_latency_ns * 0.5) p.feasible = false;
+  if (!b_lm) p.feasible = false;  // both kernels always prefetch through the ring
+  if (q_tiles == 2 && slots % 2 != 0) p.feasible = false;        // K/V alternate in the ring
   return p;
 }
 
-// Eq. 8-9 by enumeration: BN in {32, ..., 256}, slots in {2, ..., 16}, knobs in {0,1}^2.
-// Ties go to fewer slots (less shared memory), then smaller BN.
-constexpr FwdPlan fwd_plan(int D, const ArchDesc& a = kGb300) {
+// Eq. 8 for one design by enumeration over BN, slots and knobs; ties go to fewer slots.
+constexpr FwdPlan fwd_plan_variant(int D, int q_tiles, const ArchDesc& a = kGb300) {
   FwdPlan best{};
   best.feasible = false;
+  const int s_buffers = q_tiles == 2 ? 1 : 2;
   for (int bn = 32; bn <= 256; bn += 16)
     for (int slots = 2; slots <= 16; ++slots)
       for (int b_lm = 0; b_lm <= 1; ++b_lm)
         for (int b_ms = 0; b_ms <= 1; ++b_ms) {
-          FwdPlan p = fwd_eval(a, D, bn, slots, b_lm, b_ms);
+          FwdPlan p = fwd_eval(a, D, q_tiles, s_buffers, bn, slots, b_lm, b_ms);
           if (!p.feasible) continue;
-          // per-key cost: iterations scale with 1 / BN
-          const double cost = p.t_iter_ns / bn;
+          const double cost = p.t_iter_ns / bn;  // per key and query tile
           const double best_cost = best.feasible ? best.t_iter_ns / best.bn : 1e300;
           if (cost < best_cost * (1.0 - 1e-9)) best = p;
         }
   return best;
 }
 
-// Modeled time (us) of a whole prefill launch under a plan.
+// Eq. 9: the design with the lowest modeled latency.
+constexpr FwdPlan fwd_plan(int D, const ArchDesc& a = kGb300) {
+  const FwdPlan two = fwd_plan_variant(D, 2, a), one = fwd_plan_variant(D, 1, a);
+  if (!one.feasible) return two;
+  if (!two.feasible) return one;
+  return one.t_iter_ns / one.bn < two.t_iter_ns / two.bn * (1.0 - 1e-9) ? one : two;
+}
+
+// Modeled time (us) of a whole prefill launch under a plan (Eq. 5-7 over the CTA's
+// items: Q load ; for(KV tiles, pipe) ; O store, in waves over the SMs).
 constexpr double fwd_time_us(const FwdPlan& p, int B, int Hq, int Sq, int Skv, int D, int causal,
                              const ArchDesc& a = kGb300) {
   const long long rows_per_cta = 1LL * p.q_tiles * p.bm;
-  const long long pairs = cdiv(Sq, rows_per_cta);
-  const long long ctas = pairs * B * Hq;
-  // average KV tiles per CTA
-  double tiles = 0;
-  for (long long i = 0; i < pairs; ++i) {
+  const long long groups = cdiv(Sq, rows_per_cta);
+  const long long ctas = groups * B * Hq;
+  double tiles = 0;  // average KV tiles per query tile
+  for (long long i = 0; i < cdiv(Sq, p.bm); ++i) {
     long long n_kv = Skv;
     if (causal) {
-      const long long lim = (i + 1) * rows_per_cta + (Skv - Sq);
+      const long long lim = (i + 1) * p.bm + (Skv - Sq);
       n_kv = lim < Skv ? lim : Skv;
     }
     tiles += static_cast<double>(cdiv(n_kv, p.bn));
   }
-  tiles /= static_cast<double>(pairs);
-  const double t_q = 2.0 * rows_per_cta * D * 2 / a.l2_smem_gbs_sm;
+  tiles /= static_cast<double>(cdiv(Sq, p.bm));
+  const double t_q = 1.0 * rows_per_cta * D * 2 / a.l2_smem_gbs_sm;
   const double t_o = 1.0 * rows_per_cta * D * 2 / a.l2_smem_gbs_sm;
-  const double t_cta = heg_seq(heg_seq(t_q, heg_for(tiles, p.t_iter_ns)), t_o);
-  const double waves = static_cast<double>(ctas) / a.num_sms;  // fractional: LPT ordering
+  const double t_cta = heg_seq(heg_seq(t_q, heg_for(tiles * p.q_tiles, p.t_iter_ns)), t_o);
+  const double waves = static_cast<double>(ctas) / a.num_sms;  // persistent CTAs
   const double w = waves < 1.0 ? 1.0 : waves;
   return w * t_cta * 1e-3;
 }

@@ -289,6 +289,19 @@ __device__ __forceinline__ float ex2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+// 2^x on the FMA pipe (relieves MUFU when a warp cannot keep it busy): round-to-
+// nearest range reduction x = n + f, |f| <= 1/2, with n taken from the low mantissa bits
+// of x + 1.5*2^23; a cubic for 2^f fitted here by relative-error least squares on
+// [-1/2, 1/2] (max relative error 7.8e-5, below bf16 rounding); 2^n applied by adding n
+// to the exponent field.  Valid for x <= 64; inputs below -125 (and -inf) give 2^-125.
+__device__ __forceinline__ float exp2_poly(float x) {
+  x = fmaxf(x, -125.f);
+  const float t = x + 12582912.f;  // 1.5 * 2^23
+  const float f = x - (t - 12582912.f);
+  const float p = fmaf(fmaf(fmaf(0.055088684f, f, 0.24260405f), f, 0.6932762f), f, 0.99992895f);
+  return __int_as_float(__float_as_int(p) + (__float_as_int(t) << 23));
+}
+
 // Two floats -> bf16x2 (round to nearest even); `lo` lands in the low half.
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   uint32_t r;

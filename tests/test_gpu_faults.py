@@ -63,7 +63,16 @@ def test_decode_skipped_stage_times_out_and_context_survives(loom):
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "decode after timeout")
 
 
-def test_prefill_skipped_tile_times_out_and_context_survives(loom):
+@pytest.mark.parametrize("design", [2, 1])
+def test_prefill_skipped_tile_times_out_and_context_survives(loom, design):
+    loom.loom_debug_prefill_design(design)
+    try:
+        _prefill_fault_case(loom)
+    finally:
+        loom.loom_debug_prefill_design(0)
+
+
+def _prefill_fault_case(loom):
     B, H, S, D = 1, 2, 512, 128  # 4 work items, each with 4 KV tiles
     q = synth.bf16_normal(32, synth.STREAM_Q, (B, H, S, D))
     k = synth.bf16_normal(32, synth.STREAM_K, (B, H, S, D))

@@ -20,6 +20,15 @@ def loom():
     return m
 
 
+@pytest.fixture(autouse=True, params=[2, 1], ids=["two_tiles", "one_tile_double_s"])
+def design(request, loom):
+    """Run every prefill test with both kernel designs (two alternating query tiles; one
+    query tile with S double-buffered in TMEM)."""
+    loom.loom_debug_prefill_design(request.param)
+    yield request.param
+    loom.loom_debug_prefill_design(0)
+
+
 def _inputs(seed, B, Hq, Hkv, Sq, Skv, D):
     return (synth.bf16_normal(seed, synth.STREAM_Q, (B, Hq, Sq, D)),
             synth.bf16_normal(seed, synth.STREAM_K, (B, Hkv, Skv, D)),
