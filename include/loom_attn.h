@@ -127,8 +127,8 @@ loom_status loom_attn_decode_noalloc(const void* q, const void* k_cache, const v
  * selection of Eq. 8-9, solved by enumeration) with the GB300 architecture description
  * of Sec. 2.7.  The kernels are compiled with the plan these functions report.
  *
- * loom_model_fwd_plan: the prefill plan for head dimension D (64 or 128): rows per query
- *   tile, keys per KV tile, query tiles per CTA, K/V ring slots, the pipeline knob
+ * loom_model_fwd_plan: the prefill plan for head dimension D (64 or 128): the design, rows
+ *   per query tile, keys per KV tile, query tiles per CTA, S buffers, K/V ring slots, the pipeline knob
  *   (b_lm, b_ms) of Eq. 6, shared-memory bytes, TMEM columns, and the modeled latencies
  *   (ns) of one KV-tile iteration: load stage, MMA leaf, softmax leaf, and the pipe node.
  *   Returns LOOM_ERR_UNSUPPORTED for other D, LOOM_ERR_INVALID_ARG for a NULL out.
@@ -137,7 +137,8 @@ loom_status loom_attn_decode_noalloc(const void* q, const void* k_cache, const v
  *   `splits` splits on `num_sms` SMs (every sequence Skv keys); < 0 on bad sizes.
  */
 typedef struct {
-  int bm, bn, q_tiles, kv_slots, b_lm, b_ms, smem_bytes, tmem_cols;
+  int design; /* 2: two alternating query tiles; 1: one tile, S double-buffered; 3: two tiles, S ring of 3 */
+  int bm, bn, q_tiles, s_buffers, kv_slots, b_lm, b_ms, smem_bytes, tmem_cols;
   double t_load_ns, t_mma_ns, t_softmax_ns, t_iter_ns;
 } loom_fwd_plan;
 loom_status loom_model_fwd_plan(int D, loom_fwd_plan* out);
@@ -168,11 +169,12 @@ void loom_debug_inject(int mode);
 
 /*
  * Test hook: force the prefill design instead of the analytic model's choice (used to
- * measure the alternatives the model ranks).  q_tiles = 2: two query tiles per CTA that
- * alternate on the tensor pipe; q_tiles = 1: one query tile with S double-buffered in
- * TMEM; anything else: the model's choice (default).
+ * measure the alternatives the model ranks).  2: two query tiles per CTA that alternate
+ * on the tensor pipe; 1: one query tile with S double-buffered in TMEM; 3: two query
+ * tiles sharing a ring of three S buffers (D = 64 only; D = 128 falls back to 2);
+ * anything else: the model's choice (default).
  */
-void loom_debug_prefill_design(int q_tiles);
+void loom_debug_prefill_design(int design);
 
 #ifdef __cplusplus
 }

@@ -40,8 +40,8 @@ STATUS = {
 
 class FwdPlan(ctypes.Structure):
     """Mirror of ``loom_fwd_plan`` (include/loom_attn.h)."""
-    _fields_ = [(n, ctypes.c_int) for n in ("bm", "bn", "q_tiles", "kv_slots", "b_lm", "b_ms",
-                                             "smem_bytes", "tmem_cols")] + \
+    _fields_ = [(n, ctypes.c_int) for n in ("design", "bm", "bn", "q_tiles", "s_buffers", "kv_slots",
+                                             "b_lm", "b_ms", "smem_bytes", "tmem_cols")] + \
                [(n, ctypes.c_double) for n in ("t_load_ns", "t_mma_ns", "t_softmax_ns", "t_iter_ns")]
 
     def as_dict(self):
@@ -238,8 +238,8 @@ def loom_debug_inject(mode: int):
     capi().loom_debug_inject(int(mode))
 
 
-def loom_debug_prefill_design(q_tiles: int):
-    capi().loom_debug_prefill_design(int(q_tiles))
+def loom_debug_prefill_design(design: int):
+    capi().loom_debug_prefill_design(int(design))
 
 
 def loom_model_fwd_plan(D: int) -> dict:

@@ -51,7 +51,7 @@ struct FwdCfg {
   static constexpr int NSLOT = kPlan.kv_slots;  // K/V ring slots
   static_assert(BM == 128 && NQT == 2, "warp roles assume two 128-row query tiles");
   static_assert(BN == 128, "softmax holds one S row of 128 fp32 in registers, P leaves in two 64-key halves");
-  static_assert(kPlan.b_lm == 1 && NSLOT >= 4, "the loader runs ahead of the MMA by >= one tile");
+  static_assert(kPlan.b_lm == 1 && NSLOT >= 3, "the loader runs ahead of the MMA by >= one tile");
   static constexpr int THREADS = 320;               // 8 softmax warps + loader + MMA
   static constexpr int BOX_COLS = 64;               // 128-byte swizzle atom = 64 bf16
   static constexpr int NBOX = D / BOX_COLS;         // TMA boxes per row of a tile
@@ -61,9 +61,10 @@ struct FwdCfg {
   static constexpr uint32_t SLOT_BYTES = NBOX * KV_BOX_BYTES;
   static constexpr uint32_t Q_OFF = 0;
   static constexpr uint32_t RING_OFF = NQT * Q_TILE_BYTES;
-  static constexpr uint32_t BAR_OFF = RING_OFF + NSLOT * SLOT_BYTES;
-  // barriers: q_full, q_empty, full[NSLOT], empty[NSLOT], s[2], p[2][2], o[2], o_empty[2], drain
-  static constexpr int NBAR = 2 + 2 * NSLOT + 11;
+  static constexpr uint32_t STG_OFF = RING_OFF + NSLOT * SLOT_BYTES;  // O staging per tile
+  static constexpr uint32_t BAR_OFF = STG_OFF + NQT * BM * D * 2;
+  // barriers: q_full[2], q_empty[2], full[NSLOT], empty[NSLOT], s[2], p[2][2], o[2], o_empty[2], drain
+  static constexpr int NBAR = 4 + 2 * NSLOT + 11;
   static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
   static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
   static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;  // + alignment slack
@@ -80,6 +81,7 @@ struct FwdParams {
   int Hq, Hkv, Sq, Skv;
   int n_pairs;   // query-tile pairs per (b, h)
   int n_items;   // n_pairs * B * Hq work items
+  int plane_block;  // causal: (b, h) planes per block of the work order
   int causal;
   float c;       // scale * log2(e)
   KernelCtl ctl;
@@ -91,26 +93,39 @@ struct Item {
 };
 
 // The r-th item of this CTA (-1 once it has none left).  Causal items are ordered
-// heaviest first and dealt out in a snake order (CTA c takes item c of even rounds and
-// item G-1-c of odd rounds) so that long and short items even out per CTA.
+// heaviest first (within blocks of planes, see item_coords) and dealt out in a snake
+// order (CTA c takes item c of even rounds and item G-1-c of odd rounds) so that long and
+// short items even out per CTA.
 __device__ __forceinline__ int item_index(const FwdParams& p, int r) {
   const int G = static_cast<int>(gridDim.x), c = static_cast<int>(blockIdx.x);
   const long long idx = static_cast<long long>(r) * G + ((p.causal && (r & 1)) ? G - 1 - c : c);
   return idx < p.n_items ? static_cast<int>(idx) : -1;
 }
 
+// Item idx -> (position pos of its query tile or tile pair within the plane, plane bh).
+// Non-causal: consecutive items are consecutive positions of one plane (they share its
+// K/V in L2).  Causal: blocks of p.plane_block planes; within a block the bottom (longest)
+// positions of every plane go first.
+__device__ __forceinline__ void item_coords(const FwdParams& p, int idx, int& pos, int& bh) {
+  if (p.causal) {
+    const int BH = p.n_items / p.n_pairs;
+    const int per_block = p.plane_block * p.n_pairs;
+    const int blk = idx / per_block, in = idx - blk * per_block;
+    const int h0 = blk * p.plane_block;
+    const int nb = min(p.plane_block, BH - h0);
+    pos = p.n_pairs - 1 - in / nb;
+    bh = h0 + in % nb;
+  } else {
+    pos = idx % p.n_pairs;
+    bh = idx / p.n_pairs;
+  }
+}
+
 template <int D>
 __device__ __forceinline__ Item make_item(const FwdParams& p, int idx) {
   using C = FwdCfg<D>;
-  const int BH = p.n_items / p.n_pairs;
   int pair, bh;
-  if (p.causal) {  // the longest (bottom) tile pairs of every head go first
-    pair = p.n_pairs - 1 - idx / BH;
-    bh = idx % BH;
-  } else {         // consecutive items share K/V of one head in L2
-    pair = idx % p.n_pairs;
-    bh = idx / p.n_pairs;
-  }
+  item_coords(p, idx, pair, bh);
   Item it;
   it.h = bh % p.Hq;
   it.b = bh / p.Hq;
@@ -225,48 +240,79 @@ __device__ __forceinline__ bool softmax_step(uint32_t s_tm, uint32_t o_tm, uint3
   return true;
 }
 
-// Epilogue of one query row: wait for the last P.V (bar_o, par_o), read O from TMEM,
-// write O / l as bf16 and the log-sum-exp, then hand the O columns back (bar_oe).
+// Epilogue of one query row (this thread's TMEM lane): wait for the last P.V (bar_o,
+// par_o), read O from TMEM into registers as bf16 O / l and hand the O columns back to
+// the MMA warp at once (bar_oe); then write the row into this warp's staging block in
+// shared memory (D / 64 boxes of 32 rows x 128 B, 128B-swizzled like the TMA tile) and
+// let one lane store the block with TMA (rows >= Sq are clipped by the tensor map).  The
+// store completes in the background; the block is reused by this warp one item later,
+// after waiting for the store to have read it.  Finally the log-sum-exp.
 template <int D>
 __device__ __forceinline__ bool softmax_epilogue(uint32_t o_tm, uint32_t bar_o, uint32_t par_o,
                                                  uint32_t bar_oe, float m_run, float l_run,
                                                  int row, int q_z, const FwdParams& p,
-                                                 const Abort& ab) {
+                                                 const Abort& ab, const CUtensorMap* tm_o,
+                                                 uint32_t stg) {
+  const int lane = threadIdx.x & 31;
   if (!mbar_wait_warp(bar_o, par_o, p.ctl, ab)) return false;
   tc_fence_after();
   const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
-  const bool store = row < p.Sq;
-  __nv_bfloat16* orow = p.o + (static_cast<size_t>(q_z) * p.Sq + (store ? row : 0)) * D;
   const uint64_t il2 = f2(inv_l, inv_l);
-#pragma unroll 1
+  uint32_t w[D / 2];  // the row as packed bf16 pairs
+#pragma unroll
   for (int ch = 0; ch < D / 32; ++ch) {
     uint32_t rr[32];
     tmem_ld32(o_tm + ch * 32, rr);
     tmem_wait_ld();
     reg_fence32(rr);
-    uint32_t w[16];
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       const uint64_t x = mul2(f2(__uint_as_float(rr[2 * i]), __uint_as_float(rr[2 * i + 1])), il2);
-      w[i] = pack_bf16x2(f2lo(x), f2hi(x));
-    }
-    if (store) {
-      uint4* dst = reinterpret_cast<uint4*>(orow + ch * 32);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) dst[i] = make_uint4(w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+      w[ch * 16 + i] = pack_bf16x2(f2lo(x), f2hi(x));
     }
   }
   tc_fence_before();
-  mbar_arrive(bar_oe);
-  if (store && p.lse)
+  mbar_arrive(bar_oe);  // O is in registers: the next item's P.V may overwrite it
+  if (lane == 0) bulk_wait_group_read0();  // this warp's previous store has left the block
+  __syncwarp();
+  const uint32_t my_row = stg + static_cast<uint32_t>(lane) * 128u;
+#pragma unroll
+  for (int c = 0; c < D / 8; ++c) {  // 16-byte chunk c of the row: box c / 8, slot c % 8
+    const uint32_t slot = static_cast<uint32_t>((c & 7) ^ (lane & 7));
+    st_shared_v4(my_row + static_cast<uint32_t>(c >> 3) * 4096u + (slot << 4), w[4 * c], w[4 * c + 1],
+                 w[4 * c + 2], w[4 * c + 3]);
+  }
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) {
+#pragma unroll
+    for (int x = 0; x < D / 64; ++x) tma_store_3d(tm_o, stg + x * 4096u, x * 64, row, q_z);
+    bulk_commit_group();
+  }
+  if (row < p.Sq && p.lse)
     p.lse[static_cast<size_t>(q_z) * p.Sq + row] = l_run > 0.f ? (m_run + log2f(l_run)) * kLn2 : -INFINITY;
   return true;
+}
+
+// Bring the next work item's query tiles and first K/V tiles into L2 while the current
+// item still runs, so that its start waits on an L2 hit rather than HBM.
+template <int D, int NQT, int BM>
+__device__ __forceinline__ void prefetch_item_l2(const CUtensorMap* tm_q, const CUtensorMap* tm_k,
+                                                 const CUtensorMap* tm_v, int q0, int q_z, int kv_z) {
+#pragma unroll
+  for (int x = 0; x < D / 64; ++x) {
+#pragma unroll
+    for (int t = 0; t < NQT; ++t) tma_prefetch_l2_3d(tm_q, x * 64, q0 + t * BM, q_z);
+    tma_prefetch_l2_3d(tm_k, x * 64, 0, kv_z);
+    tma_prefetch_l2_3d(tm_v, x * 64, 0, kv_z);
+  }
 }
 
 template <int D>
 __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                    const __grid_constant__ CUtensorMap tm_v, const FwdParams p) {
+                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
+                    const FwdParams p) {
   using C = FwdCfg<D>;
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the 128B-swizzled tiles
@@ -275,9 +321,9 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
   uint8_t* smem = smem_raw + (sbase - raw_base);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  const uint32_t bar_q = sbase + C::BAR_OFF;       // Q tiles loaded (once per item)
-  const uint32_t bar_qe = bar_q + 8;               // Q tiles no longer read (once per item)
-  const uint32_t bar_full = bar_qe + 8;            // [NSLOT]
+  const uint32_t bar_q = sbase + C::BAR_OFF;       // [2] Q_t loaded (once per item)
+  const uint32_t bar_qe = bar_q + 16;              // [2] Q_t no longer read (once per item)
+  const uint32_t bar_full = bar_qe + 16;           // [NSLOT]
   const uint32_t bar_empty = bar_full + 8 * C::NSLOT;
   const uint32_t bar_s = bar_empty + 8 * C::NSLOT;  // [2] S_t ready
   const uint32_t bar_p = bar_s + 16;                // [2][2] half h of P_t written (h = 0: and O_t rescaled)
@@ -288,8 +334,10 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
   Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
 
   if (threadIdx.x == 0) {
-    mbar_init(bar_q, 1);
-    mbar_init(bar_qe, 1);
+    for (int t = 0; t < 2; ++t) {
+      mbar_init(bar_q + 8 * t, 1);
+      mbar_init(bar_qe + 8 * t, 1);
+    }
     for (int s = 0; s < C::NSLOT; ++s) {
       mbar_init(bar_full + 8 * s, 1);
       mbar_init(bar_empty + 8 * s, 1);
@@ -318,19 +366,31 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
       prefetch_tensormap(&tm_q);
       prefetch_tensormap(&tm_k);
       prefetch_tensormap(&tm_v);
-      int pos = 0, issued = 0, skipped = -1, q_issued = 0;
+      int pos = 0, issued = 0, skipped = -1, q_issued[2] = {0, 0};
       bool ok = true;
+      // Q_t of item r, once the previous item's S MMAs of tile t are done with its buffer
+      auto load_q = [&](int t, int r, const Item& it) -> bool {
+        if (r > 0 && !mbar_wait(bar_qe + 8 * t, (r - 1) & 1, p.ctl, ab)) return false;
+        mbar_expect_tx(bar_q + 8 * t, C::Q_TILE_BYTES);
+        for (int x = 0; x < C::NBOX; ++x)
+          tma_load_3d(sbase + C::Q_OFF + t * C::Q_TILE_BYTES + x * C::Q_BOX_BYTES, &tm_q, x * C::BOX_COLS,
+                      it.q0 + t * C::BM, it.q_z, bar_q + 8 * t);
+        q_issued[t] = r + 1;
+        return true;
+      };
       for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
         const Item it = make_item<D>(p, idx);
-        // the previous item's S MMAs must be done with the Q tiles
-        if (r > 0 && !(ok = mbar_wait(bar_qe, (r - 1) & 1, p.ctl, ab))) break;
-        mbar_expect_tx(bar_q, C::NQT * C::Q_TILE_BYTES);
-        for (int t = 0; t < C::NQT; ++t)
-          for (int x = 0; x < C::NBOX; ++x)
-            tma_load_3d(sbase + C::Q_OFF + t * C::Q_TILE_BYTES + x * C::Q_BOX_BYTES, &tm_q,
-                        x * C::BOX_COLS, it.q0 + t * C::BM, it.q_z, bar_q);
-        q_issued = r + 1;
-        for (int jj = 0; jj < 2 * it.n_tiles; ++jj, ++pos) {  // K_0, V_0, K_1, V_1, ...
+        // Q_0 first: tile 0 finishes its S MMAs of the previous item before tile 1 does
+        if (!(ok = load_q(0, r, it))) break;
+        for (int jj = 0; jj < 2 * it.n_tiles; ++jj, ++pos) {  // K_0, [Q_1], V_0, K_1, V_1, ...
+          if (jj == 1 && !(ok = load_q(1, r, it))) break;
+          if (jj == max(0, 2 * it.n_tiles - 6)) {  // three KV tiles before the end
+            const int nidx = item_index(p, r + 1);
+            if (nidx >= 0) {
+              const Item nx = make_item<D>(p, nidx);
+              prefetch_item_l2<D, C::NQT, C::BM>(&tm_q, &tm_k, &tm_v, nx.q0, nx.q_z, nx.kv_z);
+            }
+          }
           const int slot = pos % C::NSLOT, round = pos / C::NSLOT;
           if (!(ok = mbar_wait(bar_empty + 8 * slot, (round & 1) ^ 1, p.ctl, ab))) break;
           issued = pos + 1;
@@ -348,7 +408,8 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
       }
       // drain copies still in flight before the CTA may exit
       Abort no_abort{ab.flag + 1};
-      if (q_issued > 0) mbar_wait(bar_q, (q_issued - 1) & 1, p.ctl, no_abort);
+      for (int t = 0; t < 2; ++t)
+        if (q_issued[t] > 0) mbar_wait(bar_q + 8 * t, (q_issued[t] - 1) & 1, p.ctl, no_abort);
       for (int ps = max(0, issued - C::NSLOT); ps < issued; ++ps)
         if (ps != skipped)
           mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, no_abort);
@@ -392,10 +453,13 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
         tc_fence_after();
         issue_s(0, pos);
         tc_commit(bar_s);
+        if (nt0 == 1) tc_commit(bar_qe);  // every S of tile 0 issued
+        if (!(ok = mbar_wait(bar_q + 8, r & 1, p.ctl, ab))) break;
+        tc_fence_after();
         issue_s(1, pos);
         tc_commit(bar_s + 8);
         tc_commit(bar_empty + 8 * (pos % C::NSLOT));
-        if (nt == 1) tc_commit(bar_qe);  // every S of this item issued
+        if (nt == 1) tc_commit(bar_qe + 8);  // every S of tile 1 issued
         for (int j = 0; j < nt; ++j) {
           const int vpos = pos + 2 * j + 1, kpos = pos + 2 * j + 2;
           const bool more = j + 1 < nt;
@@ -417,6 +481,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
             if (j + 1 < nt0) {
               issue_s(0, kpos);
               tc_commit(bar_s);
+              if (j + 2 == nt0) tc_commit(bar_qe);  // tile 0's last S of the item
             }
           }
           if (!(ok = mbar_wait(bar_p + 16, (cnt1 + j) & 1, p.ctl, ab))) break;
@@ -432,7 +497,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
             issue_s(1, kpos);
             tc_commit(bar_s + 8);
             tc_commit(bar_empty + 8 * (kpos % C::NSLOT));
-            if (j + 2 == nt) tc_commit(bar_qe);  // that was the item's last S
+            if (j + 2 == nt) tc_commit(bar_qe + 8);  // tile 1's last S of the item
           }
         }
         cnt0 += nt0;
@@ -453,6 +518,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
     const uint32_t o_tm = tmem + lane_addr + C::O_COL + t * D;
     const uint32_t my_bar_s = bar_s + 8 * t, my_bar_p = bar_p + 16 * t, my_bar_o = bar_o + 8 * t;
     const uint32_t my_bar_oe = bar_oe + 8 * t;
+    const uint32_t stg_q = sbase + C::STG_OFF + static_cast<uint32_t>(warp) * (32 * D * 2);
     const float c = p.c;
     const uint64_t c2 = f2(c, c);
     const int off = p.Skv - p.Sq;
@@ -470,12 +536,13 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
                                     (cnt + j - 1) & 1, j == 0, j * C::BN, limit, c, c2, m_run,
                                     l_run, p.ctl, ab);
       if (!ok) break;
-      // epilogue: O / l -> bf16 rows, LSE; then hand O_t back to the MMA warp
-      if (!(ok = softmax_epilogue<D>(o_tm, my_bar_o, (cnt + my_tiles - 1) & 1, my_bar_oe, m_run,
-                                     l_run, row, it.q_z, p, ab)))
+      // epilogue: hand O_t back to the MMA warp, O / l -> bf16 rows, LSE
+      if (!(ok = softmax_epilogue<D>(o_tm, my_bar_o, (cnt + my_tiles - 1) & 1, my_bar_oe, m_run, l_run,
+                                     row, it.q_z, p, ab, &tm_o, stg_q)))
         break;
       cnt += my_tiles;
     }
+    if (lane == 0) bulk_wait_group0();  // the O stores have completed before the CTA exits
   }
 
   __syncwarp();
@@ -504,7 +571,7 @@ struct Fwd1Cfg {
   static constexpr int BM = 128;
   static constexpr int BN = kPlan.bn;
   static constexpr int NSLOT = kPlan.kv_slots;
-  static_assert(kPlan.q_tiles == 1 && kPlan.s_buffers == 2, "single-tile variant");
+  static_assert(kPlan.design == 1 && kPlan.q_tiles == 1 && kPlan.s_buffers == 2, "single-tile variant");
   static_assert(BN == 128, "softmax holds one S row of 128 fp32 in registers");
   static constexpr int THREADS = 192;
   static constexpr int BOX_COLS = 64;
@@ -515,7 +582,8 @@ struct Fwd1Cfg {
   static constexpr uint32_t SLOT_BYTES = NBOX * KV_BOX_BYTES;
   static constexpr uint32_t Q_OFF = 0;
   static constexpr uint32_t RING_OFF = Q_TILE_BYTES;
-  static constexpr uint32_t BAR_OFF = RING_OFF + NSLOT * SLOT_BYTES;
+  static constexpr uint32_t STG_OFF = RING_OFF + NSLOT * SLOT_BYTES;  // O staging, one tile
+  static constexpr uint32_t BAR_OFF = STG_OFF + BM * D * 2;
   // barriers: q_full, q_empty, full[NSLOT], empty[NSLOT], s[2], p[2][2], o[2], o_empty, drain
   static constexpr int NBAR = 2 + 2 * NSLOT + 12;
   static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
@@ -531,15 +599,8 @@ struct Fwd1Cfg {
 template <int D>
 __device__ __forceinline__ Item make_item1(const FwdParams& p, int idx) {
   using C = Fwd1Cfg<D>;
-  const int BH = p.n_items / p.n_pairs;  // n_pairs holds the query tiles per (b, h) here
-  int qt, bh;
-  if (p.causal) {
-    qt = p.n_pairs - 1 - idx / BH;
-    bh = idx % BH;
-  } else {
-    qt = idx % p.n_pairs;
-    bh = idx / p.n_pairs;
-  }
+  int qt, bh;  // n_pairs holds the query tiles per (b, h) here
+  item_coords(p, idx, qt, bh);
   Item it;
   it.h = bh % p.Hq;
   it.b = bh / p.Hq;
@@ -559,7 +620,8 @@ __device__ __forceinline__ int ring_pos_v(int j, int n) { return j == n - 1 ? 2 
 template <int D>
 __global__ void __launch_bounds__(Fwd1Cfg<D>::THREADS, 1)
     attn_fwd1_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                     const __grid_constant__ CUtensorMap tm_v, const FwdParams p) {
+                     const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
+                     const FwdParams p) {
   using C = Fwd1Cfg<D>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_base = smem_u32(smem_raw);
@@ -621,6 +683,13 @@ __global__ void __launch_bounds__(Fwd1Cfg<D>::THREADS, 1)
           tma_load_3d(sbase + C::Q_OFF + x * C::Q_BOX_BYTES, &tm_q, x * C::BOX_COLS, it.q0, it.q_z, bar_q);
         q_issued = r + 1;
         for (int sq = 0; sq < 2 * n; ++sq, ++pos) {
+          if (sq == max(0, 2 * n - 6)) {  // three KV tiles before the end
+            const int nidx = item_index(p, r + 1);
+            if (nidx >= 0) {
+              const Item nx = make_item1<D>(p, nidx);
+              prefetch_item_l2<D, 1, C::BM>(&tm_q, &tm_k, &tm_v, nx.q0, nx.q_z, nx.kv_z);
+            }
+          }
           const int slot = pos % C::NSLOT, round = pos / C::NSLOT;
           if (!(ok = mbar_wait(bar_empty + 8 * slot, (round & 1) ^ 1, p.ctl, ab))) break;
           issued = pos + 1;
@@ -719,6 +788,7 @@ __global__ void __launch_bounds__(Fwd1Cfg<D>::THREADS, 1)
     const uint32_t lane_addr = static_cast<uint32_t>(warp * 32) << 16;
     const uint32_t s_tm0 = tmem + lane_addr + C::S_COL;
     const uint32_t o_tm = tmem + lane_addr + C::O_COL;
+    const uint32_t stg_q = sbase + C::STG_OFF + static_cast<uint32_t>(warp) * (32 * D * 2);
     const float c = p.c;
     const uint64_t c2 = f2(c, c);
     const int off = p.Skv - p.Sq;
@@ -740,10 +810,11 @@ __global__ void __launch_bounds__(Fwd1Cfg<D>::THREADS, 1)
       if (!ok) break;
       const int gl = g + n - 1;  // the item's last P.V
       if (!(ok = softmax_epilogue<D>(o_tm, bar_o + 8 * (gl & 1), (gl >> 1) & 1, bar_oe, m_run, l_run,
-                                     row, it.q_z, p, ab)))
+                                     row, it.q_z, p, ab, &tm_o, stg_q)))
         break;
       g += n;
     }
+    if (lane == 0) bulk_wait_group0();  // the O stores have completed before the CTA exits
   }
 
   __syncwarp();
@@ -752,6 +823,263 @@ __global__ void __launch_bounds__(Fwd1Cfg<D>::THREADS, 1)
   if (warp == 5) {
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------- S-ring variant
+// Two 128-row query tiles share a ring of three S buffers in TMEM.  S tiles are issued
+// alternately for the two query tiles (S number k: tile k % 2, key tile k / 2 of the
+// item, buffer k % 3), and S number k + 3 is issued right after P.V of S number k has
+// freed its buffer.  Each tile's next S is therefore ready while its softmax still runs,
+// so both softmax warpgroups stay busy and the tensor pipe does not wait on one tile's
+// S -> softmax -> P.V chain.  TMEM: 3 * BN (S/P) + 2 * D (O) columns, which fits only for
+// D = 64.  Causal items run both tiles over the same n KV tiles (tile 0's last one is
+// fully masked).
+//   warps 0-3 / 4-7 softmax of tile 0 / 1, warp 8 loader, warp 9 MMA
+template <int D>
+struct Fwd3Cfg {
+  static constexpr model::FwdPlan kPlan = model::fwd_plan_variant(D, 3);
+  static constexpr bool kFeasible = kPlan.feasible;
+  static constexpr int BM = 128;
+  static constexpr int NQT = 2;
+  static constexpr int BN = 128;
+  static constexpr int NSLOT = kFeasible ? kPlan.kv_slots : 4;
+  static constexpr int THREADS = 320;
+  static constexpr int BOX_COLS = 64;
+  static constexpr int NBOX = D / BOX_COLS;
+  static constexpr uint32_t Q_BOX_BYTES = BM * 128;
+  static constexpr uint32_t Q_TILE_BYTES = NBOX * Q_BOX_BYTES;
+  static constexpr uint32_t KV_BOX_BYTES = BN * 128;
+  static constexpr uint32_t SLOT_BYTES = NBOX * KV_BOX_BYTES;
+  static constexpr uint32_t Q_OFF = 0;
+  static constexpr uint32_t RING_OFF = NQT * Q_TILE_BYTES;
+  static constexpr uint32_t STG_OFF = RING_OFF + NSLOT * SLOT_BYTES;  // O staging per tile
+  static constexpr uint32_t BAR_OFF = STG_OFF + NQT * BM * D * 2;
+  // barriers: q_full, q_empty, full[NSLOT], empty[NSLOT], s[3], p[3][2], o[2][2], o_empty[2], drain
+  static constexpr int NBAR = 2 + 2 * NSLOT + 3 + 6 + 4 + 2 + 1;
+  static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
+  static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
+  static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;
+  static constexpr uint32_t TMEM_COLS = 512;
+  static constexpr uint32_t S_COL = 0;        // + buffer * BN
+  static constexpr uint32_t O_COL = 3 * BN;   // + t * D
+  static_assert(!kFeasible || (BYTES <= 227 * 1024 && O_COL + NQT * D <= TMEM_COLS), "budgets");
+};
+
+template <int D>
+__global__ void __launch_bounds__(Fwd3Cfg<D>::THREADS, 1)
+    attn_fwd3_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                     const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
+                     const FwdParams p) {
+  using C = Fwd3Cfg<D>;
+  if constexpr (!C::kFeasible) {
+    return;
+  } else {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_base = smem_u32(smem_raw);
+  const uint32_t sbase = (raw_base + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (sbase - raw_base);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const uint32_t bar_q = sbase + C::BAR_OFF;
+  const uint32_t bar_qe = bar_q + 8;
+  const uint32_t bar_full = bar_qe + 8;                // [NSLOT]
+  const uint32_t bar_empty = bar_full + 8 * C::NSLOT;  // [NSLOT]
+  const uint32_t bar_s = bar_empty + 8 * C::NSLOT;     // [3]    S in buffer b ready
+  const uint32_t bar_p = bar_s + 24;                   // [3][2] half h of P in buffer b written
+  const uint32_t bar_o = bar_p + 48;                   // [2][2] P.V of tile t, its S number parity e
+  const uint32_t bar_oe = bar_o + 32;                  // [2]    O_t read out by the epilogue
+  const uint32_t bar_drain = bar_oe + 16;
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::TMEM_PTR_OFF);
+  Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
+
+  if (threadIdx.x == 0) {
+    mbar_init(bar_q, 1);
+    mbar_init(bar_qe, 1);
+    for (int i = 0; i < C::NSLOT; ++i) {
+      mbar_init(bar_full + 8 * i, 1);
+      mbar_init(bar_empty + 8 * i, 1);
+    }
+    for (int b = 0; b < 3; ++b) {
+      mbar_init(bar_s + 8 * b, 1);
+      mbar_init(bar_p + 16 * b, C::BM);
+      mbar_init(bar_p + 16 * b + 8, C::BM);
+    }
+    for (int i = 0; i < 4; ++i) mbar_init(bar_o + 8 * i, 1);
+    mbar_init(bar_oe, C::BM);
+    mbar_init(bar_oe + 8, C::BM);
+    mbar_init(bar_drain, 1);
+    *ab.flag = 0;
+    *(ab.flag + 1) = 0;
+    fence_barrier_init();
+  }
+  if (warp == 9) tmem_alloc(smem_u32(tmem_ptr), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_ptr;
+
+  if (warp == 8) {
+    // ------------------------------------------------------------------ loader
+    if (lane == 0) {
+      prefetch_tensormap(&tm_q);
+      prefetch_tensormap(&tm_k);
+      prefetch_tensormap(&tm_v);
+      int pos = 0, issued = 0, skipped = -1, q_issued = 0;
+      bool ok = true;
+      for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+        const Item it = make_item<D>(p, idx);
+        const int n = it.n_tiles;
+        if (r > 0 && !(ok = mbar_wait(bar_qe, (r - 1) & 1, p.ctl, ab))) break;
+        mbar_expect_tx(bar_q, C::NQT * C::Q_TILE_BYTES);
+        for (int t = 0; t < C::NQT; ++t)
+          for (int x = 0; x < C::NBOX; ++x)
+            tma_load_3d(sbase + C::Q_OFF + t * C::Q_TILE_BYTES + x * C::Q_BOX_BYTES, &tm_q,
+                        x * C::BOX_COLS, it.q0 + t * C::BM, it.q_z, bar_q);
+        q_issued = r + 1;
+        for (int sq = 0; sq < 2 * n; ++sq, ++pos) {  // K_0, K_1, V_0, K_2, V_1, ..., V_{n-1}
+          if (sq == max(0, 2 * n - 6)) {  // three KV tiles before the end
+            const int nidx = item_index(p, r + 1);
+            if (nidx >= 0) {
+              const Item nx = make_item<D>(p, nidx);
+              prefetch_item_l2<D, C::NQT, C::BM>(&tm_q, &tm_k, &tm_v, nx.q0, nx.q_z, nx.kv_z);
+            }
+          }
+          const int slot = pos % C::NSLOT, round = pos / C::NSLOT;
+          if (!(ok = mbar_wait(bar_empty + 8 * slot, (round & 1) ^ 1, p.ctl, ab))) break;
+          issued = pos + 1;
+          if (p.ctl.inject == 2 && pos == 2) {  // test hook: never load this tile
+            skipped = pos;
+            continue;
+          }
+          const bool is_v = sq != 0 && (sq == 2 * n - 1 || (sq & 1) == 0);
+          const int tile = sq == 0 ? 0 : sq == 2 * n - 1 ? n - 1 : (sq & 1) ? (sq + 1) / 2 : sq / 2 - 1;
+          mbar_expect_tx(bar_full + 8 * slot, C::SLOT_BYTES);
+          for (int x = 0; x < C::NBOX; ++x)
+            tma_load_3d(sbase + C::RING_OFF + slot * C::SLOT_BYTES + x * C::KV_BOX_BYTES,
+                        is_v ? &tm_v : &tm_k, x * C::BOX_COLS, tile * C::BN, it.kv_z, bar_full + 8 * slot);
+        }
+      }
+      Abort no_abort{ab.flag + 1};
+      if (q_issued > 0) mbar_wait(bar_q, (q_issued - 1) & 1, p.ctl, no_abort);
+      for (int ps = max(0, issued - C::NSLOT); ps < issued; ++ps)
+        if (ps != skipped)
+          mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, no_abort);
+    }
+  } else if (warp == 9) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16(C::BM, C::BN, 0, 0);
+      constexpr uint32_t idesc_pv = idesc_bf16(C::BM, D, 0, 1);
+      const uint64_t dq0 = sdesc_sw128(sbase + C::Q_OFF, 16, 1024);
+      const uint64_t dk0 = sdesc_sw128(sbase + C::RING_OFF, 16, 1024);
+      const uint64_t dv0 = sdesc_sw128(sbase + C::RING_OFF, C::KV_BOX_BYTES, 1024);
+      constexpr uint32_t kSlot16 = C::SLOT_BYTES >> 4, kQTile16 = C::Q_TILE_BYTES >> 4;
+      constexpr uint32_t kQBox16 = C::Q_BOX_BYTES >> 4, kKBox16 = C::KV_BOX_BYTES >> 4;
+      auto wait_slot = [&](int ps) {
+        return mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, ab);
+      };
+      long long gk = 0;  // S tiles issued in earlier items (both query tiles)
+      int pos = 0, cnt = 0;  // ring position of the item's K_0; per-tile S count before the item
+      bool ok = true;
+      // S number k of the item (tile k % 2, key tile k / 2) into buffer (gk + k) % 3
+      auto issue_s = [&](int k, int n) -> bool {
+        const int t = k & 1, j = k >> 1;
+        const int kp = pos + ring_pos_k(j);
+        if (!wait_slot(kp)) return false;
+        tc_fence_after();
+        const int buf = static_cast<int>((gk + k) % 3);
+        const uint64_t a = dq0 + t * kQTile16;
+        const uint64_t b = dk0 + (kp % C::NSLOT) * kSlot16;
+#pragma unroll
+        for (int x = 0; x < C::NBOX; ++x)
+          mma_ss_k64(tmem + C::S_COL + buf * C::BN, a + x * kQBox16, b + x * kKBox16, idesc_s, x > 0);
+        tc_commit(bar_s + 8 * buf);
+        if (t == 1) tc_commit(bar_empty + 8 * (kp % C::NSLOT));  // both tiles have used K_j
+        if (k == 2 * n - 1) tc_commit(bar_qe);                   // the item's last S
+        return true;
+      };
+      for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+        const Item it = make_item<D>(p, idx);
+        const int n = it.n_tiles;
+        if (!(ok = mbar_wait(bar_q, r & 1, p.ctl, ab))) break;
+        for (int k = 0; ok && k < 3 && k < 2 * n; ++k) ok = issue_s(k, n);
+        for (int m = 0; ok && m < 2 * n; ++m) {
+          const int t = m & 1, j = m >> 1;
+          const long long km = gk + m;
+          const int buf = static_cast<int>(km % 3);
+          const uint32_t par = static_cast<uint32_t>((km / 3) & 1);
+          const int vp = pos + ring_pos_v(j, n);
+          if (!(ok = wait_slot(vp))) break;
+          if (!(ok = mbar_wait(bar_p + 16 * buf, par, p.ctl, ab))) break;
+          if (j == 0 && r > 0 && !(ok = mbar_wait(bar_oe + 8 * t, (r - 1) & 1, p.ctl, ab))) break;
+          tc_fence_after();
+          const uint64_t b = dv0 + (vp % C::NSLOT) * kSlot16;
+          mma_ts_k64(tmem + C::O_COL + t * D, tmem + C::S_COL + buf * C::BN, b, idesc_pv, j > 0 ? 1u : 0u);
+          if (!(ok = mbar_wait(bar_p + 16 * buf + 8, par, p.ctl, ab))) break;
+          tc_fence_after();
+          mma_ts_k64(tmem + C::O_COL + t * D, tmem + C::S_COL + buf * C::BN + C::BN / 4,
+                     b + (C::BN / 2) * (128 >> 4), idesc_pv, 1u);
+          const int g = cnt + j;  // this tile's S number across items
+          tc_commit(bar_o + 8 * (2 * t + (g & 1)));
+          if (t == 1) tc_commit(bar_empty + 8 * (vp % C::NSLOT));  // both tiles have used V_j
+          if (m + 3 < 2 * n) ok = issue_s(m + 3, n);                // into the buffer just freed
+        }
+        gk += 2 * n;
+        cnt += n;
+        pos += 2 * n;
+      }
+      Abort no_abort{ab.flag + 1};
+      tc_commit(bar_drain);
+      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+    }
+  } else {
+    // ------------------------------------------------------------------ softmax
+    const int t = warp >> 2;
+    const int row_in_tile = (warp & 3) * 32 + lane;
+    const uint32_t lane_addr = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t s_tm0 = tmem + lane_addr + C::S_COL;
+    const uint32_t o_tm = tmem + lane_addr + C::O_COL + t * D;
+    const uint32_t stg_q = sbase + C::STG_OFF + static_cast<uint32_t>(warp) * (32 * D * 2);
+    const float c = p.c;
+    const uint64_t c2 = f2(c, c);
+    const int off = p.Skv - p.Sq;
+    long long gk = 0;
+    int cnt = 0;
+    bool ok = true;
+    for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+      const Item it = make_item<D>(p, idx);
+      const int n = it.n_tiles;
+      const int row = it.q0 + t * C::BM + row_in_tile;
+      const int limit = p.causal ? min(p.Skv, row + off + 1) : p.Skv;
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int j = 0; ok && j < n; ++j) {
+        const long long k = gk + 2 * j + t;
+        const int buf = static_cast<int>(k % 3);
+        const int g = cnt + j;
+        ok = softmax_step<D, C::BN>(s_tm0 + buf * C::BN, o_tm, bar_s + 8 * buf,
+                                    static_cast<uint32_t>((k / 3) & 1), bar_p + 16 * buf,
+                                    bar_o + 8 * (2 * t + ((g - 1) & 1)), ((g - 1) >> 1) & 1, j == 0,
+                                    j * C::BN, limit, c, c2, m_run, l_run, p.ctl, ab);
+      }
+      if (!ok) break;
+      const int gl = cnt + n - 1;
+      if (!(ok = softmax_epilogue<D>(o_tm, bar_o + 8 * (2 * t + (gl & 1)), (gl >> 1) & 1, bar_oe + 8 * t,
+                                     m_run, l_run, row, it.q_z, p, ab, &tm_o, stg_q)))
+        break;
+      gk += 2 * n;
+      cnt += n;
+    }
+    if (lane == 0) bulk_wait_group0();  // the O stores have completed before the CTA exits
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
   }
 }
 
@@ -795,10 +1123,11 @@ bool make_map(CUtensorMap* map, const void* base, int D, int rows, int planes, i
 template <int D, class C, class Kernel>
 cudaError_t launch_design(Kernel kernel, int rows_per_item, const FwdArgs& a, const KernelCtl& ctl,
                           cudaStream_t stream, unsigned long long& configured) {
-  CUtensorMap mq, mk, mv;
+  CUtensorMap mq, mk, mv, mo;
   if (!make_map(&mq, a.q, D, a.Sq, a.B * a.Hq, C::BM) ||
       !make_map(&mk, a.k, D, a.Skv, a.B * a.Hkv, C::BN) ||
-      !make_map(&mv, a.v, D, a.Skv, a.B * a.Hkv, C::BN))
+      !make_map(&mv, a.v, D, a.Skv, a.B * a.Hkv, C::BN) ||
+      !make_map(&mo, a.o, D, a.Sq, a.B * a.Hq, 32))  // epilogue: one 32-row block per warp
     return cudaErrorInvalidValue;
   int dev = 0;
   cudaGetDevice(&dev);
@@ -821,22 +1150,29 @@ cudaError_t launch_design(Kernel kernel, int rows_per_item, const FwdArgs& a, co
   const long long items = static_cast<long long>(p.n_pairs) * a.B * a.Hq;
   if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   p.n_items = static_cast<int>(items);
+  p.plane_block = model::causal_plane_block(a.B * a.Hq, a.Hq / a.Hkv, a.Skv, D);
   // persistent: one CTA per SM (shared memory / TMEM admit one), each walking its items
   int sms = 0;
   cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
   const int grid = static_cast<int>(items < sms ? items : sms);
-  kernel<<<grid, C::THREADS, C::BYTES, stream>>>(mq, mk, mv, p);
+  kernel<<<grid, C::THREADS, C::BYTES, stream>>>(mq, mk, mv, mo, p);
   return cudaGetLastError();
 }
 
 template <int D>
 cudaError_t launch_fwd_d(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
   static unsigned long long configured2 = 0, configured1 = 0;  // one bit per device
-  constexpr int kModelTiles = model::fwd_plan(D).q_tiles;
-  const int q_tiles = a.design ? a.design : kModelTiles;
-  if (q_tiles == 1)
+  static unsigned long long configured3 = 0;
+  constexpr int kModelDesign = model::fwd_plan(D).design;
+  const int design = a.design ? a.design : kModelDesign;
+  if (design == 1)
     return launch_design<D, Fwd1Cfg<D>>(attn_fwd1_kernel<D>, Fwd1Cfg<D>::BM, a, ctl, stream, configured1);
+  if constexpr (Fwd3Cfg<D>::kFeasible) {
+    if (design == 3)
+      return launch_design<D, Fwd3Cfg<D>>(attn_fwd3_kernel<D>, Fwd3Cfg<D>::NQT * Fwd3Cfg<D>::BM, a, ctl,
+                                          stream, configured3);
+  }
   return launch_design<D, FwdCfg<D>>(attn_fwd_kernel<D>, FwdCfg<D>::NQT * FwdCfg<D>::BM, a, ctl, stream,
                                      configured2);
 }

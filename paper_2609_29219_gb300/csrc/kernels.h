@@ -35,7 +35,7 @@ struct FwdArgs {
   float* lse;     // [B, Hq, Sq] or null
   int B, Hq, Hkv, Sq, Skv, D, causal;
   float scale;
-  int design;  // query tiles per CTA: 0 = the analytic model's choice, 1 or 2 forced
+  int design;  // prefill design: 0 = the analytic model's choice, 1..3 forced
 };
 
 // Bytes of workspace the decode path needs for `splits` splits.

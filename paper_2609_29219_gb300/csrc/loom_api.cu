@@ -185,6 +185,8 @@ loom_status loom_model_fwd_plan(int D, loom_fwd_plan* out) {
   if (!out) return LOOM_ERR_INVALID_ARG;
   if (D != 64 && D != 128) return LOOM_ERR_UNSUPPORTED;
   const model::FwdPlan p = model::fwd_plan(D);
+  out->design = p.design;
+  out->s_buffers = p.s_buffers;
   out->bm = p.bm;
   out->bn = p.bn;
   out->q_tiles = p.q_tiles;
@@ -216,6 +218,8 @@ void loom_debug_set_timeout_ns(uint64_t ns) { g_timeout_ns = ns ? ns : kDefaultT
 
 void loom_debug_inject(int mode) { g_inject = mode; }
 
-void loom_debug_prefill_design(int q_tiles) { g_prefill_design = (q_tiles == 1 || q_tiles == 2) ? q_tiles : 0; }
+void loom_debug_prefill_design(int design) {
+  g_prefill_design = (design >= 1 && design <= 3) ? design : 0;
+}
 
 }  // extern "C"

@@ -13,6 +13,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <initializer_list>
 
 namespace loom {
 namespace model {
@@ -38,12 +39,17 @@ struct ArchDesc {
   double cta_start_ns;      // start-up of a decode split CTA: launch, first copies (measured)
   double mma_clk_per_n;     // clocks of one 128xNx16 bf16 MMA per unit of N (measured: 0.5)
   double mma_min_clk;       // floor on one MMA's clocks (measured: 48 at N = 64)
-  double softmax_clk_per_key;  // softmax of one 128-row tile, clocks per key (measured)
+  double softmax_clk_per_key;       // softmax of one 128-row tile alone, clocks per key (measured)
+  double softmax_pair_clk_per_key;  // two tiles' softmax running together, clocks per key (measured)
+  double l2_bytes;                  // L2 cache capacity (specification)
+  double mma_issue_busy_factor;     // MMA issue stream slowdown while two softmax warpgroups
+                                    // are busy on the SM (measured: 1338 vs 512 clk per GEMM)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
-    1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.0,
+    1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
+    129.0e6, 2.6,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -64,35 +70,37 @@ constexpr double dmax(double a, double b) { return a > b ? a : b; }
 constexpr long long cdiv(long long a, long long b) { return (a + b - 1) / b; }
 
 // ------------------------------------------------------------------ prefill
-// Candidates: design (q_tiles, s_buffers) x BN keys per tile x KV ring slots x knob
-// b = (b_lm, b_ms).  BM = 128 query rows per tile (one per TMEM lane).  Two designs
-// are implemented:
-//   q_tiles = 2, s_buffers = 1: two query tiles alternate on the tensor pipe; each
-//     tile's chain S -> softmax -> P.V -> next S is serial;
-//   q_tiles = 1, s_buffers = 2: one query tile with S double-buffered in TMEM, i.e.
-//     the boundary between the S MMA and the softmax body is opened (Eq. 6 knob) at the
-//     price of a second S buffer (TMEM capacity, Eq. 8).
+// Candidates: design x BN keys per tile x KV ring slots x knob b = (b_lm, b_ms).
+// BM = 128 query rows per tile (one per TMEM lane).  Three designs are implemented:
+//   design 2: two query tiles, one S buffer each; the tiles alternate on the tensor
+//     pipe, and each tile's chain S -> softmax -> P.V -> next S is serial;
+//   design 1: one query tile, S double-buffered: the boundary between the S MMA and
+//     the softmax body is opened (Eq. 6 knob) at the price of a second S buffer;
+//   design 3: two query tiles sharing a ring of three S buffers: both tiles' next S is
+//     computed while their softmax runs, so the two softmaxes overlap each other and the
+//     MMAs (TMEM: 3 BN + 2 D columns).
 struct FwdPlan {
-  int bm, bn, q_tiles, s_buffers, kv_slots, b_lm, b_ms;
+  int design, bm, bn, q_tiles, s_buffers, kv_slots, b_lm, b_ms;
   int smem_bytes, tmem_cols;
   double t_load_ns, t_mma_ns, t_softmax_ns, t_iter_ns;  // per KV tile, per query tile
   bool feasible;
 };
 
 // Primitive latencies of one KV-tile iteration (per query tile, ns).
-constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int q_tiles, int s_buffers, int bn, int slots,
-                           int b_lm, int b_ms) {
+constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int design, int bn, int slots, int b_lm,
+                           int b_ms) {
   FwdPlan p{};
+  p.design = design;
   p.bm = 128;
-  p.q_tiles = q_tiles;
-  p.s_buffers = s_buffers;
+  p.q_tiles = design == 1 ? 1 : 2;
+  p.s_buffers = design == 1 ? 2 : design == 2 ? 1 : 3;
   p.bn = bn;
   p.kv_slots = slots;
   p.b_lm = b_lm;
   p.b_ms = b_ms;
   const double clk = a.sm_ghz;  // clocks per ns
   // load stage: K_j and V_j tiles (mostly L2 hits), shared by the CTA's query tiles
-  p.t_load_ns = 2.0 * bn * D * 2 / a.l2_smem_gbs_sm / q_tiles;
+  p.t_load_ns = 2.0 * bn * D * 2 / a.l2_smem_gbs_sm / p.q_tiles;
   // compute leaf: S = Q K^T (N = BN) and O += P V (N = D), K/16 MMAs each
   auto mma_clk = [&](int n) { return dmax(a.mma_clk_per_n * n, a.mma_min_clk); };
   p.t_mma_ns = ((D / 16.0) * mma_clk(bn) + (bn / 16.0) * mma_clk(D)) / clk;
@@ -100,59 +108,82 @@ constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int q_tiles, int s_buffers,
   p.t_softmax_ns = a.softmax_clk_per_key * bn / clk;
   const double sync = a.sync_ns;
   double body = 0.0;
-  if (q_tiles == 2) {
-    // two tiles alternate: per pair of tile-iterations the tensor pipe needs 2 * mma,
-    // and each tile's chain (softmax, then its P.V and next S) must fit in the period;
-    // the two softmaxes share the SM's MUFU and issue slots, so they do not overlap
+  if (design == 2) {
+    // per pair of tile-iterations the tensor pipe needs 2 * mma; each tile's chain
+    // (softmax, then its P.V and next S) must fit in the period; the softmaxes alternate
     body = dmax(2 * p.t_mma_ns, dmax(p.t_softmax_ns + p.t_mma_ns, 2 * p.t_softmax_ns) + 2 * sync) / 2;
+  } else if (design == 1) {
+    body = dmax(p.t_mma_ns, p.t_softmax_ns) + sync;  // softmax and MMA overlap fully
   } else {
-    // S double-buffered: softmax and MMA overlap fully; one handshake per tile
-    body = dmax(p.t_mma_ns, p.t_softmax_ns) + sync;
+    // both softmaxes run together (sharing MUFU and issue slots) and overlap the MMAs;
+    // the single MMA-issuing thread then competes with two busy warpgroups for issue
+    // slots, which stretches its stream of MMAs
+    const double pair = a.softmax_pair_clk_per_key * bn / clk;
+    body = (dmax(2 * p.t_mma_ns * a.mma_issue_busy_factor, pair) + sync) / 2;
   }
   p.t_iter_ns = heg_pipe(p.t_load_ns, body, 0.0, b_lm, b_ms);
   // resources (Eq. 8 constraints)
-  p.smem_bytes = q_tiles * p.bm * D * 2 + slots * bn * D * 2 + 1024 + 256;
-  p.tmem_cols = q_tiles * (s_buffers * bn + D);
+  // Q tiles + K/V ring + an O staging tile per query tile (TMA-store epilogue) +
+  // barriers and alignment
+  p.smem_bytes = 2 * p.q_tiles * p.bm * D * 2 + slots * bn * D * 2 + 1024 + 256;
+  p.tmem_cols = design == 1 ? 2 * bn + D : design == 2 ? 2 * (bn + D) : 3 * bn + 2 * D;
   p.feasible = true;
-  if (!((q_tiles == 2 && s_buffers == 1) || (q_tiles == 1 && s_buffers == 2))) p.feasible = false;
+  if (design < 1 || design > 3) p.feasible = false;
   if (bn % 16 != 0 || bn < 16 || bn > 256) p.feasible = false;   // MMA N for M = 128
   if (bn != 128) p.feasible = false;  // softmax: one S row of 128 fp32 per thread, P in halves
   if (D % 64 != 0) p.feasible = false;                            // 128 B swizzle atoms
   if (p.smem_bytes > a.smem_per_cta) p.feasible = false;          // L1 footprint
   if (p.tmem_cols > a.tmem_cols) p.feasible = false;
-  // an open load boundary needs the loads of the next tiles in flight while the current
-  // ones are read: at least 4 slots, enough of them to cover the memory latency
-  if (slots < 4) p.feasible = false;
-  if (b_lm && (slots / 2 - 1) * body * q_tiles < a.mem_latency_ns * 0.5) p.feasible = false;
-  if (!b_lm) p.feasible = false;  // both kernels always prefetch through the ring
-  if (q_tiles == 2 && slots % 2 != 0) p.feasible = false;        // K/V alternate in the ring
+  // an open load boundary needs loads in flight while the MMAs read the current tiles:
+  // the MMA warp holds two slots (V_j and K_{j+1}); the other slots - 2 are the
+  // look-ahead, each consumed in half a KV-tile period, which must cover the latency of
+  // an L2-resident tile (half the HBM latency)
+  if (slots < 3) p.feasible = false;
+  if (b_lm && (slots - 2) * body * p.q_tiles / 2 < a.mem_latency_ns * 0.5) p.feasible = false;
+  if (!b_lm) p.feasible = false;  // every kernel prefetches through the ring
   return p;
 }
 
-// Eq. 8 for one design by enumeration over BN, slots and knobs; ties go to fewer slots.
-constexpr FwdPlan fwd_plan_variant(int D, int q_tiles, const ArchDesc& a = kGb300) {
+// Eq. 8 for one design by enumeration over BN, slots and knobs; ties go to the deeper
+// ring (more latency slack for the same modeled time).
+constexpr FwdPlan fwd_plan_variant(int D, int design, const ArchDesc& a = kGb300) {
   FwdPlan best{};
   best.feasible = false;
-  const int s_buffers = q_tiles == 2 ? 1 : 2;
   for (int bn = 32; bn <= 256; bn += 16)
     for (int slots = 2; slots <= 16; ++slots)
       for (int b_lm = 0; b_lm <= 1; ++b_lm)
         for (int b_ms = 0; b_ms <= 1; ++b_ms) {
-          FwdPlan p = fwd_eval(a, D, q_tiles, s_buffers, bn, slots, b_lm, b_ms);
+          FwdPlan p = fwd_eval(a, D, design, bn, slots, b_lm, b_ms);
           if (!p.feasible) continue;
           const double cost = p.t_iter_ns / bn;  // per key and query tile
           const double best_cost = best.feasible ? best.t_iter_ns / best.bn : 1e300;
-          if (cost < best_cost * (1.0 - 1e-9)) best = p;
+          if (cost < best_cost * (1.0 - 1e-9) ||
+              (cost <= best_cost * (1.0 + 1e-9) && slots > best.kv_slots))
+            best = p;
         }
   return best;
 }
 
-// Eq. 9: the design with the lowest modeled latency.
+// Eq. 9: the design with the lowest modeled latency (ties keep the earlier design).
 constexpr FwdPlan fwd_plan(int D, const ArchDesc& a = kGb300) {
-  const FwdPlan two = fwd_plan_variant(D, 2, a), one = fwd_plan_variant(D, 1, a);
-  if (!one.feasible) return two;
-  if (!two.feasible) return one;
-  return one.t_iter_ns / one.bn < two.t_iter_ns / two.bn * (1.0 - 1e-9) ? one : two;
+  FwdPlan best = fwd_plan_variant(D, 2, a);
+  for (int design : {1, 3}) {
+    const FwdPlan p = fwd_plan_variant(D, design, a);
+    if (!p.feasible) continue;
+    if (!best.feasible || p.t_iter_ns / p.bn < best.t_iter_ns / best.bn * (1.0 - 1e-9)) best = p;
+  }
+  return best;
+}
+
+// Causal work order: (b, h) planes per block such that the distinct K/V bytes the block
+// streams (a K/V plane is shared by `group` query heads) stay within 40% of L2, leaving
+// room for Q, O and the next block's first tiles.  Items are dealt block by block, so
+// the CTAs working at the same time re-read K/V from L2 rather than HBM.
+constexpr int causal_plane_block(int planes, int group, int Skv, int D, const ArchDesc& a = kGb300) {
+  const double per_plane = 2.0 * Skv * D * 2 / (group > 0 ? group : 1);
+  double blk = 0.4 * a.l2_bytes / per_plane;
+  if (blk < 1.0) blk = 1.0;
+  return blk >= planes ? planes : static_cast<int>(blk);
 }
 
 // Modeled time (us) of a whole prefill launch under a plan (Eq. 5-7 over the CTA's

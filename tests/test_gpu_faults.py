@@ -63,17 +63,17 @@ def test_decode_skipped_stage_times_out_and_context_survives(loom):
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "decode after timeout")
 
 
-@pytest.mark.parametrize("design", [2, 1])
-def test_prefill_skipped_tile_times_out_and_context_survives(loom, design):
+@pytest.mark.parametrize("design,D", [(2, 128), (1, 128), (1, 64), (3, 64)])
+def test_prefill_skipped_tile_times_out_and_context_survives(loom, design, D):
     loom.loom_debug_prefill_design(design)
     try:
-        _prefill_fault_case(loom)
+        _prefill_fault_case(loom, D)
     finally:
         loom.loom_debug_prefill_design(0)
 
 
-def _prefill_fault_case(loom):
-    B, H, S, D = 1, 2, 512, 128  # 4 work items, each with 4 KV tiles
+def _prefill_fault_case(loom, D):
+    B, H, S = 1, 2, 512  # 2 to 4 work items, each with 4 KV tiles
     q = synth.bf16_normal(32, synth.STREAM_Q, (B, H, S, D))
     k = synth.bf16_normal(32, synth.STREAM_K, (B, H, S, D))
     v = synth.bf16_normal(32, synth.STREAM_V, (B, H, S, D))

@@ -20,10 +20,11 @@ def loom():
     return m
 
 
-@pytest.fixture(autouse=True, params=[2, 1], ids=["two_tiles", "one_tile_double_s"])
+@pytest.fixture(autouse=True, params=[2, 1, 3], ids=["two_tiles", "one_tile_double_s", "s_ring"])
 def design(request, loom):
-    """Run every prefill test with both kernel designs (two alternating query tiles; one
-    query tile with S double-buffered in TMEM)."""
+    """Run every prefill test with each kernel design: two alternating query tiles; one
+    query tile with S double-buffered in TMEM; two query tiles sharing a ring of three S
+    buffers (D = 64 only: at D = 128 the call runs the two-tile design)."""
     loom.loom_debug_prefill_design(request.param)
     yield request.param
     loom.loom_debug_prefill_design(0)
