@@ -132,6 +132,11 @@ loom_status loom_attn_decode_noalloc(const void* q, const void* k_cache, const v
  *   (b_lm, b_ms) of Eq. 6, shared-memory bytes, TMEM columns, and the modeled latencies
  *   (ns) of one KV-tile iteration: load stage, MMA leaf, softmax leaf, and the pipe node.
  *   Returns LOOM_ERR_UNSUPPORTED for other D, LOOM_ERR_INVALID_ARG for a NULL out.
+ * loom_model_fwd_plan_variant: the best plan of one design (1, 2 or 3) for head dimension
+ *   D, the candidates Eq. 9 ranks; LOOM_ERR_UNSUPPORTED if that design has no feasible plan
+ *   at this D (the TMEM or shared-memory capacity of Eq. 8 rules it out).
+ * loom_model_heg_pipe: Eq. 6, the latency of a three-stage pipe node with load stage l,
+ *   body m and store stage s under the pipeline knob (b_lm, b_ms), each 0 or 1.
  * loom_model_fwd_time_us: modeled time of a whole prefill launch (us); < 0 on bad sizes.
  * loom_model_decode_time_us: modeled split + merge time (us) of Flash Decode with
  *   `splits` splits on `num_sms` SMs (every sequence Skv keys); < 0 on bad sizes.
@@ -142,6 +147,8 @@ typedef struct {
   double t_load_ns, t_mma_ns, t_softmax_ns, t_iter_ns;
 } loom_fwd_plan;
 loom_status loom_model_fwd_plan(int D, loom_fwd_plan* out);
+loom_status loom_model_fwd_plan_variant(int D, int design, loom_fwd_plan* out);
+double loom_model_heg_pipe(double l, double m, double s, int b_lm, int b_ms);
 double loom_model_fwd_time_us(int B, int Hq, int Sq, int Skv, int D, int causal);
 double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms);
 

@@ -25,6 +25,7 @@ __all__ = [
     "loom_attn_decode_num_splits", "loom_attn_check_error", "loom_status_string",
     "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
     "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
+    "loom_model_fwd_plan_variant", "loom_model_heg_pipe",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -90,6 +91,10 @@ def capi() -> ctypes.CDLL:
             lib.loom_debug_prefill_design.restype = None
             lib.loom_model_fwd_plan.argtypes = [i32, ctypes.POINTER(FwdPlan)]
             lib.loom_model_fwd_plan.restype = i32
+            lib.loom_model_fwd_plan_variant.argtypes = [i32, i32, ctypes.POINTER(FwdPlan)]
+            lib.loom_model_fwd_plan_variant.restype = i32
+            lib.loom_model_heg_pipe.argtypes = [ctypes.c_double] * 3 + [i32, i32]
+            lib.loom_model_heg_pipe.restype = ctypes.c_double
             lib.loom_model_fwd_time_us.argtypes = [i32, i32, i32, i32, i32, i32]
             lib.loom_model_fwd_time_us.restype = ctypes.c_double
             lib.loom_model_decode_time_us.argtypes = [i32, i32, i32, i32, i32, i32, i32]
@@ -246,6 +251,20 @@ def loom_model_fwd_plan(D: int) -> dict:
     plan = FwdPlan()
     _check(capi().loom_model_fwd_plan(int(D), ctypes.byref(plan)), "loom_model_fwd_plan")
     return plan.as_dict()
+
+
+def loom_model_fwd_plan_variant(D: int, design: int):
+    """Best plan of one prefill design (1, 2 or 3), or None if the design is infeasible at D."""
+    plan = FwdPlan()
+    st = capi().loom_model_fwd_plan_variant(int(D), int(design), ctypes.byref(plan))
+    if st == 2:  # LOOM_ERR_UNSUPPORTED
+        return None
+    _check(st, "loom_model_fwd_plan_variant")
+    return plan.as_dict()
+
+
+def loom_model_heg_pipe(l: float, m: float, s: float, b_lm: int, b_ms: int) -> float:
+    return float(capi().loom_model_heg_pipe(float(l), float(m), float(s), int(b_lm), int(b_ms)))
 
 
 def loom_model_fwd_time_us(B, Hq, Sq, Skv, D, causal) -> float:

@@ -181,10 +181,8 @@ loom_status loom_attn_check_error(void* stream) {
   return (word & kErrTimeout) ? LOOM_ERR_TIMEOUT : LOOM_OK;
 }
 
-loom_status loom_model_fwd_plan(int D, loom_fwd_plan* out) {
-  if (!out) return LOOM_ERR_INVALID_ARG;
-  if (D != 64 && D != 128) return LOOM_ERR_UNSUPPORTED;
-  const model::FwdPlan p = model::fwd_plan(D);
+namespace {
+void fill_plan(const model::FwdPlan& p, loom_fwd_plan* out) {
   out->design = p.design;
   out->s_buffers = p.s_buffers;
   out->bm = p.bm;
@@ -199,7 +197,27 @@ loom_status loom_model_fwd_plan(int D, loom_fwd_plan* out) {
   out->t_mma_ns = p.t_mma_ns;
   out->t_softmax_ns = p.t_softmax_ns;
   out->t_iter_ns = p.t_iter_ns;
+}
+}  // namespace
+
+loom_status loom_model_fwd_plan(int D, loom_fwd_plan* out) {
+  if (!out) return LOOM_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return LOOM_ERR_UNSUPPORTED;
+  fill_plan(model::fwd_plan(D), out);
   return LOOM_OK;
+}
+
+loom_status loom_model_fwd_plan_variant(int D, int design, loom_fwd_plan* out) {
+  if (!out) return LOOM_ERR_INVALID_ARG;
+  if ((D != 64 && D != 128) || design < 1 || design > 3) return LOOM_ERR_UNSUPPORTED;
+  const model::FwdPlan p = model::fwd_plan_variant(D, design);
+  if (!p.feasible) return LOOM_ERR_UNSUPPORTED;
+  fill_plan(p, out);
+  return LOOM_OK;
+}
+
+double loom_model_heg_pipe(double l, double m, double s, int b_lm, int b_ms) {
+  return model::heg_pipe(l, m, s, b_lm != 0, b_ms != 0);
 }
 
 double loom_model_fwd_time_us(int B, int Hq, int Sq, int Skv, int D, int causal) {

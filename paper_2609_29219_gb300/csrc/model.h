@@ -109,9 +109,10 @@ constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int design, int bn, int slo
   const double sync = a.sync_ns;
   double body = 0.0;
   if (design == 2) {
-    // per pair of tile-iterations the tensor pipe needs 2 * mma; each tile's chain
-    // (softmax, then its P.V and next S) must fit in the period; the softmaxes alternate
-    body = dmax(2 * p.t_mma_ns, dmax(p.t_softmax_ns + p.t_mma_ns, 2 * p.t_softmax_ns) + 2 * sync) / 2;
+    // per pair of tile-iterations the tensor pipe needs 2 * mma; each tile's chain (its
+    // softmax, then its P.V and next S on the tensor pipe, two barrier round trips) must
+    // fit in the period, while the other tile's softmax overlaps it
+    body = dmax(2 * p.t_mma_ns, p.t_softmax_ns + p.t_mma_ns + 2 * sync) / 2;
   } else if (design == 1) {
     body = dmax(p.t_mma_ns, p.t_softmax_ns) + sync;  // softmax and MMA overlap fully
   } else {

@@ -1,0 +1,123 @@
+"""The analytic schedule model (Sec. 2.6, Eq. 5-9; architecture description of Sec. 2.7),
+checked through the C ABI on the CPU against properties that hold whatever the numbers in
+the architecture description are: Eq. 6's limiting cases, the capacity constraints of
+Eq. 8, the argmin of Eq. 9 recomputed by brute force over every candidate, the one-wave
+rule of the split decode, and the rooflines no modeled time may beat."""
+import itertools
+import math
+
+import pytest
+
+PEAK_TFLOPS = 1910.3   # measured dense bf16 (cuBLAS) on GB300
+PEAK_GBS = 6783.5      # measured HBM copy bandwidth on GB300
+NUM_SMS = 152
+
+
+@pytest.fixture(scope="module")
+def loom():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2609_29219_gb300 as m
+    return m
+
+
+# ------------------------------------------------------------------ Eq. 6
+@pytest.mark.parametrize("l,m,s", [(1.0, 2.0, 3.0), (5.0, 1.0, 1.0), (0.5, 4.0, 0.25), (2.0, 2.0, 2.0)])
+def test_heg_pipe_limits(loom, l, m, s):
+    seq = loom.loom_model_heg_pipe(l, m, s, 0, 0)
+    full = loom.loom_model_heg_pipe(l, m, s, 1, 1)
+    assert seq == pytest.approx(l + m + s)        # no boundary open: the stages run in turn
+    assert full == pytest.approx(max(l, m, s))    # both open: the slowest stage sets the pace
+    for b in itertools.product((0, 1), repeat=2):
+        t = loom.loom_model_heg_pipe(l, m, s, *b)
+        assert full - 1e-12 <= t <= seq + 1e-12   # opening a boundary never slows the pipe
+    # opening one boundary hides exactly the stage on its other side behind its neighbour
+    assert loom.loom_model_heg_pipe(l, m, s, 1, 0) == pytest.approx(max(l, m + s))
+    assert loom.loom_model_heg_pipe(l, m, s, 0, 1) == pytest.approx(max(l + m, s))
+
+
+# ------------------------------------------------------------------ Eq. 8 / 9, prefill
+@pytest.mark.parametrize("D", [64, 128])
+def test_fwd_plan_within_capacities(loom, D):
+    p = loom.loom_model_fwd_plan(D)
+    assert p["smem_bytes"] <= 227 * 1024          # dynamic shared memory per CTA
+    assert p["tmem_cols"] <= 512                  # TMEM columns per SM
+    assert p["bm"] in (64, 128)
+    assert p["bn"] % 16 == 0 and 16 <= p["bn"] <= 256
+    assert p["kv_slots"] >= 2
+    assert p["design"] in (1, 2, 3)
+    assert p["t_iter_ns"] > 0
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_fwd_plan_is_argmin_over_designs(loom, D):
+    chosen = loom.loom_model_fwd_plan(D)
+    variants = {d: loom.loom_model_fwd_plan_variant(D, d) for d in (1, 2, 3)}
+    feasible = {d: v for d, v in variants.items() if v is not None}
+    assert chosen["design"] in feasible
+    best = min(v["t_iter_ns"] / v["bn"] for v in feasible.values())
+    assert chosen["t_iter_ns"] / chosen["bn"] == pytest.approx(best)
+    for v in feasible.values():                   # every candidate obeys Eq. 8
+        assert v["smem_bytes"] <= 227 * 1024 and v["tmem_cols"] <= 512
+
+
+def test_three_s_buffers_do_not_fit_at_d128(loom):
+    # 3 S buffers of 128 columns + 2 O tiles of 128 columns = 640 > 512 TMEM columns
+    assert loom.loom_model_fwd_plan_variant(128, 3) is None
+    assert loom.loom_model_fwd_plan_variant(64, 3) is not None
+
+
+@pytest.mark.parametrize("B,Hq,S,D,causal", [(4, 32, 2048, 128, 0), (4, 32, 2048, 128, 1),
+                                            (1, 32, 8192, 128, 1), (1, 64, 8192, 64, 1),
+                                            (1, 2, 128, 64, 0)])
+def test_fwd_time_not_below_tensor_roofline(loom, B, Hq, S, D, causal):
+    t = loom.loom_model_fwd_time_us(B, Hq, S, S, D, causal)
+    pairs = S * (S + 1) / 2 if causal else S * S
+    flops = 4.0 * B * Hq * D * pairs
+    assert t > 0
+    assert t * 1e-6 >= flops / (PEAK_TFLOPS * 1e12) * 0.999
+
+
+def test_fwd_time_scales_with_work(loom):
+    t1 = loom.loom_model_fwd_time_us(8, 32, 4096, 4096, 128, 0)
+    t2 = loom.loom_model_fwd_time_us(16, 32, 4096, 4096, 128, 0)
+    assert 1.8 <= t2 / t1 <= 2.2                  # many waves: time ~ work
+    tc = loom.loom_model_fwd_time_us(8, 32, 4096, 4096, 128, 1)
+    assert tc < t1                                # the causal triangle is cheaper
+
+
+# ------------------------------------------------------------------ decode
+DECODE_SHAPES = [(16, 32, 8, 8192, 128), (1, 32, 8, 131072, 128), (1, 8, 8, 4096, 64),
+                 (4, 16, 2, 30000, 128), (2, 4, 4, 64, 128)]
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,Skv,D", DECODE_SHAPES)
+def test_decode_split_is_brute_force_argmin(loom, B, Hq, Hkv, Skv, D):
+    chosen = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
+    cands = range(1, min(1024, math.ceil(Skv / 64)) + 1)
+    times = [loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS) for s in cands]
+    best = min(times)
+    assert times[chosen - 1] == pytest.approx(best)
+    assert chosen == 1 + times.index(best)        # ties: the fewest splits
+
+
+def test_long_decode_fills_one_wave(loom):
+    # split-KV across >= one wave of CTAs over all SMs (B * Hkv * splits >= #SM)
+    s = loom.loom_attn_decode_num_splits(1, 32, 8, 131072, 128)
+    assert 8 * s >= NUM_SMS
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,Skv,D", DECODE_SHAPES)
+def test_decode_time_not_below_hbm_roofline(loom, B, Hq, Hkv, Skv, D):
+    s = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
+    t = loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS)
+    kv_bytes = 2.0 * B * Hkv * Skv * D * 2
+    assert t * 1e-6 >= kv_bytes / (PEAK_GBS * 1e9) * 0.999
+
+
+def test_decode_more_splits_than_needed_cost_more(loom):
+    # beyond the argmin, extra splits only add merge work and CTA start-up
+    B, Hq, Hkv, Skv, D = 16, 32, 8, 8192, 128
+    s = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
+    t = lambda n: loom.loom_model_decode_time_us(n, B, Hq, Hkv, Skv, D, NUM_SMS)
+    assert t(min(128, 8 * s)) > t(s)
