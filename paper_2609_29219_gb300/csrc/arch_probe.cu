@@ -4,7 +4,8 @@
 //
 // Built as a standalone program (paper_2609_29219_gb300/arch_probe.py builds and runs it)
 // and printing one JSON object:
-//   pipes : ex2.approx / fma.rn.f32 / fma.rn.f32x2 instruction-lanes per clock per SM
+//   pipes : ex2.approx / fma.rn.f32 / fma.rn.f32x2 / cvt.rn.bf16x2.f32 instruction-lanes per
+//           clock per SM, and ex2 beside the bf16x2 packs of the softmax (one per pair)
 //   mma   : clocks per tcgen05.mma kind::f16 128xNx16 (SS with N = 64, 128, 256; TS N = 128)
 //   mix   : clocks per 128x128x128 GEMM of the prefill kernel's MMA stream (P.V as TS,
 //           S = Q.K^T as SS, two query tiles) alone and under added load: bulk copies,
@@ -36,6 +37,19 @@ __global__ void pipe_kernel(float* out, long long* cyc, int iters) {
       if (MODE == 0) v[i] = ex2f_(v[i]) - 1.5f;              // 1 MUFU + 1 FADD
       if (MODE == 1) v[i] = fmaf(v[i], 0.999f, 1e-7f);       // 1 FFMA
       if (MODE == 2) asm volatile("fma.rn.f32x2 %0, %0, %1, %1;" : "+l"(w[i]) : "l"(m2));  // 1 FFMA2
+      if (MODE == 3) {  // 1 bf16x2 pack, its result fed back as the next input
+        uint32_t r;
+        asm volatile("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(v[i]), "f"(v[i]));
+        v[i] = __uint_as_float(r);
+      }
+      if (MODE == 4) {  // the softmax mix: 1 MUFU + 1 FADD per element, a bf16x2 pack per pair
+        v[i] = ex2f_(v[i]) - 1.5f;
+        if (i & 1) {
+          uint32_t r;
+          asm volatile("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(v[i - 1]), "f"(v[i]));
+          w[i] ^= r;
+        }
+      }
     }
   }
   __syncthreads();
@@ -321,13 +335,17 @@ int main() {
   // pipes: 1024 threads x 4096 iterations x 8 ops per CTA
   {
     const double ops = 1024.0 * 4096 * 8;
-    const char* names[3] = {"ex2_per_clk_sm", "ffma_lanes_per_clk_sm", "ffma2_instr_lanes_per_clk_sm"};
-    for (int mode = 0; mode < 3; ++mode) {
+    // mode 4 counts its ex2 (8 per iteration, with 4 bf16x2 packs beside them)
+    const char* names[5] = {"ex2_per_clk_sm", "ffma_lanes_per_clk_sm", "ffma2_instr_lanes_per_clk_sm",
+                            "cvt_bf16x2_per_clk_sm", "ex2_beside_cvt_per_clk_sm"};
+    for (int mode = 0; mode < 5; ++mode) {
       auto launch = [&] {
         for (int rep = 0; rep < 2; ++rep) {
           if (mode == 0) pipe_kernel<0><<<sms, 1024>>>(out, d, 4096);
           if (mode == 1) pipe_kernel<1><<<sms, 1024>>>(out, d, 4096);
           if (mode == 2) pipe_kernel<2><<<sms, 1024>>>(out, d, 4096);
+          if (mode == 3) pipe_kernel<3><<<sms, 1024>>>(out, d, 4096);
+          if (mode == 4) pipe_kernel<4><<<sms, 1024>>>(out, d, 4096);
         }
       };
       const double cyc = avg_cycles(launch, d, h, sms);
