@@ -264,6 +264,34 @@ def to_host_tensor(torch, bits):
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16)
 
 
+# ------------------------------------------------------------------ ranks
+def make_collectives(torch, world, device):
+    """The two collectives of the timed loops: a barrier around them and the maximum of a
+    time over ranks (every rank runs one independent replica; rank 0 reports the job).
+    One rank: no-ops.  `device` is where the reduction tensor lives (a GPU for NCCL, the
+    CPU for gloo)."""
+    if world <= 1:
+        return (lambda: None), (lambda x: float(x))
+    import torch.distributed as dist
+
+    def barrier():
+        dist.barrier()
+
+    def reduce_max(x):
+        t = torch.tensor([float(x)], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    return barrier, reduce_max
+
+
+def job_value(per_rank_value, world):
+    """Whole-job throughput: every rank processes the same units per step (weak scaling),
+    timed by the slowest rank, so the job's value is N times one rank's value at the
+    maximum time."""
+    return per_rank_value * world
+
+
 # ------------------------------------------------------------------ timing
 WARMUP_SECONDS = 1.0  # clocks ramp up slowly after host-side idle periods
 
@@ -312,7 +340,7 @@ def measure(torch, wl, steps, warmup, stream, barrier, world, reduce_max, peaks,
     del t_wall0
     total_ms = reduce_max(total_ms)
     ms_per_step = total_ms / steps
-    value = wl.value(ms_per_step * 1e-3) * world
+    value = job_value(wl.value(ms_per_step * 1e-3), world)
     avg_launch_ms = statistics.mean(launch_ms) if launch_ms else ms_per_step
     if wl.unit == "TFLOP/s":
         achieved = wl.flops / (avg_launch_ms * 1e-3) / 1e12
@@ -344,7 +372,7 @@ def measure_e2e(torch, wl, steps, warmup, stream, barrier, reduce_max, world):
         b.record(stream)
     torch.cuda.synchronize()
     ms = reduce_max(a.elapsed_time(b)) / steps
-    return {"value": round(wl.value(ms * 1e-3) * world, 3), "unit": wl.unit,
+    return {"value": round(job_value(wl.value(ms * 1e-3), world), 3), "unit": wl.unit,
             "h2d_bytes_per_step": int(wl.h2d), "d2h_bytes_per_step": int(wl.d2h),
             "ms_per_step": round(ms, 4)}
 
@@ -401,20 +429,7 @@ def main():
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
-
-        def barrier():
-            dist.barrier()
-
-        def reduce_max(x):
-            t = torch.tensor([float(x)], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            return float(t.item())
-    else:
-        def barrier():
-            pass
-
-        def reduce_max(x):
-            return float(x)
+    barrier, reduce_max = make_collectives(torch, world, dev)
 
     peaks, peak_src = load_peaks()
     stream = torch.cuda.Stream(dev)
