@@ -52,6 +52,28 @@ def test_tiny_config(loom, causal):
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"tiny causal={causal}")
 
 
+def test_tiny_config_matches_golden_rows(loom):
+    # the stored oracle rows of tests/golden/tiny_attention_seed0.txt
+    import os
+    import sys
+    here = os.path.dirname(os.path.abspath(__file__))
+    sys.path.insert(0, os.path.join(here, "golden"))
+    import make_golden
+    from tests.test_golden import load
+    _, rows = load()
+    q, k, v = make_golden.inputs()
+    for causal in (False, True):
+        o, lse = _run(loom, q, k, v, causal)
+        o = o_to_f64(o)
+        lse = lse.cpu().numpy()
+        for c, h, r, vals in rows:
+            if c != int(causal):
+                continue
+            assert abs(lse[0, h, r] - vals[0]) <= 1e-3, (causal, h, r)
+            got = [o[0, h, r, col] for col in make_golden.COLS]
+            assert np.max(np.abs(np.asarray(got) - np.asarray(vals[1:]))) <= 2e-2, (causal, h, r)
+
+
 @pytest.mark.parametrize("D", [64, 128])
 @pytest.mark.parametrize("causal", [False, True])
 @pytest.mark.parametrize("S", [1, 127, 129, 255, 257, 384, 515])
