@@ -82,6 +82,7 @@ struct FwdParams {
   int n_pairs;   // query-tile pairs per (b, h)
   int n_items;   // n_pairs * B * Hq work items
   int plane_block;  // causal: (b, h) planes per block of the work order
+  int last_h0;      // causal: first plane of the final block (which may be larger)
   int causal;
   float c;       // scale * log2(e)
   KernelCtl ctl;
@@ -104,15 +105,24 @@ __device__ __forceinline__ int item_index(const FwdParams& p, int r) {
 
 // Item idx -> (position pos of its query tile or tile pair within the plane, plane bh).
 // Non-causal: consecutive items are consecutive positions of one plane (they share its
-// K/V in L2).  Causal: blocks of p.plane_block planes; within a block the bottom (longest)
-// positions of every plane go first.
+// K/V in L2).  Causal: blocks of p.plane_block planes, the final block running from plane
+// p.last_h0 to the end; within a block the bottom (longest) positions of every plane go
+// first.
 __device__ __forceinline__ void item_coords(const FwdParams& p, int idx, int& pos, int& bh) {
   if (p.causal) {
     const int BH = p.n_items / p.n_pairs;
-    const int per_block = p.plane_block * p.n_pairs;
-    const int blk = idx / per_block, in = idx - blk * per_block;
-    const int h0 = blk * p.plane_block;
-    const int nb = min(p.plane_block, BH - h0);
+    int h0, nb, in;
+    if (idx >= p.last_h0 * p.n_pairs) {  // the final block: planes [last_h0, BH)
+      h0 = p.last_h0;
+      nb = BH - h0;
+      in = idx - h0 * p.n_pairs;
+    } else {
+      const int per_block = p.plane_block * p.n_pairs;
+      const int blk = idx / per_block;
+      h0 = blk * p.plane_block;
+      nb = p.plane_block;
+      in = idx - blk * per_block;
+    }
     pos = p.n_pairs - 1 - in / nb;
     bh = h0 + in % nb;
   } else {
@@ -1150,12 +1160,13 @@ cudaError_t launch_design(Kernel kernel, int rows_per_item, const FwdArgs& a, co
   const long long items = static_cast<long long>(p.n_pairs) * a.B * a.Hq;
   if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   p.n_items = static_cast<int>(items);
-  p.plane_block = model::causal_plane_block(a.B * a.Hq, a.Hq / a.Hkv, a.Skv, D);
+  // (the block layout is set below, once the grid is known)
   // persistent: one CTA per SM (shared memory / TMEM admit one), each walking its items
   int sms = 0;
   cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
   const int grid = static_cast<int>(items < sms ? items : sms);
+  p.plane_block = model::causal_block_layout(a.B * a.Hq, a.Hq / a.Hkv, a.Skv, D, p.n_pairs, grid, &p.last_h0);
   kernel<<<grid, C::THREADS, C::BYTES, stream>>>(mq, mk, mv, mo, p);
   return cudaGetLastError();
 }

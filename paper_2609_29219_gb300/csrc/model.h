@@ -187,6 +187,36 @@ constexpr int causal_plane_block(int planes, int group, int Skv, int D, const Ar
   return blk >= planes ? planes : static_cast<int>(blk);
 }
 
+// Block layout of the causal order for `grid` persistent CTAs dealing `items_per_plane`
+// items of every plane heaviest first, in a snake order (CTA c takes the c-th item of even
+// rounds and the (grid-1-c)-th of odd ones): a block whose items fill whole pairs of
+// rounds gives every CTA one item from the heavy end and one from the light end of each
+// pair, so blocks are sized to whole round pairs where the plane count allows, and the
+// remainder joins the last block (its items are then dealt heaviest first together with a
+// whole round pair, instead of forming a final round of heavy items on a few CTAs).
+// Returns the regular block size; *last_h0 is the first plane of the final block.
+constexpr int causal_block_layout(int planes, int group, int Skv, int D, int items_per_plane, int grid,
+                                  int* last_h0, const ArchDesc& a = kGb300) {
+  const int budget = causal_plane_block(planes, group, Skv, D, a);
+  *last_h0 = 0;
+  if (budget >= planes) return planes;  // everything fits: one heaviest-first order
+  const long long pair_items = 2LL * grid;
+  if (items_per_plane <= 0 || pair_items % items_per_plane != 0) {
+    *last_h0 = (planes - 1) / budget * budget;  // blocks of the budget, the last one partial
+    return budget;
+  }
+  const int unit = static_cast<int>(pair_items / items_per_plane);  // planes per round pair
+  if (unit > budget) {
+    *last_h0 = (planes - 1) / budget * budget;
+    return budget;
+  }
+  const int blk = budget / unit * unit;
+  const int full = planes / blk;              // whole blocks
+  *last_h0 = full >= 1 ? (full - 1) * blk : 0;  // the last whole block absorbs the remainder
+  if (planes % blk == 0) *last_h0 = (full - 1) * blk;
+  return blk;
+}
+
 // Modeled time (us) of a whole prefill launch under a plan (Eq. 5-7 over the CTA's
 // items: Q load ; for(KV tiles, pipe) ; O store, in waves over the SMs).
 constexpr double fwd_time_us(const FwdPlan& p, int B, int Hq, int Sq, int Skv, int D, int causal,

@@ -123,6 +123,21 @@ def test_increasing_scores_force_rescales(loom):
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "ramp")
 
 
+@pytest.mark.parametrize("B,H,S", [(4, 32, 2048), (1, 16, 8192), (1, 3, 1000), (2, 64, 512)])
+def test_causal_work_order_covers_every_row(loom, B, H, S):
+    # the causal work order (blocks of planes aligned to round pairs, a merged final
+    # block) must hand out every (plane, query tile) exactly once: O and LSE start as NaN
+    # and no NaN may survive
+    import torch
+    D = 128
+    q = torch.randn(B, H, S, D, device="cuda").to(torch.bfloat16)
+    o = torch.full_like(q, float("nan"))
+    lse = torch.full((B, H, S), float("nan"), device="cuda")
+    loom.loom_attn_fwd(q, q, q, o, lse, causal=True)
+    loom.loom_attn_check_error()
+    assert torch.isfinite(o.float()).all() and torch.isfinite(lse).all()
+
+
 @pytest.mark.slow
 @pytest.mark.parametrize("causal", [False, True])
 def test_prefill_config_full_size_sampled(loom, causal):
