@@ -127,8 +127,8 @@ class ClockSampler:
 # headline prefill kernel from the ncu capture summarised in
 # profiles/attn_fwd_d128_b4_h32_s2048_noncausal.md, and the SHA-256 of the kernel sources
 # it was taken from: the number is reported only while the sources are unchanged.
-PROFILED_TRAFFIC_BYTES = 243.9e6
-PROFILED_SOURCES_SHA256 = "59ded0ff5654f71c63cbfdbf6de1c59831dd3473352cb581d6e846cb06c37717"
+PROFILED_TRAFFIC_BYTES = 243.7e6
+PROFILED_SOURCES_SHA256 = "fcbdb092d053fa598d60aa8553bc9b2f884e3fe61f24f622bc8e60e4836896d4"
 
 
 def profiled_traffic():
@@ -410,6 +410,9 @@ def main():
     ap.add_argument("--oracle-seconds", type=float, default=12.0)
     ap.add_argument("--sweep", choices=["decode"], default=None,
                     help="model-vs-measured sweep of the decode split count (one JSON line per point)")
+    ap.add_argument("--ncu-case", default=None,
+                    help="profiling run: set up this workload (prefill, prefill_causal, long_prefill_d128, "
+                         "long_prefill_d64, batched_decode, long_decode), run --steps launches, print nothing")
     args = ap.parse_args()
     world, rank, local = dist_env()
     if args.warmup < 3:
@@ -433,6 +436,8 @@ def main():
 
     peaks, peak_src = load_peaks()
     stream = torch.cuda.Stream(dev)
+    if args.ncu_case:
+        return run_ncu_case(torch, loom, dev, stream, args)
     if args.sweep == "decode":
         return run_decode_sweep(torch, loom, dev, stream, args, peaks)
 
@@ -541,6 +546,27 @@ def run_decode_sweep(torch, loom, dev, stream, args, peaks):
                               "frac": r["roofline"]["frac"]}), flush=True)
         wl.inp = None
         torch.cuda.empty_cache()
+
+
+def all_workloads():
+    lens = synth.decode_lengths(0, 16, 4096, 8192)
+    return [Prefill("prefill", 4, 32, 32, 2048, 128, causal=False),
+            Prefill("prefill_causal", 4, 32, 32, 2048, 128, causal=True),
+            Prefill("long_prefill_d128", 1, 32, 8, 8192, 128, causal=True),
+            Prefill("long_prefill_d64", 1, 64, 16, 8192, 64, causal=True),
+            Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
+            Decode("long_decode", 1, 32, 8, 131072, 128, splits=0)]
+
+
+def run_ncu_case(torch, loom, dev, stream, args):
+    """A few launches of one workload and nothing else, for small ncu captures."""
+    wl = {w.name: w for w in all_workloads()}[args.ncu_case]
+    wl.setup(torch, dev, loom)
+    with torch.cuda.stream(stream):
+        for i in range(max(1, args.steps)):
+            wl.step(i, stream)
+    torch.cuda.synchronize()
+    loom.loom_attn_check_error(stream)
 
 
 def run_reference(args, wl, world, rank):
