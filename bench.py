@@ -191,23 +191,55 @@ class Prefill:
 
     # end to end through the public API with host buffers
     def e2e_setup(self, torch, dev):
+        """End-to-end steps through the public API: each step copies its inputs from
+        pinned host memory, runs the kernel and copies O and LSE back.  Steps are
+        pipelined over two device buffer sets, with host-to-device and device-to-host
+        copies on their own streams, so that step i's kernel overlaps step i+1's input
+        copies and step i-1's result copies."""
         q, k, v = self.host_inputs(0)
         pin = lambda a: to_host_tensor(torch, a).pin_memory()
         self.h_in = [pin(q), pin(k), pin(v)]
-        self.h_o = torch.empty(q.shape, dtype=torch.bfloat16).pin_memory()
-        self.h_lse = torch.empty((self.B, self.Hq, self.S), dtype=torch.float32).pin_memory()
-        self.d_in = [torch.empty(t.shape, dtype=t.dtype, device=dev) for t in self.h_in]
-        self.d_o = torch.empty(q.shape, dtype=torch.bfloat16, device=dev)
-        self.d_lse = torch.empty(self.h_lse.shape, dtype=torch.float32, device=dev)
+        self.h_o = [torch.empty(q.shape, dtype=torch.bfloat16).pin_memory() for _ in range(2)]
+        self.h_lse = [torch.empty((self.B, self.Hq, self.S), dtype=torch.float32).pin_memory() for _ in range(2)]
+        self.d_in2 = [[torch.empty(t.shape, dtype=t.dtype, device=dev) for t in self.h_in] for _ in range(2)]
+        self.d_o2 = [torch.empty(q.shape, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+        self.d_lse2 = [torch.empty(self.h_lse[0].shape, dtype=torch.float32, device=dev) for _ in range(2)]
+        self.s_h2d = torch.cuda.Stream(dev)
+        self.s_d2h = torch.cuda.Stream(dev)
+        self.ev_in = [torch.cuda.Event() for _ in range(2)]    # inputs of buffer set b landed
+        self.ev_done = [torch.cuda.Event() for _ in range(2)]  # kernel on set b finished
+        self.ev_out = [torch.cuda.Event() for _ in range(2)]   # results of set b copied back
+        self.e2e_i = 0
         self.h2d = sum(t.numel() * t.element_size() for t in self.h_in)
-        self.d2h = self.h_o.numel() * 2 + self.h_lse.numel() * 4
+        self.d2h = self.h_o[0].numel() * 2 + self.h_lse[0].numel() * 4
+        # the single-step form below (tests, e2e of one call) uses buffer set 0
+        self.d_in, self.d_o, self.d_lse = self.d_in2[0], self.d_o2[0], self.d_lse2[0]
 
     def e2e_step(self, stream):
-        for d, h in zip(self.d_in, self.h_in):
-            d.copy_(h, non_blocking=True)
-        self.loom.loom_attn_fwd(*self.d_in, self.d_o, self.d_lse, causal=self.causal, stream=stream)
-        self.h_o.copy_(self.d_o, non_blocking=True)
-        self.h_lse.copy_(self.d_lse, non_blocking=True)
+        torch = self.torch
+        i, b = self.e2e_i, self.e2e_i % 2
+        self.e2e_i += 1
+        if i >= 2:  # set b's previous kernel and result copies must be done with it
+            self.s_h2d.wait_event(self.ev_done[b])
+        with torch.cuda.stream(self.s_h2d):
+            for d, h in zip(self.d_in2[b], self.h_in):
+                d.copy_(h, non_blocking=True)
+            self.ev_in[b].record(self.s_h2d)
+        stream.wait_event(self.ev_in[b])
+        if i >= 2:
+            stream.wait_event(self.ev_out[b])
+        self.loom.loom_attn_fwd(*self.d_in2[b], self.d_o2[b], self.d_lse2[b], causal=self.causal, stream=stream)
+        self.ev_done[b].record(stream)
+        self.s_d2h.wait_event(self.ev_done[b])
+        with torch.cuda.stream(self.s_d2h):
+            self.h_o[b].copy_(self.d_o2[b], non_blocking=True)
+            self.h_lse[b].copy_(self.d_lse2[b], non_blocking=True)
+            self.ev_out[b].record(self.s_d2h)
+
+    def e2e_join(self, stream):
+        """Make `stream` wait for every copy issued so far."""
+        for b in range(2):
+            stream.wait_event(self.ev_out[b])
 
 
 class Decode:
@@ -358,6 +390,7 @@ def measure(torch, wl, steps, warmup, stream, barrier, world, reduce_max, peaks,
 
 
 def measure_e2e(torch, wl, steps, warmup, stream, barrier, reduce_max, world):
+    wl.torch = torch
     wl.e2e_setup(torch, stream.device)
     with torch.cuda.stream(stream):
         for _ in range(warmup):
@@ -367,8 +400,10 @@ def measure_e2e(torch, wl, steps, warmup, stream, barrier, reduce_max, world):
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         a.record(stream)
+        wl.s_h2d.wait_event(a)  # no copy of the timed steps starts before the start event
         for _ in range(steps):
             wl.e2e_step(stream)
+        wl.e2e_join(stream)     # ... and the end event follows the last result copy
         b.record(stream)
     torch.cuda.synchronize()
     ms = reduce_max(a.elapsed_time(b)) / steps
