@@ -446,8 +446,9 @@ def main():
     ap.add_argument("--sweep", choices=["decode"], default=None,
                     help="model-vs-measured sweep of the decode split count (one JSON line per point)")
     ap.add_argument("--ncu-case", default=None,
-                    help="profiling run: set up this workload (prefill, prefill_causal, long_prefill_d128, "
-                         "long_prefill_d64, batched_decode, long_decode), run --steps launches, print nothing")
+                    help="profiling run: set up this workload (tiny, tiny_causal, prefill, prefill_causal, "
+                         "long_prefill_d128, long_prefill_d64, batched_decode, long_decode), run --steps "
+                         "launches, print nothing")
     args = ap.parse_args()
     world, rank, local = dist_env()
     if args.warmup < 3:
@@ -506,9 +507,15 @@ def main():
                         clocks)
             loom.loom_attn_check_error(stream)
             r["workload"] = wl.describe()
+            if isinstance(wl, Prefill) and wl.causal:
+                # the FlashAttention convention counts half the non-causal FLOPs
+                fa = 0.5 * prefill_flops(wl.B, wl.Hq, wl.S, wl.S, wl.D, False)
+                r["value_fa_convention"] = round(r["value"] * fa / wl.flops, 3)
             if isinstance(wl, Decode):
                 r["splits"] = wl.used_splits
                 r["kv_bytes_per_step"] = int(wl.bytes)
+                # overhead beside the algorithmic bytes: the partials written and read back
+                r["workspace_bytes_per_step"] = int(2 * wl.B * wl.Hq * wl.used_splits * (wl.D + 1) * 4)
             r["gpu_launches"] = wl.launches_per_step() * max(10, args.steps // 2)
             workloads[wl.name] = r
             wl.inp = None
@@ -585,7 +592,9 @@ def run_decode_sweep(torch, loom, dev, stream, args, peaks):
 
 def all_workloads():
     lens = synth.decode_lengths(0, 16, 4096, 8192)
-    return [Prefill("prefill", 4, 32, 32, 2048, 128, causal=False),
+    return [Prefill("tiny", 1, 2, 2, 128, 64, causal=False),
+            Prefill("tiny_causal", 1, 2, 2, 128, 64, causal=True),
+            Prefill("prefill", 4, 32, 32, 2048, 128, causal=False),
             Prefill("prefill_causal", 4, 32, 32, 2048, 128, causal=True),
             Prefill("long_prefill_d128", 1, 32, 8, 8192, 128, causal=True),
             Prefill("long_prefill_d64", 1, 64, 16, 8192, 64, causal=True),
