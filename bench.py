@@ -443,8 +443,10 @@ def main():
     ap.add_argument("--only", default=None,
                     help="comma-separated subset (and order) of the extra workloads to run")
     ap.add_argument("--oracle-seconds", type=float, default=12.0)
-    ap.add_argument("--sweep", choices=["decode"], default=None,
-                    help="model-vs-measured sweep of the decode split count (one JSON line per point)")
+    ap.add_argument("--sweep", choices=["decode", "model"], default=None,
+                    help="decode: model-vs-measured sweep of the decode split count; model: the analytic "
+                         "model's ranking and accuracy over prefill designs and shapes and decode split "
+                         "counts and shapes (one JSON line per point)")
     ap.add_argument("--ncu-case", default=None,
                     help="profiling run: set up this workload (tiny, tiny_causal, prefill, prefill_causal, "
                          "long_prefill_d128, long_prefill_d64, batched_decode, long_decode), run --steps "
@@ -476,6 +478,8 @@ def main():
         return run_ncu_case(torch, loom, dev, stream, args)
     if args.sweep == "decode":
         return run_decode_sweep(torch, loom, dev, stream, args, peaks)
+    if args.sweep == "model":
+        return run_model_sweep(torch, loom, dev, stream, args, peaks)
 
     # headline: prefill non-causal, with clocks sampled during the timed loop
     headline.setup(torch, dev, loom)
@@ -586,6 +590,57 @@ def run_decode_sweep(torch, loom, dev, stream, args, peaks):
                               "model_choice": sp == chosen, "measured_us": round(r["ms_per_step"] * 1e3, 2),
                               "model_us": round(model_us, 2), "GB/s": r["value"],
                               "frac": r["roofline"]["frac"]}), flush=True)
+        wl.inp = None
+        torch.cuda.empty_cache()
+
+
+def run_model_sweep(torch, loom, dev, stream, args, peaks):
+    """The analytic model against measurement (the paper's ablations, restated for this
+    path): for prefill shapes, every feasible design's modeled and measured time (does the
+    model's top-1 design measure best?); for decode shapes with uniform lengths, the
+    model's five best split counts, measured (ranking), with the modeled and measured
+    throughput of the chosen point (accuracy)."""
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    steps = max(10, args.steps // 4)
+    prefill = [(1, 32, 32, 1024, 128, False), (4, 32, 32, 2048, 128, False), (4, 32, 32, 2048, 128, True),
+               (2, 32, 32, 4096, 128, False), (1, 32, 8, 8192, 128, True), (1, 16, 16, 16384, 128, False),
+               (16, 16, 16, 512, 128, False), (4, 32, 32, 2048, 64, False), (1, 64, 16, 8192, 64, True),
+               (2, 32, 32, 4096, 64, False)]
+    for B, H, Hkv, S, D, causal in prefill:
+        wl = Prefill("sweep", B, H, Hkv, S, D, causal=causal)
+        wl.setup(torch, dev, loom)
+        chosen = loom.loom_model_fwd_plan(D)["design"]
+        for design in (1, 2, 3):
+            model_us = loom.loom_model_fwd_time_us_design(design, B, H, S, S, D, causal)
+            if model_us < 0:
+                continue
+            loom.loom_debug_prefill_design(design)
+            r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks)
+            loom.loom_attn_check_error(stream)
+            print(json.dumps({"sweep": "model", "kind": "prefill", "workload": wl.describe(), "design": design,
+                              "model_choice": design == chosen, "measured_us": round(r["ms_per_step"] * 1e3, 2),
+                              "model_us": round(model_us, 2), "measured_tflops": r["value"],
+                              "model_tflops": round(wl.flops / (model_us * 1e-6) / 1e12, 1)}), flush=True)
+        loom.loom_debug_prefill_design(0)
+        wl.inp = None
+        torch.cuda.empty_cache()
+    decode = [(1, 32, 8, 131072, 128), (1, 32, 8, 32768, 128), (4, 32, 8, 16384, 128), (16, 32, 8, 8192, 128),
+              (64, 32, 8, 2048, 128), (1, 64, 16, 65536, 64)]
+    for B, Hq, Hkv, Skv, D in decode:
+        wl = Decode("sweep", B, Hq, Hkv, Skv, D, splits=0)
+        wl.setup(torch, dev, loom)
+        n = min(1024, (Skv + 63) // 64)
+        modeled = sorted((loom.loom_model_decode_time_us(sp, B, Hq, Hkv, Skv, D, sms), sp) for sp in range(1, n + 1))
+        for rank, (model_us, sp) in enumerate(modeled[:5]):
+            wl.splits = sp
+            nbytes = loom.loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, sp)
+            wl.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+            r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks)
+            loom.loom_attn_check_error(stream)
+            print(json.dumps({"sweep": "model", "kind": "decode", "workload": wl.describe(), "splits": sp,
+                              "model_rank": rank + 1, "measured_us": round(r["ms_per_step"] * 1e3, 2),
+                              "model_us": round(model_us, 2), "measured_gbs": r["value"],
+                              "model_gbs": round(wl.bytes / (model_us * 1e-6) / 1e9, 1)}), flush=True)
         wl.inp = None
         torch.cuda.empty_cache()
 

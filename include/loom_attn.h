@@ -150,6 +150,8 @@ loom_status loom_model_fwd_plan(int D, loom_fwd_plan* out);
 loom_status loom_model_fwd_plan_variant(int D, int design, loom_fwd_plan* out);
 double loom_model_heg_pipe(double l, double m, double s, int b_lm, int b_ms);
 double loom_model_fwd_time_us(int B, int Hq, int Sq, int Skv, int D, int causal);
+/* Modeled prefill launch time (us) with design 1, 2 or 3 forced; < 0 if infeasible. */
+double loom_model_fwd_time_us_design(int design, int B, int Hq, int Sq, int Skv, int D, int causal);
 double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms);
 
 /*

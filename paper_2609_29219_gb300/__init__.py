@@ -25,7 +25,7 @@ __all__ = [
     "loom_attn_decode_num_splits", "loom_attn_check_error", "loom_status_string",
     "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
     "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
-    "loom_model_fwd_plan_variant", "loom_model_heg_pipe",
+    "loom_model_fwd_plan_variant", "loom_model_heg_pipe", "loom_model_fwd_time_us_design",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -97,6 +97,8 @@ def capi() -> ctypes.CDLL:
             lib.loom_model_heg_pipe.restype = ctypes.c_double
             lib.loom_model_fwd_time_us.argtypes = [i32, i32, i32, i32, i32, i32]
             lib.loom_model_fwd_time_us.restype = ctypes.c_double
+            lib.loom_model_fwd_time_us_design.argtypes = [i32] * 7
+            lib.loom_model_fwd_time_us_design.restype = ctypes.c_double
             lib.loom_model_decode_time_us.argtypes = [i32, i32, i32, i32, i32, i32, i32]
             lib.loom_model_decode_time_us.restype = ctypes.c_double
             _lib = lib
@@ -265,6 +267,11 @@ def loom_model_fwd_plan_variant(D: int, design: int):
 
 def loom_model_heg_pipe(l: float, m: float, s: float, b_lm: int, b_ms: int) -> float:
     return float(capi().loom_model_heg_pipe(float(l), float(m), float(s), int(b_lm), int(b_ms)))
+
+
+def loom_model_fwd_time_us_design(design, B, Hq, Sq, Skv, D, causal) -> float:
+    """Modeled prefill time (us) with one design forced; negative if the design is infeasible."""
+    return float(capi().loom_model_fwd_time_us_design(design, B, Hq, Sq, Skv, D, int(bool(causal))))
 
 
 def loom_model_fwd_time_us(B, Hq, Sq, Skv, D, causal) -> float:

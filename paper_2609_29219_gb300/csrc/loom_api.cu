@@ -225,6 +225,13 @@ double loom_model_fwd_time_us(int B, int Hq, int Sq, int Skv, int D, int causal)
   return model::fwd_time_us(model::fwd_plan(D), B, Hq, Sq, Skv, D, causal != 0);
 }
 
+double loom_model_fwd_time_us_design(int design, int B, int Hq, int Sq, int Skv, int D, int causal) {
+  if (B <= 0 || Hq <= 0 || Sq <= 0 || Skv <= 0 || (D != 64 && D != 128) || design < 1 || design > 3) return -1.0;
+  const model::FwdPlan p = model::fwd_plan_variant(D, design);
+  if (!p.feasible) return -1.0;
+  return model::fwd_time_us(p, B, Hq, Sq, Skv, D, causal != 0);
+}
+
 double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms) {
   if (splits <= 0 || B <= 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv || Skv <= 0 || num_sms <= 0 ||
       (D != 64 && D != 128))

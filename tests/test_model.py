@@ -121,3 +121,17 @@ def test_decode_more_splits_than_needed_cost_more(loom):
     s = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
     t = lambda n: loom.loom_model_decode_time_us(n, B, Hq, Hkv, Skv, D, NUM_SMS)
     assert t(min(128, 8 * s)) > t(s)
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_per_design_time_matches_the_choice(loom, D):
+    # the per-design modeled time of the chosen design is the model's launch time; an
+    # infeasible design reports a negative time
+    chosen = loom.loom_model_fwd_plan(D)["design"]
+    args = (4, 32, 2048, 2048, D, 0)
+    assert loom.loom_model_fwd_time_us_design(chosen, *args) == pytest.approx(loom.loom_model_fwd_time_us(*args))
+    for d in (1, 2, 3):
+        t = loom.loom_model_fwd_time_us_design(d, *args)
+        assert (t < 0) == (loom.loom_model_fwd_plan_variant(D, d) is None)
+        if t > 0:
+            assert t >= loom.loom_model_fwd_time_us(*args) * (1 - 1e-9)  # the choice is the fastest
