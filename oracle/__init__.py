@@ -5,8 +5,8 @@ CPU-baseline leg of ``bench.py``, never by the product package.  It shares no co
 with the CUDA library; the only common dependency is the seeded input generator
 (``synth``), which holds no attention arithmetic.
 
-Arrays are numpy: Q [B, Hq, Sq, D], K/V [B, Hkv, Skv, D] as uint16 bfloat16 bit
-patterns, results in float64.
+Arrays are numpy: Q [B, Hq, Sq, D], K/V [B, Hkv, Skv, D] (and the GEMM operands A [M, K],
+B [K, N]) as uint16 bfloat16 bit patterns, results in float64.
 """
 from __future__ import annotations
 
@@ -160,3 +160,22 @@ def attention_naive(q, k, v, *, causal=False, scale=None):
         raise ValueError("oracle_attention_naive rejected its arguments")
     n = B * Hq * Sq
     return o[:n].reshape(B, Hq, Sq, D), lse[:n].reshape(B, Hq, Sq)
+
+
+def bf16_to_f64(bits):
+    """Exact widening of bfloat16 bit patterns (uint16) to float64."""
+    bits = np.asarray(bits, dtype=np.uint16)
+    return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def gemm(a, b, *, rows=None):
+    """C = A B in fp64 from bf16 A [M, K] and B [K, N] (the paper's third kernel, evaluated
+    on GEMM shapes): the definition, c_ij = sum_k a_ik b_kj, with the exactly widened
+    inputs and a library matmul as its one step.  ``rows`` optionally selects rows of C."""
+    A = bf16_to_f64(a)
+    Bm = bf16_to_f64(b)
+    if A.ndim != 2 or Bm.ndim != 2 or A.shape[1] != Bm.shape[0]:
+        raise ValueError("expected A [M, K] and B [K, N]")
+    if rows is not None:
+        A = A[np.asarray(rows, dtype=np.int64)]
+    return A @ Bm
