@@ -288,6 +288,42 @@ class Decode:
         return self.bytes / seconds_per_step / 1e9
 
 
+class Gemm:
+    """C = A B in bf16 with fp32 accumulation (the paper's GEMM, Sec. 4); A, B seeded N(0, 1)
+    drawn on the device.  `cublas` times torch.matmul (cuBLAS) on the same buffers."""
+
+    def __init__(self, name, M, N, K, seed=0, sets=2, cublas=False):
+        self.name, self.M, self.N, self.K, self.seed, self.sets, self.cublas = name, M, N, K, seed, sets, cublas
+        self.flops = 2.0 * M * N * K
+        self.bytes = 2 * (M * K + K * N + M * N)
+        self.unit = "TFLOP/s"
+
+    def describe(self):
+        return f"gemm M={self.M} N={self.N} K={self.K} bf16"
+
+    def setup(self, torch, dev, loom):
+        self.loom, self.torch = loom, torch
+        g = torch.Generator(device=dev).manual_seed(self.seed)
+        self.inp = []
+        for _ in range(self.sets):
+            a = torch.randn(self.M, self.K, generator=g, device=dev).to(torch.bfloat16)
+            b = torch.randn(self.K, self.N, generator=g, device=dev).to(torch.bfloat16)
+            self.inp.append((a, b, torch.empty(self.M, self.N, dtype=torch.bfloat16, device=dev)))
+
+    def launches_per_step(self):
+        return 1
+
+    def step(self, i, stream):
+        a, b, c = self.inp[i % self.sets]
+        if self.cublas:
+            self.torch.matmul(a, b, out=c)
+        else:
+            self.loom.loom_gemm_bf16(a, b, c, stream=stream)
+
+    def value(self, seconds_per_step):
+        return self.flops / seconds_per_step / 1e12
+
+
 def to_tensor(torch, bits, dev):
     return to_host_tensor(torch, bits).to(dev)
 
@@ -443,14 +479,15 @@ def main():
     ap.add_argument("--only", default=None,
                     help="comma-separated subset (and order) of the extra workloads to run")
     ap.add_argument("--oracle-seconds", type=float, default=12.0)
-    ap.add_argument("--sweep", choices=["decode", "model"], default=None,
+    ap.add_argument("--sweep", choices=["decode", "model", "gemm"], default=None,
                     help="decode: model-vs-measured sweep of the decode split count; model: the analytic "
                          "model's ranking and accuracy over prefill designs and shapes and decode split "
-                         "counts and shapes (one JSON line per point)")
+                         "counts and shapes; gemm: the BF16 GEMM over the shape grid {256, 2048, 16384}^3 "
+                         "against cuBLAS, every tile width measured (one JSON line per point)")
     ap.add_argument("--ncu-case", default=None,
                     help="profiling run: set up this workload (tiny, tiny_causal, prefill, prefill_causal, "
-                         "long_prefill_d128, long_prefill_d64, batched_decode, long_decode), run --steps "
-                         "launches, print nothing")
+                         "long_prefill_d128, long_prefill_d64, batched_decode, long_decode, gemm_4096, "
+                         "gemm_16k_256_16k), run --steps launches, print nothing")
     args = ap.parse_args()
     world, rank, local = dist_env()
     if args.warmup < 3:
@@ -480,6 +517,8 @@ def main():
         return run_decode_sweep(torch, loom, dev, stream, args, peaks)
     if args.sweep == "model":
         return run_model_sweep(torch, loom, dev, stream, args, peaks)
+    if args.sweep == "gemm":
+        return run_gemm_sweep(torch, loom, dev, stream, args, peaks)
 
     # headline: prefill non-causal, with clocks sampled during the timed loop
     headline.setup(torch, dev, loom)
@@ -645,6 +684,46 @@ def run_model_sweep(torch, loom, dev, stream, args, peaks):
         torch.cuda.empty_cache()
 
 
+GEMM_DIMS = (256, 2048, 16384)
+
+
+def run_gemm_sweep(torch, loom, dev, stream, args, peaks):
+    """The BF16 GEMM over the paper's shape range (every M, N, K in {256, 2048, 16384}):
+    cuBLAS (torch.matmul), this library with the model's tile width, and every tile width
+    forced (does the model's choice measure best?), all on the same buffers and stream."""
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    for M in GEMM_DIMS:
+        for N in GEMM_DIMS:
+            for K in GEMM_DIMS:
+                wl = Gemm("sweep", M, N, K)
+                wl.setup(torch, dev, loom)
+                steps = int(min(500, max(10, 0.05 / (wl.flops / 1.5e15))))
+                chosen = loom.loom_gemm_tile_n(M, N, K)
+                row = {"sweep": "gemm", "workload": wl.describe(), "model_tile_n": chosen}
+                wl.cublas = True
+                row["cublas_tflops"] = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float,
+                                               peaks)["value"]
+                a, b, c = wl.inp[0]
+                ref = c.float()
+                wl.cublas = False
+                for bn in (0, 64, 128, 192, 256):
+                    loom.loom_debug_gemm_tile_n(bn)
+                    r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks)
+                    loom.loom_attn_check_error(stream)
+                    key = "loom_tflops" if bn == 0 else f"bn{bn}_tflops"
+                    row[key] = r["value"]
+                    if bn == 0:
+                        diff = (c.float() - ref).abs().max().item() / max(ref.abs().max().item(), 1e-30)
+                        row["max_rel_diff_vs_cublas"] = float(f"{diff:.3g}")
+                        row["model_us"] = round(loom.loom_model_gemm_time_us(M, N, K, chosen, sms), 2)
+                loom.loom_debug_gemm_tile_n(0)
+                row["vs_cublas"] = round(row["loom_tflops"] / row["cublas_tflops"], 3)
+                row["frac_of_peak"] = round(row["loom_tflops"] / peaks["bf16_tflops"], 4)
+                print(json.dumps(row), flush=True)
+                wl.inp = None
+                torch.cuda.empty_cache()
+
+
 def all_workloads():
     lens = synth.decode_lengths(0, 16, 4096, 8192)
     return [Prefill("tiny", 1, 2, 2, 128, 64, causal=False),
@@ -659,7 +738,10 @@ def all_workloads():
 
 def run_ncu_case(torch, loom, dev, stream, args):
     """A few launches of one workload and nothing else, for small ncu captures."""
-    wl = {w.name: w for w in all_workloads()}[args.ncu_case]
+    cases = {w.name: w for w in all_workloads()}
+    cases["gemm_4096"] = Gemm("gemm_4096", 4096, 4096, 4096)
+    cases["gemm_16k_256_16k"] = Gemm("gemm_16k_256_16k", 16384, 256, 16384)
+    wl = cases[args.ncu_case]
     wl.setup(torch, dev, loom)
     with torch.cuda.stream(stream):
         for i in range(max(1, args.steps)):

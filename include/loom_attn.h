@@ -155,6 +155,25 @@ double loom_model_fwd_time_us_design(int design, int B, int Hq, int Sq, int Skv,
 double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms);
 
 /*
+ * BF16 GEMM, the third kernel the paper evaluates (GEMM shapes, Sec. 4): C = A B with
+ *   a  [M, K] bf16 row-major, read
+ *   b  [K, N] bf16 row-major, read
+ *   c  [M, N] bf16 row-major, written (fp32 accumulation, rounded to nearest even)
+ * The caller owns the buffers; the call is asynchronous on `stream`.  The tile width
+ * (64, 128, 192 or 256 columns of C per 128 rows) and ring depth come from the analytic
+ * model (loom_gemm_tile_n reports the width chosen for a shape).
+ * Errors: INVALID_ARG (NULL pointer, M, N or K < 1), MISALIGNED (pointer not 16-byte
+ * aligned), UNSUPPORTED (K or N not a multiple of 8: rows must be 16-byte multiples for
+ * the tensor-memory-access copies), CUDA (launch failure).
+ */
+loom_status loom_gemm_bf16(const void* a, const void* b, void* c, int M, int N, int K, void* stream);
+int loom_gemm_tile_n(int M, int N, int K);
+/* Modeled GEMM launch time (us) with tile width tile_n on num_sms SMs; < 0 if infeasible. */
+double loom_model_gemm_time_us(int M, int N, int K, int tile_n, int num_sms);
+/* Test hook: force the GEMM tile width (64, 128, 192, 256); anything else restores the model's choice. */
+void loom_debug_gemm_tile_n(int tile_n);
+
+/*
  * Synchronises `stream`, then reads and clears the current device's error word.
  * Returns LOOM_OK, LOOM_ERR_TIMEOUT if a kernel abandoned a bounded wait since the last
  * check, or LOOM_ERR_CUDA if the synchronisation itself failed.
@@ -169,7 +188,8 @@ const char* loom_status_string(loom_status status);
  * loom_debug_set_timeout_ns: upper bound, in nanoseconds of %globaltimer, on every
  *   internal wait of the kernels (default 2e9).  0 restores the default.
  * loom_debug_inject: 0 = off; 1 = the decode split kernel's loader skips the copy of
- *   its second stage; 2 = the prefill kernel's loader skips its second K tile.  The
+ *   its second stage; 2 = the prefill kernel's loader skips its second K tile; 3 = the
+ *   GEMM loader skips its third stage.  The
  *   waits on the skipped data then expire, the kernel unwinds and the next
  *   loom_attn_check_error returns LOOM_ERR_TIMEOUT.  Host-side switch; no fault.
  */

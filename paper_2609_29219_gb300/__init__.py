@@ -26,6 +26,7 @@ __all__ = [
     "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
     "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
     "loom_model_fwd_plan_variant", "loom_model_heg_pipe", "loom_model_fwd_time_us_design",
+    "loom_gemm_bf16", "loom_gemm_tile_n", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -99,6 +100,14 @@ def capi() -> ctypes.CDLL:
             lib.loom_model_fwd_time_us.restype = ctypes.c_double
             lib.loom_model_fwd_time_us_design.argtypes = [i32] * 7
             lib.loom_model_fwd_time_us_design.restype = ctypes.c_double
+            lib.loom_gemm_bf16.argtypes = [vp, vp, vp, i32, i32, i32, vp]
+            lib.loom_gemm_bf16.restype = i32
+            lib.loom_gemm_tile_n.argtypes = [i32, i32, i32]
+            lib.loom_gemm_tile_n.restype = i32
+            lib.loom_model_gemm_time_us.argtypes = [i32] * 5
+            lib.loom_model_gemm_time_us.restype = ctypes.c_double
+            lib.loom_debug_gemm_tile_n.argtypes = [i32]
+            lib.loom_debug_gemm_tile_n.restype = None
             lib.loom_model_decode_time_us.argtypes = [i32, i32, i32, i32, i32, i32, i32]
             lib.loom_model_decode_time_us.restype = ctypes.c_double
             _lib = lib
@@ -267,6 +276,38 @@ def loom_model_fwd_plan_variant(D: int, design: int):
 
 def loom_model_heg_pipe(l: float, m: float, s: float, b_lm: int, b_ms: int) -> float:
     return float(capi().loom_model_heg_pipe(float(l), float(m), float(s), int(b_lm), int(b_ms)))
+
+
+def loom_gemm_bf16(a, b, c=None, *, stream=None):
+    """C = A B (bf16, fp32 accumulation): a [M, K], b [K, N] bf16 CUDA tensors; writes and
+    returns c ([M, N] bf16, allocated if None)."""
+    torch = _torch()
+    bf16 = torch.bfloat16
+    ap = _dev_ptr(a, "a", bf16, 2)
+    bp = _dev_ptr(b, "b", bf16, 2)
+    M, K = a.shape
+    K2, N = b.shape
+    if K2 != K:
+        raise ValueError(f"a is [M, {K}] but b is [{K2}, N]")
+    if c is None:
+        c = torch.empty((M, N), dtype=bf16, device=a.device)
+    cp = _dev_ptr(c, "c", bf16, 2)
+    if tuple(c.shape) != (M, N):
+        raise ValueError("c must be [M, N]")
+    _check(capi().loom_gemm_bf16(ap, bp, cp, M, N, K, _stream_ptr(stream, a.device)), "loom_gemm_bf16")
+    return c
+
+
+def loom_gemm_tile_n(M, N, K) -> int:
+    return int(capi().loom_gemm_tile_n(M, N, K))
+
+
+def loom_model_gemm_time_us(M, N, K, tile_n, num_sms) -> float:
+    return float(capi().loom_model_gemm_time_us(M, N, K, tile_n, num_sms))
+
+
+def loom_debug_gemm_tile_n(tile_n: int):
+    capi().loom_debug_gemm_tile_n(int(tile_n))
 
 
 def loom_model_fwd_time_us_design(design, B, Hq, Sq, Skv, D, causal) -> float:

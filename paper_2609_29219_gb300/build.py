@@ -14,7 +14,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libloomattn.so")
-SOURCES = ["loom_api.cu", "attn_fwd.cu", "attn_decode.cu", "loom_noalloc.cu"]
+SOURCES = ["loom_api.cu", "attn_fwd.cu", "attn_decode.cu", "loom_noalloc.cu", "gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "--expt-relaxed-constexpr",
                 "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall"]

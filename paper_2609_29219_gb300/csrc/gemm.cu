@@ -1,0 +1,325 @@
+// BF16 GEMM for GB300 (sm_103a): C = A B, the third kernel the paper evaluates (GEMM,
+// Sec. 4), with tile width and ring depth from the analytic model (Eq. 6-9).
+//
+// Persistent CTAs walk the output tiles (BM = 128 rows x BN columns) in groups of 8 tile
+// rows, so that CTAs working at the same time share A rows and B columns in L2:
+//
+//   warp 4 (loader, 1 thread)   A tile 128 x 64 and B tile 64 x BN per K stage into an
+//                               NSTAGE-deep ring of 128B-swizzled slots (TMA, full/empty
+//                               mbarriers)
+//   warp 5 (MMA, 1 thread)      tcgen05.mma kind::f16, M = 128, N = BN, K = 16: A K-major,
+//                               B MN-major (rows of B are contiguous in N), fp32 into one of
+//                               two TMEM accumulators
+//   warps 0-3 (epilogue)        thread = row of the tile (= TMEM lane): fp32 -> bf16 in
+//                               64-column chunks, staged per warp in shared memory and
+//                               stored with TMA; the accumulator is released as soon as it
+//                               is in registers, so the next-but-one tile may reuse it.
+//
+// TMEM: [0, BN) accumulator 0 | [BN, 2 BN) accumulator 1.
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include <mutex>
+
+#include "kernels.h"
+#include "model.h"
+#include "ptx.cuh"
+
+namespace loom {
+namespace {
+
+template <int BN>
+struct GemmCfg {
+  static constexpr model::GemmPlan kPlan = model::gemm_plan_variant(BN);
+  static_assert(kPlan.feasible, "no feasible GEMM plan for this tile width");
+  static constexpr int BM = 128, BK = 64;
+  static constexpr int NSTAGE = kPlan.stages;
+  static constexpr int THREADS = 192;                       // 4 epilogue warps, loader, MMA
+  static constexpr int NB = BN / 64;                        // 64-column boxes of a B stage
+  static constexpr uint32_t A_BYTES = BM * BK * 2;          // one 128B-swizzled box
+  static constexpr uint32_t B_BOX_BYTES = BK * 64 * 2;      // 64 K-rows x 64 N-columns
+  static constexpr uint32_t STAGE_BYTES = A_BYTES + NB * B_BOX_BYTES;
+  static constexpr uint32_t STG_OFF = NSTAGE * STAGE_BYTES;  // epilogue staging
+  static constexpr uint32_t STG_WARP = 2 * 32 * 128;         // 2 buffers x 32 rows x 128 B
+  static constexpr uint32_t BAR_OFF = STG_OFF + 4 * STG_WARP;
+  // barriers: full[NSTAGE], empty[NSTAGE], acc_full[2], acc_empty[2], drain
+  static constexpr int NBAR = 2 * NSTAGE + 5;
+  static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
+  static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
+  static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;  // + alignment slack
+  static constexpr uint32_t TMEM_COLS = 2 * BN <= 32 ? 32 : 2 * BN <= 64 ? 64 : 2 * BN <= 128 ? 128
+                                        : 2 * BN <= 256 ? 256 : 512;
+  static_assert(STG_WARP * 4 == model::kGemmStagingBytes, "staging layout matches the model");
+  static_assert(BYTES <= 227 * 1024, "shared memory budget");
+};
+
+struct GemmParams {
+  __nv_bfloat16* c;
+  int M, N, K;
+  int tiles_m, tiles_n, k_iters;
+  KernelCtl ctl;
+};
+
+// Tile t -> (tm, tn): groups of 8 tile rows, column-major inside a group.
+__device__ __forceinline__ void tile_coords(const GemmParams& p, int t, int& tm, int& tn) {
+  constexpr int kGroup = 8;
+  const int per_group = kGroup * p.tiles_n;
+  const int g = t / per_group;
+  const int first = g * kGroup;
+  const int rows = min(kGroup, p.tiles_m - first);
+  const int in = t - g * per_group;
+  tm = first + in % rows;
+  tn = in / rows;
+}
+
+template <int BN>
+__global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
+                const __grid_constant__ CUtensorMap tm_c, const GemmParams p) {
+  using C = GemmCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_base = smem_u32(smem_raw);
+  const uint32_t sbase = (raw_base + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (sbase - raw_base);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const uint32_t bar_full = sbase + C::BAR_OFF;         // [NSTAGE] stage loaded
+  const uint32_t bar_empty = bar_full + 8 * C::NSTAGE;  // [NSTAGE] stage read by the MMAs
+  const uint32_t bar_acc = bar_empty + 8 * C::NSTAGE;   // [2] accumulator b complete
+  const uint32_t bar_acce = bar_acc + 16;               // [2] accumulator b read out
+  const uint32_t bar_drain = bar_acce + 16;
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::TMEM_PTR_OFF);
+  Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
+  const int tiles = p.tiles_m * p.tiles_n;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSTAGE; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(bar_acc + 8 * b, 1);
+      mbar_init(bar_acce + 8 * b, C::BM);
+    }
+    mbar_init(bar_drain, 1);
+    *ab.flag = 0;
+    *(ab.flag + 1) = 0;
+    fence_barrier_init();
+  }
+  if (warp == 5) tmem_alloc(smem_u32(tmem_ptr), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_ptr;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------------ loader
+    if (lane == 0) {
+      prefetch_tensormap(&tm_a);
+      prefetch_tensormap(&tm_b);
+      int it = 0, issued = 0, skipped = -1;
+      bool ok = true;
+      for (int t = blockIdx.x; ok && t < tiles; t += gridDim.x) {
+        int tm, tn;
+        tile_coords(p, t, tm, tn);
+        for (int ks = 0; ks < p.k_iters; ++ks, ++it) {
+          const int s = it % C::NSTAGE;
+          if (!(ok = mbar_wait(bar_empty + 8 * s, ((it / C::NSTAGE) & 1) ^ 1, p.ctl, ab))) break;
+          issued = it + 1;
+          if (p.ctl.inject == 3 && it == 2) {  // test hook: never load this stage
+            skipped = it;
+            continue;
+          }
+          const uint32_t dst = sbase + s * C::STAGE_BYTES;
+          mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
+          tma_load_3d(dst, &tm_a, ks * C::BK, tm * C::BM, 0, bar_full + 8 * s);
+#pragma unroll
+          for (int x = 0; x < C::NB; ++x)
+            tma_load_3d(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b, tn * BN + x * 64, ks * C::BK, 0,
+                        bar_full + 8 * s);
+        }
+      }
+      Abort no_abort{ab.flag + 1};
+      for (int i = max(0, issued - C::NSTAGE); i < issued; ++i)
+        if (i != skipped) mbar_wait(bar_full + 8 * (i % C::NSTAGE), (i / C::NSTAGE) & 1, p.ctl, no_abort);
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16(C::BM, BN, 0, 1);  // A K-major, B MN-major
+      // A: K-major, 8-row groups 1024 B apart, K-step +32 B inside the swizzle row.
+      // B: MN-major, 64-column boxes B_BOX_BYTES apart (LBO), 8 K-rows 1024 B apart (SBO),
+      //    K-step +16 rows = +2048 B.
+      const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
+      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, C::B_BOX_BYTES, 1024);
+      constexpr uint32_t kStage16 = C::STAGE_BYTES >> 4;
+      int it = 0, lt = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; ok && t < tiles; t += gridDim.x, ++lt) {
+        const int b = lt & 1, use = lt >> 1;
+        // the epilogue has read this accumulator's previous tile out
+        if (lt >= 2 && !(ok = mbar_wait(bar_acce + 8 * b, (use - 1) & 1, p.ctl, ab))) break;
+        tc_fence_after();
+        const uint32_t d = tmem + static_cast<uint32_t>(b * BN);
+        for (int ks = 0; ks < p.k_iters; ++ks, ++it) {
+          const int s = it % C::NSTAGE;
+          if (!(ok = mbar_wait(bar_full + 8 * s, (it / C::NSTAGE) & 1, p.ctl, ab))) break;
+          tc_fence_after();
+          const uint64_t da = da0 + s * kStage16, db = db0 + s * kStage16;
+#pragma unroll
+          for (int kk = 0; kk < C::BK / 16; ++kk)
+            mma_ss(d, da + kk * 2, db + kk * 128, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
+          tc_commit(bar_empty + 8 * s);
+        }
+        if (!ok) break;
+        tc_commit(bar_acc + 8 * b);  // the tile's accumulator is complete
+      }
+      Abort no_abort{ab.flag + 1};
+      tc_commit(bar_drain);
+      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue
+    const uint32_t lane_addr = static_cast<uint32_t>(warp * 32) << 16;
+    const uint32_t stg = sbase + C::STG_OFF + static_cast<uint32_t>(warp) * C::STG_WARP;
+    int lt = 0, chunk = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; ok && t < tiles; t += gridDim.x, ++lt) {
+      int tm, tn;
+      tile_coords(p, t, tm, tn);
+      const int b = lt & 1, use = lt >> 1;
+      if (!(ok = mbar_wait_warp(bar_acc + 8 * b, use & 1, p.ctl, ab))) break;
+      tc_fence_after();
+      const uint32_t src = tmem + lane_addr + static_cast<uint32_t>(b * BN);
+#pragma unroll 1
+      for (int c = 0; c < C::NB; ++c) {
+        uint32_t r0[32], r1[32];
+        tmem_ld32(src + c * 64, r0);
+        tmem_ld32(src + c * 64 + 32, r1);
+        tmem_wait_ld();
+        reg_fence32(r0);
+        reg_fence32(r1);
+        if (c == C::NB - 1) {  // the accumulator is in registers: hand it back
+          tc_fence_before();
+          mbar_arrive(bar_acce + 8 * b);
+        }
+        // a chunk lying wholly outside C stores nothing (and takes no staging buffer)
+        if (tn * BN + c * 64 >= p.N || tm * C::BM + warp * 32 >= p.M) continue;
+        uint32_t w[32];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          w[i] = pack_bf16x2(__uint_as_float(r0[2 * i]), __uint_as_float(r0[2 * i + 1]));
+          w[16 + i] = pack_bf16x2(__uint_as_float(r1[2 * i]), __uint_as_float(r1[2 * i + 1]));
+        }
+        // staging buffer chunk % 2: the store issued from it two stored chunks ago has read it
+        const uint32_t buf = stg + static_cast<uint32_t>(chunk & 1) * (32 * 128);
+        ++chunk;
+        if (lane == 0) bulk_wait_group_read1();
+        __syncwarp();
+        const uint32_t row = buf + static_cast<uint32_t>(lane) * 128u;
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          st_shared_v4(row + (static_cast<uint32_t>(q ^ (lane & 7)) << 4), w[4 * q], w[4 * q + 1], w[4 * q + 2],
+                       w[4 * q + 3]);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_3d(&tm_c, buf, tn * BN + c * 64, tm * C::BM + warp * 32, 0);
+          bulk_commit_group();
+        }
+      }
+    }
+    if (lane == 0) bulk_wait_group0();  // the C stores have completed before the CTA exits
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------- host side
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult qres;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &qres) ==
+            cudaSuccess &&
+        qres == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+// 2-D row-major bf16 matrix [rows, cols] as a 3-D tensor with a unit third dimension.
+bool matrix_map(CUtensorMap* map, const void* base, int rows, int cols, int box_cols, int box_rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows), 1};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(cols) * 2, static_cast<cuuint64_t>(cols) * 2 * rows};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(box_cols), static_cast<cuuint32_t>(box_rows), 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN>
+cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int sms) {
+  using C = GemmCfg<BN>;
+  static unsigned long long configured = 0;  // one bit per device
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (!(configured & (1ull << (dev & 63)))) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::BYTES);
+    if (e != cudaSuccess) return e;
+    configured |= 1ull << (dev & 63);
+  }
+  CUtensorMap ma, mb, mc;
+  if (!matrix_map(&ma, a.a, a.M, a.K, 64, C::BM) || !matrix_map(&mb, a.b, a.K, a.N, 64, C::BK) ||
+      !matrix_map(&mc, a.c, a.M, a.N, 64, 32))
+    return cudaErrorInvalidValue;
+  GemmParams p;
+  p.c = static_cast<__nv_bfloat16*>(a.c);
+  p.M = a.M;
+  p.N = a.N;
+  p.K = a.K;
+  p.tiles_m = (a.M + C::BM - 1) / C::BM;
+  p.tiles_n = (a.N + BN - 1) / BN;
+  p.k_iters = (a.K + C::BK - 1) / C::BK;
+  p.ctl = ctl;
+  const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
+  if (tiles > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  const int grid = static_cast<int>(tiles < sms ? tiles : sms);
+  gemm_kernel<BN><<<grid, C::THREADS, C::BYTES, stream>>>(ma, mb, mc, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int gemm_tile_n(int M, int N, int K, int sms) { return model::gemm_choose_bn(M, N, K, sms); }
+
+cudaError_t launch_gemm(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const int bn = a.tile_n ? a.tile_n : gemm_tile_n(a.M, a.N, a.K, sms);
+  switch (bn) {
+    case 64: return launch_bn<64>(a, ctl, stream, sms);
+    case 128: return launch_bn<128>(a, ctl, stream, sms);
+    case 192: return launch_bn<192>(a, ctl, stream, sms);
+    default: return launch_bn<256>(a, ctl, stream, sms);
+  }
+}
+
+}  // namespace loom

@@ -21,6 +21,7 @@ constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // 2 s
 uint64_t g_timeout_ns = kDefaultTimeoutNs;
 int g_inject = 0;
 int g_prefill_design = 0;
+int g_gemm_tile_n = 0;  // test hook: forced GEMM tile width (0: the model's choice)
 
 constexpr int kMaxDevices = 64;
 uint32_t* g_err_ptr[kMaxDevices] = {};
@@ -166,6 +167,35 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
                num_splits, scale};
   return launch_decode(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                  : LOOM_ERR_CUDA;
+}
+
+loom_status loom_gemm_bf16(const void* a, const void* b, void* c, int M, int N, int K, void* stream) {
+  if (!a || !b || !c) return LOOM_ERR_INVALID_ARG;
+  if (M <= 0 || N <= 0 || K <= 0) return LOOM_ERR_INVALID_ARG;
+  if (!aligned16(a) || !aligned16(b) || !aligned16(c)) return LOOM_ERR_MISALIGNED;
+  if (K % 8 != 0 || N % 8 != 0) return LOOM_ERR_UNSUPPORTED;  // 16-byte row strides for TMA
+  KernelCtl ctl;
+  if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
+  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n};
+  return launch_gemm(g, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK : LOOM_ERR_CUDA;
+}
+
+int loom_gemm_tile_n(int M, int N, int K) {
+  if (M <= 0 || N <= 0 || K <= 0) return 0;
+  int sms = current_sm_count();
+  if (sms <= 0) sms = model::kGb300.num_sms;
+  return gemm_tile_n(M, N, K, sms);
+}
+
+double loom_model_gemm_time_us(int M, int N, int K, int tile_n, int num_sms) {
+  if (M <= 0 || N <= 0 || K <= 0 || num_sms <= 0) return -1.0;
+  const model::GemmPlan p = model::gemm_plan_variant(tile_n);
+  if (!p.feasible || (tile_n != 64 && tile_n != 128 && tile_n != 192 && tile_n != 256)) return -1.0;
+  return model::gemm_time_us(p, M, N, K, num_sms);
+}
+
+void loom_debug_gemm_tile_n(int tile_n) {
+  g_gemm_tile_n = (tile_n == 64 || tile_n == 128 || tile_n == 192 || tile_n == 256) ? tile_n : 0;
 }
 
 loom_status loom_attn_check_error(void* stream) {

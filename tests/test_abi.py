@@ -100,3 +100,19 @@ def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
     monkeypatch.setattr(loom, "_LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="no fallback"):
         loom.capi()
+
+
+def test_gemm_rejects_bad_arguments(lib):
+    # every call is rejected during validation, before any device work
+    odd = FAKE + 8
+    assert lib.loom_gemm_bf16(None, FAKE, FAKE, 8, 8, 8, None) == 1   # INVALID_ARG: null
+    assert lib.loom_gemm_bf16(FAKE, FAKE, FAKE, 0, 8, 8, None) == 1   # INVALID_ARG: M = 0
+    assert lib.loom_gemm_bf16(FAKE, odd, FAKE, 8, 8, 8, None) == 3    # MISALIGNED
+    assert lib.loom_gemm_bf16(FAKE, FAKE, FAKE, 8, 8, 12, None) == 2  # UNSUPPORTED: K % 8
+    assert lib.loom_gemm_bf16(FAKE, FAKE, FAKE, 8, 20, 8, None) == 2  # UNSUPPORTED: N % 8
+
+
+def test_gemm_tile_choice_is_a_supported_width(lib):
+    for M, N, K in [(1, 8, 8), (128, 256, 64), (4096, 4096, 4096), (8192, 1024, 8192)]:
+        assert lib.loom_gemm_tile_n(M, N, K) in (64, 128, 192, 256)
+    assert lib.loom_gemm_tile_n(0, 8, 8) == 0
