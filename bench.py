@@ -364,13 +364,13 @@ def job_value(per_rank_value, world):
 WARMUP_SECONDS = 1.0  # clocks ramp up slowly after host-side idle periods
 
 
-def time_steps(torch, wl, steps, warmup, stream, barrier, per_launch_events=True):
-    """Warm up (at least `warmup` steps and WARMUP_SECONDS of back-to-back work), then
+def time_steps(torch, wl, steps, warmup, stream, barrier, per_launch_events=True, warm_s=WARMUP_SECONDS):
+    """Warm up (at least `warmup` steps and `warm_s` seconds of back-to-back work), then
     time exactly `steps` steps with CUDA events on `stream`."""
     t0 = time.perf_counter()
     i = 0
     with torch.cuda.stream(stream):
-        while i < warmup or time.perf_counter() - t0 < WARMUP_SECONDS:
+        while i < warmup or time.perf_counter() - t0 < warm_s:
             for _ in range(max(1, warmup)):
                 wl.step(i, stream)
                 i += 1
@@ -400,9 +400,9 @@ def time_steps(torch, wl, steps, warmup, stream, barrier, per_launch_events=True
     return total_ms, launch_ms
 
 
-def measure(torch, wl, steps, warmup, stream, barrier, world, reduce_max, peaks, clocks=None):
+def measure(torch, wl, steps, warmup, stream, barrier, world, reduce_max, peaks, clocks=None, warm_s=WARMUP_SECONDS):
     t_wall0 = time.time()
-    total_ms, launch_ms = time_steps(torch, wl, steps, warmup, stream, barrier)
+    total_ms, launch_ms = time_steps(torch, wl, steps, warmup, stream, barrier, warm_s=warm_s)
     t_wall1 = time.time()
     window = (t_wall1 - total_ms * 1e-3, t_wall1)  # the timed loop ends at the final sync
     del t_wall0
@@ -689,8 +689,10 @@ GEMM_DIMS = (256, 2048, 16384)
 
 def run_gemm_sweep(torch, loom, dev, stream, args, peaks):
     """The BF16 GEMM over the paper's shape range (every M, N, K in {256, 2048, 16384}):
-    cuBLAS (torch.matmul), this library with the model's tile width, and every tile width
-    forced (does the model's choice measure best?), all on the same buffers and stream."""
+    cuBLAS (torch.matmul); this library with the model's (tile width, split count); every
+    tile width with persistent tiles (S = 1); and, at the model's tile width, every split
+    count that leaves each CTA two K stages or more (does the model's choice measure
+    best?).  All on the same buffers and stream."""
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     for M in GEMM_DIMS:
         for N in GEMM_DIMS:
@@ -698,29 +700,39 @@ def run_gemm_sweep(torch, loom, dev, stream, args, peaks):
                 wl = Gemm("sweep", M, N, K)
                 wl.setup(torch, dev, loom)
                 steps = int(min(500, max(10, 0.05 / (wl.flops / 1.5e15))))
-                chosen = loom.loom_gemm_tile_n(M, N, K)
-                row = {"sweep": "gemm", "workload": wl.describe(), "model_tile_n": chosen}
-                wl.cublas = True
-                row["cublas_tflops"] = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float,
-                                               peaks)["value"]
-                a, b, c = wl.inp[0]
-                ref = c.float()
-                wl.cublas = False
-                for bn in (0, 64, 128, 192, 256):
-                    loom.loom_debug_gemm_tile_n(bn)
-                    r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks)
+                bn, sp = loom.loom_gemm_tile_n(M, N, K), loom.loom_gemm_splits(M, N, K)
+                row = {"sweep": "gemm", "workload": wl.describe(), "model_tile_n": bn, "model_splits": sp,
+                       "model_us": round(loom.loom_model_gemm_time_us(M, N, K, bn, sp, sms), 2)}
+
+                def timed():
+                    r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks, warm_s=0.25)
                     loom.loom_attn_check_error(stream)
-                    key = "loom_tflops" if bn == 0 else f"bn{bn}_tflops"
-                    row[key] = r["value"]
-                    if bn == 0:
-                        diff = (c.float() - ref).abs().max().item() / max(ref.abs().max().item(), 1e-30)
-                        row["max_rel_diff_vs_cublas"] = float(f"{diff:.3g}")
-                        row["model_us"] = round(loom.loom_model_gemm_time_us(M, N, K, chosen, sms), 2)
+                    return r["value"]
+
+                wl.cublas = True
+                row["cublas_tflops"] = timed()
+                ref = wl.inp[0][2].float()
+                wl.cublas = False
+                row["loom_tflops"] = timed()
+                c = wl.inp[0][2].float()
+                row["max_rel_diff_vs_cublas"] = float(f"{(c - ref).abs().max().item() / max(ref.abs().max().item(), 1e-30):.3g}")
+                for t in (64, 128, 192, 256):
+                    loom.loom_debug_gemm_tile_n(t)
+                    loom.loom_debug_gemm_splits(1)
+                    row[f"bn{t}_s1_tflops"] = timed()
+                loom.loom_debug_gemm_tile_n(bn)
+                for s_ in (2, 4, 8, 16):
+                    if (K + 63) // 64 < 2 * s_:
+                        break
+                    loom.loom_debug_gemm_splits(s_)
+                    row[f"bn{bn}_s{s_}_tflops"] = timed()
                 loom.loom_debug_gemm_tile_n(0)
+                loom.loom_debug_gemm_splits(0)
                 row["vs_cublas"] = round(row["loom_tflops"] / row["cublas_tflops"], 3)
                 row["frac_of_peak"] = round(row["loom_tflops"] / peaks["bf16_tflops"], 4)
                 print(json.dumps(row), flush=True)
                 wl.inp = None
+                del ref, c
                 torch.cuda.empty_cache()
 
 

@@ -159,19 +159,30 @@ double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, in
  *   a  [M, K] bf16 row-major, read
  *   b  [K, N] bf16 row-major, read
  *   c  [M, N] bf16 row-major, written (fp32 accumulation, rounded to nearest even)
- * The caller owns the buffers; the call is asynchronous on `stream`.  The tile width
- * (64, 128, 192 or 256 columns of C per 128 rows) and ring depth come from the analytic
- * model (loom_gemm_tile_n reports the width chosen for a shape).
+ * The caller owns the buffers; the call is asynchronous on `stream` and needs no
+ * workspace.  The analytic model picks the tile width (64, 128, 192 or 256 columns of C
+ * per 128 rows), the ring depth and the split count S: S = 1 walks the tiles with
+ * persistent CTAs; S = 2, 4, 8 or 16 gives each tile a cluster of S CTAs that split K and
+ * sum their fp32 partials through distributed shared memory in a fixed order (so the
+ * result depends on S but not on timing).  loom_gemm_tile_n / loom_gemm_splits report the
+ * choice for a shape on the current device.
  * Errors: INVALID_ARG (NULL pointer, M, N or K < 1), MISALIGNED (pointer not 16-byte
  * aligned), UNSUPPORTED (K or N not a multiple of 8: rows must be 16-byte multiples for
  * the tensor-memory-access copies), CUDA (launch failure).
  */
 loom_status loom_gemm_bf16(const void* a, const void* b, void* c, int M, int N, int K, void* stream);
+/* The model's tile width / split count for this shape (0 for a non-positive size).  Without a
+ * device the cluster occupancy is estimated as whole clusters in 8 equal SM groups. */
 int loom_gemm_tile_n(int M, int N, int K);
-/* Modeled GEMM launch time (us) with tile width tile_n on num_sms SMs; < 0 if infeasible. */
-double loom_model_gemm_time_us(int M, int N, int K, int tile_n, int num_sms);
-/* Test hook: force the GEMM tile width (64, 128, 192, 256); anything else restores the model's choice. */
+int loom_gemm_splits(int M, int N, int K);
+/* Modeled GEMM launch time (us) with tile width tile_n and split count splits on num_sms SMs
+ * (cluster occupancy estimated as above); < 0 if infeasible. */
+double loom_model_gemm_time_us(int M, int N, int K, int tile_n, int splits, int num_sms);
+/* Test hooks: force the GEMM tile width (64, 128, 192, 256) / split count (1, 2, 4, 8, 16);
+ * any other value restores the model's choice.  A forced split may leave CTAs no K stage:
+ * their partial is zero. */
 void loom_debug_gemm_tile_n(int tile_n);
+void loom_debug_gemm_splits(int splits);
 
 /*
  * Synchronises `stream`, then reads and clears the current device's error word.
@@ -189,7 +200,7 @@ const char* loom_status_string(loom_status status);
  *   internal wait of the kernels (default 2e9).  0 restores the default.
  * loom_debug_inject: 0 = off; 1 = the decode split kernel's loader skips the copy of
  *   its second stage; 2 = the prefill kernel's loader skips its second K tile; 3 = the
- *   GEMM loader skips its third stage.  The
+ *   GEMM loader skips its third stage (of each CTA's K range).  The
  *   waits on the skipped data then expire, the kernel unwinds and the next
  *   loom_attn_check_error returns LOOM_ERR_TIMEOUT.  Host-side switch; no fault.
  */

@@ -26,7 +26,8 @@ __all__ = [
     "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
     "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
     "loom_model_fwd_plan_variant", "loom_model_heg_pipe", "loom_model_fwd_time_us_design",
-    "loom_gemm_bf16", "loom_gemm_tile_n", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
+    "loom_gemm_bf16", "loom_gemm_tile_n", "loom_gemm_splits", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
+    "loom_debug_gemm_splits",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -104,10 +105,14 @@ def capi() -> ctypes.CDLL:
             lib.loom_gemm_bf16.restype = i32
             lib.loom_gemm_tile_n.argtypes = [i32, i32, i32]
             lib.loom_gemm_tile_n.restype = i32
-            lib.loom_model_gemm_time_us.argtypes = [i32] * 5
+            lib.loom_gemm_splits.argtypes = [i32, i32, i32]
+            lib.loom_gemm_splits.restype = i32
+            lib.loom_model_gemm_time_us.argtypes = [i32] * 6
             lib.loom_model_gemm_time_us.restype = ctypes.c_double
             lib.loom_debug_gemm_tile_n.argtypes = [i32]
             lib.loom_debug_gemm_tile_n.restype = None
+            lib.loom_debug_gemm_splits.argtypes = [i32]
+            lib.loom_debug_gemm_splits.restype = None
             lib.loom_model_decode_time_us.argtypes = [i32, i32, i32, i32, i32, i32, i32]
             lib.loom_model_decode_time_us.restype = ctypes.c_double
             _lib = lib
@@ -302,12 +307,20 @@ def loom_gemm_tile_n(M, N, K) -> int:
     return int(capi().loom_gemm_tile_n(M, N, K))
 
 
-def loom_model_gemm_time_us(M, N, K, tile_n, num_sms) -> float:
-    return float(capi().loom_model_gemm_time_us(M, N, K, tile_n, num_sms))
+def loom_gemm_splits(M, N, K) -> int:
+    return int(capi().loom_gemm_splits(M, N, K))
+
+
+def loom_model_gemm_time_us(M, N, K, tile_n, splits, num_sms) -> float:
+    return float(capi().loom_model_gemm_time_us(M, N, K, tile_n, splits, num_sms))
 
 
 def loom_debug_gemm_tile_n(tile_n: int):
     capi().loom_debug_gemm_tile_n(int(tile_n))
+
+
+def loom_debug_gemm_splits(splits: int):
+    capi().loom_debug_gemm_splits(int(splits))
 
 
 def loom_model_fwd_time_us_design(design, B, Hq, Sq, Skv, D, causal) -> float:

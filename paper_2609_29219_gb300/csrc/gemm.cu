@@ -21,12 +21,43 @@
 
 #include <mutex>
 
-#include "kernels.h"
-#include "model.h"
+#include "gemm.h"
+#include "gemm_model.h"
 #include "ptx.cuh"
 
 namespace loom {
 namespace {
+
+// Wait until at most one committed bulk store of this thread has not yet read its source.
+__device__ __forceinline__ void bulk_wait_group_read1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+
+// ---------------------------------------------------------------- cluster primitives
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// All threads of every CTA of the cluster; orders this thread's earlier shared-memory
+// writes before the peers' later reads (release / acquire at cluster scope).
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared-memory offset in CTA `rank` of this cluster.
+__device__ __forceinline__ uint32_t map_shared_rank(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float4 ld_dsmem_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
 
 template <int BN>
 struct GemmCfg {
@@ -57,6 +88,7 @@ struct GemmParams {
   __nv_bfloat16* c;
   int M, N, K;
   int tiles_m, tiles_n, k_iters;
+  int splits;  // split-K kernel: CTAs per cluster (= per tile)
   KernelCtl ctl;
 };
 
@@ -241,6 +273,178 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
   }
 }
 
+// ---------------------------------------------------------------- split-K clusters
+// One cluster of S = p.splits CTAs per C tile; CTA r of the cluster multiplies the K
+// stages [r k_iters / S, (r + 1) k_iters / S) into its TMEM accumulator with the same
+// loader / MMA roles as above.  The epilogue warps then park the fp32 partial tile in the
+// CTA's own shared memory (over the ring, which is idle by then), rows 128 B-swizzled in
+// 16-byte chunks; after a cluster barrier CTA r sums rows [r 128 / S, (r + 1) 128 / S)
+// over the S partials in the order s = 0 .. S - 1, reading its peers' shared memory,
+// and stores them as bf16.  A second cluster barrier keeps every partial alive until all
+// peers have read it.  The summation order does not depend on timing, so the result is
+// deterministic for a given S.
+template <int BN>
+__global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
+    gemm_splitk_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
+                       const GemmParams p) {
+  using C = GemmCfg<BN>;
+  constexpr uint32_t kCols = BN <= 64 ? 64 : BN <= 128 ? 128 : 256;  // one accumulator
+  constexpr uint32_t kRowBytes = BN * 4;                                // fp32 partial row
+  static_assert(C::BM * kRowBytes <= C::STG_OFF, "the partial tile fits in the ring");
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_base = smem_u32(smem_raw);
+  const uint32_t sbase = (raw_base + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (sbase - raw_base);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const uint32_t bar_full = sbase + C::BAR_OFF;
+  const uint32_t bar_empty = bar_full + 8 * C::NSTAGE;
+  const uint32_t bar_acc = bar_empty + 8 * C::NSTAGE;  // accumulator complete
+  const uint32_t bar_drain = bar_acc + 32;
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::TMEM_PTR_OFF);
+  Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
+
+  const int S = p.splits;
+  const uint32_t rank = cluster_ctarank();
+  const int tile = static_cast<int>(blockIdx.x) / S;
+  int tm, tn;
+  tile_coords(p, tile, tm, tn);
+  const int k0 = static_cast<int>(static_cast<long long>(p.k_iters) * rank / S);
+  const int k1 = static_cast<int>(static_cast<long long>(p.k_iters) * (rank + 1) / S);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSTAGE; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, 1);
+    }
+    mbar_init(bar_acc, 1);
+    mbar_init(bar_drain, 1);
+    *ab.flag = 0;
+    *(ab.flag + 1) = 0;
+    fence_barrier_init();
+  }
+  if (warp == 5) tmem_alloc(smem_u32(tmem_ptr), kCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_ptr;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------------ loader
+    if (lane == 0) {
+      prefetch_tensormap(&tm_a);
+      prefetch_tensormap(&tm_b);
+      int issued = 0, skipped = -1;
+      for (int ks = k0, it = 0; ks < k1; ++ks, ++it) {
+        const int s = it % C::NSTAGE;
+        if (!mbar_wait(bar_empty + 8 * s, ((it / C::NSTAGE) & 1) ^ 1, p.ctl, ab)) break;
+        issued = it + 1;
+        if (p.ctl.inject == 3 && it == 2) {  // test hook: never load this stage
+          skipped = it;
+          continue;
+        }
+        const uint32_t dst = sbase + s * C::STAGE_BYTES;
+        mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
+        tma_load_3d(dst, &tm_a, ks * C::BK, tm * C::BM, 0, bar_full + 8 * s);
+#pragma unroll
+        for (int x = 0; x < C::NB; ++x)
+          tma_load_3d(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b, tn * BN + x * 64, ks * C::BK, 0,
+                      bar_full + 8 * s);
+      }
+      Abort no_abort{ab.flag + 1};
+      for (int i = max(0, issued - C::NSTAGE); i < issued; ++i)
+        if (i != skipped) mbar_wait(bar_full + 8 * (i % C::NSTAGE), (i / C::NSTAGE) & 1, p.ctl, no_abort);
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16(C::BM, BN, 0, 1);
+      const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
+      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, C::B_BOX_BYTES, 1024);
+      constexpr uint32_t kStage16 = C::STAGE_BYTES >> 4;
+      bool ok = true;
+      for (int ks = k0, it = 0; ks < k1; ++ks, ++it) {
+        const int s = it % C::NSTAGE;
+        if (!(ok = mbar_wait(bar_full + 8 * s, (it / C::NSTAGE) & 1, p.ctl, ab))) break;
+        tc_fence_after();
+        const uint64_t da = da0 + s * kStage16, db = db0 + s * kStage16;
+#pragma unroll
+        for (int kk = 0; kk < C::BK / 16; ++kk)
+          mma_ss(tmem, da + kk * 2, db + kk * 128, idesc, (it > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(bar_empty + 8 * s);
+      }
+      if (ok) tc_commit(bar_acc);  // with no stages at all this arrives at once
+      Abort no_abort{ab.flag + 1};
+      tc_commit(bar_drain);
+      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+    }
+  } else {
+    // ------------------------------------------------------------------ partial tile -> smem
+    const int row = warp * 32 + lane;
+    const uint32_t prow = sbase + static_cast<uint32_t>(row) * kRowBytes;
+    if (mbar_wait_warp(bar_acc, 0, p.ctl, ab)) {
+      tc_fence_after();
+      fence_proxy_async_smem();  // the ring's last TMA writes and MMA reads are complete
+      const uint32_t src = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        uint32_t r[32];
+        if (k1 > k0) {
+          tmem_ld32(src + c * 32, r);
+          tmem_wait_ld();
+          reg_fence32(r);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) r[i] = 0u;
+        }
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const uint32_t chunk = static_cast<uint32_t>(c * 8 + q) ^ static_cast<uint32_t>(row & 7);
+          st_shared_v4(prow + chunk * 16u, r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]);
+        }
+      }
+    }
+  }
+
+  __syncwarp();
+  cluster_sync_all();  // every partial tile is in its CTA's shared memory
+
+  if (warp < 4 && !ab.raised()) {
+    // ------------------------------------------------------------------ reduce rows, store
+    const int rows = C::BM / S;
+    constexpr int kChunks = BN / 4;  // 16-byte chunks of a partial row
+    const int r_first = static_cast<int>(rank) * rows;
+    for (int i = threadIdx.x; i < rows * kChunks; i += 128) {
+      const int r = r_first + i / kChunks, j = i % kChunks;
+      const uint32_t off = static_cast<uint32_t>(r) * kRowBytes + ((static_cast<uint32_t>(j) ^ (r & 7)) << 4);
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int s = 0; s < S; ++s) {
+        const float4 v = ld_dsmem_f4(map_shared_rank(sbase + off, static_cast<uint32_t>(s)));
+        acc.x += v.x;
+        acc.y += v.y;
+        acc.z += v.z;
+        acc.w += v.w;
+      }
+      const int grow = tm * C::BM + r, gcol = tn * BN + j * 4;
+      if (grow < p.M && gcol < p.N) {  // N % 8 == 0: the 4 columns are all inside C
+        uint2 w;
+        w.x = pack_bf16x2(acc.x, acc.y);
+        w.y = pack_bf16x2(acc.z, acc.w);
+        *reinterpret_cast<uint2*>(p.c + static_cast<size_t>(grow) * p.N + gcol) = w;
+      }
+    }
+  }
+
+  __syncwarp();
+  cluster_sync_all();  // no CTA leaves while a peer may still read its partial
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kCols);
+  }
+}
+
 // ---------------------------------------------------------------- host side
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                    const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -274,29 +478,43 @@ bool matrix_map(CUtensorMap* map, const void* base, int rows, int cols, int box_
 }
 
 template <int BN>
-cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int sms) {
-  using C = GemmCfg<BN>;
-  static unsigned long long configured = 0;  // one bit per device
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (!(configured & (1ull << (dev & 63)))) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::BYTES);
-    if (e != cudaSuccess) return e;
-    configured |= 1ull << (dev & 63);
-  }
-  CUtensorMap ma, mb, mc;
-  if (!matrix_map(&ma, a.a, a.M, a.K, 64, C::BM) || !matrix_map(&mb, a.b, a.K, a.N, 64, C::BK) ||
-      !matrix_map(&mc, a.c, a.M, a.N, 64, 32))
-    return cudaErrorInvalidValue;
+bool set_smem_attr(const void* fn, int& done_mask, int bit) {
+  // one opt-in per kernel and device (the mask is per template instance)
+  if (done_mask & (1 << bit)) return true;
+  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmCfg<BN>::BYTES) != cudaSuccess)
+    return false;
+  done_mask |= 1 << bit;
+  return true;
+}
+
+bool make_maps(const GemmArgs& a, int bm, CUtensorMap* ma, CUtensorMap* mb, CUtensorMap* mc) {
+  return matrix_map(ma, a.a, a.M, a.K, 64, bm) && matrix_map(mb, a.b, a.K, a.N, 64, 64) &&
+         (mc == nullptr || matrix_map(mc, a.c, a.M, a.N, 64, 32));
+}
+
+GemmParams make_params(const GemmArgs& a, const KernelCtl& ctl, int bn, int splits) {
   GemmParams p;
   p.c = static_cast<__nv_bfloat16*>(a.c);
   p.M = a.M;
   p.N = a.N;
   p.K = a.K;
-  p.tiles_m = (a.M + C::BM - 1) / C::BM;
-  p.tiles_n = (a.N + BN - 1) / BN;
-  p.k_iters = (a.K + C::BK - 1) / C::BK;
+  p.tiles_m = (a.M + 127) / 128;
+  p.tiles_n = (a.N + bn - 1) / bn;
+  p.k_iters = (a.K + 63) / 64;
+  p.splits = splits;
   p.ctl = ctl;
+  return p;
+}
+
+template <int BN>
+cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int dev, int sms) {
+  using C = GemmCfg<BN>;
+  static int configured = 0;  // bit per device (devices 0..30)
+  if (dev < 31 && !set_smem_attr<BN>(reinterpret_cast<const void*>(gemm_kernel<BN>), configured, dev))
+    return cudaErrorInvalidValue;
+  CUtensorMap ma, mb, mc;
+  if (!make_maps(a, C::BM, &ma, &mb, &mc)) return cudaErrorInvalidValue;
+  const GemmParams p = make_params(a, ctl, BN, 1);
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   const int grid = static_cast<int>(tiles < sms ? tiles : sms);
@@ -304,21 +522,113 @@ cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stre
   return cudaGetLastError();
 }
 
+template <int BN>
+cudaLaunchConfig_t splitk_config(int grid, int S, cudaStream_t stream, cudaLaunchAttribute* attr) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
+  cfg.blockDim = dim3(GemmCfg<BN>::THREADS, 1, 1);
+  cfg.dynamicSmemBytes = GemmCfg<BN>::BYTES;
+  cfg.stream = stream;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(S);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cfg;
+}
+
+template <int BN>
+bool prepare_splitk(int dev) {
+  static int configured = 0;
+  static int nonportable = 0;
+  const void* fn = reinterpret_cast<const void*>(gemm_splitk_kernel<BN>);
+  if (dev >= 31) return false;
+  if (!set_smem_attr<BN>(fn, configured, dev)) return false;
+  if (!(nonportable & (1 << dev))) {
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) return false;
+    nonportable |= 1 << dev;
+  }
+  return true;
+}
+
+// CTAs of clusters of S that fit on the device at once (0: none, or cannot be queried).
+template <int BN>
+int splitk_slots(int dev, int S) {
+  static int cache[31][5];  // [device][log2 S], value + 1 once known
+  int lg = 0;
+  while ((1 << lg) < S) ++lg;
+  if (dev >= 31 || lg > 4 || (1 << lg) != S) return 0;
+  if (cache[dev][lg] != 0) return cache[dev][lg] - 1;
+  int clusters = 0;
+  if (prepare_splitk<BN>(dev)) {
+    cudaLaunchAttribute attr[1];
+    cudaLaunchConfig_t cfg = splitk_config<BN>(S * 64, S, nullptr, attr);
+    if (cudaOccupancyMaxActiveClusters(&clusters, gemm_splitk_kernel<BN>, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      clusters = 0;
+    }
+  }
+  cache[dev][lg] = clusters * S + 1;
+  return clusters * S;
+}
+
+int splitk_slots_any(int dev, int bn, int S) {
+  switch (bn) {
+    case 64: return splitk_slots<64>(dev, S);
+    case 128: return splitk_slots<128>(dev, S);
+    case 192: return splitk_slots<192>(dev, S);
+    default: return splitk_slots<256>(dev, S);
+  }
+}
+
+template <int BN>
+cudaError_t launch_splitk(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int dev, int S) {
+  if (!prepare_splitk<BN>(dev)) return cudaErrorInvalidValue;
+  CUtensorMap ma, mb;
+  if (!make_maps(a, GemmCfg<BN>::BM, &ma, &mb, nullptr)) return cudaErrorInvalidValue;
+  const GemmParams p = make_params(a, ctl, BN, S);
+  const long long ctas = static_cast<long long>(p.tiles_m) * p.tiles_n * S;
+  if (ctas > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = splitk_config<BN>(static_cast<int>(ctas), S, stream, attr);
+  return cudaLaunchKernelEx(&cfg, gemm_splitk_kernel<BN>, ma, mb, p);
+}
+
+bool device_sms(int* dev, int* sms) {
+  if (cudaGetDevice(dev) != cudaSuccess) return false;
+  return cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, *dev) == cudaSuccess && *sms > 0;
+}
+
 }  // namespace
 
-int gemm_tile_n(int M, int N, int K, int sms) { return model::gemm_choose_bn(M, N, K, sms); }
+GemmChoice gemm_choice(int M, int N, int K, GemmChoice forced) {
+  int dev = 0, sms = 0;
+  if (!device_sms(&dev, &sms)) return {0, 0};
+  const model::GemmChoiceModel c = model::gemm_choose(
+      M, N, K, sms, [dev](int bn, int S) { return splitk_slots_any(dev, bn, S); }, model::kGb300, forced.tile_n,
+      forced.splits);
+  return {c.bn, c.splits};
+}
 
 cudaError_t launch_gemm(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
   int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (e != cudaSuccess) return e;
-  const int bn = a.tile_n ? a.tile_n : gemm_tile_n(a.M, a.N, a.K, sms);
-  switch (bn) {
-    case 64: return launch_bn<64>(a, ctl, stream, sms);
-    case 128: return launch_bn<128>(a, ctl, stream, sms);
-    case 192: return launch_bn<192>(a, ctl, stream, sms);
-    default: return launch_bn<256>(a, ctl, stream, sms);
+  if (!device_sms(&dev, &sms)) return cudaErrorNoDevice;
+  const GemmChoice c = gemm_choice(a.M, a.N, a.K, {a.tile_n, a.splits});
+  if (c.tile_n == 0) return cudaErrorInvalidConfiguration;
+  if (c.splits > 1) {
+    switch (c.tile_n) {
+      case 64: return launch_splitk<64>(a, ctl, stream, dev, c.splits);
+      case 128: return launch_splitk<128>(a, ctl, stream, dev, c.splits);
+      case 192: return launch_splitk<192>(a, ctl, stream, dev, c.splits);
+      default: return launch_splitk<256>(a, ctl, stream, dev, c.splits);
+    }
+  }
+  switch (c.tile_n) {
+    case 64: return launch_bn<64>(a, ctl, stream, dev, sms);
+    case 128: return launch_bn<128>(a, ctl, stream, dev, sms);
+    case 192: return launch_bn<192>(a, ctl, stream, dev, sms);
+    default: return launch_bn<256>(a, ctl, stream, dev, sms);
   }
 }
 

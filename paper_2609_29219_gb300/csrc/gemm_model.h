@@ -1,0 +1,159 @@
+// Analytic model of the BF16 GEMM (C = A B), the paper's third kernel (Sec. 4): the HEG
+// latency composition of Eq. 5-7 and the enumerated choice of Eq. 8-9, restated for one
+// GB300 SM.  It shares the architecture description and the HEG operators of model.h.
+#pragma once
+
+#include "model.h"
+
+namespace loom {
+namespace model {
+
+// ------------------------------------------------------------------ persistent tiles
+// The paper's third kernel.  A CTA computes BM = 128 rows x BN columns of C at a time,
+// with K in BK = 64 stages through an NSTAGE ring (Eq. 6 with the load boundary open)
+// and the accumulator double-buffered in TMEM, so that one tile's epilogue overlaps the
+// next tile's MMAs.  Candidates: BN in {64, 128, 192, 256} x ring depth.
+struct GemmPlan {
+  int bm, bn, bk, stages, smem_bytes, tmem_cols;
+  double t_load_ns, t_mma_ns, t_iter_ns, t_epi_ns;
+  bool feasible;
+};
+
+constexpr int kGemmStagingBytes = 4 * 2 * 32 * 128;  // 4 epilogue warps x 2 buffers x 32 rows x 128 B
+
+constexpr GemmPlan gemm_eval(const ArchDesc& a, int bn, int stages) {
+  GemmPlan p{};
+  p.bm = 128;
+  p.bn = bn;
+  p.bk = 64;
+  p.stages = stages;
+  const double stage_bytes = (p.bm + bn) * p.bk * 2.0;
+  p.t_load_ns = stage_bytes / a.l2_smem_gbs_sm;  // A and B tiles from L2
+  p.t_mma_ns = (p.bk / 16.0) * dmax(a.mma_clk_per_n * bn, a.mma_min_clk) / a.sm_ghz;
+  p.t_iter_ns = heg_pipe(p.t_load_ns, p.t_mma_ns, 0.0, 1, 0);
+  p.t_epi_ns = p.bm * bn * 2.0 / a.l2_smem_gbs_sm;  // the C tile leaves through L2
+  p.smem_bytes = static_cast<int>(stages * stage_bytes) + kGemmStagingBytes + 1024 + 256;
+  p.tmem_cols = 2 * bn;
+  p.feasible = p.smem_bytes <= a.smem_per_cta && p.tmem_cols <= a.tmem_cols && stages >= 2 && bn % 64 == 0 &&
+               bn >= 64 && bn <= 256 && (stages - 1) * p.t_iter_ns >= a.mem_latency_ns * 0.5;
+  return p;
+}
+
+// Eq. 8 for one tile width: the ring depth with the lowest modeled iteration, ties to the
+// deeper ring.
+constexpr GemmPlan gemm_plan_variant(int bn, const ArchDesc& a = kGb300) {
+  GemmPlan best{};
+  best.feasible = false;
+  for (int stages = 2; stages <= 12; ++stages) {
+    const GemmPlan p = gemm_eval(a, bn, stages);
+    if (!p.feasible) continue;
+    if (!best.feasible || p.t_iter_ns < best.t_iter_ns * (1.0 - 1e-9) ||
+        (p.t_iter_ns <= best.t_iter_ns * (1.0 + 1e-9) && p.stages > best.stages))
+      best = p;
+  }
+  return best;
+}
+
+// Eq. 5-7 for a whole launch: the busiest SM runs ceil(tiles / SMs) tiles of ceil(K / BK)
+// iterations back to back; the first load and the last epilogue are exposed.
+constexpr double gemm_time_us(const GemmPlan& p, long long M, long long N, long long K, int num_sms,
+                              const ArchDesc& a = kGb300) {
+  const long long tiles = cdiv(M, p.bm) * cdiv(N, p.bn);
+  const long long per_sm = cdiv(tiles, num_sms);
+  const double t = heg_seq(heg_seq(p.t_load_ns, heg_for(per_sm * cdiv(K, p.bk), p.t_iter_ns)), p.t_epi_ns);
+  return (t + a.launch_ns * 0.2) * 1e-3;
+}
+
+// Eq. 9: the tile width with the lowest modeled launch time (ties to the wider tile).
+constexpr int gemm_choose_bn(long long M, long long N, long long K, int num_sms, const ArchDesc& a = kGb300) {
+  int best_bn = 0;
+  double best_t = 1e300;
+  for (int bn = 256; bn >= 64; bn -= 64) {
+    const GemmPlan p = gemm_plan_variant(bn, a);
+    if (!p.feasible) continue;
+    const double t = gemm_time_us(p, M, N, K, num_sms, a);
+    if (t < best_t * (1.0 - 1e-9)) {
+      best_t = t;
+      best_bn = bn;
+    }
+  }
+  return best_bn;
+}
+
+// ------------------------------------------------------------------ split-K clusters
+// When there are few C tiles for the SMs (small M x N, long K), a cluster of S CTAs shares
+// one tile, each CTA taking a contiguous 1/S of the K stages into its own TMEM
+// accumulator.  The S fp32 partial tiles are then summed through distributed shared
+// memory: every CTA parks its partial in its own shared memory and, after a cluster
+// barrier, reduces BM / S rows of the tile over all S CTAs and stores them.  So each CTA
+// reads one tile's worth of fp32 over DSMEM, and the reduction adds two cluster barriers.
+struct GemmClusterArch {
+  double dsmem_gbs_sm;    // distributed-shared-memory read rate of one SM, GB/s (assumed)
+  double cluster_sync_ns; // one cluster-wide barrier.cluster round trip (assumed)
+};
+inline constexpr GemmClusterArch kGb300Cluster = {120.0, 300.0};
+
+constexpr int kGemmMaxSplits = 16;
+
+// Time of one launch with split S (S >= 2) when `cta_slots` CTAs of clusters of S fit on the
+// GPU at once: every CTA of the busiest wave loads and multiplies ceil(k_iters / S) stages,
+// then reduces and stores its BM / S rows.
+constexpr double gemm_splitk_time_us(const GemmPlan& p, long long M, long long N, long long K, int S, int cta_slots,
+                                     const ArchDesc& a = kGb300, const GemmClusterArch& c = kGb300Cluster) {
+  const long long tiles = cdiv(M, p.bm) * cdiv(N, p.bn);
+  const long long units = tiles * S;
+  const long long waves = cdiv(units, cta_slots < S ? S : cta_slots);
+  const long long iters = cdiv(cdiv(K, p.bk), S);
+  const double t_red = p.bm * p.bn * 4.0 / c.dsmem_gbs_sm + 2.0 * c.cluster_sync_ns;
+  const double t_unit = heg_seq(heg_seq(p.t_load_ns, heg_for(iters, p.t_iter_ns)), t_red + p.t_epi_ns / S);
+  return (static_cast<double>(waves) * t_unit + a.launch_ns * 0.2) * 1e-3;
+}
+
+// Split counts the kernel supports, and the plan of the split-K kernel for one tile width
+// (the same ring as the persistent kernel: the partial tile reuses the ring's memory).
+constexpr bool gemm_split_supported(int S) { return S == 1 || S == 2 || S == 4 || S == 8 || S == 16; }
+
+// Eq. 9 over (tile width, split count).  `slots(bn, S)` is the number of CTAs of clusters
+// of S that fit on the GPU at once with tile width bn; zero rules the split out.  A
+// non-zero `only_bn` / `only_splits` restricts the search to that value (and a forced
+// split may leave a CTA fewer than two stages).  Ties go to the wider tile and then to
+// fewer splits; bn = 0 when nothing is feasible.
+struct GemmChoiceModel {
+  int bn, splits;
+  double t_us;
+};
+
+template <typename SlotsFn>
+constexpr GemmChoiceModel gemm_choose(long long M, long long N, long long K, int num_sms, SlotsFn slots,
+                                      const ArchDesc& a = kGb300, int only_bn = 0, int only_splits = 0) {
+  GemmChoiceModel best{0, 0, 1e300};
+  for (int bn = 256; bn >= 64; bn -= 64) {
+    if (only_bn != 0 && bn != only_bn) continue;
+    const GemmPlan p = gemm_plan_variant(bn, a);
+    if (!p.feasible) continue;
+    for (int S = 1; S <= kGemmMaxSplits; S *= 2) {
+      if (only_splits != 0 && S != only_splits) continue;
+      double t;
+      if (S == 1) {
+        t = gemm_time_us(p, M, N, K, num_sms, a);
+      } else {
+        if (only_splits == 0 && cdiv(K, p.bk) < 2LL * S) break;  // every CTA takes two stages or more
+        const int s = slots(bn, S);
+        if (s <= 0) continue;
+        t = gemm_splitk_time_us(p, M, N, K, S, s, a);
+      }
+      if (t < best.t_us * (1.0 - 1e-9)) best = {bn, S, t};
+    }
+  }
+  return best;
+}
+
+// Cluster slots when nothing better is known: whole clusters of S on `num_sms` SMs with the
+// GPU's SMs in 8 groups (GPCs) of equal size; a cluster never spans two groups.
+constexpr int gemm_default_slots(int num_sms, int S) {
+  const int per_gpc = num_sms / 8;
+  return (per_gpc / S) * S * 8;
+}
+
+}  // namespace model
+}  // namespace loom

@@ -46,17 +46,7 @@ inline size_t decode_workspace_bytes(int B, int Hq, int D, int splits) {
   return ((opart + 255) / 256) * 256 + ((lpart + 255) / 256) * 256;
 }
 
-struct GemmArgs {
-  const void* a;  // [M, K] bf16 row-major
-  const void* b;  // [K, N] bf16 row-major
-  void* c;        // [M, N] bf16 row-major
-  int M, N, K;
-  int tile_n;     // 0: the analytic model's choice, else 64, 128, 192 or 256
-};
-
 cudaError_t launch_decode(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream);
-cudaError_t launch_gemm(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream);
-int gemm_tile_n(int M, int N, int K, int sms);
 cudaError_t launch_fwd(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream);
 
 }  // namespace loom

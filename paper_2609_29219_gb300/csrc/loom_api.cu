@@ -9,6 +9,8 @@
 #include <vector>
 
 #include "../../include/loom_attn.h"
+#include "gemm.h"
+#include "gemm_model.h"
 #include "kernels.h"
 #include "model.h"
 
@@ -22,6 +24,7 @@ uint64_t g_timeout_ns = kDefaultTimeoutNs;
 int g_inject = 0;
 int g_prefill_design = 0;
 int g_gemm_tile_n = 0;  // test hook: forced GEMM tile width (0: the model's choice)
+int g_gemm_splits = 0;  // test hook: forced GEMM split count (0: the model's choice)
 
 constexpr int kMaxDevices = 64;
 uint32_t* g_err_ptr[kMaxDevices] = {};
@@ -176,27 +179,50 @@ loom_status loom_gemm_bf16(const void* a, const void* b, void* c, int M, int N, 
   if (K % 8 != 0 || N % 8 != 0) return LOOM_ERR_UNSUPPORTED;  // 16-byte row strides for TMA
   KernelCtl ctl;
   if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
-  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n};
+  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n, g_gemm_splits};
   return launch_gemm(g, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK : LOOM_ERR_CUDA;
 }
 
+namespace {
+// The model's GEMM choice: with the device's cluster occupancy when a device answers, else
+// with the estimate of whole clusters in 8 equal SM groups of a GB300.
+GemmChoice gemm_choice_any(int M, int N, int K, GemmChoice forced) {
+  const GemmChoice c = gemm_choice(M, N, K, forced);
+  if (c.tile_n != 0) return c;
+  cudaGetLastError();
+  const int sms = model::kGb300.num_sms;
+  const model::GemmChoiceModel m = model::gemm_choose(
+      M, N, K, sms, [sms](int, int S) { return model::gemm_default_slots(sms, S); }, model::kGb300,
+      forced.tile_n, forced.splits);
+  return {m.bn, m.splits};
+}
+}  // namespace
+
 int loom_gemm_tile_n(int M, int N, int K) {
   if (M <= 0 || N <= 0 || K <= 0) return 0;
-  int sms = current_sm_count();
-  if (sms <= 0) sms = model::kGb300.num_sms;
-  return gemm_tile_n(M, N, K, sms);
+  return gemm_choice_any(M, N, K, {g_gemm_tile_n, g_gemm_splits}).tile_n;
 }
 
-double loom_model_gemm_time_us(int M, int N, int K, int tile_n, int num_sms) {
+int loom_gemm_splits(int M, int N, int K) {
+  if (M <= 0 || N <= 0 || K <= 0) return 0;
+  return gemm_choice_any(M, N, K, {g_gemm_tile_n, g_gemm_splits}).splits;
+}
+
+double loom_model_gemm_time_us(int M, int N, int K, int tile_n, int splits, int num_sms) {
   if (M <= 0 || N <= 0 || K <= 0 || num_sms <= 0) return -1.0;
+  if (tile_n != 64 && tile_n != 128 && tile_n != 192 && tile_n != 256) return -1.0;
+  if (!model::gemm_split_supported(splits)) return -1.0;
   const model::GemmPlan p = model::gemm_plan_variant(tile_n);
-  if (!p.feasible || (tile_n != 64 && tile_n != 128 && tile_n != 192 && tile_n != 256)) return -1.0;
-  return model::gemm_time_us(p, M, N, K, num_sms);
+  if (!p.feasible) return -1.0;
+  if (splits == 1) return model::gemm_time_us(p, M, N, K, num_sms);
+  return model::gemm_splitk_time_us(p, M, N, K, splits, model::gemm_default_slots(num_sms, splits));
 }
 
 void loom_debug_gemm_tile_n(int tile_n) {
   g_gemm_tile_n = (tile_n == 64 || tile_n == 128 || tile_n == 192 || tile_n == 256) ? tile_n : 0;
 }
+
+void loom_debug_gemm_splits(int splits) { g_gemm_splits = model::gemm_split_supported(splits) ? splits : 0; }
 
 loom_status loom_attn_check_error(void* stream) {
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return LOOM_ERR_CUDA;

@@ -242,78 +242,6 @@ constexpr double fwd_time_us(const FwdPlan& p, int B, int Hq, int Sq, int Skv, i
   return w * t_cta * 1e-3;
 }
 
-// ------------------------------------------------------------------ GEMM (C = A B)
-// The paper's third kernel.  A CTA computes BM = 128 rows x BN columns of C at a time,
-// with K in BK = 64 stages through an NSTAGE ring (Eq. 6 with the load boundary open)
-// and the accumulator double-buffered in TMEM, so that one tile's epilogue overlaps the
-// next tile's MMAs.  Candidates: BN in {64, 128, 192, 256} x ring depth.
-struct GemmPlan {
-  int bm, bn, bk, stages, smem_bytes, tmem_cols;
-  double t_load_ns, t_mma_ns, t_iter_ns, t_epi_ns;
-  bool feasible;
-};
-
-constexpr int kGemmStagingBytes = 4 * 2 * 32 * 128;  // 4 epilogue warps x 2 buffers x 32 rows x 128 B
-
-constexpr GemmPlan gemm_eval(const ArchDesc& a, int bn, int stages) {
-  GemmPlan p{};
-  p.bm = 128;
-  p.bn = bn;
-  p.bk = 64;
-  p.stages = stages;
-  const double stage_bytes = (p.bm + bn) * p.bk * 2.0;
-  p.t_load_ns = stage_bytes / a.l2_smem_gbs_sm;  // A and B tiles from L2
-  p.t_mma_ns = (p.bk / 16.0) * dmax(a.mma_clk_per_n * bn, a.mma_min_clk) / a.sm_ghz;
-  p.t_iter_ns = heg_pipe(p.t_load_ns, p.t_mma_ns, 0.0, 1, 0);
-  p.t_epi_ns = p.bm * bn * 2.0 / a.l2_smem_gbs_sm;  // the C tile leaves through L2
-  p.smem_bytes = static_cast<int>(stages * stage_bytes) + kGemmStagingBytes + 1024 + 256;
-  p.tmem_cols = 2 * bn;
-  p.feasible = p.smem_bytes <= a.smem_per_cta && p.tmem_cols <= a.tmem_cols && stages >= 2 && bn % 64 == 0 &&
-               bn >= 64 && bn <= 256 && (stages - 1) * p.t_iter_ns >= a.mem_latency_ns * 0.5;
-  return p;
-}
-
-// Eq. 8 for one tile width: the ring depth with the lowest modeled iteration, ties to the
-// deeper ring.
-constexpr GemmPlan gemm_plan_variant(int bn, const ArchDesc& a = kGb300) {
-  GemmPlan best{};
-  best.feasible = false;
-  for (int stages = 2; stages <= 12; ++stages) {
-    const GemmPlan p = gemm_eval(a, bn, stages);
-    if (!p.feasible) continue;
-    if (!best.feasible || p.t_iter_ns < best.t_iter_ns * (1.0 - 1e-9) ||
-        (p.t_iter_ns <= best.t_iter_ns * (1.0 + 1e-9) && p.stages > best.stages))
-      best = p;
-  }
-  return best;
-}
-
-// Eq. 5-7 for a whole launch: the busiest SM runs ceil(tiles / SMs) tiles of ceil(K / BK)
-// iterations back to back; the first load and the last epilogue are exposed.
-constexpr double gemm_time_us(const GemmPlan& p, long long M, long long N, long long K, int num_sms,
-                              const ArchDesc& a = kGb300) {
-  const long long tiles = cdiv(M, p.bm) * cdiv(N, p.bn);
-  const long long per_sm = cdiv(tiles, num_sms);
-  const double t = heg_seq(heg_seq(p.t_load_ns, heg_for(per_sm * cdiv(K, p.bk), p.t_iter_ns)), p.t_epi_ns);
-  return (t + a.launch_ns * 0.2) * 1e-3;
-}
-
-// Eq. 9: the tile width with the lowest modeled launch time (ties to the wider tile).
-constexpr int gemm_choose_bn(long long M, long long N, long long K, int num_sms, const ArchDesc& a = kGb300) {
-  int best_bn = 0;
-  double best_t = 1e300;
-  for (int bn = 256; bn >= 64; bn -= 64) {
-    const GemmPlan p = gemm_plan_variant(bn, a);
-    if (!p.feasible) continue;
-    const double t = gemm_time_us(p, M, N, K, num_sms, a);
-    if (t < best_t * (1.0 - 1e-9)) {
-      best_t = t;
-      best_bn = bn;
-    }
-  }
-  return best_bn;
-}
-
 // ------------------------------------------------------------------ decode
 // Stage plan of the split kernel: T keys per stage, NSTAGE ring depth, CTAs per SM.
 struct DecodeStagePlan {

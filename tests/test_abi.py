@@ -112,7 +112,23 @@ def test_gemm_rejects_bad_arguments(lib):
     assert lib.loom_gemm_bf16(FAKE, FAKE, FAKE, 8, 20, 8, None) == 2  # UNSUPPORTED: N % 8
 
 
-def test_gemm_tile_choice_is_a_supported_width(lib):
-    for M, N, K in [(1, 8, 8), (128, 256, 64), (4096, 4096, 4096), (8192, 1024, 8192)]:
+def test_gemm_choice_is_supported(lib):
+    for M, N, K in [(1, 8, 8), (128, 256, 64), (4096, 4096, 4096), (8192, 1024, 8192), (256, 256, 16384)]:
         assert lib.loom_gemm_tile_n(M, N, K) in (64, 128, 192, 256)
+        assert lib.loom_gemm_splits(M, N, K) in (1, 2, 4, 8, 16)
     assert lib.loom_gemm_tile_n(0, 8, 8) == 0
+    assert lib.loom_gemm_splits(8, 0, 8) == 0
+
+
+def test_gemm_splits_only_when_tiles_are_few(lib):
+    # few C tiles and a long K: the model splits K over clusters
+    assert lib.loom_gemm_splits(256, 256, 16384) > 1
+    assert lib.loom_gemm_splits(256, 2048, 16384) > 1
+    # enough tiles for every SM, or a single K stage: no split
+    assert lib.loom_gemm_splits(16384, 16384, 16384) == 1
+    assert lib.loom_gemm_splits(256, 256, 64) == 1
+    t1 = lib.loom_model_gemm_time_us(256, 256, 16384, 64, 1, 152)
+    t8 = lib.loom_model_gemm_time_us(256, 256, 16384, 64, 8, 152)
+    assert 0 < t8 < t1
+    assert lib.loom_model_gemm_time_us(256, 256, 16384, 64, 3, 152) < 0  # unsupported split
+    assert lib.loom_model_gemm_time_us(256, 256, 16384, 96, 1, 152) < 0  # unsupported width

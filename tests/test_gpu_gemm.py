@@ -2,7 +2,8 @@
 
 Bound: C is rounded to bf16 once (at most 2^-9 relative error, written here as 2^-8 for
 margin), and the fp32 accumulation over K adds at most ~K * 2^-24 * sum_k |a_ik b_kj|,
-which for N(0,1) inputs stays below 1e-6 * K in absolute terms at these sizes."""
+which for N(0,1) inputs stays below 1e-6 * K in absolute terms at these sizes.  The same
+bound holds for every split count: the split only regroups the fp32 sum."""
 import numpy as np
 import pytest
 
@@ -11,6 +12,9 @@ import synth
 from tests.gpu_util import to_dev
 
 pytestmark = pytest.mark.gpu
+
+TILE_WIDTHS = (64, 128, 192, 256)
+SPLITS = (2, 4, 8, 16)
 
 
 @pytest.fixture(scope="module")
@@ -21,14 +25,23 @@ def loom():
     import __graft_entry__
     __graft_entry__.build()
     import paper_2609_29219_gb300 as m
-    return m
+    yield m
+    m.loom_debug_gemm_tile_n(0)
+    m.loom_debug_gemm_splits(0)
+    m.loom_debug_inject(0)
+    m.loom_debug_set_timeout_ns(0)
 
 
-@pytest.fixture(autouse=True, params=[0, 64, 128, 192, 256], ids=["model", "bn64", "bn128", "bn192", "bn256"])
-def tile_n(request, loom):
-    loom.loom_debug_gemm_tile_n(request.param)
-    yield request.param
+@pytest.fixture
+def forced(loom):
+    """forced(tile_n, splits): pin the kernel variant for one test (0 = the model's choice)."""
+    def set_(tile_n=0, splits=0):
+        loom.loom_debug_gemm_tile_n(tile_n)
+        loom.loom_debug_gemm_splits(splits)
+        assert tile_n == 0 or loom.loom_gemm_tile_n(8, 8, 8) == tile_n
+    yield set_
     loom.loom_debug_gemm_tile_n(0)
+    loom.loom_debug_gemm_splits(0)
 
 
 def _inputs(seed, M, K, N):
@@ -36,48 +49,102 @@ def _inputs(seed, M, K, N):
 
 
 def _check(c_gpu, c_ref, K, what):
+    assert np.all(np.isfinite(c_gpu)), f"{what}: non-finite output"
     diff = np.abs(c_gpu - c_ref)
     bound = 2.0 ** -8 * np.abs(c_ref) + 1e-6 * K + 1e-6
     worst = np.max(diff - bound)
     assert worst <= 0, f"{what}: max excess {worst:.3g} (max |diff| {diff.max():.3g})"
 
 
-def _run(loom, a, b):
-    import torch
-    c = loom.loom_gemm_bf16(to_dev(a), to_dev(b))
+def _run_dev(loom, ad, bd):
+    c = loom.loom_gemm_bf16(ad, bd)
     loom.loom_attn_check_error()
-    return c.float().cpu().numpy().astype(np.float64)
+    return c
 
 
+def _run(loom, a, b):
+    return _run_dev(loom, to_dev(a), to_dev(b)).float().cpu().numpy().astype(np.float64)
+
+
+# ---------------------------------------------------------------- persistent tiles (S = 1)
+@pytest.mark.parametrize("tile_n", [0, *TILE_WIDTHS], ids=["model", *[f"bn{b}" for b in TILE_WIDTHS]])
 @pytest.mark.parametrize("M,K,N", [(128, 64, 256), (1, 8, 8), (200, 136, 304), (130, 72, 264), (255, 1000, 520),
                                    (1000, 1000, 1000), (64, 4096, 64), (2048, 256, 256)])
-def test_full_parity(loom, M, K, N):
+def test_full_parity(loom, forced, tile_n, M, K, N):
+    forced(tile_n, 1 if tile_n else 0)
     a, b = _inputs(M + K + N, M, K, N)
-    _check(_run(loom, a, b), oracle.gemm(a, b), K, f"{M}x{K}x{N}")
+    _check(_run(loom, a, b), oracle.gemm(a, b), K, f"{M}x{K}x{N} bn={tile_n}")
 
 
+@pytest.mark.parametrize("tile_n", [0, 64, 256], ids=["model", "bn64", "bn256"])
 @pytest.mark.parametrize("M,K,N", [(4096, 4096, 4096), (8192, 2048, 1024)])
-def test_large_sampled_rows(loom, M, K, N):
+def test_large_sampled_rows(loom, forced, tile_n, M, K, N):
+    forced(tile_n, 1 if tile_n else 0)
     a, b = _inputs(7, M, K, N)
     c = _run(loom, a, b)
     rng = np.random.default_rng(0)
     rows = np.unique(np.concatenate([[0, 127, 128, M - 1], rng.integers(0, M, 60)]))
-    _check(c[rows], oracle.gemm(a, b, rows=rows), K, f"{M}x{K}x{N} sampled")
+    _check(c[rows], oracle.gemm(a, b, rows=rows), K, f"{M}x{K}x{N} sampled bn={tile_n}")
 
 
-def test_identity_and_zeros(loom):
+# ---------------------------------------------------------------- split-K clusters
+@pytest.mark.parametrize("splits", SPLITS, ids=[f"s{s}" for s in SPLITS])
+@pytest.mark.parametrize("tile_n", TILE_WIDTHS, ids=[f"bn{b}" for b in TILE_WIDTHS])
+@pytest.mark.parametrize("M,K,N", [(128, 1024, 256), (200, 1000, 304), (130, 4096, 520), (384, 2048, 1000)])
+def test_split_parity(loom, forced, tile_n, splits, M, K, N):
+    forced(tile_n, splits)
+    a, b = _inputs(3 * M + K + N, M, K, N)
+    _check(_run(loom, a, b), oracle.gemm(a, b), K, f"{M}x{K}x{N} bn={tile_n} S={splits}")
+
+
+@pytest.mark.parametrize("splits", SPLITS, ids=[f"s{s}" for s in SPLITS])
+def test_split_with_idle_ctas(loom, forced, splits):
+    """K = 64 is one stage: all but one CTA of each cluster get no stage and add zeros."""
+    forced(64, splits)
+    M, K, N = 256, 64, 192
+    a, b = _inputs(5, M, K, N)
+    _check(_run(loom, a, b), oracle.gemm(a, b), K, f"idle CTAs S={splits}")
+
+
+@pytest.mark.parametrize("M,K,N", [(256, 16384, 256), (256, 16384, 2048), (2048, 2048, 256)])
+def test_model_choice_long_k(loom, forced, M, K, N):
+    """Shapes with few tiles and long K, on whatever (tile width, split) the model picks."""
+    forced(0, 0)
+    a, b = _inputs(9, M, K, N)
+    c = _run(loom, a, b)
+    rows = np.unique(np.concatenate([[0, 1, 127, 128, M - 1], np.random.default_rng(1).integers(0, M, 40)]))
+    _check(c[rows], oracle.gemm(a, b, rows=rows), K,
+           f"{M}x{K}x{N} model bn={loom.loom_gemm_tile_n(M, N, K)} S={loom.loom_gemm_splits(M, N, K)}")
+
+
+@pytest.mark.parametrize("splits", [1, 4, 16])
+def test_deterministic(loom, forced, splits):
+    forced(128, splits)
+    a, b = _inputs(13, 384, 4096, 512)
+    ad, bd = to_dev(a), to_dev(b)
+    import torch
+    x1 = _run_dev(loom, ad, bd).view(torch.int16).cpu().numpy()
+    x2 = _run_dev(loom, ad, bd).view(torch.int16).cpu().numpy()
+    np.testing.assert_array_equal(x1, x2)
+
+
+def test_identity_and_zeros(loom, forced):
     K, N = 256, 512
     eye = np.zeros((K, K), np.uint16)
     eye[np.arange(K), np.arange(K)] = 0x3F80
     b = synth.bf16_normal(3, synth.STREAM_V, (K, N))
-    np.testing.assert_array_equal(_run(loom, eye, b), oracle.bf16_to_f64(b))  # exact: one product per entry
-    z = np.zeros((K, N), np.uint16)
-    np.testing.assert_array_equal(_run(loom, eye, z), 0.0)
+    for tile_n, splits in [(0, 0), (64, 2), (256, 4)]:
+        forced(tile_n, splits)
+        np.testing.assert_array_equal(_run(loom, eye, b), oracle.bf16_to_f64(b))  # one product per entry
+        np.testing.assert_array_equal(_run(loom, eye, np.zeros((K, N), np.uint16)), 0.0)
 
 
-def test_timeout_is_reported_and_context_survives(loom, tile_n):
-    if tile_n not in (0, 256):
-        pytest.skip("one tile width is enough")
+# ---------------------------------------------------------------- bounded waits
+@pytest.mark.parametrize("tile_n,splits", [(256, 1), (64, 4)])
+def test_timeout_is_reported_and_context_survives(loom, forced, tile_n, splits):
+    """The loader skips one stage (per CTA); the waits on it run out, every CTA (and, split,
+    every cluster) unwinds, the error word says TIMEOUT, and the next call is correct."""
+    forced(tile_n, splits)
     M, K, N = 256, 1024, 512
     a, b = _inputs(11, M, K, N)
     ad, bd = to_dev(a), to_dev(b)
@@ -92,6 +159,5 @@ def test_timeout_is_reported_and_context_survives(loom, tile_n):
     finally:
         loom.loom_debug_inject(0)
         loom.loom_debug_set_timeout_ns(0)
-    c = loom.loom_gemm_bf16(ad, bd)
-    loom.loom_attn_check_error()
+    c = _run_dev(loom, ad, bd)
     _check(c.float().cpu().numpy().astype(np.float64), oracle.gemm(a, b), K, "after timeout")
