@@ -6,7 +6,8 @@ with the CUDA library; the only common dependency is the seeded input generator
 (``synth``), which holds no attention arithmetic.
 
 Arrays are numpy: Q [B, Hq, Sq, D], K/V [B, Hkv, Skv, D] (and the GEMM operands A [M, K],
-B [K, N]) as uint16 bfloat16 bit patterns, results in float64.
+B [K, N]; a paged KV cache [num_pages, page_size, Hkv, D]; packed ragged batches
+[total_tokens, H, D]) as uint16 bfloat16 bit patterns, results in float64.
 """
 from __future__ import annotations
 
@@ -179,3 +180,38 @@ def gemm(a, b, *, rows=None):
     if rows is not None:
         A = A[np.asarray(rows, dtype=np.int64)]
     return A @ Bm
+
+
+def paged_gather(cache, block_table, seqlens, page_size):
+    """The logical K (or V) [B, Hkv, Skv_max, D] of a paged cache [num_pages, page_size,
+    Hkv, D]: key t of sequence b is row t mod page_size of physical page
+    block_table[b, t div page_size] (the usual paged-KV convention; the paper has none).
+    Skv_max = block_table.shape[1] * page_size; positions at or past seqlens[b] are left
+    zero, and their table entries are not read (they may be anything)."""
+    cache = _u16(cache)
+    table = np.asarray(block_table, dtype=np.int64)
+    lens = np.asarray(seqlens, dtype=np.int64)
+    npages, P, Hkv, D = cache.shape
+    if P != page_size:
+        raise ValueError("cache rows per page != page_size")
+    B, max_pages = table.shape
+    out = np.zeros((B, Hkv, max_pages * P, D), dtype=np.uint16)
+    for b in range(B):
+        n = int(min(max(lens[b], 0), max_pages * P))
+        for j in range((n + P - 1) // P):
+            page = int(table[b, j])
+            if not 0 <= page < npages:
+                raise ValueError(f"block_table[{b}, {j}] = {page} is not a page of the cache")
+            r = min(P, n - j * P)
+            out[b, :, j * P:j * P + r, :] = cache[page, :r].transpose(1, 0, 2)
+    return out
+
+
+def decode_paged(q, k_cache, v_cache, block_table, seqlens, *, page_size, scale=None, nthreads=0):
+    """Decode (one query row per head) over a paged KV cache: the attention definition on
+    the logical K/V that ``paged_gather`` assembles.  q [B, Hq, 1, D].  Returns
+    ``(o [B, Hq, D], lse [B, Hq])``."""
+    k = paged_gather(k_cache, block_table, seqlens, page_size)
+    v = paged_gather(v_cache, block_table, seqlens, page_size)
+    o, lse = attention(q, k, v, scale=scale, seqlens_k=np.asarray(seqlens, dtype=np.int32), nthreads=nthreads)
+    return o[:, :, 0, :], lse[:, :, 0]
