@@ -288,6 +288,49 @@ class Decode:
         return self.bytes / seconds_per_step / 1e9
 
 
+class PagedDecode(Decode):
+    """The batched decode over a paged cache [num_pages, page_size, Hkv, D]: each sequence's
+    pages are dealt in a seeded shuffled order across the cache (a cache that has served
+    many requests), so consecutive logical pages are scattered in HBM."""
+
+    def __init__(self, name, B, Hq, Hkv, Skv, D, splits, page_size, lengths, seed=0, sets=2):
+        super().__init__(name, B, Hq, Hkv, Skv, D, splits, lengths=lengths, seed=seed, sets=sets)
+        self.P = page_size
+
+    def describe(self):
+        return super().describe().replace("decode ", f"paged decode page_size={self.P} ", 1)
+
+    def paged(self, k, v, s):
+        B, Hkv, S, D, P = self.B, self.Hkv, self.Skv, self.D, self.P
+        npg = S // P
+        order = np.random.default_rng(self.seed + s).permutation(B * npg).astype(np.int32)
+        kc = np.empty((B * npg, P, Hkv, D), np.uint16)
+        vc = np.empty_like(kc)
+        kc[order] = k.reshape(B, Hkv, npg, P, D).transpose(0, 2, 3, 1, 4).reshape(B * npg, P, Hkv, D)
+        vc[order] = v.reshape(B, Hkv, npg, P, D).transpose(0, 2, 3, 1, 4).reshape(B * npg, P, Hkv, D)
+        return kc, vc, order.reshape(B, npg)
+
+    def setup(self, torch, dev, loom):
+        self.loom = loom
+        self.inp = []
+        self.sl = torch.from_numpy(self.lens).to(dev)
+        nbytes = loom.loom_attn_decode_workspace_bytes(self.B, self.Hq, self.Hkv, self.Skv, self.D, self.splits)
+        self.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        self.used_splits = self.splits or loom.loom_attn_decode_num_splits(self.B, self.Hq, self.Hkv, self.Skv, self.D)
+        for s in range(self.sets):
+            q, k, v = self.host_inputs(s)
+            kc, vc, table = self.paged(k, v, s)
+            q = to_tensor(torch, q, dev)
+            self.inp.append((q, to_tensor(torch, kc, dev), to_tensor(torch, vc, dev),
+                             torch.from_numpy(np.ascontiguousarray(table)).to(dev), torch.empty_like(q),
+                             torch.empty((self.B, self.Hq), dtype=torch.float32, device=dev)))
+
+    def step(self, i, stream):
+        q, kc, vc, table, o, lse = self.inp[i % self.sets]
+        self.loom.loom_attn_decode_paged(q, kc, vc, table, self.sl, o, lse, self.ws, num_splits=self.splits,
+                                         stream=stream)
+
+
 class Gemm:
     """C = A B in bf16 with fp32 accumulation (the paper's GEMM, Sec. 4); A, B seeded N(0, 1)
     drawn on the device.  `cublas` times torch.matmul (cuBLAS) on the same buffers."""
@@ -486,7 +529,8 @@ def main():
                          "against cuBLAS, every tile width measured (one JSON line per point)")
     ap.add_argument("--ncu-case", default=None,
                     help="profiling run: set up this workload (tiny, tiny_causal, prefill, prefill_causal, "
-                         "long_prefill_d128, long_prefill_d64, batched_decode, long_decode, gemm_4096, "
+                         "long_prefill_d128, long_prefill_d64, batched_decode, paged_decode_p16, paged_decode_p64, long_decode, "
+                         "gemm_4096, "
                          "gemm_16k_256_16k), run --steps launches, print nothing")
     args = ap.parse_args()
     world, rank, local = dist_env()
@@ -539,6 +583,8 @@ def main():
             Prefill("long_prefill_d128", 1, 32, 8, 8192, 128, causal=True),
             Prefill("long_prefill_d64", 1, 64, 16, 8192, 64, causal=True),
             Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
+            PagedDecode("paged_decode_p16", 16, 32, 8, 8192, 128, splits=16, page_size=16, lengths=lens),
+            PagedDecode("paged_decode_p64", 16, 32, 8, 8192, 128, splits=16, page_size=64, lengths=lens),
             Decode("long_decode", 1, 32, 8, 131072, 128, splits=0),
         ]
         if args.only:
@@ -745,6 +791,8 @@ def all_workloads():
             Prefill("long_prefill_d128", 1, 32, 8, 8192, 128, causal=True),
             Prefill("long_prefill_d64", 1, 64, 16, 8192, 64, causal=True),
             Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
+            PagedDecode("paged_decode_p16", 16, 32, 8, 8192, 128, splits=16, page_size=16, lengths=lens),
+            PagedDecode("paged_decode_p64", 16, 32, 8, 8192, 128, splits=16, page_size=64, lengths=lens),
             Decode("long_decode", 1, 32, 8, 131072, 128, splits=0)]
 
 

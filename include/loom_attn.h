@@ -100,6 +100,33 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
                              float scale, int num_splits, void* stream);
 
 /*
+ * Flash Decode over a paged KV cache (the layout of paged serving engines; the paper has
+ * no counterpart -- it belongs to the irregular grids its Sec. 2.6 scope note sets aside).
+ *   q            [B, Hq, 1, D]                     bf16, read
+ *   k_cache,
+ *   v_cache      [num_pages, page_size, Hkv, D]    bf16, read; a page holds page_size
+ *                consecutive keys of one sequence, with the rows of all kv heads adjacent
+ *   block_table  [B, max_pages] int32 on the device: key t of sequence b is row
+ *                t % page_size of page block_table[b * max_pages + t / page_size].  Only
+ *                the first ceil(len_b / page_size) entries of a row are read; an entry
+ *                outside [0, num_pages) reads zeros (no fault).
+ *   seqlens_k    [B] int32 on the device (required): 0 .. max_pages * page_size, clamped
+ *   o, lse, workspace, num_splits, scale: as loom_attn_decode, with Skv = max_pages *
+ *                page_size in loom_attn_decode_workspace_bytes / loom_attn_decode_num_splits.
+ * page_size: 8, 16, 32 or a multiple of 64.  The split rule and results are those of
+ * loom_attn_decode on the gathered (logical) cache.
+ * Errors: INVALID_ARG (NULL q/k/v/o/block_table/seqlens_k, a size <= 0, Hq % Hkv, scale),
+ * UNSUPPORTED (D, page_size, more than 2^31 - 1 keys in the cache or per sequence, too many
+ * splits), MISALIGNED (q, caches, o, workspace not 16-byte aligned; block_table, seqlens_k,
+ * lse not 4-byte aligned), WORKSPACE, CUDA.
+ */
+loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const void* v_cache,
+                                   const int32_t* block_table, const int32_t* seqlens_k, void* o,
+                                   float* lse, void* workspace, size_t workspace_bytes, int B, int Hq,
+                                   int Hkv, int num_pages, int page_size, int max_pages, int D,
+                                   float scale, int num_splits, void* stream);
+
+/*
  * Flash Decode without any allocation and without a workspace argument.  The paper has
  * no counterpart; this entry point exists for callers that cannot obtain device scratch
  * memory for a call -- serving engines that reserve all device memory at start-up and

@@ -26,7 +26,7 @@ __all__ = [
     "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
     "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
     "loom_model_fwd_plan_variant", "loom_model_heg_pipe", "loom_model_fwd_time_us_design",
-    "loom_gemm_bf16", "loom_gemm_tile_n", "loom_gemm_splits", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
+    "loom_attn_decode_paged", "loom_gemm_bf16", "loom_gemm_tile_n", "loom_gemm_splits", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
     "loom_debug_gemm_splits",
 ]
 
@@ -101,6 +101,9 @@ def capi() -> ctypes.CDLL:
             lib.loom_model_fwd_time_us.restype = ctypes.c_double
             lib.loom_model_fwd_time_us_design.argtypes = [i32] * 7
             lib.loom_model_fwd_time_us_design.restype = ctypes.c_double
+            lib.loom_attn_decode_paged.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, sz, i32, i32, i32, i32,
+                                                   i32, i32, i32, f32, i32, vp]
+            lib.loom_attn_decode_paged.restype = i32
             lib.loom_gemm_bf16.argtypes = [vp, vp, vp, i32, i32, i32, vp]
             lib.loom_gemm_bf16.restype = i32
             lib.loom_gemm_tile_n.argtypes = [i32, i32, i32]
@@ -238,6 +241,51 @@ def loom_attn_decode(q, k_cache, v_cache, seqlens_k=None, o=None, lse=None, work
                                  B, Hq, Hkv, Skv, D, float(scale), int(num_splits),
                                  _stream_ptr(stream, q.device))
     _check(st, "loom_attn_decode")
+    return (o, lse) if (return_lse or lse is not None) else o
+
+
+def loom_attn_decode_paged(q, k_cache, v_cache, block_table, seqlens_k, o=None, lse=None, workspace=None, *,
+                           scale=None, num_splits=0, stream=None, return_lse=False):
+    """Flash Decode over a paged cache.  q [B,Hq,1,D]; k_cache/v_cache [num_pages, page_size,
+    Hkv, D] bf16; block_table [B, max_pages] int32; seqlens_k [B] int32 (all on the device).
+    Returns ``o`` or ``(o, lse)``."""
+    torch = _torch()
+    bf16 = torch.bfloat16
+    qp = _dev_ptr(q, "q", bf16, 4)
+    kp = _dev_ptr(k_cache, "k_cache", bf16, 4)
+    vp_ = _dev_ptr(v_cache, "v_cache", bf16, 4)
+    B, Hq, Sq, D = q.shape
+    num_pages, page_size, Hkv, Dk = k_cache.shape
+    if Sq != 1 or tuple(v_cache.shape) != tuple(k_cache.shape) or Dk != D:
+        raise ValueError("paged decode takes q [B,Hq,1,D] and caches [num_pages, page_size, Hkv, D]")
+    if block_table.dim() != 2 or block_table.shape[0] != B:
+        raise ValueError("block_table must be [B, max_pages]")
+    max_pages = block_table.shape[1]
+    tp = _dev_ptr(block_table, "block_table", torch.int32, 2)
+    if tuple(seqlens_k.shape) != (B,):
+        raise ValueError("seqlens_k must be [B]")
+    sp = _dev_ptr(seqlens_k, "seqlens_k", torch.int32)
+    if o is None:
+        o = torch.empty_like(q)
+    op = _dev_ptr(o, "o", bf16, 4)
+    if lse is None and return_lse:
+        lse = torch.empty((B, Hq), dtype=torch.float32, device=q.device)
+    lp = None
+    if lse is not None:
+        if lse.numel() != B * Hq:
+            raise ValueError("lse must hold B*Hq values")
+        lp = _dev_ptr(lse, "lse", torch.float32)
+    Skv = max_pages * page_size
+    if workspace is None:
+        need = loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, num_splits)
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=q.device)
+    wp = _dev_ptr(workspace, "workspace")
+    if scale is None:
+        scale = D ** -0.5
+    st = capi().loom_attn_decode_paged(qp, kp, vp_, tp, sp, op, lp, wp, workspace.numel() * workspace.element_size(),
+                                       B, Hq, Hkv, num_pages, page_size, max_pages, D, float(scale),
+                                       int(num_splits), _stream_ptr(stream, q.device))
+    _check(st, "loom_attn_decode_paged")
     return (o, lse) if (return_lse or lse is not None) else o
 
 

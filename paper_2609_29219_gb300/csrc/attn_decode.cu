@@ -8,6 +8,9 @@
 //   * a loader warp streams the split's K and V rows with 1-D bulk copies
 //     (cp.async.bulk, 16 KB per tile) into an NSTAGE-deep shared-memory ring guarded by
 //     full/empty mbarriers, so that 2 CTAs x 3 stages x 32 KB are in flight per SM;
+//     with a paged cache it reads the sequence's block table 32 entries at a time (one
+//     per lane) and lane j copies the stage's j-th page piece with a 3-D TMA load of
+//     the cache viewed as [keys of all pages, Hkv, D];
 //   * 8 compute warps each take T/8 tokens of every stage; they read K rows with
 //     128-bit shared loads, form the scores of all GT query heads of the kv head at
 //     once (fp32 FMA), reduce them across lanes with a transposing butterfly, run an
@@ -18,12 +21,16 @@
 //   w_i = exp(lse_i - L), O = sum w_i O_i / sum w_i -> bf16, lse = L + ln sum w_i.
 //   It is launched with programmatic dependent launch so its launch overlaps the
 //   split kernel's tail.
+#include <cuda.h>
 #include <cuda_bf16.h>
 
 #include <cmath>
+#include <cstring>
+#include <mutex>
 
 #include "kernels.h"
 #include "model.h"
+#include "paged.h"
 #include "ptx.cuh"
 
 namespace loom {
@@ -107,12 +114,21 @@ __device__ __forceinline__ int head_of_lane(int lane) {
   return h;
 }
 
-template <int D, int GT>
+// Where a paged split kernel finds its keys (unused by the contiguous instantiation).
+struct PagedView {
+  const int32_t* block_table;
+  int page_size, max_pages;
+  int num_keys;  // num_pages * page_size (< 2^31)
+};
+
+template <int D, int GT, bool PAGED>
 __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_SM)
     decode_split_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
                         const __nv_bfloat16* __restrict__ v, const int32_t* __restrict__ seqlens,
                         float* __restrict__ o_part, float* __restrict__ lse_part, int Hq, int Hkv,
-                        int Skv, int splits, int n_groups, float c, KernelCtl ctl) {
+                        int Skv, int splits, int n_groups, float c, KernelCtl ctl,
+                        const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                        PagedView pv) {
   using C = DecodeCfg<D>;
   using L = DecodeSmem<D, GT>;
   extern __shared__ __align__(128) uint8_t smem[];
@@ -162,7 +178,57 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
 
   if (warp == C::NCW) {
     // ------------------------------------------------------------ loader warp
-    if (lane == 0) {
+    if constexpr (PAGED) {
+      static_assert(C::T % kDecodeChunkAlign == 0, "stages start on a copy boundary");
+      // Copies of `rows` keys: a 64-key piece of one page (page_size a multiple of 64) or
+      // one whole page (page_size 8, 16 or 32).  Stages start on a multiple of 64 keys, so
+      // no copy crosses a page; a stage takes at most T / 8 copies.
+      const int P = pv.page_size;
+      const int rows = P < kDecodeChunkAlign ? P : kDecodeChunkAlign;
+      const uint32_t copy_bytes = static_cast<uint32_t>(rows) * D * 2;
+      const int32_t* tbl = pv.block_table + static_cast<size_t>(b) * pv.max_pages;
+      int win = 0, entry = 0;
+      bool have = false;
+      int issued = 0, skipped = -1;
+      for (int it = 0; it < n_stages; ++it) {
+        const int slot = it % C::NSTAGE, round = it / C::NSTAGE;
+        if (!mbar_wait_warp(bar_empty + 8 * slot, (round & 1) ^ 1, ctl, ab)) break;
+        const int tok0 = t_begin + it * C::T;
+        const int ncopy = (min(C::T, t_end - tok0) + rows - 1) / rows;
+        const int lp_first = tok0 / P, lp_last = (tok0 + (ncopy - 1) * rows) / P;
+        if (!have || lp_first < win || lp_last >= win + 32) {  // refill the table window
+          win = lp_first;
+          entry = (win + lane < pv.max_pages) ? tbl[win + lane] : 0;
+          have = true;
+        }
+        issued = it + 1;
+        if (ctl.inject == 1 && it == 1) {  // test hook: never fill this stage
+          skipped = it;
+          continue;
+        }
+        const uint32_t dst = s_base + slot * C::STAGE_BYTES;
+        if (lane == 0) mbar_expect_tx(bar_full + 8 * slot, 2u * ncopy * copy_bytes);
+        __syncwarp();
+        const int t = tok0 + lane * rows;
+        const int page = __shfl_sync(0xffffffffu, entry, (t / P - win) & 31);
+        if (lane < ncopy) {
+          // an out-of-range page (a caller error) is sent past the last key, where the
+          // copy engine reads zeros
+          const long long zl = static_cast<long long>(page) * P + t % P;
+          const int z = (page < 0 || zl >= pv.num_keys) ? pv.num_keys : static_cast<int>(zl);
+          tma_load_3d(dst + lane * copy_bytes, &tm_k, 0, hk, z, bar_full + 8 * slot);
+          tma_load_3d(dst + C::TILE_BYTES + lane * copy_bytes, &tm_v, 0, hk, z, bar_full + 8 * slot);
+        }
+      }
+      if (lane == 0) {
+        Abort no_abort{reinterpret_cast<volatile int*>(smem + L::ABORT_OFF + 4)};
+        *no_abort.flag = 0;
+        for (int it = max(0, issued - C::NSTAGE); it < issued; ++it) {
+          if (it == skipped) continue;
+          mbar_wait(bar_full + 8 * (it % C::NSTAGE), (it / C::NSTAGE) & 1, ctl, no_abort);
+        }
+      }
+    } else if (lane == 0) {
       int issued = 0, skipped = -1;
       for (int it = 0; it < n_stages; ++it) {
         const int slot = it % C::NSTAGE, round = it / C::NSTAGE;
@@ -422,26 +488,72 @@ __global__ void __launch_bounds__(D) decode_merge_kernel(const float* __restrict
   if (lse && d == 0) lse[bh] = any ? M + log2f(W) * kLn2 : -INFINITY;
 }
 
-template <int D, int GT>
-cudaError_t launch_split(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult qres;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &qres) ==
+            cudaSuccess &&
+        qres == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+// A paged cache [num_pages, page_size, Hkv, D] viewed as the 3-D tensor
+// [num_pages * page_size keys, Hkv, D] (innermost first: D, Hkv, keys); one box is
+// `rows` keys of one kv head, landing in shared memory as rows x D contiguous bf16.
+bool paged_map(CUtensorMap* map, const void* cache, const PagedKV& pk, int Hkv, int D, int rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(Hkv),
+                        static_cast<cuuint64_t>(pk.num_pages) * pk.page_size};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(Hkv) * D * 2};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(D), 1, static_cast<cuuint32_t>(rows)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(cache), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D, int GT, bool PAGED>
+cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
   using C = DecodeCfg<D>;
   constexpr uint32_t smem = DecodeSmem<D, GT>::BYTES;
   static unsigned long long configured = 0;  // one bit per device
   int dev = 0;
   cudaGetDevice(&dev);
   if (!(configured & (1ull << (dev & 63)))) {
-    cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D, GT>,
+    cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D, GT, PAGED>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     configured |= 1ull << (dev & 63);
   }
+  CUtensorMap tk, tv;
+  PagedView view{nullptr, 0, 0, 0};
+  if constexpr (PAGED) {
+    const int rows = pk->page_size < kDecodeChunkAlign ? pk->page_size : kDecodeChunkAlign;
+    if (!paged_map(&tk, a.k, *pk, a.Hkv, D, rows) || !paged_map(&tv, a.v, *pk, a.Hkv, D, rows))
+      return cudaErrorInvalidValue;
+    view = PagedView{pk->block_table, pk->page_size, pk->max_pages, pk->num_pages * pk->page_size};
+  } else {
+    (void)pk;
+    memset(&tk, 0, sizeof(tk));
+    memset(&tv, 0, sizeof(tv));
+  }
   const int G = a.Hq / a.Hkv;
   const int n_groups = (G + GT - 1) / GT;
   dim3 grid(a.splits, a.Hkv * n_groups, a.B);
-  decode_split_kernel<D, GT><<<grid, C::THREADS, smem, stream>>>(
+  decode_split_kernel<D, GT, PAGED><<<grid, C::THREADS, smem, stream>>>(
       static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.k),
       static_cast<const __nv_bfloat16*>(a.v), a.seqlens, a.o_part, a.lse_part, a.Hq, a.Hkv, a.Skv,
-      a.splits, n_groups, a.scale * kLog2e, ctl);
+      a.splits, n_groups, a.scale * kLog2e, ctl, tk, tv, view);
   return cudaGetLastError();
 }
 
@@ -462,14 +574,14 @@ cudaError_t launch_merge(const DecodeArgs& a, cudaStream_t stream) {
                             static_cast<__nv_bfloat16*>(a.o), a.lse, a.splits);
 }
 
-template <int D>
-cudaError_t launch_decode_d(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+template <int D, bool PAGED>
+cudaError_t launch_decode_d(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
   const int G = a.Hq / a.Hkv;
   cudaError_t e;
-  if (G >= 8) e = launch_split<D, 8>(a, ctl, stream);
-  else if (G >= 4) e = launch_split<D, 4>(a, ctl, stream);
-  else if (G >= 2) e = launch_split<D, 2>(a, ctl, stream);
-  else e = launch_split<D, 1>(a, ctl, stream);
+  if (G >= 8) e = launch_split<D, 8, PAGED>(a, pk, ctl, stream);
+  else if (G >= 4) e = launch_split<D, 4, PAGED>(a, pk, ctl, stream);
+  else if (G >= 2) e = launch_split<D, 2, PAGED>(a, pk, ctl, stream);
+  else e = launch_split<D, 1, PAGED>(a, pk, ctl, stream);
   if (e != cudaSuccess) return e;
   return launch_merge<D>(a, stream);
 }
@@ -477,8 +589,14 @@ cudaError_t launch_decode_d(const DecodeArgs& a, const KernelCtl& ctl, cudaStrea
 }  // namespace
 
 cudaError_t launch_decode(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
-  if (a.D == 128) return launch_decode_d<128>(a, ctl, stream);
-  return launch_decode_d<64>(a, ctl, stream);
+  if (a.D == 128) return launch_decode_d<128, false>(a, nullptr, ctl, stream);
+  return launch_decode_d<64, false>(a, nullptr, ctl, stream);
+}
+
+cudaError_t launch_decode_paged(const DecodeArgs& a, const PagedKV& pk, const KernelCtl& ctl, cudaStream_t stream) {
+  if (!paged_page_size_ok(pk.page_size) || !a.seqlens || !pk.block_table) return cudaErrorInvalidValue;
+  if (a.D == 128) return launch_decode_d<128, true>(a, &pk, ctl, stream);
+  return launch_decode_d<64, true>(a, &pk, ctl, stream);
 }
 
 }  // namespace loom

@@ -13,6 +13,7 @@
 #include "gemm_model.h"
 #include "kernels.h"
 #include "model.h"
+#include "paged.h"
 
 namespace loom {
 namespace {
@@ -170,6 +171,49 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
                num_splits, scale};
   return launch_decode(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                  : LOOM_ERR_CUDA;
+}
+
+loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const void* v_cache,
+                                   const int32_t* block_table, const int32_t* seqlens_k, void* o,
+                                   float* lse, void* workspace, size_t workspace_bytes, int B, int Hq,
+                                   int Hkv, int num_pages, int page_size, int max_pages, int D,
+                                   float scale, int num_splits, void* stream) {
+  if (!q || !k_cache || !v_cache || !o || !block_table || !seqlens_k) return LOOM_ERR_INVALID_ARG;
+  if (B <= 0 || Hq <= 0 || Hkv <= 0 || num_pages <= 0 || page_size <= 0 || max_pages <= 0 || D <= 0)
+    return LOOM_ERR_INVALID_ARG;
+  if (Hq % Hkv != 0) return LOOM_ERR_INVALID_ARG;
+  if (!std::isfinite(scale) || scale <= 0.f) return LOOM_ERR_INVALID_ARG;
+  if (num_splits < 0) return LOOM_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return LOOM_ERR_UNSUPPORTED;
+  if (!paged_page_size_ok(page_size)) return LOOM_ERR_UNSUPPORTED;
+  if (static_cast<long long>(num_pages) * page_size > 0x7fffffffLL ||
+      static_cast<long long>(max_pages) * page_size > 0x7fffffffLL ||
+      static_cast<long long>(B) * max_pages > 0x7fffffffLL)
+    return LOOM_ERR_UNSUPPORTED;
+  if (num_splits > kMaxDecodeSplits) return LOOM_ERR_UNSUPPORTED;
+  if (static_cast<long long>(B) * Hq * (num_splits ? num_splits : 1) > 0x7fffffffLL ||
+      static_cast<long long>(B) > 65535)
+    return LOOM_ERR_UNSUPPORTED;
+  if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(o)) return LOOM_ERR_MISALIGNED;
+  if ((reinterpret_cast<uintptr_t>(block_table) & 3u) || (reinterpret_cast<uintptr_t>(seqlens_k) & 3u) ||
+      (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
+    return LOOM_ERR_MISALIGNED;
+  const int Skv = max_pages * page_size;
+  if (num_splits == 0) num_splits = loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D);
+  if (num_splits <= 0) return LOOM_ERR_INVALID_ARG;
+  const size_t need = decode_workspace_bytes(B, Hq, D, num_splits);
+  if (!workspace || workspace_bytes < need) return LOOM_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return LOOM_ERR_MISALIGNED;
+  KernelCtl ctl;
+  if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
+  const size_t rows = static_cast<size_t>(B) * Hq * num_splits;
+  float* o_part = static_cast<float*>(workspace);
+  float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
+                                             (rows * D * sizeof(float) + 255) / 256 * 256);
+  DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D, num_splits, scale};
+  PagedKV pk{block_table, num_pages, page_size, max_pages};
+  return launch_decode_paged(a, pk, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
+                                                                                          : LOOM_ERR_CUDA;
 }
 
 loom_status loom_gemm_bf16(const void* a, const void* b, void* c, int M, int N, int K, void* stream) {

@@ -132,3 +132,26 @@ def test_gemm_splits_only_when_tiles_are_few(lib):
     assert 0 < t8 < t1
     assert lib.loom_model_gemm_time_us(256, 256, 16384, 64, 3, 152) < 0  # unsupported split
     assert lib.loom_model_gemm_time_us(256, 256, 16384, 96, 1, 152) < 0  # unsupported width
+
+
+def test_paged_decode_rejects_bad_arguments(lib):
+    ok = dict(q=FAKE, k=FAKE, v=FAKE, tbl=FAKE, sl=FAKE, o=FAKE, lse=None, ws=FAKE, wsb=1 << 24, B=2, Hq=8,
+              Hkv=2, npages=64, P=16, maxp=8, D=128, scale=0.08, splits=4, stream=None)
+    names = list(ok)
+
+    def call(**kw):
+        a = dict(ok)
+        a.update(kw)
+        return lib.loom_attn_decode_paged(*[a[n] for n in names])
+
+    assert call(tbl=None) == 1
+    assert call(sl=None) == 1
+    assert call(P=0) == 1
+    assert call(Hq=7) == 1
+    assert call(P=24) == 2          # UNSUPPORTED page size
+    assert call(P=96) == 2
+    assert call(D=80) == 2
+    assert call(npages=1 << 30, P=64) == 2
+    assert call(tbl=FAKE + 2) == 3  # MISALIGNED
+    assert call(q=FAKE + 8) == 3
+    assert call(wsb=16) == 4        # WORKSPACE
