@@ -215,3 +215,47 @@ def decode_paged(q, k_cache, v_cache, block_table, seqlens, *, page_size, scale=
     v = paged_gather(v_cache, block_table, seqlens, page_size)
     o, lse = attention(q, k, v, scale=scale, seqlens_k=np.asarray(seqlens, dtype=np.int32), nthreads=nthreads)
     return o[:, :, 0, :], lse[:, :, 0]
+
+
+def attention_varlen(q, k, v, cu_seqlens_q, cu_seqlens_k, *, causal=False, scale=None, nthreads=0):
+    """Attention over a ragged batch packed token-major: q [total_q, Hq, D], k/v
+    [total_k, Hkv, D]; sequence b owns query tokens cu_seqlens_q[b] .. cu_seqlens_q[b+1]
+    and key tokens cu_seqlens_k[b] .. cu_seqlens_k[b+1] (the packed-varlen convention; the
+    paper has none).  Each sequence is the attention definition on its own tokens, causal
+    masking bottom-right aligned per sequence.  Returns ``(o [total_q, Hq, D],
+    lse [Hq, total_q])``; a query with no visible key has O = 0 and LSE = -inf."""
+    q, k, v = _u16(q), _u16(k), _u16(v)
+    cq = np.asarray(cu_seqlens_q, dtype=np.int64)
+    ck = np.asarray(cu_seqlens_k, dtype=np.int64)
+    total_q, Hq, D = q.shape
+    total_k, Hkv, Dk = k.shape
+    if v.shape != k.shape or Dk != D or cq.shape != ck.shape or cq.ndim != 1 or cq.size < 2:
+        raise ValueError("expected q [total_q, Hq, D], k/v [total_k, Hkv, D], cu_seqlens [B + 1]")
+    if cq[0] != 0 or ck[0] != 0 or cq[-1] != total_q or ck[-1] != total_k or np.any(np.diff(cq) < 0) \
+            or np.any(np.diff(ck) < 0):
+        raise ValueError("cu_seqlens must run from 0 to the token totals without decreasing")
+    if scale is None:
+        scale = 1.0 / np.sqrt(D)
+    o = np.zeros((total_q, Hq, D), dtype=np.float64)
+    lse = np.full((Hq, total_q), -np.inf, dtype=np.float64)
+    for b in range(cq.size - 1):
+        q0, q1, k0, k1 = int(cq[b]), int(cq[b + 1]), int(ck[b]), int(ck[b + 1])
+        if q1 == q0:
+            continue
+        if k1 == k0:
+            continue  # no keys: O = 0, LSE = -inf
+        qb = np.ascontiguousarray(q[q0:q1].transpose(1, 0, 2))[None]
+        kb = np.ascontiguousarray(k[k0:k1].transpose(1, 0, 2))[None]
+        vb = np.ascontiguousarray(v[k0:k1].transpose(1, 0, 2))[None]
+        if causal and q1 - q0 > k1 - k0:
+            # rows with no visible key (i < Sq - Skv) are left at O = 0, LSE = -inf; the
+            # others see keys j <= i + (Skv - Sq) as in the definition
+            skip = (q1 - q0) - (k1 - k0)
+            ob, lb = attention(qb[:, :, skip:], kb, vb, causal=True, scale=scale, nthreads=nthreads)
+            o[q0 + skip:q1] = ob[0].transpose(1, 0, 2)
+            lse[:, q0 + skip:q1] = lb[0]
+        else:
+            ob, lb = attention(qb, kb, vb, causal=causal, scale=scale, nthreads=nthreads)
+            o[q0:q1] = ob[0].transpose(1, 0, 2)
+            lse[:, q0:q1] = lb[0]
+    return o, lse
