@@ -127,8 +127,8 @@ class ClockSampler:
 # headline prefill kernel from the ncu capture summarised in
 # profiles/attn_fwd_d128_b4_h32_s2048_noncausal.md, and the SHA-256 of the kernel sources
 # it was taken from: the number is reported only while the sources are unchanged.
-PROFILED_TRAFFIC_BYTES = 243.7e6
-PROFILED_SOURCES_SHA256 = "fcbdb092d053fa598d60aa8553bc9b2f884e3fe61f24f622bc8e60e4836896d4"
+PROFILED_TRAFFIC_BYTES = 243.0e6
+PROFILED_SOURCES_SHA256 = "a5337da4db4328d01e4b9572cd34abcef84271cdf34a13326326fab0712b5a9f"
 
 
 def profiled_traffic():
@@ -331,6 +331,49 @@ class PagedDecode(Decode):
                                          stream=stream)
 
 
+class VarlenPrefill:
+    """Prefill over a ragged batch packed [total, H, D]: seeded lengths U[lo, hi], causal
+    (each sequence attends to itself), FLOPs = 4 D per visible (query, key) pair."""
+
+    def __init__(self, name, B, Hq, Hkv, lo, hi, D, causal=True, seed=0, sets=2):
+        self.name, self.B, self.Hq, self.Hkv, self.D, self.causal = name, B, Hq, Hkv, D, causal
+        self.seed, self.sets, self.lo, self.hi = seed, sets, lo, hi
+        self.lens = synth.decode_lengths(seed + 1, B, lo, hi).astype(np.int64)
+        self.cu = np.concatenate([[0], np.cumsum(self.lens)]).astype(np.int32)
+        self.total = int(self.cu[-1])
+        self.flops = float(sum(prefill_flops(1, Hq, int(n), int(n), D, causal) for n in self.lens))
+        self.bytes = 2 * (self.total * Hq * D * 2 + self.total * Hkv * D * 2) + self.total * Hq * 4
+        self.unit = "TFLOP/s"
+
+    def describe(self):
+        return (f"varlen prefill B={self.B} lengths U[{self.lo},{self.hi}] (total {self.total} tokens) "
+                f"Hq={self.Hq} Hkv={self.Hkv} D={self.D} {'causal' if self.causal else 'non-causal'}")
+
+    def setup(self, torch, dev, loom):
+        self.loom = loom
+        self.inp = []
+        self.cq = torch.from_numpy(self.cu).to(dev)
+        self.maxq = int(self.lens.max())
+        for s in range(self.sets):
+            seed = self.seed + s
+            q = to_tensor(torch, synth.bf16_normal(seed, synth.STREAM_Q, (self.total, self.Hq, self.D)), dev)
+            k = to_tensor(torch, synth.bf16_normal(seed, synth.STREAM_K, (self.total, self.Hkv, self.D)), dev)
+            v = to_tensor(torch, synth.bf16_normal(seed, synth.STREAM_V, (self.total, self.Hkv, self.D)), dev)
+            self.inp.append((q, k, v, torch.empty_like(q),
+                             torch.empty((self.Hq, self.total), dtype=torch.float32, device=dev)))
+
+    def launches_per_step(self):
+        return 1
+
+    def step(self, i, stream):
+        q, k, v, o, lse = self.inp[i % self.sets]
+        self.loom.loom_attn_fwd_varlen(q, k, v, self.cq, self.cq, self.maxq, o, lse, causal=self.causal,
+                                       stream=stream)
+
+    def value(self, seconds_per_step):
+        return self.flops / seconds_per_step / 1e12
+
+
 class Gemm:
     """C = A B in bf16 with fp32 accumulation (the paper's GEMM, Sec. 4); A, B seeded N(0, 1)
     drawn on the device.  `cublas` times torch.matmul (cuBLAS) on the same buffers."""
@@ -529,7 +572,8 @@ def main():
                          "against cuBLAS, every tile width measured (one JSON line per point)")
     ap.add_argument("--ncu-case", default=None,
                     help="profiling run: set up this workload (tiny, tiny_causal, prefill, prefill_causal, "
-                         "long_prefill_d128, long_prefill_d64, batched_decode, paged_decode_p16, paged_decode_p64, long_decode, "
+                         "long_prefill_d128, long_prefill_d64, varlen_prefill, batched_decode, paged_decode_p16, paged_decode_p64, "
+                         "long_decode, "
                          "gemm_4096, "
                          "gemm_16k_256_16k), run --steps launches, print nothing")
     args = ap.parse_args()
@@ -582,6 +626,7 @@ def main():
             Prefill("prefill_causal", 4, 32, 32, 2048, 128, causal=True),
             Prefill("long_prefill_d128", 1, 32, 8, 8192, 128, causal=True),
             Prefill("long_prefill_d64", 1, 64, 16, 8192, 64, causal=True),
+            VarlenPrefill("varlen_prefill", 16, 32, 8, 1024, 8192, 128, causal=True),
             Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
             PagedDecode("paged_decode_p16", 16, 32, 8, 8192, 128, splits=16, page_size=16, lengths=lens),
             PagedDecode("paged_decode_p64", 16, 32, 8, 8192, 128, splits=16, page_size=64, lengths=lens),
@@ -790,6 +835,7 @@ def all_workloads():
             Prefill("prefill_causal", 4, 32, 32, 2048, 128, causal=True),
             Prefill("long_prefill_d128", 1, 32, 8, 8192, 128, causal=True),
             Prefill("long_prefill_d64", 1, 64, 16, 8192, 64, causal=True),
+            VarlenPrefill("varlen_prefill", 16, 32, 8, 1024, 8192, 128, causal=True),
             Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
             PagedDecode("paged_decode_p16", 16, 32, 8, 8192, 128, splits=16, page_size=16, lengths=lens),
             PagedDecode("paged_decode_p64", 16, 32, 8, 8192, 128, splits=16, page_size=64, lengths=lens),

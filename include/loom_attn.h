@@ -63,6 +63,33 @@ loom_status loom_attn_fwd(const void* q, const void* k, const void* v, void* o, 
                           void* stream);
 
 /*
+ * Prefill over a ragged batch packed token-major (the packed-varlen layout; the paper has
+ * no counterpart -- irregular grids are outside its Sec. 2.6 scope note).
+ *   q             [total_q, Hq, D]   bf16, read
+ *   k, v          [total_k, Hkv, D]  bf16, read
+ *   o             [total_q, Hq, D]   bf16, written
+ *   lse           [Hq, total_q]      fp32, written (natural log); may be NULL
+ *   cu_seqlens_q,
+ *   cu_seqlens_k  [B + 1] int32 on the device: sequence b owns query tokens
+ *                 cu_seqlens_q[b] .. cu_seqlens_q[b+1] - 1 and key tokens likewise; both
+ *                 start at 0, never decrease and end at total_q / total_k.
+ *   max_seqlen_q  an upper bound of the query lengths (it only sizes the launch; every
+ *                 sequence is computed whatever its value).
+ * Each sequence is attention on its own tokens (GQA as loom_attn_fwd); causal masking is
+ * bottom-right aligned per sequence, and a query with no visible key (causal with more
+ * queries than keys, or no keys) gets O = 0 and LSE = -inf.  Runs the two-tile prefill
+ * kernel (design 2) with a sequence cursor over the offsets.
+ * Errors: INVALID_ARG (NULL pointer, B, Hq, Hkv or D <= 0, total_q, total_k or
+ * max_seqlen_q < 0, Hq % Hkv, scale), UNSUPPORTED (D not 64 or 128; total_k = 0 while
+ * total_q > 0; more than 2^31 work items), MISALIGNED (q, k, v, o not 16-byte aligned;
+ * cu_seqlens, lse not 4-byte aligned), CUDA.  total_q = 0 returns LOOM_OK at once.
+ */
+loom_status loom_attn_fwd_varlen(const void* q, const void* k, const void* v, void* o, float* lse,
+                                 const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int B,
+                                 int Hq, int Hkv, int total_q, int total_k, int max_seqlen_q, int D,
+                                 int causal, float scale, void* stream);
+
+/*
  * Number of KV splits the decode path uses for this problem when the caller passes
  * num_splits = 0: the analytic model's choice (one wave of split CTAs over the GPU's
  * SMs, Sec. 2.6 Eq. 8-9 restated for GB300).  Returns 0 on invalid sizes.

@@ -26,7 +26,7 @@ __all__ = [
     "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
     "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
     "loom_model_fwd_plan_variant", "loom_model_heg_pipe", "loom_model_fwd_time_us_design",
-    "loom_attn_decode_paged", "loom_gemm_bf16", "loom_gemm_tile_n", "loom_gemm_splits", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
+    "loom_attn_decode_paged", "loom_attn_fwd_varlen", "loom_gemm_bf16", "loom_gemm_tile_n", "loom_gemm_splits", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
     "loom_debug_gemm_splits",
 ]
 
@@ -104,6 +104,9 @@ def capi() -> ctypes.CDLL:
             lib.loom_attn_decode_paged.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, sz, i32, i32, i32, i32,
                                                    i32, i32, i32, f32, i32, vp]
             lib.loom_attn_decode_paged.restype = i32
+            lib.loom_attn_fwd_varlen.argtypes = [vp, vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32,
+                                                 i32, f32, vp]
+            lib.loom_attn_fwd_varlen.restype = i32
             lib.loom_gemm_bf16.argtypes = [vp, vp, vp, i32, i32, i32, vp]
             lib.loom_gemm_bf16.restype = i32
             lib.loom_gemm_tile_n.argtypes = [i32, i32, i32]
@@ -241,6 +244,44 @@ def loom_attn_decode(q, k_cache, v_cache, seqlens_k=None, o=None, lse=None, work
                                  B, Hq, Hkv, Skv, D, float(scale), int(num_splits),
                                  _stream_ptr(stream, q.device))
     _check(st, "loom_attn_decode")
+    return (o, lse) if (return_lse or lse is not None) else o
+
+
+def loom_attn_fwd_varlen(q, k, v, cu_seqlens_q, cu_seqlens_k, max_seqlen_q, o=None, lse=None, *, causal=False,
+                         scale=None, stream=None, return_lse=False):
+    """Prefill over a ragged batch.  q [total_q, Hq, D], k/v [total_k, Hkv, D] bf16;
+    cu_seqlens_q / cu_seqlens_k [B + 1] int32 on the device; max_seqlen_q an int.
+    Returns ``o`` ([total_q, Hq, D]) or ``(o, lse)`` with lse [Hq, total_q]."""
+    torch = _torch()
+    bf16 = torch.bfloat16
+    qp = _dev_ptr(q, "q", bf16, 3)
+    kp = _dev_ptr(k, "k", bf16, 3)
+    vp_ = _dev_ptr(v, "v", bf16, 3)
+    total_q, Hq, D = q.shape
+    total_k, Hkv, Dk = k.shape
+    if tuple(v.shape) != tuple(k.shape) or Dk != D:
+        raise ValueError("varlen prefill takes q [total_q, Hq, D] and k/v [total_k, Hkv, D]")
+    cqp = _dev_ptr(cu_seqlens_q, "cu_seqlens_q", torch.int32, 1)
+    ckp = _dev_ptr(cu_seqlens_k, "cu_seqlens_k", torch.int32, 1)
+    if cu_seqlens_q.numel() != cu_seqlens_k.numel() or cu_seqlens_q.numel() < 2:
+        raise ValueError("cu_seqlens_q and cu_seqlens_k must both be [B + 1]")
+    B = cu_seqlens_q.numel() - 1
+    if o is None:
+        o = torch.empty_like(q)
+    op = _dev_ptr(o, "o", bf16, 3)
+    if lse is None and return_lse:
+        lse = torch.empty((Hq, total_q), dtype=torch.float32, device=q.device)
+    lp = None
+    if lse is not None:
+        if lse.numel() != Hq * total_q:
+            raise ValueError("lse must hold Hq*total_q values")
+        lp = _dev_ptr(lse, "lse", torch.float32)
+    if scale is None:
+        scale = D ** -0.5
+    st = capi().loom_attn_fwd_varlen(qp, kp, vp_, op, lp, cqp, ckp, B, Hq, Hkv, total_q, total_k,
+                                     int(max_seqlen_q), D, int(bool(causal)), float(scale),
+                                     _stream_ptr(stream, q.device))
+    _check(st, "loom_attn_fwd_varlen")
     return (o, lse) if (return_lse or lse is not None) else o
 
 

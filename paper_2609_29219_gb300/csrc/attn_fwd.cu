@@ -27,9 +27,11 @@
 #include <cuda_bf16.h>
 
 #include <cmath>
+#include <cstring>
 #include <mutex>
 
 #include "kernels.h"
+#include "varlen.h"
 #include "model.h"
 #include "ptx.cuh"
 
@@ -86,11 +88,16 @@ struct FwdParams {
   int causal;
   float c;       // scale * log2(e)
   KernelCtl ctl;
+  // ragged batches (Q/K/V/O packed [total, H, D]; unused by the dense instantiations)
+  const int32_t* cu_q;  // [B + 1] first query token of each sequence
+  const int32_t* cu_k;  // [B + 1] first key token of each sequence
+  int B, total_q;       // sequences; query tokens (the row stride of LSE [Hq, total_q])
 };
 
 // One work item of a persistent CTA: a pair of 128-row query tiles of one (b, h).
 struct Item {
   int b, h, q_z, kv_z, q0, n_tiles0, n_tiles;
+  int sq, skv, qb, kb;  // ragged batches: the sequence's lengths and first tokens
 };
 
 // The r-th item of this CTA (-1 once it has none left).  Causal items are ordered
@@ -153,6 +160,88 @@ __device__ __forceinline__ Item make_item(const FwdParams& p, int idx) {
   it.n_tiles0 = (n_kv0 + C::BN - 1) / C::BN;
   it.n_tiles = (n_kv1 + C::BN - 1) / C::BN;
   return it;
+}
+
+// ---------------------------------------------------------------- ragged batches
+// Items are (sequence, head, query-tile pair) in sequence order; sequence b, with sq_b
+// query rows, owns ceil(sq_b / rows_per_item) pairs per head.  Every role walks its items
+// with a cursor over the sequence offsets -- a CTA's item indices only grow -- so no item
+// list is stored and an empty sequence costs one step of the cursor.
+struct SeqCursor {
+  int b;            // sequence of the last located item
+  long long first;  // index of that sequence's first item
+  int pairs;        // its query-tile pairs per head
+};
+
+template <int ROWS>
+__device__ __forceinline__ int seq_pairs(const FwdParams& p, int b) {
+  const int sq = p.cu_q[b + 1] - p.cu_q[b];
+  return sq > 0 ? (sq + ROWS - 1) / ROWS : 0;
+}
+
+template <int ROWS>
+__device__ __forceinline__ SeqCursor seq_cursor(const FwdParams& p) {
+  return SeqCursor{0, 0, p.B > 0 ? seq_pairs<ROWS>(p, 0) : 0};
+}
+
+// Dense: the r-th item's index (see item_index).  Ragged: the same dealing over the
+// unbounded index space, with the cursor moved to the item's sequence; -1 past the last.
+template <int ROWS, bool VARLEN>
+__device__ __forceinline__ int item_index_t(const FwdParams& p, int r, SeqCursor& cur) {
+  if constexpr (!VARLEN) {
+    (void)cur;
+    return item_index(p, r);
+  } else {
+    const int G = static_cast<int>(gridDim.x), c = static_cast<int>(blockIdx.x);
+    const long long idx = static_cast<long long>(r) * G + ((p.causal && (r & 1)) ? G - 1 - c : c);
+    while (cur.b < p.B && idx >= cur.first + static_cast<long long>(cur.pairs) * p.Hq) {
+      cur.first += static_cast<long long>(cur.pairs) * p.Hq;
+      ++cur.b;
+      cur.pairs = cur.b < p.B ? seq_pairs<ROWS>(p, cur.b) : 0;
+    }
+    return cur.b < p.B ? static_cast<int>(idx) : -1;
+  }
+}
+
+// Ragged item: causal takes a sequence's heaviest pairs (last rows) first over all heads;
+// non-causal takes one head's pairs in a row (they share its K/V in L2).  At least one KV
+// tile is processed even when no key is visible (fully masked: O = 0, LSE = -inf).
+template <int D, bool VARLEN>
+__device__ __forceinline__ Item make_item_t(const FwdParams& p, const SeqCursor& cur, int idx) {
+  using C = FwdCfg<D>;
+  if constexpr (!VARLEN) {
+    (void)cur;
+    return make_item<D>(p, idx);
+  } else {
+    const int in = static_cast<int>(idx - cur.first);
+    int pos, h;
+    if (p.causal) {
+      pos = cur.pairs - 1 - in / p.Hq;
+      h = in % p.Hq;
+    } else {
+      pos = in % cur.pairs;
+      h = in / cur.pairs;
+    }
+    Item it;
+    it.b = cur.b;
+    it.h = h;
+    it.q_z = h;
+    it.kv_z = h / (p.Hq / p.Hkv);
+    it.qb = p.cu_q[cur.b];
+    it.sq = p.cu_q[cur.b + 1] - it.qb;
+    it.kb = p.cu_k[cur.b];
+    it.skv = p.cu_k[cur.b + 1] - it.kb;
+    it.q0 = pos * (C::NQT * C::BM);
+    const int off = it.skv - it.sq;
+    int n_kv0 = it.skv, n_kv1 = it.skv;
+    if (p.causal) {
+      n_kv0 = min(it.skv, it.q0 + C::BM + off);
+      n_kv1 = min(it.skv, it.q0 + 2 * C::BM + off);
+    }
+    it.n_tiles0 = max(1, (n_kv0 + C::BN - 1) / C::BN);
+    it.n_tiles = max(it.n_tiles0, (n_kv1 + C::BN - 1) / C::BN);
+    return it;
+  }
 }
 
 // One online-softmax step of one query row (this thread's TMEM lane) over a BN-key
@@ -257,12 +346,15 @@ __device__ __forceinline__ bool softmax_step(uint32_t s_tm, uint32_t o_tm, uint3
 // let one lane store the block with TMA (rows >= Sq are clipped by the tensor map).  The
 // store completes in the background; the block is reused by this warp one item later,
 // after waiting for the store to have read it.  Finally the log-sum-exp.
-template <int D>
+// Ragged batches (VARLEN): O is [total_q, Hq, D] and the store box is 32 rows of one head;
+// a warp whose 32 rows run past its sequence's end writes its valid rows with plain
+// stores instead (a TMA store would spill into the next sequence), and LSE is [Hq, total_q].
+template <int D, bool VARLEN = false>
 __device__ __forceinline__ bool softmax_epilogue(uint32_t o_tm, uint32_t bar_o, uint32_t par_o,
                                                  uint32_t bar_oe, float m_run, float l_run,
                                                  int row, int q_z, const FwdParams& p,
                                                  const Abort& ab, const CUtensorMap* tm_o,
-                                                 uint32_t stg) {
+                                                 uint32_t stg, int qb = 0, int sq = 0) {
   const int lane = threadIdx.x & 31;
   if (!mbar_wait_warp(bar_o, par_o, p.ctl, ab)) return false;
   tc_fence_after();
@@ -283,6 +375,20 @@ __device__ __forceinline__ bool softmax_epilogue(uint32_t o_tm, uint32_t bar_o, 
   }
   tc_fence_before();
   mbar_arrive(bar_oe);  // O is in registers: the next item's P.V may overwrite it
+  if constexpr (VARLEN) {
+    const int row0 = row - lane;  // the warp's rows are row0 .. row0 + 31
+    if (row0 + 32 > sq) {
+      if (row < sq) {
+        uint4* dst = reinterpret_cast<uint4*>(p.o + (static_cast<size_t>(qb + row) * p.Hq + q_z) * D);
+#pragma unroll
+        for (int c = 0; c < D / 8; ++c) dst[c] = make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+        if (p.lse)
+          p.lse[static_cast<size_t>(q_z) * p.total_q + qb + row] =
+              l_run > 0.f ? (m_run + log2f(l_run)) * kLn2 : -INFINITY;
+      }
+      return true;
+    }
+  }
   if (lane == 0) bulk_wait_group_read0();  // this warp's previous store has left the block
   __syncwarp();
   const uint32_t my_row = stg + static_cast<uint32_t>(lane) * 128u;
@@ -294,6 +400,16 @@ __device__ __forceinline__ bool softmax_epilogue(uint32_t o_tm, uint32_t bar_o, 
   }
   fence_proxy_async_smem();
   __syncwarp();
+  if constexpr (VARLEN) {
+    if (lane == 0) {
+#pragma unroll
+      for (int x = 0; x < D / 64; ++x) tma_store_3d(tm_o, stg + x * 4096u, x * 64, q_z, qb + row);
+      bulk_commit_group();
+    }
+    if (p.lse)
+      p.lse[static_cast<size_t>(q_z) * p.total_q + qb + row] = l_run > 0.f ? (m_run + log2f(l_run)) * kLn2 : -INFINITY;
+    return true;
+  }
   if (lane == 0) {
 #pragma unroll
     for (int x = 0; x < D / 64; ++x) tma_store_3d(tm_o, stg + x * 4096u, x * 64, row, q_z);
@@ -306,24 +422,35 @@ __device__ __forceinline__ bool softmax_epilogue(uint32_t o_tm, uint32_t bar_o, 
 
 // Bring the next work item's query tiles and first K/V tiles into L2 while the current
 // item still runs, so that its start waits on an L2 hit rather than HBM.
-template <int D, int NQT, int BM>
+template <int D, int NQT, int BM, bool VARLEN = false>
 __device__ __forceinline__ void prefetch_item_l2(const CUtensorMap* tm_q, const CUtensorMap* tm_k,
-                                                 const CUtensorMap* tm_v, int q0, int q_z, int kv_z) {
+                                                 const CUtensorMap* tm_v, int q0, int q_z, int kv_z,
+                                                 int qb = 0, int kb = 0) {
 #pragma unroll
   for (int x = 0; x < D / 64; ++x) {
+    if constexpr (VARLEN) {
 #pragma unroll
-    for (int t = 0; t < NQT; ++t) tma_prefetch_l2_3d(tm_q, x * 64, q0 + t * BM, q_z);
-    tma_prefetch_l2_3d(tm_k, x * 64, 0, kv_z);
-    tma_prefetch_l2_3d(tm_v, x * 64, 0, kv_z);
+      for (int t = 0; t < NQT; ++t) tma_prefetch_l2_3d(tm_q, x * 64, q_z, qb + q0 + t * BM);
+      tma_prefetch_l2_3d(tm_k, x * 64, kv_z, kb);
+      tma_prefetch_l2_3d(tm_v, x * 64, kv_z, kb);
+    } else {
+#pragma unroll
+      for (int t = 0; t < NQT; ++t) tma_prefetch_l2_3d(tm_q, x * 64, q0 + t * BM, q_z);
+      tma_prefetch_l2_3d(tm_k, x * 64, 0, kv_z);
+      tma_prefetch_l2_3d(tm_v, x * 64, 0, kv_z);
+    }
   }
 }
 
-template <int D>
+// VARLEN: a ragged batch packed [total, H, D]: the tensor maps are [total, H, D] views
+// (coordinates: column, head, token) and items come from the sequence cursor.
+template <int D, bool VARLEN = false>
 __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                     const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
                     const FwdParams p) {
   using C = FwdCfg<D>;
+  constexpr int kRows = C::NQT * C::BM;  // query rows of one item
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the 128B-swizzled tiles
   const uint32_t raw_base = smem_u32(smem_raw);
@@ -378,27 +505,32 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
       prefetch_tensormap(&tm_v);
       int pos = 0, issued = 0, skipped = -1, q_issued[2] = {0, 0};
       bool ok = true;
+      SeqCursor cur = VARLEN ? seq_cursor<kRows>(p) : SeqCursor{0, 0, 0};
       // Q_t of item r, once the previous item's S MMAs of tile t are done with its buffer
       auto load_q = [&](int t, int r, const Item& it) -> bool {
         if (r > 0 && !mbar_wait(bar_qe + 8 * t, (r - 1) & 1, p.ctl, ab)) return false;
         mbar_expect_tx(bar_q + 8 * t, C::Q_TILE_BYTES);
+        const int qy = VARLEN ? it.q_z : it.q0 + t * C::BM;
+        const int qz = VARLEN ? it.qb + it.q0 + t * C::BM : it.q_z;
         for (int x = 0; x < C::NBOX; ++x)
           tma_load_3d(sbase + C::Q_OFF + t * C::Q_TILE_BYTES + x * C::Q_BOX_BYTES, &tm_q, x * C::BOX_COLS,
-                      it.q0 + t * C::BM, it.q_z, bar_q + 8 * t);
+                      qy, qz, bar_q + 8 * t);
         q_issued[t] = r + 1;
         return true;
       };
-      for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
-        const Item it = make_item<D>(p, idx);
+      for (int r = 0, idx; ok && (idx = item_index_t<kRows, VARLEN>(p, r, cur)) >= 0; ++r) {
+        const Item it = make_item_t<D, VARLEN>(p, cur, idx);
         // Q_0 first: tile 0 finishes its S MMAs of the previous item before tile 1 does
         if (!(ok = load_q(0, r, it))) break;
         for (int jj = 0; jj < 2 * it.n_tiles; ++jj, ++pos) {  // K_0, [Q_1], V_0, K_1, V_1, ...
           if (jj == 1 && !(ok = load_q(1, r, it))) break;
           if (jj == max(0, 2 * it.n_tiles - 6)) {  // three KV tiles before the end
-            const int nidx = item_index(p, r + 1);
+            SeqCursor nc = cur;
+            const int nidx = item_index_t<kRows, VARLEN>(p, r + 1, nc);
             if (nidx >= 0) {
-              const Item nx = make_item<D>(p, nidx);
-              prefetch_item_l2<D, C::NQT, C::BM>(&tm_q, &tm_k, &tm_v, nx.q0, nx.q_z, nx.kv_z);
+              const Item nx = make_item_t<D, VARLEN>(p, nc, nidx);
+              prefetch_item_l2<D, C::NQT, C::BM, VARLEN>(&tm_q, &tm_k, &tm_v, nx.q0, nx.q_z, nx.kv_z, nx.qb,
+                                                         nx.kb);
             }
           }
           const int slot = pos % C::NSLOT, round = pos / C::NSLOT;
@@ -410,10 +542,11 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
           }
           const CUtensorMap* map = (jj & 1) ? &tm_v : &tm_k;
           const int row = (jj >> 1) * C::BN;
+          const int ky = VARLEN ? it.kv_z : row, kz = VARLEN ? it.kb + row : it.kv_z;
           mbar_expect_tx(bar_full + 8 * slot, C::SLOT_BYTES);
           for (int x = 0; x < C::NBOX; ++x)
             tma_load_3d(sbase + C::RING_OFF + slot * C::SLOT_BYTES + x * C::KV_BOX_BYTES, map,
-                        x * C::BOX_COLS, row, it.kv_z, bar_full + 8 * slot);
+                        x * C::BOX_COLS, ky, kz, bar_full + 8 * slot);
         }
       }
       // drain copies still in flight before the CTA may exit
@@ -456,8 +589,9 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
       };
       int pos = 0, cnt0 = 0, cnt1 = 0;  // ring position of K_0; S/P/O uses so far per tile
       bool ok = true;
-      for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
-        const Item it = make_item<D>(p, idx);
+      SeqCursor cur = VARLEN ? seq_cursor<kRows>(p) : SeqCursor{0, 0, 0};
+      for (int r = 0, idx; ok && (idx = item_index_t<kRows, VARLEN>(p, r, cur)) >= 0; ++r) {
+        const Item it = make_item_t<D, VARLEN>(p, cur, idx);
         const int nt0 = it.n_tiles0, nt = it.n_tiles;
         if (!(ok = mbar_wait(bar_q, r & 1, p.ctl, ab) && wait_slot(pos))) break;
         tc_fence_after();
@@ -535,10 +669,13 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
 
     int cnt = 0;  // S tiles of this query tile processed in earlier items
     bool ok = true;
-    for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
-      const Item it = make_item<D>(p, idx);
+    SeqCursor cur = VARLEN ? seq_cursor<kRows>(p) : SeqCursor{0, 0, 0};
+    for (int r = 0, idx; ok && (idx = item_index_t<kRows, VARLEN>(p, r, cur)) >= 0; ++r) {
+      const Item it = make_item_t<D, VARLEN>(p, cur, idx);
       const int row = it.q0 + t * C::BM + row_in_tile;
-      const int limit = p.causal ? min(p.Skv, row + off + 1) : p.Skv;  // keys [0, limit) visible
+      const int skv = VARLEN ? it.skv : p.Skv;
+      const int offv = VARLEN ? it.skv - it.sq : off;
+      const int limit = p.causal ? min(skv, row + offv + 1) : skv;  // keys [0, limit) visible
       const int my_tiles = t == 0 ? it.n_tiles0 : it.n_tiles;
       float m_run = -INFINITY, l_run = 0.f;
       for (int j = 0; ok && j < my_tiles; ++j)
@@ -547,8 +684,9 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
                                     l_run, p.ctl, ab);
       if (!ok) break;
       // epilogue: hand O_t back to the MMA warp, O / l -> bf16 rows, LSE
-      if (!(ok = softmax_epilogue<D>(o_tm, my_bar_o, (cnt + my_tiles - 1) & 1, my_bar_oe, m_run, l_run,
-                                     row, it.q_z, p, ab, &tm_o, stg_q)))
+      if (!(ok = softmax_epilogue<D, VARLEN>(o_tm, my_bar_o, (cnt + my_tiles - 1) & 1, my_bar_oe, m_run,
+                                             l_run, row, it.q_z, p, ab, &tm_o, stg_q,
+                                             VARLEN ? it.qb : 0, VARLEN ? it.sq : 0)))
         break;
       cnt += my_tiles;
     }
@@ -1128,6 +1266,64 @@ bool make_map(CUtensorMap* map, const void* base, int D, int rows, int planes, i
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D view [total, H, D] of a packed [total, H, D] bf16 tensor (innermost first: D, H,
+// tokens) with a 64-column x 1-head x box_rows box, which lands in shared memory exactly
+// like the dense 64 x box_rows box.
+bool make_map_tokens(CUtensorMap* map, const void* base, int D, int H, int total, int box_rows) {
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(total)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(D) * 2 * static_cast<cuuint64_t>(H)};
+  cuuint32_t box[3] = {64, 1, static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D>
+cudaError_t launch_varlen_d(const FwdVarlenArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  using C = FwdCfg<D>;
+  static unsigned long long configured = 0;  // one bit per device
+  CUtensorMap mq, mk, mv, mo;
+  if (!make_map_tokens(&mq, a.q, D, a.Hq, a.total_q, C::BM) ||
+      !make_map_tokens(&mk, a.k, D, a.Hkv, a.total_k, C::BN) ||
+      !make_map_tokens(&mv, a.v, D, a.Hkv, a.total_k, C::BN) ||
+      !make_map_tokens(&mo, a.o, D, a.Hq, a.total_q, 32))
+    return cudaErrorInvalidValue;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (!(configured & (1ull << (dev & 63)))) {
+    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         C::BYTES);
+    if (e != cudaSuccess) return e;
+    configured |= 1ull << (dev & 63);
+  }
+  FwdParams p;
+  memset(&p, 0, sizeof(p));
+  p.o = static_cast<__nv_bfloat16*>(a.o);
+  p.lse = a.lse;
+  p.Hq = a.Hq;
+  p.Hkv = a.Hkv;
+  p.causal = a.causal;
+  p.c = a.scale * kLog2e;
+  p.ctl = ctl;
+  p.cu_q = a.cu_q;
+  p.cu_k = a.cu_k;
+  p.B = a.B;
+  p.total_q = a.total_q;
+  int sms = 0;
+  cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  // items: at most B * Hq * ceil(max_seqlen_q / rows) (the persistent loop takes them all
+  // whatever the grid; max_seqlen_q only caps the CTAs launched)
+  constexpr int kRows = C::NQT * C::BM;
+  const long long bound = static_cast<long long>(a.B) * a.Hq * ((a.max_seqlen_q + kRows - 1) / kRows);
+  const int grid = static_cast<int>(bound > 0 && bound < sms ? bound : sms);
+  attn_fwd_kernel<D, true><<<grid, C::THREADS, C::BYTES, stream>>>(mq, mk, mv, mo, p);
+  return cudaGetLastError();
+}
+
 // Launch one design: C is its configuration, rows_per_item the query rows of one work
 // item (C::NQT * C::BM).
 template <int D, class C, class Kernel>
@@ -1193,6 +1389,11 @@ cudaError_t launch_fwd_d(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t st
 cudaError_t launch_fwd(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
   if (a.D == 128) return launch_fwd_d<128>(a, ctl, stream);
   return launch_fwd_d<64>(a, ctl, stream);
+}
+
+cudaError_t launch_fwd_varlen(const FwdVarlenArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  if (a.D == 128) return launch_varlen_d<128>(a, ctl, stream);
+  return launch_varlen_d<64>(a, ctl, stream);
 }
 
 }  // namespace loom

@@ -14,6 +14,7 @@
 #include "kernels.h"
 #include "model.h"
 #include "paged.h"
+#include "varlen.h"
 
 namespace loom {
 namespace {
@@ -171,6 +172,31 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
                num_splits, scale};
   return launch_decode(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                  : LOOM_ERR_CUDA;
+}
+
+loom_status loom_attn_fwd_varlen(const void* q, const void* k, const void* v, void* o, float* lse,
+                                 const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int B,
+                                 int Hq, int Hkv, int total_q, int total_k, int max_seqlen_q, int D,
+                                 int causal, float scale, void* stream) {
+  if (!q || !k || !v || !o || !cu_seqlens_q || !cu_seqlens_k) return LOOM_ERR_INVALID_ARG;
+  if (B <= 0 || Hq <= 0 || Hkv <= 0 || D <= 0 || total_q < 0 || total_k < 0 || max_seqlen_q < 0)
+    return LOOM_ERR_INVALID_ARG;
+  if (Hq % Hkv != 0) return LOOM_ERR_INVALID_ARG;
+  if (!std::isfinite(scale) || scale <= 0.f) return LOOM_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return LOOM_ERR_UNSUPPORTED;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o)) return LOOM_ERR_MISALIGNED;
+  if ((reinterpret_cast<uintptr_t>(cu_seqlens_q) & 3u) || (reinterpret_cast<uintptr_t>(cu_seqlens_k) & 3u) ||
+      (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
+    return LOOM_ERR_MISALIGNED;
+  if (total_q == 0) return LOOM_OK;
+  if (total_k == 0) return LOOM_ERR_UNSUPPORTED;
+  // work items (query-tile pairs x heads) are at most (total_q / 256 + B) * Hq
+  if ((static_cast<long long>(total_q) / 256 + B) * Hq > 0x7fffffffLL) return LOOM_ERR_UNSUPPORTED;
+  KernelCtl ctl;
+  if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
+  FwdVarlenArgs a{q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, B, Hq, Hkv, total_q, total_k, max_seqlen_q, D,
+                  causal ? 1 : 0, scale};
+  return launch_fwd_varlen(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK : LOOM_ERR_CUDA;
 }
 
 loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const void* v_cache,

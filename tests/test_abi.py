@@ -155,3 +155,25 @@ def test_paged_decode_rejects_bad_arguments(lib):
     assert call(tbl=FAKE + 2) == 3  # MISALIGNED
     assert call(q=FAKE + 8) == 3
     assert call(wsb=16) == 4        # WORKSPACE
+
+
+def test_varlen_prefill_rejects_bad_arguments(lib):
+    ok = dict(q=FAKE, k=FAKE, v=FAKE, o=FAKE, lse=None, cq=FAKE, ck=FAKE, B=2, Hq=8, Hkv=2, tq=100, tk=100,
+              maxq=60, D=128, causal=1, scale=0.08, stream=None)
+    names = list(ok)
+
+    def call(**kw):
+        a = dict(ok)
+        a.update(kw)
+        return lib.loom_attn_fwd_varlen(*[a[n] for n in names])
+
+    assert call(cq=None) == 1
+    assert call(B=0) == 1
+    assert call(tq=-1) == 1
+    assert call(Hq=7) == 1
+    assert call(scale=0.0) == 1
+    assert call(D=96) == 2
+    assert call(tk=0) == 2          # queries but no keys at all
+    assert call(q=FAKE + 8) == 3
+    assert call(ck=FAKE + 2) == 3
+    assert call(tq=0) == 0          # nothing to do
