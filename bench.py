@@ -780,10 +780,10 @@ GEMM_DIMS = (256, 2048, 16384)
 
 def run_gemm_sweep(torch, loom, dev, stream, args, peaks):
     """The BF16 GEMM over the paper's shape range (every M, N, K in {256, 2048, 16384}):
-    cuBLAS (torch.matmul); this library with the model's (tile width, split count); every
-    tile width with persistent tiles (S = 1); and, at the model's tile width, every split
-    count that leaves each CTA two K stages or more (does the model's choice measure
-    best?).  All on the same buffers and stream."""
+    cuBLAS (torch.matmul); this library with the model's choice; CTA-pair tiles; every tile
+    width with single-CTA persistent tiles (S = 1); and, at the model's single-CTA tile
+    width, every split count that leaves each CTA two K stages or more (does the model's
+    choice measure best?).  All on the same buffers and stream."""
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     for M in GEMM_DIMS:
         for N in GEMM_DIMS:
@@ -792,8 +792,10 @@ def run_gemm_sweep(torch, loom, dev, stream, args, peaks):
                 wl.setup(torch, dev, loom)
                 steps = int(min(500, max(10, 0.05 / (wl.flops / 1.5e15))))
                 bn, sp = loom.loom_gemm_tile_n(M, N, K), loom.loom_gemm_splits(M, N, K)
+                pair = loom.loom_gemm_cta_pair(M, N, K)
                 row = {"sweep": "gemm", "workload": wl.describe(), "model_tile_n": bn, "model_splits": sp,
-                       "model_us": round(loom.loom_model_gemm_time_us(M, N, K, bn, sp, sms), 2)}
+                       "model_cta_pair": pair,
+                       "model_us": round(loom.loom_model_gemm_time_us(M, N, K, 512 if pair else bn, sp, sms), 2)}
 
                 def timed():
                     r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks, warm_s=0.25)
@@ -807,18 +809,25 @@ def run_gemm_sweep(torch, loom, dev, stream, args, peaks):
                 row["loom_tflops"] = timed()
                 c = wl.inp[0][2].float()
                 row["max_rel_diff_vs_cublas"] = float(f"{(c - ref).abs().max().item() / max(ref.abs().max().item(), 1e-30):.3g}")
+                loom.loom_debug_gemm_cta_pair(1)
+                row["pair_tflops"] = timed()
+                loom.loom_debug_gemm_cta_pair(-1)
                 for t in (64, 128, 192, 256):
                     loom.loom_debug_gemm_tile_n(t)
                     loom.loom_debug_gemm_splits(1)
                     row[f"bn{t}_s1_tflops"] = timed()
-                loom.loom_debug_gemm_tile_n(bn)
+                loom.loom_debug_gemm_tile_n(0)
+                loom.loom_debug_gemm_splits(0)
+                sbn = loom.loom_gemm_tile_n(M, N, K)  # the model's single-CTA width (pairs forbidden)
+                loom.loom_debug_gemm_tile_n(sbn)
                 for s_ in (2, 4, 8, 16):
                     if (K + 63) // 64 < 2 * s_:
                         break
                     loom.loom_debug_gemm_splits(s_)
-                    row[f"bn{bn}_s{s_}_tflops"] = timed()
+                    row[f"bn{sbn}_s{s_}_tflops"] = timed()
                 loom.loom_debug_gemm_tile_n(0)
                 loom.loom_debug_gemm_splits(0)
+                loom.loom_debug_gemm_cta_pair(0)
                 row["vs_cublas"] = round(row["loom_tflops"] / row["cublas_tflops"], 3)
                 row["frac_of_peak"] = round(row["loom_tflops"] / peaks["bf16_tflops"], 4)
                 print(json.dumps(row), flush=True)

@@ -214,11 +214,11 @@ double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, in
  *   b  [K, N] bf16 row-major, read
  *   c  [M, N] bf16 row-major, written (fp32 accumulation, rounded to nearest even)
  * The caller owns the buffers; the call is asynchronous on `stream` and needs no
- * workspace.  The analytic model picks the tile width (64, 128, 192 or 256 columns of C
- * per 128 rows), the ring depth and the split count S: S = 1 walks the tiles with
- * persistent CTAs; S = 2, 4, 8 or 16 gives each tile a cluster of S CTAs that split K and
- * sum their fp32 partials through distributed shared memory in a fixed order (so the
- * result depends on S but not on timing).  loom_gemm_tile_n / loom_gemm_splits report the
+ * workspace.  The analytic model picks the kernel: persistent CTAs over 128-row tiles of
+ * 64, 128, 192 or 256 columns; persistent CTA pairs over 256 x 256 tiles; or, for few
+ * tiles and a long K, split-K over clusters of S = 2, 4, 8 or 16 CTAs that sum their fp32
+ * partials through distributed shared memory in a fixed order (so the result depends on
+ * S but not on timing).  loom_gemm_tile_n / loom_gemm_splits report the
  * choice for a shape on the current device.
  * Errors: INVALID_ARG (NULL pointer, M, N or K < 1), MISALIGNED (pointer not 16-byte
  * aligned), UNSUPPORTED (K or N not a multiple of 8: rows must be 16-byte multiples for
@@ -229,14 +229,20 @@ loom_status loom_gemm_bf16(const void* a, const void* b, void* c, int M, int N, 
  * device the cluster occupancy is estimated as whole clusters in 8 equal SM groups. */
 int loom_gemm_tile_n(int M, int N, int K);
 int loom_gemm_splits(int M, int N, int K);
+/* 1 if the model computes this shape with CTA-pair tiles: a cluster of two CTAs per 256 x 256
+ * tile of C with M = 256 pair MMAs (each SM holds its 128 rows of A and half of B), else 0. */
+int loom_gemm_cta_pair(int M, int N, int K);
 /* Modeled GEMM launch time (us) with tile width tile_n and split count splits on num_sms SMs
- * (cluster occupancy estimated as above); < 0 if infeasible. */
+ * (cluster occupancy estimated as above; tile_n = 512 with splits = 1 prices the CTA-pair
+ * tiles); < 0 if infeasible. */
 double loom_model_gemm_time_us(int M, int N, int K, int tile_n, int splits, int num_sms);
 /* Test hooks: force the GEMM tile width (64, 128, 192, 256) / split count (1, 2, 4, 8, 16);
  * any other value restores the model's choice.  A forced split may leave CTAs no K stage:
  * their partial is zero. */
 void loom_debug_gemm_tile_n(int tile_n);
 void loom_debug_gemm_splits(int splits);
+/* Test hook: 1 forces CTA-pair tiles, -1 forbids them, anything else restores the model's choice. */
+void loom_debug_gemm_cta_pair(int mode);
 
 /*
  * Synchronises `stream`, then reads and clears the current device's error word.

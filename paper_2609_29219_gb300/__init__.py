@@ -26,8 +26,8 @@ __all__ = [
     "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
     "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
     "loom_model_fwd_plan_variant", "loom_model_heg_pipe", "loom_model_fwd_time_us_design",
-    "loom_attn_decode_paged", "loom_attn_fwd_varlen", "loom_gemm_bf16", "loom_gemm_tile_n", "loom_gemm_splits", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
-    "loom_debug_gemm_splits",
+    "loom_attn_decode_paged", "loom_attn_fwd_varlen", "loom_gemm_bf16", "loom_gemm_tile_n", "loom_gemm_splits", "loom_gemm_cta_pair", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
+    "loom_debug_gemm_splits", "loom_debug_gemm_cta_pair",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -113,12 +113,16 @@ def capi() -> ctypes.CDLL:
             lib.loom_gemm_tile_n.restype = i32
             lib.loom_gemm_splits.argtypes = [i32, i32, i32]
             lib.loom_gemm_splits.restype = i32
+            lib.loom_gemm_cta_pair.argtypes = [i32, i32, i32]
+            lib.loom_gemm_cta_pair.restype = i32
             lib.loom_model_gemm_time_us.argtypes = [i32] * 6
             lib.loom_model_gemm_time_us.restype = ctypes.c_double
             lib.loom_debug_gemm_tile_n.argtypes = [i32]
             lib.loom_debug_gemm_tile_n.restype = None
             lib.loom_debug_gemm_splits.argtypes = [i32]
             lib.loom_debug_gemm_splits.restype = None
+            lib.loom_debug_gemm_cta_pair.argtypes = [i32]
+            lib.loom_debug_gemm_cta_pair.restype = None
             lib.loom_model_decode_time_us.argtypes = [i32, i32, i32, i32, i32, i32, i32]
             lib.loom_model_decode_time_us.restype = ctypes.c_double
             _lib = lib
@@ -410,6 +414,14 @@ def loom_debug_gemm_tile_n(tile_n: int):
 
 def loom_debug_gemm_splits(splits: int):
     capi().loom_debug_gemm_splits(int(splits))
+
+
+def loom_gemm_cta_pair(M, N, K) -> int:
+    return int(capi().loom_gemm_cta_pair(M, N, K))
+
+
+def loom_debug_gemm_cta_pair(mode: int):
+    capi().loom_debug_gemm_cta_pair(int(mode))
 
 
 def loom_model_fwd_time_us_design(design, B, Hq, Sq, Skv, D, causal) -> float:

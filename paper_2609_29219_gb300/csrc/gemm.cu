@@ -445,6 +445,247 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
   }
 }
 
+// ---------------------------------------------------------------- CTA-pair tiles
+// A cluster of two CTAs (a CTA pair) computes 256 x 256 tiles of C with
+// tcgen05.mma.cta_group::2 (M = 256, N = 256, issued by the even CTA): each CTA holds its
+// own 128 rows of A and one half (128 columns) of B per K stage, and its TMEM receives
+// its 128 rows x 256 columns of the accumulator.  Per K stage an SM thus loads 32 KB
+// instead of the 48 KB of a 128 x 256 single-CTA tile, and six stages fit.  Both CTAs'
+// copies complete on the even CTA's full barrier (armed once for 64 KB); the even CTA's
+// commits signal stage-free and accumulator-ready on both CTAs at once; each CTA's four
+// epilogue warps tell the even CTA that an accumulator has been read (8 arrivals).
+struct GemmPairCfg {
+  static constexpr int BM = 128, BN = 256, BK = 64;   // per CTA: 128 rows x 256 columns of C
+  static constexpr int NSTAGE = 6;
+  static constexpr int THREADS = 192;
+  static constexpr int NBH = 2;                        // 64-column boxes of this CTA's half of B
+  static constexpr uint32_t A_BYTES = BM * BK * 2;
+  static constexpr uint32_t B_BOX_BYTES = BK * 64 * 2;
+  static constexpr uint32_t STAGE_BYTES = A_BYTES + NBH * B_BOX_BYTES;  // 32 KB
+  static constexpr uint32_t STG_OFF = NSTAGE * STAGE_BYTES;
+  static constexpr uint32_t STG_WARP = 2 * 32 * 128;
+  static constexpr uint32_t BAR_OFF = STG_OFF + 4 * STG_WARP;
+  static constexpr int NBAR = 2 * NSTAGE + 5;  // full, empty, acc_full[2], acc_empty[2], drain
+  static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
+  static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
+  static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;
+  static constexpr uint32_t TMEM_COLS = 512;  // two accumulators of 256 columns
+  static_assert(BYTES <= 227 * 1024, "shared memory budget");
+};
+
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t dst, uint32_t ncols) {
+  // one warp of each CTA of the pair, together: the same columns in both SMs
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+// 3-D TMA load into this CTA's shared memory completing on `bar`, which may be the peer
+// CTA's barrier (a shared::cluster address).
+__device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap* map, int x, int y, int z,
+                                                 uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2 [%0], [%1, "
+      "{%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void mma_ss_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on the barrier at the same offset in both CTAs of the pair once the MMAs issued
+// so far have completed.
+__device__ __forceinline__ void tc_commit_pair_both(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+__device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar) : "memory");
+}
+
+__global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
+    gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
+                     const __grid_constant__ CUtensorMap tm_c, const GemmParams p) {
+  using C = GemmPairCfg;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_base = smem_u32(smem_raw);
+  const uint32_t sbase = (raw_base + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (sbase - raw_base);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();  // 0: issues the MMAs; 1: its peer
+  const int pair = static_cast<int>(blockIdx.x) >> 1, n_pairs = static_cast<int>(gridDim.x) >> 1;
+
+  const uint32_t bar_full = sbase + C::BAR_OFF;
+  const uint32_t bar_empty = bar_full + 8 * C::NSTAGE;
+  const uint32_t bar_acc = bar_empty + 8 * C::NSTAGE;
+  const uint32_t bar_acce = bar_acc + 16;
+  const uint32_t bar_drain = bar_acce + 16;
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::TMEM_PTR_OFF);
+  Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
+  const int tiles = p.tiles_m * p.tiles_n;  // 256 x 256 tiles
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSTAGE; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(bar_acc + 8 * b, 1);
+      mbar_init(bar_acce + 8 * b, 8);  // 4 epilogue warps x 2 CTAs
+    }
+    mbar_init(bar_drain, 1);
+    *ab.flag = 0;
+    *(ab.flag + 1) = 0;
+    fence_barrier_init();
+  }
+  if (warp == 5) tmem_alloc_pair(smem_u32(tmem_ptr), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // both CTAs' barriers initialised, TMEM allocated in both
+  tc_fence_after();
+  const uint32_t tmem = *tmem_ptr;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------------ loader (both CTAs)
+    if (lane == 0) {
+      prefetch_tensormap(&tm_a);
+      prefetch_tensormap(&tm_b);
+      int it = 0, issued = 0, skipped = -1;
+      bool ok = true;
+      for (int t = pair; ok && t < tiles; t += n_pairs) {
+        int tm, tn;
+        tile_coords(p, t, tm, tn);
+        for (int ks = 0; ks < p.k_iters; ++ks, ++it) {
+          const int s = it % C::NSTAGE;
+          if (!(ok = mbar_wait(bar_empty + 8 * s, ((it / C::NSTAGE) & 1) ^ 1, p.ctl, ab))) break;
+          issued = it + 1;
+          if (p.ctl.inject == 3 && it == 2 && rank == 0) {  // test hook: never arm this stage
+            skipped = it;
+            continue;
+          }
+          const uint32_t full0 = map_shared_rank(bar_full + 8 * s, 0);  // the even CTA's barrier
+          if (rank == 0) mbar_expect_tx(bar_full + 8 * s, 2 * C::STAGE_BYTES);
+          const uint32_t dst = sbase + s * C::STAGE_BYTES;
+          tma_load_3d_pair(dst, &tm_a, ks * C::BK, tm * 256 + static_cast<int>(rank) * C::BM, 0, full0);
+#pragma unroll
+          for (int x = 0; x < C::NBH; ++x)
+            tma_load_3d_pair(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b,
+                             tn * C::BN + static_cast<int>(rank) * 128 + x * 64, ks * C::BK, 0, full0);
+        }
+      }
+      if (rank == 0) {  // the even CTA's barriers count both CTAs' copies
+        Abort no_abort{ab.flag + 1};
+        for (int i = max(0, issued - C::NSTAGE); i < issued; ++i)
+          if (i != skipped) mbar_wait(bar_full + 8 * (i % C::NSTAGE), (i / C::NSTAGE) & 1, p.ctl, no_abort);
+      }
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------------ MMA issuer (even CTA)
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_bf16(256, C::BN, 0, 1);
+      const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
+      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, C::B_BOX_BYTES, 1024);
+      constexpr uint32_t kStage16 = C::STAGE_BYTES >> 4;
+      int it = 0, lt = 0;
+      bool ok = true;
+      for (int t = pair; ok && t < tiles; t += n_pairs, ++lt) {
+        const int b = lt & 1, use = lt >> 1;
+        if (lt >= 2 && !(ok = mbar_wait(bar_acce + 8 * b, (use - 1) & 1, p.ctl, ab))) break;
+        tc_fence_after();
+        const uint32_t d = tmem + static_cast<uint32_t>(b * C::BN);
+        for (int ks = 0; ks < p.k_iters; ++ks, ++it) {
+          const int s = it % C::NSTAGE;
+          if (!(ok = mbar_wait(bar_full + 8 * s, (it / C::NSTAGE) & 1, p.ctl, ab))) break;
+          tc_fence_after();
+          const uint64_t da = da0 + s * kStage16, db = db0 + s * kStage16;
+#pragma unroll
+          for (int kk = 0; kk < C::BK / 16; ++kk)
+            mma_ss_pair(d, da + kk * 2, db + kk * 128, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
+          tc_commit_pair_both(bar_empty + 8 * s);
+        }
+        if (!ok) break;
+        tc_commit_pair_both(bar_acc + 8 * b);
+      }
+      Abort no_abort{ab.flag + 1};
+      tc_commit_pair(bar_drain);
+      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue (both CTAs)
+    const uint32_t lane_addr = static_cast<uint32_t>(warp * 32) << 16;
+    const uint32_t stg = sbase + C::STG_OFF + static_cast<uint32_t>(warp) * C::STG_WARP;
+    int lt = 0, chunk = 0;
+    bool ok = true;
+    for (int t = pair; ok && t < tiles; t += n_pairs, ++lt) {
+      int tm, tn;
+      tile_coords(p, t, tm, tn);
+      const int b = lt & 1, use = lt >> 1;
+      if (!(ok = mbar_wait_warp(bar_acc + 8 * b, use & 1, p.ctl, ab))) break;
+      tc_fence_after();
+      const uint32_t src = tmem + lane_addr + static_cast<uint32_t>(b * C::BN);
+      const int row0 = tm * 256 + static_cast<int>(rank) * C::BM + warp * 32;
+#pragma unroll 1
+      for (int c = 0; c < C::BN / 64; ++c) {
+        uint32_t r0[32], r1[32];
+        tmem_ld32(src + c * 64, r0);
+        tmem_ld32(src + c * 64 + 32, r1);
+        tmem_wait_ld();
+        reg_fence32(r0);
+        reg_fence32(r1);
+        if (c == C::BN / 64 - 1) {  // the accumulator is in registers: hand it back
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(map_shared_rank(bar_acce + 8 * b, 0));
+        }
+        if (tn * C::BN + c * 64 >= p.N || row0 >= p.M) continue;
+        uint32_t w[32];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          w[i] = pack_bf16x2(__uint_as_float(r0[2 * i]), __uint_as_float(r0[2 * i + 1]));
+          w[16 + i] = pack_bf16x2(__uint_as_float(r1[2 * i]), __uint_as_float(r1[2 * i + 1]));
+        }
+        const uint32_t buf = stg + static_cast<uint32_t>(chunk & 1) * (32 * 128);
+        ++chunk;
+        if (lane == 0) bulk_wait_group_read1();
+        __syncwarp();
+        const uint32_t row = buf + static_cast<uint32_t>(lane) * 128u;
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          st_shared_v4(row + (static_cast<uint32_t>(q ^ (lane & 7)) << 4), w[4 * q], w[4 * q + 1], w[4 * q + 2],
+                       w[4 * q + 3]);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_3d(&tm_c, buf, tn * C::BN + c * 64, row0, 0);
+          bulk_commit_group();
+        }
+      }
+    }
+    if (lane == 0) bulk_wait_group0();
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // the pair's MMAs, copies and TMEM reads are over in both CTAs
+  if (warp == 5) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, C::TMEM_COLS);
+  }
+}
+
 // ---------------------------------------------------------------- host side
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                    const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -595,6 +836,65 @@ cudaError_t launch_splitk(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t 
   return cudaLaunchKernelEx(&cfg, gemm_splitk_kernel<BN>, ma, mb, p);
 }
 
+bool prepare_pair(int dev) {
+  static int configured = 0;
+  if (dev >= 31) return false;
+  const void* fn = reinterpret_cast<const void*>(gemm_pair_kernel);
+  if (configured & (1 << dev)) return true;
+  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmPairCfg::BYTES) != cudaSuccess)
+    return false;
+  configured |= 1 << dev;
+  return true;
+}
+
+cudaLaunchConfig_t pair_config(int grid, cudaStream_t stream, cudaLaunchAttribute* attr) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
+  cfg.blockDim = dim3(GemmPairCfg::THREADS, 1, 1);
+  cfg.dynamicSmemBytes = GemmPairCfg::BYTES;
+  cfg.stream = stream;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cfg;
+}
+
+// CTAs of CTA pairs that fit on the device at once (0: none, or cannot be queried).
+int pair_slots(int dev) {
+  static int cache[31];  // value + 1 once known
+  if (dev >= 31) return 0;
+  if (cache[dev] != 0) return cache[dev] - 1;
+  int clusters = 0;
+  if (prepare_pair(dev)) {
+    cudaLaunchAttribute attr[1];
+    cudaLaunchConfig_t cfg = pair_config(128, nullptr, attr);
+    if (cudaOccupancyMaxActiveClusters(&clusters, gemm_pair_kernel, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      clusters = 0;
+    }
+  }
+  cache[dev] = 2 * clusters + 1;
+  return 2 * clusters;
+}
+
+cudaError_t launch_pair(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int dev) {
+  const int slots = pair_slots(dev);
+  if (slots < 2 || !prepare_pair(dev)) return cudaErrorInvalidConfiguration;
+  CUtensorMap ma, mb, mc;
+  if (!make_maps(a, GemmPairCfg::BM, &ma, &mb, &mc)) return cudaErrorInvalidValue;
+  GemmParams p = make_params(a, ctl, GemmPairCfg::BN, 1);
+  p.tiles_m = (a.M + 255) / 256;  // 256-row tiles of the pair
+  const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
+  if (tiles > 0x3fffffffLL) return cudaErrorInvalidConfiguration;
+  const long long pairs = tiles < slots / 2 ? tiles : slots / 2;
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = pair_config(static_cast<int>(2 * pairs), stream, attr);
+  return cudaLaunchKernelEx(&cfg, gemm_pair_kernel, ma, mb, mc, p);
+}
+
 bool device_sms(int* dev, int* sms) {
   if (cudaGetDevice(dev) != cudaSuccess) return false;
   return cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, *dev) == cudaSuccess && *sms > 0;
@@ -607,15 +907,16 @@ GemmChoice gemm_choice(int M, int N, int K, GemmChoice forced) {
   if (!device_sms(&dev, &sms)) return {0, 0};
   const model::GemmChoiceModel c = model::gemm_choose(
       M, N, K, sms, [dev](int bn, int S) { return splitk_slots_any(dev, bn, S); }, model::kGb300, forced.tile_n,
-      forced.splits);
-  return {c.bn, c.splits};
+      forced.splits, forced.pair >= 0 ? pair_slots(dev) : 0, forced.pair);
+  return {c.bn, c.splits, c.pair ? 1 : 0};
 }
 
 cudaError_t launch_gemm(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
   int dev = 0, sms = 0;
   if (!device_sms(&dev, &sms)) return cudaErrorNoDevice;
-  const GemmChoice c = gemm_choice(a.M, a.N, a.K, {a.tile_n, a.splits});
+  const GemmChoice c = gemm_choice(a.M, a.N, a.K, {a.tile_n, a.splits, a.pair});
   if (c.tile_n == 0) return cudaErrorInvalidConfiguration;
+  if (c.pair == 1) return launch_pair(a, ctl, stream, dev);
   if (c.splits > 1) {
     switch (c.tile_n) {
       case 64: return launch_splitk<64>(a, ctl, stream, dev, c.splits);

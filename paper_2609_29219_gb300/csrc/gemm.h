@@ -14,15 +14,18 @@ struct GemmArgs {
   int M, N, K;
   int tile_n;     // 0: the analytic model's choice, else 64, 128, 192 or 256
   int splits;     // 0: the model's choice, else 1 (persistent tiles) or 2, 4, 8, 16 (split-K clusters)
+  int pair;       // 0: the model's choice, 1: CTA-pair 256 x 256 tiles, -1: never CTA pairs
 };
 
 struct GemmChoice {
   int tile_n, splits;
+  int pair;  // as a choice: 1 = CTA-pair tiles; as a restriction: see GemmArgs::pair
 };
 
 cudaError_t launch_gemm(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream);
-// The model's (tile width, split count) for this shape on the current device; fields of
-// `forced` that are non-zero are kept.  {0, 0} if the device cannot be queried.
+// The model's (tile width, split count, CTA pair) for this shape on the current device;
+// fields of `forced` that are non-zero restrict the choice.  tile_n = 0 if the device
+// cannot be queried or nothing fits the restriction.
 GemmChoice gemm_choice(int M, int N, int K, GemmChoice forced);
 
 }  // namespace loom

@@ -16,10 +16,18 @@ namespace model {
 struct GemmPlan {
   int bm, bn, bk, stages, smem_bytes, tmem_cols;
   double t_load_ns, t_mma_ns, t_iter_ns, t_epi_ns;
+  double t_epi_tile_ns;  // the epilogue's time for one tile: it bounds the tile rate when K is short
   bool feasible;
 };
 
 constexpr int kGemmStagingBytes = 4 * 2 * 32 * 128;  // 4 epilogue warps x 2 buffers x 32 rows x 128 B
+// Epilogue of one tile by the four epilogue warps: a fixed part plus one 64-column chunk
+// (TMEM -> registers -> bf16 -> staging -> TMA store) at a time, and the extra cost of a
+// CTA pair's cross-SM accumulator release (fitted to K = 256 tiles: 128 x 256 take 2.8 us,
+// 128 x 128 1.55 us, and a pair's 128 x 256 per SM 3.4 us).
+constexpr double kGemmEpiTileNs = 400.0;
+constexpr double kGemmEpiChunkNs = 600.0;
+constexpr double kGemmPairEpiFactor = 1.2;
 
 constexpr GemmPlan gemm_eval(const ArchDesc& a, int bn, int stages) {
   GemmPlan p{};
@@ -32,6 +40,7 @@ constexpr GemmPlan gemm_eval(const ArchDesc& a, int bn, int stages) {
   p.t_mma_ns = (p.bk / 16.0) * dmax(a.mma_clk_per_n * bn, a.mma_min_clk) / a.sm_ghz;
   p.t_iter_ns = heg_pipe(p.t_load_ns, p.t_mma_ns, 0.0, 1, 0);
   p.t_epi_ns = p.bm * bn * 2.0 / a.l2_smem_gbs_sm;  // the C tile leaves through L2
+  p.t_epi_tile_ns = kGemmEpiTileNs + (bn / 64) * kGemmEpiChunkNs;
   p.smem_bytes = static_cast<int>(stages * stage_bytes) + kGemmStagingBytes + 1024 + 256;
   p.tmem_cols = 2 * bn;
   p.feasible = p.smem_bytes <= a.smem_per_cta && p.tmem_cols <= a.tmem_cols && stages >= 2 && bn % 64 == 0 &&
@@ -60,7 +69,10 @@ constexpr double gemm_time_us(const GemmPlan& p, long long M, long long N, long 
                               const ArchDesc& a = kGb300) {
   const long long tiles = cdiv(M, p.bm) * cdiv(N, p.bn);
   const long long per_sm = cdiv(tiles, num_sms);
-  const double t = heg_seq(heg_seq(p.t_load_ns, heg_for(per_sm * cdiv(K, p.bk), p.t_iter_ns)), p.t_epi_ns);
+  // the next tile's K loop overlaps this tile's epilogue (two accumulators): a tile takes
+  // the longer of the two
+  const double t_tile = dmax(heg_for(cdiv(K, p.bk), p.t_iter_ns), p.t_epi_tile_ns);
+  const double t = heg_seq(heg_seq(p.t_load_ns, heg_for(per_sm, t_tile)), p.t_epi_ns);
   return (t + a.launch_ns * 0.2) * 1e-3;
 }
 
@@ -121,12 +133,55 @@ constexpr bool gemm_split_supported(int S) { return S == 1 || S == 2 || S == 4 |
 struct GemmChoiceModel {
   int bn, splits;
   double t_us;
+  bool pair;  // CTA-pair 256 x 256 tiles (bn = 256, splits = 1)
 };
 
+// ------------------------------------------------------------------ CTA pairs
+// Two CTAs of a cluster compute a 256 x 256 tile with one M = 256 MMA stream: each SM
+// loads its 128 rows of A and half of B, (128 + 128) x 64 x 2 = 32 KB per K stage, against
+// the same four 128 x 256 x 16 MMAs per SM as a 128 x 256 single-CTA tile (48 KB).
+constexpr GemmPlan gemm_pair_plan(const ArchDesc& a = kGb300) {
+  GemmPlan p{};
+  p.bm = 256;
+  p.bn = 256;
+  p.bk = 64;
+  p.stages = 6;
+  const double stage_bytes = (128 + 128) * p.bk * 2.0;
+  p.t_load_ns = stage_bytes / a.l2_smem_gbs_sm;
+  p.t_mma_ns = (p.bk / 16.0) * dmax(a.mma_clk_per_n * 256, a.mma_min_clk) / a.sm_ghz;
+  p.t_iter_ns = heg_pipe(p.t_load_ns, p.t_mma_ns, 0.0, 1, 0);
+  p.t_epi_ns = 128 * 256 * 2.0 / a.l2_smem_gbs_sm;
+  p.t_epi_tile_ns = (kGemmEpiTileNs + (256 / 64) * kGemmEpiChunkNs) * kGemmPairEpiFactor;
+  p.smem_bytes = static_cast<int>(p.stages * stage_bytes) + kGemmStagingBytes + 1024 + 256;
+  p.tmem_cols = 512;
+  p.feasible = p.smem_bytes <= a.smem_per_cta && p.tmem_cols <= a.tmem_cols;
+  return p;
+}
+
+// `pair_ctas` CTAs (whole pairs) fit on the GPU at once.
+constexpr double gemm_pair_time_us(long long M, long long N, long long K, int pair_ctas, const ArchDesc& a = kGb300) {
+  const GemmPlan p = gemm_pair_plan(a);
+  const long long tiles = cdiv(M, 256) * cdiv(N, 256);
+  const long long pairs = pair_ctas / 2 > 0 ? pair_ctas / 2 : 1;
+  const long long per_pair = cdiv(tiles, pairs);
+  const double t_tile = dmax(heg_for(cdiv(K, p.bk), p.t_iter_ns), p.t_epi_tile_ns);
+  const double t = heg_seq(heg_seq(p.t_load_ns, heg_for(per_pair, t_tile)), p.t_epi_ns);
+  return (t + a.launch_ns * 0.2) * 1e-3;
+}
+
+// Eq. 9 over the kernel variants.  only_pair: 0 = the model decides, 1 = the pair kernel
+// only, -1 = never the pair kernel.
 template <typename SlotsFn>
 constexpr GemmChoiceModel gemm_choose(long long M, long long N, long long K, int num_sms, SlotsFn slots,
-                                      const ArchDesc& a = kGb300, int only_bn = 0, int only_splits = 0) {
-  GemmChoiceModel best{0, 0, 1e300};
+                                      const ArchDesc& a = kGb300, int only_bn = 0, int only_splits = 0,
+                                      int pair_ctas = 0, int only_pair = 0) {
+  GemmChoiceModel best{0, 0, 1e300, false};
+  if (only_pair >= 0 && pair_ctas >= 2 && (only_bn == 0 || only_bn == 256) && only_splits <= 1 &&
+      gemm_pair_plan(a).feasible) {
+    best = {256, 1, gemm_pair_time_us(M, N, K, pair_ctas, a), true};
+    if (only_pair == 1) return best;
+  }
+  if (only_pair == 1) return GemmChoiceModel{0, 0, 1e300, false};
   for (int bn = 256; bn >= 64; bn -= 64) {
     if (only_bn != 0 && bn != only_bn) continue;
     const GemmPlan p = gemm_plan_variant(bn, a);
@@ -142,7 +197,7 @@ constexpr GemmChoiceModel gemm_choose(long long M, long long N, long long K, int
         if (s <= 0) continue;
         t = gemm_splitk_time_us(p, M, N, K, S, s, a);
       }
-      if (t < best.t_us * (1.0 - 1e-9)) best = {bn, S, t};
+      if (t < best.t_us * (1.0 - 1e-9)) best = {bn, S, t, false};
     }
   }
   return best;

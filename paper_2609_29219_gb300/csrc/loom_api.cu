@@ -27,6 +27,7 @@ int g_inject = 0;
 int g_prefill_design = 0;
 int g_gemm_tile_n = 0;  // test hook: forced GEMM tile width (0: the model's choice)
 int g_gemm_splits = 0;  // test hook: forced GEMM split count (0: the model's choice)
+int g_gemm_pair = 0;    // test hook: 1 forces CTA-pair tiles, -1 forbids them, 0: the model's choice
 
 constexpr int kMaxDevices = 64;
 uint32_t* g_err_ptr[kMaxDevices] = {};
@@ -249,7 +250,7 @@ loom_status loom_gemm_bf16(const void* a, const void* b, void* c, int M, int N, 
   if (K % 8 != 0 || N % 8 != 0) return LOOM_ERR_UNSUPPORTED;  // 16-byte row strides for TMA
   KernelCtl ctl;
   if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
-  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n, g_gemm_splits};
+  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n, g_gemm_splits, g_gemm_pair};
   return launch_gemm(g, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK : LOOM_ERR_CUDA;
 }
 
@@ -263,23 +264,30 @@ GemmChoice gemm_choice_any(int M, int N, int K, GemmChoice forced) {
   const int sms = model::kGb300.num_sms;
   const model::GemmChoiceModel m = model::gemm_choose(
       M, N, K, sms, [sms](int, int S) { return model::gemm_default_slots(sms, S); }, model::kGb300,
-      forced.tile_n, forced.splits);
-  return {m.bn, m.splits};
+      forced.tile_n, forced.splits, forced.pair >= 0 ? model::gemm_default_slots(sms, 2) : 0, forced.pair);
+  return {m.bn, m.splits, m.pair ? 1 : 0};
 }
 }  // namespace
 
 int loom_gemm_tile_n(int M, int N, int K) {
   if (M <= 0 || N <= 0 || K <= 0) return 0;
-  return gemm_choice_any(M, N, K, {g_gemm_tile_n, g_gemm_splits}).tile_n;
+  return gemm_choice_any(M, N, K, {g_gemm_tile_n, g_gemm_splits, g_gemm_pair}).tile_n;
 }
 
 int loom_gemm_splits(int M, int N, int K) {
   if (M <= 0 || N <= 0 || K <= 0) return 0;
-  return gemm_choice_any(M, N, K, {g_gemm_tile_n, g_gemm_splits}).splits;
+  return gemm_choice_any(M, N, K, {g_gemm_tile_n, g_gemm_splits, g_gemm_pair}).splits;
+}
+
+int loom_gemm_cta_pair(int M, int N, int K) {
+  if (M <= 0 || N <= 0 || K <= 0) return 0;
+  return gemm_choice_any(M, N, K, {g_gemm_tile_n, g_gemm_splits, g_gemm_pair}).pair;
 }
 
 double loom_model_gemm_time_us(int M, int N, int K, int tile_n, int splits, int num_sms) {
   if (M <= 0 || N <= 0 || K <= 0 || num_sms <= 0) return -1.0;
+  if (tile_n == 512 && splits == 1)  // CTA-pair 256 x 256 tiles
+    return model::gemm_pair_time_us(M, N, K, model::gemm_default_slots(num_sms, 2));
   if (tile_n != 64 && tile_n != 128 && tile_n != 192 && tile_n != 256) return -1.0;
   if (!model::gemm_split_supported(splits)) return -1.0;
   const model::GemmPlan p = model::gemm_plan_variant(tile_n);
@@ -293,6 +301,8 @@ void loom_debug_gemm_tile_n(int tile_n) {
 }
 
 void loom_debug_gemm_splits(int splits) { g_gemm_splits = model::gemm_split_supported(splits) ? splits : 0; }
+
+void loom_debug_gemm_cta_pair(int mode) { g_gemm_pair = (mode == 1 || mode == -1) ? mode : 0; }
 
 loom_status loom_attn_check_error(void* stream) {
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return LOOM_ERR_CUDA;

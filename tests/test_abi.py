@@ -134,6 +134,16 @@ def test_gemm_splits_only_when_tiles_are_few(lib):
     assert lib.loom_model_gemm_time_us(256, 256, 16384, 96, 1, 152) < 0  # unsupported width
 
 
+def test_gemm_pair_tiles_for_large_shapes(lib):
+    # operand traffic per SM decides: CTA pairs for large C, never for a single K stage tile
+    assert lib.loom_gemm_cta_pair(16384, 16384, 16384) == 1
+    assert lib.loom_gemm_tile_n(16384, 16384, 16384) == 256
+    assert lib.loom_gemm_cta_pair(256, 256, 16384) == 0
+    tp = lib.loom_model_gemm_time_us(16384, 16384, 16384, 512, 1, 152)
+    t1 = lib.loom_model_gemm_time_us(16384, 16384, 16384, 256, 1, 152)
+    assert 0 < tp < t1
+
+
 def test_paged_decode_rejects_bad_arguments(lib):
     ok = dict(q=FAKE, k=FAKE, v=FAKE, tbl=FAKE, sl=FAKE, o=FAKE, lse=None, ws=FAKE, wsb=1 << 24, B=2, Hq=8,
               Hkv=2, npages=64, P=16, maxp=8, D=128, scale=0.08, splits=4, stream=None)

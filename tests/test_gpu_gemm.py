@@ -28,20 +28,27 @@ def loom():
     yield m
     m.loom_debug_gemm_tile_n(0)
     m.loom_debug_gemm_splits(0)
+    m.loom_debug_gemm_cta_pair(0)
     m.loom_debug_inject(0)
     m.loom_debug_set_timeout_ns(0)
 
 
 @pytest.fixture
 def forced(loom):
-    """forced(tile_n, splits): pin the kernel variant for one test (0 = the model's choice)."""
-    def set_(tile_n=0, splits=0):
+    """forced(tile_n, splits, pair): pin the kernel variant for one test (0 = the model's
+    choice; pair 1 = CTA-pair 256 x 256 tiles, -1 = single-CTA kernels only)."""
+    def set_(tile_n=0, splits=0, pair=None):
+        if pair is None:
+            pair = -1 if (tile_n or splits) else 0
         loom.loom_debug_gemm_tile_n(tile_n)
         loom.loom_debug_gemm_splits(splits)
+        loom.loom_debug_gemm_cta_pair(pair)
         assert tile_n == 0 or loom.loom_gemm_tile_n(8, 8, 8) == tile_n
+        assert pair != 1 or loom.loom_gemm_cta_pair(8, 8, 8) == 1
     yield set_
     loom.loom_debug_gemm_tile_n(0)
     loom.loom_debug_gemm_splits(0)
+    loom.loom_debug_gemm_cta_pair(0)
 
 
 def _inputs(seed, M, K, N):
@@ -67,19 +74,25 @@ def _run(loom, a, b):
 
 
 # ---------------------------------------------------------------- persistent tiles (S = 1)
-@pytest.mark.parametrize("tile_n", [0, *TILE_WIDTHS], ids=["model", *[f"bn{b}" for b in TILE_WIDTHS]])
+@pytest.mark.parametrize("tile_n", [0, *TILE_WIDTHS, "pair"], ids=["model", *[f"bn{b}" for b in TILE_WIDTHS], "pair"])
 @pytest.mark.parametrize("M,K,N", [(128, 64, 256), (1, 8, 8), (200, 136, 304), (130, 72, 264), (255, 1000, 520),
-                                   (1000, 1000, 1000), (64, 4096, 64), (2048, 256, 256)])
+                                   (1000, 1000, 1000), (64, 4096, 64), (2048, 256, 256), (384, 320, 768)])
 def test_full_parity(loom, forced, tile_n, M, K, N):
-    forced(tile_n, 1 if tile_n else 0)
+    if tile_n == "pair":
+        forced(0, 0, 1)
+    else:
+        forced(tile_n, 1 if tile_n else 0)
     a, b = _inputs(M + K + N, M, K, N)
     _check(_run(loom, a, b), oracle.gemm(a, b), K, f"{M}x{K}x{N} bn={tile_n}")
 
 
-@pytest.mark.parametrize("tile_n", [0, 64, 256], ids=["model", "bn64", "bn256"])
+@pytest.mark.parametrize("tile_n", [0, 64, 256, "pair"], ids=["model", "bn64", "bn256", "pair"])
 @pytest.mark.parametrize("M,K,N", [(4096, 4096, 4096), (8192, 2048, 1024)])
 def test_large_sampled_rows(loom, forced, tile_n, M, K, N):
-    forced(tile_n, 1 if tile_n else 0)
+    if tile_n == "pair":
+        forced(0, 0, 1)
+    else:
+        forced(tile_n, 1 if tile_n else 0)
     a, b = _inputs(7, M, K, N)
     c = _run(loom, a, b)
     rng = np.random.default_rng(0)
@@ -117,9 +130,12 @@ def test_model_choice_long_k(loom, forced, M, K, N):
            f"{M}x{K}x{N} model bn={loom.loom_gemm_tile_n(M, N, K)} S={loom.loom_gemm_splits(M, N, K)}")
 
 
-@pytest.mark.parametrize("splits", [1, 4, 16])
+@pytest.mark.parametrize("splits", [1, 4, 16, "pair"])
 def test_deterministic(loom, forced, splits):
-    forced(128, splits)
+    if splits == "pair":
+        forced(0, 0, 1)
+    else:
+        forced(128, splits)
     a, b = _inputs(13, 384, 4096, 512)
     ad, bd = to_dev(a), to_dev(b)
     import torch
@@ -133,18 +149,19 @@ def test_identity_and_zeros(loom, forced):
     eye = np.zeros((K, K), np.uint16)
     eye[np.arange(K), np.arange(K)] = 0x3F80
     b = synth.bf16_normal(3, synth.STREAM_V, (K, N))
-    for tile_n, splits in [(0, 0), (64, 2), (256, 4)]:
-        forced(tile_n, splits)
+    for tile_n, splits, pair in [(0, 0, 0), (64, 2, -1), (256, 4, -1), (0, 0, 1)]:
+        forced(tile_n, splits, pair)
         np.testing.assert_array_equal(_run(loom, eye, b), oracle.bf16_to_f64(b))  # one product per entry
         np.testing.assert_array_equal(_run(loom, eye, np.zeros((K, N), np.uint16)), 0.0)
 
 
 # ---------------------------------------------------------------- bounded waits
-@pytest.mark.parametrize("tile_n,splits", [(256, 1), (64, 4)])
-def test_timeout_is_reported_and_context_survives(loom, forced, tile_n, splits):
-    """The loader skips one stage (per CTA); the waits on it run out, every CTA (and, split,
-    every cluster) unwinds, the error word says TIMEOUT, and the next call is correct."""
-    forced(tile_n, splits)
+@pytest.mark.parametrize("tile_n,splits,pair", [(256, 1, -1), (64, 4, -1), (0, 0, 1)])
+def test_timeout_is_reported_and_context_survives(loom, forced, tile_n, splits, pair):
+    """The loader skips one stage (per CTA; for CTA pairs the even CTA never arms it); the
+    waits on it run out, every CTA (and every cluster) unwinds, the error word says TIMEOUT,
+    and the next call is correct."""
+    forced(tile_n, splits, pair)
     M, K, N = 256, 1024, 512
     a, b = _inputs(11, M, K, N)
     ad, bd = to_dev(a), to_dev(b)
