@@ -4,16 +4,17 @@
 // Persistent CTAs walk the output tiles (BM = 128 rows x BN columns) in groups of 8 tile
 // rows, so that CTAs working at the same time share A rows and B columns in L2:
 //
-//   warp 4 (loader, 1 thread)   A tile 128 x 64 and B tile 64 x BN per K stage into an
+//   warp 8 (loader, 1 thread)   A tile 128 x 64 and B tile 64 x BN per K stage into an
 //                               NSTAGE-deep ring of 128B-swizzled slots (TMA, full/empty
 //                               mbarriers)
-//   warp 5 (MMA, 1 thread)      tcgen05.mma kind::f16, M = 128, N = BN, K = 16: A K-major,
+//   warp 9 (MMA, 1 thread)      tcgen05.mma kind::f16, M = 128, N = BN, K = 16: A K-major,
 //                               B MN-major (rows of B are contiguous in N), fp32 into one of
 //                               two TMEM accumulators
-//   warps 0-3 (epilogue)        thread = row of the tile (= TMEM lane): fp32 -> bf16 in
-//                               64-column chunks, staged per warp in shared memory and
-//                               stored with TMA; the accumulator is released as soon as it
-//                               is in registers, so the next-but-one tile may reuse it.
+//   warps 0-7 (epilogue)        warp w reads TMEM lanes 32 (w mod 4) .. + 31 (its 32 rows
+//                               of the tile) and every other 64-column chunk from w div 4:
+//                               fp32 -> bf16, staged per warp in shared memory and stored
+//                               with TMA; the accumulator is released as soon as it is in
+//                               registers, so the next-but-one tile may reuse it.
 //
 // TMEM: [0, BN) accumulator 0 | [BN, 2 BN) accumulator 1.
 #include <cuda.h>
@@ -27,11 +28,6 @@
 
 namespace loom {
 namespace {
-
-// Wait until at most one committed bulk store of this thread has not yet read its source.
-__device__ __forceinline__ void bulk_wait_group_read1() {
-  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-}
 
 // ---------------------------------------------------------------- cluster primitives
 __device__ __forceinline__ uint32_t cluster_ctarank() {
@@ -50,6 +46,10 @@ __device__ __forceinline__ uint32_t map_shared_rank(uint32_t saddr, uint32_t ran
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
   return r;
 }
+// Arrive on an mbarrier of any CTA of the cluster (a shared::cluster address).
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar) : "memory");
+}
 __device__ __forceinline__ float4 ld_dsmem_f4(uint32_t addr) {
   float4 v;
   asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
@@ -65,14 +65,15 @@ struct GemmCfg {
   static_assert(kPlan.feasible, "no feasible GEMM plan for this tile width");
   static constexpr int BM = 128, BK = 64;
   static constexpr int NSTAGE = kPlan.stages;
-  static constexpr int THREADS = 192;                       // 4 epilogue warps, loader, MMA
+  static constexpr int THREADS = 320;                       // 8 epilogue warps, loader, MMA
+  static constexpr int SPLIT_THREADS = 192;                 // split-K: 4 epilogue warps, loader, MMA
   static constexpr int NB = BN / 64;                        // 64-column boxes of a B stage
   static constexpr uint32_t A_BYTES = BM * BK * 2;          // one 128B-swizzled box
   static constexpr uint32_t B_BOX_BYTES = BK * 64 * 2;      // 64 K-rows x 64 N-columns
   static constexpr uint32_t STAGE_BYTES = A_BYTES + NB * B_BOX_BYTES;
   static constexpr uint32_t STG_OFF = NSTAGE * STAGE_BYTES;  // epilogue staging
-  static constexpr uint32_t STG_WARP = 2 * 32 * 128;         // 2 buffers x 32 rows x 128 B
-  static constexpr uint32_t BAR_OFF = STG_OFF + 4 * STG_WARP;
+  static constexpr uint32_t STG_WARP = 32 * 128;             // one 32-row x 128 B block per warp
+  static constexpr uint32_t BAR_OFF = STG_OFF + 8 * STG_WARP;
   // barriers: full[NSTAGE], empty[NSTAGE], acc_full[2], acc_empty[2], drain
   static constexpr int NBAR = 2 * NSTAGE + 5;
   static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
@@ -80,7 +81,7 @@ struct GemmCfg {
   static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;  // + alignment slack
   static constexpr uint32_t TMEM_COLS = 2 * BN <= 32 ? 32 : 2 * BN <= 64 ? 64 : 2 * BN <= 128 ? 128
                                         : 2 * BN <= 256 ? 256 : 512;
-  static_assert(STG_WARP * 4 == model::kGemmStagingBytes, "staging layout matches the model");
+  static_assert(STG_WARP * 8 == model::kGemmStagingBytes, "staging layout matches the model");
   static_assert(BYTES <= 227 * 1024, "shared memory budget");
 };
 
@@ -102,6 +103,65 @@ __device__ __forceinline__ void tile_coords(const GemmParams& p, int t, int& tm,
   const int in = t - g * per_group;
   tm = first + in % rows;
   tn = in / rows;
+}
+
+// One epilogue warp's share of a finished accumulator: its 32 TMEM lanes (rows row0 ..
+// row0 + 31 of C) and the 64-column chunks c = h, h + 2, ... < NB of the accumulator at
+// `acc`.  Once its last chunk is in registers the warp arrives on `release` (the even
+// CTA's barrier, over the cluster, when `remote`), so the MMA warp may reuse the
+// accumulator while the stores drain.  A chunk goes through the warp's 4 KB staging block
+// (128B-swizzled like the TMA box) and leaves with a TMA store; chunks wholly outside C
+// are not stored.
+template <int NB>
+__device__ __forceinline__ void epilogue_warp(const CUtensorMap* tm_c, uint32_t acc, uint32_t stg, int h, int col0,
+                                              int row0, int M, int N, uint32_t release, bool remote) {
+  const int lane = threadIdx.x & 31;
+  bool released = false;
+#pragma unroll 1
+  for (int c = h; c < NB; c += 2) {
+    uint32_t r0[32], r1[32];
+    tmem_ld32(acc + c * 64, r0);
+    tmem_ld32(acc + c * 64 + 32, r1);
+    tmem_wait_ld();
+    reg_fence32(r0);
+    reg_fence32(r1);
+    if (c + 2 >= NB) {
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (remote) mbar_arrive_cluster(release);
+        else mbar_arrive(release);
+      }
+      released = true;
+    }
+    if (col0 + c * 64 >= N || row0 >= M) continue;
+    uint32_t w[32];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      w[i] = pack_bf16x2(__uint_as_float(r0[2 * i]), __uint_as_float(r0[2 * i + 1]));
+      w[16 + i] = pack_bf16x2(__uint_as_float(r1[2 * i]), __uint_as_float(r1[2 * i + 1]));
+    }
+    if (lane == 0) bulk_wait_group_read0();  // this warp's previous store has read the block
+    __syncwarp();
+    const uint32_t row = stg + static_cast<uint32_t>(lane) * 128u;
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      st_shared_v4(row + (static_cast<uint32_t>(q ^ (lane & 7)) << 4), w[4 * q], w[4 * q + 1], w[4 * q + 2],
+                   w[4 * q + 3]);
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_3d(tm_c, stg, col0 + c * 64, row0, 0);
+      bulk_commit_group();
+    }
+  }
+  if (!released) {  // no chunk for this warp (a 64-column tile): nothing read, release at once
+    __syncwarp();
+    if (lane == 0) {
+      if (remote) mbar_arrive_cluster(release);
+      else mbar_arrive(release);
+    }
+  }
 }
 
 template <int BN>
@@ -131,20 +191,20 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(bar_acc + 8 * b, 1);
-      mbar_init(bar_acce + 8 * b, C::BM);
+      mbar_init(bar_acce + 8 * b, 8);  // one arrive per epilogue warp
     }
     mbar_init(bar_drain, 1);
     *ab.flag = 0;
     *(ab.flag + 1) = 0;
     fence_barrier_init();
   }
-  if (warp == 5) tmem_alloc(smem_u32(tmem_ptr), C::TMEM_COLS);
+  if (warp == 9) tmem_alloc(smem_u32(tmem_ptr), C::TMEM_COLS);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_ptr;
 
-  if (warp == 4) {
+  if (warp == 8) {
     // ------------------------------------------------------------------ loader
     if (lane == 0) {
       prefetch_tensormap(&tm_a);
@@ -175,7 +235,7 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
       for (int i = max(0, issued - C::NSTAGE); i < issued; ++i)
         if (i != skipped) mbar_wait(bar_full + 8 * (i % C::NSTAGE), (i / C::NSTAGE) & 1, p.ctl, no_abort);
     }
-  } else if (warp == 5) {
+  } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(C::BM, BN, 0, 1);  // A K-major, B MN-major
@@ -211,10 +271,11 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
       mbar_wait(bar_drain, 0, p.ctl, no_abort);
     }
   } else {
-    // ------------------------------------------------------------------ epilogue
-    const uint32_t lane_addr = static_cast<uint32_t>(warp * 32) << 16;
+    // ------------------------------------------------------------------ epilogue (warps 0-7)
+    const int quarter = warp & 3, half = warp >> 2;
+    const uint32_t lane_addr = static_cast<uint32_t>(quarter * 32) << 16;
     const uint32_t stg = sbase + C::STG_OFF + static_cast<uint32_t>(warp) * C::STG_WARP;
-    int lt = 0, chunk = 0;
+    int lt = 0;
     bool ok = true;
     for (int t = blockIdx.x; ok && t < tiles; t += gridDim.x, ++lt) {
       int tm, tn;
@@ -222,44 +283,8 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
       const int b = lt & 1, use = lt >> 1;
       if (!(ok = mbar_wait_warp(bar_acc + 8 * b, use & 1, p.ctl, ab))) break;
       tc_fence_after();
-      const uint32_t src = tmem + lane_addr + static_cast<uint32_t>(b * BN);
-#pragma unroll 1
-      for (int c = 0; c < C::NB; ++c) {
-        uint32_t r0[32], r1[32];
-        tmem_ld32(src + c * 64, r0);
-        tmem_ld32(src + c * 64 + 32, r1);
-        tmem_wait_ld();
-        reg_fence32(r0);
-        reg_fence32(r1);
-        if (c == C::NB - 1) {  // the accumulator is in registers: hand it back
-          tc_fence_before();
-          mbar_arrive(bar_acce + 8 * b);
-        }
-        // a chunk lying wholly outside C stores nothing (and takes no staging buffer)
-        if (tn * BN + c * 64 >= p.N || tm * C::BM + warp * 32 >= p.M) continue;
-        uint32_t w[32];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          w[i] = pack_bf16x2(__uint_as_float(r0[2 * i]), __uint_as_float(r0[2 * i + 1]));
-          w[16 + i] = pack_bf16x2(__uint_as_float(r1[2 * i]), __uint_as_float(r1[2 * i + 1]));
-        }
-        // staging buffer chunk % 2: the store issued from it two stored chunks ago has read it
-        const uint32_t buf = stg + static_cast<uint32_t>(chunk & 1) * (32 * 128);
-        ++chunk;
-        if (lane == 0) bulk_wait_group_read1();
-        __syncwarp();
-        const uint32_t row = buf + static_cast<uint32_t>(lane) * 128u;
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          st_shared_v4(row + (static_cast<uint32_t>(q ^ (lane & 7)) << 4), w[4 * q], w[4 * q + 1], w[4 * q + 2],
-                       w[4 * q + 3]);
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) {
-          tma_store_3d(&tm_c, buf, tn * BN + c * 64, tm * C::BM + warp * 32, 0);
-          bulk_commit_group();
-        }
-      }
+      epilogue_warp<C::NB>(&tm_c, tmem + lane_addr + static_cast<uint32_t>(b * BN), stg, half, tn * BN,
+                           tm * C::BM + quarter * 32, p.M, p.N, bar_acce + 8 * b, false);
     }
     if (lane == 0) bulk_wait_group0();  // the C stores have completed before the CTA exits
   }
@@ -267,7 +292,7 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
   __syncwarp();
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == 9) {
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
@@ -284,7 +309,7 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
 // peers have read it.  The summation order does not depend on timing, so the result is
 // deterministic for a given S.
 template <int BN>
-__global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
+__global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
     gemm_splitk_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                        const GemmParams p) {
   using C = GemmCfg<BN>;
@@ -452,19 +477,19 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
 // its 128 rows x 256 columns of the accumulator.  Per K stage an SM thus loads 32 KB
 // instead of the 48 KB of a 128 x 256 single-CTA tile, and six stages fit.  Both CTAs'
 // copies complete on the even CTA's full barrier (armed once for 64 KB); the even CTA's
-// commits signal stage-free and accumulator-ready on both CTAs at once; each CTA's four
-// epilogue warps tell the even CTA that an accumulator has been read (8 arrivals).
+// commits signal stage-free and accumulator-ready on both CTAs at once; each CTA's eight
+// epilogue warps tell the even CTA that an accumulator has been read (16 arrivals).
 struct GemmPairCfg {
   static constexpr int BM = 128, BN = 256, BK = 64;   // per CTA: 128 rows x 256 columns of C
   static constexpr int NSTAGE = 6;
-  static constexpr int THREADS = 192;
+  static constexpr int THREADS = 320;                  // 8 epilogue warps, loader, MMA
   static constexpr int NBH = 2;                        // 64-column boxes of this CTA's half of B
   static constexpr uint32_t A_BYTES = BM * BK * 2;
   static constexpr uint32_t B_BOX_BYTES = BK * 64 * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + NBH * B_BOX_BYTES;  // 32 KB
   static constexpr uint32_t STG_OFF = NSTAGE * STAGE_BYTES;
-  static constexpr uint32_t STG_WARP = 2 * 32 * 128;
-  static constexpr uint32_t BAR_OFF = STG_OFF + 4 * STG_WARP;
+  static constexpr uint32_t STG_WARP = 32 * 128;
+  static constexpr uint32_t BAR_OFF = STG_OFF + 8 * STG_WARP;
   static constexpr int NBAR = 2 * NSTAGE + 5;  // full, empty, acc_full[2], acc_empty[2], drain
   static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
   static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
@@ -511,9 +536,6 @@ __device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
                : "memory");
 }
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_bar) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar) : "memory");
-}
 
 __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
@@ -543,21 +565,21 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(bar_acc + 8 * b, 1);
-      mbar_init(bar_acce + 8 * b, 8);  // 4 epilogue warps x 2 CTAs
+      mbar_init(bar_acce + 8 * b, 16);  // 8 epilogue warps x 2 CTAs
     }
     mbar_init(bar_drain, 1);
     *ab.flag = 0;
     *(ab.flag + 1) = 0;
     fence_barrier_init();
   }
-  if (warp == 5) tmem_alloc_pair(smem_u32(tmem_ptr), C::TMEM_COLS);
+  if (warp == 9) tmem_alloc_pair(smem_u32(tmem_ptr), C::TMEM_COLS);
   tc_fence_before();
   __syncthreads();
   cluster_sync_all();  // both CTAs' barriers initialised, TMEM allocated in both
   tc_fence_after();
   const uint32_t tmem = *tmem_ptr;
 
-  if (warp == 4) {
+  if (warp == 8) {
     // ------------------------------------------------------------------ loader (both CTAs)
     if (lane == 0) {
       prefetch_tensormap(&tm_a);
@@ -591,7 +613,7 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
           if (i != skipped) mbar_wait(bar_full + 8 * (i % C::NSTAGE), (i / C::NSTAGE) & 1, p.ctl, no_abort);
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer (even CTA)
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = idesc_bf16(256, C::BN, 0, 1);
@@ -623,10 +645,11 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
       mbar_wait(bar_drain, 0, p.ctl, no_abort);
     }
   } else {
-    // ------------------------------------------------------------------ epilogue (both CTAs)
-    const uint32_t lane_addr = static_cast<uint32_t>(warp * 32) << 16;
+    // ------------------------------------------------------------------ epilogue (both CTAs, warps 0-7)
+    const int quarter = warp & 3, half = warp >> 2;
+    const uint32_t lane_addr = static_cast<uint32_t>(quarter * 32) << 16;
     const uint32_t stg = sbase + C::STG_OFF + static_cast<uint32_t>(warp) * C::STG_WARP;
-    int lt = 0, chunk = 0;
+    int lt = 0;
     bool ok = true;
     for (int t = pair; ok && t < tiles; t += n_pairs, ++lt) {
       int tm, tn;
@@ -634,44 +657,9 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
       const int b = lt & 1, use = lt >> 1;
       if (!(ok = mbar_wait_warp(bar_acc + 8 * b, use & 1, p.ctl, ab))) break;
       tc_fence_after();
-      const uint32_t src = tmem + lane_addr + static_cast<uint32_t>(b * C::BN);
-      const int row0 = tm * 256 + static_cast<int>(rank) * C::BM + warp * 32;
-#pragma unroll 1
-      for (int c = 0; c < C::BN / 64; ++c) {
-        uint32_t r0[32], r1[32];
-        tmem_ld32(src + c * 64, r0);
-        tmem_ld32(src + c * 64 + 32, r1);
-        tmem_wait_ld();
-        reg_fence32(r0);
-        reg_fence32(r1);
-        if (c == C::BN / 64 - 1) {  // the accumulator is in registers: hand it back
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive_cluster(map_shared_rank(bar_acce + 8 * b, 0));
-        }
-        if (tn * C::BN + c * 64 >= p.N || row0 >= p.M) continue;
-        uint32_t w[32];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          w[i] = pack_bf16x2(__uint_as_float(r0[2 * i]), __uint_as_float(r0[2 * i + 1]));
-          w[16 + i] = pack_bf16x2(__uint_as_float(r1[2 * i]), __uint_as_float(r1[2 * i + 1]));
-        }
-        const uint32_t buf = stg + static_cast<uint32_t>(chunk & 1) * (32 * 128);
-        ++chunk;
-        if (lane == 0) bulk_wait_group_read1();
-        __syncwarp();
-        const uint32_t row = buf + static_cast<uint32_t>(lane) * 128u;
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          st_shared_v4(row + (static_cast<uint32_t>(q ^ (lane & 7)) << 4), w[4 * q], w[4 * q + 1], w[4 * q + 2],
-                       w[4 * q + 3]);
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) {
-          tma_store_3d(&tm_c, buf, tn * C::BN + c * 64, row0, 0);
-          bulk_commit_group();
-        }
-      }
+      epilogue_warp<C::BN / 64>(&tm_c, tmem + lane_addr + static_cast<uint32_t>(b * C::BN), stg, half, tn * C::BN,
+                                tm * 256 + static_cast<int>(rank) * C::BM + quarter * 32, p.M, p.N,
+                                map_shared_rank(bar_acce + 8 * b, 0), true);
     }
     if (lane == 0) bulk_wait_group0();
   }
@@ -680,7 +668,7 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
   tc_fence_before();
   __syncthreads();
   cluster_sync_all();  // the pair's MMAs, copies and TMEM reads are over in both CTAs
-  if (warp == 5) {
+  if (warp == 9) {
     tc_fence_after();
     tmem_dealloc_pair(tmem, C::TMEM_COLS);
   }
@@ -767,7 +755,7 @@ template <int BN>
 cudaLaunchConfig_t splitk_config(int grid, int S, cudaStream_t stream, cudaLaunchAttribute* attr) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
-  cfg.blockDim = dim3(GemmCfg<BN>::THREADS, 1, 1);
+  cfg.blockDim = dim3(GemmCfg<BN>::SPLIT_THREADS, 1, 1);
   cfg.dynamicSmemBytes = GemmCfg<BN>::BYTES;
   cfg.stream = stream;
   attr[0].id = cudaLaunchAttributeClusterDimension;

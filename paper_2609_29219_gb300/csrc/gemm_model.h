@@ -20,14 +20,14 @@ struct GemmPlan {
   bool feasible;
 };
 
-constexpr int kGemmStagingBytes = 4 * 2 * 32 * 128;  // 4 epilogue warps x 2 buffers x 32 rows x 128 B
-// Epilogue of one tile by the four epilogue warps: a fixed part plus one 64-column chunk
-// (TMEM -> registers -> bf16 -> staging -> TMA store) at a time, and the extra cost of a
-// CTA pair's cross-SM accumulator release (fitted to K = 256 tiles: 128 x 256 take 2.8 us,
-// 128 x 128 1.55 us, and a pair's 128 x 256 per SM 3.4 us).
-constexpr double kGemmEpiTileNs = 400.0;
-constexpr double kGemmEpiChunkNs = 600.0;
-constexpr double kGemmPairEpiFactor = 1.2;
+constexpr int kGemmStagingBytes = 8 * 32 * 128;  // 8 epilogue warps x 32 rows x 128 B
+// Epilogue of one tile by the eight epilogue warps: a fixed part plus 64-column chunks
+// (TMEM -> registers -> bf16 -> staging -> TMA store), and the factor of a CTA pair's
+// cross-SM accumulator release (fitted to K = 256 tiles in steady state, 54 tiles per SM:
+// 128 x 256 take 2.89 us single and 2.89 us per SM as a pair, 128 x 128 1.66 us).
+constexpr double kGemmEpiTileNs = 430.0;
+constexpr double kGemmEpiChunkNs = 615.0;
+constexpr double kGemmPairEpiFactor = 1.0;
 
 constexpr GemmPlan gemm_eval(const ArchDesc& a, int bn, int stages) {
   GemmPlan p{};
