@@ -574,7 +574,8 @@ def main():
                     help="profiling run: set up this workload (tiny, tiny_causal, prefill, prefill_causal, "
                          "long_prefill_d128, long_prefill_d64, varlen_prefill, batched_decode, paged_decode_p16, paged_decode_p64, "
                          "long_decode, "
-                         "gemm_4096, gemm_16k_256_16k, gemm_256_256_16k, varlen_prefill_small), run --steps "
+                         "gemm_4096, gemm_16k_256_16k, gemm_256_256_16k, gemm_8192, cublas_8192 (torch.matmul), "
+                         "varlen_prefill_small), run --steps "
                          "launches, print nothing")
     args = ap.parse_args()
     world, rank, local = dist_env()
@@ -860,6 +861,8 @@ def run_ncu_case(torch, loom, dev, stream, args):
     cases["gemm_4096"] = Gemm("gemm_4096", 4096, 4096, 4096)
     cases["gemm_16k_256_16k"] = Gemm("gemm_16k_256_16k", 16384, 256, 16384)
     cases["gemm_256_256_16k"] = Gemm("gemm_256_256_16k", 256, 256, 16384)
+    cases["gemm_8192"] = Gemm("gemm_8192", 8192, 8192, 8192)
+    cases["cublas_8192"] = Gemm("cublas_8192", 8192, 8192, 8192, cublas=True)
     cases["varlen_prefill_small"] = VarlenPrefill("varlen_prefill_small", 8, 32, 8, 512, 2048, 128, causal=True)
     wl = cases[args.ncu_case]
     wl.sets = 1  # one input set: the smallest device footprint for a capture
