@@ -4,8 +4,9 @@
 //
 // Built as a standalone program (paper_2609_29219_gb300/arch_probe.py builds and runs it)
 // and printing one JSON object:
-//   pipes : ex2.approx / fma.rn.f32 / fma.rn.f32x2 / cvt.rn.bf16x2.f32 instruction-lanes per
-//           clock per SM, and ex2 beside the bf16x2 packs of the softmax (one per pair)
+//   pipes : ex2.approx / fma.rn.f32 / fma.rn.f32x2 / cvt.rn.bf16x2.f32 / ex2.approx.bf16x2
+//           instruction-lanes per clock per SM, and ex2 beside the bf16x2 packs of the softmax
+//           (one per pair)
 //   mma   : clocks per tcgen05.mma kind::f16 128xNx16 (SS with N = 64, 128, 256; TS N = 128)
 //   mix   : clocks per 128x128x128 GEMM of the prefill kernel's MMA stream (P.V as TS,
 //           S = Q.K^T as SS, two query tiles) alone and under added load: bulk copies,
@@ -41,6 +42,11 @@ __global__ void pipe_kernel(float* out, long long* cyc, int iters) {
         uint32_t r;
         asm volatile("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(v[i]), "f"(v[i]));
         v[i] = __uint_as_float(r);
+      }
+      if (MODE == 5) {  // packed exponential: one MUFU instruction for two bf16 results
+        uint32_t r = __float_as_uint(v[i]);
+        asm volatile("ex2.approx.ftz.bf16x2 %0, %0;" : "+r"(r));
+        v[i] = __uint_as_float(r ^ 0x80008000u);  // both halves negative again: results stay in (0, 1]
       }
       if (MODE == 4) {  // the softmax mix: 1 MUFU + 1 FADD per element, a bf16x2 pack per pair
         v[i] = ex2f_(v[i]) - 1.5f;
@@ -336,9 +342,10 @@ int main() {
   {
     const double ops = 1024.0 * 4096 * 8;
     // mode 4 counts its ex2 (8 per iteration, with 4 bf16x2 packs beside them)
-    const char* names[5] = {"ex2_per_clk_sm", "ffma_lanes_per_clk_sm", "ffma2_instr_lanes_per_clk_sm",
-                            "cvt_bf16x2_per_clk_sm", "ex2_beside_cvt_per_clk_sm"};
-    for (int mode = 0; mode < 5; ++mode) {
+    // mode 5 counts instructions (each gives two bf16 exponentials)
+    const char* names[6] = {"ex2_per_clk_sm", "ffma_lanes_per_clk_sm", "ffma2_instr_lanes_per_clk_sm",
+                            "cvt_bf16x2_per_clk_sm", "ex2_beside_cvt_per_clk_sm", "ex2_bf16x2_instr_per_clk_sm"};
+    for (int mode = 0; mode < 6; ++mode) {
       auto launch = [&] {
         for (int rep = 0; rep < 2; ++rep) {
           if (mode == 0) pipe_kernel<0><<<sms, 1024>>>(out, d, 4096);
@@ -346,6 +353,7 @@ int main() {
           if (mode == 2) pipe_kernel<2><<<sms, 1024>>>(out, d, 4096);
           if (mode == 3) pipe_kernel<3><<<sms, 1024>>>(out, d, 4096);
           if (mode == 4) pipe_kernel<4><<<sms, 1024>>>(out, d, 4096);
+          if (mode == 5) pipe_kernel<5><<<sms, 1024>>>(out, d, 4096);
         }
       };
       const double cyc = avg_cycles(launch, d, h, sms);
