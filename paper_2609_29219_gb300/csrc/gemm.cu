@@ -50,6 +50,34 @@ __device__ __forceinline__ uint32_t map_shared_rank(uint32_t saddr, uint32_t ran
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_bar) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar) : "memory");
 }
+// Bounded wait by one thread on a barrier that the peer CTA arrives on (release at cluster
+// scope): acquire at cluster scope, so the peer's writes before its arrival are visible.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, const KernelCtl& ctl,
+                                                  const Abort& ab) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 16; ++i)
+      if (mbar_try_wait_cluster(bar, parity)) return true;
+    if (ab.raised()) return false;
+    if (globaltimer_ns() - t0 > ctl.timeout_ns) {
+      ab.raise(ctl);
+      return false;
+    }
+  }
+}
 __device__ __forceinline__ float4 ld_dsmem_f4(uint32_t addr) {
   float4 v;
   asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
@@ -624,7 +652,7 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
       bool ok = true;
       for (int t = pair; ok && t < tiles; t += n_pairs, ++lt) {
         const int b = lt & 1, use = lt >> 1;
-        if (lt >= 2 && !(ok = mbar_wait(bar_acce + 8 * b, (use - 1) & 1, p.ctl, ab))) break;
+        if (lt >= 2 && !(ok = mbar_wait_cluster(bar_acce + 8 * b, (use - 1) & 1, p.ctl, ab))) break;
         tc_fence_after();
         const uint32_t d = tmem + static_cast<uint32_t>(b * C::BN);
         for (int ks = 0; ks < p.k_iters; ++ks, ++it) {
