@@ -178,3 +178,12 @@ def test_timeout_is_reported_and_context_survives(loom, forced, tile_n, splits, 
         loom.loom_debug_set_timeout_ns(0)
     c = _run_dev(loom, ad, bd)
     _check(c.float().cpu().numpy().astype(np.float64), oracle.gemm(a, b), K, "after timeout")
+
+
+@pytest.mark.parametrize("M,K,N", [(1, 64, 512), (257, 128, 248), (3000, 640, 40), (512, 2048, 8)])
+def test_pair_tiles_on_thin_shapes(loom, forced, M, K, N):
+    """CTA-pair tiles on shapes far from 256 x 256 multiples: the odd CTA's rows (or most
+    columns) fall outside C and are neither stored nor allowed to disturb the even CTA."""
+    forced(0, 0, 1)
+    a, b = _inputs(M * 7 + N, M, K, N)
+    _check(_run(loom, a, b), oracle.gemm(a, b), K, f"pair {M}x{K}x{N}")

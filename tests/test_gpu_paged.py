@@ -168,3 +168,14 @@ def test_timeout_is_reported_and_context_survives(loom):
     loom.loom_attn_check_error()
     o_ref, lse_ref = oracle.decode_paged(q, kc, vc, table, sl, page_size=P)
     assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, "after timeout")
+
+
+def test_large_pages_and_long_table(loom):
+    """512-key pages (eight 64-key copies per page) and a 40-entry block table."""
+    B, Hq, Hkv, P, D = 3, 8, 2, 512, 128
+    lens = [20000, 513, 9000]
+    q, kc, vc, table, sl = paged_case(41, B, Hq, Hkv, P, lens, D, spare=2)
+    for splits in (0, 3):
+        o, lse = run_paged(loom, q, kc, vc, table, sl, splits)
+        o_ref, lse_ref = oracle.decode_paged(q, kc, vc, table, sl, page_size=P)
+        assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"P=512 splits={splits}")

@@ -135,3 +135,28 @@ def test_timeout_is_reported_and_context_survives(loom):
     loom.loom_attn_check_error()
     o_ref, lse_ref = oracle.attention_varlen(q, k, v, cq, ck, causal=True)
     assert_parity(o.float().cpu().numpy(), o_ref, lse.cpu().numpy(), lse_ref, "after timeout")
+
+
+@pytest.mark.parametrize("causal", [False, True], ids=["nc", "causal"])
+def test_many_short_sequences(loom, causal):
+    """300 sequences of 0-300 tokens (many empty or single-token), D = 64: the sequence
+    cursor steps over empty runs and items never cross a sequence."""
+    rng = np.random.default_rng(17)
+    lens = rng.integers(0, 301, 300)
+    lens[rng.integers(0, 300, 40)] = 0
+    lens[rng.integers(0, 300, 40)] = 1
+    q, k, v, cq, ck = case(23, lens, lens, 4, 1, 64)
+    o, lse = run(loom, q, k, v, cq, ck, causal)
+    o_ref, lse_ref = oracle.attention_varlen(q, k, v, cq, ck, causal=causal)
+    assert_parity(o, o_ref, lse, lse_ref, f"300 short sequences causal={causal}")
+
+
+def test_cross_attention_lengths(loom):
+    """Every sequence has its own query and key counts (cross attention, non-causal)."""
+    rng = np.random.default_rng(29)
+    lq = rng.integers(1, 700, 10)
+    lk = rng.integers(1, 1500, 10)
+    q, k, v, cq, ck = case(31, lq, lk, 8, 2, 128)
+    o, lse = run(loom, q, k, v, cq, ck, False)
+    o_ref, lse_ref = oracle.attention_varlen(q, k, v, cq, ck, causal=False)
+    assert_parity(o, o_ref, lse, lse_ref, "cross attention")
