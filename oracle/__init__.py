@@ -182,13 +182,18 @@ def gemm(a, b, *, rows=None):
     return A @ Bm
 
 
-def paged_gather(cache, block_table, seqlens, page_size):
-    """The logical K (or V) [B, Hkv, Skv_max, D] of a paged cache [num_pages, page_size,
-    Hkv, D]: key t of sequence b is row t mod page_size of physical page
-    block_table[b, t div page_size] (the usual paged-KV convention; the paper has none).
-    Skv_max = block_table.shape[1] * page_size; positions at or past seqlens[b] are left
-    zero, and their table entries are not read (they may be anything)."""
+def paged_gather(cache, block_table, seqlens, page_size, layout="nhd"):
+    """The logical K (or V) [B, Hkv, Skv_max, D] of a paged cache: key t of sequence b is
+    row t mod page_size of physical page block_table[b, t div page_size] (the usual
+    paged-KV convention; the paper has none).  layout "nhd": cache [num_pages, page_size,
+    Hkv, D]; "hnd": cache [num_pages, Hkv, page_size, D].  Skv_max = block_table.shape[1] *
+    page_size; positions at or past seqlens[b] are left zero, and their table entries are
+    not read (they may be anything)."""
     cache = _u16(cache)
+    if layout == "hnd":
+        cache = cache.transpose(0, 2, 1, 3)
+    elif layout != "nhd":
+        raise ValueError("layout is 'nhd' or 'hnd'")
     table = np.asarray(block_table, dtype=np.int64)
     lens = np.asarray(seqlens, dtype=np.int64)
     npages, P, Hkv, D = cache.shape
@@ -207,12 +212,12 @@ def paged_gather(cache, block_table, seqlens, page_size):
     return out
 
 
-def decode_paged(q, k_cache, v_cache, block_table, seqlens, *, page_size, scale=None, nthreads=0):
+def decode_paged(q, k_cache, v_cache, block_table, seqlens, *, page_size, scale=None, nthreads=0, layout="nhd"):
     """Decode (one query row per head) over a paged KV cache: the attention definition on
     the logical K/V that ``paged_gather`` assembles.  q [B, Hq, 1, D].  Returns
     ``(o [B, Hq, D], lse [B, Hq])``."""
-    k = paged_gather(k_cache, block_table, seqlens, page_size)
-    v = paged_gather(v_cache, block_table, seqlens, page_size)
+    k = paged_gather(k_cache, block_table, seqlens, page_size, layout)
+    v = paged_gather(v_cache, block_table, seqlens, page_size, layout)
     o, lse = attention(q, k, v, scale=scale, seqlens_k=np.asarray(seqlens, dtype=np.int32), nthreads=nthreads)
     return o[:, :, 0, :], lse[:, :, 0]
 

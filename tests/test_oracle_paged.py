@@ -162,3 +162,19 @@ def test_brute_force_catches_planted_gather_mistakes(kind, monkeypatch):
     monkeypatch.setattr(oracle, "paged_gather", _mutant_gather(kind))
     o, _ = oracle.decode_paged(q, kc, vc, table, sl, page_size=P, scale=0.3)
     assert not np.allclose(o, ob, atol=1e-6)
+
+
+def test_hnd_layout_is_the_same_cache_transposed():
+    """The head-major page layout [pages, Hkv, page_size, D] holds the same keys: gathering
+    it equals gathering its NHD transpose, and the brute force agrees."""
+    P, lens = 8, [13, 30]
+    q, kc, vc, table, sl = _paged_case(51, 2, 4, 2, P, 5, lens, D=16)
+    kh = np.ascontiguousarray(kc.transpose(0, 2, 1, 3))
+    vh = np.ascontiguousarray(vc.transpose(0, 2, 1, 3))
+    np.testing.assert_array_equal(oracle.paged_gather(kh, table, sl, P, "hnd"), oracle.paged_gather(kc, table, sl, P))
+    o, lse = oracle.decode_paged(q, kh, vh, table, sl, page_size=P, scale=0.3, layout="hnd")
+    ob, lb = _brute(q, kc, vc, table, sl, P, 0.3)
+    np.testing.assert_allclose(o, ob, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(lse, lb, rtol=0, atol=1e-12)
+    with pytest.raises(ValueError):
+        oracle.paged_gather(kc, table, sl, P, "nhwd")
