@@ -135,7 +135,7 @@ def test_empty_sequence_and_bad_table():
 
 
 def _mutant_gather(kind):
-    def gather(cache, block_table, seqlens, page_size):
+    def gather(cache, block_table, seqlens, page_size, layout="nhd"):
         cache = np.asarray(cache, dtype=np.uint16)
         table = np.asarray(block_table, dtype=np.int64)
         npages, P, Hkv, D = cache.shape
