@@ -293,12 +293,12 @@ class PagedDecode(Decode):
     pages are dealt in a seeded shuffled order across the cache (a cache that has served
     many requests), so consecutive logical pages are scattered in HBM."""
 
-    def __init__(self, name, B, Hq, Hkv, Skv, D, splits, page_size, lengths, seed=0, sets=2):
+    def __init__(self, name, B, Hq, Hkv, Skv, D, splits, page_size, lengths, seed=0, sets=2, layout="nhd"):
         super().__init__(name, B, Hq, Hkv, Skv, D, splits, lengths=lengths, seed=seed, sets=sets)
-        self.P = page_size
+        self.P, self.layout = page_size, layout
 
     def describe(self):
-        return super().describe().replace("decode ", f"paged decode page_size={self.P} ", 1)
+        return super().describe().replace("decode ", f"paged decode ({self.layout}) page_size={self.P} ", 1)
 
     def paged(self, k, v, s):
         B, Hkv, S, D, P = self.B, self.Hkv, self.Skv, self.D, self.P
@@ -308,6 +308,9 @@ class PagedDecode(Decode):
         vc = np.empty_like(kc)
         kc[order] = k.reshape(B, Hkv, npg, P, D).transpose(0, 2, 3, 1, 4).reshape(B * npg, P, Hkv, D)
         vc[order] = v.reshape(B, Hkv, npg, P, D).transpose(0, 2, 3, 1, 4).reshape(B * npg, P, Hkv, D)
+        if self.layout == "hnd":
+            kc = np.ascontiguousarray(kc.transpose(0, 2, 1, 3))
+            vc = np.ascontiguousarray(vc.transpose(0, 2, 1, 3))
         return kc, vc, order.reshape(B, npg)
 
     def setup(self, torch, dev, loom):
@@ -328,7 +331,7 @@ class PagedDecode(Decode):
     def step(self, i, stream):
         q, kc, vc, table, o, lse = self.inp[i % self.sets]
         self.loom.loom_attn_decode_paged(q, kc, vc, table, self.sl, o, lse, self.ws, num_splits=self.splits,
-                                         stream=stream)
+                                         stream=stream, layout=self.layout)
 
 
 class VarlenPrefill:
@@ -573,6 +576,7 @@ def main():
     ap.add_argument("--ncu-case", default=None,
                     help="profiling run: set up this workload (tiny, tiny_causal, prefill, prefill_causal, "
                          "long_prefill_d128, long_prefill_d64, varlen_prefill, batched_decode, paged_decode_p16, paged_decode_p64, "
+                         "paged_decode_hnd_p16, "
                          "long_decode, "
                          "gemm_4096, gemm_16k_256_16k, gemm_256_256_16k, gemm_8192, cublas_8192 (torch.matmul), "
                          "varlen_prefill_small), run --steps "
@@ -631,6 +635,8 @@ def main():
             Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
             PagedDecode("paged_decode_p16", 16, 32, 8, 8192, 128, splits=16, page_size=16, lengths=lens),
             PagedDecode("paged_decode_p64", 16, 32, 8, 8192, 128, splits=16, page_size=64, lengths=lens),
+            PagedDecode("paged_decode_hnd_p16", 16, 32, 8, 8192, 128, splits=16, page_size=16, lengths=lens,
+                        layout="hnd"),
             Decode("long_decode", 1, 32, 8, 131072, 128, splits=0),
         ]
         if args.only:
@@ -852,6 +858,8 @@ def all_workloads():
             Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
             PagedDecode("paged_decode_p16", 16, 32, 8, 8192, 128, splits=16, page_size=16, lengths=lens),
             PagedDecode("paged_decode_p64", 16, 32, 8, 8192, 128, splits=16, page_size=64, lengths=lens),
+            PagedDecode("paged_decode_hnd_p16", 16, 32, 8, 8192, 128, splits=16, page_size=16, lengths=lens,
+                        layout="hnd"),
             Decode("long_decode", 1, 32, 8, 131072, 128, splits=0)]
 
 

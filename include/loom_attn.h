@@ -131,8 +131,10 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
  * no counterpart -- it belongs to the irregular grids its Sec. 2.6 scope note sets aside).
  *   q            [B, Hq, 1, D]                     bf16, read
  *   k_cache,
- *   v_cache      [num_pages, page_size, Hkv, D]    bf16, read; a page holds page_size
- *                consecutive keys of one sequence, with the rows of all kv heads adjacent
+ *   v_cache      bf16, read; a page holds page_size consecutive keys of one sequence:
+ *                kv_layout 0 (NHD): [num_pages, page_size, Hkv, D], a key's rows of all kv
+ *                heads adjacent; kv_layout 1 (HND): [num_pages, Hkv, page_size, D], a page's
+ *                rows of one kv head contiguous
  *   block_table  [B, max_pages] int32 on the device: key t of sequence b is row
  *                t % page_size of page block_table[b * max_pages + t / page_size].  Only
  *                the first ceil(len_b / page_size) entries of a row are read; an entry
@@ -142,16 +144,16 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
  *                page_size in loom_attn_decode_workspace_bytes / loom_attn_decode_num_splits.
  * page_size: 8, 16, 32 or a multiple of 64.  The split rule and results are those of
  * loom_attn_decode on the gathered (logical) cache.
- * Errors: INVALID_ARG (NULL q/k/v/o/block_table/seqlens_k, a size <= 0, Hq % Hkv, scale),
- * UNSUPPORTED (D, page_size, more than 2^31 - 1 keys in the cache or per sequence, too many
- * splits), MISALIGNED (q, caches, o, workspace not 16-byte aligned; block_table, seqlens_k,
+ * Errors: INVALID_ARG (NULL q/k/v/o/block_table/seqlens_k, a size <= 0, Hq % Hkv, scale,
+ * kv_layout not 0 or 1), UNSUPPORTED (D, page_size, more than 2^31 - 1 keys in the cache or
+ * per sequence, too many splits), MISALIGNED (q, caches, o, workspace not 16-byte aligned; block_table, seqlens_k,
  * lse not 4-byte aligned), WORKSPACE, CUDA.
  */
 loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const void* v_cache,
                                    const int32_t* block_table, const int32_t* seqlens_k, void* o,
                                    float* lse, void* workspace, size_t workspace_bytes, int B, int Hq,
-                                   int Hkv, int num_pages, int page_size, int max_pages, int D,
-                                   float scale, int num_splits, void* stream);
+                                   int Hkv, int num_pages, int page_size, int max_pages, int kv_layout,
+                                   int D, float scale, int num_splits, void* stream);
 
 /*
  * Flash Decode without any allocation and without a workspace argument.  The paper has

@@ -102,7 +102,7 @@ def capi() -> ctypes.CDLL:
             lib.loom_model_fwd_time_us_design.argtypes = [i32] * 7
             lib.loom_model_fwd_time_us_design.restype = ctypes.c_double
             lib.loom_attn_decode_paged.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, sz, i32, i32, i32, i32,
-                                                   i32, i32, i32, f32, i32, vp]
+                                                   i32, i32, i32, i32, f32, i32, vp]
             lib.loom_attn_decode_paged.restype = i32
             lib.loom_attn_fwd_varlen.argtypes = [vp, vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32,
                                                  i32, f32, vp]
@@ -290,19 +290,25 @@ def loom_attn_fwd_varlen(q, k, v, cu_seqlens_q, cu_seqlens_k, max_seqlen_q, o=No
 
 
 def loom_attn_decode_paged(q, k_cache, v_cache, block_table, seqlens_k, o=None, lse=None, workspace=None, *,
-                           scale=None, num_splits=0, stream=None, return_lse=False):
-    """Flash Decode over a paged cache.  q [B,Hq,1,D]; k_cache/v_cache [num_pages, page_size,
-    Hkv, D] bf16; block_table [B, max_pages] int32; seqlens_k [B] int32 (all on the device).
-    Returns ``o`` or ``(o, lse)``."""
+                           scale=None, num_splits=0, stream=None, return_lse=False, layout="nhd"):
+    """Flash Decode over a paged cache.  q [B,Hq,1,D]; k_cache/v_cache bf16, [num_pages,
+    page_size, Hkv, D] (layout "nhd") or [num_pages, Hkv, page_size, D] (layout "hnd");
+    block_table [B, max_pages] int32; seqlens_k [B] int32 (all on the device).  Returns
+    ``o`` or ``(o, lse)``."""
     torch = _torch()
     bf16 = torch.bfloat16
     qp = _dev_ptr(q, "q", bf16, 4)
     kp = _dev_ptr(k_cache, "k_cache", bf16, 4)
     vp_ = _dev_ptr(v_cache, "v_cache", bf16, 4)
     B, Hq, Sq, D = q.shape
-    num_pages, page_size, Hkv, Dk = k_cache.shape
+    if layout not in ("nhd", "hnd"):
+        raise ValueError("layout is 'nhd' or 'hnd'")
+    if layout == "nhd":
+        num_pages, page_size, Hkv, Dk = k_cache.shape
+    else:
+        num_pages, Hkv, page_size, Dk = k_cache.shape
     if Sq != 1 or tuple(v_cache.shape) != tuple(k_cache.shape) or Dk != D:
-        raise ValueError("paged decode takes q [B,Hq,1,D] and caches [num_pages, page_size, Hkv, D]")
+        raise ValueError("paged decode takes q [B,Hq,1,D] and two caches of one shape")
     if block_table.dim() != 2 or block_table.shape[0] != B:
         raise ValueError("block_table must be [B, max_pages]")
     max_pages = block_table.shape[1]
@@ -328,7 +334,8 @@ def loom_attn_decode_paged(q, k_cache, v_cache, block_table, seqlens_k, o=None, 
     if scale is None:
         scale = D ** -0.5
     st = capi().loom_attn_decode_paged(qp, kp, vp_, tp, sp, op, lp, wp, workspace.numel() * workspace.element_size(),
-                                       B, Hq, Hkv, num_pages, page_size, max_pages, D, float(scale),
+                                       B, Hq, Hkv, num_pages, page_size, max_pages, 0 if layout == "nhd" else 1,
+                                       D, float(scale),
                                        int(num_splits), _stream_ptr(stream, q.device))
     _check(st, "loom_attn_decode_paged")
     return (o, lse) if (return_lse or lse is not None) else o

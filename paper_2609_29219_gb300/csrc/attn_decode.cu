@@ -118,7 +118,8 @@ __device__ __forceinline__ int head_of_lane(int lane) {
 struct PagedView {
   const int32_t* block_table;
   int page_size, max_pages;
-  int num_keys;  // num_pages * page_size (< 2^31)
+  int num_pages;
+  int hnd;  // 1: [num_pages, Hkv, page_size, D]; 0: [num_pages, page_size, Hkv, D]
 };
 
 template <int D, int GT, bool PAGED>
@@ -212,12 +213,20 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
         const int t = tok0 + lane * rows;
         const int page = __shfl_sync(0xffffffffu, entry, (t / P - win) & 31);
         if (lane < ncopy) {
-          // an out-of-range page (a caller error) is sent past the last key, where the
-          // copy engine reads zeros
-          const long long zl = static_cast<long long>(page) * P + t % P;
-          const int z = (page < 0 || zl >= pv.num_keys) ? pv.num_keys : static_cast<int>(zl);
-          tma_load_3d(dst + lane * copy_bytes, &tm_k, 0, hk, z, bar_full + 8 * slot);
-          tma_load_3d(dst + C::TILE_BYTES + lane * copy_bytes, &tm_v, 0, hk, z, bar_full + 8 * slot);
+          // An out-of-range page (a caller error) is sent past the end of the cache, where
+          // the copy engine reads zeros.  NHD view [keys of all pages, Hkv, D]: (0, hk, key);
+          // HND view [pages x Hkv, page_size, D]: (0, row in page, page x Hkv + hk).
+          const bool bad = page < 0 || page >= pv.num_pages;
+          int y, z;
+          if (pv.hnd) {
+            y = t % P;
+            z = bad ? pv.num_pages * Hkv : page * Hkv + hk;
+          } else {
+            y = hk;
+            z = bad ? pv.num_pages * P : page * P + t % P;
+          }
+          tma_load_3d(dst + lane * copy_bytes, &tm_k, 0, y, z, bar_full + 8 * slot);
+          tma_load_3d(dst + C::TILE_BYTES + lane * copy_bytes, &tm_v, 0, y, z, bar_full + 8 * slot);
         }
       }
       if (lane == 0) {
@@ -506,16 +515,21 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// A paged cache [num_pages, page_size, Hkv, D] viewed as the 3-D tensor
-// [num_pages * page_size keys, Hkv, D] (innermost first: D, Hkv, keys); one box is
-// `rows` keys of one kv head, landing in shared memory as rows x D contiguous bf16.
+// A paged cache as a 3-D tensor whose box is `rows` keys of one kv head, landing in
+// shared memory as rows x D contiguous bf16:
+//   NHD [num_pages, page_size, Hkv, D] -> [num_pages * page_size keys, Hkv, D], box D x 1 x rows
+//   HND [num_pages, Hkv, page_size, D] -> [num_pages * Hkv, page_size, D],      box D x rows x 1
 bool paged_map(CUtensorMap* map, const void* cache, const PagedKV& pk, int Hkv, int D, int rows) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return false;
-  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(Hkv),
-                        static_cast<cuuint64_t>(pk.num_pages) * pk.page_size};
-  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(Hkv) * D * 2};
-  cuuint32_t box[3] = {static_cast<cuuint32_t>(D), 1, static_cast<cuuint32_t>(rows)};
+  const bool hnd = pk.layout == kPagedHND;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D),
+                        static_cast<cuuint64_t>(hnd ? pk.page_size : Hkv),
+                        static_cast<cuuint64_t>(pk.num_pages) * (hnd ? Hkv : pk.page_size)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2,
+                           static_cast<cuuint64_t>(hnd ? pk.page_size : Hkv) * D * 2};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(D), static_cast<cuuint32_t>(hnd ? rows : 1),
+                       static_cast<cuuint32_t>(hnd ? 1 : rows)};
   cuuint32_t estr[3] = {1, 1, 1};
   return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(cache), dims, strides, box, estr,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -536,12 +550,12 @@ cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl
     configured |= 1ull << (dev & 63);
   }
   CUtensorMap tk, tv;
-  PagedView view{nullptr, 0, 0, 0};
+  PagedView view{nullptr, 0, 0, 0, 0};
   if constexpr (PAGED) {
     const int rows = pk->page_size < kDecodeChunkAlign ? pk->page_size : kDecodeChunkAlign;
     if (!paged_map(&tk, a.k, *pk, a.Hkv, D, rows) || !paged_map(&tv, a.v, *pk, a.Hkv, D, rows))
       return cudaErrorInvalidValue;
-    view = PagedView{pk->block_table, pk->page_size, pk->max_pages, pk->num_pages * pk->page_size};
+    view = PagedView{pk->block_table, pk->page_size, pk->max_pages, pk->num_pages, pk->layout == kPagedHND ? 1 : 0};
   } else {
     (void)pk;
     memset(&tk, 0, sizeof(tk));
@@ -594,7 +608,9 @@ cudaError_t launch_decode(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_
 }
 
 cudaError_t launch_decode_paged(const DecodeArgs& a, const PagedKV& pk, const KernelCtl& ctl, cudaStream_t stream) {
-  if (!paged_page_size_ok(pk.page_size) || !a.seqlens || !pk.block_table) return cudaErrorInvalidValue;
+  if (!paged_page_size_ok(pk.page_size) || !a.seqlens || !pk.block_table ||
+      (pk.layout != kPagedNHD && pk.layout != kPagedHND))
+    return cudaErrorInvalidValue;
   if (a.D == 128) return launch_decode_d<128, true>(a, &pk, ctl, stream);
   return launch_decode_d<64, true>(a, &pk, ctl, stream);
 }

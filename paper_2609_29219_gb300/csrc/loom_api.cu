@@ -203,17 +203,19 @@ loom_status loom_attn_fwd_varlen(const void* q, const void* k, const void* v, vo
 loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const void* v_cache,
                                    const int32_t* block_table, const int32_t* seqlens_k, void* o,
                                    float* lse, void* workspace, size_t workspace_bytes, int B, int Hq,
-                                   int Hkv, int num_pages, int page_size, int max_pages, int D,
-                                   float scale, int num_splits, void* stream) {
+                                   int Hkv, int num_pages, int page_size, int max_pages, int kv_layout,
+                                   int D, float scale, int num_splits, void* stream) {
   if (!q || !k_cache || !v_cache || !o || !block_table || !seqlens_k) return LOOM_ERR_INVALID_ARG;
   if (B <= 0 || Hq <= 0 || Hkv <= 0 || num_pages <= 0 || page_size <= 0 || max_pages <= 0 || D <= 0)
     return LOOM_ERR_INVALID_ARG;
   if (Hq % Hkv != 0) return LOOM_ERR_INVALID_ARG;
   if (!std::isfinite(scale) || scale <= 0.f) return LOOM_ERR_INVALID_ARG;
   if (num_splits < 0) return LOOM_ERR_INVALID_ARG;
+  if (kv_layout != kPagedNHD && kv_layout != kPagedHND) return LOOM_ERR_INVALID_ARG;
   if (D != 64 && D != 128) return LOOM_ERR_UNSUPPORTED;
   if (!paged_page_size_ok(page_size)) return LOOM_ERR_UNSUPPORTED;
   if (static_cast<long long>(num_pages) * page_size > 0x7fffffffLL ||
+      static_cast<long long>(num_pages) * Hkv > 0x7fffffffLL ||
       static_cast<long long>(max_pages) * page_size > 0x7fffffffLL ||
       static_cast<long long>(B) * max_pages > 0x7fffffffLL)
     return LOOM_ERR_UNSUPPORTED;
@@ -238,7 +240,7 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D, num_splits, scale};
-  PagedKV pk{block_table, num_pages, page_size, max_pages};
+  PagedKV pk{block_table, num_pages, page_size, max_pages, kv_layout};
   return launch_decode_paged(a, pk, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                           : LOOM_ERR_CUDA;
 }

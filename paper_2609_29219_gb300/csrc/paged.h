@@ -8,14 +8,18 @@
 
 namespace loom {
 
-// The cache is [num_pages, page_size, Hkv, D] bf16 (a key's rows of all kv heads are
-// adjacent; a page holds page_size consecutive keys of one sequence).  Key t of sequence
-// b lives in row t % page_size of page block_table[b * max_pages + t / page_size].
+// A page holds page_size consecutive keys of one sequence.  Key t of sequence b lives in
+// row t % page_size of page block_table[b * max_pages + t / page_size].  Layouts (bf16):
+//   kPagedNHD  [num_pages, page_size, Hkv, D]  (a key's rows of all kv heads adjacent)
+//   kPagedHND  [num_pages, Hkv, page_size, D]  (a page's rows of one kv head contiguous)
+constexpr int kPagedNHD = 0, kPagedHND = 1;
+
 struct PagedKV {
   const int32_t* block_table;  // [B, max_pages]
   int num_pages;               // pages in each of the K and V caches
   int page_size;               // keys per page
   int max_pages;               // logical pages per sequence (row stride of block_table)
+  int layout;                  // kPagedNHD or kPagedHND
 };
 
 // Page sizes the loader supports: each 64-key copy (the split-chunk alignment) lies in one

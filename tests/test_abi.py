@@ -146,7 +146,7 @@ def test_gemm_pair_tiles_for_large_shapes(lib):
 
 def test_paged_decode_rejects_bad_arguments(lib):
     ok = dict(q=FAKE, k=FAKE, v=FAKE, tbl=FAKE, sl=FAKE, o=FAKE, lse=None, ws=FAKE, wsb=1 << 24, B=2, Hq=8,
-              Hkv=2, npages=64, P=16, maxp=8, D=128, scale=0.08, splits=4, stream=None)
+              Hkv=2, npages=64, P=16, maxp=8, layout=0, D=128, scale=0.08, splits=4, stream=None)
     names = list(ok)
 
     def call(**kw):
@@ -158,6 +158,7 @@ def test_paged_decode_rejects_bad_arguments(lib):
     assert call(sl=None) == 1
     assert call(P=0) == 1
     assert call(Hq=7) == 1
+    assert call(layout=2) == 1      # INVALID_ARG layout
     assert call(P=24) == 2          # UNSUPPORTED page size
     assert call(P=96) == 2
     assert call(D=80) == 2

@@ -53,23 +53,32 @@ def paged_case(seed, B, Hq, Hkv, P, lens, D, spare=5, poison=True, shuffle=True)
     return q, kc, vc, table, lens
 
 
-def run_paged(loom, q, kc, vc, table, lens, splits=0):
+def run_paged(loom, q, kc, vc, table, lens, splits=0, layout="nhd"):
+    """kc / vc are token-major [pages, page_size, Hkv, D]; layout "hnd" hands the kernel
+    the same pages head-major [pages, Hkv, page_size, D]."""
     import torch
+    if layout == "hnd":
+        kc = np.ascontiguousarray(kc.transpose(0, 2, 1, 3))
+        vc = np.ascontiguousarray(vc.transpose(0, 2, 1, 3))
     o, lse = loom.loom_attn_decode_paged(to_dev(q), to_dev(kc), to_dev(vc),
                                          torch.from_numpy(table).cuda(), torch.from_numpy(lens).cuda(),
-                                         num_splits=splits, return_lse=True)
+                                         num_splits=splits, return_lse=True, layout=layout)
     loom.loom_attn_check_error()
     return o, lse
 
 
+LAYOUTS = pytest.mark.parametrize("layout", ["nhd", "hnd"])
+
+
+@LAYOUTS
 @pytest.mark.parametrize("D", [64, 128])
 @pytest.mark.parametrize("P", [8, 16, 32, 64, 128, 256])
-def test_page_sizes(loom, P, D):
+def test_page_sizes(loom, P, D, layout):
     B, Hq, Hkv = 4, 8, 2
     lens = [1, P - 1, 3 * P + 1, 700]
     q, kc, vc, table, sl = paged_case(P + D, B, Hq, Hkv, P, lens, D)
     for splits in (1, 0, 7):
-        o, lse = run_paged(loom, q, kc, vc, table, sl, splits)
+        o, lse = run_paged(loom, q, kc, vc, table, sl, splits, layout)
         o_ref, lse_ref = oracle.decode_paged(q, kc, vc, table, sl, page_size=P)
         assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"P={P} D={D} splits={splits}")
 
@@ -83,19 +92,21 @@ def test_gqa_groups(loom, G):
     assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"G={G}")
 
 
-def test_edge_lengths_and_empty(loom):
+@LAYOUTS
+def test_edge_lengths_and_empty(loom, layout):
     B, Hq, Hkv, P, D = 8, 4, 1, 16, 64
     lens = [0, 1, 15, 16, 17, 63, 64, 65]
     q, kc, vc, table, sl = paged_case(4, B, Hq, Hkv, P, lens, D)
     for splits in (1, 3, 64):
-        o, lse = run_paged(loom, q, kc, vc, table, sl, splits)
+        o, lse = run_paged(loom, q, kc, vc, table, sl, splits, layout)
         o_ref, lse_ref = oracle.decode_paged(q, kc, vc, table, sl, page_size=P)
         assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"edges splits={splits}")
         assert np.all(o_to_f64(o)[0] == 0.0) and np.all(np.isneginf(lse.cpu().numpy()[0]))
 
 
+@LAYOUTS
 @pytest.mark.parametrize("P", [16, 64])
-def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P):
+def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P, layout):
     """With page j of sequence b at physical index b * pages + j, the paged and the
     contiguous kernels copy identical rows to identical places: outputs are equal bit for bit."""
     import torch
@@ -109,7 +120,7 @@ def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P):
     table = np.arange(B * npg, dtype=np.int32).reshape(B, npg)
     lens = np.array([S, 777, 64], dtype=np.int32)
     for splits in (1, 5):
-        o1, l1 = run_paged(loom, q, kc, vc, table, lens, splits)
+        o1, l1 = run_paged(loom, q, kc, vc, table, lens, splits, layout)
         o2, l2 = loom.loom_attn_decode(to_dev(q), to_dev(k), to_dev(v), torch.from_numpy(lens).cuda(),
                                        num_splits=splits, return_lse=True)
         loom.loom_attn_check_error()
@@ -117,19 +128,21 @@ def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P):
         assert torch.equal(l1, l2)
 
 
+@LAYOUTS
 @pytest.mark.parametrize("P", [16, 64])
-def test_batched_serving_shape(loom, P):
+def test_batched_serving_shape(loom, P, layout):
     """The batched decode shape (B=16, Hq=32, Hkv=8, D=128, lengths U[4096, 8192]) paged,
     pages shuffled, model-chosen splits."""
     B, Hq, Hkv, D = 16, 32, 8, 128
     lens = synth.decode_lengths(0, B, 4096, 8192)
     q, kc, vc, table, sl = paged_case(0, B, Hq, Hkv, P, lens, D, spare=0, poison=False)
-    o, lse = run_paged(loom, q, kc, vc, table, sl, 16)
+    o, lse = run_paged(loom, q, kc, vc, table, sl, 16, layout)
     o_ref, lse_ref = oracle.decode_paged(q, kc, vc, table, sl, page_size=P)
-    assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"batched paged P={P}")
+    assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"batched paged P={P} {layout}")
 
 
-def test_out_of_range_page_reads_zeros_without_fault(loom):
+@LAYOUTS
+def test_out_of_range_page_reads_zeros_without_fault(loom, layout):
     """A table entry outside the cache (a caller error) is bounded by the copy engine: the
     keys it names read as zeros, so the call completes and reports no error."""
     import torch
@@ -137,7 +150,7 @@ def test_out_of_range_page_reads_zeros_without_fault(loom):
     q, kc, vc, table, sl = paged_case(12, B, Hq, Hkv, P, [48], D, poison=False)
     bad = table.copy()
     bad[0, 1] = kc.shape[0] + 1000
-    o, lse = run_paged(loom, q, kc, vc, bad, sl, 1)
+    o, lse = run_paged(loom, q, kc, vc, bad, sl, 1, layout)
     kz, vz = kc.copy(), vc.copy()
     zero_page = np.zeros((1, P, Hkv, D), np.uint16)
     kz = np.concatenate([kz, zero_page])
