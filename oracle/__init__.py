@@ -169,14 +169,17 @@ def bf16_to_f64(bits):
     return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
 
 
-def gemm(a, b, *, rows=None):
+def gemm(a, b, *, rows=None, b_transposed=False):
     """C = A B in fp64 from bf16 A [M, K] and B [K, N] (the paper's third kernel, evaluated
     on GEMM shapes): the definition, c_ij = sum_k a_ik b_kj, with the exactly widened
-    inputs and a library matmul as its one step.  ``rows`` optionally selects rows of C."""
+    inputs and a library matmul as its one step.  ``b_transposed``: b is given [N, K] and
+    C = A b^T (c_ij = sum_k a_ik b_jk).  ``rows`` optionally selects rows of C."""
     A = bf16_to_f64(a)
     Bm = bf16_to_f64(b)
+    if b_transposed:
+        Bm = Bm.T
     if A.ndim != 2 or Bm.ndim != 2 or A.shape[1] != Bm.shape[0]:
-        raise ValueError("expected A [M, K] and B [K, N]")
+        raise ValueError("expected A [M, K] and B [K, N] ([N, K] when transposed)")
     if rows is not None:
         A = A[np.asarray(rows, dtype=np.int64)]
     return A @ Bm

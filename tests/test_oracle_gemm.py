@@ -67,3 +67,19 @@ def test_row_selection():
 def test_shape_mismatch_rejected():
     with pytest.raises(ValueError):
         oracle.gemm(_bits(7, 0, (4, 5)), _bits(7, 1, (6, 3)))
+
+
+def test_transposed_b_matches_triple_loop():
+    """b given [N, K]: c_ij = sum_k a_ik b_jk, checked element by element in plain Python."""
+    rng = np.random.default_rng(7)
+    M, K, N = 5, 7, 3
+    a = synth.f32_to_bf16(rng.standard_normal((M, K)).astype(np.float32))
+    bt = synth.f32_to_bf16(rng.standard_normal((N, K)).astype(np.float32))
+    c = oracle.gemm(a, bt, b_transposed=True)
+    A, Bt = oracle.bf16_to_f64(a), oracle.bf16_to_f64(bt)
+    for i in range(M):
+        for j in range(N):
+            ref = sum(float(A[i, k]) * float(Bt[j, k]) for k in range(K))
+            assert abs(c[i, j] - ref) <= 1e-12 * max(1.0, abs(ref))
+    with pytest.raises(ValueError):
+        oracle.gemm(a, bt)  # [N, K] taken as [K, N]: the inner sizes disagree
