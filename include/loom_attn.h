@@ -227,6 +227,10 @@ double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, in
  * the tensor-memory-access copies), CUDA (launch failure).
  */
 loom_status loom_gemm_bf16(const void* a, const void* b, void* c, int M, int N, int K, void* stream);
+/* C = A B^T with b [N, K] bf16 row-major (a linear layer's weight layout: c_ij = sum_k a_ik
+ * b_jk); B's tiles are then K-major like A's.  Everything else as loom_gemm_bf16, including
+ * the model's choice of kernel (it depends on the shape only). */
+loom_status loom_gemm_bf16_bt(const void* a, const void* b, void* c, int M, int N, int K, void* stream);
 /* The model's tile width / split count for this shape (0 for a non-positive size).  Without a
  * device the cluster occupancy is estimated as whole clusters in 8 equal SM groups. */
 int loom_gemm_tile_n(int M, int N, int K);

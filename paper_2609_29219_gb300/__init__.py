@@ -26,7 +26,7 @@ __all__ = [
     "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
     "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
     "loom_model_fwd_plan_variant", "loom_model_heg_pipe", "loom_model_fwd_time_us_design",
-    "loom_attn_decode_paged", "loom_attn_fwd_varlen", "loom_gemm_bf16", "loom_gemm_tile_n", "loom_gemm_splits", "loom_gemm_cta_pair", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
+    "loom_attn_decode_paged", "loom_attn_fwd_varlen", "loom_gemm_bf16", "loom_gemm_bf16_bt", "loom_gemm_tile_n", "loom_gemm_splits", "loom_gemm_cta_pair", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
     "loom_debug_gemm_splits", "loom_debug_gemm_cta_pair",
 ]
 
@@ -109,6 +109,8 @@ def capi() -> ctypes.CDLL:
             lib.loom_attn_fwd_varlen.restype = i32
             lib.loom_gemm_bf16.argtypes = [vp, vp, vp, i32, i32, i32, vp]
             lib.loom_gemm_bf16.restype = i32
+            lib.loom_gemm_bf16_bt.argtypes = [vp, vp, vp, i32, i32, i32, vp]
+            lib.loom_gemm_bf16_bt.restype = i32
             lib.loom_gemm_tile_n.argtypes = [i32, i32, i32]
             lib.loom_gemm_tile_n.restype = i32
             lib.loom_gemm_splits.argtypes = [i32, i32, i32]
@@ -383,23 +385,28 @@ def loom_model_heg_pipe(l: float, m: float, s: float, b_lm: int, b_ms: int) -> f
     return float(capi().loom_model_heg_pipe(float(l), float(m), float(s), int(b_lm), int(b_ms)))
 
 
-def loom_gemm_bf16(a, b, c=None, *, stream=None):
-    """C = A B (bf16, fp32 accumulation): a [M, K], b [K, N] bf16 CUDA tensors; writes and
-    returns c ([M, N] bf16, allocated if None)."""
+def loom_gemm_bf16(a, b, c=None, *, stream=None, b_transposed=False):
+    """C = A B (bf16, fp32 accumulation): a [M, K] and b [K, N] bf16 CUDA tensors, or with
+    ``b_transposed`` b [N, K] and C = A b^T (a linear layer's weight); writes and returns c
+    ([M, N] bf16, allocated if None)."""
     torch = _torch()
     bf16 = torch.bfloat16
     ap = _dev_ptr(a, "a", bf16, 2)
     bp = _dev_ptr(b, "b", bf16, 2)
     M, K = a.shape
-    K2, N = b.shape
+    if b_transposed:
+        N, K2 = b.shape
+    else:
+        K2, N = b.shape
     if K2 != K:
-        raise ValueError(f"a is [M, {K}] but b is [{K2}, N]")
+        raise ValueError(f"a is [M, {K}] but b has {K2} along K")
     if c is None:
         c = torch.empty((M, N), dtype=bf16, device=a.device)
     cp = _dev_ptr(c, "c", bf16, 2)
     if tuple(c.shape) != (M, N):
         raise ValueError("c must be [M, N]")
-    _check(capi().loom_gemm_bf16(ap, bp, cp, M, N, K, _stream_ptr(stream, a.device)), "loom_gemm_bf16")
+    fn = capi().loom_gemm_bf16_bt if b_transposed else capi().loom_gemm_bf16
+    _check(fn(ap, bp, cp, M, N, K, _stream_ptr(stream, a.device)), "loom_gemm_bf16")
     return c
 
 

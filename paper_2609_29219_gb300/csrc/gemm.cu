@@ -117,7 +117,8 @@ struct GemmParams {
   __nv_bfloat16* c;
   int M, N, K;
   int tiles_m, tiles_n, k_iters;
-  int splits;  // split-K kernel: CTAs per cluster (= per tile)
+  int splits;    // split-K kernel: CTAs per cluster (= per tile)
+  int b_kmajor;  // 1: B given [N, K] (C = A B^T), its tiles K-major like A's; 0: B [K, N]
   KernelCtl ctl;
 };
 
@@ -253,10 +254,14 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
           const uint32_t dst = sbase + s * C::STAGE_BYTES;
           mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
           tma_load_3d(dst, &tm_a, ks * C::BK, tm * C::BM, 0, bar_full + 8 * s);
+          if (p.b_kmajor) {  // BN rows of B [N, K], 64 K-columns: one box
+            tma_load_3d(dst + C::A_BYTES, &tm_b, ks * C::BK, tn * BN, 0, bar_full + 8 * s);
+          } else {
 #pragma unroll
-          for (int x = 0; x < C::NB; ++x)
-            tma_load_3d(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b, tn * BN + x * 64, ks * C::BK, 0,
-                        bar_full + 8 * s);
+            for (int x = 0; x < C::NB; ++x)
+              tma_load_3d(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b, tn * BN + x * 64, ks * C::BK, 0,
+                          bar_full + 8 * s);
+          }
         }
       }
       Abort no_abort{ab.flag + 1};
@@ -266,12 +271,13 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16(C::BM, BN, 0, 1);  // A K-major, B MN-major
       // A: K-major, 8-row groups 1024 B apart, K-step +32 B inside the swizzle row.
-      // B: MN-major, 64-column boxes B_BOX_BYTES apart (LBO), 8 K-rows 1024 B apart (SBO),
-      //    K-step +16 rows = +2048 B.
+      // B [K, N]: MN-major, 64-column boxes B_BOX_BYTES apart (LBO), 8 K-rows 1024 B apart
+      //    (SBO), K-step +16 rows = +2048 B.  B [N, K]: K-major like A.
+      const uint32_t idesc = idesc_bf16(C::BM, BN, 0, p.b_kmajor ? 0 : 1);
+      const uint32_t kstep_b = p.b_kmajor ? 2u : 128u;
       const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
-      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, C::B_BOX_BYTES, 1024);
+      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, p.b_kmajor ? 16u : C::B_BOX_BYTES, 1024);
       constexpr uint32_t kStage16 = C::STAGE_BYTES >> 4;
       int it = 0, lt = 0;
       bool ok = true;
@@ -288,7 +294,7 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
           const uint64_t da = da0 + s * kStage16, db = db0 + s * kStage16;
 #pragma unroll
           for (int kk = 0; kk < C::BK / 16; ++kk)
-            mma_ss(d, da + kk * 2, db + kk * 128, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
+            mma_ss(d, da + kk * 2, db + kk * kstep_b, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
           tc_commit(bar_empty + 8 * s);
         }
         if (!ok) break;
@@ -399,10 +405,14 @@ __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
         const uint32_t dst = sbase + s * C::STAGE_BYTES;
         mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
         tma_load_3d(dst, &tm_a, ks * C::BK, tm * C::BM, 0, bar_full + 8 * s);
+        if (p.b_kmajor) {
+          tma_load_3d(dst + C::A_BYTES, &tm_b, ks * C::BK, tn * BN, 0, bar_full + 8 * s);
+        } else {
 #pragma unroll
-        for (int x = 0; x < C::NB; ++x)
-          tma_load_3d(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b, tn * BN + x * 64, ks * C::BK, 0,
-                      bar_full + 8 * s);
+          for (int x = 0; x < C::NB; ++x)
+            tma_load_3d(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b, tn * BN + x * 64, ks * C::BK, 0,
+                        bar_full + 8 * s);
+        }
       }
       Abort no_abort{ab.flag + 1};
       for (int i = max(0, issued - C::NSTAGE); i < issued; ++i)
@@ -411,9 +421,10 @@ __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
   } else if (warp == 5) {
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16(C::BM, BN, 0, 1);
+      const uint32_t idesc = idesc_bf16(C::BM, BN, 0, p.b_kmajor ? 0 : 1);
+      const uint32_t kstep_b = p.b_kmajor ? 2u : 128u;
       const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
-      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, C::B_BOX_BYTES, 1024);
+      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, p.b_kmajor ? 16u : C::B_BOX_BYTES, 1024);
       constexpr uint32_t kStage16 = C::STAGE_BYTES >> 4;
       bool ok = true;
       for (int ks = k0, it = 0; ks < k1; ++ks, ++it) {
@@ -423,7 +434,7 @@ __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
         const uint64_t da = da0 + s * kStage16, db = db0 + s * kStage16;
 #pragma unroll
         for (int kk = 0; kk < C::BK / 16; ++kk)
-          mma_ss(tmem, da + kk * 2, db + kk * 128, idesc, (it > 0 || kk > 0) ? 1u : 0u);
+          mma_ss(tmem, da + kk * 2, db + kk * kstep_b, idesc, (it > 0 || kk > 0) ? 1u : 0u);
         tc_commit(bar_empty + 8 * s);
       }
       if (ok) tc_commit(bar_acc);  // with no stages at all this arrives at once
@@ -629,10 +640,14 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
           if (rank == 0) mbar_expect_tx(bar_full + 8 * s, 2 * C::STAGE_BYTES);
           const uint32_t dst = sbase + s * C::STAGE_BYTES;
           tma_load_3d_pair(dst, &tm_a, ks * C::BK, tm * 256 + static_cast<int>(rank) * C::BM, 0, full0);
+          if (p.b_kmajor) {  // this CTA's 128 rows of B [N, K], 64 K-columns: one box
+            tma_load_3d_pair(dst + C::A_BYTES, &tm_b, ks * C::BK, tn * C::BN + static_cast<int>(rank) * 128, 0, full0);
+          } else {
 #pragma unroll
-          for (int x = 0; x < C::NBH; ++x)
-            tma_load_3d_pair(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b,
-                             tn * C::BN + static_cast<int>(rank) * 128 + x * 64, ks * C::BK, 0, full0);
+            for (int x = 0; x < C::NBH; ++x)
+              tma_load_3d_pair(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b,
+                               tn * C::BN + static_cast<int>(rank) * 128 + x * 64, ks * C::BK, 0, full0);
+          }
         }
       }
       if (rank == 0) {  // the even CTA's barriers count both CTAs' copies
@@ -644,9 +659,10 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer (even CTA)
     if (lane == 0 && rank == 0) {
-      constexpr uint32_t idesc = idesc_bf16(256, C::BN, 0, 1);
+      const uint32_t idesc = idesc_bf16(256, C::BN, 0, p.b_kmajor ? 0 : 1);
+      const uint32_t kstep_b = p.b_kmajor ? 2u : 128u;
       const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
-      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, C::B_BOX_BYTES, 1024);
+      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, p.b_kmajor ? 16u : C::B_BOX_BYTES, 1024);
       constexpr uint32_t kStage16 = C::STAGE_BYTES >> 4;
       int it = 0, lt = 0;
       bool ok = true;
@@ -662,7 +678,7 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
           const uint64_t da = da0 + s * kStage16, db = db0 + s * kStage16;
 #pragma unroll
           for (int kk = 0; kk < C::BK / 16; ++kk)
-            mma_ss_pair(d, da + kk * 2, db + kk * 128, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
+            mma_ss_pair(d, da + kk * 2, db + kk * kstep_b, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
           tc_commit_pair_both(bar_empty + 8 * s);
         }
         if (!ok) break;
@@ -744,9 +760,10 @@ bool set_smem_attr(const void* fn, int& done_mask, int bit) {
   return true;
 }
 
-bool make_maps(const GemmArgs& a, int bm, CUtensorMap* ma, CUtensorMap* mb, CUtensorMap* mc) {
-  return matrix_map(ma, a.a, a.M, a.K, 64, bm) && matrix_map(mb, a.b, a.K, a.N, 64, 64) &&
-         (mc == nullptr || matrix_map(mc, a.c, a.M, a.N, 64, 32));
+// B's box: 64 columns x 64 K-rows of B [K, N], or 64 K-columns x b_rows rows of B [N, K].
+bool make_maps(const GemmArgs& a, int bm, int b_rows, CUtensorMap* ma, CUtensorMap* mb, CUtensorMap* mc) {
+  const bool b_ok = a.b_kmajor ? matrix_map(mb, a.b, a.N, a.K, 64, b_rows) : matrix_map(mb, a.b, a.K, a.N, 64, 64);
+  return matrix_map(ma, a.a, a.M, a.K, 64, bm) && b_ok && (mc == nullptr || matrix_map(mc, a.c, a.M, a.N, 64, 32));
 }
 
 GemmParams make_params(const GemmArgs& a, const KernelCtl& ctl, int bn, int splits) {
@@ -759,6 +776,7 @@ GemmParams make_params(const GemmArgs& a, const KernelCtl& ctl, int bn, int spli
   p.tiles_n = (a.N + bn - 1) / bn;
   p.k_iters = (a.K + 63) / 64;
   p.splits = splits;
+  p.b_kmajor = a.b_kmajor;
   p.ctl = ctl;
   return p;
 }
@@ -770,7 +788,7 @@ cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stre
   if (dev < 31 && !set_smem_attr<BN>(reinterpret_cast<const void*>(gemm_kernel<BN>), configured, dev))
     return cudaErrorInvalidValue;
   CUtensorMap ma, mb, mc;
-  if (!make_maps(a, C::BM, &ma, &mb, &mc)) return cudaErrorInvalidValue;
+  if (!make_maps(a, C::BM, BN, &ma, &mb, &mc)) return cudaErrorInvalidValue;
   const GemmParams p = make_params(a, ctl, BN, 1);
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
@@ -843,7 +861,7 @@ template <int BN>
 cudaError_t launch_splitk(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int dev, int S) {
   if (!prepare_splitk<BN>(dev)) return cudaErrorInvalidValue;
   CUtensorMap ma, mb;
-  if (!make_maps(a, GemmCfg<BN>::BM, &ma, &mb, nullptr)) return cudaErrorInvalidValue;
+  if (!make_maps(a, GemmCfg<BN>::BM, BN, &ma, &mb, nullptr)) return cudaErrorInvalidValue;
   const GemmParams p = make_params(a, ctl, BN, S);
   const long long ctas = static_cast<long long>(p.tiles_m) * p.tiles_n * S;
   if (ctas > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
@@ -900,7 +918,7 @@ cudaError_t launch_pair(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t st
   const int slots = pair_slots(dev);
   if (slots < 2 || !prepare_pair(dev)) return cudaErrorInvalidConfiguration;
   CUtensorMap ma, mb, mc;
-  if (!make_maps(a, GemmPairCfg::BM, &ma, &mb, &mc)) return cudaErrorInvalidValue;
+  if (!make_maps(a, GemmPairCfg::BM, 128, &ma, &mb, &mc)) return cudaErrorInvalidValue;
   GemmParams p = make_params(a, ctl, GemmPairCfg::BN, 1);
   p.tiles_m = (a.M + 255) / 256;  // 256-row tiles of the pair
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;

@@ -9,12 +9,13 @@ namespace loom {
 
 struct GemmArgs {
   const void* a;  // [M, K] bf16 row-major
-  const void* b;  // [K, N] bf16 row-major
+  const void* b;  // [K, N] bf16 row-major ([N, K] when b_kmajor)
   void* c;        // [M, N] bf16 row-major
   int M, N, K;
   int tile_n;     // 0: the analytic model's choice, else 64, 128, 192 or 256
   int splits;     // 0: the model's choice, else 1 (persistent tiles) or 2, 4, 8, 16 (split-K clusters)
   int pair;       // 0: the model's choice, 1: CTA-pair 256 x 256 tiles, -1: never CTA pairs
+  int b_kmajor;   // 1: b is [N, K] row-major and C = A B^T
 };
 
 struct GemmChoice {

@@ -245,15 +245,25 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
                                                                                           : LOOM_ERR_CUDA;
 }
 
-loom_status loom_gemm_bf16(const void* a, const void* b, void* c, int M, int N, int K, void* stream) {
+namespace {
+loom_status gemm_call(const void* a, const void* b, void* c, int M, int N, int K, int b_kmajor, void* stream) {
   if (!a || !b || !c) return LOOM_ERR_INVALID_ARG;
   if (M <= 0 || N <= 0 || K <= 0) return LOOM_ERR_INVALID_ARG;
   if (!aligned16(a) || !aligned16(b) || !aligned16(c)) return LOOM_ERR_MISALIGNED;
   if (K % 8 != 0 || N % 8 != 0) return LOOM_ERR_UNSUPPORTED;  // 16-byte row strides for TMA
   KernelCtl ctl;
   if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
-  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n, g_gemm_splits, g_gemm_pair};
+  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n, g_gemm_splits, g_gemm_pair, b_kmajor};
   return launch_gemm(g, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK : LOOM_ERR_CUDA;
+}
+}  // namespace
+
+loom_status loom_gemm_bf16(const void* a, const void* b, void* c, int M, int N, int K, void* stream) {
+  return gemm_call(a, b, c, M, N, K, 0, stream);
+}
+
+loom_status loom_gemm_bf16_bt(const void* a, const void* b, void* c, int M, int N, int K, void* stream) {
+  return gemm_call(a, b, c, M, N, K, 1, stream);
 }
 
 namespace {

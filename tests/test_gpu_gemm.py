@@ -187,3 +187,30 @@ def test_pair_tiles_on_thin_shapes(loom, forced, M, K, N):
     forced(0, 0, 1)
     a, b = _inputs(M * 7 + N, M, K, N)
     _check(_run(loom, a, b), oracle.gemm(a, b), K, f"pair {M}x{K}x{N}")
+
+
+@pytest.mark.parametrize("variant", ["model", "bn128", "bn256", "split4", "pair"])
+@pytest.mark.parametrize("M,K,N", [(200, 136, 304), (1000, 1000, 1000), (256, 4096, 264), (130, 64, 8)])
+def test_transposed_b(loom, forced, variant, M, K, N):
+    """b given [N, K] (C = A b^T): its tiles are K-major, in every kernel."""
+    forced(*{"model": (0, 0, 0), "bn128": (128, 1, -1), "bn256": (256, 1, -1), "split4": (128, 4, -1),
+             "pair": (0, 0, 1)}[variant])
+    a = synth.bf16_normal(M + 5, synth.STREAM_Q, (M, K))
+    bt = synth.bf16_normal(M + 5, synth.STREAM_K, (N, K))
+    c = loom.loom_gemm_bf16(to_dev(a), to_dev(bt), b_transposed=True)
+    loom.loom_attn_check_error()
+    _check(c.float().cpu().numpy().astype(np.float64), oracle.gemm(a, bt, b_transposed=True), K,
+           f"A B^T {M}x{K}x{N} {variant}")
+
+
+def test_transposed_b_matches_plain_layout_bitwise(loom, forced):
+    """The same product from B and from B^T stored [N, K]: identical fp32 sums, identical bits."""
+    import torch
+    forced(0, 0, 0)
+    M, K, N = 512, 1024, 768
+    a = to_dev(synth.bf16_normal(2, synth.STREAM_Q, (M, K)))
+    b = to_dev(synth.bf16_normal(2, synth.STREAM_K, (K, N)))
+    c1 = loom.loom_gemm_bf16(a, b)
+    c2 = loom.loom_gemm_bf16(a, b.t().contiguous(), b_transposed=True)
+    loom.loom_attn_check_error()
+    assert torch.equal(c1.view(torch.int16), c2.view(torch.int16))
