@@ -117,8 +117,7 @@ struct GemmParams {
   __nv_bfloat16* c;
   int M, N, K;
   int tiles_m, tiles_n, k_iters;
-  int splits;    // split-K kernel: CTAs per cluster (= per tile)
-  int b_kmajor;  // 1: B given [N, K] (C = A B^T), its tiles K-major like A's; 0: B [K, N]
+  int splits;  // split-K kernel: CTAs per cluster (= per tile)
   KernelCtl ctl;
 };
 
@@ -193,7 +192,8 @@ __device__ __forceinline__ void epilogue_warp(const CUtensorMap* tm_c, uint32_t 
   }
 }
 
-template <int BN>
+// BK_MAJOR: B given [N, K] (C = A B^T), its tiles K-major like A's; else B [K, N].
+template <int BN, bool BK_MAJOR>
 __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                 const __grid_constant__ CUtensorMap tm_c, const GemmParams p) {
@@ -254,7 +254,7 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
           const uint32_t dst = sbase + s * C::STAGE_BYTES;
           mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
           tma_load_3d(dst, &tm_a, ks * C::BK, tm * C::BM, 0, bar_full + 8 * s);
-          if (p.b_kmajor) {  // BN rows of B [N, K], 64 K-columns: one box
+          if constexpr (BK_MAJOR) {  // BN rows of B [N, K], 64 K-columns: one box
             tma_load_3d(dst + C::A_BYTES, &tm_b, ks * C::BK, tn * BN, 0, bar_full + 8 * s);
           } else {
 #pragma unroll
@@ -274,10 +274,10 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
       // A: K-major, 8-row groups 1024 B apart, K-step +32 B inside the swizzle row.
       // B [K, N]: MN-major, 64-column boxes B_BOX_BYTES apart (LBO), 8 K-rows 1024 B apart
       //    (SBO), K-step +16 rows = +2048 B.  B [N, K]: K-major like A.
-      const uint32_t idesc = idesc_bf16(C::BM, BN, 0, p.b_kmajor ? 0 : 1);
-      const uint32_t kstep_b = p.b_kmajor ? 2u : 128u;
+      constexpr uint32_t idesc = idesc_bf16(C::BM, BN, 0, BK_MAJOR ? 0 : 1);
+      constexpr uint32_t kstep_b = BK_MAJOR ? 2u : 128u;
       const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
-      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, p.b_kmajor ? 16u : C::B_BOX_BYTES, 1024);
+      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, BK_MAJOR ? 16u : C::B_BOX_BYTES, 1024);
       constexpr uint32_t kStage16 = C::STAGE_BYTES >> 4;
       int it = 0, lt = 0;
       bool ok = true;
@@ -342,7 +342,7 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
 // and stores them as bf16.  A second cluster barrier keeps every partial alive until all
 // peers have read it.  The summation order does not depend on timing, so the result is
 // deterministic for a given S.
-template <int BN>
+template <int BN, bool BK_MAJOR>
 __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
     gemm_splitk_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                        const GemmParams p) {
@@ -405,7 +405,7 @@ __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
         const uint32_t dst = sbase + s * C::STAGE_BYTES;
         mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
         tma_load_3d(dst, &tm_a, ks * C::BK, tm * C::BM, 0, bar_full + 8 * s);
-        if (p.b_kmajor) {
+        if constexpr (BK_MAJOR) {
           tma_load_3d(dst + C::A_BYTES, &tm_b, ks * C::BK, tn * BN, 0, bar_full + 8 * s);
         } else {
 #pragma unroll
@@ -421,10 +421,10 @@ __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
   } else if (warp == 5) {
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(C::BM, BN, 0, p.b_kmajor ? 0 : 1);
-      const uint32_t kstep_b = p.b_kmajor ? 2u : 128u;
+      constexpr uint32_t idesc = idesc_bf16(C::BM, BN, 0, BK_MAJOR ? 0 : 1);
+      constexpr uint32_t kstep_b = BK_MAJOR ? 2u : 128u;
       const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
-      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, p.b_kmajor ? 16u : C::B_BOX_BYTES, 1024);
+      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, BK_MAJOR ? 16u : C::B_BOX_BYTES, 1024);
       constexpr uint32_t kStage16 = C::STAGE_BYTES >> 4;
       bool ok = true;
       for (int ks = k0, it = 0; ks < k1; ++ks, ++it) {
@@ -576,6 +576,7 @@ __device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
                : "memory");
 }
 
+template <bool BK_MAJOR>
 __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                      const __grid_constant__ CUtensorMap tm_c, const GemmParams p) {
@@ -640,7 +641,7 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
           if (rank == 0) mbar_expect_tx(bar_full + 8 * s, 2 * C::STAGE_BYTES);
           const uint32_t dst = sbase + s * C::STAGE_BYTES;
           tma_load_3d_pair(dst, &tm_a, ks * C::BK, tm * 256 + static_cast<int>(rank) * C::BM, 0, full0);
-          if (p.b_kmajor) {  // this CTA's 128 rows of B [N, K], 64 K-columns: one box
+          if constexpr (BK_MAJOR) {  // this CTA's 128 rows of B [N, K], 64 K-columns: one box
             tma_load_3d_pair(dst + C::A_BYTES, &tm_b, ks * C::BK, tn * C::BN + static_cast<int>(rank) * 128, 0, full0);
           } else {
 #pragma unroll
@@ -659,10 +660,10 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer (even CTA)
     if (lane == 0 && rank == 0) {
-      const uint32_t idesc = idesc_bf16(256, C::BN, 0, p.b_kmajor ? 0 : 1);
-      const uint32_t kstep_b = p.b_kmajor ? 2u : 128u;
+      constexpr uint32_t idesc = idesc_bf16(256, C::BN, 0, BK_MAJOR ? 0 : 1);
+      constexpr uint32_t kstep_b = BK_MAJOR ? 2u : 128u;
       const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
-      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, p.b_kmajor ? 16u : C::B_BOX_BYTES, 1024);
+      const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, BK_MAJOR ? 16u : C::B_BOX_BYTES, 1024);
       constexpr uint32_t kStage16 = C::STAGE_BYTES >> 4;
       int it = 0, lt = 0;
       bool ok = true;
@@ -776,16 +777,15 @@ GemmParams make_params(const GemmArgs& a, const KernelCtl& ctl, int bn, int spli
   p.tiles_n = (a.N + bn - 1) / bn;
   p.k_iters = (a.K + 63) / 64;
   p.splits = splits;
-  p.b_kmajor = a.b_kmajor;
   p.ctl = ctl;
   return p;
 }
 
-template <int BN>
+template <int BN, bool BKM>
 cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int dev, int sms) {
   using C = GemmCfg<BN>;
   static int configured = 0;  // bit per device (devices 0..30)
-  if (dev < 31 && !set_smem_attr<BN>(reinterpret_cast<const void*>(gemm_kernel<BN>), configured, dev))
+  if (dev < 31 && !set_smem_attr<BN>(reinterpret_cast<const void*>(gemm_kernel<BN, BKM>), configured, dev))
     return cudaErrorInvalidValue;
   CUtensorMap ma, mb, mc;
   if (!make_maps(a, C::BM, BN, &ma, &mb, &mc)) return cudaErrorInvalidValue;
@@ -793,7 +793,7 @@ cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stre
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   const int grid = static_cast<int>(tiles < sms ? tiles : sms);
-  gemm_kernel<BN><<<grid, C::THREADS, C::BYTES, stream>>>(ma, mb, mc, p);
+  gemm_kernel<BN, BKM><<<grid, C::THREADS, C::BYTES, stream>>>(ma, mb, mc, p);
   return cudaGetLastError();
 }
 
@@ -813,11 +813,11 @@ cudaLaunchConfig_t splitk_config(int grid, int S, cudaStream_t stream, cudaLaunc
   return cfg;
 }
 
-template <int BN>
+template <int BN, bool BKM>
 bool prepare_splitk(int dev) {
   static int configured = 0;
   static int nonportable = 0;
-  const void* fn = reinterpret_cast<const void*>(gemm_splitk_kernel<BN>);
+  const void* fn = reinterpret_cast<const void*>(gemm_splitk_kernel<BN, BKM>);
   if (dev >= 31) return false;
   if (!set_smem_attr<BN>(fn, configured, dev)) return false;
   if (!(nonportable & (1 << dev))) {
@@ -827,7 +827,8 @@ bool prepare_splitk(int dev) {
   return true;
 }
 
-// CTAs of clusters of S that fit on the device at once (0: none, or cannot be queried).
+// CTAs of clusters of S that fit on the device at once (0: none, or cannot be queried); both
+// B layouts have the same resources, so the [K, N] instance answers for both.
 template <int BN>
 int splitk_slots(int dev, int S) {
   static int cache[31][5];  // [device][log2 S], value + 1 once known
@@ -836,10 +837,10 @@ int splitk_slots(int dev, int S) {
   if (dev >= 31 || lg > 4 || (1 << lg) != S) return 0;
   if (cache[dev][lg] != 0) return cache[dev][lg] - 1;
   int clusters = 0;
-  if (prepare_splitk<BN>(dev)) {
+  if (prepare_splitk<BN, false>(dev)) {
     cudaLaunchAttribute attr[1];
     cudaLaunchConfig_t cfg = splitk_config<BN>(S * 64, S, nullptr, attr);
-    if (cudaOccupancyMaxActiveClusters(&clusters, gemm_splitk_kernel<BN>, &cfg) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&clusters, gemm_splitk_kernel<BN, false>, &cfg) != cudaSuccess) {
       cudaGetLastError();
       clusters = 0;
     }
@@ -857,9 +858,9 @@ int splitk_slots_any(int dev, int bn, int S) {
   }
 }
 
-template <int BN>
+template <int BN, bool BKM>
 cudaError_t launch_splitk(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int dev, int S) {
-  if (!prepare_splitk<BN>(dev)) return cudaErrorInvalidValue;
+  if (!prepare_splitk<BN, BKM>(dev)) return cudaErrorInvalidValue;
   CUtensorMap ma, mb;
   if (!make_maps(a, GemmCfg<BN>::BM, BN, &ma, &mb, nullptr)) return cudaErrorInvalidValue;
   const GemmParams p = make_params(a, ctl, BN, S);
@@ -867,13 +868,14 @@ cudaError_t launch_splitk(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t 
   if (ctas > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = splitk_config<BN>(static_cast<int>(ctas), S, stream, attr);
-  return cudaLaunchKernelEx(&cfg, gemm_splitk_kernel<BN>, ma, mb, p);
+  return cudaLaunchKernelEx(&cfg, gemm_splitk_kernel<BN, BKM>, ma, mb, p);
 }
 
+template <bool BKM>
 bool prepare_pair(int dev) {
   static int configured = 0;
   if (dev >= 31) return false;
-  const void* fn = reinterpret_cast<const void*>(gemm_pair_kernel);
+  const void* fn = reinterpret_cast<const void*>(gemm_pair_kernel<BKM>);
   if (configured & (1 << dev)) return true;
   if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmPairCfg::BYTES) != cudaSuccess)
     return false;
@@ -902,10 +904,10 @@ int pair_slots(int dev) {
   if (dev >= 31) return 0;
   if (cache[dev] != 0) return cache[dev] - 1;
   int clusters = 0;
-  if (prepare_pair(dev)) {
+  if (prepare_pair<false>(dev)) {
     cudaLaunchAttribute attr[1];
     cudaLaunchConfig_t cfg = pair_config(128, nullptr, attr);
-    if (cudaOccupancyMaxActiveClusters(&clusters, gemm_pair_kernel, &cfg) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&clusters, gemm_pair_kernel<false>, &cfg) != cudaSuccess) {
       cudaGetLastError();
       clusters = 0;
     }
@@ -914,9 +916,10 @@ int pair_slots(int dev) {
   return 2 * clusters;
 }
 
+template <bool BKM>
 cudaError_t launch_pair(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int dev) {
   const int slots = pair_slots(dev);
-  if (slots < 2 || !prepare_pair(dev)) return cudaErrorInvalidConfiguration;
+  if (slots < 2 || !prepare_pair<BKM>(dev)) return cudaErrorInvalidConfiguration;
   CUtensorMap ma, mb, mc;
   if (!make_maps(a, GemmPairCfg::BM, 128, &ma, &mb, &mc)) return cudaErrorInvalidValue;
   GemmParams p = make_params(a, ctl, GemmPairCfg::BN, 1);
@@ -926,7 +929,27 @@ cudaError_t launch_pair(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t st
   const long long pairs = tiles < slots / 2 ? tiles : slots / 2;
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = pair_config(static_cast<int>(2 * pairs), stream, attr);
-  return cudaLaunchKernelEx(&cfg, gemm_pair_kernel, ma, mb, mc, p);
+  return cudaLaunchKernelEx(&cfg, gemm_pair_kernel<BKM>, ma, mb, mc, p);
+}
+
+template <bool BKM>
+cudaError_t launch_choice(const GemmArgs& a, const GemmChoice& c, const KernelCtl& ctl, cudaStream_t stream, int dev,
+                          int sms) {
+  if (c.pair == 1) return launch_pair<BKM>(a, ctl, stream, dev);
+  if (c.splits > 1) {
+    switch (c.tile_n) {
+      case 64: return launch_splitk<64, BKM>(a, ctl, stream, dev, c.splits);
+      case 128: return launch_splitk<128, BKM>(a, ctl, stream, dev, c.splits);
+      case 192: return launch_splitk<192, BKM>(a, ctl, stream, dev, c.splits);
+      default: return launch_splitk<256, BKM>(a, ctl, stream, dev, c.splits);
+    }
+  }
+  switch (c.tile_n) {
+    case 64: return launch_bn<64, BKM>(a, ctl, stream, dev, sms);
+    case 128: return launch_bn<128, BKM>(a, ctl, stream, dev, sms);
+    case 192: return launch_bn<192, BKM>(a, ctl, stream, dev, sms);
+    default: return launch_bn<256, BKM>(a, ctl, stream, dev, sms);
+  }
 }
 
 bool device_sms(int* dev, int* sms) {
@@ -950,21 +973,8 @@ cudaError_t launch_gemm(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t st
   if (!device_sms(&dev, &sms)) return cudaErrorNoDevice;
   const GemmChoice c = gemm_choice(a.M, a.N, a.K, {a.tile_n, a.splits, a.pair});
   if (c.tile_n == 0) return cudaErrorInvalidConfiguration;
-  if (c.pair == 1) return launch_pair(a, ctl, stream, dev);
-  if (c.splits > 1) {
-    switch (c.tile_n) {
-      case 64: return launch_splitk<64>(a, ctl, stream, dev, c.splits);
-      case 128: return launch_splitk<128>(a, ctl, stream, dev, c.splits);
-      case 192: return launch_splitk<192>(a, ctl, stream, dev, c.splits);
-      default: return launch_splitk<256>(a, ctl, stream, dev, c.splits);
-    }
-  }
-  switch (c.tile_n) {
-    case 64: return launch_bn<64>(a, ctl, stream, dev, sms);
-    case 128: return launch_bn<128>(a, ctl, stream, dev, sms);
-    case 192: return launch_bn<192>(a, ctl, stream, dev, sms);
-    default: return launch_bn<256>(a, ctl, stream, dev, sms);
-  }
+  return a.b_kmajor ? launch_choice<true>(a, c, ctl, stream, dev, sms)
+                    : launch_choice<false>(a, c, ctl, stream, dev, sms);
 }
 
 }  // namespace loom
