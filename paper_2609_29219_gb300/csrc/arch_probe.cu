@@ -23,6 +23,29 @@
 namespace {
 using namespace loom;
 __device__ __forceinline__ float ex2f_(float x){float y; asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x)); return y;}
+// One tcgen05.mma issued by the warp's elected lane while every lane runs the surrounding
+// code, so that operands and control flow are warp-uniform.
+__device__ __forceinline__ void mma_ss_el(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p, e;\n\tsetp.ne.b32 p, %4, 0;\n\telect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+__device__ __forceinline__ void mma_ts_el(uint32_t d, uint32_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p, e;\n\tsetp.ne.b32 p, %4, 0;\n\telect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+      "r"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+__device__ __forceinline__ void tc_commit_el(uint32_t bar) {
+  asm volatile(
+      "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(bar)
+      : "memory");
+}
+
 template <int MODE>
 __global__ void pipe_kernel(float* out, long long* cyc, int iters) {
   float v[8];
@@ -106,7 +129,10 @@ __global__ void __launch_bounds__(128, 1) mma_kernel(long long* out, int iters) 
 }
 // and concurrent tcgen05.ld/st traffic by 8 other warps.  Reports clocks per 128^3 GEMM.
 // smem: Q 2x32K at 0, ring 4x32K at 64K  (total 192K + 1K align)
-template <int MODE>  // bit0: bulk copies; bit1: tcgen05.ld/st traffic; bit2: busy ALU warps; bit3: commit per GEMM
+// bit0: bulk copies; bit1: tcgen05.ld/st traffic; bit2: busy ALU warps; bit3: commit per GEMM;
+// bit4: random operands; bit5: fence per GEMM; bit6: high-ILP FMA warps; bit7: prebuilt
+// descriptors; bit8: polling warps; bit9: the whole MMA warp runs the issue loop (elected lane issues)
+template <int MODE>
 __global__ void __launch_bounds__(320, 1) mix_kernel(long long* out, const uint8_t* __restrict__ g, int iters) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -131,7 +157,7 @@ __global__ void __launch_bounds__(320, 1) mix_kernel(long long* out, const uint8
   if (warp == 9) tmem_alloc(smem_u32(&tptr), 512);
   tc_fence_before(); __syncthreads(); tc_fence_after();
   const uint32_t tmem = tptr;
-  if (warp == 9 && lane == 0) {
+  if (warp == 9 && (lane == 0 || (MODE & 512))) {
     const uint32_t ids = idesc_bf16(128, 128, 0, 0), idpv = idesc_bf16(128, 128, 0, 1);
     long long t0 = 0;
     for (int rep = 0; rep < 2; ++rep) {
@@ -145,13 +171,22 @@ __global__ void __launch_bounds__(320, 1) mix_kernel(long long* out, const uint8
 #pragma unroll
           for (int t = 0; t < 2; ++t) {
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              mma_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8, dv + vs + kk * (2048 >> 4), idpv, 1);
+            for (int kk = 0; kk < 8; ++kk) {
+              if (MODE & 512)
+                mma_ts_el(tmem + 256 + t * 128, tmem + t * 128 + kk * 8, dv + vs + kk * (2048 >> 4), idpv, 1);
+              else
+                mma_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8, dv + vs + kk * (2048 >> 4), idpv, 1);
+            }
             const uint64_t dq = t ? dq1 : dq0;
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              mma_ss(tmem + t * 128, dq + ((kk / 4) * 16384 + (kk % 4) * 32) / 16,
-                     dk + ks + ((kk / 4) * 16384 + (kk % 4) * 32) / 16, ids, 1);
+            for (int kk = 0; kk < 8; ++kk) {
+              if (MODE & 512)
+                mma_ss_el(tmem + t * 128, dq + ((kk / 4) * 16384 + (kk % 4) * 32) / 16,
+                          dk + ks + ((kk / 4) * 16384 + (kk % 4) * 32) / 16, ids, 1);
+              else
+                mma_ss(tmem + t * 128, dq + ((kk / 4) * 16384 + (kk % 4) * 32) / 16,
+                       dk + ks + ((kk / 4) * 16384 + (kk % 4) * 32) / 16, ids, 1);
+            }
           }
         }
       } else
@@ -172,10 +207,13 @@ __global__ void __launch_bounds__(320, 1) mix_kernel(long long* out, const uint8
           if (MODE & 8) { tc_commit(smem_u32(&bars[3])); tc_commit(smem_u32(&bars[3])); }
         }
       }
-      tc_commit(smem_u32(&bars[0]));
+      if (MODE & 512)
+        tc_commit_el(smem_u32(&bars[0]));
+      else
+        tc_commit(smem_u32(&bars[0]));
       for (long long spin = 0; spin < (1LL << 26) && !mbar_try_wait(smem_u32(&bars[0]), rep & 1); ++spin) {}
     }
-    out[blockIdx.x] = clock64() - t0;
+    if (lane == 0) out[blockIdx.x] = clock64() - t0;
     done = 1;
   } else if (warp == 8 && lane == 0 && (MODE & 1)) {
     // bulk copies of 32 KB into the ring slots, back to back, until the MMA stream is done
@@ -415,13 +453,13 @@ int main() {
   // prefill-like MMA stream under load
   {
     const int iters = 500, smem = 6 * 32768 + 1024;
-    const int modes[12] = {0, 1, 2, 3, 4, 8, 16, 26, 32, 64, 192, 256};
-    const char* names[12] = {"alone", "bulk_copies", "tmem_ld_st", "copies_and_tmem", "mufu_warps",
+    const int modes[14] = {0, 1, 2, 3, 4, 8, 16, 26, 32, 64, 192, 256, 640, 704};
+    const char* names[14] = {"alone", "bulk_copies", "tmem_ld_st", "copies_and_tmem", "mufu_warps",
                              "commit_per_gemm", "random_operands", "random_commits_tmem",
                              "fence_per_gemm", "ilp_fma_warps", "ilp_fma_warps_lean_issue",
-                             "polling_warps"};
+                             "polling_warps", "lean_issue_warp_wide", "ilp_fma_warps_lean_issue_warp_wide"};
     printf(", \"mix_clk_per_gemm\": {");
-    for (int i = 0; i < 12; ++i) {
+    for (int i = 0; i < 14; ++i) {
       auto launch = [&] {
 #define LOOM_MIX(M)                                                                        \
   if (modes[i] == M) {                                                                     \
@@ -429,7 +467,7 @@ int main() {
     mix_kernel<M><<<sms, 320, smem>>>(d, g, iters);                                        \
   }
         LOOM_MIX(0) LOOM_MIX(1) LOOM_MIX(2) LOOM_MIX(3) LOOM_MIX(4) LOOM_MIX(8) LOOM_MIX(16)
-        LOOM_MIX(26) LOOM_MIX(32) LOOM_MIX(64) LOOM_MIX(192) LOOM_MIX(256)
+        LOOM_MIX(26) LOOM_MIX(32) LOOM_MIX(64) LOOM_MIX(192) LOOM_MIX(256) LOOM_MIX(640) LOOM_MIX(704)
 #undef LOOM_MIX
       };
       const double cyc = avg_cycles(launch, d, h, sms);

@@ -559,11 +559,13 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
     }
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // The whole warp runs this role (warp-uniform operands and waits); one elected lane
+    // issues the MMAs and commits.
+    {
       constexpr uint32_t idesc_s = idesc_bf16(C::BM, C::BN, 0, 0);  // Q, K both K-major
       constexpr uint32_t idesc_pv = idesc_bf16(C::BM, D, 0, 1);     // P from TMEM, V MN-major
       auto wait_slot = [&](int ps) {
-        return mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, ab);
+        return mbar_wait_warp(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, ab);
       };
       // Base descriptors, built once: Q tile t, and ring slot s read as K (K-major) or V
       // (MN-major); a slot or box step is a constant added to the start-address field.
@@ -578,13 +580,13 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
         const uint64_t b = dk0 + (kpos % C::NSLOT) * kSlot16;
 #pragma unroll
         for (int x = 0; x < C::NBOX; ++x)
-          mma_ss_k64(tmem + C::S_COL + t * C::BN, a + x * kQBox16, b + x * kKBox16, idesc_s, x > 0);
+          mma_ss_k64_el(tmem + C::S_COL + t * C::BN, a + x * kQBox16, b + x * kKBox16, idesc_s, x > 0);
       };
       // O_t += P_t[:, half] V_j[half, :] over K = BN/2 keys
       auto issue_pv = [&](int t, int vpos, bool acc, int half) {
         const uint64_t b = dv0 + (vpos % C::NSLOT) * kSlot16 + half * (C::BN / 2) * (128 >> 4);
         static_assert(C::BN / 2 == 64, "a half of P is one 64-key block of four K-steps");
-        mma_ts_k64(tmem + C::O_COL + t * D, tmem + C::S_COL + t * C::BN + half * (C::BN / 4), b, idesc_pv,
+        mma_ts_k64_el(tmem + C::O_COL + t * D, tmem + C::S_COL + t * C::BN + half * (C::BN / 4), b, idesc_pv,
                    acc ? 1u : 0u);
       };
       int pos = 0, cnt0 = 0, cnt1 = 0;  // ring position of K_0; S/P/O uses so far per tile
@@ -593,55 +595,55 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
       for (int r = 0, idx; ok && (idx = item_index_t<kRows, VARLEN>(p, r, cur)) >= 0; ++r) {
         const Item it = make_item_t<D, VARLEN>(p, cur, idx);
         const int nt0 = it.n_tiles0, nt = it.n_tiles;
-        if (!(ok = mbar_wait(bar_q, r & 1, p.ctl, ab) && wait_slot(pos))) break;
+        if (!(ok = mbar_wait_warp(bar_q, r & 1, p.ctl, ab) && wait_slot(pos))) break;
         tc_fence_after();
         issue_s(0, pos);
-        tc_commit(bar_s);
-        if (nt0 == 1) tc_commit(bar_qe);  // every S of tile 0 issued
-        if (!(ok = mbar_wait(bar_q + 8, r & 1, p.ctl, ab))) break;
+        tc_commit_el(bar_s);
+        if (nt0 == 1) tc_commit_el(bar_qe);  // every S of tile 0 issued
+        if (!(ok = mbar_wait_warp(bar_q + 8, r & 1, p.ctl, ab))) break;
         tc_fence_after();
         issue_s(1, pos);
-        tc_commit(bar_s + 8);
-        tc_commit(bar_empty + 8 * (pos % C::NSLOT));
-        if (nt == 1) tc_commit(bar_qe + 8);  // every S of tile 1 issued
+        tc_commit_el(bar_s + 8);
+        tc_commit_el(bar_empty + 8 * (pos % C::NSLOT));
+        if (nt == 1) tc_commit_el(bar_qe + 8);  // every S of tile 1 issued
         for (int j = 0; j < nt; ++j) {
           const int vpos = pos + 2 * j + 1, kpos = pos + 2 * j + 2;
           const bool more = j + 1 < nt;
           if (!(ok = wait_slot(vpos))) break;
           if (j < nt0) {  // query tile 0 stops at its own diagonal
-            if (!(ok = mbar_wait(bar_p, (cnt0 + j) & 1, p.ctl, ab))) break;
+            if (!(ok = mbar_wait_warp(bar_p, (cnt0 + j) & 1, p.ctl, ab))) break;
             // O_0 of the previous item must have been read out
-            if (j == 0 && r > 0 && !(ok = mbar_wait(bar_oe, (r - 1) & 1, p.ctl, ab))) break;
+            if (j == 0 && r > 0 && !(ok = mbar_wait_warp(bar_oe, (r - 1) & 1, p.ctl, ab))) break;
             tc_fence_after();
             issue_pv(0, vpos, j > 0, 0);
-            if (!(ok = mbar_wait(bar_p + 8, (cnt0 + j) & 1, p.ctl, ab))) break;
+            if (!(ok = mbar_wait_warp(bar_p + 8, (cnt0 + j) & 1, p.ctl, ab))) break;
             tc_fence_after();
             issue_pv(0, vpos, true, 1);
-            tc_commit(bar_o);
+            tc_commit_el(bar_o);
           }
           if (more) {
             if (!(ok = wait_slot(kpos))) break;
             tc_fence_after();
             if (j + 1 < nt0) {
               issue_s(0, kpos);
-              tc_commit(bar_s);
-              if (j + 2 == nt0) tc_commit(bar_qe);  // tile 0's last S of the item
+              tc_commit_el(bar_s);
+              if (j + 2 == nt0) tc_commit_el(bar_qe);  // tile 0's last S of the item
             }
           }
-          if (!(ok = mbar_wait(bar_p + 16, (cnt1 + j) & 1, p.ctl, ab))) break;
-          if (j == 0 && r > 0 && !(ok = mbar_wait(bar_oe + 8, (r - 1) & 1, p.ctl, ab))) break;
+          if (!(ok = mbar_wait_warp(bar_p + 16, (cnt1 + j) & 1, p.ctl, ab))) break;
+          if (j == 0 && r > 0 && !(ok = mbar_wait_warp(bar_oe + 8, (r - 1) & 1, p.ctl, ab))) break;
           tc_fence_after();
           issue_pv(1, vpos, j > 0, 0);
-          if (!(ok = mbar_wait(bar_p + 24, (cnt1 + j) & 1, p.ctl, ab))) break;
+          if (!(ok = mbar_wait_warp(bar_p + 24, (cnt1 + j) & 1, p.ctl, ab))) break;
           tc_fence_after();
           issue_pv(1, vpos, true, 1);
-          tc_commit(bar_o + 8);
-          tc_commit(bar_empty + 8 * (vpos % C::NSLOT));
+          tc_commit_el(bar_o + 8);
+          tc_commit_el(bar_empty + 8 * (vpos % C::NSLOT));
           if (more) {
             issue_s(1, kpos);
-            tc_commit(bar_s + 8);
-            tc_commit(bar_empty + 8 * (kpos % C::NSLOT));
-            if (j + 2 == nt) tc_commit(bar_qe + 8);  // tile 1's last S of the item
+            tc_commit_el(bar_s + 8);
+            tc_commit_el(bar_empty + 8 * (kpos % C::NSLOT));
+            if (j + 2 == nt) tc_commit_el(bar_qe + 8);  // tile 1's last S of the item
           }
         }
         cnt0 += nt0;
@@ -650,8 +652,8 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
       }
       // wait for every MMA issued above before TMEM may be released
       Abort no_abort{ab.flag + 1};
-      tc_commit(bar_drain);
-      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+      tc_commit_el(bar_drain);
+      mbar_wait_warp(bar_drain, 0, p.ctl, no_abort);
     }
   } else {
     // ------------------------------------------------------------------ softmax
@@ -862,7 +864,8 @@ __global__ void __launch_bounds__(Fwd1Cfg<D>::THREADS, 1)
     }
   } else if (warp == 5) {
     // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // The whole warp runs this role; one elected lane issues the MMAs and commits.
+    {
       constexpr uint32_t idesc_s = idesc_bf16(C::BM, C::BN, 0, 0);
       constexpr uint32_t idesc_pv = idesc_bf16(C::BM, D, 0, 1);
       const uint64_t dq = sdesc_sw128(sbase + C::Q_OFF, 16, 1024);
@@ -871,17 +874,17 @@ __global__ void __launch_bounds__(Fwd1Cfg<D>::THREADS, 1)
       constexpr uint32_t kSlot16 = C::SLOT_BYTES >> 4, kQBox16 = C::Q_BOX_BYTES >> 4;
       constexpr uint32_t kKBox16 = C::KV_BOX_BYTES >> 4;
       auto wait_slot = [&](int ps) {
-        return mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, ab);
+        return mbar_wait_warp(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, ab);
       };
       auto issue_s = [&](int buf, int kpos) {
         const uint64_t b = dk0 + (kpos % C::NSLOT) * kSlot16;
 #pragma unroll
         for (int x = 0; x < C::NBOX; ++x)
-          mma_ss_k64(tmem + C::S_COL + buf * C::BN, dq + x * kQBox16, b + x * kKBox16, idesc_s, x > 0);
+          mma_ss_k64_el(tmem + C::S_COL + buf * C::BN, dq + x * kQBox16, b + x * kKBox16, idesc_s, x > 0);
       };
       auto issue_pv = [&](int buf, int vpos, bool acc, int half) {
         const uint64_t b = dv0 + (vpos % C::NSLOT) * kSlot16 + half * (C::BN / 2) * (128 >> 4);
-        mma_ts_k64(tmem + C::O_COL, tmem + C::S_COL + buf * C::BN + half * (C::BN / 4), b, idesc_pv,
+        mma_ts_k64_el(tmem + C::O_COL, tmem + C::S_COL + buf * C::BN + half * (C::BN / 4), b, idesc_pv,
                    acc ? 1u : 0u);
       };
       int pos = 0, g = 0;  // ring position of the item's first tile; S tiles issued so far
@@ -889,47 +892,47 @@ __global__ void __launch_bounds__(Fwd1Cfg<D>::THREADS, 1)
       for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
         const Item it = make_item1<D>(p, idx);
         const int n = it.n_tiles;
-        if (!(ok = mbar_wait(bar_q, r & 1, p.ctl, ab))) break;
+        if (!(ok = mbar_wait_warp(bar_q, r & 1, p.ctl, ab))) break;
         // S_0 and S_1 of the item into the two buffers
         for (int j = 0; j < 2 && j < n; ++j) {
           const int kp = pos + ring_pos_k(j);
           if (!(ok = wait_slot(kp))) break;
           tc_fence_after();
           issue_s((g + j) & 1, kp);
-          tc_commit(bar_s + 8 * ((g + j) & 1));
-          tc_commit(bar_empty + 8 * (kp % C::NSLOT));
+          tc_commit_el(bar_s + 8 * ((g + j) & 1));
+          tc_commit_el(bar_empty + 8 * (kp % C::NSLOT));
         }
         if (!ok) break;
-        if (n <= 2) tc_commit(bar_qe);  // every S of this item issued
+        if (n <= 2) tc_commit_el(bar_qe);  // every S of this item issued
         for (int j = 0; j < n; ++j) {
           const int gj = g + j, buf = gj & 1;
           const int vp = pos + ring_pos_v(j, n);
           if (!(ok = wait_slot(vp))) break;
-          if (!(ok = mbar_wait(bar_p + 16 * buf, (gj >> 1) & 1, p.ctl, ab))) break;
-          if (j == 0 && r > 0 && !(ok = mbar_wait(bar_oe, (r - 1) & 1, p.ctl, ab))) break;
+          if (!(ok = mbar_wait_warp(bar_p + 16 * buf, (gj >> 1) & 1, p.ctl, ab))) break;
+          if (j == 0 && r > 0 && !(ok = mbar_wait_warp(bar_oe, (r - 1) & 1, p.ctl, ab))) break;
           tc_fence_after();
           issue_pv(buf, vp, j > 0, 0);
-          if (!(ok = mbar_wait(bar_p + 16 * buf + 8, (gj >> 1) & 1, p.ctl, ab))) break;
+          if (!(ok = mbar_wait_warp(bar_p + 16 * buf + 8, (gj >> 1) & 1, p.ctl, ab))) break;
           tc_fence_after();
           issue_pv(buf, vp, true, 1);
-          tc_commit(bar_o + 8 * buf);
-          tc_commit(bar_empty + 8 * (vp % C::NSLOT));
+          tc_commit_el(bar_o + 8 * buf);
+          tc_commit_el(bar_empty + 8 * (vp % C::NSLOT));
           if (j + 2 < n) {  // S_{j+2} into the buffer P_j V_j has just been issued from
             const int kp = pos + ring_pos_k(j + 2);
             if (!(ok = wait_slot(kp))) break;
             tc_fence_after();
             issue_s(buf, kp);
-            tc_commit(bar_s + 8 * buf);
-            tc_commit(bar_empty + 8 * (kp % C::NSLOT));
-            if (j + 3 == n) tc_commit(bar_qe);
+            tc_commit_el(bar_s + 8 * buf);
+            tc_commit_el(bar_empty + 8 * (kp % C::NSLOT));
+            if (j + 3 == n) tc_commit_el(bar_qe);
           }
         }
         g += n;
         pos += 2 * n;
       }
       Abort no_abort{ab.flag + 1};
-      tc_commit(bar_drain);
-      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+      tc_commit_el(bar_drain);
+      mbar_wait_warp(bar_drain, 0, p.ctl, no_abort);
     }
   } else {
     // ------------------------------------------------------------------ softmax
@@ -1116,7 +1119,8 @@ __global__ void __launch_bounds__(Fwd3Cfg<D>::THREADS, 1)
     }
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // The whole warp runs this role; one elected lane issues the MMAs and commits.
+    {
       constexpr uint32_t idesc_s = idesc_bf16(C::BM, C::BN, 0, 0);
       constexpr uint32_t idesc_pv = idesc_bf16(C::BM, D, 0, 1);
       const uint64_t dq0 = sdesc_sw128(sbase + C::Q_OFF, 16, 1024);
@@ -1125,7 +1129,7 @@ __global__ void __launch_bounds__(Fwd3Cfg<D>::THREADS, 1)
       constexpr uint32_t kSlot16 = C::SLOT_BYTES >> 4, kQTile16 = C::Q_TILE_BYTES >> 4;
       constexpr uint32_t kQBox16 = C::Q_BOX_BYTES >> 4, kKBox16 = C::KV_BOX_BYTES >> 4;
       auto wait_slot = [&](int ps) {
-        return mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, ab);
+        return mbar_wait_warp(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, ab);
       };
       long long gk = 0;  // S tiles issued in earlier items (both query tiles)
       int pos = 0, cnt = 0;  // ring position of the item's K_0; per-tile S count before the item
@@ -1141,16 +1145,16 @@ __global__ void __launch_bounds__(Fwd3Cfg<D>::THREADS, 1)
         const uint64_t b = dk0 + (kp % C::NSLOT) * kSlot16;
 #pragma unroll
         for (int x = 0; x < C::NBOX; ++x)
-          mma_ss_k64(tmem + C::S_COL + buf * C::BN, a + x * kQBox16, b + x * kKBox16, idesc_s, x > 0);
-        tc_commit(bar_s + 8 * buf);
-        if (t == 1) tc_commit(bar_empty + 8 * (kp % C::NSLOT));  // both tiles have used K_j
-        if (k == 2 * n - 1) tc_commit(bar_qe);                   // the item's last S
+          mma_ss_k64_el(tmem + C::S_COL + buf * C::BN, a + x * kQBox16, b + x * kKBox16, idesc_s, x > 0);
+        tc_commit_el(bar_s + 8 * buf);
+        if (t == 1) tc_commit_el(bar_empty + 8 * (kp % C::NSLOT));  // both tiles have used K_j
+        if (k == 2 * n - 1) tc_commit_el(bar_qe);                   // the item's last S
         return true;
       };
       for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
         const Item it = make_item<D>(p, idx);
         const int n = it.n_tiles;
-        if (!(ok = mbar_wait(bar_q, r & 1, p.ctl, ab))) break;
+        if (!(ok = mbar_wait_warp(bar_q, r & 1, p.ctl, ab))) break;
         for (int k = 0; ok && k < 3 && k < 2 * n; ++k) ok = issue_s(k, n);
         for (int m = 0; ok && m < 2 * n; ++m) {
           const int t = m & 1, j = m >> 1;
@@ -1159,18 +1163,18 @@ __global__ void __launch_bounds__(Fwd3Cfg<D>::THREADS, 1)
           const uint32_t par = static_cast<uint32_t>((km / 3) & 1);
           const int vp = pos + ring_pos_v(j, n);
           if (!(ok = wait_slot(vp))) break;
-          if (!(ok = mbar_wait(bar_p + 16 * buf, par, p.ctl, ab))) break;
-          if (j == 0 && r > 0 && !(ok = mbar_wait(bar_oe + 8 * t, (r - 1) & 1, p.ctl, ab))) break;
+          if (!(ok = mbar_wait_warp(bar_p + 16 * buf, par, p.ctl, ab))) break;
+          if (j == 0 && r > 0 && !(ok = mbar_wait_warp(bar_oe + 8 * t, (r - 1) & 1, p.ctl, ab))) break;
           tc_fence_after();
           const uint64_t b = dv0 + (vp % C::NSLOT) * kSlot16;
-          mma_ts_k64(tmem + C::O_COL + t * D, tmem + C::S_COL + buf * C::BN, b, idesc_pv, j > 0 ? 1u : 0u);
-          if (!(ok = mbar_wait(bar_p + 16 * buf + 8, par, p.ctl, ab))) break;
+          mma_ts_k64_el(tmem + C::O_COL + t * D, tmem + C::S_COL + buf * C::BN, b, idesc_pv, j > 0 ? 1u : 0u);
+          if (!(ok = mbar_wait_warp(bar_p + 16 * buf + 8, par, p.ctl, ab))) break;
           tc_fence_after();
-          mma_ts_k64(tmem + C::O_COL + t * D, tmem + C::S_COL + buf * C::BN + C::BN / 4,
+          mma_ts_k64_el(tmem + C::O_COL + t * D, tmem + C::S_COL + buf * C::BN + C::BN / 4,
                      b + (C::BN / 2) * (128 >> 4), idesc_pv, 1u);
           const int g = cnt + j;  // this tile's S number across items
-          tc_commit(bar_o + 8 * (2 * t + (g & 1)));
-          if (t == 1) tc_commit(bar_empty + 8 * (vp % C::NSLOT));  // both tiles have used V_j
+          tc_commit_el(bar_o + 8 * (2 * t + (g & 1)));
+          if (t == 1) tc_commit_el(bar_empty + 8 * (vp % C::NSLOT));  // both tiles have used V_j
           if (m + 3 < 2 * n) ok = issue_s(m + 3, n);                // into the buffer just freed
         }
         gk += 2 * n;
@@ -1178,8 +1182,8 @@ __global__ void __launch_bounds__(Fwd3Cfg<D>::THREADS, 1)
         pos += 2 * n;
       }
       Abort no_abort{ab.flag + 1};
-      tc_commit(bar_drain);
-      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+      tc_commit_el(bar_drain);
+      mbar_wait_warp(bar_drain, 0, p.ctl, no_abort);
     }
   } else {
     // ------------------------------------------------------------------ softmax
