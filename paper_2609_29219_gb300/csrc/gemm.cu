@@ -78,6 +78,22 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity,
     }
   }
 }
+// Warp-wide form of mbar_wait_cluster (warp-uniform result).
+__device__ __forceinline__ bool mbar_wait_cluster_warp(uint32_t bar, uint32_t parity, const KernelCtl& ctl,
+                                                       const Abort& ab) {
+  if (__all_sync(0xffffffffu, mbar_try_wait_cluster(bar, parity))) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 16; ++i)
+      if (__all_sync(0xffffffffu, mbar_try_wait_cluster(bar, parity))) return true;
+    const bool give_up = ab.raised() || (globaltimer_ns() - t0 > ctl.timeout_ns);
+    if (__any_sync(0xffffffffu, give_up)) {
+      if ((threadIdx.x & 31) == 0) ab.raise(ctl);
+      return false;
+    }
+  }
+}
 __device__ __forceinline__ float4 ld_dsmem_f4(uint32_t addr) {
   float4 v;
   asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
@@ -270,7 +286,7 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
     }
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    {  // the whole warp runs this role; one elected lane issues
       // A: K-major, 8-row groups 1024 B apart, K-step +32 B inside the swizzle row.
       // B [K, N]: MN-major, 64-column boxes B_BOX_BYTES apart (LBO), 8 K-rows 1024 B apart
       //    (SBO), K-step +16 rows = +2048 B.  B [N, K]: K-major like A.
@@ -284,25 +300,25 @@ __global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
       for (int t = blockIdx.x; ok && t < tiles; t += gridDim.x, ++lt) {
         const int b = lt & 1, use = lt >> 1;
         // the epilogue has read this accumulator's previous tile out
-        if (lt >= 2 && !(ok = mbar_wait(bar_acce + 8 * b, (use - 1) & 1, p.ctl, ab))) break;
+        if (lt >= 2 && !(ok = mbar_wait_warp(bar_acce + 8 * b, (use - 1) & 1, p.ctl, ab))) break;
         tc_fence_after();
         const uint32_t d = tmem + static_cast<uint32_t>(b * BN);
         for (int ks = 0; ks < p.k_iters; ++ks, ++it) {
           const int s = it % C::NSTAGE;
-          if (!(ok = mbar_wait(bar_full + 8 * s, (it / C::NSTAGE) & 1, p.ctl, ab))) break;
+          if (!(ok = mbar_wait_warp(bar_full + 8 * s, (it / C::NSTAGE) & 1, p.ctl, ab))) break;
           tc_fence_after();
           const uint64_t da = da0 + s * kStage16, db = db0 + s * kStage16;
 #pragma unroll
           for (int kk = 0; kk < C::BK / 16; ++kk)
-            mma_ss(d, da + kk * 2, db + kk * kstep_b, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
-          tc_commit(bar_empty + 8 * s);
+            mma_ss_el(d, da + kk * 2, db + kk * kstep_b, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
+          tc_commit_el(bar_empty + 8 * s);
         }
         if (!ok) break;
-        tc_commit(bar_acc + 8 * b);  // the tile's accumulator is complete
+        tc_commit_el(bar_acc + 8 * b);  // the tile's accumulator is complete
       }
       Abort no_abort{ab.flag + 1};
-      tc_commit(bar_drain);
-      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+      tc_commit_el(bar_drain);
+      mbar_wait_warp(bar_drain, 0, p.ctl, no_abort);
     }
   } else {
     // ------------------------------------------------------------------ epilogue (warps 0-7)
@@ -420,7 +436,7 @@ __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
     }
   } else if (warp == 5) {
     // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    {  // the whole warp runs this role; one elected lane issues
       constexpr uint32_t idesc = idesc_bf16(C::BM, BN, 0, BK_MAJOR ? 0 : 1);
       constexpr uint32_t kstep_b = BK_MAJOR ? 2u : 128u;
       const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
@@ -429,18 +445,18 @@ __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
       bool ok = true;
       for (int ks = k0, it = 0; ks < k1; ++ks, ++it) {
         const int s = it % C::NSTAGE;
-        if (!(ok = mbar_wait(bar_full + 8 * s, (it / C::NSTAGE) & 1, p.ctl, ab))) break;
+        if (!(ok = mbar_wait_warp(bar_full + 8 * s, (it / C::NSTAGE) & 1, p.ctl, ab))) break;
         tc_fence_after();
         const uint64_t da = da0 + s * kStage16, db = db0 + s * kStage16;
 #pragma unroll
         for (int kk = 0; kk < C::BK / 16; ++kk)
-          mma_ss(tmem, da + kk * 2, db + kk * kstep_b, idesc, (it > 0 || kk > 0) ? 1u : 0u);
-        tc_commit(bar_empty + 8 * s);
+          mma_ss_el(tmem, da + kk * 2, db + kk * kstep_b, idesc, (it > 0 || kk > 0) ? 1u : 0u);
+        tc_commit_el(bar_empty + 8 * s);
       }
-      if (ok) tc_commit(bar_acc);  // with no stages at all this arrives at once
+      if (ok) tc_commit_el(bar_acc);  // with no stages at all this arrives at once
       Abort no_abort{ab.flag + 1};
-      tc_commit(bar_drain);
-      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+      tc_commit_el(bar_drain);
+      mbar_wait_warp(bar_drain, 0, p.ctl, no_abort);
     }
   } else {
     // ------------------------------------------------------------------ partial tile -> smem
@@ -555,11 +571,13 @@ __device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
       : "memory");
 }
+// The pair MMA and its commits, executed by the whole issuing warp with one elected lane
+// issuing (see mma_ss_el).
 __device__ __forceinline__ void mma_ss_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                             uint32_t accumulate) {
   asm volatile(
-      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "{\n\t.reg .pred p, e;\n\tsetp.ne.b32 p, %4, 0;\n\telect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
@@ -567,13 +585,16 @@ __device__ __forceinline__ void mma_ss_pair(uint32_t d_tmem, uint64_t a_desc, ui
 // so far have completed.
 __device__ __forceinline__ void tc_commit_pair_both(uint32_t bar) {
   asm volatile(
-      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n\t}" ::"r"(bar),
       "h"(static_cast<uint16_t>(3))
       : "memory");
 }
 __device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
-  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-               : "memory");
+  asm volatile(
+      "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(bar)
+      : "memory");
 }
 
 template <bool BK_MAJOR>
@@ -659,7 +680,7 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
     }
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer (even CTA)
-    if (lane == 0 && rank == 0) {
+    if (rank == 0) {  // the whole warp; one elected lane issues
       constexpr uint32_t idesc = idesc_bf16(256, C::BN, 0, BK_MAJOR ? 0 : 1);
       constexpr uint32_t kstep_b = BK_MAJOR ? 2u : 128u;
       const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
@@ -669,12 +690,12 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
       bool ok = true;
       for (int t = pair; ok && t < tiles; t += n_pairs, ++lt) {
         const int b = lt & 1, use = lt >> 1;
-        if (lt >= 2 && !(ok = mbar_wait_cluster(bar_acce + 8 * b, (use - 1) & 1, p.ctl, ab))) break;
+        if (lt >= 2 && !(ok = mbar_wait_cluster_warp(bar_acce + 8 * b, (use - 1) & 1, p.ctl, ab))) break;
         tc_fence_after();
         const uint32_t d = tmem + static_cast<uint32_t>(b * C::BN);
         for (int ks = 0; ks < p.k_iters; ++ks, ++it) {
           const int s = it % C::NSTAGE;
-          if (!(ok = mbar_wait(bar_full + 8 * s, (it / C::NSTAGE) & 1, p.ctl, ab))) break;
+          if (!(ok = mbar_wait_warp(bar_full + 8 * s, (it / C::NSTAGE) & 1, p.ctl, ab))) break;
           tc_fence_after();
           const uint64_t da = da0 + s * kStage16, db = db0 + s * kStage16;
 #pragma unroll
@@ -687,7 +708,7 @@ __global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
       }
       Abort no_abort{ab.flag + 1};
       tc_commit_pair(bar_drain);
-      mbar_wait(bar_drain, 0, p.ctl, no_abort);
+      mbar_wait_warp(bar_drain, 0, p.ctl, no_abort);
     }
   } else {
     // ------------------------------------------------------------------ epilogue (both CTAs, warps 0-7)
