@@ -42,14 +42,15 @@ struct ArchDesc {
   double softmax_clk_per_key;       // softmax of one 128-row tile alone, clocks per key (measured)
   double softmax_pair_clk_per_key;  // two tiles' softmax running together, clocks per key (measured)
   double l2_bytes;                  // L2 cache capacity (specification)
-  double mma_issue_busy_factor;     // MMA issue stream slowdown while two softmax warpgroups
-                                    // are busy on the SM (measured: 1338 vs 512 clk per GEMM)
+  double mma_issue_busy_factor;     // MMA stream slowdown while high-ILP warps share the SM with
+                                    // the MMA warp issuing warp-wide (measured: 546 vs 512 clk
+                                    // per 128^3 GEMM; 1338 when a lone lane issues)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 2.6,
+    129.0e6, 1.07,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -110,17 +111,21 @@ constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int design, int bn, int slo
   double body = 0.0;
   if (design == 2) {
     // per pair of tile-iterations the tensor pipe needs 2 * mma; each tile's chain (its
-    // softmax, then its P.V and next S on the tensor pipe, two barrier round trips) must
-    // fit in the period, while the other tile's softmax overlaps it
-    body = dmax(2 * p.t_mma_ns, p.t_softmax_ns + p.t_mma_ns + 2 * sync) / 2;
+    // softmax, then its P.V and next S on the tensor pipe, one barrier round trip: the
+    // warp-wide MMA issuer picks P up at once) must fit in the period, while the other
+    // tile's softmax overlaps it
+    body = dmax(2 * p.t_mma_ns, p.t_softmax_ns + p.t_mma_ns + sync) / 2;
   } else if (design == 1) {
     body = dmax(p.t_mma_ns, p.t_softmax_ns) + sync;  // softmax and MMA overlap fully
   } else {
-    // both softmaxes run together (sharing MUFU and issue slots) and overlap the MMAs;
-    // the single MMA-issuing thread then competes with two busy warpgroups for issue
-    // slots, which stretches its stream of MMAs
+    // both softmaxes run together (sharing MUFU and issue slots) and overlap the MMAs,
+    // whose stream is stretched by the busy warps; yet every S is issued behind a P.V of
+    // the other tile on the single MMA stream, so a tile's chain still holds its softmax,
+    // a P.V + S and two barrier round trips (in-kernel clock counters: the softmax waits
+    // ~1060 clk per step for S, against ~760 in design 2)
     const double pair = a.softmax_pair_clk_per_key * bn / clk;
-    body = (dmax(2 * p.t_mma_ns * a.mma_issue_busy_factor, pair) + sync) / 2;
+    body = dmax(dmax(2 * p.t_mma_ns * a.mma_issue_busy_factor, pair),
+                p.t_softmax_ns + p.t_mma_ns + 2 * sync) / 2;
   }
   p.t_iter_ns = heg_pipe(p.t_load_ns, body, 0.0, b_lm, b_ms);
   // resources (Eq. 8 constraints)
