@@ -246,54 +246,17 @@ __device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
-// Issue-lean GEMM blocks: the MMA-issuing warp shares its SM sub-partition with
-// softmax warps that can issue every cycle, so every instruction on the issue path
-// delays the tensor pipe.  These helpers issue several K=16 MMAs from one asm block:
-// descriptors advance by immediate offsets (16-byte units in the start-address field),
-// and the accumulate predicate is set up once.
+// Issue-lean MMA blocks, executed by a whole (converged) warp with warp-uniform operands,
+// one elected lane issuing.  The MMA warp shares its SM sub-partition with softmax or
+// epilogue warps that can issue every cycle; a lone issuing lane in divergent code loses
+// most of its issue slots to them (a 128x128x128 GEMM stream: 1338 clk against 546
+// warp-wide, 512 alone).  Each block issues four K=16 MMAs from one asm statement:
+// descriptors advance by immediate offsets (16-byte units in the start-address field) and
+// the accumulate predicate is set up once.  Every call of one warp elects the same lane,
+// so that lane's commits (tc_commit_el) track its own MMAs.
 //
 // Four K-steps of 128-byte-swizzled K-major A and B: A/B advance by 32 bytes (2 units)
 // per step within a 64-element swizzle row.
-__device__ __forceinline__ void mma_ss_k64(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
-                                           uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p, q;\n\t.reg .b64 a1, a2, a3, b1, b2, b3;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "setp.eq.b32 q, %3, %3;\n\t"
-      "add.s64 a1, %1, 2;\n\tadd.s64 b1, %2, 2;\n\t"
-      "add.s64 a2, %1, 4;\n\tadd.s64 b2, %2, 4;\n\t"
-      "add.s64 a3, %1, 6;\n\tadd.s64 b3, %2, 6;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], a1, b1, %3, q;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], a2, b2, %3, q;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], a3, b3, %3, q;\n\t}" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// Four K-steps with A in TMEM (advancing 8 columns = 16 bf16 per step) and an MN-major
-// B whose K rows advance by 16 rows x 128 bytes (128 units) per step.
-__device__ __forceinline__ void mma_ts_k64(uint32_t d_tmem, uint32_t a_tmem, uint64_t b,
-                                           uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p, q;\n\t.reg .b64 b1, b2, b3;\n\t.reg .b32 t1, t2, t3;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "setp.eq.b32 q, %3, %3;\n\t"
-      "add.s32 t1, %1, 8;\n\tadd.s64 b1, %2, 128;\n\t"
-      "add.s32 t2, %1, 16;\n\tadd.s64 b2, %2, 256;\n\t"
-      "add.s32 t3, %1, 24;\n\tadd.s64 b3, %2, 384;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [t1], b1, %3, q;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [t2], b2, %3, q;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [t3], b3, %3, q;\n\t}" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-// Warp-wide forms of the two blocks above and of tc_commit below: the whole (converged)
-// warp executes them with warp-uniform operands and one elected lane issues.  A lone
-// issuing lane in divergent code loses most of its issue slots to high-ILP warps on its
-// SM sub-partition (a 128x128x128 GEMM stream: 1338 clk against 546 warp-wide, 512 alone);
-// every call of one warp elects the same lane, so its commits track its own MMAs.
 __device__ __forceinline__ void mma_ss_k64_el(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
                                               uint32_t accumulate) {
   asm volatile(
@@ -311,6 +274,8 @@ __device__ __forceinline__ void mma_ss_k64_el(uint32_t d_tmem, uint64_t a, uint6
       "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// Four K-steps with A in TMEM (advancing 8 columns = 16 bf16 per step) and an MN-major
+// B whose K rows advance by 16 rows x 128 bytes (128 units) per step.
 __device__ __forceinline__ void mma_ts_k64_el(uint32_t d_tmem, uint32_t a_tmem, uint64_t b,
                                               uint32_t idesc, uint32_t accumulate) {
   asm volatile(
@@ -328,6 +293,7 @@ __device__ __forceinline__ void mma_ts_k64_el(uint32_t d_tmem, uint32_t a_tmem, 
       "r"(a_tmem), "l"(b), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// One K=16 step, both operands in shared memory.
 __device__ __forceinline__ void mma_ss_el(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                           uint32_t accumulate) {
   asm volatile(
