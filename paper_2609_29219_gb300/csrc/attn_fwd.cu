@@ -11,7 +11,8 @@
 //
 //   warp 8 (loader, 1 thread)   Q0, Q1 once; then K_0, V_0, K_1, V_1, ... into an
 //                               NSLOT-deep ring of 128B-swizzled shared-memory slots
-//   warp 9 (MMA, 1 thread)      S_t = Q_t K_j^T          (SS MMA, fp32 in TMEM)
+//   warp 9 (MMA, whole warp,    S_t = Q_t K_j^T          (SS MMA, fp32 in TMEM)
+//     one elected lane issues)
 //                               O_t += P_t V_j           (TS MMA: P read from TMEM)
 //                               issue order S0 S1 | PV0 S0' | PV1 S1' | ... so the
 //                               tensor pipe works on one tile while the other tile's

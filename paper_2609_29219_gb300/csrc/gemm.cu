@@ -7,7 +7,8 @@
 //   warp 8 (loader, 1 thread)   A tile 128 x 64 and B tile 64 x BN per K stage into an
 //                               NSTAGE-deep ring of 128B-swizzled slots (TMA, full/empty
 //                               mbarriers)
-//   warp 9 (MMA, 1 thread)      tcgen05.mma kind::f16, M = 128, N = BN, K = 16: A K-major,
+//   warp 9 (MMA, whole warp,    tcgen05.mma kind::f16, M = 128, N = BN, K = 16: A K-major,
+//     one elected lane issues)
 //                               B MN-major (rows of B are contiguous in N), fp32 into one of
 //                               two TMEM accumulators
 //   warps 0-7 (epilogue)        warp w reads TMEM lanes 32 (w mod 4) .. + 31 (its 32 rows
