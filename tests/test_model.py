@@ -61,6 +61,17 @@ def test_fwd_plan_is_argmin_over_designs(loom, D):
         assert v["smem_bytes"] <= 227 * 1024 and v["tmem_cols"] <= 512
 
 
+@pytest.mark.parametrize("D", [64, 128])
+def test_fwd_plan_ranks_the_measured_best_design_first(loom, D):
+    # GB300 same-box measurements (warp-wide MMA issue): design 2 leads at both head
+    # dimensions (D=128: 1481 vs 1370 TFLOP/s for design 1; D=64: 1010 vs 874 for design 3
+    # and 813 for design 1), and at D=64 design 3 measures ahead of design 1
+    t = {d: loom.loom_model_fwd_plan_variant(D, d) for d in (1, 2, 3)}
+    assert loom.loom_model_fwd_plan(D)["design"] == 2
+    if D == 64:
+        assert t[2]["t_iter_ns"] < t[3]["t_iter_ns"] < t[1]["t_iter_ns"]
+
+
 def test_three_s_buffers_do_not_fit_at_d128(loom):
     # 3 S buffers of 128 columns + 2 O tiles of 128 columns = 640 > 512 TMEM columns
     assert loom.loom_model_fwd_plan_variant(128, 3) is None
