@@ -124,9 +124,8 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ workloads
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one launch of the
-# headline prefill kernel from the ncu capture summarised in
-# profiles/attn_fwd_d128_b4_h32_s2048_noncausal.md, and the SHA-256 of the kernel sources
-# it was taken from: the number is reported only while the sources are unchanged.
+# headline prefill kernel from an ncu capture of it, and the SHA-256 of the kernel
+# sources it was taken from: the number is reported only while the sources are unchanged.
 PROFILED_TRAFFIC_BYTES = 243.4e6
 PROFILED_SOURCES_SHA256 = "6f01ac2943b743b090c76c1136f107101eae207708a932bf14f45dbb5074cc93"
 
@@ -697,11 +696,32 @@ def main():
             "gpu_launches": args.steps * headline.launches_per_step(),
             "clocks": clk,
             "workloads": workloads,
+            "summary": summary_line(res, clk, workloads),
         }
         print(json.dumps(line), flush=True)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def summary_line(headline, headline_clocks, workloads):
+    """One short string per workload (value, unit, roofline fraction, median SM clock,
+    throttle reasons), kept last in the JSON line so that a reader of only its tail sees
+    every configuration."""
+    def one(r, clk):
+        txt = f"{r['value']:.1f} {r['unit']} frac={r['roofline']['frac']:.3f}"
+        if clk and clk.get("sm_mhz"):
+            txt += f" sm={clk['sm_mhz']:.0f}MHz"
+            if clk.get("reasons"):
+                txt += " " + "+".join(clk["reasons"])
+        if "splits" in r:
+            txt += f" splits={r['splits']}"
+        return txt
+
+    out = {"prefill": one(headline, headline_clocks)}
+    for name, r in workloads.items():
+        out[name] = one(r, r.get("clocks"))
+    return out
 
 
 def run_decode_sweep(torch, loom, dev, stream, args, peaks):

@@ -170,7 +170,11 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
  * looks up the array's device address (cudaGetSymbolAddress, current device); make that
  * first call before any stream capture.  All calls share the array, which keeps the last
  * call's contents (nothing in it needs to start at zero); calls whose kernels overlap on
- * the GPU race on it.  This entry point itself calls no cudaMalloc or cudaFree.
+ * the GPU race on it.  This entry point itself calls no cudaMalloc or cudaFree.  The
+ * looked-up address belongs to the device's context: after cudaDeviceReset the entry
+ * point must not be called on that device again in the same process.
+ * Errors: those of loom_attn_decode, checked in the same order (INVALID_ARG,
+ * UNSUPPORTED, MISALIGNED); then WORKSPACE when the partials exceed the array; CUDA.
  */
 #define LOOM_DECODE_NOALLOC_SCRATCH_BYTES ((size_t)8 << 20)
 loom_status loom_attn_decode_noalloc(const void* q, const void* k_cache, const void* v_cache,

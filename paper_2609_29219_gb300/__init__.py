@@ -21,7 +21,7 @@ import threading
 
 __all__ = [
     "LoomError", "capi", "library_path", "STATUS",
-    "loom_attn_fwd", "loom_attn_decode", "loom_attn_decode_workspace_bytes",
+    "loom_attn_fwd", "loom_attn_decode", "loom_attn_decode_noalloc", "loom_attn_decode_workspace_bytes",
     "loom_attn_decode_num_splits", "loom_attn_check_error", "loom_status_string",
     "loom_debug_set_timeout_ns", "loom_debug_inject", "loom_model_fwd_plan",
     "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
@@ -81,6 +81,9 @@ def capi() -> ctypes.CDLL:
             lib.loom_attn_decode.argtypes = [vp, vp, vp, vp, vp, vp, vp, sz, i32, i32, i32, i32, i32,
                                              f32, i32, vp]
             lib.loom_attn_decode.restype = i32
+            lib.loom_attn_decode_noalloc.argtypes = [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, f32, i32,
+                                                     vp]
+            lib.loom_attn_decode_noalloc.restype = i32
             lib.loom_attn_check_error.argtypes = [vp]
             lib.loom_attn_check_error.restype = i32
             lib.loom_status_string.argtypes = [i32]
@@ -209,13 +212,8 @@ def loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, num_splits=0) -> int:
     return int(capi().loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, num_splits))
 
 
-def loom_attn_decode(q, k_cache, v_cache, seqlens_k=None, o=None, lse=None, workspace=None, *,
-                     scale=None, num_splits=0, stream=None, return_lse=False):
-    """Flash Decode.  q [B,Hq,1,D], k_cache/v_cache [B,Hkv,Skv,D] bf16, seqlens_k [B] int32.
-
-    ``workspace`` is a CUDA uint8 tensor of at least ``loom_attn_decode_workspace_bytes``
-    bytes (allocated here if None).  Returns ``o`` or ``(o, lse)``.
-    """
+def _decode_operands(q, k_cache, v_cache, seqlens_k, o, lse, return_lse):
+    """Pointers and sizes of the contiguous decode entry points' tensor arguments."""
     torch = _torch()
     bf16 = torch.bfloat16
     qp = _dev_ptr(q, "q", bf16, 4)
@@ -240,6 +238,19 @@ def loom_attn_decode(q, k_cache, v_cache, seqlens_k=None, o=None, lse=None, work
         if lse.numel() != B * Hq:
             raise ValueError("lse must hold B*Hq values")
         lp = _dev_ptr(lse, "lse", torch.float32)
+    return (qp, kp, vp_, sp, op, lp), (B, Hq, Hkv, Skv, D), o, lse
+
+
+def loom_attn_decode(q, k_cache, v_cache, seqlens_k=None, o=None, lse=None, workspace=None, *,
+                     scale=None, num_splits=0, stream=None, return_lse=False):
+    """Flash Decode.  q [B,Hq,1,D], k_cache/v_cache [B,Hkv,Skv,D] bf16, seqlens_k [B] int32.
+
+    ``workspace`` is a CUDA uint8 tensor of at least ``loom_attn_decode_workspace_bytes``
+    bytes (allocated here if None).  Returns ``o`` or ``(o, lse)``.
+    """
+    torch = _torch()
+    (qp, kp, vp_, sp, op, lp), (B, Hq, Hkv, Skv, D), o, lse = _decode_operands(
+        q, k_cache, v_cache, seqlens_k, o, lse, return_lse)
     if workspace is None:
         need = loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, num_splits)
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=q.device)
@@ -250,6 +261,21 @@ def loom_attn_decode(q, k_cache, v_cache, seqlens_k=None, o=None, lse=None, work
                                  B, Hq, Hkv, Skv, D, float(scale), int(num_splits),
                                  _stream_ptr(stream, q.device))
     _check(st, "loom_attn_decode")
+    return (o, lse) if (return_lse or lse is not None) else o
+
+
+def loom_attn_decode_noalloc(q, k_cache, v_cache, seqlens_k=None, o=None, lse=None, *, scale=None,
+                             num_splits=0, stream=None, return_lse=False):
+    """Flash Decode with the partials in the library's built-in scratch array (no
+    workspace argument, no device allocation by the library).  Arguments and results as
+    ``loom_attn_decode``; problems whose partials exceed the array raise LOOM_ERR_WORKSPACE."""
+    (qp, kp, vp_, sp, op, lp), (B, Hq, Hkv, Skv, D), o, lse = _decode_operands(
+        q, k_cache, v_cache, seqlens_k, o, lse, return_lse)
+    if scale is None:
+        scale = D ** -0.5
+    st = capi().loom_attn_decode_noalloc(qp, kp, vp_, sp, op, lp, B, Hq, Hkv, Skv, D, float(scale),
+                                         int(num_splits), _stream_ptr(stream, q.device))
+    _check(st, "loom_attn_decode_noalloc")
     return (o, lse) if (return_lse or lse is not None) else o
 
 

@@ -540,15 +540,14 @@ template <int D, int GT, bool PAGED>
 cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
   using C = DecodeCfg<D>;
   constexpr uint32_t smem = DecodeSmem<D, GT>::BYTES;
-  static unsigned long long configured = 0;  // one bit per device
+  static PerDeviceOnce configured;
   int dev = 0;
   cudaGetDevice(&dev);
-  if (!(configured & (1ull << (dev & 63)))) {
-    cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D, GT, PAGED>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    configured |= 1ull << (dev & 63);
-  }
+  if (!configured.run(dev, [&] {
+        return cudaFuncSetAttribute(decode_split_kernel<D, GT, PAGED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    smem) == cudaSuccess;
+      }))
+    return cudaErrorInvalidValue;
   CUtensorMap tk, tv;
   PagedView view{nullptr, 0, 0, 0, 0};
   if constexpr (PAGED) {

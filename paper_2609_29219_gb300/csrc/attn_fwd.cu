@@ -4,7 +4,7 @@
 // Paper: Sec. 3.2.2 evaluates Flash Attention as fused "matrix multiplication, softmax,
 // and value aggregation"; the pipelining of its load, compute and store stages through
 // counted circular buffers is the virtual-buffer protocol of Sec. 2.3, and the tile and
-// stage constants come from the latency model of Sec. 2.6 (Eq. 6-9, see model.cpp).
+// stage constants come from the latency model of Sec. 2.6 (Eq. 6-9, in model.h).
 //
 // One CTA owns NQT = 2 query tiles of BM = 128 rows (tile 0 and tile 1) of one
 // (batch, query head) and walks the key/value sequence in tiles of BN = 128 rows:
@@ -1289,7 +1289,7 @@ bool make_map_tokens(CUtensorMap* map, const void* base, int D, int H, int total
 template <int D>
 cudaError_t launch_varlen_d(const FwdVarlenArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
   using C = FwdCfg<D>;
-  static unsigned long long configured = 0;  // one bit per device
+  static PerDeviceOnce configured;
   CUtensorMap mq, mk, mv, mo;
   if (!make_map_tokens(&mq, a.q, D, a.Hq, a.total_q, C::BM) ||
       !make_map_tokens(&mk, a.k, D, a.Hkv, a.total_k, C::BN) ||
@@ -1298,12 +1298,11 @@ cudaError_t launch_varlen_d(const FwdVarlenArgs& a, const KernelCtl& ctl, cudaSt
     return cudaErrorInvalidValue;
   int dev = 0;
   cudaGetDevice(&dev);
-  if (!(configured & (1ull << (dev & 63)))) {
-    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         C::BYTES);
-    if (e != cudaSuccess) return e;
-    configured |= 1ull << (dev & 63);
-  }
+  if (!configured.run(dev, [] {
+        return cudaFuncSetAttribute(attn_fwd_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    C::BYTES) == cudaSuccess;
+      }))
+    return cudaErrorInvalidValue;
   FwdParams p;
   memset(&p, 0, sizeof(p));
   p.o = static_cast<__nv_bfloat16*>(a.o);
@@ -1333,7 +1332,7 @@ cudaError_t launch_varlen_d(const FwdVarlenArgs& a, const KernelCtl& ctl, cudaSt
 // item (C::NQT * C::BM).
 template <int D, class C, class Kernel>
 cudaError_t launch_design(Kernel kernel, int rows_per_item, const FwdArgs& a, const KernelCtl& ctl,
-                          cudaStream_t stream, unsigned long long& configured) {
+                          cudaStream_t stream, PerDeviceOnce& configured) {
   CUtensorMap mq, mk, mv, mo;
   if (!make_map(&mq, a.q, D, a.Sq, a.B * a.Hq, C::BM) ||
       !make_map(&mk, a.k, D, a.Skv, a.B * a.Hkv, C::BN) ||
@@ -1342,11 +1341,10 @@ cudaError_t launch_design(Kernel kernel, int rows_per_item, const FwdArgs& a, co
     return cudaErrorInvalidValue;
   int dev = 0;
   cudaGetDevice(&dev);
-  if (!(configured & (1ull << (dev & 63)))) {
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::BYTES);
-    if (e != cudaSuccess) return e;
-    configured |= 1ull << (dev & 63);
-  }
+  if (!configured.run(dev, [&] {
+        return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::BYTES) == cudaSuccess;
+      }))
+    return cudaErrorInvalidValue;
   FwdParams p;
   p.o = static_cast<__nv_bfloat16*>(a.o);
   p.lse = a.lse;
@@ -1374,8 +1372,7 @@ cudaError_t launch_design(Kernel kernel, int rows_per_item, const FwdArgs& a, co
 
 template <int D>
 cudaError_t launch_fwd_d(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
-  static unsigned long long configured2 = 0, configured1 = 0;  // one bit per device
-  static unsigned long long configured3 = 0;
+  static PerDeviceOnce configured1, configured2, configured3;
   constexpr int kModelDesign = model::fwd_plan(D).design;
   const int design = a.design ? a.design : kModelDesign;
   if (design == 1)

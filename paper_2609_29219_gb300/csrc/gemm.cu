@@ -21,10 +21,12 @@
 #include <cuda.h>
 #include <cuda_bf16.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "gemm.h"
 #include "gemm_model.h"
+#include "kernels.h"
 #include "ptx.cuh"
 
 namespace loom {
@@ -773,14 +775,15 @@ bool matrix_map(CUtensorMap* map, const void* base, int rows, int cols, int box_
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Devices whose cluster occupancy answers are cached (others query on every call).
+constexpr int kSlotCacheDevices = 64;
+
 template <int BN>
-bool set_smem_attr(const void* fn, int& done_mask, int bit) {
-  // one opt-in per kernel and device (the mask is per template instance)
-  if (done_mask & (1 << bit)) return true;
-  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmCfg<BN>::BYTES) != cudaSuccess)
-    return false;
-  done_mask |= 1 << bit;
-  return true;
+bool set_smem_attr(const void* fn, PerDeviceOnce& done, int dev) {
+  // one opt-in per kernel and device (the flags are per template instance)
+  return done.run(dev, [fn] {
+    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmCfg<BN>::BYTES) == cudaSuccess;
+  });
 }
 
 // B's box: 64 columns x 64 K-rows of B [K, N], or 64 K-columns x b_rows rows of B [N, K].
@@ -806,8 +809,8 @@ GemmParams make_params(const GemmArgs& a, const KernelCtl& ctl, int bn, int spli
 template <int BN, bool BKM>
 cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int dev, int sms) {
   using C = GemmCfg<BN>;
-  static int configured = 0;  // bit per device (devices 0..30)
-  if (dev < 31 && !set_smem_attr<BN>(reinterpret_cast<const void*>(gemm_kernel<BN, BKM>), configured, dev))
+  static PerDeviceOnce configured;
+  if (!set_smem_attr<BN>(reinterpret_cast<const void*>(gemm_kernel<BN, BKM>), configured, dev))
     return cudaErrorInvalidValue;
   CUtensorMap ma, mb, mc;
   if (!make_maps(a, C::BM, BN, &ma, &mb, &mc)) return cudaErrorInvalidValue;
@@ -837,27 +840,27 @@ cudaLaunchConfig_t splitk_config(int grid, int S, cudaStream_t stream, cudaLaunc
 
 template <int BN, bool BKM>
 bool prepare_splitk(int dev) {
-  static int configured = 0;
-  static int nonportable = 0;
+  static PerDeviceOnce configured, nonportable;
   const void* fn = reinterpret_cast<const void*>(gemm_splitk_kernel<BN, BKM>);
-  if (dev >= 31) return false;
   if (!set_smem_attr<BN>(fn, configured, dev)) return false;
-  if (!(nonportable & (1 << dev))) {
-    if (cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) return false;
-    nonportable |= 1 << dev;
-  }
-  return true;
+  return nonportable.run(dev, [fn] {
+    return cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
+  });
 }
 
 // CTAs of clusters of S that fit on the device at once (0: none, or cannot be queried); both
 // B layouts have the same resources, so the [K, N] instance answers for both.
 template <int BN>
 int splitk_slots(int dev, int S) {
-  static int cache[31][5];  // [device][log2 S], value + 1 once known
+  static std::atomic<int> cache[kSlotCacheDevices][5];  // [device][log2 S], value + 1 once known
   int lg = 0;
   while ((1 << lg) < S) ++lg;
-  if (dev >= 31 || lg > 4 || (1 << lg) != S) return 0;
-  if (cache[dev][lg] != 0) return cache[dev][lg] - 1;
+  if (dev < 0 || lg > 4 || (1 << lg) != S) return 0;
+  const bool cached = dev < kSlotCacheDevices;
+  if (cached) {
+    const int c = cache[dev][lg].load(std::memory_order_relaxed);
+    if (c != 0) return c - 1;
+  }
   int clusters = 0;
   if (prepare_splitk<BN, false>(dev)) {
     cudaLaunchAttribute attr[1];
@@ -867,7 +870,7 @@ int splitk_slots(int dev, int S) {
       clusters = 0;
     }
   }
-  cache[dev][lg] = clusters * S + 1;
+  if (cached) cache[dev][lg].store(clusters * S + 1, std::memory_order_relaxed);
   return clusters * S;
 }
 
@@ -895,14 +898,11 @@ cudaError_t launch_splitk(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t 
 
 template <bool BKM>
 bool prepare_pair(int dev) {
-  static int configured = 0;
-  if (dev >= 31) return false;
+  static PerDeviceOnce configured;
   const void* fn = reinterpret_cast<const void*>(gemm_pair_kernel<BKM>);
-  if (configured & (1 << dev)) return true;
-  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmPairCfg::BYTES) != cudaSuccess)
-    return false;
-  configured |= 1 << dev;
-  return true;
+  return configured.run(dev, [fn] {
+    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmPairCfg::BYTES) == cudaSuccess;
+  });
 }
 
 cudaLaunchConfig_t pair_config(int grid, cudaStream_t stream, cudaLaunchAttribute* attr) {
@@ -922,9 +922,13 @@ cudaLaunchConfig_t pair_config(int grid, cudaStream_t stream, cudaLaunchAttribut
 
 // CTAs of CTA pairs that fit on the device at once (0: none, or cannot be queried).
 int pair_slots(int dev) {
-  static int cache[31];  // value + 1 once known
-  if (dev >= 31) return 0;
-  if (cache[dev] != 0) return cache[dev] - 1;
+  static std::atomic<int> cache[kSlotCacheDevices];  // value + 1 once known
+  if (dev < 0) return 0;
+  const bool cached = dev < kSlotCacheDevices;
+  if (cached) {
+    const int c = cache[dev].load(std::memory_order_relaxed);
+    if (c != 0) return c - 1;
+  }
   int clusters = 0;
   if (prepare_pair<false>(dev)) {
     cudaLaunchAttribute attr[1];
@@ -934,7 +938,7 @@ int pair_slots(int dev) {
       clusters = 0;
     }
   }
-  cache[dev] = 2 * clusters + 1;
+  if (cached) cache[dev].store(2 * clusters + 1, std::memory_order_relaxed);
   return 2 * clusters;
 }
 

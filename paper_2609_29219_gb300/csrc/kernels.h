@@ -1,6 +1,7 @@
 // Internal launch interface between the C ABI (loom_api.cu) and the kernel files.
 #pragma once
 
+#include <atomic>
 #include <cstddef>
 #include <cstdint>
 #include <cuda_runtime.h>
@@ -8,6 +9,26 @@
 #include "ptx.cuh"
 
 namespace loom {
+
+// One-time set-up per device (a kernel's shared-memory opt-in, a cluster-size opt-in),
+// safe when several host threads launch at once: the first call on a device runs `fn`,
+// later calls skip it once it has succeeded.  Devices beyond the 64 tracked bits run `fn`
+// on every call (the set-up calls it guards are idempotent).
+class PerDeviceOnce {
+ public:
+  template <class F>
+  bool run(int dev, F&& fn) {
+    if (dev < 0 || dev >= 64) return fn();
+    const unsigned long long bit = 1ull << dev;
+    if (bits_.load(std::memory_order_acquire) & bit) return true;
+    if (!fn()) return false;
+    bits_.fetch_or(bit, std::memory_order_acq_rel);
+    return true;
+  }
+
+ private:
+  std::atomic<unsigned long long> bits_{0};
+};
 
 // Split rule of the decode path: chunk length of a sequence of `len` keys cut into
 // `splits` pieces, ceil(len / splits) rounded up to a multiple of kDecodeChunkAlign.
@@ -45,6 +66,12 @@ inline size_t decode_workspace_bytes(int B, int Hq, int D, int splits) {
   const size_t lpart = rows * sizeof(float);
   return ((opart + 255) / 256) * 256 + ((lpart + 255) / 256) * 256;
 }
+
+// Argument checks of the contiguous decode entry points, in their order, up to (not
+// including) the workspace; returns a loom_status value and, on success, the split count.
+int decode_check_args(const void* q, const void* k_cache, const void* v_cache, const int32_t* seqlens_k,
+                      const void* o, const float* lse, int B, int Hq, int Hkv, int Skv, int D, float scale,
+                      int num_splits, int* splits);
 
 cudaError_t launch_decode(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream);
 cudaError_t launch_fwd(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream);

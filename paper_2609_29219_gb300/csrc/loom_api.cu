@@ -139,10 +139,14 @@ size_t loom_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int Skv, int D, 
   return decode_workspace_bytes(B, Hq, D, num_splits);
 }
 
-loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_cache,
-                             const int32_t* seqlens_k, void* o, float* lse, void* workspace,
-                             size_t workspace_bytes, int B, int Hq, int Hkv, int Skv, int D,
-                             float scale, int num_splits, void* stream) {
+}  // extern "C"
+
+namespace loom {
+// Every check of the contiguous decode entry points that comes before the workspace: on
+// LOOM_OK, *splits is the split count the call will use (the model's when num_splits = 0).
+int decode_check_args(const void* q, const void* k_cache, const void* v_cache, const int32_t* seqlens_k,
+                      const void* o, const float* lse, int B, int Hq, int Hkv, int Skv, int D, float scale,
+                      int num_splits, int* splits) {
   if (!q || !k_cache || !v_cache || !o) return LOOM_ERR_INVALID_ARG;
   if (B <= 0 || Hq <= 0 || Hkv <= 0 || Skv <= 0 || D <= 0) return LOOM_ERR_INVALID_ARG;
   if (Hq % Hkv != 0) return LOOM_ERR_INVALID_ARG;
@@ -160,6 +164,20 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
     return LOOM_ERR_MISALIGNED;
   if (num_splits == 0) num_splits = loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D);
   if (num_splits <= 0) return LOOM_ERR_INVALID_ARG;
+  *splits = num_splits;
+  return LOOM_OK;
+}
+}  // namespace loom
+
+extern "C" {
+
+loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_cache,
+                             const int32_t* seqlens_k, void* o, float* lse, void* workspace,
+                             size_t workspace_bytes, int B, int Hq, int Hkv, int Skv, int D,
+                             float scale, int num_splits, void* stream) {
+  const int st = decode_check_args(q, k_cache, v_cache, seqlens_k, o, lse, B, Hq, Hkv, Skv, D, scale, num_splits,
+                                   &num_splits);
+  if (st != LOOM_OK) return static_cast<loom_status>(st);
   const size_t need = decode_workspace_bytes(B, Hq, D, num_splits);
   if (!workspace || workspace_bytes < need) return LOOM_ERR_WORKSPACE;
   if (!aligned16(workspace)) return LOOM_ERR_MISALIGNED;

@@ -15,7 +15,12 @@
 // any stream capture.  All calls share the array and it keeps the last call's contents;
 // nothing in it needs to start at zero (the split kernel writes every partial, empty
 // splits included, before the merge kernel reads them).  Calls whose kernels overlap on
-// the GPU (concurrent streams, or two host threads) race on the array.
+// the GPU (concurrent streams, or two host threads) race on the array.  The cached
+// address belongs to the device's context: after cudaDeviceReset on a device this entry
+// point must not be called there again in the same process.
+//
+// Arguments are checked exactly as loom_attn_decode checks them, in the same order; only
+// then is the problem's need compared with the array's size (LOOM_ERR_WORKSPACE).
 #include <mutex>
 
 #include "../../include/loom_attn.h"
@@ -53,15 +58,13 @@ extern "C" loom_status loom_attn_decode_noalloc(const void* q, const void* k_cac
                                                 void* o, float* lse, int B, int Hq, int Hkv,
                                                 int Skv, int D, float scale, int num_splits,
                                                 void* stream) {
-  if (num_splits < 0) return LOOM_ERR_INVALID_ARG;
-  const size_t need = loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, num_splits);
-  if (need == 0) {  // sizes the workspace query rejects: let the full validation report why
-    return loom_attn_decode(q, k_cache, v_cache, seqlens_k, o, lse, nullptr, 0, B, Hq, Hkv, Skv, D,
-                            scale, num_splits, stream);
-  }
-  if (need > loom::kNoallocScratchBytes) return LOOM_ERR_WORKSPACE;
+  int splits = 0;
+  const int st = loom::decode_check_args(q, k_cache, v_cache, seqlens_k, o, lse, B, Hq, Hkv, Skv, D, scale,
+                                         num_splits, &splits);
+  if (st != LOOM_OK) return static_cast<loom_status>(st);
+  if (loom::decode_workspace_bytes(B, Hq, D, splits) > loom::kNoallocScratchBytes) return LOOM_ERR_WORKSPACE;
   void* scratch = loom::scratch_ptr();
   if (!scratch) return LOOM_ERR_CUDA;
   return loom_attn_decode(q, k_cache, v_cache, seqlens_k, o, lse, scratch, loom::kNoallocScratchBytes,
-                          B, Hq, Hkv, Skv, D, scale, num_splits, stream);
+                          B, Hq, Hkv, Skv, D, scale, splits, stream);
 }

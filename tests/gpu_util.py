@@ -1,4 +1,4 @@
-"""Helpers shared by the GPU parity tests: device upload, tolerance checks, sampling."""
+"""Helpers shared by the GPU parity tests: device upload and tolerance checks."""
 import numpy as np
 
 # Parity bar (fp64 oracle vs the CUDA path on identical bf16 inputs)
@@ -31,16 +31,3 @@ def assert_parity(o_gpu, o_ref, lse_gpu=None, lse_ref=None, what=""):
     assert err.max() <= TOL_MAX_ABS, msg
     assert err.mean() <= TOL_MEAN_ABS, msg
     return msg
-
-
-def sample_rows(B, H, S, n, seed=0, tile=128):
-    """Flat row indices (b*H + h)*S + i: every tile edge of a few heads plus random rows."""
-    rng = np.random.default_rng(seed)
-    rows = set()
-    for _ in range(4):
-        b, h = int(rng.integers(B)), int(rng.integers(H))
-        for i in {0, 1, S - 1, S - 2, tile - 1, tile, min(S - 1, 2 * tile - 1), min(S - 1, 2 * tile)}:
-            if 0 <= i < S:
-                rows.add((b * H + h) * S + i)
-    rows.update(int(x) for x in rng.integers(0, B * H * S, size=n))
-    return np.array(sorted(rows), dtype=np.int64)

@@ -188,3 +188,23 @@ def test_varlen_prefill_rejects_bad_arguments(lib):
     assert call(q=FAKE + 8) == 3
     assert call(ck=FAKE + 2) == 3
     assert call(tq=0) == 0          # nothing to do
+
+
+def test_noalloc_decode_checks_arguments_before_its_scratch_size(lib):
+    # a problem far beyond the built-in scratch array: argument errors are still reported
+    # first, in loom_attn_decode's order; only valid arguments get LOOM_ERR_WORKSPACE
+    ok = dict(q=FAKE, k=FAKE, v=FAKE, sl=None, o=FAKE, lse=None, B=64, Hq=64, Hkv=8, Skv=65536, D=128,
+              scale=0.08, splits=1024, stream=None)
+    names = list(ok)
+
+    def call(**kw):
+        a = dict(ok)
+        a.update(kw)
+        return lib.loom_attn_decode_noalloc(*[a[n] for n in names])
+
+    assert call(q=None) == 1
+    assert call(Hq=7) == 1
+    assert call(D=80) == 2
+    assert call(o=FAKE + 8) == 3
+    assert call(sl=FAKE + 2) == 3
+    assert call() == 4

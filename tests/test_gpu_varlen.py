@@ -90,29 +90,16 @@ def test_equal_lengths_match_dense_kernel_bitwise(loom, S, causal):
     assert torch.equal(lse, ld.contiguous())
 
 
-def test_large_ragged_batch_sampled(loom):
-    """12 sequences of U[512, 4096] tokens, Hq = 32, Hkv = 8, D = 128, causal: every row of
-    four sequences' tile edges and random rows, checked against the oracle one by one."""
-    import torch
+def test_large_ragged_batch_full(loom):
+    """12 sequences of U[512, 4096] tokens, Hq = 32, Hkv = 8, D = 128, causal: every row
+    of O and LSE against the oracle."""
     rng = np.random.default_rng(3)
     lens = rng.integers(512, 4097, 12)
     Hq, Hkv, D = 32, 8, 128
     q, k, v, cq, ck = case(11, lens, lens, Hq, Hkv, D)
     o, lse = run(loom, q, k, v, cq, ck, True)
-    for b in (0, 3, 7, 11):
-        S = int(lens[b])
-        qb = np.ascontiguousarray(q[cq[b]:cq[b + 1]].transpose(1, 0, 2))[None]
-        kb = np.ascontiguousarray(k[ck[b]:ck[b + 1]].transpose(1, 0, 2))[None]
-        vb = np.ascontiguousarray(v[ck[b]:ck[b + 1]].transpose(1, 0, 2))[None]
-        hs = rng.integers(0, Hq, 3)
-        rows = sorted({int(h) * S + i for h in hs for i in
-                       {0, 1, 127, 128, 255, 256, S - 1, S - 2, *rng.integers(0, S, 6).tolist()} if 0 <= i < S})
-        o_ref, lse_ref = oracle.attention(qb, kb, vb, causal=True, rows=np.array(rows))
-        idx_h = np.array(rows) // S
-        idx_i = np.array(rows) % S
-        o_got = o[cq[b] + idx_i, idx_h]
-        lse_got = lse[idx_h, cq[b] + idx_i]
-        assert_parity(o_got, o_ref, lse_got, lse_ref, f"seq {b} (S={S})")
+    o_ref, lse_ref = oracle.attention_varlen(q, k, v, cq, ck, causal=True)
+    assert_parity(o, o_ref, lse, lse_ref, f"12 sequences, {int(cq[-1])} tokens")
 
 
 def test_timeout_is_reported_and_context_survives(loom):
