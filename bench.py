@@ -733,20 +733,31 @@ def run_decode_sweep(torch, loom, dev, stream, args, peaks):
         (Decode("long_decode", 1, 32, 8, 131072, 128, splits=0), [8, 16, 19, 24, 32, 38, 48, 57, 64, 76, 96, 114, 152]),
         (Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens), [1, 2, 3, 4, 6, 8, 12, 16, 19, 24, 32]),
     ]
+    G = 32 // 8
     for wl, splits in cases:
         wl.setup(torch, dev, loom)
         chosen = loom.loom_attn_decode_num_splits(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D)
+        chosen_form = loom.loom_attn_decode_cluster_form(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, 0)
         for sp in sorted(set(splits + [chosen])):
             wl.splits = sp
             nbytes = loom.loom_attn_decode_workspace_bytes(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sp)
             wl.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
-            r = measure(torch, wl, max(10, args.steps // 4), args.warmup, stream, lambda: None, 1, float, peaks)
-            loom.loom_attn_check_error(stream)
-            model_us = loom.loom_model_decode_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sms)
-            print(json.dumps({"sweep": "decode", "workload": wl.describe(), "splits": sp,
-                              "model_choice": sp == chosen, "measured_us": round(r["ms_per_step"] * 1e3, 2),
-                              "model_us": round(model_us, 2), "GB/s": r["value"],
-                              "frac": r["roofline"]["frac"]}), flush=True)
+            slots = loom.loom_decode_cluster_slots(wl.D, G, sp)
+            for form in ((-1, 1) if sp <= 16 and slots >= sp else (-1,)):
+                loom.loom_debug_decode_cluster(form)
+                r = measure(torch, wl, max(10, args.steps // 4), args.warmup, stream, lambda: None, 1, float, peaks)
+                loom.loom_attn_check_error(stream)
+                if form == 1:
+                    model_us = loom.loom_model_decode_fused_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, slots)
+                else:
+                    model_us = loom.loom_model_decode_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sms)
+                print(json.dumps({"sweep": "decode", "workload": wl.describe(), "splits": sp,
+                                  "form": "cluster" if form == 1 else "split+merge", "cluster_slots": slots,
+                                  "model_choice": sp == chosen and (form == 1) == (chosen_form == 1),
+                                  "measured_us": round(r["ms_per_step"] * 1e3, 2),
+                                  "model_us": round(model_us, 2), "GB/s": r["value"],
+                                  "frac": r["roofline"]["frac"]}), flush=True)
+            loom.loom_debug_decode_cluster(0)
         wl.inp = None
         torch.cuda.empty_cache()
 

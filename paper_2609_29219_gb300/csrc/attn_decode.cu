@@ -21,9 +21,18 @@
 //   w_i = exp(lse_i - L), O = sum w_i O_i / sum w_i -> bf16, lse = L + ln sum w_i.
 //   It is launched with programmatic dependent launch so its launch overlaps the
 //   split kernel's tail.
+// Single-kernel form (FUSED instantiation of kernel 1, at most 16 splits): the splits of
+// one (batch, kv head, head group) are one thread-block cluster.  Each CTA keeps its
+// partial (O_i, lse_i) in its own shared memory; after a cluster barrier CTA r gathers
+// outputs [r n / splits, (r + 1) n / splits) of the unit's n = heads x D outputs from
+// all the cluster's CTAs over distributed shared memory (in the order i = 0 .. splits-1,
+// so the result does not depend on timing), applies the global softmax and the final
+// scaling, and writes O (bf16) and LSE; a second cluster barrier keeps every partial
+// alive until all peers have read it.  No workspace, no second launch.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -63,7 +72,7 @@ struct DecodeCfg {
   static_assert(TW % TPR == 0, "whole 128-bit load rounds per warp");
 };
 
-template <int D, int GT>
+template <int D, int GT, bool FUSED = false>
 struct DecodeSmem {
   using C = DecodeCfg<D>;
   // ring first (16-byte aligned bulk-copy destinations), then the small arrays
@@ -71,7 +80,10 @@ struct DecodeSmem {
   static constexpr uint32_t ALPHA_OFF = P_OFF + C::NCW * C::TW * GT * 4;  // [NCW][GT] f32
   static constexpr uint32_t WM_OFF = ALPHA_OFF + C::NCW * GT * 4;       // [NCW][GT] f32
   static constexpr uint32_t WL_OFF = WM_OFF + C::NCW * GT * 4;          // [NCW][GT] f32
-  static constexpr uint32_t BAR_OFF = ((WL_OFF + C::NCW * GT * 4) + 7) / 8 * 8;
+  // single-kernel form: the CTA's partial, read by the cluster's CTAs over DSMEM
+  static constexpr uint32_t PART_O_OFF = (WL_OFF + C::NCW * GT * 4 + 15) / 16 * 16;  // [GT][D] f32
+  static constexpr uint32_t PART_L_OFF = PART_O_OFF + (FUSED ? GT * D * 4 : 0);      // [GT] f32
+  static constexpr uint32_t BAR_OFF = ((PART_L_OFF + (FUSED ? GT * 4 : 0)) + 7) / 8 * 8;
   static constexpr uint32_t ABORT_OFF = BAR_OFF + 2 * C::NSTAGE * 8;
   static constexpr uint32_t BYTES = ABORT_OFF + 16;
   // the cross-warp merge reuses the ring: [NCW][GT][D] f32
@@ -122,20 +134,62 @@ struct PagedView {
   int hnd;  // 1: [num_pages, Hkv, page_size, D]; 0: [num_pages, page_size, Hkv, D]
 };
 
-template <int D, int GT, bool PAGED>
+// Gather, global softmax and final scaling of one unit's partials across its cluster (the
+// single-kernel form), run by every thread of every CTA of the cluster: the partials
+// (part_o [GT][D], part_l [GT] at these shared-memory offsets) of all `splits` CTAs are
+// complete after the first barrier; CTA r combines its share of the nh x D outputs, reading
+// each split i = 0 .. splits-1 in order; the second barrier keeps the partials alive until
+// every peer has read them.  o_row0 = row of O (and index of LSE) of the unit's first head.
+template <int D>
+__device__ __forceinline__ void cluster_gather(uint32_t part_o, uint32_t part_l, int nh, int splits,
+                                               __nv_bfloat16* __restrict__ o, float* __restrict__ lse,
+                                               size_t o_row0) {
+  cluster_sync_all();
+  const int total = nh * D;
+  const int per = (total + splits - 1) / splits;
+  const int e0 = static_cast<int>(cluster_ctarank()) * per;
+  const int e1 = min(total, e0 + per);
+  for (int e = e0 + static_cast<int>(threadIdx.x); e < e1; e += static_cast<int>(blockDim.x)) {
+    const int h = e / D, d = e % D;
+    float l[model::kMaxFusedSplits];
+    float M = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < model::kMaxFusedSplits; ++i) {
+      l[i] = i < splits ? ld_dsmem_f32(map_shared_rank(part_l + 4u * h, i)) : -INFINITY;
+      M = fmaxf(M, l[i]);
+    }
+    float W = 0.f, acc = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int i = 0; i < model::kMaxFusedSplits; ++i) {
+        if (i < splits) {
+          const float w = ex2((l[i] - M) * kLog2e);  // 0 for empty splits
+          W += w;
+          acc = fmaf(w, ld_dsmem_f32(map_shared_rank(part_o + 4u * e, i)), acc);
+        }
+      }
+    }
+    const bool any = W > 0.f;
+    o[(o_row0 + h) * D + d] = __float2bfloat16_rn(any ? acc / W : 0.f);
+    if (lse && d == 0) lse[o_row0 + h] = any ? M + log2f(W) * kLn2 : -INFINITY;
+  }
+  cluster_sync_all();
+}
+
+template <int D, int GT, bool PAGED, bool FUSED>
 __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_SM)
     decode_split_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
                         const __nv_bfloat16* __restrict__ v, const int32_t* __restrict__ seqlens,
                         float* __restrict__ o_part, float* __restrict__ lse_part, int Hq, int Hkv,
                         int Skv, int splits, int n_groups, float c, KernelCtl ctl,
                         const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
-                        PagedView pv) {
+                        PagedView pv, __nv_bfloat16* __restrict__ o_out, float* __restrict__ lse_out) {
   using C = DecodeCfg<D>;
-  using L = DecodeSmem<D, GT>;
+  using L = DecodeSmem<D, GT, FUSED>;
   extern __shared__ __align__(128) uint8_t smem[];
 
   // Let the merge grid launch as soon as every split CTA is resident.
-  asm volatile("griddepcontrol.launch_dependents;");
+  if constexpr (!FUSED) asm volatile("griddepcontrol.launch_dependents;");
 
   const int split = blockIdx.x;
   const int hk = blockIdx.y / n_groups, grp = blockIdx.y % n_groups;
@@ -152,11 +206,20 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
   const int t_begin = min(split * chunk, len);
   const int t_end = min(t_begin + chunk, len);
   const size_t row0 = (static_cast<size_t>(b) * Hq + h0) * splits + split;  // head h0's partial
+  const uint32_t part_o = smem_u32(smem) + L::PART_O_OFF, part_l = smem_u32(smem) + L::PART_L_OFF;
+  const size_t o_row0 = static_cast<size_t>(b) * Hq + h0;  // single-kernel form: first output row
 
   if (t_begin >= t_end) {  // empty split: contributes nothing to the merge
-    for (int i = threadIdx.x; i < nh * D; i += blockDim.x)
-      o_part[(row0 + static_cast<size_t>(i / D) * splits) * D + i % D] = 0.f;
-    if (threadIdx.x < nh) lse_part[row0 + static_cast<size_t>(threadIdx.x) * splits] = -INFINITY;
+    if constexpr (FUSED) {
+      float* po = reinterpret_cast<float*>(smem + L::PART_O_OFF);
+      for (int i = threadIdx.x; i < nh * D; i += blockDim.x) po[i] = 0.f;
+      if (threadIdx.x < nh) reinterpret_cast<float*>(smem + L::PART_L_OFF)[threadIdx.x] = -INFINITY;
+      cluster_gather<D>(part_o, part_l, nh, splits, o_out, lse_out, o_row0);
+    } else {
+      for (int i = threadIdx.x; i < nh * D; i += blockDim.x)
+        o_part[(row0 + static_cast<size_t>(i / D) * splits) * D + i % D] = 0.f;
+      if (threadIdx.x < nh) lse_part[row0 + static_cast<size_t>(threadIdx.x) * splits] = -INFINITY;
+    }
     return;
   }
   const int n_stages = (t_end - t_begin + C::T - 1) / C::T;
@@ -261,6 +324,10 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
         if (it == skipped) continue;
         mbar_wait(bar_full + 8 * (it % C::NSTAGE), (it / C::NSTAGE) & 1, ctl, no_abort);
       }
+    }
+    if constexpr (FUSED) {  // the loader warp takes its share of the cluster gather
+      __syncwarp();
+      cluster_gather<D>(part_o, part_l, nh, splits, o_out, lse_out, o_row0);
     }
     return;
   }
@@ -435,11 +502,17 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
         osum = fmaf(a, wo[(w * GT + h) * D + d], osum);
       }
     }
-    const size_t row = row0 + static_cast<size_t>(h) * splits;
     const bool any = lsum > 0.f;
-    o_part[row * D + d] = any ? osum / lsum : 0.f;
-    if (d == 0) lse_part[row] = any ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+    if constexpr (FUSED) {
+      reinterpret_cast<float*>(smem + L::PART_O_OFF)[idx] = any ? osum / lsum : 0.f;
+      if (d == 0) reinterpret_cast<float*>(smem + L::PART_L_OFF)[h] = any ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+    } else {
+      const size_t row = row0 + static_cast<size_t>(h) * splits;
+      o_part[row * D + d] = any ? osum / lsum : 0.f;
+      if (d == 0) lse_part[row] = any ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+    }
   }
+  if constexpr (FUSED) cluster_gather<D>(part_o, part_l, nh, splits, o_out, lse_out, o_row0);
 }
 
 // One CTA (D threads) per (batch, query head).  The split log-sum-exps are read in
@@ -536,18 +609,70 @@ bool paged_map(CUtensorMap* map, const void* cache, const PagedKV& pk, int Hkv, 
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int D, int GT, bool PAGED>
-cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
-  using C = DecodeCfg<D>;
-  constexpr uint32_t smem = DecodeSmem<D, GT>::BYTES;
+// Per-device set-up of one kernel instance: the shared-memory opt-in and, for the cluster
+// form, clusters of up to 16 CTAs (beyond the portable 8).
+template <int D, int GT, bool PAGED, bool FUSED>
+bool prepare_split() {
   static PerDeviceOnce configured;
   int dev = 0;
-  cudaGetDevice(&dev);
-  if (!configured.run(dev, [&] {
-        return cudaFuncSetAttribute(decode_split_kernel<D, GT, PAGED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    smem) == cudaSuccess;
-      }))
-    return cudaErrorInvalidValue;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  return configured.run(dev, [] {
+    const void* fn = reinterpret_cast<const void*>(decode_split_kernel<D, GT, PAGED, FUSED>);
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, DecodeSmem<D, GT, FUSED>::BYTES) !=
+        cudaSuccess)
+      return false;
+    if constexpr (FUSED) return cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
+    return true;
+  });
+}
+
+template <int D, int GT, bool FUSED>
+cudaLaunchConfig_t split_config(dim3 grid, int cluster, cudaStream_t stream, cudaLaunchAttribute* attr) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(DecodeCfg<D>::THREADS);
+  cfg.dynamicSmemBytes = DecodeSmem<D, GT, FUSED>::BYTES;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 0;
+  if (FUSED) {
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = static_cast<unsigned>(cluster);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.numAttrs = 1;
+  }
+  return cfg;
+}
+
+// CTA slots of the cluster form with clusters of `splits` CTAs on the current device: whole
+// clusters that fit at once (cudaOccupancyMaxActiveClusters) x splits; 0 if none fit or the
+// device cannot be asked.  Cached per device and cluster size.
+template <int D, int GT, bool PAGED>
+int cluster_slots(int splits) {
+  static std::atomic<int> cache[64][model::kMaxFusedSplits + 1];  // value + 1 once known
+  int dev = 0;
+  if (splits < 1 || splits > model::kMaxFusedSplits || cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 0;
+  if (dev < 64) {
+    const int c = cache[dev][splits].load(std::memory_order_relaxed);
+    if (c != 0) return c - 1;
+  }
+  int clusters = 0;
+  if (prepare_split<D, GT, PAGED, true>()) {
+    cudaLaunchAttribute attr[1];
+    const cudaLaunchConfig_t cfg = split_config<D, GT, true>(dim3(splits, 64, 1), splits, nullptr, attr);
+    if (cudaOccupancyMaxActiveClusters(&clusters, decode_split_kernel<D, GT, PAGED, true>, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      clusters = 0;
+    }
+  }
+  if (dev < 64) cache[dev][splits].store(clusters * splits + 1, std::memory_order_relaxed);
+  return clusters * splits;
+}
+
+template <int D, int GT, bool PAGED, bool FUSED>
+cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
+  if (!prepare_split<D, GT, PAGED, FUSED>()) return cudaErrorInvalidValue;
   CUtensorMap tk, tv;
   PagedView view{nullptr, 0, 0, 0, 0};
   if constexpr (PAGED) {
@@ -562,12 +687,13 @@ cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl
   }
   const int G = a.Hq / a.Hkv;
   const int n_groups = (G + GT - 1) / GT;
-  dim3 grid(a.splits, a.Hkv * n_groups, a.B);
-  decode_split_kernel<D, GT, PAGED><<<grid, C::THREADS, smem, stream>>>(
-      static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.k),
-      static_cast<const __nv_bfloat16*>(a.v), a.seqlens, a.o_part, a.lse_part, a.Hq, a.Hkv, a.Skv,
-      a.splits, n_groups, a.scale * kLog2e, ctl, tk, tv, view);
-  return cudaGetLastError();
+  cudaLaunchAttribute attr[1];
+  const cudaLaunchConfig_t cfg =
+      split_config<D, GT, FUSED>(dim3(a.splits, a.Hkv * n_groups, a.B), a.splits, stream, attr);
+  return cudaLaunchKernelEx(&cfg, decode_split_kernel<D, GT, PAGED, FUSED>, static_cast<const __nv_bfloat16*>(a.q),
+                            static_cast<const __nv_bfloat16*>(a.k), static_cast<const __nv_bfloat16*>(a.v),
+                            a.seqlens, a.o_part, a.lse_part, a.Hq, a.Hkv, a.Skv, a.splits, n_groups,
+                            a.scale * kLog2e, ctl, tk, tv, view, static_cast<__nv_bfloat16*>(a.o), a.lse);
 }
 
 template <int D>
@@ -587,16 +713,53 @@ cudaError_t launch_merge(const DecodeArgs& a, cudaStream_t stream) {
                             static_cast<__nv_bfloat16*>(a.o), a.lse, a.splits);
 }
 
+// Which form runs: the cluster form when it is forced (a.fused = 1) or the model prefers
+// it (a.fused = 0), provided the split count is a cluster size and such clusters fit.
+template <int D, int GT, bool PAGED>
+bool use_cluster_form(const DecodeArgs& a) {
+  if (a.fused < 0 || a.splits > model::kMaxFusedSplits) return false;
+  const int slots = cluster_slots<D, GT, PAGED>(a.splits);
+  if (slots < a.splits) return false;
+  if (a.fused == 1) return true;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
+                                                cudaSuccess)
+    return false;
+  return model::decode_fused_wins(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms, slots);
+}
+
+template <int D, int GT, bool PAGED>
+cudaError_t launch_form(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
+  if (use_cluster_form<D, GT, PAGED>(a)) return launch_split<D, GT, PAGED, true>(a, pk, ctl, stream);
+  const cudaError_t e = launch_split<D, GT, PAGED, false>(a, pk, ctl, stream);
+  if (e != cudaSuccess) return e;
+  return launch_merge<D>(a, stream);
+}
+
 template <int D, bool PAGED>
 cudaError_t launch_decode_d(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
   const int G = a.Hq / a.Hkv;
-  cudaError_t e;
-  if (G >= 8) e = launch_split<D, 8, PAGED>(a, pk, ctl, stream);
-  else if (G >= 4) e = launch_split<D, 4, PAGED>(a, pk, ctl, stream);
-  else if (G >= 2) e = launch_split<D, 2, PAGED>(a, pk, ctl, stream);
-  else e = launch_split<D, 1, PAGED>(a, pk, ctl, stream);
-  if (e != cudaSuccess) return e;
-  return launch_merge<D>(a, stream);
+  if (G >= 8) return launch_form<D, 8, PAGED>(a, pk, ctl, stream);
+  if (G >= 4) return launch_form<D, 4, PAGED>(a, pk, ctl, stream);
+  if (G >= 2) return launch_form<D, 2, PAGED>(a, pk, ctl, stream);
+  return launch_form<D, 1, PAGED>(a, pk, ctl, stream);
+}
+
+template <int D, bool PAGED>
+bool cluster_form_d(const DecodeArgs& a) {
+  const int G = a.Hq / a.Hkv;
+  if (G >= 8) return use_cluster_form<D, 8, PAGED>(a);
+  if (G >= 4) return use_cluster_form<D, 4, PAGED>(a);
+  if (G >= 2) return use_cluster_form<D, 2, PAGED>(a);
+  return use_cluster_form<D, 1, PAGED>(a);
+}
+
+template <int D>
+int cluster_slots_d(int G, int splits) {
+  if (G >= 8) return cluster_slots<D, 8, false>(splits);
+  if (G >= 4) return cluster_slots<D, 4, false>(splits);
+  if (G >= 2) return cluster_slots<D, 2, false>(splits);
+  return cluster_slots<D, 1, false>(splits);
 }
 
 }  // namespace
@@ -612,6 +775,15 @@ cudaError_t launch_decode_paged(const DecodeArgs& a, const PagedKV& pk, const Ke
     return cudaErrorInvalidValue;
   if (a.D == 128) return launch_decode_d<128, true>(a, &pk, ctl, stream);
   return launch_decode_d<64, true>(a, &pk, ctl, stream);
+}
+
+bool decode_cluster_form(const DecodeArgs& a, bool paged) {
+  if (a.D == 128) return paged ? cluster_form_d<128, true>(a) : cluster_form_d<128, false>(a);
+  return paged ? cluster_form_d<64, true>(a) : cluster_form_d<64, false>(a);
+}
+
+int decode_cluster_slots(int D, int G, int splits) {
+  return D == 128 ? cluster_slots_d<128>(G, splits) : cluster_slots_d<64>(G, splits);
 }
 
 }  // namespace loom

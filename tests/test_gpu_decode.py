@@ -1,4 +1,6 @@
-"""GPU parity of the Flash Decode kernels (split + merge, through the C ABI)."""
+"""GPU parity of the Flash Decode kernels through the C ABI, in both forms: split kernel +
+merge kernel, and the single kernel whose splits of a (batch, kv head) form a cluster and
+merge over distributed shared memory (at most 16 splits)."""
 import numpy as np
 import pytest
 
@@ -20,6 +22,24 @@ def loom():
     return m
 
 
+@pytest.fixture(autouse=True, params=[0, 1, -1], ids=["model_form", "cluster_form", "split_merge"])
+def form(request, loom):
+    """Every test runs with the model's choice of form, with the cluster form forced
+    wherever it can run (at most 16 splits), and with split + merge kernels forced."""
+    loom.loom_debug_decode_cluster(request.param)
+    yield request.param
+    loom.loom_debug_decode_cluster(0)
+
+
+def _expect_form(loom, form, B, Hq, Hkv, Skv, D, splits):
+    used = loom.loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, splits)
+    if form == -1:
+        assert used == 0
+    elif form == 1:
+        s = splits or loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
+        assert used == (1 if s <= 16 else 0)
+
+
 def _inputs(seed, B, Hq, Hkv, Skv, D):
     return (synth.bf16_normal(seed, synth.STREAM_Q, (B, Hq, 1, D)),
             synth.bf16_normal(seed, synth.STREAM_K, (B, Hkv, Skv, D)),
@@ -35,9 +55,10 @@ def _run(loom, q, k, v, lens, num_splits, workspace=None):
     return o, lse
 
 
-def test_batched_decode_config(loom):
+def test_batched_decode_config(loom, form):
     # B=16, Hq=32, Hkv=8, Skv=8192, lengths U[4096, 8192] (stream 3), D=128, 16 splits
     B, Hq, Hkv, Skv, D = 16, 32, 8, 8192, 128
+    _expect_form(loom, form, B, Hq, Hkv, Skv, D, 16)
     q, k, v = _inputs(0, B, Hq, Hkv, Skv, D)
     lens = synth.decode_lengths(0, B, 4096, 8192)
     o, lse = _run(loom, q, k, v, lens, 16)
@@ -58,30 +79,35 @@ def test_long_context_decode_config(loom):
 
 
 @pytest.mark.parametrize("D", [64, 128])
-def test_edge_lengths(loom, D):
-    # empty sequence, single key, chunk-1, chunk+1, full
+def test_edge_lengths(loom, form, D):
+    # empty sequence, single key, chunk-1, chunk+1, full; splits that leave whole empty
+    # CTAs in a cluster (16 splits of 300 keys: chunks of 64, splits 5..15 empty)
     B, Hq, Hkv, Skv = 6, 4, 2, 300
     q, k, v = _inputs(3, B, Hq, Hkv, Skv, D)
     lens = np.array([0, 1, 63, 65, 129, 300], np.int32)
-    for splits in (1, 3, 16, 64):
+    for splits in (1, 2, 3, 7, 16, 64):
+        _expect_form(loom, form, B, Hq, Hkv, Skv, D, splits)
         o, lse = _run(loom, q, k, v, lens, splits)
         o_ref, lse_ref = oracle.attention(q, k, v, seqlens_k=lens)
         assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"D={D} splits={splits}")
 
 
 @pytest.mark.parametrize("Hq,Hkv", [(1, 1), (3, 1), (8, 8), (16, 2), (32, 1), (12, 4)])
-def test_group_sizes(loom, Hq, Hkv):
+def test_group_sizes(loom, form, Hq, Hkv):
     B, Skv, D = 2, 777, 128
     q, k, v = _inputs(Hq + Hkv, B, Hq, Hkv, Skv, D)
-    for splits in (1, 5):
+    for splits in (1, 5, 13):
+        _expect_form(loom, form, B, Hq, Hkv, Skv, D, splits)
         o, lse = _run(loom, q, k, v, None, splits)
         o_ref, lse_ref = oracle.attention(q, k, v)
         assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"Hq={Hq} Hkv={Hkv} splits={splits}")
 
 
-def test_partials_match_oracle_split_form(loom):
-    """The workspace holds the per-split partial (O_i, lse_i) of the Flash Decode form."""
+def test_partials_match_oracle_split_form(loom, form):
+    """The workspace holds the per-split partial (O_i, lse_i) of the Flash Decode form
+    (split + merge kernels; the cluster form keeps its partials in shared memory)."""
     import torch
+    loom.loom_debug_decode_cluster(-1)
     B, Hq, Hkv, Skv, D, S = 2, 8, 2, 1000, 128, 5
     q, k, v = _inputs(9, B, Hq, Hkv, Skv, D)
     lens = np.array([1000, 333], np.int32)
@@ -107,3 +133,16 @@ def test_workspace_and_argument_errors(loom):
     with pytest.raises(loom.LoomError) as e:
         loom.loom_attn_decode(to_dev(q), to_dev(k), to_dev(v), None, num_splits=2000)
     assert e.value.status == 2
+
+
+def test_cluster_form_is_deterministic(loom, form):
+    """The cluster form reads the splits in a fixed order: repeated calls agree bit for bit."""
+    import torch
+    B, Hq, Hkv, Skv, D = 3, 16, 4, 5000, 128
+    q, k, v = (to_dev(x) for x in _inputs(13, B, Hq, Hkv, Skv, D))
+    sl = torch.tensor([5000, 4097, 100], dtype=torch.int32, device="cuda")
+    outs = [loom.loom_attn_decode(q, k, v, sl, num_splits=11, return_lse=True) for _ in range(3)]
+    loom.loom_attn_check_error()
+    for o, lse in outs[1:]:
+        assert torch.equal(o.view(torch.int16), outs[0][0].view(torch.int16))
+        assert torch.equal(lse, outs[0][1])

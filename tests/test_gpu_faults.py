@@ -7,6 +7,7 @@ TMEM) and sets the device error word.  These tests check that loom_attn_check_er
 reports LOOM_ERR_TIMEOUT and that the context stays usable: the very next normal call
 matches the oracle and reports no error.
 """
+import numpy as np
 import pytest
 
 import oracle
@@ -61,6 +62,36 @@ def test_decode_skipped_stage_times_out_and_context_survives(loom):
     loom.loom_attn_check_error()
     o_ref, lse_ref = oracle.attention(q, k, v)
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "decode after timeout")
+
+
+@pytest.mark.parametrize("lens,splits", [(2048, 2), (160, 2), (2048, 16)], ids=["both_abort", "one_aborts", "c16"])
+def test_cluster_decode_skipped_stage_times_out_and_context_survives(loom, lens, splits):
+    """The single-kernel cluster form: every CTA whose chunk has a second stage gives up on
+    it and unwinds; all CTAs (those that gave up and those that finished) still meet at the
+    cluster barriers, so the launch ends and the next call is correct."""
+    import torch
+    B, Hq, Hkv, Skv, D = 1, 4, 1, 2048, 128
+    q = synth.bf16_normal(37, synth.STREAM_Q, (B, Hq, 1, D))
+    k = synth.bf16_normal(37, synth.STREAM_K, (B, Hkv, Skv, D))
+    v = synth.bf16_normal(37, synth.STREAM_V, (B, Hkv, Skv, D))
+    qd, kd, vd = to_dev(q), to_dev(k), to_dev(v)
+    sl_h = np.array([lens], np.int32)
+    sl = torch.from_numpy(sl_h).cuda()
+    loom.loom_debug_decode_cluster(1)
+    try:
+        assert loom.loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, splits) == 1
+
+        def bad():
+            loom.loom_debug_inject(1)
+            loom.loom_attn_decode(qd, kd, vd, sl, num_splits=splits)
+
+        _expect_timeout(loom, bad)
+        o, lse = loom.loom_attn_decode(qd, kd, vd, sl, num_splits=splits, return_lse=True)
+        loom.loom_attn_check_error()
+    finally:
+        loom.loom_debug_decode_cluster(0)
+    o_ref, lse_ref = oracle.attention(q, k, v, seqlens_k=sl_h)
+    assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "cluster decode after timeout")
 
 
 @pytest.mark.parametrize("design,D", [(2, 128), (1, 128), (1, 64), (3, 64)])

@@ -26,6 +26,15 @@ def loom():
     m.loom_debug_set_timeout_ns(0)
 
 
+@pytest.fixture(autouse=True, params=[1, -1], ids=["cluster_form", "split_merge"])
+def form(request, loom):
+    """Every test runs with the single-kernel cluster form forced wherever it can run (at
+    most 16 splits) and with split + merge kernels forced."""
+    loom.loom_debug_decode_cluster(request.param)
+    yield request.param
+    loom.loom_debug_decode_cluster(0)
+
+
 def paged_case(seed, B, Hq, Hkv, P, lens, D, spare=5, poison=True, shuffle=True):
     """Pages dealt to the sequences in a (shuffled) order; rows past each sequence's end
     and the spare pages hold NaN, table entries past a sequence's last page hold -1."""
@@ -130,13 +139,15 @@ def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P, layout):
 
 @LAYOUTS
 @pytest.mark.parametrize("P", [16, 64])
-def test_batched_serving_shape(loom, P, layout):
+def test_batched_serving_shape(loom, form, P, layout):
     """The batched decode shape (B=16, Hq=32, Hkv=8, D=128, lengths U[4096, 8192]) paged,
     pages shuffled, model-chosen splits."""
     B, Hq, Hkv, D = 16, 32, 8, 128
     lens = synth.decode_lengths(0, B, 4096, 8192)
     q, kc, vc, table, sl = paged_case(0, B, Hq, Hkv, P, lens, D, spare=0, poison=False)
     o, lse = run_paged(loom, q, kc, vc, table, sl, 16, layout)
+    assert loom.loom_attn_decode_cluster_form(B, Hq, Hkv, table.shape[1] * P, D, 16, paged=True) == \
+        (1 if form == 1 else 0)
     o_ref, lse_ref = oracle.decode_paged(q, kc, vc, table, sl, page_size=P)
     assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"batched paged P={P} {layout}")
 

@@ -102,14 +102,41 @@ DECODE_SHAPES = [(16, 32, 8, 8192, 128), (1, 32, 8, 131072, 128), (1, 8, 8, 4096
                  (4, 16, 2, 30000, 128), (2, 4, 4, 64, 128)]
 
 
+def _decode_candidates(loom, B, Hq, Hkv, Skv, D):
+    """Modeled time of every (form, split count) candidate: the two-kernel form for every
+    split count, the cluster form for split counts up to 16 with the slots it is priced at."""
+    cands = []
+    for s in range(1, min(1024, math.ceil(Skv / 64)) + 1):
+        cands.append((loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS), 0, s))
+    for s in range(1, min(16, math.ceil(Skv / 64)) + 1):
+        t = loom.loom_model_decode_fused_time_us(s, B, Hq, Hkv, Skv, D, loom.loom_decode_cluster_slots(D, Hq // Hkv, s))
+        if t > 0:
+            cands.append((t, 1, s))
+    return cands
+
+
 @pytest.mark.parametrize("B,Hq,Hkv,Skv,D", DECODE_SHAPES)
 def test_decode_split_is_brute_force_argmin(loom, B, Hq, Hkv, Skv, D):
+    # Eq. 9 over both Flash Decode forms: the chosen (form, splits) is the fastest candidate
     chosen = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
-    cands = range(1, min(1024, math.ceil(Skv / 64)) + 1)
-    times = [loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS) for s in cands]
-    best = min(times)
-    assert times[chosen - 1] == pytest.approx(best)
-    assert chosen == 1 + times.index(best)        # ties: the fewest splits
+    cands = _decode_candidates(loom, B, Hq, Hkv, Skv, D)
+    best = min(t for t, _, _ in cands)
+    winners = sorted((f, s) for t, f, s in cands if t <= best * (1 + 1e-9))
+    assert winners[0][1] == chosen                # ties: the two-kernel form, then the fewest splits
+    form = loom.loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, 0)
+    assert form == winners[0][0]
+
+
+def test_cluster_form_limits(loom):
+    B, Hq, Hkv, Skv, D = 16, 32, 8, 8192, 128
+    slots = loom.loom_decode_cluster_slots(D, 4, 16)
+    assert slots > 0 and slots % 16 == 0
+    assert loom.loom_model_decode_fused_time_us(17, B, Hq, Hkv, Skv, D, 10 ** 6) < 0   # > 16 CTAs per cluster
+    assert loom.loom_model_decode_fused_time_us(16, B, Hq, Hkv, Skv, D, 15) < 0       # no whole cluster fits
+    # fewer slots never make it faster; the HBM roof bounds it
+    t = [loom.loom_model_decode_fused_time_us(16, B, Hq, Hkv, Skv, D, n) for n in (64, 128, 256, 304)]
+    assert all(a >= b * (1 - 1e-9) for a, b in zip(t, t[1:]))
+    assert t[-1] * 1e-6 >= 2.0 * B * Hkv * Skv * D * 2 / (PEAK_GBS * 1e9) * 0.999
 
 
 def test_long_decode_fills_one_wave(loom):
@@ -121,7 +148,9 @@ def test_long_decode_fills_one_wave(loom):
 @pytest.mark.parametrize("B,Hq,Hkv,Skv,D", DECODE_SHAPES)
 def test_decode_time_not_below_hbm_roofline(loom, B, Hq, Hkv, Skv, D):
     s = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
-    t = loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS)
+    t = min(loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS),
+            loom.loom_model_decode_fused_time_us(s, B, Hq, Hkv, Skv, D, loom.loom_decode_cluster_slots(D, Hq // Hkv, s))
+            if s <= 16 else 1e30)
     kv_bytes = 2.0 * B * Hkv * Skv * D * 2
     assert t * 1e-6 >= kv_bytes / (PEAK_GBS * 1e9) * 0.999
 
