@@ -742,18 +742,21 @@ def run_decode_sweep(torch, loom, dev, stream, args, peaks):
             wl.splits = sp
             nbytes = loom.loom_attn_decode_workspace_bytes(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sp)
             wl.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
-            slots = loom.loom_decode_cluster_slots(wl.D, G, sp)
-            for form in ((-1, 1) if sp <= 16 and slots >= sp else (-1,)):
-                loom.loom_debug_decode_cluster(form)
+            # split + merge, then the cluster form with every power-of-two cluster size dividing sp
+            for cs in [0] + [c for c in (1, 2, 4, 8, 16) if sp % c == 0]:
+                n_fit = loom.loom_decode_max_clusters(wl.D, G, cs) if cs else 0
+                if cs and n_fit < 1:
+                    continue
+                loom.loom_debug_decode_cluster(1 if cs else -1, cs)
                 r = measure(torch, wl, max(10, args.steps // 4), args.warmup, stream, lambda: None, 1, float, peaks)
                 loom.loom_attn_check_error(stream)
-                if form == 1:
-                    model_us = loom.loom_model_decode_fused_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, slots)
+                if cs:
+                    model_us = loom.loom_model_decode_cluster_time_us(sp, cs, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, n_fit)
                 else:
                     model_us = loom.loom_model_decode_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sms)
                 print(json.dumps({"sweep": "decode", "workload": wl.describe(), "splits": sp,
-                                  "form": "cluster" if form == 1 else "split+merge", "cluster_slots": slots,
-                                  "model_choice": sp == chosen and (form == 1) == (chosen_form == 1),
+                                  "form": f"cluster{cs}" if cs else "split+merge", "resident_clusters": n_fit,
+                                  "model_choice": sp == chosen and cs == chosen_form,
                                   "measured_us": round(r["ms_per_step"] * 1e3, 2),
                                   "model_us": round(model_us, 2), "GB/s": r["value"],
                                   "frac": r["roofline"]["frac"]}), flush=True)

@@ -121,10 +121,11 @@ size_t loom_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int Skv, int D, 
  * length 0 yields O = 0 and LSE = -inf.
  * Two forms compute it, chosen by the analytic model (see loom_attn_decode_cluster_form):
  * a split kernel writing the partials (O_i, lse_i) into the workspace followed by a merge
- * kernel (the gather, global softmax and final scaling of the Flash Decode HEG), or, for
- * at most 16 splits, one kernel whose splits of a (batch, kv head) form a thread-block
- * cluster and merge their partials over distributed shared memory; that form leaves the
- * workspace untouched, but the call checks and requires it all the same.
+ * kernel (the gather, global softmax and final scaling of the Flash Decode HEG), or one
+ * persistent kernel in which clusters of cs CTAs (cs divides num_splits, cs <= 16) walk
+ * the (batch, kv head) pairs, CTA r taking splits r, r + cs, ... of each, and merge their
+ * partials over distributed shared memory; that form leaves the workspace untouched, but
+ * the call checks and requires it all the same.
  * Errors: INVALID_ARG, UNSUPPORTED, MISALIGNED, WORKSPACE, CUDA.
  */
 loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_cache,
@@ -219,23 +220,26 @@ double loom_model_fwd_time_us(int B, int Hq, int Sq, int Skv, int D, int causal)
 /* Modeled prefill launch time (us) with design 1, 2 or 3 forced; < 0 if infeasible. */
 double loom_model_fwd_time_us_design(int design, int B, int Hq, int Sq, int Skv, int D, int causal);
 double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms);
-/* Modeled time (us) of the single-kernel (cluster) Flash Decode with `splits` splits
- * (1..16) when `slots` CTAs of its clusters fit on the GPU at once; < 0 on bad sizes. */
-double loom_model_decode_fused_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int slots);
+/* Modeled time (us) of the single-kernel (cluster) Flash Decode with `splits` splits and
+ * clusters of `cluster` CTAs (dividing splits, at most 16) when `clusters` such clusters
+ * fit on the GPU at once; < 0 on bad sizes. */
+double loom_model_decode_cluster_time_us(int splits, int cluster, int B, int Hq, int Hkv, int Skv, int D,
+                                         int clusters);
 
 /*
- * Which Flash Decode form a call with these sizes runs on the current device: 1 = the
- * single-kernel cluster form (Sec. 2.6's gather, global softmax and final scaling done
- * inside one kernel, over distributed shared memory), 0 = split kernel + merge kernel,
- * -1 = invalid sizes.  num_splits = 0 means the model's split count; paged = 1 asks about
- * loom_attn_decode_paged (Skv = max_pages * page_size).  Follows loom_debug_decode_cluster.
- * loom_decode_cluster_slots: CTAs of clusters of `splits` decode CTAs (G query heads per
- * kv head, head dimension D) that fit on the current device at once, 0 if none; with no
- * device, the model's GB300 estimate (whole clusters in 8 equal groups of SMs).  These are
- * the slots the split-count choice (num_splits = 0) prices the cluster form with.
+ * Which Flash Decode form a call with these sizes runs on the current device: cs > 0 = the
+ * single-kernel cluster form with clusters of cs CTAs (Sec. 2.6's gather, global softmax
+ * and final scaling done inside one kernel, over distributed shared memory), 0 = split
+ * kernel + merge kernel, -1 = invalid sizes.  num_splits = 0 means the model's split
+ * count; paged = 1 asks about loom_attn_decode_paged (Skv = max_pages * page_size).
+ * Follows loom_debug_decode_cluster.
+ * loom_decode_max_clusters: clusters of `cluster` decode CTAs (G query heads per kv head,
+ * head dimension D) resident on the current device at once, 0 if none; with no device, the
+ * model's GB300 estimate (whole clusters in 8 equal groups of SMs).  These are what the
+ * split-count choice (num_splits = 0) prices the cluster form with.
  */
 int loom_attn_decode_cluster_form(int B, int Hq, int Hkv, int Skv, int D, int num_splits, int paged);
-int loom_decode_cluster_slots(int D, int G, int splits);
+int loom_decode_max_clusters(int D, int G, int cluster);
 
 /*
  * BF16 GEMM, the third kernel the paper evaluates (GEMM shapes, Sec. 4): C = A B with
@@ -310,11 +314,12 @@ void loom_debug_inject(int mode);
 void loom_debug_prefill_design(int design);
 
 /*
- * Test hook: the Flash Decode form.  1 = the single-kernel cluster form wherever it can
- * run (at most 16 splits and such clusters fit on the GPU); -1 = always split + merge
- * kernels; anything else: the analytic model's choice (default).
+ * Test hook: the Flash Decode form.  mode 1 = the single-kernel cluster form wherever some
+ * cluster size runs; -1 = always split + merge kernels; anything else: the analytic model's
+ * choice (default).  cluster in 1..16 pins the cluster form's cluster size (honoured when
+ * it divides the split count and such clusters fit); 0: the model's size.
  */
-void loom_debug_decode_cluster(int mode);
+void loom_debug_decode_cluster(int mode, int cluster);
 
 #ifdef __cplusplus
 }

@@ -27,8 +27,8 @@ __all__ = [
     "loom_model_fwd_time_us", "loom_model_decode_time_us", "FwdPlan", "loom_debug_prefill_design",
     "loom_model_fwd_plan_variant", "loom_model_heg_pipe", "loom_model_fwd_time_us_design",
     "loom_attn_decode_paged", "loom_attn_fwd_varlen", "loom_gemm_bf16", "loom_gemm_bf16_bt", "loom_gemm_tile_n", "loom_gemm_splits", "loom_gemm_cta_pair", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
-    "loom_debug_gemm_splits", "loom_debug_gemm_cta_pair", "loom_model_decode_fused_time_us",
-    "loom_attn_decode_cluster_form", "loom_decode_cluster_slots", "loom_debug_decode_cluster",
+    "loom_debug_gemm_splits", "loom_debug_gemm_cta_pair", "loom_model_decode_cluster_time_us",
+    "loom_attn_decode_cluster_form", "loom_decode_max_clusters", "loom_debug_decode_cluster",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -131,13 +131,13 @@ def capi() -> ctypes.CDLL:
             lib.loom_debug_gemm_cta_pair.restype = None
             lib.loom_model_decode_time_us.argtypes = [i32, i32, i32, i32, i32, i32, i32]
             lib.loom_model_decode_time_us.restype = ctypes.c_double
-            lib.loom_model_decode_fused_time_us.argtypes = [i32] * 7
-            lib.loom_model_decode_fused_time_us.restype = ctypes.c_double
+            lib.loom_model_decode_cluster_time_us.argtypes = [i32] * 8
+            lib.loom_model_decode_cluster_time_us.restype = ctypes.c_double
             lib.loom_attn_decode_cluster_form.argtypes = [i32] * 7
             lib.loom_attn_decode_cluster_form.restype = i32
-            lib.loom_decode_cluster_slots.argtypes = [i32, i32, i32]
-            lib.loom_decode_cluster_slots.restype = i32
-            lib.loom_debug_decode_cluster.argtypes = [i32]
+            lib.loom_decode_max_clusters.argtypes = [i32, i32, i32]
+            lib.loom_decode_max_clusters.restype = i32
+            lib.loom_debug_decode_cluster.argtypes = [i32, i32]
             lib.loom_debug_decode_cluster.restype = None
             _lib = lib
     return _lib
@@ -486,19 +486,19 @@ def loom_model_decode_time_us(splits, B, Hq, Hkv, Skv, D, num_sms) -> float:
     return float(capi().loom_model_decode_time_us(splits, B, Hq, Hkv, Skv, D, num_sms))
 
 
-def loom_model_decode_fused_time_us(splits, B, Hq, Hkv, Skv, D, slots) -> float:
-    return float(capi().loom_model_decode_fused_time_us(splits, B, Hq, Hkv, Skv, D, slots))
+def loom_model_decode_cluster_time_us(splits, cluster, B, Hq, Hkv, Skv, D, clusters) -> float:
+    return float(capi().loom_model_decode_cluster_time_us(splits, cluster, B, Hq, Hkv, Skv, D, clusters))
 
 
 def loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, num_splits=0, paged=False) -> int:
-    """1 if a decode call with these sizes runs the single-kernel cluster form, 0 if the
-    split + merge kernels, -1 on invalid sizes."""
+    """The cluster size if a decode call with these sizes runs the single-kernel cluster
+    form, 0 if the split + merge kernels, -1 on invalid sizes."""
     return int(capi().loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, num_splits, int(bool(paged))))
 
 
-def loom_decode_cluster_slots(D, G, splits) -> int:
-    return int(capi().loom_decode_cluster_slots(D, G, splits))
+def loom_decode_max_clusters(D, G, cluster) -> int:
+    return int(capi().loom_decode_max_clusters(D, G, cluster))
 
 
-def loom_debug_decode_cluster(mode: int) -> None:
-    capi().loom_debug_decode_cluster(int(mode))
+def loom_debug_decode_cluster(mode: int, cluster: int = 0) -> None:
+    capi().loom_debug_decode_cluster(int(mode), int(cluster))

@@ -1,9 +1,10 @@
-// Flash Decode for GB300: split-KV partial attention + log-sum-exp merge.
+// Flash Decode for GB300: split-KV partial attention + log-sum-exp merge, in two forms.
 //
 // Paper: Sec. 2.6 (the Flash Decode HEG is a sequential composition of a local
 // softmax loop, a gather of partial results, a global softmax and a final scaling) and
 // Sec. 3.2.3 (the sequence axis, the reduction axis, is split across cores).
 //
+// Split + merge form.
 // Kernel 1, decode_split_kernel -- one CTA per (split, kv head, head group, batch):
 //   * a loader warp streams the split's K and V rows with 1-D bulk copies
 //     (cp.async.bulk, 16 KB per tile) into an NSTAGE-deep shared-memory ring guarded by
@@ -21,14 +22,22 @@
 //   w_i = exp(lse_i - L), O = sum w_i O_i / sum w_i -> bf16, lse = L + ln sum w_i.
 //   It is launched with programmatic dependent launch so its launch overlaps the
 //   split kernel's tail.
-// Single-kernel form (FUSED instantiation of kernel 1, at most 16 splits): the splits of
-// one (batch, kv head, head group) are one thread-block cluster.  Each CTA keeps its
-// partial (O_i, lse_i) in its own shared memory; after a cluster barrier CTA r gathers
-// outputs [r n / splits, (r + 1) n / splits) of the unit's n = heads x D outputs from
-// all the cluster's CTAs over distributed shared memory (in the order i = 0 .. splits-1,
-// so the result does not depend on timing), applies the global softmax and the final
-// scaling, and writes O (bf16) and LSE; a second cluster barrier keeps every partial
-// alive until all peers have read it.  No workspace, no second launch.
+//
+// Single-kernel (cluster) form, decode_cluster_kernel -- persistent clusters of CS CTAs
+// (CS divides the split count, CS <= 16).  A unit is one (batch, kv head, head group);
+// each cluster walks its units (dealt in a snake order over the units sorted by
+// sequence length), and for every unit CTA r of the cluster streams the unit's splits
+// r, r + CS, ... with the same loader ring and compute warps as kernel 1, without a
+// break between units: the loader fetches the next unit's q and first K/V stages while
+// the compute warps finish the current one.  At a unit's end the compute warps merge
+// their states in the ring slot of the unit's last stage into the CTA's partial
+// (O_r, lse_r), kept in shared memory; once every CTA of the cluster has signalled its
+// partial (a remote mbarrier arrive), CTA r gathers outputs [r n / CS, (r + 1) n / CS)
+// of the unit's n = heads x D outputs from the CS partials over distributed shared
+// memory (in rank order, so the result does not depend on timing), applies the global
+// softmax and the final scaling, writes O (bf16) and LSE, and signals that it has read
+// the partials, so that their owners may overwrite them with the next unit's.  No
+// workspace and no second launch.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -72,7 +81,7 @@ struct DecodeCfg {
   static_assert(TW % TPR == 0, "whole 128-bit load rounds per warp");
 };
 
-template <int D, int GT, bool FUSED = false>
+template <int D, int GT>
 struct DecodeSmem {
   using C = DecodeCfg<D>;
   // ring first (16-byte aligned bulk-copy destinations), then the small arrays
@@ -80,10 +89,7 @@ struct DecodeSmem {
   static constexpr uint32_t ALPHA_OFF = P_OFF + C::NCW * C::TW * GT * 4;  // [NCW][GT] f32
   static constexpr uint32_t WM_OFF = ALPHA_OFF + C::NCW * GT * 4;       // [NCW][GT] f32
   static constexpr uint32_t WL_OFF = WM_OFF + C::NCW * GT * 4;          // [NCW][GT] f32
-  // single-kernel form: the CTA's partial, read by the cluster's CTAs over DSMEM
-  static constexpr uint32_t PART_O_OFF = (WL_OFF + C::NCW * GT * 4 + 15) / 16 * 16;  // [GT][D] f32
-  static constexpr uint32_t PART_L_OFF = PART_O_OFF + (FUSED ? GT * D * 4 : 0);      // [GT] f32
-  static constexpr uint32_t BAR_OFF = ((PART_L_OFF + (FUSED ? GT * 4 : 0)) + 7) / 8 * 8;
+  static constexpr uint32_t BAR_OFF = ((WL_OFF + C::NCW * GT * 4) + 7) / 8 * 8;
   static constexpr uint32_t ABORT_OFF = BAR_OFF + 2 * C::NSTAGE * 8;
   static constexpr uint32_t BYTES = ABORT_OFF + 16;
   // the cross-warp merge reuses the ring: [NCW][GT][D] f32
@@ -134,62 +140,245 @@ struct PagedView {
   int hnd;  // 1: [num_pages, Hkv, page_size, D]; 0: [num_pages, page_size, Hkv, D]
 };
 
-// Gather, global softmax and final scaling of one unit's partials across its cluster (the
-// single-kernel form), run by every thread of every CTA of the cluster: the partials
-// (part_o [GT][D], part_l [GT] at these shared-memory offsets) of all `splits` CTAs are
-// complete after the first barrier; CTA r combines its share of the nh x D outputs, reading
-// each split i = 0 .. splits-1 in order; the second barrier keeps the partials alive until
-// every peer has read them.  o_row0 = row of O (and index of LSE) of the unit's first head.
-template <int D>
-__device__ __forceinline__ void cluster_gather(uint32_t part_o, uint32_t part_l, int nh, int splits,
-                                               __nv_bfloat16* __restrict__ o, float* __restrict__ lse,
-                                               size_t o_row0) {
-  cluster_sync_all();
-  const int total = nh * D;
-  const int per = (total + splits - 1) / splits;
-  const int e0 = static_cast<int>(cluster_ctarank()) * per;
-  const int e1 = min(total, e0 + per);
-  for (int e = e0 + static_cast<int>(threadIdx.x); e < e1; e += static_cast<int>(blockDim.x)) {
-    const int h = e / D, d = e % D;
-    float l[model::kMaxFusedSplits];
-    float M = -INFINITY;
+// Compute-warp lane roles of one stage: lane = (token within a load round, 16-byte column
+// of the K row); one primary lane per (token, head) keeps the head's probability.
+template <int D, int GT>
+struct LaneRole {
+  using C = DecodeCfg<D>;
+  int kl, tg, hl;
+  bool primary;
+  __device__ __forceinline__ explicit LaneRole(int lane)
+      : kl(lane % C::KL), tg(lane / C::KL), hl(head_of_lane<C::KL, GT>(lane)),
+        primary(((lane % C::KL) & (C::KL / GT - 1)) == 0) {}
+};
+
+// q of the GT heads at q_rows (row h = head h0 + h; rows >= nh are zero), pre-multiplied by
+// scale * log2(e) so that scores come out in base 2.  q_rows may be global or shared.
+template <int D, int GT>
+__device__ __forceinline__ void load_q(const __nv_bfloat16* q_rows, int nh, int kl, float c, float (&qf)[GT][8]) {
 #pragma unroll
-    for (int i = 0; i < model::kMaxFusedSplits; ++i) {
-      l[i] = i < splits ? ld_dsmem_f32(map_shared_rank(part_l + 4u * h, i)) : -INFINITY;
-      M = fmaxf(M, l[i]);
-    }
-    float W = 0.f, acc = 0.f;
-    if (M != -INFINITY) {
+  for (int h = 0; h < GT; ++h) {
+    if (h < nh) {
+      const uint4 raw = *reinterpret_cast<const uint4*>(q_rows + static_cast<size_t>(h) * D + kl * 8);
+      const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
 #pragma unroll
-      for (int i = 0; i < model::kMaxFusedSplits; ++i) {
-        if (i < splits) {
-          const float w = ex2((l[i] - M) * kLog2e);  // 0 for empty splits
-          W += w;
-          acc = fmaf(w, ld_dsmem_f32(map_shared_rank(part_o + 4u * e, i)), acc);
-        }
+      for (int i = 0; i < 4; ++i) {
+        qf[h][2 * i] = bf16lo(w[i]) * c;
+        qf[h][2 * i + 1] = bf16hi(w[i]) * c;
       }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) qf[h][i] = 0.f;
     }
-    const bool any = W > 0.f;
-    o[(o_row0 + h) * D + d] = __float2bfloat16_rn(any ? acc / W : 0.f);
-    if (lse && d == 0) lse[o_row0 + h] = any ? M + log2f(W) * kLn2 : -INFINITY;
   }
-  cluster_sync_all();
 }
 
-template <int D, int GT, bool PAGED, bool FUSED>
+// One compute warp's work on one stage of the ring (K tile ks, V tile vs, ntok valid
+// keys): the scores of its TW tokens for the GT heads (base 2), the online softmax per
+// head with a lazily moved running max (m_run, l_run), and P.V into acc_o.  ps and alpha_s
+// are this warp's shared-memory P [TW][GT] and rescale factors [GT].
+template <int D, int GT>
+__device__ __forceinline__ void decode_stage(const uint8_t* ks, const uint8_t* vs, int ntok, int warp, int lane,
+                                             const LaneRole<D, GT>& lr, const float (&qf)[GT][8], float& m_run,
+                                             float& l_run, float (&acc_o)[GT][DecodeCfg<D>::VD], float* ps,
+                                             float* alpha_s) {
+  using C = DecodeCfg<D>;
+  // scores of this warp's TW tokens, in base-2 units
+  float sc[C::KROUNDS];
+#pragma unroll
+  for (int r = 0; r < C::KROUNDS; ++r) {
+    const int tl = warp * C::TW + r * C::TPR + lr.tg;
+    const uint4 raw = *reinterpret_cast<const uint4*>(ks + tl * (D * 2) + lr.kl * 16);
+    const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+    float kf[8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      kf[2 * i] = bf16lo(w[i]);
+      kf[2 * i + 1] = bf16hi(w[i]);
+    }
+    float acc[GT];
+#pragma unroll
+    for (int h = 0; h < GT; ++h) {
+      float s = 0.f;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) s = fmaf(qf[h][i], kf[i], s);
+      acc[h] = s;
+    }
+    const float s = transpose_reduce<C::KL, GT>(acc, lane);
+    sc[r] = (tl < ntok) ? s : -INFINITY;
+  }
+
+  // online softmax (per head, over this warp's tokens)
+  float mx = sc[0];
+#pragma unroll
+  for (int r = 1; r < C::KROUNDS; ++r) mx = fmaxf(mx, sc[r]);
+#pragma unroll
+  for (int off = C::KL; off < 32; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  const float m_new = fmaxf(m_run, mx);
+  const bool need = m_new > m_run + kRescaleThreshold;
+  const float alpha = need ? ex2(m_run - m_new) : 1.f;
+  if (need) m_run = m_new;
+  const float ms = (m_run == -INFINITY) ? 0.f : m_run;
+  float psum = 0.f;
+  __syncwarp();
+#pragma unroll
+  for (int r = 0; r < C::KROUNDS; ++r) {
+    const float p = ex2(sc[r] - ms);
+    psum += p;
+    if (lr.primary) ps[(r * C::TPR + lr.tg) * GT + lr.hl] = p;
+  }
+  l_run = l_run * alpha + psum;
+  if (lr.primary && lr.tg == 0) alpha_s[lr.hl] = alpha;
+  __syncwarp();
+
+  if (__any_sync(0xffffffffu, need)) {
+#pragma unroll
+    for (int h = 0; h < GT; ++h) {
+      const float a = alpha_s[h];
+#pragma unroll
+      for (int d = 0; d < C::VD; ++d) acc_o[h][d] *= a;
+    }
+  }
+
+  // P.V over this warp's tokens; lane owns dims [lane*VD, lane*VD + VD)
+  const int nmine = min(C::TW, ntok - warp * C::TW);
+#pragma unroll 4
+  for (int tt = 0; tt < nmine; ++tt) {
+    const int tl = warp * C::TW + tt;
+    float vf[C::VD];
+    if constexpr (C::VD == 4) {
+      const uint2 raw = *reinterpret_cast<const uint2*>(vs + tl * (D * 2) + lane * 8);
+      vf[0] = bf16lo(raw.x);
+      vf[1] = bf16hi(raw.x);
+      vf[2] = bf16lo(raw.y);
+      vf[3] = bf16hi(raw.y);
+    } else {
+      const uint32_t raw = *reinterpret_cast<const uint32_t*>(vs + tl * (D * 2) + lane * 4);
+      vf[0] = bf16lo(raw);
+      vf[1] = bf16hi(raw);
+    }
+    float pv[GT];
+    if constexpr (GT % 4 == 0) {
+#pragma unroll
+      for (int h = 0; h < GT; h += 4) {
+        const float4 p4 = *reinterpret_cast<const float4*>(ps + tt * GT + h);
+        pv[h] = p4.x;
+        pv[h + 1] = p4.y;
+        pv[h + 2] = p4.z;
+        pv[h + 3] = p4.w;
+      }
+    } else {
+#pragma unroll
+      for (int h = 0; h < GT; ++h) pv[h] = ps[tt * GT + h];
+    }
+#pragma unroll
+    for (int h = 0; h < GT; ++h)
+#pragma unroll
+      for (int d = 0; d < C::VD; ++d) acc_o[h][d] = fmaf(pv[h], vf[d], acc_o[h][d]);
+  }
+}
+
+// Merge of the NCW compute warps' states (run by all of them) into one partial per
+// (head, dim): wo is an [NCW][GT][D] fp32 scratch that no warp reads any more when this is
+// called, wm / wl [NCW][GT].  emit(idx = h * D + d, h, d, O value, LSE (natural log; valid
+// where d == 0)) receives each of the nh x D results.
+template <int D, int GT, class Emit>
+__device__ __forceinline__ void merge_warps(float* wo, float* wm, float* wl, int nh, int warp, int lane,
+                                            const LaneRole<D, GT>& lr, float m_run, float l_run,
+                                            const float (&acc_o)[GT][DecodeCfg<D>::VD], Emit emit) {
+  using C = DecodeCfg<D>;
+#pragma unroll
+  for (int off = C::KL; off < 32; off <<= 1) l_run += __shfl_xor_sync(0xffffffffu, l_run, off);
+  asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");  // the scratch is no longer read
+  if (lr.primary && lr.tg == 0) {
+    wm[warp * GT + lr.hl] = m_run;
+    wl[warp * GT + lr.hl] = l_run;
+  }
+#pragma unroll
+  for (int h = 0; h < GT; ++h)
+#pragma unroll
+    for (int d = 0; d < C::VD; ++d) wo[(warp * GT + h) * D + lane * C::VD + d] = acc_o[h][d];
+  asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");
+
+  for (int idx = threadIdx.x; idx < nh * D; idx += C::NCW * 32) {
+    const int h = idx / D, d = idx % D;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < C::NCW; ++w) M = fmaxf(M, wm[w * GT + h]);
+    float lsum = 0.f, osum = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < C::NCW; ++w) {
+        const float a = ex2(wm[w * GT + h] - M);  // 0 for warps that saw no key
+        lsum = fmaf(a, wl[w * GT + h], lsum);
+        osum = fmaf(a, wo[(w * GT + h) * D + d], osum);
+      }
+    }
+    const bool any = lsum > 0.f;
+    emit(idx, h, d, any ? osum / lsum : 0.f, any ? (M + log2f(lsum)) * kLn2 : -INFINITY);
+  }
+}
+
+// Loader of a paged cache for one kv head of one sequence: the block table is read 32
+// entries at a time (one per lane) and lane j issues the stage's j-th copy pair.  Copies
+// hold `rows` keys: a 64-key piece of one page (page_size a multiple of 64) or one whole
+// page (page_size 8, 16 or 32).  Stages start on a multiple of 64 keys, so no copy
+// crosses a page.  Run by the whole loader warp.
+struct PagedLoader {
+  int win = 0, entry = 0;
+  bool have = false;
+  __device__ __forceinline__ void reset() { have = false; }
+  template <int D>
+  __device__ __forceinline__ void stage(const PagedView& pv, const int32_t* tbl, int Hkv, int hk, int tok0, int ntok,
+                                        uint32_t dst, uint32_t bar, uint32_t tile_bytes, const CUtensorMap* tm_k,
+                                        const CUtensorMap* tm_v, int lane) {
+    const int P = pv.page_size;
+    const int rows = P < kDecodeChunkAlign ? P : kDecodeChunkAlign;
+    const uint32_t copy_bytes = static_cast<uint32_t>(rows) * D * 2;
+    const int ncopy = (ntok + rows - 1) / rows;
+    const int lp_first = tok0 / P, lp_last = (tok0 + (ncopy - 1) * rows) / P;
+    if (!have || lp_first < win || lp_last >= win + 32) {  // refill the table window
+      win = lp_first;
+      entry = (win + lane < pv.max_pages) ? tbl[win + lane] : 0;
+      have = true;
+    }
+    if (lane == 0) mbar_expect_tx(bar, 2u * ncopy * copy_bytes);
+    __syncwarp();
+    const int t = tok0 + lane * rows;
+    const int page = __shfl_sync(0xffffffffu, entry, (t / P - win) & 31);
+    if (lane < ncopy) {
+      // An out-of-range page (a caller error) is sent past the end of the cache, where
+      // the copy engine reads zeros.  NHD view [keys of all pages, Hkv, D]: (0, hk, key);
+      // HND view [pages x Hkv, page_size, D]: (0, row in page, page x Hkv + hk).
+      const bool bad = page < 0 || page >= pv.num_pages;
+      int y, z;
+      if (pv.hnd) {
+        y = t % P;
+        z = bad ? pv.num_pages * Hkv : page * Hkv + hk;
+      } else {
+        y = hk;
+        z = bad ? pv.num_pages * P : page * P + t % P;
+      }
+      tma_load_3d(dst + lane * copy_bytes, tm_k, 0, y, z, bar);
+      tma_load_3d(dst + tile_bytes + lane * copy_bytes, tm_v, 0, y, z, bar);
+    }
+  }
+};
+
+template <int D, int GT, bool PAGED>
 __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_SM)
     decode_split_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
                         const __nv_bfloat16* __restrict__ v, const int32_t* __restrict__ seqlens,
                         float* __restrict__ o_part, float* __restrict__ lse_part, int Hq, int Hkv,
                         int Skv, int splits, int n_groups, float c, KernelCtl ctl,
                         const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
-                        PagedView pv, __nv_bfloat16* __restrict__ o_out, float* __restrict__ lse_out) {
+                        PagedView pv) {
   using C = DecodeCfg<D>;
-  using L = DecodeSmem<D, GT, FUSED>;
+  using L = DecodeSmem<D, GT>;
   extern __shared__ __align__(128) uint8_t smem[];
 
   // Let the merge grid launch as soon as every split CTA is resident.
-  if constexpr (!FUSED) asm volatile("griddepcontrol.launch_dependents;");
+  asm volatile("griddepcontrol.launch_dependents;");
 
   const int split = blockIdx.x;
   const int hk = blockIdx.y / n_groups, grp = blockIdx.y % n_groups;
@@ -206,20 +395,11 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
   const int t_begin = min(split * chunk, len);
   const int t_end = min(t_begin + chunk, len);
   const size_t row0 = (static_cast<size_t>(b) * Hq + h0) * splits + split;  // head h0's partial
-  const uint32_t part_o = smem_u32(smem) + L::PART_O_OFF, part_l = smem_u32(smem) + L::PART_L_OFF;
-  const size_t o_row0 = static_cast<size_t>(b) * Hq + h0;  // single-kernel form: first output row
 
   if (t_begin >= t_end) {  // empty split: contributes nothing to the merge
-    if constexpr (FUSED) {
-      float* po = reinterpret_cast<float*>(smem + L::PART_O_OFF);
-      for (int i = threadIdx.x; i < nh * D; i += blockDim.x) po[i] = 0.f;
-      if (threadIdx.x < nh) reinterpret_cast<float*>(smem + L::PART_L_OFF)[threadIdx.x] = -INFINITY;
-      cluster_gather<D>(part_o, part_l, nh, splits, o_out, lse_out, o_row0);
-    } else {
-      for (int i = threadIdx.x; i < nh * D; i += blockDim.x)
-        o_part[(row0 + static_cast<size_t>(i / D) * splits) * D + i % D] = 0.f;
-      if (threadIdx.x < nh) lse_part[row0 + static_cast<size_t>(threadIdx.x) * splits] = -INFINITY;
-    }
+    for (int i = threadIdx.x; i < nh * D; i += blockDim.x)
+      o_part[(row0 + static_cast<size_t>(i / D) * splits) * D + i % D] = 0.f;
+    if (threadIdx.x < nh) lse_part[row0 + static_cast<size_t>(threadIdx.x) * splits] = -INFINITY;
     return;
   }
   const int n_stages = (t_end - t_begin + C::T - 1) / C::T;
@@ -244,53 +424,20 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
     // ------------------------------------------------------------ loader warp
     if constexpr (PAGED) {
       static_assert(C::T % kDecodeChunkAlign == 0, "stages start on a copy boundary");
-      // Copies of `rows` keys: a 64-key piece of one page (page_size a multiple of 64) or
-      // one whole page (page_size 8, 16 or 32).  Stages start on a multiple of 64 keys, so
-      // no copy crosses a page; a stage takes at most T / 8 copies.
-      const int P = pv.page_size;
-      const int rows = P < kDecodeChunkAlign ? P : kDecodeChunkAlign;
-      const uint32_t copy_bytes = static_cast<uint32_t>(rows) * D * 2;
       const int32_t* tbl = pv.block_table + static_cast<size_t>(b) * pv.max_pages;
-      int win = 0, entry = 0;
-      bool have = false;
+      PagedLoader pl;
       int issued = 0, skipped = -1;
       for (int it = 0; it < n_stages; ++it) {
         const int slot = it % C::NSTAGE, round = it / C::NSTAGE;
         if (!mbar_wait_warp(bar_empty + 8 * slot, (round & 1) ^ 1, ctl, ab)) break;
-        const int tok0 = t_begin + it * C::T;
-        const int ncopy = (min(C::T, t_end - tok0) + rows - 1) / rows;
-        const int lp_first = tok0 / P, lp_last = (tok0 + (ncopy - 1) * rows) / P;
-        if (!have || lp_first < win || lp_last >= win + 32) {  // refill the table window
-          win = lp_first;
-          entry = (win + lane < pv.max_pages) ? tbl[win + lane] : 0;
-          have = true;
-        }
         issued = it + 1;
         if (ctl.inject == 1 && it == 1) {  // test hook: never fill this stage
           skipped = it;
           continue;
         }
-        const uint32_t dst = s_base + slot * C::STAGE_BYTES;
-        if (lane == 0) mbar_expect_tx(bar_full + 8 * slot, 2u * ncopy * copy_bytes);
-        __syncwarp();
-        const int t = tok0 + lane * rows;
-        const int page = __shfl_sync(0xffffffffu, entry, (t / P - win) & 31);
-        if (lane < ncopy) {
-          // An out-of-range page (a caller error) is sent past the end of the cache, where
-          // the copy engine reads zeros.  NHD view [keys of all pages, Hkv, D]: (0, hk, key);
-          // HND view [pages x Hkv, page_size, D]: (0, row in page, page x Hkv + hk).
-          const bool bad = page < 0 || page >= pv.num_pages;
-          int y, z;
-          if (pv.hnd) {
-            y = t % P;
-            z = bad ? pv.num_pages * Hkv : page * Hkv + hk;
-          } else {
-            y = hk;
-            z = bad ? pv.num_pages * P : page * P + t % P;
-          }
-          tma_load_3d(dst + lane * copy_bytes, &tm_k, 0, y, z, bar_full + 8 * slot);
-          tma_load_3d(dst + C::TILE_BYTES + lane * copy_bytes, &tm_v, 0, y, z, bar_full + 8 * slot);
-        }
+        const int tok0 = t_begin + it * C::T;
+        pl.stage<D>(pv, tbl, Hkv, hk, tok0, min(C::T, t_end - tok0), s_base + slot * C::STAGE_BYTES,
+                    bar_full + 8 * slot, C::TILE_BYTES, &tm_k, &tm_v, lane);
       }
       if (lane == 0) {
         Abort no_abort{reinterpret_cast<volatile int*>(smem + L::ABORT_OFF + 4)};
@@ -325,37 +472,13 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
         mbar_wait(bar_full + 8 * (it % C::NSTAGE), (it / C::NSTAGE) & 1, ctl, no_abort);
       }
     }
-    if constexpr (FUSED) {  // the loader warp takes its share of the cluster gather
-      __syncwarp();
-      cluster_gather<D>(part_o, part_l, nh, splits, o_out, lse_out, o_row0);
-    }
     return;
   }
 
   // -------------------------------------------------------------- compute warps
-  const int kl = lane % C::KL;   // 16-byte column of the K row this lane reads
-  const int tg = lane / C::KL;   // token within a load round
-  const int hl = head_of_lane<C::KL, GT>(lane);
-  const bool primary = ((lane % C::KL) & (C::KL / GT - 1)) == 0;  // one lane per (token, head)
-
-  // q of the GT heads, pre-multiplied by scale*log2(e) so scores come out in base 2
+  const LaneRole<D, GT> lr(lane);
   float qf[GT][8];
-#pragma unroll
-  for (int h = 0; h < GT; ++h) {
-    if (h < nh) {
-      const uint4 raw = *reinterpret_cast<const uint4*>(
-          q + (static_cast<size_t>(b) * Hq + h0 + h) * D + kl * 8);
-      const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        qf[h][2 * i] = bf16lo(w[i]) * c;
-        qf[h][2 * i + 1] = bf16hi(w[i]) * c;
-      }
-    } else {
-#pragma unroll
-      for (int i = 0; i < 8; ++i) qf[h][i] = 0.f;
-    }
-  }
+  load_q<D, GT>(q + (static_cast<size_t>(b) * Hq + h0) * D, nh, lr.kl, c, qf);
 
   float m_run = -INFINITY, l_run = 0.f;
   float acc_o[GT][C::VD];
@@ -370,149 +493,292 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
   for (int it = 0; it < n_stages; ++it) {
     const int slot = it % C::NSTAGE;
     if (!mbar_wait_warp(bar_full + 8 * slot, (it / C::NSTAGE) & 1, ctl, ab)) break;
-    const int ntok = min(C::T, t_end - (t_begin + it * C::T));
     const uint8_t* ks = smem + slot * C::STAGE_BYTES;
-    const uint8_t* vs = ks + C::TILE_BYTES;
-
-    // scores of this warp's TW tokens, in base-2 units
-    float sc[C::KROUNDS];
-#pragma unroll
-    for (int r = 0; r < C::KROUNDS; ++r) {
-      const int tl = warp * C::TW + r * C::TPR + tg;
-      const uint4 raw = *reinterpret_cast<const uint4*>(ks + tl * (D * 2) + kl * 16);
-      const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
-      float kf[8];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        kf[2 * i] = bf16lo(w[i]);
-        kf[2 * i + 1] = bf16hi(w[i]);
-      }
-      float acc[GT];
-#pragma unroll
-      for (int h = 0; h < GT; ++h) {
-        float s = 0.f;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) s = fmaf(qf[h][i], kf[i], s);
-        acc[h] = s;
-      }
-      const float s = transpose_reduce<C::KL, GT>(acc, lane);
-      sc[r] = (tl < ntok) ? s : -INFINITY;
-    }
-
-    // online softmax (per head, over this warp's tokens)
-    float mx = sc[0];
-#pragma unroll
-    for (int r = 1; r < C::KROUNDS; ++r) mx = fmaxf(mx, sc[r]);
-#pragma unroll
-    for (int off = C::KL; off < 32; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-    const float m_new = fmaxf(m_run, mx);
-    const bool need = m_new > m_run + kRescaleThreshold;
-    const float alpha = need ? ex2(m_run - m_new) : 1.f;
-    if (need) m_run = m_new;
-    const float ms = (m_run == -INFINITY) ? 0.f : m_run;
-    float psum = 0.f;
-    __syncwarp();
-#pragma unroll
-    for (int r = 0; r < C::KROUNDS; ++r) {
-      const float p = ex2(sc[r] - ms);
-      psum += p;
-      if (primary) ps[(r * C::TPR + tg) * GT + hl] = p;
-    }
-    l_run = l_run * alpha + psum;
-    if (primary && tg == 0) alpha_s[hl] = alpha;
-    __syncwarp();
-
-    if (__any_sync(0xffffffffu, need)) {
-#pragma unroll
-      for (int h = 0; h < GT; ++h) {
-        const float a = alpha_s[h];
-#pragma unroll
-        for (int d = 0; d < C::VD; ++d) acc_o[h][d] *= a;
-      }
-    }
-
-    // P.V over this warp's tokens; lane owns dims [lane*VD, lane*VD + VD)
-    const int nmine = min(C::TW, ntok - warp * C::TW);
-#pragma unroll 4
-    for (int tt = 0; tt < nmine; ++tt) {
-      const int tl = warp * C::TW + tt;
-      float vf[C::VD];
-      if constexpr (C::VD == 4) {
-        const uint2 raw = *reinterpret_cast<const uint2*>(vs + tl * (D * 2) + lane * 8);
-        vf[0] = bf16lo(raw.x);
-        vf[1] = bf16hi(raw.x);
-        vf[2] = bf16lo(raw.y);
-        vf[3] = bf16hi(raw.y);
-      } else {
-        const uint32_t raw = *reinterpret_cast<const uint32_t*>(vs + tl * (D * 2) + lane * 4);
-        vf[0] = bf16lo(raw);
-        vf[1] = bf16hi(raw);
-      }
-      float pv[GT];
-      if constexpr (GT % 4 == 0) {
-#pragma unroll
-        for (int h = 0; h < GT; h += 4) {
-          const float4 p4 = *reinterpret_cast<const float4*>(ps + tt * GT + h);
-          pv[h] = p4.x;
-          pv[h + 1] = p4.y;
-          pv[h + 2] = p4.z;
-          pv[h + 3] = p4.w;
-        }
-      } else {
-#pragma unroll
-        for (int h = 0; h < GT; ++h) pv[h] = ps[tt * GT + h];
-      }
-#pragma unroll
-      for (int h = 0; h < GT; ++h)
-#pragma unroll
-        for (int d = 0; d < C::VD; ++d) acc_o[h][d] = fmaf(pv[h], vf[d], acc_o[h][d]);
-    }
+    decode_stage<D, GT>(ks, ks + C::TILE_BYTES, min(C::T, t_end - (t_begin + it * C::T)), warp, lane, lr, qf, m_run,
+                        l_run, acc_o, ps, alpha_s);
     __syncwarp();
     if (lane == 0) mbar_arrive(bar_empty + 8 * slot);
   }
 
-  // ---------------------------------------------------------------- merge the 8 warps
-#pragma unroll
-  for (int off = C::KL; off < 32; off <<= 1) l_run += __shfl_xor_sync(0xffffffffu, l_run, off);
-  asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");  // ring no longer read
-  float* wm = reinterpret_cast<float*>(smem + L::WM_OFF);
-  float* wl = reinterpret_cast<float*>(smem + L::WL_OFF);
-  float* wo = reinterpret_cast<float*>(smem);  // [NCW][GT][D], reuses the ring
-  if (primary && tg == 0) {
-    wm[warp * GT + hl] = m_run;
-    wl[warp * GT + hl] = l_run;
-  }
-#pragma unroll
-  for (int h = 0; h < GT; ++h)
-#pragma unroll
-    for (int d = 0; d < C::VD; ++d) wo[(warp * GT + h) * D + lane * C::VD + d] = acc_o[h][d];
-  asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");
+  // the 8 warps' states -> the split's partial in the workspace (the drained ring is the scratch)
+  merge_warps<D, GT>(reinterpret_cast<float*>(smem), reinterpret_cast<float*>(smem + L::WM_OFF),
+                     reinterpret_cast<float*>(smem + L::WL_OFF), nh, warp, lane, lr, m_run, l_run, acc_o,
+                     [&](int, int h, int d, float ov, float lv) {
+                       const size_t row = row0 + static_cast<size_t>(h) * splits;
+                       o_part[row * D + d] = ov;
+                       if (d == 0) lse_part[row] = lv;
+                     });
+}
 
-  for (int idx = threadIdx.x; idx < nh * D; idx += C::NCW * 32) {
-    const int h = idx / D, d = idx % D;
-    float M = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < C::NCW; ++w) M = fmaxf(M, wm[w * GT + h]);
-    float lsum = 0.f, osum = 0.f;
-    if (M != -INFINITY) {
-#pragma unroll
-      for (int w = 0; w < C::NCW; ++w) {
-        const float a = ex2(wm[w * GT + h] - M);  // 0 for warps that saw no key
-        lsum = fmaf(a, wl[w * GT + h], lsum);
-        osum = fmaf(a, wo[(w * GT + h) * D + d], osum);
+// ---------------------------------------------------------------- single-kernel form
+template <int D, int GT>
+struct ClusterSmem {
+  using C = DecodeCfg<D>;
+  static constexpr int kMaxSortedB = 256;  // sequences sorted by length for the dealing
+  // ring first (16-byte aligned bulk-copy destinations), then the small arrays
+  static constexpr uint32_t P_OFF = C::RING_BYTES;                        // [NCW][TW][GT] f32
+  static constexpr uint32_t ALPHA_OFF = P_OFF + C::NCW * C::TW * GT * 4;  // [NCW][GT] f32
+  static constexpr uint32_t WM_OFF = ALPHA_OFF + C::NCW * GT * 4;         // [NCW][GT] f32
+  static constexpr uint32_t WL_OFF = WM_OFF + C::NCW * GT * 4;            // [NCW][GT] f32
+  static constexpr uint32_t Q_OFF = (WL_OFF + C::NCW * GT * 4 + 15) / 16 * 16;  // [GT][D] bf16, q of a unit
+  static constexpr uint32_t PO_OFF = Q_OFF + GT * D * 2;                 // [GT][D] f32, this CTA's partial O
+  static constexpr uint32_t PL_OFF = PO_OFF + GT * D * 4;                // [GT] f32, its log-sum-exps
+  static constexpr uint32_t ORDER_OFF = (PL_OFF + GT * 4 + 15) / 16 * 16;  // [kMaxSortedB] int32
+  static constexpr uint32_t BAR_OFF = ORDER_OFF + kMaxSortedB * 4;
+  // full[NSTAGE], empty[NSTAGE], q_full, q_empty, ready, consumed
+  static constexpr uint32_t ABORT_OFF = BAR_OFF + (2 * C::NSTAGE + 4) * 8;
+  static constexpr uint32_t BYTES = ABORT_OFF + 16;
+  static_assert(C::NCW * GT * D * 4 <= C::STAGE_BYTES, "the warps' merge fits in one ring slot");
+  static_assert(C::CTAS_PER_SM * (BYTES + 1024) <= 228 * 1024, "CTAs per SM of the stage plan");
+};
+
+// The k-th unit of cluster `cid` of n_clusters: units sorted by sequence length (longest
+// first), dealt in a snake order (even rounds left to right, odd rounds right to left);
+// -1 past the last.
+__device__ __forceinline__ int cluster_unit(int kk, int cid, int n_clusters, int n_units) {
+  const long long i = static_cast<long long>(kk) * n_clusters + ((kk & 1) ? n_clusters - 1 - cid : cid);
+  return i < n_units ? static_cast<int>(i) : -1;
+}
+
+template <int D, int GT, bool PAGED>
+__global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_SM)
+    decode_cluster_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
+                          const __nv_bfloat16* __restrict__ v, const int32_t* __restrict__ seqlens,
+                          __nv_bfloat16* __restrict__ o, float* __restrict__ lse, int B, int Hq, int Hkv, int Skv,
+                          int splits, int n_groups, float c, KernelCtl ctl,
+                          const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                          PagedView pv) {
+  using C = DecodeCfg<D>;
+  using L = ClusterSmem<D, GT>;
+  extern __shared__ __align__(128) uint8_t smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int cs = static_cast<int>(cluster_nctarank());
+  const int rank = static_cast<int>(cluster_ctarank());
+  const int cid = static_cast<int>(blockIdx.x) / cs;
+  const int n_clusters = static_cast<int>(gridDim.x) / cs;
+  const int G = Hq / Hkv;
+  const int upb = Hkv * n_groups;  // units per sequence
+  const int n_units = B * upb;
+  const int per_cta = splits / cs;  // splits r, r + cs, ... of every unit belong to CTA r
+
+  const uint32_t s_base = smem_u32(smem);
+  const uint32_t bar_full = s_base + L::BAR_OFF;
+  const uint32_t bar_empty = bar_full + C::NSTAGE * 8;
+  const uint32_t bar_qf = bar_empty + C::NSTAGE * 8;
+  const uint32_t bar_qe = bar_qf + 8;
+  const uint32_t bar_ready = bar_qe + 8;     // every CTA's partial of the current unit is written
+  const uint32_t bar_consumed = bar_ready + 8;  // every CTA has read this CTA's partial
+  Abort ab{reinterpret_cast<volatile int*>(smem + L::ABORT_OFF)};
+
+  // the sequences in order of decreasing length (ties by index): the dealing order
+  int* order = reinterpret_cast<int*>(smem + L::ORDER_OFF);
+  const bool sorted = seqlens != nullptr && B <= L::kMaxSortedB;
+  if (sorted) {
+    for (int bb = threadIdx.x; bb < B; bb += blockDim.x) {
+      const int lb = seqlens[bb];
+      int r = 0;
+      for (int x = 0; x < B; ++x) {
+        const int lx = seqlens[x];
+        r += (lx > lb) || (lx == lb && x < bb);
+      }
+      order[r] = bb;
+    }
+  }
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSTAGE; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, C::NCW);
+    }
+    mbar_init(bar_qf, 1);
+    mbar_init(bar_qe, C::NCW);
+    mbar_init(bar_ready, cs);
+    mbar_init(bar_consumed, cs);
+    *ab.flag = 0;
+    *(ab.flag + 1) = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+  cluster_sync_all();  // every CTA's barriers exist before a peer arrives on them
+
+  // unit i (sorted order) -> sequence, kv head, head group, and the sequence's chunk length
+  struct Unit {
+    int b, hk, grp, h0, nh, len, chunk;
+  };
+  auto unit = [&](int i) {
+    Unit u;
+    const int br = i / upb, j = i % upb;
+    u.b = sorted ? order[br] : br;
+    u.hk = j / n_groups;
+    u.grp = j % n_groups;
+    u.h0 = u.hk * G + u.grp * GT;
+    u.nh = min(GT, G - u.grp * GT);
+    u.len = max(0, min(seqlens ? seqlens[u.b] : Skv, Skv));
+    const int ch = (u.len + splits - 1) / splits;
+    u.chunk = (ch + kDecodeChunkAlign - 1) / kDecodeChunkAlign * kDecodeChunkAlign;
+    return u;
+  };
+  // keys [*t0, *t1) of this CTA's jj-th split of unit u
+  auto split_range = [&](const Unit& u, int jj, int* t0, int* t1) {
+    const int s = rank + jj * cs;
+    *t0 = min(s * u.chunk, u.len);
+    *t1 = min(*t0 + u.chunk, u.len);
+  };
+
+  if (warp == C::NCW) {
+    // ------------------------------------------------------------ loader warp (whole warp)
+    PagedLoader pl;
+    int pos = 0, skipped = -1, q_loads = 0;
+    bool ok = true;
+    for (int kk = 0, ui; ok && (ui = cluster_unit(kk, cid, n_clusters, n_units)) >= 0; ++kk) {
+      const Unit u = unit(ui);
+      // the unit's q rows (one bulk copy), once the compute warps have read the previous unit's
+      if (kk > 0 && !(ok = mbar_wait_warp(bar_qe, (kk - 1) & 1, ctl, ab))) break;
+      if (lane == 0) {
+        const uint32_t qbytes = static_cast<uint32_t>(u.nh) * D * 2;
+        mbar_expect_tx(bar_qf, qbytes);
+        bulk_g2s(s_base + L::Q_OFF, q + (static_cast<size_t>(u.b) * Hq + u.h0) * D, qbytes, bar_qf);
+      }
+      q_loads = kk + 1;
+      if constexpr (PAGED) pl.reset();
+      const size_t kv_row0 = (static_cast<size_t>(u.b) * Hkv + u.hk) * Skv;
+      const int32_t* tbl = PAGED ? pv.block_table + static_cast<size_t>(u.b) * pv.max_pages : nullptr;
+      for (int jj = 0; ok && jj < per_cta; ++jj) {
+        int t0, t1;
+        split_range(u, jj, &t0, &t1);
+        for (int tok0 = t0; tok0 < t1; tok0 += C::T, ++pos) {
+          const int slot = pos % C::NSTAGE, round = pos / C::NSTAGE;
+          if (!(ok = mbar_wait_warp(bar_empty + 8 * slot, (round & 1) ^ 1, ctl, ab))) break;
+          if (ctl.inject == 1 && pos == 1) {  // test hook: never fill this stage
+            skipped = pos;
+            continue;
+          }
+          const int ntok = min(C::T, t1 - tok0);
+          const uint32_t dst = s_base + slot * C::STAGE_BYTES;
+          if constexpr (PAGED) {
+            pl.stage<D>(pv, tbl, Hkv, u.hk, tok0, ntok, dst, bar_full + 8 * slot, C::TILE_BYTES, &tm_k, &tm_v,
+                        lane);
+          } else if (lane == 0) {
+            const uint32_t bytes = static_cast<uint32_t>(ntok) * D * 2;
+            mbar_expect_tx(bar_full + 8 * slot, 2 * bytes);
+            bulk_g2s(dst, k + (kv_row0 + tok0) * D, bytes, bar_full + 8 * slot);
+            bulk_g2s(dst + C::TILE_BYTES, v + (kv_row0 + tok0) * D, bytes, bar_full + 8 * slot);
+          }
+        }
       }
     }
-    const bool any = lsum > 0.f;
-    if constexpr (FUSED) {
-      reinterpret_cast<float*>(smem + L::PART_O_OFF)[idx] = any ? osum / lsum : 0.f;
-      if (d == 0) reinterpret_cast<float*>(smem + L::PART_L_OFF)[h] = any ? (M + log2f(lsum)) * kLn2 : -INFINITY;
-    } else {
-      const size_t row = row0 + static_cast<size_t>(h) * splits;
-      o_part[row * D + d] = any ? osum / lsum : 0.f;
-      if (d == 0) lse_part[row] = any ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+    // Drain: never leave the CTA with copies still landing in its shared memory.
+    if (lane == 0) {
+      Abort no_abort{ab.flag + 1};
+      for (int it = max(0, pos - C::NSTAGE); it < pos; ++it)
+        if (it != skipped) mbar_wait(bar_full + 8 * (it % C::NSTAGE), (it / C::NSTAGE) & 1, ctl, no_abort);
+      if (q_loads > 0) mbar_wait(bar_qf, (q_loads - 1) & 1, ctl, no_abort);
+    }
+    __syncwarp();
+  } else {
+    // -------------------------------------------------------------- compute warps
+    const LaneRole<D, GT> lr(lane);
+    float* ps = reinterpret_cast<float*>(smem + L::P_OFF) + warp * C::TW * GT;
+    float* alpha_s = reinterpret_cast<float*>(smem + L::ALPHA_OFF) + warp * GT;
+    float* part_o = reinterpret_cast<float*>(smem + L::PO_OFF);
+    float* part_l = reinterpret_cast<float*>(smem + L::PL_OFF);
+    int pos = 0;
+    // A failed (timed-out) wait is made known to all compute warps at the unit's next
+    // common point (a barrier reduction), so that they leave together and none is left
+    // waiting at a barrier of the merge.
+    for (int kk = 0, ui; (ui = cluster_unit(kk, cid, n_clusters, n_units)) >= 0; ++kk) {
+      const Unit u = unit(ui);
+      bool ok = mbar_wait_warp(bar_qf, kk & 1, ctl, ab);
+      float qf[GT][8];
+      load_q<D, GT>(reinterpret_cast<const __nv_bfloat16*>(smem + L::Q_OFF), u.nh, lr.kl, c, qf);
+      __syncwarp();
+      if (ok && lane == 0) mbar_arrive(bar_qe);
+
+      float m_run = -INFINITY, l_run = 0.f;
+      float acc_o[GT][C::VD];
+#pragma unroll
+      for (int h = 0; h < GT; ++h)
+#pragma unroll
+        for (int d = 0; d < C::VD; ++d) acc_o[h][d] = 0.f;
+
+      int n_st = 0;  // this CTA's stages of the unit
+      for (int jj = 0; jj < per_cta; ++jj) {
+        int t0, t1;
+        split_range(u, jj, &t0, &t1);
+        n_st += (t1 - t0 + C::T - 1) / C::T;
+      }
+      int st = 0;
+      for (int jj = 0; ok && jj < per_cta; ++jj) {
+        int t0, t1;
+        split_range(u, jj, &t0, &t1);
+        for (int tok0 = t0; tok0 < t1; tok0 += C::T, ++pos, ++st) {
+          const int slot = pos % C::NSTAGE;
+          if (!(ok = mbar_wait_warp(bar_full + 8 * slot, (pos / C::NSTAGE) & 1, ctl, ab))) break;
+          const uint8_t* ks = smem + slot * C::STAGE_BYTES;
+          decode_stage<D, GT>(ks, ks + C::TILE_BYTES, min(C::T, t1 - tok0), warp, lane, lr, qf, m_run, l_run, acc_o,
+                              ps, alpha_s);
+          __syncwarp();
+          // the unit's last slot stays held: it is the scratch of the merge below
+          if (st + 1 < n_st && lane == 0) mbar_arrive(bar_empty + 8 * slot);
+        }
+      }
+      // this CTA's partial of the unit, once every CTA has read its previous one
+      if (ok && kk > 0) ok = mbar_wait_cluster_warp(bar_consumed, (kk - 1) & 1, ctl, ab);
+      if (named_bar_any(1, C::NCW * 32, !ok)) break;
+      if (n_st > 0) {
+        const int last = (pos - 1) % C::NSTAGE;
+        merge_warps<D, GT>(reinterpret_cast<float*>(smem + last * C::STAGE_BYTES),
+                           reinterpret_cast<float*>(smem + L::WM_OFF), reinterpret_cast<float*>(smem + L::WL_OFF),
+                           u.nh, warp, lane, lr, m_run, l_run, acc_o, [&](int idx, int h, int d, float ov, float lv) {
+                             part_o[idx] = ov;
+                             if (d == 0) part_l[h] = lv;
+                           });
+        asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");  // partial written, slot read
+        if (lane == 0) mbar_arrive(bar_empty + 8 * last);
+      } else {  // no key of the unit falls to this CTA
+        for (int idx = threadIdx.x; idx < u.nh * D; idx += C::NCW * 32) part_o[idx] = 0.f;
+        if (threadIdx.x < u.nh) part_l[threadIdx.x] = -INFINITY;
+        asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");
+      }
+      if (static_cast<int>(threadIdx.x) < cs) mbar_arrive_cluster(map_shared_rank(bar_ready, threadIdx.x));
+      ok = mbar_wait_cluster_warp(bar_ready, kk & 1, ctl, ab);
+      if (named_bar_any(1, C::NCW * 32, !ok)) break;
+
+      // gather, global softmax and final scaling of this CTA's share of the unit's outputs
+      const int total = u.nh * D;
+      const int per = (total + cs - 1) / cs;
+      const int e1 = min(total, (rank + 1) * per);
+      const size_t o_row0 = static_cast<size_t>(u.b) * Hq + u.h0;
+      for (int e = rank * per + static_cast<int>(threadIdx.x); e < e1; e += C::NCW * 32) {
+        const int h = e / D, d = e % D;
+        float l[model::kMaxClusterSize];
+        float M = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < model::kMaxClusterSize; ++i) {
+          l[i] = i < cs ? ld_dsmem_f32(map_shared_rank(s_base + L::PL_OFF + 4u * h, i)) : -INFINITY;
+          M = fmaxf(M, l[i]);
+        }
+        float W = 0.f, acc = 0.f;
+        if (M != -INFINITY) {
+#pragma unroll
+          for (int i = 0; i < model::kMaxClusterSize; ++i) {
+            if (i < cs) {
+              const float w = ex2((l[i] - M) * kLog2e);  // 0 for a CTA without keys
+              W += w;
+              acc = fmaf(w, ld_dsmem_f32(map_shared_rank(s_base + L::PO_OFF + 4u * e, i)), acc);
+            }
+          }
+        }
+        const bool any = W > 0.f;
+        o[(o_row0 + h) * D + d] = __float2bfloat16_rn(any ? acc / W : 0.f);
+        if (lse && d == 0) lse[o_row0 + h] = any ? M + log2f(W) * kLn2 : -INFINITY;
+      }
+      asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");  // this CTA's reads are done
+      if (static_cast<int>(threadIdx.x) < cs) mbar_arrive_cluster(map_shared_rank(bar_consumed, threadIdx.x));
     }
   }
-  if constexpr (FUSED) cluster_gather<D>(part_o, part_l, nh, splits, o_out, lse_out, o_row0);
+  // Leave together: no CTA exits while a peer may still read its partial or arrive on its
+  // barriers.
+  cluster_sync_all();
 }
 
 // One CTA (D threads) per (batch, query head).  The split log-sum-exps are read in
@@ -609,33 +875,42 @@ bool paged_map(CUtensorMap* map, const void* cache, const PagedKV& pk, int Hkv, 
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+
 // Per-device set-up of one kernel instance: the shared-memory opt-in and, for the cluster
-// form, clusters of up to 16 CTAs (beyond the portable 8).
-template <int D, int GT, bool PAGED, bool FUSED>
-bool prepare_split() {
-  static PerDeviceOnce configured;
+// kernel, clusters of up to 16 CTAs (beyond the portable 8).
+template <class Kernel>
+bool prepare_kernel(Kernel kernel, uint32_t smem, bool cluster, PerDeviceOnce& once) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
-  return configured.run(dev, [] {
-    const void* fn = reinterpret_cast<const void*>(decode_split_kernel<D, GT, PAGED, FUSED>);
-    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, DecodeSmem<D, GT, FUSED>::BYTES) !=
-        cudaSuccess)
-      return false;
-    if constexpr (FUSED) return cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
-    return true;
+  return once.run(dev, [&] {
+    const void* fn = reinterpret_cast<const void*>(kernel);
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess) return false;
+    return !cluster || cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
   });
 }
 
-template <int D, int GT, bool FUSED>
-cudaLaunchConfig_t split_config(dim3 grid, int cluster, cudaStream_t stream, cudaLaunchAttribute* attr) {
+template <int D, int GT, bool PAGED>
+bool prepare_split() {
+  static PerDeviceOnce once;
+  return prepare_kernel(decode_split_kernel<D, GT, PAGED>, DecodeSmem<D, GT>::BYTES, false, once);
+}
+
+template <int D, int GT, bool PAGED>
+bool prepare_cluster() {
+  static PerDeviceOnce once;
+  return prepare_kernel(decode_cluster_kernel<D, GT, PAGED>, ClusterSmem<D, GT>::BYTES, true, once);
+}
+
+cudaLaunchConfig_t launch_config(dim3 grid, uint32_t smem, int cluster, cudaStream_t stream, cudaLaunchAttribute* attr) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
-  cfg.blockDim = dim3(DecodeCfg<D>::THREADS);
-  cfg.dynamicSmemBytes = DecodeSmem<D, GT, FUSED>::BYTES;
+  cfg.blockDim = dim3(DecodeCfg<128>::THREADS);
+  static_assert(DecodeCfg<128>::THREADS == DecodeCfg<64>::THREADS, "one block shape");
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 0;
-  if (FUSED) {
+  if (cluster > 0) {
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = static_cast<unsigned>(cluster);
     attr[0].val.clusterDim.y = 1;
@@ -645,55 +920,86 @@ cudaLaunchConfig_t split_config(dim3 grid, int cluster, cudaStream_t stream, cud
   return cfg;
 }
 
-// CTA slots of the cluster form with clusters of `splits` CTAs on the current device: whole
-// clusters that fit at once (cudaOccupancyMaxActiveClusters) x splits; 0 if none fit or the
-// device cannot be asked.  Cached per device and cluster size.
+// Clusters of `cs` cluster-kernel CTAs that fit on the current device at once
+// (cudaOccupancyMaxActiveClusters); 0 if none or the device cannot be asked.  Cached per
+// device and cluster size.
 template <int D, int GT, bool PAGED>
-int cluster_slots(int splits) {
-  static std::atomic<int> cache[64][model::kMaxFusedSplits + 1];  // value + 1 once known
+int max_clusters(int cs) {
+  static std::atomic<int> cache[64][model::kMaxClusterSize + 1];  // value + 1 once known
   int dev = 0;
-  if (splits < 1 || splits > model::kMaxFusedSplits || cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 0;
+  if (cs < 1 || cs > model::kMaxClusterSize || cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 0;
   if (dev < 64) {
-    const int c = cache[dev][splits].load(std::memory_order_relaxed);
+    const int c = cache[dev][cs].load(std::memory_order_relaxed);
     if (c != 0) return c - 1;
   }
   int clusters = 0;
-  if (prepare_split<D, GT, PAGED, true>()) {
+  if (prepare_cluster<D, GT, PAGED>()) {
     cudaLaunchAttribute attr[1];
-    const cudaLaunchConfig_t cfg = split_config<D, GT, true>(dim3(splits, 64, 1), splits, nullptr, attr);
-    if (cudaOccupancyMaxActiveClusters(&clusters, decode_split_kernel<D, GT, PAGED, true>, &cfg) != cudaSuccess) {
+    const cudaLaunchConfig_t cfg = launch_config(dim3(cs * 64), ClusterSmem<D, GT>::BYTES, cs, nullptr, attr);
+    if (cudaOccupancyMaxActiveClusters(&clusters, decode_cluster_kernel<D, GT, PAGED>, &cfg) != cudaSuccess) {
       cudaGetLastError();
       clusters = 0;
     }
   }
-  if (dev < 64) cache[dev][splits].store(clusters * splits + 1, std::memory_order_relaxed);
-  return clusters * splits;
+  if (dev < 64) cache[dev][cs].store(clusters + 1, std::memory_order_relaxed);
+  return clusters;
 }
 
-template <int D, int GT, bool PAGED, bool FUSED>
-cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
-  if (!prepare_split<D, GT, PAGED, FUSED>()) return cudaErrorInvalidValue;
-  CUtensorMap tk, tv;
-  PagedView view{nullptr, 0, 0, 0, 0};
+// Views of the K and V caches for the split kernels' loaders: paged caches as TMA tensors,
+// contiguous caches need none (1-D bulk copies).
+template <int D, bool PAGED>
+bool kv_views(const DecodeArgs& a, const PagedKV* pk, CUtensorMap* tk, CUtensorMap* tv, PagedView* view) {
+  *view = PagedView{nullptr, 0, 0, 0, 0};
   if constexpr (PAGED) {
     const int rows = pk->page_size < kDecodeChunkAlign ? pk->page_size : kDecodeChunkAlign;
-    if (!paged_map(&tk, a.k, *pk, a.Hkv, D, rows) || !paged_map(&tv, a.v, *pk, a.Hkv, D, rows))
-      return cudaErrorInvalidValue;
-    view = PagedView{pk->block_table, pk->page_size, pk->max_pages, pk->num_pages, pk->layout == kPagedHND ? 1 : 0};
+    if (!paged_map(tk, a.k, *pk, a.Hkv, D, rows) || !paged_map(tv, a.v, *pk, a.Hkv, D, rows)) return false;
+    *view = PagedView{pk->block_table, pk->page_size, pk->max_pages, pk->num_pages, pk->layout == kPagedHND ? 1 : 0};
   } else {
+    (void)a;
     (void)pk;
-    memset(&tk, 0, sizeof(tk));
-    memset(&tv, 0, sizeof(tv));
+    memset(tk, 0, sizeof(*tk));
+    memset(tv, 0, sizeof(*tv));
   }
+  return true;
+}
+
+template <int D, int GT, bool PAGED>
+cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
+  if (!prepare_split<D, GT, PAGED>()) return cudaErrorInvalidValue;
+  CUtensorMap tk, tv;
+  PagedView view;
+  if (!kv_views<D, PAGED>(a, pk, &tk, &tv, &view)) return cudaErrorInvalidValue;
   const int G = a.Hq / a.Hkv;
   const int n_groups = (G + GT - 1) / GT;
+  dim3 grid(a.splits, a.Hkv * n_groups, a.B);
+  decode_split_kernel<D, GT, PAGED><<<grid, DecodeCfg<D>::THREADS, DecodeSmem<D, GT>::BYTES, stream>>>(
+      static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.k),
+      static_cast<const __nv_bfloat16*>(a.v), a.seqlens, a.o_part, a.lse_part, a.Hq, a.Hkv, a.Skv,
+      a.splits, n_groups, a.scale * kLog2e, ctl, tk, tv, view);
+  return cudaGetLastError();
+}
+
+// The cluster kernel with clusters of cs CTAs: as many clusters as fit at once, at most one
+// per unit.
+template <int D, int GT, bool PAGED>
+cudaError_t launch_cluster(const DecodeArgs& a, int cs, const PagedKV* pk, const KernelCtl& ctl,
+                           cudaStream_t stream) {
+  const int fit = max_clusters<D, GT, PAGED>(cs);
+  if (fit < 1 || !prepare_cluster<D, GT, PAGED>()) return cudaErrorInvalidConfiguration;
+  CUtensorMap tk, tv;
+  PagedView view;
+  if (!kv_views<D, PAGED>(a, pk, &tk, &tv, &view)) return cudaErrorInvalidValue;
+  const int G = a.Hq / a.Hkv;
+  const int n_groups = (G + GT - 1) / GT;
+  const long long units = static_cast<long long>(a.B) * a.Hkv * n_groups;
+  const long long n_clusters = units < fit ? units : fit;
   cudaLaunchAttribute attr[1];
   const cudaLaunchConfig_t cfg =
-      split_config<D, GT, FUSED>(dim3(a.splits, a.Hkv * n_groups, a.B), a.splits, stream, attr);
-  return cudaLaunchKernelEx(&cfg, decode_split_kernel<D, GT, PAGED, FUSED>, static_cast<const __nv_bfloat16*>(a.q),
+      launch_config(dim3(static_cast<unsigned>(n_clusters * cs)), ClusterSmem<D, GT>::BYTES, cs, stream, attr);
+  return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<D, GT, PAGED>, static_cast<const __nv_bfloat16*>(a.q),
                             static_cast<const __nv_bfloat16*>(a.k), static_cast<const __nv_bfloat16*>(a.v),
-                            a.seqlens, a.o_part, a.lse_part, a.Hq, a.Hkv, a.Skv, a.splits, n_groups,
-                            a.scale * kLog2e, ctl, tk, tv, view, static_cast<__nv_bfloat16*>(a.o), a.lse);
+                            a.seqlens, static_cast<__nv_bfloat16*>(a.o), a.lse, a.B, a.Hq, a.Hkv, a.Skv, a.splits,
+                            n_groups, a.scale * kLog2e, ctl, tk, tv, view);
 }
 
 template <int D>
@@ -713,25 +1019,30 @@ cudaError_t launch_merge(const DecodeArgs& a, cudaStream_t stream) {
                             static_cast<__nv_bfloat16*>(a.o), a.lse, a.splits);
 }
 
-// Which form runs: the cluster form when it is forced (a.fused = 1) or the model prefers
-// it (a.fused = 0), provided the split count is a cluster size and such clusters fit.
+// The Flash Decode form of a launch: 0 = split + merge kernels, cs > 0 = the cluster kernel
+// with clusters of cs CTAs.  a.fused = -1 forbids the cluster form; a.fused = 1 takes it
+// with the model's cluster size whenever some cluster size runs; a.fused = 0 lets the model
+// decide (Eq. 9 over both forms at the call's split count); a.cluster > 0 pins the size
+// (when it divides the split count and such clusters fit).
 template <int D, int GT, bool PAGED>
-bool use_cluster_form(const DecodeArgs& a) {
-  if (a.fused < 0 || a.splits > model::kMaxFusedSplits) return false;
-  const int slots = cluster_slots<D, GT, PAGED>(a.splits);
-  if (slots < a.splits) return false;
-  if (a.fused == 1) return true;
+int decode_form(const DecodeArgs& a) {
+  if (a.fused < 0) return 0;
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
                                                 cudaSuccess)
-    return false;
-  return model::decode_fused_wins(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms, slots);
+    return 0;
+  const model::DecodeClusterChoice ch = model::choose_decode_cluster(
+      a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, [](int cs) { return max_clusters<D, GT, PAGED>(cs); }, a.cluster);
+  if (ch.cs == 0) return 0;
+  if (a.fused == 1) return ch.cs;
+  return ch.t_us < model::decode_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms) * (1.0 - 1e-9) ? ch.cs : 0;
 }
 
 template <int D, int GT, bool PAGED>
 cudaError_t launch_form(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
-  if (use_cluster_form<D, GT, PAGED>(a)) return launch_split<D, GT, PAGED, true>(a, pk, ctl, stream);
-  const cudaError_t e = launch_split<D, GT, PAGED, false>(a, pk, ctl, stream);
+  const int cs = decode_form<D, GT, PAGED>(a);
+  if (cs > 0) return launch_cluster<D, GT, PAGED>(a, cs, pk, ctl, stream);
+  const cudaError_t e = launch_split<D, GT, PAGED>(a, pk, ctl, stream);
   if (e != cudaSuccess) return e;
   return launch_merge<D>(a, stream);
 }
@@ -746,20 +1057,20 @@ cudaError_t launch_decode_d(const DecodeArgs& a, const PagedKV* pk, const Kernel
 }
 
 template <int D, bool PAGED>
-bool cluster_form_d(const DecodeArgs& a) {
+int decode_form_d(const DecodeArgs& a) {
   const int G = a.Hq / a.Hkv;
-  if (G >= 8) return use_cluster_form<D, 8, PAGED>(a);
-  if (G >= 4) return use_cluster_form<D, 4, PAGED>(a);
-  if (G >= 2) return use_cluster_form<D, 2, PAGED>(a);
-  return use_cluster_form<D, 1, PAGED>(a);
+  if (G >= 8) return decode_form<D, 8, PAGED>(a);
+  if (G >= 4) return decode_form<D, 4, PAGED>(a);
+  if (G >= 2) return decode_form<D, 2, PAGED>(a);
+  return decode_form<D, 1, PAGED>(a);
 }
 
 template <int D>
-int cluster_slots_d(int G, int splits) {
-  if (G >= 8) return cluster_slots<D, 8, false>(splits);
-  if (G >= 4) return cluster_slots<D, 4, false>(splits);
-  if (G >= 2) return cluster_slots<D, 2, false>(splits);
-  return cluster_slots<D, 1, false>(splits);
+int max_clusters_d(int G, int cs) {
+  if (G >= 8) return max_clusters<D, 8, false>(cs);
+  if (G >= 4) return max_clusters<D, 4, false>(cs);
+  if (G >= 2) return max_clusters<D, 2, false>(cs);
+  return max_clusters<D, 1, false>(cs);
 }
 
 }  // namespace
@@ -777,13 +1088,11 @@ cudaError_t launch_decode_paged(const DecodeArgs& a, const PagedKV& pk, const Ke
   return launch_decode_d<64, true>(a, &pk, ctl, stream);
 }
 
-bool decode_cluster_form(const DecodeArgs& a, bool paged) {
-  if (a.D == 128) return paged ? cluster_form_d<128, true>(a) : cluster_form_d<128, false>(a);
-  return paged ? cluster_form_d<64, true>(a) : cluster_form_d<64, false>(a);
+int decode_cluster_form(const DecodeArgs& a, bool paged) {
+  if (a.D == 128) return paged ? decode_form_d<128, true>(a) : decode_form_d<128, false>(a);
+  return paged ? decode_form_d<64, true>(a) : decode_form_d<64, false>(a);
 }
 
-int decode_cluster_slots(int D, int G, int splits) {
-  return D == 128 ? cluster_slots_d<128>(G, splits) : cluster_slots_d<64>(G, splits);
-}
+int decode_max_clusters(int D, int G, int cs) { return D == 128 ? max_clusters_d<128>(G, cs) : max_clusters_d<64>(G, cs); }
 
 }  // namespace loom

@@ -46,7 +46,8 @@ struct DecodeArgs {
   float* lse_part;          // [B, Hq, splits] fp32 (workspace)
   int B, Hq, Hkv, Skv, D, splits;
   float scale;
-  int fused;  // 0: the model's form; 1: the cluster form wherever it can run; -1: split + merge kernels
+  int fused;    // 0: the model's form; 1: the cluster form wherever it can run; -1: split + merge kernels
+  int cluster;  // cluster form: 0 = the model's cluster size, else this size (if it divides splits and fits)
 };
 
 struct FwdArgs {
@@ -75,11 +76,12 @@ int decode_check_args(const void* q, const void* k_cache, const void* v_cache, c
                       int num_splits, int* splits);
 
 cudaError_t launch_decode(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream);
-// Whether a decode launch with these arguments runs the single-kernel cluster form.
-bool decode_cluster_form(const DecodeArgs& a, bool paged);
-// CTA slots of the cluster form with clusters of `splits` CTAs (G query heads per kv head)
-// on the current device; 0 if such clusters cannot run or the device cannot be asked.
-int decode_cluster_slots(int D, int G, int splits);
+// The form a decode launch with these arguments runs: 0 = split + merge kernels, cs > 0 =
+// the single-kernel cluster form with clusters of cs CTAs.
+int decode_cluster_form(const DecodeArgs& a, bool paged);
+// Clusters of cs cluster-decode CTAs (G query heads per kv head) resident at once on the
+// current device; 0 if none fit or the device cannot be asked.
+int decode_max_clusters(int D, int G, int cs);
 cudaError_t launch_fwd(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream);
 
 }  // namespace loom

@@ -28,7 +28,8 @@ int g_prefill_design = 0;
 int g_gemm_tile_n = 0;  // test hook: forced GEMM tile width (0: the model's choice)
 int g_gemm_splits = 0;  // test hook: forced GEMM split count (0: the model's choice)
 int g_gemm_pair = 0;    // test hook: 1 forces CTA-pair tiles, -1 forbids them, 0: the model's choice
-int g_decode_fused = 0;  // test hook: 1 forces the cluster decode form, -1 forbids it, 0: the model's choice
+int g_decode_fused = 0;    // test hook: 1 forces the cluster decode form, -1 forbids it, 0: the model's choice
+int g_decode_cluster = 0;  // test hook: the cluster decode form's cluster size (0: the model's)
 
 constexpr int kMaxDevices = 64;
 uint32_t* g_err_ptr[kMaxDevices] = {};
@@ -130,9 +131,8 @@ int loom_attn_decode_num_splits(int B, int Hq, int Hkv, int Skv, int D) {
   // device, or from the GB300 estimate when no device answers.
   const bool device = current_sm_count() > 0;
   const int G = Hq / Hkv;
-  const int splits = model::choose_decode_plan(B, Hq, Hkv, Skv, D, sms, [&](int s) {
-                       return device ? decode_cluster_slots(D, G, s)
-                                     : model::decode_default_cluster_slots(sms, s, D);
+  const int splits = model::choose_decode_plan(B, Hq, Hkv, Skv, D, sms, [&](int cs) {
+                       return device ? decode_max_clusters(D, G, cs) : model::decode_default_clusters(sms, cs, D);
                      }).splits;
   std::lock_guard<std::mutex> lock(g_split_mutex);
   if (g_split_cache.size() >= 256) g_split_cache.erase(g_split_cache.begin());
@@ -196,7 +196,7 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D,
-               num_splits, scale, g_decode_fused};
+               num_splits, scale, g_decode_fused, g_decode_cluster};
   return launch_decode(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                  : LOOM_ERR_CUDA;
 }
@@ -266,7 +266,7 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D, num_splits, scale,
-               g_decode_fused};
+               g_decode_fused, g_decode_cluster};
   PagedKV pk{block_table, num_pages, page_size, max_pages, kv_layout};
   return launch_decode_paged(a, pk, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                           : LOOM_ERR_CUDA;
@@ -428,29 +428,34 @@ int loom_attn_decode_cluster_form(int B, int Hq, int Hkv, int Skv, int D, int nu
   a.D = D;
   a.splits = num_splits;
   a.fused = g_decode_fused;
-  const bool c = decode_cluster_form(a, paged != 0);
+  a.cluster = g_decode_cluster;
+  const int cs = decode_cluster_form(a, paged != 0);
   cudaGetLastError();
-  return c ? 1 : 0;
+  return cs;
 }
 
-double loom_model_decode_fused_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int slots) {
-  if (splits <= 0 || B <= 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv || Skv <= 0 || slots <= 0 ||
+double loom_model_decode_cluster_time_us(int splits, int cluster, int B, int Hq, int Hkv, int Skv, int D,
+                                         int clusters) {
+  if (splits <= 0 || B <= 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv || Skv <= 0 || clusters <= 0 ||
       (D != 64 && D != 128))
     return -1.0;
-  const double t = model::decode_fused_time_us(splits, B, Hq, Hkv, Skv, D, slots);
+  const double t = model::decode_cluster_time_us(splits, cluster, B, Hq, Hkv, Skv, D, clusters);
   return t > 1e299 ? -1.0 : t;
 }
 
-int loom_decode_cluster_slots(int D, int G, int splits) {
-  if ((D != 64 && D != 128) || G <= 0 || splits <= 0) return 0;
+int loom_decode_max_clusters(int D, int G, int cluster) {
+  if ((D != 64 && D != 128) || G <= 0 || cluster <= 0 || cluster > model::kMaxClusterSize) return 0;
   const int sms = current_sm_count();
-  if (sms <= 0) return model::decode_default_cluster_slots(model::kGb300.num_sms, splits, D);
-  const int s = decode_cluster_slots(D, G, splits);
+  if (sms <= 0) return model::decode_default_clusters(model::kGb300.num_sms, cluster, D);
+  const int n = decode_max_clusters(D, G, cluster);
   cudaGetLastError();
-  return s;
+  return n;
 }
 
-void loom_debug_decode_cluster(int mode) { g_decode_fused = (mode == 1 || mode == -1) ? mode : 0; }
+void loom_debug_decode_cluster(int mode, int cluster) {
+  g_decode_fused = (mode == 1 || mode == -1) ? mode : 0;
+  g_decode_cluster = (cluster >= 1 && cluster <= model::kMaxClusterSize) ? cluster : 0;
+}
 
 void loom_debug_set_timeout_ns(uint64_t ns) { g_timeout_ns = ns ? ns : kDefaultTimeoutNs; }
 

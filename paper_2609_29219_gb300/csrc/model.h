@@ -45,14 +45,14 @@ struct ArchDesc {
   double mma_issue_busy_factor;     // MMA stream slowdown while high-ILP warps share the SM with
                                     // the MMA warp issuing warp-wide (measured: 546 vs 512 clk
                                     // per 128^3 GEMM; 1338 when a lone lane issues)
-  double cluster_merge_ns;          // gather of a decode cluster's partials over DSMEM: two
-                                    // cluster barriers and the reads (assumed)
+  double cluster_merge_ns;          // per unit of the cluster decode: the warps' merge, the
+                                    // cluster handshakes and the DSMEM gather (assumed)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 1000.0,
+    129.0e6, 1.07, 500.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -305,13 +305,13 @@ constexpr const DecodeStagePlan& decode_stage(int D) { return D == 64 ? kDecodeS
 
 struct DecodeSplitPlan {
   int splits;
-  double t_us;   // modeled split + merge time
-  bool fused;    // the splits of a unit run as one cluster and merge over DSMEM
+  double t_us;  // modeled time of the chosen form
+  int cluster;  // 0: split kernel + merge kernel; cs > 0: the cluster kernel, clusters of cs CTAs
 };
 
-// Largest split count of the single-kernel (cluster) Flash Decode: a unit's splits form one
-// thread-block cluster, and 16 CTAs is the largest (non-portable) cluster size.
-constexpr int kMaxFusedSplits = 16;
+// Largest cluster of the single-kernel (cluster) Flash Decode: 16 CTAs, the largest
+// (non-portable) thread-block cluster.
+constexpr int kMaxClusterSize = 16;
 
 // Number of q heads one split CTA serves (must match the kernel dispatch).
 constexpr int decode_group_tile(int G) { return G >= 8 ? 8 : G >= 4 ? 4 : G >= 2 ? 2 : 1; }
@@ -319,10 +319,9 @@ constexpr int decode_group_tile(int G) { return G >= 8 ? 8 : G >= 4 ? 4 : G >= 2
 // The split loop of Flash Decode (Eq. 6-7 with an open load boundary), evaluated on the
 // busiest SM: it runs ceil(CTAs / SMs) split CTAs in rounds of at most CTAs-per-SM at a
 // time; a round of k CTAs streams at min(the SM's share of HBM / k, the rate one CTA
-// sustains), and each round pays the CTA start-up (launch and first copies) and `round_ns`
-// more.  `sms` may be fractional: SM-equivalents of CTA slots.
-constexpr double decode_split_loop_ns(int splits, int B, int Hq, int Hkv, int Skv, int D, double sms,
-                                      double round_ns, const ArchDesc& a) {
+// sustains), and each round pays the CTA start-up (launch and first copies).
+constexpr double decode_split_loop_ns(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms,
+                                      const ArchDesc& a) {
   const DecodeStagePlan& sp = decode_stage(D);
   const int G = Hq / Hkv;
   const int gt = decode_group_tile(G);
@@ -330,10 +329,8 @@ constexpr double decode_split_loop_ns(int splits, int B, int Hq, int Hkv, int Sk
   const long long ctas = units * splits;
   const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
   const double chunk_bytes = 2.0 * chunk * D * 2;
-  const double per_sm_d = static_cast<double>(ctas) / sms;
-  long long per_sm = static_cast<long long>(per_sm_d);
-  if (static_cast<double>(per_sm) < per_sm_d) ++per_sm;
-  const double active_sms = static_cast<double>(ctas) < sms ? static_cast<double>(ctas) : sms;
+  const long long per_sm = cdiv(ctas, num_sms);
+  const double active_sms = static_cast<double>(ctas < num_sms ? ctas : num_sms);
   const double share = a.hbm_gbs / active_sms;  // bytes/ns for one SM
   double t_split = 0.0;
   for (long long left = per_sm; left > 0;) {
@@ -341,72 +338,94 @@ constexpr double decode_split_loop_ns(int splits, int B, int Hq, int Hkv, int Sk
     left -= k;
     double bw = share / static_cast<double>(k);
     if (bw > a.decode_cta_gbs) bw = a.decode_cta_gbs;
-    t_split += heg_seq(heg_seq(a.cta_start_ns, chunk_bytes / bw), round_ns);
+    t_split += heg_seq(a.cta_start_ns, chunk_bytes / bw);
   }
   return t_split;
 }
 
-// Eq. 5 for Flash Decode: T = T_split-loop ; T_merge (gather + global softmax + scale), the
-// merge a second, dependent launch that reads the partials back.
+// Eq. 5 for Flash Decode in the split + merge form: T = T_split-loop ; T_merge (gather +
+// global softmax + final scaling), the merge a second, dependent launch that reads the
+// partials back.
 constexpr double decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms,
                                 const ArchDesc& a = kGb300) {
-  const double t_split = decode_split_loop_ns(splits, B, Hq, Hkv, Skv, D, num_sms, 0.0, a);
+  const double t_split = decode_split_loop_ns(splits, B, Hq, Hkv, Skv, D, num_sms, a);
   const double part_bytes = 1.0 * B * Hq * splits * (D + 1) * 4;
   const double t_merge = a.launch_ns * 0.2 + 2.0 * part_bytes / a.hbm_gbs;
   return heg_seq(t_split, t_merge) * 1e-3;
 }
 
-// Single-kernel Flash Decode: the `splits` CTAs of one unit form a thread-block cluster and
-// gather, globally softmax and scale their partials over distributed shared memory, so the
-// merge launch and the workspace round trip are gone.  The gather is paid inside every
-// round (two cluster barriers and splits DSMEM reads per output); and a cluster's CTAs are
-// placed together, so only `slots` CTAs (whole clusters per GPC) run at once.
-constexpr double decode_fused_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int slots,
-                                      const ArchDesc& a = kGb300) {
-  if (splits < 1 || splits > kMaxFusedSplits || slots < splits) return 1e300;
-  const double sms = static_cast<double>(slots) / decode_stage(D).ctas_per_sm;
-  return decode_split_loop_ns(splits, B, Hq, Hkv, Skv, D, sms, a.cluster_merge_ns, a) * 1e-3;
+// Eq. 5 for the single-kernel form: persistent clusters of cs CTAs (cs divides the split
+// count); the min(fit_clusters, units) clusters each walk ceil(units / clusters) units, and
+// a CTA streams splits / cs chunks of every unit at min(its share of HBM, the rate one CTA
+// sustains), without a break between units.  Per unit it pays the gather + global softmax +
+// scaling over DSMEM (cluster_merge_ns); the start-up once.  No merge launch, no workspace.
+constexpr double decode_cluster_time_us(int splits, int cs, int B, int Hq, int Hkv, int Skv, int D,
+                                        int fit_clusters, const ArchDesc& a = kGb300) {
+  if (cs < 1 || cs > kMaxClusterSize || splits < cs || splits % cs != 0 || fit_clusters < 1) return 1e300;
+  const int G = Hq / Hkv;
+  const long long units = 1LL * B * Hkv * cdiv(G, decode_group_tile(G));
+  const long long clusters = units < fit_clusters ? units : fit_clusters;
+  const double ctas = static_cast<double>(clusters * cs);
+  const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
+  const double cta_unit_bytes = static_cast<double>(splits / cs) * 2.0 * chunk * D * 2;
+  double rate = a.hbm_gbs / ctas;
+  if (rate > a.decode_cta_gbs) rate = a.decode_cta_gbs;
+  const double per_unit = heg_seq(cta_unit_bytes / rate, a.cluster_merge_ns);
+  return heg_seq(a.cta_start_ns, heg_for(static_cast<double>(cdiv(units, clusters)), per_unit)) * 1e-3;
 }
 
-// CTA slots of clusters of `splits` decode CTAs when no device can be asked: whole clusters
-// in 8 equal SM groups (GPCs) at the stage plan's CTAs per SM.
-constexpr int decode_default_cluster_slots(int num_sms, int splits, int D) {
-  if (splits < 1) return 0;
+// Clusters of cs decode CTAs in one GPC-sized group when no device can be asked: whole
+// clusters in 8 equal groups of SMs at the stage plan's CTAs per SM.
+constexpr int decode_default_clusters(int num_sms, int cs, int D) {
+  if (cs < 1) return 0;
   const int per_gpc = num_sms / 8 * decode_stage(D).ctas_per_sm;
-  return per_gpc / splits * splits * 8;
+  return per_gpc / cs * 8;
 }
 
-// Eq. 9 over both Flash Decode forms: every split count of the two-kernel form and every
-// split count up to kMaxFusedSplits of the cluster form; `slots(s)` gives the CTA slots of
-// clusters of s CTAs (0: that cluster size cannot run).  Ties keep the two-kernel form
-// and the smaller split count.
-template <class Slots>
-constexpr DecodeSplitPlan choose_decode_plan(int B, int Hq, int Hkv, int Skv, int D, int num_sms, Slots slots,
-                                             const ArchDesc& a = kGb300) {
-  DecodeSplitPlan best{1, 1e300, false};
-  const long long max_splits = cdiv(Skv, 64) < 1024 ? cdiv(Skv, 64) : 1024;
-  for (int s = 1; s <= max_splits; ++s) {
-    const double t = decode_time_us(s, B, Hq, Hkv, Skv, D, num_sms, a);
-    if (t < best.t_us * (1.0 - 1e-9)) best = {s, t, false};
-  }
-  for (int s = 1; s <= max_splits && s <= kMaxFusedSplits; ++s) {
-    const double t = decode_fused_time_us(s, B, Hq, Hkv, Skv, D, slots(s), a);
-    if (t < best.t_us * (1.0 - 1e-9)) best = {s, t, true};
+struct DecodeClusterChoice {
+  int cs;       // 0: no cluster size can run
+  double t_us;
+};
+
+// The cluster size of the single-kernel form for a split count: Eq. 9 over the sizes that
+// divide it and fit (fit(cs): clusters of cs CTAs resident at once, 0 if none); forced_cs
+// > 0 admits that size only.  Ties keep the smaller cluster.
+template <class Fit>
+constexpr DecodeClusterChoice choose_decode_cluster(int splits, int B, int Hq, int Hkv, int Skv, int D, Fit fit,
+                                                    int forced_cs = 0, const ArchDesc& a = kGb300) {
+  DecodeClusterChoice best{0, 1e300};
+  for (int cs = 1; cs <= kMaxClusterSize && cs <= splits; ++cs) {
+    if (splits % cs != 0 || (forced_cs > 0 && cs != forced_cs)) continue;
+    const int f = fit(cs);
+    if (f < 1) continue;
+    const double t = decode_cluster_time_us(splits, cs, B, Hq, Hkv, Skv, D, f, a);
+    if (t < best.t_us * (1.0 - 1e-9)) best = {cs, t};
   }
   return best;
 }
 
-// The two-kernel form alone (Eq. 9 over its split counts).
+// Eq. 9 over both Flash Decode forms and every split count; fit(cs) as above (always 0:
+// the split + merge form alone).  Ties keep the split + merge form and fewer splits.
+template <class Fit>
+constexpr DecodeSplitPlan choose_decode_plan(int B, int Hq, int Hkv, int Skv, int D, int num_sms, Fit fit,
+                                             const ArchDesc& a = kGb300) {
+  DecodeSplitPlan best{1, 1e300, 0};
+  const long long max_splits = cdiv(Skv, 64) < 1024 ? cdiv(Skv, 64) : 1024;
+  for (int s = 1; s <= max_splits; ++s) {
+    const double t = decode_time_us(s, B, Hq, Hkv, Skv, D, num_sms, a);
+    if (t < best.t_us * (1.0 - 1e-9)) best = {s, t, 0};
+  }
+  for (int s = 1; s <= max_splits; ++s) {
+    const DecodeClusterChoice c = choose_decode_cluster(s, B, Hq, Hkv, Skv, D, fit, 0, a);
+    if (c.cs > 0 && c.t_us < best.t_us * (1.0 - 1e-9)) best = {s, c.t_us, c.cs};
+  }
+  return best;
+}
+
+// The split + merge form alone (Eq. 9 over its split counts).
 constexpr DecodeSplitPlan choose_decode_splits(int B, int Hq, int Hkv, int Skv, int D, int num_sms,
                                                const ArchDesc& a = kGb300) {
   return choose_decode_plan(B, Hq, Hkv, Skv, D, num_sms, [](int) { return 0; }, a);
-}
-
-// For a given split count: does the cluster form beat the two-kernel form?
-constexpr bool decode_fused_wins(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms, int slots,
-                                 const ArchDesc& a = kGb300) {
-  return decode_fused_time_us(splits, B, Hq, Hkv, Skv, D, slots, a) <
-         decode_time_us(splits, B, Hq, Hkv, Skv, D, num_sms, a) * (1.0 - 1e-9);
 }
 
 }  // namespace model

@@ -1,6 +1,6 @@
 """GPU parity of the Flash Decode kernels through the C ABI, in both forms: split kernel +
-merge kernel, and the single kernel whose splits of a (batch, kv head) form a cluster and
-merge over distributed shared memory (at most 16 splits)."""
+merge kernel, and the single persistent kernel whose clusters of CTAs walk the (batch, kv
+head) pairs and merge their partials over distributed shared memory."""
 import numpy as np
 import pytest
 
@@ -24,8 +24,8 @@ def loom():
 
 @pytest.fixture(autouse=True, params=[0, 1, -1], ids=["model_form", "cluster_form", "split_merge"])
 def form(request, loom):
-    """Every test runs with the model's choice of form, with the cluster form forced
-    wherever it can run (at most 16 splits), and with split + merge kernels forced."""
+    """Every test runs with the model's choice of form, with the cluster form forced (the
+    model's cluster size), and with split + merge kernels forced."""
     loom.loom_debug_decode_cluster(request.param)
     yield request.param
     loom.loom_debug_decode_cluster(0)
@@ -37,7 +37,7 @@ def _expect_form(loom, form, B, Hq, Hkv, Skv, D, splits):
         assert used == 0
     elif form == 1:
         s = splits or loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
-        assert used == (1 if s <= 16 else 0)
+        assert used >= 1 and s % used == 0
 
 
 def _inputs(seed, B, Hq, Hkv, Skv, D):
@@ -67,15 +67,39 @@ def test_batched_decode_config(loom, form):
 
 
 @pytest.mark.slow
-def test_long_context_decode_config(loom):
+def test_long_context_decode_config(loom, form):
     # B=1, Hq=32, Hkv=8, Skv=131072, D=128, model-chosen splits (>= one wave of CTAs)
     B, Hq, Hkv, Skv, D = 1, 32, 8, 131072, 128
+    _expect_form(loom, form, B, Hq, Hkv, Skv, D, 0)
     q, k, v = _inputs(0, B, Hq, Hkv, Skv, D)
     splits = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
     assert splits * Hkv >= 148
     o, lse = _run(loom, q, k, v, None, 0)
     o_ref, lse_ref = oracle.attention(q, k, v)
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "long decode")
+
+
+@pytest.mark.parametrize("splits,clusters", [(16, (1, 2, 4, 8, 16)), (12, (3, 6, 12)), (5, (5,)), (38, (2, 19))])
+def test_every_cluster_size(loom, form, splits, clusters):
+    """The cluster form with each cluster size pinned (CTA r takes splits r, r + cs, ...):
+    sequences of 0 .. Skv keys over a batch that leaves clusters several units each."""
+    import torch
+    if form != 1:
+        pytest.skip("cluster sizes are pinned under the forced cluster form")
+    B, Hq, Hkv, Skv, D = 9, 16, 4, 4000, 128
+    q, k, v = _inputs(splits, B, Hq, Hkv, Skv, D)
+    lens = np.array([4000, 0, 1, 63, 65, 1000, 3999, 2048, 777], np.int32)
+    o_ref, lse_ref = oracle.attention(q, k, v, seqlens_k=lens)
+    for cs in clusters:
+        loom.loom_debug_decode_cluster(1, cs)
+        used = loom.loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, splits)
+        if splits % cs == 0 and cs <= 16:
+            assert used == cs
+        else:
+            assert used != cs
+        o, lse = _run(loom, q, k, v, lens, splits)
+        assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"splits={splits} cluster={cs}")
+    loom.loom_debug_decode_cluster(1, 0)
 
 
 @pytest.mark.parametrize("D", [64, 128])

@@ -66,9 +66,10 @@ def test_decode_skipped_stage_times_out_and_context_survives(loom):
 
 @pytest.mark.parametrize("lens,splits", [(2048, 2), (160, 2), (2048, 16)], ids=["both_abort", "one_aborts", "c16"])
 def test_cluster_decode_skipped_stage_times_out_and_context_survives(loom, lens, splits):
-    """The single-kernel cluster form: every CTA whose chunk has a second stage gives up on
-    it and unwinds; all CTAs (those that gave up and those that finished) still meet at the
-    cluster barriers, so the launch ends and the next call is correct."""
+    """The single-kernel cluster form (one cluster of `splits` CTAs): every CTA with a
+    second stage gives up on it and unwinds; its peers give up on the partial it never
+    signals; all CTAs still meet at the final cluster barrier, so the launch ends and the
+    next call is correct."""
     import torch
     B, Hq, Hkv, Skv, D = 1, 4, 1, 2048, 128
     q = synth.bf16_normal(37, synth.STREAM_Q, (B, Hq, 1, D))
@@ -77,9 +78,9 @@ def test_cluster_decode_skipped_stage_times_out_and_context_survives(loom, lens,
     qd, kd, vd = to_dev(q), to_dev(k), to_dev(v)
     sl_h = np.array([lens], np.int32)
     sl = torch.from_numpy(sl_h).cuda()
-    loom.loom_debug_decode_cluster(1)
+    loom.loom_debug_decode_cluster(1, splits)
     try:
-        assert loom.loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, splits) == 1
+        assert loom.loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, splits) == splits
 
         def bad():
             loom.loom_debug_inject(1)

@@ -28,8 +28,8 @@ def loom():
 
 @pytest.fixture(autouse=True, params=[1, -1], ids=["cluster_form", "split_merge"])
 def form(request, loom):
-    """Every test runs with the single-kernel cluster form forced wherever it can run (at
-    most 16 splits) and with split + merge kernels forced."""
+    """Every test runs with the single-kernel cluster form forced (the model's cluster size)
+    and with split + merge kernels forced."""
     loom.loom_debug_decode_cluster(request.param)
     yield request.param
     loom.loom_debug_decode_cluster(0)
@@ -146,8 +146,8 @@ def test_batched_serving_shape(loom, form, P, layout):
     lens = synth.decode_lengths(0, B, 4096, 8192)
     q, kc, vc, table, sl = paged_case(0, B, Hq, Hkv, P, lens, D, spare=0, poison=False)
     o, lse = run_paged(loom, q, kc, vc, table, sl, 16, layout)
-    assert loom.loom_attn_decode_cluster_form(B, Hq, Hkv, table.shape[1] * P, D, 16, paged=True) == \
-        (1 if form == 1 else 0)
+    assert (loom.loom_attn_decode_cluster_form(B, Hq, Hkv, table.shape[1] * P, D, 16, paged=True) > 0) == \
+        (form == 1)
     o_ref, lse_ref = oracle.decode_paged(q, kc, vc, table, sl, page_size=P)
     assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"batched paged P={P} {layout}")
 

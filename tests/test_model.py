@@ -104,14 +104,18 @@ DECODE_SHAPES = [(16, 32, 8, 8192, 128), (1, 32, 8, 131072, 128), (1, 8, 8, 4096
 
 def _decode_candidates(loom, B, Hq, Hkv, Skv, D):
     """Modeled time of every (form, split count) candidate: the two-kernel form for every
-    split count, the cluster form for split counts up to 16 with the slots it is priced at."""
+    split count, the cluster form for every split count and cluster size dividing it, with
+    the clusters it is priced at."""
     cands = []
+    G = Hq // Hkv
     for s in range(1, min(1024, math.ceil(Skv / 64)) + 1):
         cands.append((loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS), 0, s))
-    for s in range(1, min(16, math.ceil(Skv / 64)) + 1):
-        t = loom.loom_model_decode_fused_time_us(s, B, Hq, Hkv, Skv, D, loom.loom_decode_cluster_slots(D, Hq // Hkv, s))
-        if t > 0:
-            cands.append((t, 1, s))
+        for cs in range(1, min(16, s) + 1):
+            if s % cs:
+                continue
+            t = loom.loom_model_decode_cluster_time_us(s, cs, B, Hq, Hkv, Skv, D, loom.loom_decode_max_clusters(D, G, cs))
+            if t > 0:
+                cands.append((t, cs, s))
     return cands
 
 
@@ -121,22 +125,21 @@ def test_decode_split_is_brute_force_argmin(loom, B, Hq, Hkv, Skv, D):
     chosen = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
     cands = _decode_candidates(loom, B, Hq, Hkv, Skv, D)
     best = min(t for t, _, _ in cands)
-    winners = sorted((f, s) for t, f, s in cands if t <= best * (1 + 1e-9))
-    assert winners[0][1] == chosen                # ties: the two-kernel form, then the fewest splits
-    form = loom.loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, 0)
-    assert form == winners[0][0]
+    winners = [(f > 0, s, f) for t, f, s in cands if t <= best * (1 + 1e-9)]
+    assert min(winners)[1] == chosen              # ties: the two-kernel form, then the fewest splits
 
 
 def test_cluster_form_limits(loom):
     B, Hq, Hkv, Skv, D = 16, 32, 8, 8192, 128
-    slots = loom.loom_decode_cluster_slots(D, 4, 16)
-    assert slots > 0 and slots % 16 == 0
-    assert loom.loom_model_decode_fused_time_us(17, B, Hq, Hkv, Skv, D, 10 ** 6) < 0   # > 16 CTAs per cluster
-    assert loom.loom_model_decode_fused_time_us(16, B, Hq, Hkv, Skv, D, 15) < 0       # no whole cluster fits
-    # fewer slots never make it faster; the HBM roof bounds it
-    t = [loom.loom_model_decode_fused_time_us(16, B, Hq, Hkv, Skv, D, n) for n in (64, 128, 256, 304)]
-    assert all(a >= b * (1 - 1e-9) for a, b in zip(t, t[1:]))
-    assert t[-1] * 1e-6 >= 2.0 * B * Hkv * Skv * D * 2 / (PEAK_GBS * 1e9) * 0.999
+    assert loom.loom_decode_max_clusters(D, 4, 16) > 0
+    t = lambda s, cs, n: loom.loom_model_decode_cluster_time_us(s, cs, B, Hq, Hkv, Skv, D, n)
+    assert t(32, 17, 100) < 0      # more than 16 CTAs per cluster
+    assert t(16, 3, 100) < 0       # the cluster size must divide the split count
+    assert t(16, 16, 0) < 0        # no cluster fits
+    # more resident clusters never make it slower; the HBM roof bounds it
+    ts = [t(16, 16, n) for n in (1, 2, 4, 8, 14, 32)]
+    assert all(a >= b * (1 - 1e-9) for a, b in zip(ts, ts[1:]))
+    assert ts[-1] * 1e-6 >= 2.0 * B * Hkv * Skv * D * 2 / (PEAK_GBS * 1e9) * 0.999
 
 
 def test_long_decode_fills_one_wave(loom):
@@ -148,9 +151,7 @@ def test_long_decode_fills_one_wave(loom):
 @pytest.mark.parametrize("B,Hq,Hkv,Skv,D", DECODE_SHAPES)
 def test_decode_time_not_below_hbm_roofline(loom, B, Hq, Hkv, Skv, D):
     s = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
-    t = min(loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS),
-            loom.loom_model_decode_fused_time_us(s, B, Hq, Hkv, Skv, D, loom.loom_decode_cluster_slots(D, Hq // Hkv, s))
-            if s <= 16 else 1e30)
+    t = min(t for t, _, n in _decode_candidates(loom, B, Hq, Hkv, Skv, D) if n == s)
     kv_bytes = 2.0 * B * Hkv * Skv * D * 2
     assert t * 1e-6 >= kv_bytes / (PEAK_GBS * 1e9) * 0.999
 
