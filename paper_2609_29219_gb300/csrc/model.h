@@ -45,14 +45,16 @@ struct ArchDesc {
   double mma_issue_busy_factor;     // MMA stream slowdown while high-ILP warps share the SM with
                                     // the MMA warp issuing warp-wide (measured: 546 vs 512 clk
                                     // per 128^3 GEMM; 1338 when a lone lane issues)
-  double cluster_merge_ns;          // per unit of the cluster decode: the warps' merge, the
-                                    // cluster handshakes and the DSMEM gather (assumed)
+  double cluster_merge_ns;          // per unit and CTA of a cluster-decode cluster: the warps'
+                                    // merge, the handshakes waiting on the slowest CTA and the
+                                    // DSMEM gather (fitted: 147 / 103 / 93 us measured with
+                                    // clusters of 16 / 8 / 2 on the batched decode)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 500.0,
+    129.0e6, 1.07, 300.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -358,7 +360,9 @@ constexpr double decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int
 // count); the min(fit_clusters, units) clusters each walk ceil(units / clusters) units, and
 // a CTA streams splits / cs chunks of every unit at min(its share of HBM, the rate one CTA
 // sustains), without a break between units.  Per unit it pays the gather + global softmax +
-// scaling over DSMEM (cluster_merge_ns); the start-up once.  No merge launch, no workspace.
+// scaling over DSMEM and the handshakes, which wait for the slowest of the cluster's CTAs
+// (cluster_merge_ns per CTA of the cluster); the start-up once.  No merge launch, no
+// workspace.
 constexpr double decode_cluster_time_us(int splits, int cs, int B, int Hq, int Hkv, int Skv, int D,
                                         int fit_clusters, const ArchDesc& a = kGb300) {
   if (cs < 1 || cs > kMaxClusterSize || splits < cs || splits % cs != 0 || fit_clusters < 1) return 1e300;
@@ -370,7 +374,7 @@ constexpr double decode_cluster_time_us(int splits, int cs, int B, int Hq, int H
   const double cta_unit_bytes = static_cast<double>(splits / cs) * 2.0 * chunk * D * 2;
   double rate = a.hbm_gbs / ctas;
   if (rate > a.decode_cta_gbs) rate = a.decode_cta_gbs;
-  const double per_unit = heg_seq(cta_unit_bytes / rate, a.cluster_merge_ns);
+  const double per_unit = heg_seq(cta_unit_bytes / rate, a.cluster_merge_ns * cs);
   return heg_seq(a.cta_start_ns, heg_for(static_cast<double>(cdiv(units, clusters)), per_unit)) * 1e-3;
 }
 
