@@ -314,6 +314,26 @@ void loom_debug_inject(int mode);
 void loom_debug_prefill_design(int design);
 
 /*
+ * Block-size ablation hooks (the paper's block-size ablation, Sec. 3 "Ablation Studies":
+ * the neighbourhood of the solver's choice, measured).  Each pins a compiled neighbour of
+ * the analytic model's constant and returns 1, or returns 0 (and restores the model's
+ * constant) when that value is not compiled:
+ * loom_debug_prefill_slots: the two-tile prefill's K/V ring depth for head dimension D
+ *   (compiled beside the model's 3 at D = 128: 2; beside 10 at D = 64: 3, 6, 9; deeper
+ *   rings do not fit in shared memory).  0 restores the model's.
+ * loom_debug_decode_stage_plan: the decode split kernel's keys per stage, ring stages and
+ *   CTAs per SM (contiguous cache, D = 128, 4 query heads per kv head, split + merge form;
+ *   compiled: 32x2x2, 32x3x2, 32x4x2, 64x2x2, 64x4x1, 128x2x1, 128x3x1 beside the model's
+ *   64x3x2).  tokens = 0 restores the model's.
+ * loom_debug_gemm_stages: the GEMM's K-stage ring depth ([K, N] B): the CTA pair with 5
+ *   (model: 6), 256-wide persistent tiles with 3 (model: 4), 128-wide with 5 (model: 6);
+ *   other values or kernels run the model's depth.  0 restores the model's.
+ */
+int loom_debug_prefill_slots(int D, int slots);
+int loom_debug_decode_stage_plan(int tokens, int stages, int ctas_per_sm);
+void loom_debug_gemm_stages(int stages);
+
+/*
  * Test hook: the Flash Decode form.  mode 1 = the single-kernel cluster form wherever some
  * cluster size runs; -1 = always split + merge kernels; anything else: the analytic model's
  * choice (default).  cluster in 1..16 pins the cluster form's cluster size (honoured when

@@ -29,6 +29,7 @@ __all__ = [
     "loom_attn_decode_paged", "loom_attn_fwd_varlen", "loom_gemm_bf16", "loom_gemm_bf16_bt", "loom_gemm_tile_n", "loom_gemm_splits", "loom_gemm_cta_pair", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
     "loom_debug_gemm_splits", "loom_debug_gemm_cta_pair", "loom_model_decode_cluster_time_us",
     "loom_attn_decode_cluster_form", "loom_decode_max_clusters", "loom_debug_decode_cluster",
+    "loom_debug_prefill_slots", "loom_debug_decode_stage_plan", "loom_debug_gemm_stages",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -139,6 +140,12 @@ def capi() -> ctypes.CDLL:
             lib.loom_decode_max_clusters.restype = i32
             lib.loom_debug_decode_cluster.argtypes = [i32, i32]
             lib.loom_debug_decode_cluster.restype = None
+            lib.loom_debug_prefill_slots.argtypes = [i32, i32]
+            lib.loom_debug_prefill_slots.restype = i32
+            lib.loom_debug_decode_stage_plan.argtypes = [i32, i32, i32]
+            lib.loom_debug_decode_stage_plan.restype = i32
+            lib.loom_debug_gemm_stages.argtypes = [i32]
+            lib.loom_debug_gemm_stages.restype = None
             _lib = lib
     return _lib
 
@@ -502,3 +509,18 @@ def loom_decode_max_clusters(D, G, cluster) -> int:
 
 def loom_debug_decode_cluster(mode: int, cluster: int = 0) -> None:
     capi().loom_debug_decode_cluster(int(mode), int(cluster))
+
+
+def loom_debug_prefill_slots(D: int, slots: int) -> bool:
+    """Pin the two-tile prefill's K/V ring depth (0: the model's); False if not compiled."""
+    return bool(capi().loom_debug_prefill_slots(int(D), int(slots)))
+
+
+def loom_debug_decode_stage_plan(tokens: int, stages: int = 0, ctas_per_sm: int = 0) -> bool:
+    """Pin the decode split kernel's stage plan (tokens 0: the model's); False if not compiled."""
+    return bool(capi().loom_debug_decode_stage_plan(int(tokens), int(stages), int(ctas_per_sm)))
+
+
+def loom_debug_gemm_stages(stages: int) -> None:
+    """Pin the GEMM's K-stage ring depth where a neighbour is compiled (0: the model's)."""
+    capi().loom_debug_gemm_stages(int(stages))

@@ -60,14 +60,16 @@ constexpr float kLn2 = 0.6931471805599453f;
 // exceeds it by more than this many base-2 units; P stays <= 2^8, exact in fp32.
 constexpr float kRescaleThreshold = 8.0f;
 
-// Stage constants: the analytic model's choice for this head dimension.
-template <int D>
+// Stage constants: the analytic model's choice for this head dimension.  Non-zero T_,
+// NSTAGE_, CTAS_ override it (the neighbours measured by the block-size ablation).
+template <int D, int T_ = 0, int NSTAGE_ = 0, int CTAS_ = 0>
 struct DecodeCfg {
   static constexpr model::DecodeStagePlan kPlan = model::decode_stage_plan(D);
   static_assert(kPlan.feasible, "no feasible decode stage plan");
-  static constexpr int T = kPlan.tokens;           // tokens per stage
-  static constexpr int NSTAGE = kPlan.stages;
-  static constexpr int CTAS_PER_SM = kPlan.ctas_per_sm;
+  static constexpr int DIM = D;
+  static constexpr int T = T_ ? T_ : kPlan.tokens;  // tokens per stage
+  static constexpr int NSTAGE = NSTAGE_ ? NSTAGE_ : kPlan.stages;
+  static constexpr int CTAS_PER_SM = CTAS_ ? CTAS_ : kPlan.ctas_per_sm;
   static constexpr int NCW = 8;                    // compute warps
   static constexpr int THREADS = (NCW + 1) * 32;   // + loader warp
   static constexpr int TW = T / NCW;               // tokens per warp per stage
@@ -81,9 +83,8 @@ struct DecodeCfg {
   static_assert(TW % TPR == 0, "whole 128-bit load rounds per warp");
 };
 
-template <int D, int GT>
+template <class C, int GT>
 struct DecodeSmem {
-  using C = DecodeCfg<D>;
   // ring first (16-byte aligned bulk-copy destinations), then the small arrays
   static constexpr uint32_t P_OFF = C::RING_BYTES;                      // [NCW][TW][GT] f32
   static constexpr uint32_t ALPHA_OFF = P_OFF + C::NCW * C::TW * GT * 4;  // [NCW][GT] f32
@@ -93,7 +94,7 @@ struct DecodeSmem {
   static constexpr uint32_t ABORT_OFF = BAR_OFF + 2 * C::NSTAGE * 8;
   static constexpr uint32_t BYTES = ABORT_OFF + 16;
   // the cross-warp merge reuses the ring: [NCW][GT][D] f32
-  static_assert(C::NCW * GT * D * 4 <= C::RING_BYTES, "merge buffer must fit in the ring");
+  static_assert(C::NCW * GT * C::DIM * 4 <= C::RING_BYTES, "merge buffer must fit in the ring");
 };
 
 // Sum over the KL lanes of a K row of the GT per-head partial dot products.  Each
@@ -177,12 +178,12 @@ __device__ __forceinline__ void load_q(const __nv_bfloat16* q_rows, int nh, int 
 // keys): the scores of its TW tokens for the GT heads (base 2), the online softmax per
 // head with a lazily moved running max (m_run, l_run), and P.V into acc_o.  ps and alpha_s
 // are this warp's shared-memory P [TW][GT] and rescale factors [GT].
-template <int D, int GT>
+template <class C, int GT>
 __device__ __forceinline__ void decode_stage(const uint8_t* ks, const uint8_t* vs, int ntok, int warp, int lane,
-                                             const LaneRole<D, GT>& lr, const float (&qf)[GT][8], float& m_run,
-                                             float& l_run, float (&acc_o)[GT][DecodeCfg<D>::VD], float* ps,
+                                             const LaneRole<C::DIM, GT>& lr, const float (&qf)[GT][8],
+                                             float& m_run, float& l_run, float (&acc_o)[GT][C::VD], float* ps,
                                              float* alpha_s) {
-  using C = DecodeCfg<D>;
+  constexpr int D = C::DIM;
   // scores of this warp's TW tokens, in base-2 units
   float sc[C::KROUNDS];
 #pragma unroll
@@ -365,16 +366,16 @@ struct PagedLoader {
   }
 };
 
-template <int D, int GT, bool PAGED>
-__global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_SM)
+template <int D, int GT, bool PAGED, class C = DecodeCfg<D>>
+__global__ void __launch_bounds__(C::THREADS, C::CTAS_PER_SM)
     decode_split_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
                         const __nv_bfloat16* __restrict__ v, const int32_t* __restrict__ seqlens,
                         float* __restrict__ o_part, float* __restrict__ lse_part, int Hq, int Hkv,
                         int Skv, int splits, int n_groups, float c, KernelCtl ctl,
                         const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                         PagedView pv) {
-  using C = DecodeCfg<D>;
-  using L = DecodeSmem<D, GT>;
+  static_assert(C::DIM == D, "configuration of this head dimension");
+  using L = DecodeSmem<C, GT>;
   extern __shared__ __align__(128) uint8_t smem[];
 
   // Let the merge grid launch as soon as every split CTA is resident.
@@ -494,7 +495,7 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
     const int slot = it % C::NSTAGE;
     if (!mbar_wait_warp(bar_full + 8 * slot, (it / C::NSTAGE) & 1, ctl, ab)) break;
     const uint8_t* ks = smem + slot * C::STAGE_BYTES;
-    decode_stage<D, GT>(ks, ks + C::TILE_BYTES, min(C::T, t_end - (t_begin + it * C::T)), warp, lane, lr, qf, m_run,
+    decode_stage<C, GT>(ks, ks + C::TILE_BYTES, min(C::T, t_end - (t_begin + it * C::T)), warp, lane, lr, qf, m_run,
                         l_run, acc_o, ps, alpha_s);
     __syncwarp();
     if (lane == 0) mbar_arrive(bar_empty + 8 * slot);
@@ -714,7 +715,7 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
           const int slot = pos % C::NSTAGE;
           if (!(ok = mbar_wait_warp(bar_full + 8 * slot, (pos / C::NSTAGE) & 1, ctl, ab))) break;
           const uint8_t* ks = smem + slot * C::STAGE_BYTES;
-          decode_stage<D, GT>(ks, ks + C::TILE_BYTES, min(C::T, t1 - tok0), warp, lane, lr, qf, m_run, l_run, acc_o,
+          decode_stage<C, GT>(ks, ks + C::TILE_BYTES, min(C::T, t1 - tok0), warp, lane, lr, qf, m_run, l_run, acc_o,
                               ps, alpha_s);
           __syncwarp();
           // the unit's last slot stays held: it is the scratch of the merge below
@@ -889,10 +890,10 @@ bool prepare_kernel(Kernel kernel, uint32_t smem, bool cluster, PerDeviceOnce& o
   });
 }
 
-template <int D, int GT, bool PAGED>
+template <int D, int GT, bool PAGED, class Cfg = DecodeCfg<D>>
 bool prepare_split() {
   static PerDeviceOnce once;
-  return prepare_kernel(decode_split_kernel<D, GT, PAGED>, DecodeSmem<D, GT>::BYTES, false, once);
+  return prepare_kernel(decode_split_kernel<D, GT, PAGED, Cfg>, DecodeSmem<Cfg, GT>::BYTES, false, once);
 }
 
 template <int D, int GT, bool PAGED>
@@ -963,16 +964,16 @@ bool kv_views(const DecodeArgs& a, const PagedKV* pk, CUtensorMap* tk, CUtensorM
   return true;
 }
 
-template <int D, int GT, bool PAGED>
+template <int D, int GT, bool PAGED, class Cfg = DecodeCfg<D>>
 cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
-  if (!prepare_split<D, GT, PAGED>()) return cudaErrorInvalidValue;
+  if (!prepare_split<D, GT, PAGED, Cfg>()) return cudaErrorInvalidValue;
   CUtensorMap tk, tv;
   PagedView view;
   if (!kv_views<D, PAGED>(a, pk, &tk, &tv, &view)) return cudaErrorInvalidValue;
   const int G = a.Hq / a.Hkv;
   const int n_groups = (G + GT - 1) / GT;
   dim3 grid(a.splits, a.Hkv * n_groups, a.B);
-  decode_split_kernel<D, GT, PAGED><<<grid, DecodeCfg<D>::THREADS, DecodeSmem<D, GT>::BYTES, stream>>>(
+  decode_split_kernel<D, GT, PAGED, Cfg><<<grid, Cfg::THREADS, DecodeSmem<Cfg, GT>::BYTES, stream>>>(
       static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.k),
       static_cast<const __nv_bfloat16*>(a.v), a.seqlens, a.o_part, a.lse_part, a.Hq, a.Hkv, a.Skv,
       a.splits, n_groups, a.scale * kLog2e, ctl, tk, tv, view);
@@ -1038,8 +1039,36 @@ int decode_form(const DecodeArgs& a) {
   return ch.t_us < model::decode_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms) * (1.0 - 1e-9) ? ch.cs : 0;
 }
 
+// Stage plans compiled beside the model's for the block-size ablation (contiguous cache,
+// D = 128, four query heads per CTA, split + merge form): {tokens per stage, stages, CTAs
+// per SM}; index + 1 is DecodeArgs::stage_plan.
+constexpr int kDecodeAblationPlans[][3] = {{32, 2, 2}, {32, 3, 2}, {32, 4, 2}, {64, 2, 2},
+                                           {64, 4, 1}, {128, 2, 1}, {128, 3, 1}};
+
+template <int I>
+cudaError_t launch_ablation_split(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  constexpr const int* P = kDecodeAblationPlans[I];
+  return launch_split<128, 4, false, DecodeCfg<128, P[0], P[1], P[2]>>(a, nullptr, ctl, stream);
+}
+
+cudaError_t launch_ablation(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  cudaError_t e;
+  switch (a.stage_plan) {
+    case 1: e = launch_ablation_split<0>(a, ctl, stream); break;
+    case 2: e = launch_ablation_split<1>(a, ctl, stream); break;
+    case 3: e = launch_ablation_split<2>(a, ctl, stream); break;
+    case 4: e = launch_ablation_split<3>(a, ctl, stream); break;
+    case 5: e = launch_ablation_split<4>(a, ctl, stream); break;
+    case 6: e = launch_ablation_split<5>(a, ctl, stream); break;
+    default: e = launch_ablation_split<6>(a, ctl, stream); break;
+  }
+  if (e != cudaSuccess) return e;
+  return launch_merge<128>(a, stream);
+}
+
 template <int D, int GT, bool PAGED>
 cudaError_t launch_form(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
+  if (D == 128 && GT == 4 && !PAGED && a.stage_plan > 0) return launch_ablation(a, ctl, stream);
   const int cs = decode_form<D, GT, PAGED>(a);
   if (cs > 0) return launch_cluster<D, GT, PAGED>(a, cs, pk, ctl, stream);
   const cudaError_t e = launch_split<D, GT, PAGED>(a, pk, ctl, stream);
@@ -1094,5 +1123,13 @@ int decode_cluster_form(const DecodeArgs& a, bool paged) {
 }
 
 int decode_max_clusters(int D, int G, int cs) { return D == 128 ? max_clusters_d<128>(G, cs) : max_clusters_d<64>(G, cs); }
+
+int decode_ablation_plan(int tokens, int stages, int ctas_per_sm) {
+  for (int i = 0; i < static_cast<int>(sizeof(kDecodeAblationPlans) / sizeof(kDecodeAblationPlans[0])); ++i)
+    if (kDecodeAblationPlans[i][0] == tokens && kDecodeAblationPlans[i][1] == stages &&
+        kDecodeAblationPlans[i][2] == ctas_per_sm)
+      return i + 1;
+  return 0;
+}
 
 }  // namespace loom

@@ -43,18 +43,21 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescaleThreshold = 8.0f;  // base-2 units; P <= 2^8 between rescales
 
-// Tile and stage constants: the analytic model's argmin for this head dimension.
-template <int D>
+// Tile and stage constants: the analytic model's argmin for this head dimension.  SLOTS
+// other than 0 overrides the ring depth (the neighbours of the model's choice, measured by
+// the block-size ablation; 2 slots leave the loader no tile of look-ahead but cannot
+// deadlock: every slot the MMA warp waits for is released earlier in its own order).
+template <int D, int SLOTS = 0>
 struct FwdCfg {
   static constexpr model::FwdPlan kPlan = model::fwd_plan_variant(D, 2);
   static_assert(kPlan.feasible, "no feasible two-tile prefill schedule");
   static constexpr int BM = kPlan.bm;         // rows per query tile (= TMEM lanes)
   static constexpr int NQT = kPlan.q_tiles;   // query tiles per CTA
   static constexpr int BN = kPlan.bn;         // keys per KV tile
-  static constexpr int NSLOT = kPlan.kv_slots;  // K/V ring slots
+  static constexpr int NSLOT = SLOTS ? SLOTS : kPlan.kv_slots;  // K/V ring slots
   static_assert(BM == 128 && NQT == 2, "warp roles assume two 128-row query tiles");
   static_assert(BN == 128, "softmax holds one S row of 128 fp32 in registers, P leaves in two 64-key halves");
-  static_assert(kPlan.b_lm == 1 && NSLOT >= 3, "the loader runs ahead of the MMA by >= one tile");
+  static_assert(kPlan.b_lm == 1 && NSLOT >= 2, "a K and a V slot at least");
   static constexpr int THREADS = 320;               // 8 softmax warps + loader + MMA
   static constexpr int BOX_COLS = 64;               // 128-byte swizzle atom = 64 bf16
   static constexpr int NBOX = D / BOX_COLS;         // TMA boxes per row of a tile
@@ -444,13 +447,14 @@ __device__ __forceinline__ void prefetch_item_l2(const CUtensorMap* tm_q, const 
 }
 
 // VARLEN: a ragged batch packed [total, H, D]: the tensor maps are [total, H, D] views
-// (coordinates: column, head, token) and items come from the sequence cursor.
-template <int D, bool VARLEN = false>
-__global__ void __launch_bounds__(FwdCfg<D>::THREADS, 1)
+// (coordinates: column, head, token) and items come from the sequence cursor.  SLOTS: the
+// ring depth (0: the model's).
+template <int D, bool VARLEN = false, int SLOTS = 0>
+__global__ void __launch_bounds__(FwdCfg<D, SLOTS>::THREADS, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                     const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
                     const FwdParams p) {
-  using C = FwdCfg<D>;
+  using C = FwdCfg<D, SLOTS>;
   constexpr int kRows = C::NQT * C::BM;  // query rows of one item
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the 128B-swizzled tiles
@@ -1370,11 +1374,35 @@ cudaError_t launch_design(Kernel kernel, int rows_per_item, const FwdArgs& a, co
   return cudaGetLastError();
 }
 
+// Ring depths compiled for the block-size ablation of the two-tile design (the model's
+// depth and its neighbours that fit in shared memory, plus a shallow point).
+template <int D>
+cudaError_t launch_two_tile_slots(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream, bool* handled) {
+  *handled = true;
+  constexpr int kRows = FwdCfg<D>::NQT * FwdCfg<D>::BM;
+  if constexpr (D == 128) {
+    static PerDeviceOnce once2;
+    if (a.slots == 2) return launch_design<D, FwdCfg<D, 2>>(attn_fwd_kernel<D, false, 2>, kRows, a, ctl, stream, once2);
+  } else {
+    static PerDeviceOnce once3, once6, once9;
+    if (a.slots == 3) return launch_design<D, FwdCfg<D, 3>>(attn_fwd_kernel<D, false, 3>, kRows, a, ctl, stream, once3);
+    if (a.slots == 6) return launch_design<D, FwdCfg<D, 6>>(attn_fwd_kernel<D, false, 6>, kRows, a, ctl, stream, once6);
+    if (a.slots == 9) return launch_design<D, FwdCfg<D, 9>>(attn_fwd_kernel<D, false, 9>, kRows, a, ctl, stream, once9);
+  }
+  *handled = false;
+  return cudaSuccess;
+}
+
 template <int D>
 cudaError_t launch_fwd_d(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
   static PerDeviceOnce configured1, configured2, configured3;
   constexpr int kModelDesign = model::fwd_plan(D).design;
   const int design = a.design ? a.design : kModelDesign;
+  if (design == 2 && a.slots > 0 && a.slots != FwdCfg<D>::NSLOT) {
+    bool handled = false;
+    const cudaError_t e = launch_two_tile_slots<D>(a, ctl, stream, &handled);
+    if (handled) return e;
+  }
   if (design == 1)
     return launch_design<D, Fwd1Cfg<D>>(attn_fwd1_kernel<D>, Fwd1Cfg<D>::BM, a, ctl, stream, configured1);
   if constexpr (Fwd3Cfg<D>::kFeasible) {

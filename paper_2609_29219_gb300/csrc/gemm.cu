@@ -32,12 +32,14 @@
 namespace loom {
 namespace {
 
-template <int BN>
+// NS other than 0 overrides the model's ring depth (the neighbours measured by the
+// block-size ablation).
+template <int BN, int NS = 0>
 struct GemmCfg {
   static constexpr model::GemmPlan kPlan = model::gemm_plan_variant(BN);
   static_assert(kPlan.feasible, "no feasible GEMM plan for this tile width");
   static constexpr int BM = 128, BK = 64;
-  static constexpr int NSTAGE = kPlan.stages;
+  static constexpr int NSTAGE = NS ? NS : kPlan.stages;
   static constexpr int THREADS = 320;                       // 8 epilogue warps, loader, MMA
   static constexpr int SPLIT_THREADS = 192;                 // split-K: 4 epilogue warps, loader, MMA
   static constexpr int NB = BN / 64;                        // 64-column boxes of a B stage
@@ -138,11 +140,11 @@ __device__ __forceinline__ void epilogue_warp(const CUtensorMap* tm_c, uint32_t 
 }
 
 // BK_MAJOR: B given [N, K] (C = A B^T), its tiles K-major like A's; else B [K, N].
-template <int BN, bool BK_MAJOR>
-__global__ void __launch_bounds__(GemmCfg<BN>::THREADS, 1)
+template <int BN, bool BK_MAJOR, int NS = 0>
+__global__ void __launch_bounds__(GemmCfg<BN, NS>::THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                 const __grid_constant__ CUtensorMap tm_c, const GemmParams p) {
-  using C = GemmCfg<BN>;
+  using C = GemmCfg<BN, NS>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_base = smem_u32(smem_raw);
   const uint32_t sbase = (raw_base + 1023u) & ~1023u;
@@ -463,9 +465,10 @@ __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
 // copies complete on the even CTA's full barrier (armed once for 64 KB); the even CTA's
 // commits signal stage-free and accumulator-ready on both CTAs at once; each CTA's eight
 // epilogue warps tell the even CTA that an accumulator has been read (16 arrivals).
-struct GemmPairCfg {
+template <int NS = 6>
+struct GemmPairCfgT {
   static constexpr int BM = 128, BN = 256, BK = 64;   // per CTA: 128 rows x 256 columns of C
-  static constexpr int NSTAGE = 6;
+  static constexpr int NSTAGE = NS;                    // 6: the model's depth (the deepest that fits)
   static constexpr int THREADS = 320;                  // 8 epilogue warps, loader, MMA
   static constexpr int NBH = 2;                        // 64-column boxes of this CTA's half of B
   static constexpr uint32_t A_BYTES = BM * BK * 2;
@@ -481,6 +484,7 @@ struct GemmPairCfg {
   static constexpr uint32_t TMEM_COLS = 512;  // two accumulators of 256 columns
   static_assert(BYTES <= 227 * 1024, "shared memory budget");
 };
+using GemmPairCfg = GemmPairCfgT<6>;
 
 __device__ __forceinline__ void tmem_alloc_pair(uint32_t dst, uint32_t ncols) {
   // one warp of each CTA of the pair, together: the same columns in both SMs
@@ -526,11 +530,11 @@ __device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
       : "memory");
 }
 
-template <bool BK_MAJOR>
-__global__ void __launch_bounds__(GemmPairCfg::THREADS, 1)
+template <bool BK_MAJOR, int NS = 6>
+__global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                      const __grid_constant__ CUtensorMap tm_c, const GemmParams p) {
-  using C = GemmPairCfg;
+  using C = GemmPairCfgT<NS>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_base = smem_u32(smem_raw);
   const uint32_t sbase = (raw_base + 1023u) & ~1023u;
@@ -704,11 +708,12 @@ bool matrix_map(CUtensorMap* map, const void* base, int rows, int cols, int box_
 // Devices whose cluster occupancy answers are cached (others query on every call).
 constexpr int kSlotCacheDevices = 64;
 
-template <int BN>
+template <int BN, int NS = 0>
 bool set_smem_attr(const void* fn, PerDeviceOnce& done, int dev) {
   // one opt-in per kernel and device (the flags are per template instance)
   return done.run(dev, [fn] {
-    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmCfg<BN>::BYTES) == cudaSuccess;
+    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmCfg<BN, NS>::BYTES) ==
+           cudaSuccess;
   });
 }
 
@@ -732,11 +737,11 @@ GemmParams make_params(const GemmArgs& a, const KernelCtl& ctl, int bn, int spli
   return p;
 }
 
-template <int BN, bool BKM>
+template <int BN, bool BKM, int NS = 0>
 cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int dev, int sms) {
-  using C = GemmCfg<BN>;
+  using C = GemmCfg<BN, NS>;
   static PerDeviceOnce configured;
-  if (!set_smem_attr<BN>(reinterpret_cast<const void*>(gemm_kernel<BN, BKM>), configured, dev))
+  if (!set_smem_attr<BN, NS>(reinterpret_cast<const void*>(gemm_kernel<BN, BKM, NS>), configured, dev))
     return cudaErrorInvalidValue;
   CUtensorMap ma, mb, mc;
   if (!make_maps(a, C::BM, BN, &ma, &mb, &mc)) return cudaErrorInvalidValue;
@@ -744,7 +749,7 @@ cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stre
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   const int grid = static_cast<int>(tiles < sms ? tiles : sms);
-  gemm_kernel<BN, BKM><<<grid, C::THREADS, C::BYTES, stream>>>(ma, mb, mc, p);
+  gemm_kernel<BN, BKM, NS><<<grid, C::THREADS, C::BYTES, stream>>>(ma, mb, mc, p);
   return cudaGetLastError();
 }
 
@@ -822,20 +827,22 @@ cudaError_t launch_splitk(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t 
   return cudaLaunchKernelEx(&cfg, gemm_splitk_kernel<BN, BKM>, ma, mb, p);
 }
 
-template <bool BKM>
+template <bool BKM, int NS = 6>
 bool prepare_pair(int dev) {
   static PerDeviceOnce configured;
-  const void* fn = reinterpret_cast<const void*>(gemm_pair_kernel<BKM>);
+  const void* fn = reinterpret_cast<const void*>(gemm_pair_kernel<BKM, NS>);
   return configured.run(dev, [fn] {
-    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmPairCfg::BYTES) == cudaSuccess;
+    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmPairCfgT<NS>::BYTES) ==
+           cudaSuccess;
   });
 }
 
+template <int NS = 6>
 cudaLaunchConfig_t pair_config(int grid, cudaStream_t stream, cudaLaunchAttribute* attr) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
-  cfg.blockDim = dim3(GemmPairCfg::THREADS, 1, 1);
-  cfg.dynamicSmemBytes = GemmPairCfg::BYTES;
+  cfg.blockDim = dim3(GemmPairCfgT<NS>::THREADS, 1, 1);
+  cfg.dynamicSmemBytes = GemmPairCfgT<NS>::BYTES;
   cfg.stream = stream;
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
@@ -868,10 +875,10 @@ int pair_slots(int dev) {
   return 2 * clusters;
 }
 
-template <bool BKM>
+template <bool BKM, int NS = 6>
 cudaError_t launch_pair(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stream, int dev) {
   const int slots = pair_slots(dev);
-  if (slots < 2 || !prepare_pair<BKM>(dev)) return cudaErrorInvalidConfiguration;
+  if (slots < 2 || !prepare_pair<BKM, NS>(dev)) return cudaErrorInvalidConfiguration;
   CUtensorMap ma, mb, mc;
   if (!make_maps(a, GemmPairCfg::BM, 128, &ma, &mb, &mc)) return cudaErrorInvalidValue;
   GemmParams p = make_params(a, ctl, GemmPairCfg::BN, 1);
@@ -880,8 +887,24 @@ cudaError_t launch_pair(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t st
   if (tiles > 0x3fffffffLL) return cudaErrorInvalidConfiguration;
   const long long pairs = tiles < slots / 2 ? tiles : slots / 2;
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = pair_config(static_cast<int>(2 * pairs), stream, attr);
-  return cudaLaunchKernelEx(&cfg, gemm_pair_kernel<BKM>, ma, mb, mc, p);
+  cudaLaunchConfig_t cfg = pair_config<NS>(static_cast<int>(2 * pairs), stream, attr);
+  return cudaLaunchKernelEx(&cfg, gemm_pair_kernel<BKM, NS>, ma, mb, mc, p);
+}
+
+// Ring depths compiled beside the model's for the block-size ablation ([K, N] B only): the
+// CTA pair with 5 stages (model: 6), persistent 256-wide tiles with 3 (model: 4), 128-wide
+// tiles with 5 (model: 6); the deeper neighbours do not fit in shared memory.
+bool gemm_stages_compiled(const GemmChoice& c, int stages) {
+  if (c.pair == 1) return stages == 5;
+  if (c.splits > 1) return false;
+  return (c.tile_n == 256 && stages == 3) || (c.tile_n == 128 && stages == 5);
+}
+
+cudaError_t launch_ablation(const GemmArgs& a, const GemmChoice& c, const KernelCtl& ctl, cudaStream_t stream,
+                            int dev, int sms) {
+  if (c.pair == 1) return launch_pair<false, 5>(a, ctl, stream, dev);
+  if (c.tile_n == 256) return launch_bn<256, false, 3>(a, ctl, stream, dev, sms);
+  return launch_bn<128, false, 5>(a, ctl, stream, dev, sms);
 }
 
 template <bool BKM>
@@ -925,6 +948,8 @@ cudaError_t launch_gemm(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t st
   if (!device_sms(&dev, &sms)) return cudaErrorNoDevice;
   const GemmChoice c = gemm_choice(a.M, a.N, a.K, {a.tile_n, a.splits, a.pair});
   if (c.tile_n == 0) return cudaErrorInvalidConfiguration;
+  if (a.stages > 0 && !a.b_kmajor && gemm_stages_compiled(c, a.stages))
+    return launch_ablation(a, c, ctl, stream, dev, sms);
   return a.b_kmajor ? launch_choice<true>(a, c, ctl, stream, dev, sms)
                     : launch_choice<false>(a, c, ctl, stream, dev, sms);
 }

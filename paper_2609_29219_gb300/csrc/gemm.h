@@ -16,6 +16,7 @@ struct GemmArgs {
   int splits;     // 0: the model's choice, else 1 (persistent tiles) or 2, 4, 8, 16 (split-K clusters)
   int pair;       // 0: the model's choice, 1: CTA-pair 256 x 256 tiles, -1: never CTA pairs
   int b_kmajor;   // 1: b is [N, K] row-major and C = A B^T
+  int stages;     // 0: the model's ring depth; a compiled neighbour of it otherwise (block-size ablation)
 };
 
 struct GemmChoice {

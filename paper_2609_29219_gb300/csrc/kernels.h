@@ -48,6 +48,7 @@ struct DecodeArgs {
   float scale;
   int fused;    // 0: the model's form; 1: the cluster form wherever it can run; -1: split + merge kernels
   int cluster;  // cluster form: 0 = the model's cluster size, else this size (if it divides splits and fits)
+  int stage_plan;  // 0: the model's stage plan; i > 0: the i-th compiled ablation plan (split + merge form)
 };
 
 struct FwdArgs {
@@ -59,7 +60,14 @@ struct FwdArgs {
   int B, Hq, Hkv, Sq, Skv, D, causal;
   float scale;
   int design;  // prefill design: 0 = the analytic model's choice, 1..3 forced
+  int slots;   // two-tile design's K/V ring depth: 0 = the model's; a compiled neighbour otherwise
 };
+
+// K/V ring depths of the two-tile prefill compiled beside the model's, for the block-size
+// ablation (D = 128: 2; D = 64: 3, 6, 9).
+inline bool fwd_slots_compiled(int D, int slots) {
+  return D == 128 ? slots == 2 : (slots == 3 || slots == 6 || slots == 9);
+}
 
 // Bytes of workspace the decode path needs for `splits` splits.
 inline size_t decode_workspace_bytes(int B, int Hq, int D, int splits) {
@@ -82,6 +90,9 @@ int decode_cluster_form(const DecodeArgs& a, bool paged);
 // Clusters of cs cluster-decode CTAs (G query heads per kv head) resident at once on the
 // current device; 0 if none fit or the device cannot be asked.
 int decode_max_clusters(int D, int G, int cs);
+// Index (> 0) of a compiled ablation stage plan of the decode split kernel (contiguous
+// cache, D = 128, 4 query heads per kv head), 0 if that plan is not compiled.
+int decode_ablation_plan(int tokens, int stages, int ctas_per_sm);
 cudaError_t launch_fwd(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t stream);
 
 }  // namespace loom

@@ -25,11 +25,14 @@ constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // 2 s
 uint64_t g_timeout_ns = kDefaultTimeoutNs;
 int g_inject = 0;
 int g_prefill_design = 0;
+int g_prefill_slots = 0;  // test hook: the two-tile prefill's K/V ring depth (0: the model's)
 int g_gemm_tile_n = 0;  // test hook: forced GEMM tile width (0: the model's choice)
 int g_gemm_splits = 0;  // test hook: forced GEMM split count (0: the model's choice)
 int g_gemm_pair = 0;    // test hook: 1 forces CTA-pair tiles, -1 forbids them, 0: the model's choice
+int g_gemm_stages = 0;  // test hook: GEMM ring depth (0: the model's; a compiled neighbour otherwise)
 int g_decode_fused = 0;    // test hook: 1 forces the cluster decode form, -1 forbids it, 0: the model's choice
 int g_decode_cluster = 0;  // test hook: the cluster decode form's cluster size (0: the model's)
+int g_decode_stage_plan = 0;  // test hook: a compiled ablation stage plan of the decode split kernel
 
 constexpr int kMaxDevices = 64;
 uint32_t* g_err_ptr[kMaxDevices] = {};
@@ -110,7 +113,7 @@ loom_status loom_attn_fwd(const void* q, const void* k, const void* v, void* o, 
     return LOOM_ERR_UNSUPPORTED;
   KernelCtl ctl;
   if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
-  FwdArgs a{q, k, v, o, lse, B, Hq, Hkv, Sq, Skv, D, causal, scale, g_prefill_design};
+  FwdArgs a{q, k, v, o, lse, B, Hq, Hkv, Sq, Skv, D, causal, scale, g_prefill_design, g_prefill_slots};
   return launch_fwd(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                : LOOM_ERR_CUDA;
 }
@@ -196,7 +199,7 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D,
-               num_splits, scale, g_decode_fused, g_decode_cluster};
+               num_splits, scale, g_decode_fused, g_decode_cluster, g_decode_stage_plan};
   return launch_decode(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                  : LOOM_ERR_CUDA;
 }
@@ -266,7 +269,7 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D, num_splits, scale,
-               g_decode_fused, g_decode_cluster};
+               g_decode_fused, g_decode_cluster, 0};
   PagedKV pk{block_table, num_pages, page_size, max_pages, kv_layout};
   return launch_decode_paged(a, pk, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                           : LOOM_ERR_CUDA;
@@ -280,7 +283,7 @@ loom_status gemm_call(const void* a, const void* b, void* c, int M, int N, int K
   if (K % 8 != 0 || N % 8 != 0) return LOOM_ERR_UNSUPPORTED;  // 16-byte row strides for TMA
   KernelCtl ctl;
   if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
-  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n, g_gemm_splits, g_gemm_pair, b_kmajor};
+  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n, g_gemm_splits, g_gemm_pair, b_kmajor, g_gemm_stages};
   return launch_gemm(g, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK : LOOM_ERR_CUDA;
 }
 }  // namespace
@@ -342,6 +345,8 @@ void loom_debug_gemm_tile_n(int tile_n) {
 void loom_debug_gemm_splits(int splits) { g_gemm_splits = model::gemm_split_supported(splits) ? splits : 0; }
 
 void loom_debug_gemm_cta_pair(int mode) { g_gemm_pair = (mode == 1 || mode == -1) ? mode : 0; }
+
+void loom_debug_gemm_stages(int stages) { g_gemm_stages = stages > 0 ? stages : 0; }
 
 loom_status loom_attn_check_error(void* stream) {
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return LOOM_ERR_CUDA;
@@ -457,12 +462,32 @@ void loom_debug_decode_cluster(int mode, int cluster) {
   g_decode_cluster = (cluster >= 1 && cluster <= model::kMaxClusterSize) ? cluster : 0;
 }
 
+int loom_debug_decode_stage_plan(int tokens, int stages, int ctas_per_sm) {
+  const model::DecodeStagePlan& m = model::decode_stage(128);
+  if (tokens == 0 || (tokens == m.tokens && stages == m.stages && ctas_per_sm == m.ctas_per_sm)) {
+    g_decode_stage_plan = 0;
+    return 1;
+  }
+  g_decode_stage_plan = decode_ablation_plan(tokens, stages, ctas_per_sm);
+  return g_decode_stage_plan > 0 ? 1 : 0;
+}
+
 void loom_debug_set_timeout_ns(uint64_t ns) { g_timeout_ns = ns ? ns : kDefaultTimeoutNs; }
 
 void loom_debug_inject(int mode) { g_inject = mode; }
 
 void loom_debug_prefill_design(int design) {
   g_prefill_design = (design >= 1 && design <= 3) ? design : 0;
+}
+
+int loom_debug_prefill_slots(int D, int slots) {
+  if (slots == 0 || (D == 128 && slots == model::fwd_plan_variant(128, 2).kv_slots) ||
+      (D == 64 && slots == model::fwd_plan_variant(64, 2).kv_slots) || fwd_slots_compiled(D, slots)) {
+    g_prefill_slots = slots;
+    return 1;
+  }
+  g_prefill_slots = 0;
+  return 0;
 }
 
 }  // extern "C"
