@@ -574,6 +574,8 @@ def main():
                          "against cuBLAS, every tile width measured (one JSON line per point); ablation: "
                          "the block-size ablation, every compiled neighbour of the model's prefill ring "
                          "depth, decode stage plan and GEMM ring depth measured beside the model's choice")
+    ap.add_argument("--prefill-design", type=int, default=0,
+                    help="with --ncu-case: force this prefill design (1-4) instead of the model's choice")
     ap.add_argument("--ncu-case", default=None,
                     help="profiling run: set up this workload (tiny, tiny_causal, prefill, prefill_causal, "
                          "long_prefill_d128, long_prefill_d64, varlen_prefill, batched_decode, paged_decode_p16, paged_decode_p64, "
@@ -785,7 +787,7 @@ def run_model_sweep(torch, loom, dev, stream, args, peaks):
         wl = Prefill("sweep", B, H, Hkv, S, D, causal=causal)
         wl.setup(torch, dev, loom)
         chosen = loom.loom_model_fwd_plan(D)["design"]
-        for design in (1, 2, 3):
+        for design in (1, 2, 3, 4):
             model_us = loom.loom_model_fwd_time_us_design(design, B, H, S, S, D, causal)
             if model_us < 0:
                 continue
@@ -982,7 +984,14 @@ def run_ncu_case(torch, loom, dev, stream, args):
     cases["gemm_8192"] = Gemm("gemm_8192", 8192, 8192, 8192)
     cases["cublas_8192"] = Gemm("cublas_8192", 8192, 8192, 8192, cublas=True)
     cases["varlen_prefill_small"] = VarlenPrefill("varlen_prefill_small", 8, 32, 8, 512, 2048, 128, causal=True)
+    cases["prefill_d64_small"] = Prefill("prefill_d64_small", 1, 16, 4, 8192, 64, causal=True)
+    cases["batched_decode_cluster"] = Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16,
+                                             lengths=synth.decode_lengths(0, 16, 4096, 8192))
     wl = cases[args.ncu_case]
+    if args.prefill_design:
+        loom.loom_debug_prefill_design(args.prefill_design)
+    if args.ncu_case == "batched_decode_cluster":
+        loom.loom_debug_decode_cluster(1, 2)
     wl.sets = 1  # one input set: the smallest device footprint for a capture
     wl.setup(torch, dev, loom)
     with torch.cuda.stream(stream):

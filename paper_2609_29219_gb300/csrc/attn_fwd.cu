@@ -296,22 +296,32 @@ __device__ __forceinline__ bool softmax_step(uint32_t s_tm, uint32_t o_tm, uint3
   if (need) m_run = m_new;
   const float ms = (m_run == -INFINITY) ? 0.f : m_run;
   const uint64_t nms2 = f2(-ms, -ms);
-  // p = 2^(s*c - m): packed FMA, one MUFU ex2 per score, 4 packed partial sums
+  // p = 2^(s*c - m): packed FMA, one MUFU ex2 per score, 4 packed partial sums.  P leaves
+  // in two halves of H0 and BN - H0 keys (64 + 64, or 64 + 32 for 96-key tiles), each
+  // written as packed bf16 pairs over the first columns of its keys' S.
+  static_assert(BN == 128 || BN == 96, "P halves of 64 + 64 or 64 + 32 keys");
+  constexpr int H0 = 64;
   uint64_t acc[4] = {0, 0, 0, 0};
 #pragma unroll
   for (int half = 0; half < 2; ++half) {
-    uint32_t pk[BN / 4];
+    const int k0 = half == 0 ? 0 : H0;
+    const int nk = half == 0 ? H0 : BN - H0;
+    uint32_t pk[H0 / 2];
 #pragma unroll
-    for (int i = 0; i < BN / 4; ++i) {
-      const int e = half * (BN / 2) + 2 * i;
-      const uint64_t x = fma2(f2(__uint_as_float(s[e]), __uint_as_float(s[e + 1])), c2, nms2);
-      const float p0 = ex2(f2lo(x));
-      const float p1 = ex2(f2hi(x));
-      acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
-      pk[i] = pack_bf16x2(p0, p1);
+    for (int i = 0; i < H0 / 2; ++i) {
+      if (i < nk / 2) {
+        const int e = k0 + 2 * i;
+        const uint64_t x = fma2(f2(__uint_as_float(s[e]), __uint_as_float(s[e + 1])), c2, nms2);
+        const float p0 = ex2(f2lo(x));
+        const float p1 = ex2(f2hi(x));
+        acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
+        pk[i] = pack_bf16x2(p0, p1);
+      }
     }
-#pragma unroll
-    for (int ch = 0; ch < BN / 128; ++ch) tmem_st32(s_tm + half * (BN / 4) + ch * 32, pk + ch * 32);
+    if (nk == 64)
+      tmem_st32(s_tm + k0 / 2, pk);
+    else
+      tmem_st16(s_tm + k0 / 2, pk);
     tmem_wait_st();
     // O must hold the previous P.V before it is rescaled, and be rescaled before this
     // tile's P.V starts (the first-half arrive below).
@@ -365,17 +375,22 @@ __device__ __forceinline__ bool softmax_epilogue(uint32_t o_tm, uint32_t bar_o, 
   const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
   const uint64_t il2 = f2(inv_l, inv_l);
   uint32_t w[D / 2];  // the row as packed bf16 pairs
+  // 64 columns per TMEM round trip: two loads in flight before each wait
 #pragma unroll
-  for (int ch = 0; ch < D / 32; ++ch) {
-    uint32_t rr[32];
-    tmem_ld32(o_tm + ch * 32, rr);
+  for (int ch = 0; ch < D / 32; ch += 2) {
+    uint32_t rr[2][32];
+    tmem_ld32(o_tm + ch * 32, rr[0]);
+    tmem_ld32(o_tm + ch * 32 + 32, rr[1]);
     tmem_wait_ld();
-    reg_fence32(rr);
+    reg_fence32(rr[0]);
+    reg_fence32(rr[1]);
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const uint64_t x = mul2(f2(__uint_as_float(rr[2 * i]), __uint_as_float(rr[2 * i + 1])), il2);
-      w[ch * 16 + i] = pack_bf16x2(f2lo(x), f2hi(x));
-    }
+    for (int u = 0; u < 2; ++u)
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const uint64_t x = mul2(f2(__uint_as_float(rr[u][2 * i]), __uint_as_float(rr[u][2 * i + 1])), il2);
+        w[(ch + u) * 16 + i] = pack_bf16x2(f2lo(x), f2hi(x));
+      }
   }
   tc_fence_before();
   mbar_arrive(bar_oe);  // O is in registers: the next item's P.V may overwrite it
@@ -1240,6 +1255,295 @@ __global__ void __launch_bounds__(Fwd3Cfg<D>::THREADS, 1)
   }
 }
 
+// ---------------------------------------------------------------- three-tile variant
+// Three 128-row query tiles per CTA over KV tiles of BN = 96 keys (D = 64 only).  The MMA
+// warp issues S0 S1 S2 | PV0 S0' | PV1 S1' | PV2 S2' | ...: while one tile's softmax
+// runs, the tensor pipe works through the other two tiles' P.V and next S, so each tile's
+// chain S -> softmax -> P.V has two tiles' MMAs to hide behind (design 2 has one).  P is
+// handed over in halves of 64 and 32 keys.  A query tile wholly past Sq (the last item of
+// a plane when Sq is not a multiple of 384) runs one KV tile only; its rows are clipped
+// by the O tensor map and get no LSE.
+//   warps 0-3 / 4-7 / 8-11 softmax of tile 0 / 1 / 2, warp 12 loader, warp 13 MMA
+//   TMEM (512 columns): tile t's S/P at t * 160 (96 columns), its O at t * 160 + 96 (64)
+template <int D>
+struct Fwd4Cfg {
+  static constexpr model::FwdPlan kPlan = model::fwd_plan_variant(D, 4);
+  static constexpr bool kFeasible = kPlan.feasible;
+  static constexpr int BM = 128;
+  static constexpr int NQT = 3;
+  static constexpr int BN = 96;
+  static constexpr int NSLOT = kFeasible ? kPlan.kv_slots : 3;
+  static constexpr int THREADS = 448;
+  static constexpr int BOX_COLS = 64;
+  static constexpr int NBOX = D / BOX_COLS;
+  static constexpr uint32_t Q_BOX_BYTES = BM * 128;
+  static constexpr uint32_t Q_TILE_BYTES = NBOX * Q_BOX_BYTES;
+  static constexpr uint32_t KV_BOX_BYTES = BN * 128;
+  static constexpr uint32_t SLOT_BYTES = NBOX * KV_BOX_BYTES;
+  static constexpr uint32_t Q_OFF = 0;
+  static constexpr uint32_t RING_OFF = NQT * Q_TILE_BYTES;
+  static constexpr uint32_t STG_OFF = RING_OFF + NSLOT * SLOT_BYTES;  // O staging, one block per warp
+  static constexpr uint32_t BAR_OFF = STG_OFF + NQT * BM * D * 2;
+  // barriers: q_full[3], q_empty[3], full[NSLOT], empty[NSLOT], s[3], p[3][2], o[3], o_empty[3], drain
+  static constexpr int NBAR = 6 + 2 * NSLOT + 3 + 6 + 3 + 3 + 1;
+  static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
+  static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
+  static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;
+  static constexpr uint32_t TMEM_COLS = 512;
+  static constexpr uint32_t TILE_COLS = 160;  // tile t: S/P at t * 160, O at t * 160 + BN
+  static_assert(!kFeasible || D == 64, "three S buffers and O accumulators fit TMEM at D = 64 only");
+  static_assert(!kFeasible || (BYTES <= 227 * 1024 && NQT * TILE_COLS <= TMEM_COLS && BN + D <= TILE_COLS),
+                "budgets");
+  static_assert(KV_BOX_BYTES % 1024 == 0, "128B-swizzled tiles start on 1024-byte boundaries");
+};
+
+// KV tiles of BN keys that query tile t (rows q0 + t * 128 ..) of an item needs: up to the
+// diagonal of its last row when causal; one for a tile wholly past Sq.
+__device__ __forceinline__ int fwd4_tiles(const FwdParams& p, int q0, int t) {
+  const int r0 = q0 + t * Fwd4Cfg<64>::BM;
+  if (r0 >= p.Sq) return 1;
+  int n_kv = p.Skv;
+  if (p.causal) n_kv = min(p.Skv, r0 + Fwd4Cfg<64>::BM + (p.Skv - p.Sq));
+  return (n_kv + Fwd4Cfg<64>::BN - 1) / Fwd4Cfg<64>::BN;
+}
+
+template <int D>
+__global__ void __launch_bounds__(Fwd4Cfg<D>::THREADS, 1)
+    attn_fwd4_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                     const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
+                     const FwdParams p) {
+  using C = Fwd4Cfg<D>;
+  if constexpr (!C::kFeasible) {
+    return;
+  } else {
+  constexpr int kRows = C::NQT * C::BM;  // query rows of one item
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_base = smem_u32(smem_raw);
+  const uint32_t sbase = (raw_base + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (sbase - raw_base);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const uint32_t bar_q = sbase + C::BAR_OFF;           // [3] Q_t loaded
+  const uint32_t bar_qe = bar_q + 24;                  // [3] Q_t no longer read
+  const uint32_t bar_full = bar_qe + 24;               // [NSLOT]
+  const uint32_t bar_empty = bar_full + 8 * C::NSLOT;  // [NSLOT]
+  const uint32_t bar_s = bar_empty + 8 * C::NSLOT;     // [3] S_t ready
+  const uint32_t bar_p = bar_s + 24;                   // [3][2] half h of P_t written (h = 0: and O_t rescaled)
+  const uint32_t bar_o = bar_p + 48;                   // [3] P_t V_j accumulated into O_t
+  const uint32_t bar_oe = bar_o + 24;                  // [3] O_t read out by the epilogue
+  const uint32_t bar_drain = bar_oe + 24;
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::TMEM_PTR_OFF);
+  Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
+
+  if (threadIdx.x == 0) {
+    for (int t = 0; t < C::NQT; ++t) {
+      mbar_init(bar_q + 8 * t, 1);
+      mbar_init(bar_qe + 8 * t, 1);
+      mbar_init(bar_s + 8 * t, 1);
+      mbar_init(bar_p + 16 * t, C::BM);
+      mbar_init(bar_p + 16 * t + 8, C::BM);
+      mbar_init(bar_o + 8 * t, 1);
+      mbar_init(bar_oe + 8 * t, C::BM);
+    }
+    for (int s = 0; s < C::NSLOT; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, 1);
+    }
+    mbar_init(bar_drain, 1);
+    *ab.flag = 0;
+    *(ab.flag + 1) = 0;
+    fence_barrier_init();
+  }
+  if (warp == 13) tmem_alloc(smem_u32(tmem_ptr), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_ptr;
+
+  if (warp == 12) {
+    // ------------------------------------------------------------------ loader
+    if (lane == 0) {
+      prefetch_tensormap(&tm_q);
+      prefetch_tensormap(&tm_k);
+      prefetch_tensormap(&tm_v);
+      int pos = 0, issued = 0, skipped = -1, q_issued[3] = {0, 0, 0};
+      bool ok = true;
+      // Q_t of item r, once the previous item's S MMAs of tile t are done with its buffer
+      auto load_q = [&](int t, int r, const Item& it) -> bool {
+        if (r > 0 && !mbar_wait(bar_qe + 8 * t, (r - 1) & 1, p.ctl, ab)) return false;
+        mbar_expect_tx(bar_q + 8 * t, C::Q_TILE_BYTES);
+        for (int x = 0; x < C::NBOX; ++x)
+          tma_load_3d(sbase + C::Q_OFF + t * C::Q_TILE_BYTES + x * C::Q_BOX_BYTES, &tm_q, x * C::BOX_COLS,
+                      it.q0 + t * C::BM, it.q_z, bar_q + 8 * t);
+        q_issued[t] = r + 1;
+        return true;
+      };
+      for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+        const Item it = make_item<D>(p, idx);  // b, h, q_z, kv_z (the 256-row fields are unused)
+        Item it4 = it;
+        int pos_item, bh;
+        item_coords(p, idx, pos_item, bh);
+        it4.q0 = pos_item * kRows;
+        const int nmax = max(fwd4_tiles(p, it4.q0, 0), max(fwd4_tiles(p, it4.q0, 1), fwd4_tiles(p, it4.q0, 2)));
+        if (!(ok = load_q(0, r, it4))) break;
+        for (int jj = 0; jj < 2 * nmax; ++jj, ++pos) {  // K_0, [Q_1, Q_2], V_0, K_1, V_1, ...
+          if (jj == 1 && !((ok = load_q(1, r, it4)) && (ok = load_q(2, r, it4)))) break;
+          if (jj == max(0, 2 * nmax - 6)) {  // three KV tiles before the end
+            const int nidx = item_index(p, r + 1);
+            if (nidx >= 0) {
+              const Item nx = make_item<D>(p, nidx);
+              int npos, nbh;
+              item_coords(p, nidx, npos, nbh);
+              prefetch_item_l2<D, C::NQT, C::BM>(&tm_q, &tm_k, &tm_v, npos * kRows, nx.q_z, nx.kv_z);
+            }
+          }
+          const int slot = pos % C::NSLOT, round = pos / C::NSLOT;
+          if (!(ok = mbar_wait(bar_empty + 8 * slot, (round & 1) ^ 1, p.ctl, ab))) break;
+          issued = pos + 1;
+          if (p.ctl.inject == 2 && pos == 2) {  // test hook: never load this tile
+            skipped = pos;
+            continue;
+          }
+          mbar_expect_tx(bar_full + 8 * slot, C::SLOT_BYTES);
+          for (int x = 0; x < C::NBOX; ++x)
+            tma_load_3d(sbase + C::RING_OFF + slot * C::SLOT_BYTES + x * C::KV_BOX_BYTES, (jj & 1) ? &tm_v : &tm_k,
+                        x * C::BOX_COLS, (jj >> 1) * C::BN, it4.kv_z, bar_full + 8 * slot);
+        }
+      }
+      // drain copies still in flight before the CTA may exit
+      Abort no_abort{ab.flag + 1};
+      for (int t = 0; t < C::NQT; ++t)
+        if (q_issued[t] > 0) mbar_wait(bar_q + 8 * t, (q_issued[t] - 1) & 1, p.ctl, no_abort);
+      for (int ps = max(0, issued - C::NSLOT); ps < issued; ++ps)
+        if (ps != skipped) mbar_wait(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, no_abort);
+    }
+  } else if (warp == 13) {
+    // ------------------------------------------------------------------ MMA issuer
+    // The whole warp runs this role (warp-uniform operands and waits); one elected lane
+    // issues the MMAs and commits.
+    {
+      constexpr uint32_t idesc_s = idesc_bf16(C::BM, C::BN, 0, 0);  // Q, K both K-major
+      constexpr uint32_t idesc_pv = idesc_bf16(C::BM, D, 0, 1);     // P from TMEM, V MN-major
+      auto wait_slot = [&](int ps) {
+        return mbar_wait_warp(bar_full + 8 * (ps % C::NSLOT), (ps / C::NSLOT) & 1, p.ctl, ab);
+      };
+      const uint64_t dq0 = sdesc_sw128(sbase + C::Q_OFF, 16, 1024);
+      const uint64_t dk0 = sdesc_sw128(sbase + C::RING_OFF, 16, 1024);
+      const uint64_t dv0 = sdesc_sw128(sbase + C::RING_OFF, C::KV_BOX_BYTES, 1024);
+      constexpr uint32_t kSlot16 = C::SLOT_BYTES >> 4, kQTile16 = C::Q_TILE_BYTES >> 4;
+      // S_t = Q_t K^T (K = D = 64: one 64-wide box)
+      auto issue_s = [&](int t, int kpos) {
+        mma_ss_k64_el(tmem + t * C::TILE_COLS, dq0 + t * kQTile16, dk0 + (kpos % C::NSLOT) * kSlot16, idesc_s, 0u);
+      };
+      // O_t += P_t V_j: keys 0-63 (P columns 0-31), then keys 64-95 (P columns 32-47)
+      auto issue_pv = [&](int t, int vpos, bool acc, int half) {
+        const uint64_t b = dv0 + (vpos % C::NSLOT) * kSlot16 + half * 64 * (128 >> 4);
+        const uint32_t o = tmem + t * C::TILE_COLS + C::BN;
+        if (half == 0)
+          mma_ts_k64_el(o, tmem + t * C::TILE_COLS, b, idesc_pv, acc ? 1u : 0u);
+        else
+          mma_ts_k32_el(o, tmem + t * C::TILE_COLS + 32, b, idesc_pv, 1u);
+      };
+      int pos = 0, cnt[3] = {0, 0, 0};  // ring position of K_0; S/P/O uses so far per tile
+      bool ok = true;
+      for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+        int pos_item, bh;
+        item_coords(p, idx, pos_item, bh);
+        const int q0 = pos_item * kRows;
+        int nt[3];
+        for (int t = 0; t < 3; ++t) nt[t] = fwd4_tiles(p, q0, t);
+        const int nmax = max(nt[0], max(nt[1], nt[2]));
+        for (int t = 0; ok && t < 3; ++t) {
+          if (!(ok = mbar_wait_warp(bar_q + 8 * t, r & 1, p.ctl, ab) && (t > 0 || wait_slot(pos)))) break;
+          tc_fence_after();
+          issue_s(t, pos);
+          tc_commit_el(bar_s + 8 * t);
+          if (nt[t] == 1) tc_commit_el(bar_qe + 8 * t);  // every S of tile t issued
+        }
+        if (!ok) break;
+        tc_commit_el(bar_empty + 8 * (pos % C::NSLOT));  // K_0 read by the three S MMAs
+        for (int j = 0; ok && j < nmax; ++j) {
+          const int vpos = pos + 2 * j + 1, kpos = pos + 2 * j + 2;
+          const bool more = j + 1 < nmax;
+          if (!(ok = wait_slot(vpos))) break;
+          bool k_ready = false;
+          for (int t = 0; ok && t < 3; ++t) {
+            if (j < nt[t]) {
+              if (!(ok = mbar_wait_warp(bar_p + 16 * t, (cnt[t] + j) & 1, p.ctl, ab))) break;
+              // O_t of the previous item must have been read out
+              if (j == 0 && r > 0 && !(ok = mbar_wait_warp(bar_oe + 8 * t, (r - 1) & 1, p.ctl, ab))) break;
+              tc_fence_after();
+              issue_pv(t, vpos, j > 0, 0);
+              if (!(ok = mbar_wait_warp(bar_p + 16 * t + 8, (cnt[t] + j) & 1, p.ctl, ab))) break;
+              tc_fence_after();
+              issue_pv(t, vpos, true, 1);
+              tc_commit_el(bar_o + 8 * t);
+            }
+            if (j + 1 < nt[t]) {
+              if (!k_ready && !(ok = k_ready = wait_slot(kpos))) break;
+              tc_fence_after();
+              issue_s(t, kpos);
+              tc_commit_el(bar_s + 8 * t);
+              if (j + 2 == nt[t]) tc_commit_el(bar_qe + 8 * t);  // tile t's last S of the item
+            }
+          }
+          if (!ok) break;
+          tc_commit_el(bar_empty + 8 * (vpos % C::NSLOT));
+          if (more) tc_commit_el(bar_empty + 8 * (kpos % C::NSLOT));
+        }
+        for (int t = 0; t < 3; ++t) cnt[t] += nt[t];
+        pos += 2 * nmax;
+      }
+      // wait for every MMA issued above before TMEM may be released
+      Abort no_abort{ab.flag + 1};
+      tc_commit_el(bar_drain);
+      mbar_wait_warp(bar_drain, 0, p.ctl, no_abort);
+    }
+  } else {
+    // ------------------------------------------------------------------ softmax
+    const int t = warp >> 2;                        // query tile of this warpgroup
+    const int row_in_tile = (warp & 3) * 32 + lane;  // == TMEM lane
+    const uint32_t lane_addr = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t s_tm = tmem + lane_addr + t * C::TILE_COLS;
+    const uint32_t o_tm = s_tm + C::BN;
+    const uint32_t my_bar_s = bar_s + 8 * t, my_bar_p = bar_p + 16 * t, my_bar_o = bar_o + 8 * t;
+    const uint32_t my_bar_oe = bar_oe + 8 * t;
+    const uint32_t stg_q = sbase + C::STG_OFF + static_cast<uint32_t>(warp) * (32 * D * 2);
+    const float c = p.c;
+    const uint64_t c2 = f2(c, c);
+    const int off = p.Skv - p.Sq;
+    int cnt = 0;  // S tiles of this query tile processed in earlier items
+    bool ok = true;
+    for (int r = 0, idx; ok && (idx = item_index(p, r)) >= 0; ++r) {
+      int pos_item, bh;
+      item_coords(p, idx, pos_item, bh);
+      const int q0 = pos_item * kRows;
+      const int row = q0 + t * C::BM + row_in_tile;
+      const int limit = p.causal ? min(p.Skv, row + off + 1) : p.Skv;  // keys [0, limit) visible
+      const int my_tiles = fwd4_tiles(p, q0, t);
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int j = 0; ok && j < my_tiles; ++j)
+        ok = softmax_step<D, C::BN>(s_tm, o_tm, my_bar_s, (cnt + j) & 1, my_bar_p, my_bar_o, (cnt + j - 1) & 1,
+                                    j == 0, j * C::BN, limit, c, c2, m_run, l_run, p.ctl, ab);
+      if (!ok) break;
+      if (!(ok = softmax_epilogue<D>(o_tm, my_bar_o, (cnt + my_tiles - 1) & 1, my_bar_oe, m_run, l_run, row, bh, p,
+                                     ab, &tm_o, stg_q)))
+        break;
+      cnt += my_tiles;
+    }
+    if (lane == 0) bulk_wait_group0();  // the O stores have completed before the CTA exits
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 13) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+  }
+}
+
 // ---------------------------------------------------------------- host side
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                    const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
@@ -1409,6 +1713,12 @@ cudaError_t launch_fwd_d(const FwdArgs& a, const KernelCtl& ctl, cudaStream_t st
     if (design == 3)
       return launch_design<D, Fwd3Cfg<D>>(attn_fwd3_kernel<D>, Fwd3Cfg<D>::NQT * Fwd3Cfg<D>::BM, a, ctl,
                                           stream, configured3);
+  }
+  if constexpr (Fwd4Cfg<D>::kFeasible) {
+    static PerDeviceOnce configured4;
+    if (design == 4)
+      return launch_design<D, Fwd4Cfg<D>>(attn_fwd4_kernel<D>, Fwd4Cfg<D>::NQT * Fwd4Cfg<D>::BM, a, ctl,
+                                          stream, configured4);
   }
   return launch_design<D, FwdCfg<D>>(attn_fwd_kernel<D>, FwdCfg<D>::NQT * FwdCfg<D>::BM, a, ctl, stream,
                                      configured2);

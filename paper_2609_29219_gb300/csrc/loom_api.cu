@@ -389,7 +389,7 @@ loom_status loom_model_fwd_plan(int D, loom_fwd_plan* out) {
 
 loom_status loom_model_fwd_plan_variant(int D, int design, loom_fwd_plan* out) {
   if (!out) return LOOM_ERR_INVALID_ARG;
-  if ((D != 64 && D != 128) || design < 1 || design > 3) return LOOM_ERR_UNSUPPORTED;
+  if ((D != 64 && D != 128) || design < 1 || design > 4) return LOOM_ERR_UNSUPPORTED;
   const model::FwdPlan p = model::fwd_plan_variant(D, design);
   if (!p.feasible) return LOOM_ERR_UNSUPPORTED;
   fill_plan(p, out);
@@ -406,7 +406,7 @@ double loom_model_fwd_time_us(int B, int Hq, int Sq, int Skv, int D, int causal)
 }
 
 double loom_model_fwd_time_us_design(int design, int B, int Hq, int Sq, int Skv, int D, int causal) {
-  if (B <= 0 || Hq <= 0 || Sq <= 0 || Skv <= 0 || (D != 64 && D != 128) || design < 1 || design > 3) return -1.0;
+  if (B <= 0 || Hq <= 0 || Sq <= 0 || Skv <= 0 || (D != 64 && D != 128) || design < 1 || design > 4) return -1.0;
   const model::FwdPlan p = model::fwd_plan_variant(D, design);
   if (!p.feasible) return -1.0;
   return model::fwd_time_us(p, B, Hq, Sq, Skv, D, causal != 0);
@@ -477,7 +477,7 @@ void loom_debug_set_timeout_ns(uint64_t ns) { g_timeout_ns = ns ? ns : kDefaultT
 void loom_debug_inject(int mode) { g_inject = mode; }
 
 void loom_debug_prefill_design(int design) {
-  g_prefill_design = (design >= 1 && design <= 3) ? design : 0;
+  g_prefill_design = (design >= 1 && design <= 4) ? design : 0;
 }
 
 int loom_debug_prefill_slots(int D, int slots) {

@@ -45,6 +45,9 @@ struct ArchDesc {
   double mma_issue_busy_factor;     // MMA stream slowdown while high-ILP warps share the SM with
                                     // the MMA warp issuing warp-wide (measured: 546 vs 512 clk
                                     // per 128^3 GEMM; 1338 when a lone lane issues)
+  double softmax_triple_clk_per_key;  // three tiles' softmax running together (design 4, 96-key
+                                      // tiles, 14 warps at 128 registers), clocks per key of a
+                                      // round (measured: 876 TFLOP/s on B1 H64 S8192 D64 causal)
   double cluster_merge_ns;          // per unit and CTA of a cluster-decode cluster: the warps'
                                     // merge, the handshakes waiting on the slowest CTA and the
                                     // DSMEM gather (fitted: 147 / 103 / 93 us measured with
@@ -54,7 +57,7 @@ struct ArchDesc {
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 300.0,
+    129.0e6, 1.07, 28.4, 300.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -84,6 +87,9 @@ constexpr long long cdiv(long long a, long long b) { return (a + b - 1) / b; }
 //   design 3: two query tiles sharing a ring of three S buffers: both tiles' next S is
 //     computed while their softmax runs, so the two softmaxes overlap each other and the
 //     MMAs (TMEM: 3 BN + 2 D columns).
+//   design 4: three query tiles, one S buffer each, over KV tiles of BN = 96 keys (TMEM:
+//     3 (BN + D) columns, D = 64 only): the tiles take turns on the tensor pipe like
+//     design 2's two, so each tile's chain has two other tiles' MMAs to hide behind.
 struct FwdPlan {
   int design, bm, bn, q_tiles, s_buffers, kv_slots, b_lm, b_ms;
   int smem_bytes, tmem_cols;
@@ -97,8 +103,8 @@ constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int design, int bn, int slo
   FwdPlan p{};
   p.design = design;
   p.bm = 128;
-  p.q_tiles = design == 1 ? 1 : 2;
-  p.s_buffers = design == 1 ? 2 : design == 2 ? 1 : 3;
+  p.q_tiles = design == 1 ? 1 : design == 4 ? 3 : 2;
+  p.s_buffers = design == 1 ? 2 : design == 3 ? 3 : 1;
   p.bn = bn;
   p.kv_slots = slots;
   p.b_lm = b_lm;
@@ -113,12 +119,16 @@ constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int design, int bn, int slo
   p.t_softmax_ns = a.softmax_clk_per_key * bn / clk;
   const double sync = a.sync_ns;
   double body = 0.0;
-  if (design == 2) {
-    // per pair of tile-iterations the tensor pipe needs 2 * mma; each tile's chain (its
-    // softmax, then its P.V and next S on the tensor pipe, one barrier round trip: the
-    // warp-wide MMA issuer picks P up at once) must fit in the period, while the other
-    // tile's softmax overlaps it
-    body = dmax(2 * p.t_mma_ns, p.t_softmax_ns + p.t_mma_ns + sync) / 2;
+  if (design == 2 || design == 4) {
+    // per round of tile-iterations (one per query tile) the tensor pipe needs q_tiles *
+    // mma; each tile's chain (its softmax, then its P.V and next S on the tensor pipe, one
+    // barrier round trip: the warp-wide MMA issuer picks P up at once) must fit in the
+    // round, while the other tiles' softmaxes overlap it.  With three tiles the three
+    // softmaxes share the SM sub-partitions' MUFU and issue slots (and 14 warps cap a thread
+    // at 128 registers): a round takes at least their measured joint time.
+    body = dmax(p.q_tiles * p.t_mma_ns, p.t_softmax_ns + p.t_mma_ns + sync);
+    if (design == 4) body = dmax(body, a.softmax_triple_clk_per_key * bn / clk);
+    body /= p.q_tiles;
   } else if (design == 1) {
     body = dmax(p.t_mma_ns, p.t_softmax_ns) + sync;  // softmax and MMA overlap fully
   } else {
@@ -136,11 +146,16 @@ constexpr FwdPlan fwd_eval(const ArchDesc& a, int D, int design, int bn, int slo
   // Q tiles + K/V ring + an O staging tile per query tile (TMA-store epilogue) +
   // barriers and alignment
   p.smem_bytes = 2 * p.q_tiles * p.bm * D * 2 + slots * bn * D * 2 + 1024 + 256;
-  p.tmem_cols = design == 1 ? 2 * bn + D : design == 2 ? 2 * (bn + D) : 3 * bn + 2 * D;
+  // design 4 keeps each tile's S and O adjacent at 32-column aligned bases (t * 160)
+  p.tmem_cols = design == 1 ? 2 * bn + D : design == 2 ? 2 * (bn + D) : design == 3 ? 3 * bn + 2 * D
+                                                                      : 3 * (bn + D);
   p.feasible = true;
-  if (design < 1 || design > 3) p.feasible = false;
+  if (design < 1 || design > 4) p.feasible = false;
   if (bn % 16 != 0 || bn < 16 || bn > 256) p.feasible = false;   // MMA N for M = 128
-  if (bn != 128) p.feasible = false;  // softmax: one S row of 128 fp32 per thread, P in halves
+  // softmax: one S row per thread, P handed over in two halves: 128 keys (64 + 64) for
+  // designs 1-3, 96 keys (64 + 32) for design 4
+  if (bn != (design == 4 ? 96 : 128)) p.feasible = false;
+  if (design == 4 && D != 64) p.feasible = false;  // 3 S buffers + 3 O accumulators in 512 columns
   if (D % 64 != 0) p.feasible = false;                            // 128 B swizzle atoms
   if (p.smem_bytes > a.smem_per_cta) p.feasible = false;          // L1 footprint
   if (p.tmem_cols > a.tmem_cols) p.feasible = false;
@@ -177,7 +192,7 @@ constexpr FwdPlan fwd_plan_variant(int D, int design, const ArchDesc& a = kGb300
 // Eq. 9: the design with the lowest modeled latency (ties keep the earlier design).
 constexpr FwdPlan fwd_plan(int D, const ArchDesc& a = kGb300) {
   FwdPlan best = fwd_plan_variant(D, 2, a);
-  for (int design : {1, 3}) {
+  for (int design : {1, 3, 4}) {
     const FwdPlan p = fwd_plan_variant(D, design, a);
     if (!p.feasible) continue;
     if (!best.feasible || p.t_iter_ns / p.bn < best.t_iter_ns / best.bn * (1.0 - 1e-9)) best = p;

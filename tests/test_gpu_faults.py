@@ -95,7 +95,7 @@ def test_cluster_decode_skipped_stage_times_out_and_context_survives(loom, lens,
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "cluster decode after timeout")
 
 
-@pytest.mark.parametrize("design,D", [(2, 128), (1, 128), (1, 64), (3, 64)])
+@pytest.mark.parametrize("design,D", [(2, 128), (1, 128), (1, 64), (3, 64), (4, 64)])
 def test_prefill_skipped_tile_times_out_and_context_survives(loom, design, D):
     loom.loom_debug_prefill_design(design)
     try:

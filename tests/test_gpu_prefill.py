@@ -20,11 +20,12 @@ def loom():
     return m
 
 
-@pytest.fixture(autouse=True, params=[2, 1, 3], ids=["two_tiles", "one_tile_double_s", "s_ring"])
+@pytest.fixture(autouse=True, params=[2, 1, 3, 4], ids=["two_tiles", "one_tile_double_s", "s_ring", "three_tiles"])
 def design(request, loom):
     """Run every prefill test with each kernel design: two alternating query tiles; one
     query tile with S double-buffered in TMEM; two query tiles sharing a ring of three S
-    buffers (D = 64 only: at D = 128 the call runs the two-tile design)."""
+    buffers; three alternating query tiles over 96-key KV tiles (the last two D = 64 only:
+    at D = 128 the call runs the two-tile design)."""
     loom.loom_debug_prefill_design(request.param)
     yield request.param
     loom.loom_debug_prefill_design(0)

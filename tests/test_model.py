@@ -45,14 +45,14 @@ def test_fwd_plan_within_capacities(loom, D):
     assert p["bm"] in (64, 128)
     assert p["bn"] % 16 == 0 and 16 <= p["bn"] <= 256
     assert p["kv_slots"] >= 2
-    assert p["design"] in (1, 2, 3)
+    assert p["design"] in (1, 2, 3, 4)
     assert p["t_iter_ns"] > 0
 
 
 @pytest.mark.parametrize("D", [64, 128])
 def test_fwd_plan_is_argmin_over_designs(loom, D):
     chosen = loom.loom_model_fwd_plan(D)
-    variants = {d: loom.loom_model_fwd_plan_variant(D, d) for d in (1, 2, 3)}
+    variants = {d: loom.loom_model_fwd_plan_variant(D, d) for d in (1, 2, 3, 4)}
     feasible = {d: v for d, v in variants.items() if v is not None}
     assert chosen["design"] in feasible
     best = min(v["t_iter_ns"] / v["bn"] for v in feasible.values())
@@ -64,18 +64,25 @@ def test_fwd_plan_is_argmin_over_designs(loom, D):
 @pytest.mark.parametrize("D", [64, 128])
 def test_fwd_plan_ranks_the_measured_best_design_first(loom, D):
     # GB300 same-box measurements (warp-wide MMA issue): design 2 leads at both head
-    # dimensions (D=128: 1481 vs 1370 TFLOP/s for design 1; D=64: 1010 vs 874 for design 3
-    # and 813 for design 1), and at D=64 design 3 measures ahead of design 1
-    t = {d: loom.loom_model_fwd_plan_variant(D, d) for d in (1, 2, 3)}
+    # dimensions (D=128: 1481 vs 1370 TFLOP/s for design 1; D=64 (B1 H64 S8192 causal): 1004
+    # vs 876 for design 4, 874 for design 3 and 813 for design 1), and at D=64 designs 3
+    # and 4 measure ahead of design 1 (cost per key: t_iter / bn)
+    t = {d: loom.loom_model_fwd_plan_variant(D, d) for d in (1, 2, 3, 4)}
     assert loom.loom_model_fwd_plan(D)["design"] == 2
     if D == 64:
-        assert t[2]["t_iter_ns"] < t[3]["t_iter_ns"] < t[1]["t_iter_ns"]
+        cost = {d: t[d]["t_iter_ns"] / t[d]["bn"] for d in (1, 2, 3, 4)}
+        assert cost[2] < cost[3] < cost[1]
+        assert cost[2] < cost[4] < cost[1]
 
 
 def test_three_s_buffers_do_not_fit_at_d128(loom):
-    # 3 S buffers of 128 columns + 2 O tiles of 128 columns = 640 > 512 TMEM columns
+    # 3 S buffers of 128 columns + 2 O tiles of 128 columns = 640 > 512 TMEM columns;
+    # three tiles of 96-key S and 128-column O: 3 x 224 = 672 > 512
     assert loom.loom_model_fwd_plan_variant(128, 3) is None
     assert loom.loom_model_fwd_plan_variant(64, 3) is not None
+    assert loom.loom_model_fwd_plan_variant(128, 4) is None
+    p4 = loom.loom_model_fwd_plan_variant(64, 4)
+    assert p4 is not None and p4["q_tiles"] == 3 and p4["bn"] == 96 and p4["tmem_cols"] == 480
 
 
 @pytest.mark.parametrize("B,Hq,S,D,causal", [(4, 32, 2048, 128, 0), (4, 32, 2048, 128, 1),
@@ -171,7 +178,7 @@ def test_per_design_time_matches_the_choice(loom, D):
     chosen = loom.loom_model_fwd_plan(D)["design"]
     args = (4, 32, 2048, 2048, D, 0)
     assert loom.loom_model_fwd_time_us_design(chosen, *args) == pytest.approx(loom.loom_model_fwd_time_us(*args))
-    for d in (1, 2, 3):
+    for d in (1, 2, 3, 4):
         t = loom.loom_model_fwd_time_us_design(d, *args)
         assert (t < 0) == (loom.loom_model_fwd_plan_variant(D, d) is None)
         if t > 0:
