@@ -45,6 +45,9 @@ struct ArchDesc {
   double mma_issue_busy_factor;     // MMA stream slowdown while high-ILP warps share the SM with
                                     // the MMA warp issuing warp-wide (measured: 546 vs 512 clk
                                     // per 128^3 GEMM; 1338 when a lone lane issues)
+  double item_boundary_ns;  // prefill: between two work items of a CTA, the last P.V, the O
+                            // read-out and the next item's first S (in-kernel clock trace:
+                            // ~2400 clk at the 1.447 GHz reference clock)
   double softmax_triple_clk_per_key;  // three tiles' softmax running together (design 4, 96-key
                                       // tiles, 14 warps at 128 registers), clocks per key of a
                                       // round (measured: 876 TFLOP/s on B1 H64 S8192 D64 causal)
@@ -57,7 +60,7 @@ struct ArchDesc {
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 28.4, 300.0,
+    129.0e6, 1.07, 1660.0, 28.4, 300.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -242,28 +245,39 @@ constexpr int causal_block_layout(int planes, int group, int Skv, int D, int ite
 }
 
 // Modeled time (us) of a whole prefill launch under a plan (Eq. 5-7 over the CTA's
-// items: Q load ; for(KV tiles, pipe) ; O store, in waves over the SMs).
+// items: item boundary ; for(KV tiles, pipe), in waves over the SMs).  The query tiles of
+// an item take turns on the tensor pipe, so a KV-tile step costs a full round of
+// q_tiles iterations even when some tile (causal: the item's upper tiles) has no work left
+// in it: an item costs its slowest tile's KV tiles x q_tiles x t_iter.  The boundary
+// between items (the last P.V, the O read-out and the next item's first S: ~2400 clk in an
+// in-kernel clock trace) is item_boundary_ns.
 constexpr double fwd_time_us(const FwdPlan& p, int B, int Hq, int Sq, int Skv, int D, int causal,
                              const ArchDesc& a = kGb300) {
-  const long long rows_per_cta = 1LL * p.q_tiles * p.bm;
-  const long long groups = cdiv(Sq, rows_per_cta);
-  const long long ctas = groups * B * Hq;
-  double tiles = 0;  // average KV tiles per query tile
-  for (long long i = 0; i < cdiv(Sq, p.bm); ++i) {
-    long long n_kv = Skv;
-    if (causal) {
-      const long long lim = (i + 1) * p.bm + (Skv - Sq);
-      n_kv = lim < Skv ? lim : Skv;
+  (void)D;
+  const long long rows_per_item = 1LL * p.q_tiles * p.bm;
+  const long long groups = cdiv(Sq, rows_per_item);
+  const long long items = groups * B * Hq;
+  double item_tiles = 0;  // average over an item's of its slowest query tile's KV tiles
+  for (long long g = 0; g < groups; ++g) {
+    long long n_max = 0;
+    for (long long t = 0; t < p.q_tiles; ++t) {
+      const long long i = g * p.q_tiles + t;  // query tile
+      if (i * p.bm >= Sq) break;
+      long long n_kv = Skv;
+      if (causal) {
+        const long long lim = (i + 1) * p.bm + (Skv - Sq);
+        n_kv = lim < Skv ? lim : Skv;
+      }
+      const long long n = cdiv(n_kv, p.bn);
+      n_max = n > n_max ? n : n_max;
     }
-    tiles += static_cast<double>(cdiv(n_kv, p.bn));
+    item_tiles += static_cast<double>(n_max);
   }
-  tiles /= static_cast<double>(cdiv(Sq, p.bm));
-  const double t_q = 1.0 * rows_per_cta * D * 2 / a.l2_smem_gbs_sm;
-  const double t_o = 1.0 * rows_per_cta * D * 2 / a.l2_smem_gbs_sm;
-  const double t_cta = heg_seq(heg_seq(t_q, heg_for(tiles * p.q_tiles, p.t_iter_ns)), t_o);
-  const double waves = static_cast<double>(ctas) / a.num_sms;  // persistent CTAs
+  item_tiles /= static_cast<double>(groups);
+  const double t_item = heg_seq(a.item_boundary_ns, heg_for(item_tiles * p.q_tiles, p.t_iter_ns));
+  const double waves = static_cast<double>(items) / a.num_sms;  // persistent CTAs
   const double w = waves < 1.0 ? 1.0 : waves;
-  return w * t_cta * 1e-3;
+  return w * t_item * 1e-3;
 }
 
 // ------------------------------------------------------------------ decode
