@@ -743,30 +743,34 @@ def run_decode_sweep(torch, loom, dev, stream, args, peaks):
     for wl, splits in cases:
         wl.setup(torch, dev, loom)
         chosen = loom.loom_attn_decode_num_splits(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D)
-        chosen_form = loom.loom_attn_decode_cluster_form(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, 0)
+        chosen_form = loom.loom_attn_decode_form(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, 0)
+        slots = loom.loom_decode_persistent_slots(wl.D, G)
         for sp in sorted(set(splits + [chosen])):
             wl.splits = sp
             nbytes = loom.loom_attn_decode_workspace_bytes(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sp)
             wl.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
-            # split + merge, then the cluster form with every power-of-two cluster size dividing sp
-            for cs in [0] + [c for c in (1, 2, 4, 8, 16) if sp % c == 0]:
+            # split + merge, the persistent split kernel + merge, then the cluster form with
+            # every power-of-two cluster size dividing sp
+            for form, cs in [(1, 0), (2, 0)] + [(3, c) for c in (2, 4, 8, 16) if sp % c == 0]:
                 n_fit = loom.loom_decode_max_clusters(wl.D, G, cs) if cs else 0
                 if cs and n_fit < 1:
                     continue
-                loom.loom_debug_decode_cluster(1 if cs else -1, cs)
+                loom.loom_debug_decode_form(form, cs)
                 r = measure(torch, wl, max(10, args.steps // 4), args.warmup, stream, lambda: None, 1, float, peaks)
                 loom.loom_attn_check_error(stream)
-                if cs:
+                if form == 3:
                     model_us = loom.loom_model_decode_cluster_time_us(sp, cs, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, n_fit)
+                elif form == 2:
+                    model_us = loom.loom_model_decode_persistent_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, slots)
                 else:
                     model_us = loom.loom_model_decode_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sms)
-                print(json.dumps({"sweep": "decode", "workload": wl.describe(), "splits": sp,
-                                  "form": f"cluster{cs}" if cs else "split+merge", "resident_clusters": n_fit,
-                                  "model_choice": sp == chosen and cs == chosen_form,
+                name = {1: "split+merge", 2: "persistent+merge", 3: f"cluster{cs}"}[form]
+                print(json.dumps({"sweep": "decode", "workload": wl.describe(), "splits": sp, "form": name,
+                                  "model_choice": sp == chosen and (form, cs if form == 3 else 0) == chosen_form,
                                   "measured_us": round(r["ms_per_step"] * 1e3, 2),
                                   "model_us": round(model_us, 2), "GB/s": r["value"],
                                   "frac": r["roofline"]["frac"]}), flush=True)
-            loom.loom_debug_decode_cluster(0)
+            loom.loom_debug_decode_form(0)
         wl.inp = None
         torch.cuda.empty_cache()
 
@@ -855,7 +859,7 @@ def run_ablation_sweep(torch, loom, dev, stream, args, peaks):
 
     # decode: keys per stage x ring stages x CTAs per SM of the split kernel (split + merge form)
     plans = [(64, 3, 2), (32, 2, 2), (32, 3, 2), (32, 4, 2), (64, 2, 2), (64, 4, 1), (128, 2, 1), (128, 3, 1)]
-    loom.loom_debug_decode_cluster(-1)
+    loom.loom_debug_decode_form(1)
     for wl in (Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
                Decode("long_decode", 1, 32, 8, 131072, 128, splits=0)):
         wl.setup(torch, dev, loom)
@@ -867,7 +871,7 @@ def run_ablation_sweep(torch, loom, dev, stream, args, peaks):
         loom.loom_debug_decode_stage_plan(0)
         wl.inp = None
         torch.cuda.empty_cache()
-    loom.loom_debug_decode_cluster(0)
+    loom.loom_debug_decode_form(0)
 
     # GEMM: K-stage ring depth of the kernel the model picks (deeper rings do not fit)
     for (M, N, K), kernel, depths in [((8192, 8192, 8192), "pair", (5, 6)), ((16384, 16384, 16384), "pair", (5, 6)),
@@ -985,13 +989,13 @@ def run_ncu_case(torch, loom, dev, stream, args):
     cases["cublas_8192"] = Gemm("cublas_8192", 8192, 8192, 8192, cublas=True)
     cases["varlen_prefill_small"] = VarlenPrefill("varlen_prefill_small", 8, 32, 8, 512, 2048, 128, causal=True)
     cases["prefill_d64_small"] = Prefill("prefill_d64_small", 1, 16, 4, 8192, 64, causal=True)
-    cases["batched_decode_cluster"] = Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16,
+    cases["batched_decode_persistent"] = Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16,
                                              lengths=synth.decode_lengths(0, 16, 4096, 8192))
     wl = cases[args.ncu_case]
     if args.prefill_design:
         loom.loom_debug_prefill_design(args.prefill_design)
-    if args.ncu_case == "batched_decode_cluster":
-        loom.loom_debug_decode_cluster(1, 2)
+    if args.ncu_case == "batched_decode_persistent":
+        loom.loom_debug_decode_form(2)
     wl.sets = 1  # one input set: the smallest device footprint for a capture
     wl.setup(torch, dev, loom)
     with torch.cuda.stream(stream):

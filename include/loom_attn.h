@@ -119,13 +119,17 @@ size_t loom_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int Skv, int D, 
  * Split i of sequence b covers keys [i*C, min((i+1)*C, len_b)), C = ceil(len_b/splits)
  * rounded up to a multiple of 64; empty splits contribute nothing.  A sequence of
  * length 0 yields O = 0 and LSE = -inf.
- * Two forms compute it, chosen by the analytic model (see loom_attn_decode_cluster_form):
- * a split kernel writing the partials (O_i, lse_i) into the workspace followed by a merge
- * kernel (the gather, global softmax and final scaling of the Flash Decode HEG), or one
- * persistent kernel in which clusters of cs CTAs (cs divides num_splits, cs <= 16) walk
- * the (batch, kv head) pairs, CTA r taking splits r, r + cs, ... of each, and merge their
- * partials over distributed shared memory; that form leaves the workspace untouched, but
- * the call checks and requires it all the same.
+ * Three forms compute it, chosen by the analytic model (see loom_attn_decode_form):
+ *   1  a split kernel of one CTA per (split, batch, kv head) writing the partials (O_i,
+ *      lse_i) into the workspace, then a merge kernel (the gather, global softmax and
+ *      final scaling of the Flash Decode HEG);
+ *   2  the same partials and merge kernel, with a persistent split kernel whose CTAs walk
+ *      the (split, batch, kv head) items, streaming K/V across item boundaries;
+ *   3  one persistent kernel in which clusters of cs CTAs (cs divides num_splits, cs <= 16)
+ *      walk the (batch, kv head) pairs, CTA r taking splits r, r + cs, ... of each, and
+ *      merge their partials over distributed shared memory; it leaves the workspace
+ *      untouched, but the call checks and requires it all the same.
+ * All three follow the split rule above and give the same result up to rounding order.
  * Errors: INVALID_ARG, UNSUPPORTED, MISALIGNED, WORKSPACE, CUDA.
  */
 loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_cache,
@@ -226,20 +230,28 @@ double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, in
 double loom_model_decode_cluster_time_us(int splits, int cluster, int B, int Hq, int Hkv, int Skv, int D,
                                          int clusters);
 
+/* Modeled time (us) of the persistent split kernel + merge with `splits` splits on `ctas`
+ * resident CTAs; < 0 on bad sizes. */
+double loom_model_decode_persistent_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int ctas);
+
 /*
- * Which Flash Decode form a call with these sizes runs on the current device: cs > 0 = the
- * single-kernel cluster form with clusters of cs CTAs (Sec. 2.6's gather, global softmax
- * and final scaling done inside one kernel, over distributed shared memory), 0 = split
- * kernel + merge kernel, -1 = invalid sizes.  num_splits = 0 means the model's split
- * count; paged = 1 asks about loom_attn_decode_paged (Skv = max_pages * page_size).
- * Follows loom_debug_decode_cluster.
+ * Which Flash Decode form a call with these sizes runs on the current device: 1 = split
+ * kernel + merge kernel, 2 = persistent split kernel + merge kernel, 3 = the single-kernel
+ * cluster form (Sec. 2.6's gather, global softmax and final scaling done inside one kernel,
+ * over distributed shared memory) with *cluster CTAs per cluster; -1 = invalid sizes.
+ * num_splits = 0 means the model's split count; paged = 1 asks about
+ * loom_attn_decode_paged (Skv = max_pages * page_size).  cluster may be NULL.  Follows
+ * loom_debug_decode_form.
  * loom_decode_max_clusters: clusters of `cluster` decode CTAs (G query heads per kv head,
  * head dimension D) resident on the current device at once, 0 if none; with no device, the
- * model's GB300 estimate (whole clusters in 8 equal groups of SMs).  These are what the
- * split-count choice (num_splits = 0) prices the cluster form with.
+ * model's GB300 estimate (whole clusters in 8 equal groups of SMs).
+ * loom_decode_persistent_slots: CTAs of the persistent split kernel resident at once (with
+ * no device: the model's 2 per SM x 152 SMs).  These are what the split-count choice
+ * (num_splits = 0) prices the persistent forms with.
  */
-int loom_attn_decode_cluster_form(int B, int Hq, int Hkv, int Skv, int D, int num_splits, int paged);
+int loom_attn_decode_form(int B, int Hq, int Hkv, int Skv, int D, int num_splits, int paged, int* cluster);
 int loom_decode_max_clusters(int D, int G, int cluster);
+int loom_decode_persistent_slots(int D, int G);
 
 /*
  * BF16 GEMM, the third kernel the paper evaluates (GEMM shapes, Sec. 4): C = A B with
@@ -334,12 +346,13 @@ int loom_debug_decode_stage_plan(int tokens, int stages, int ctas_per_sm);
 void loom_debug_gemm_stages(int stages);
 
 /*
- * Test hook: the Flash Decode form.  mode 1 = the single-kernel cluster form wherever some
- * cluster size runs; -1 = always split + merge kernels; anything else: the analytic model's
- * choice (default).  cluster in 1..16 pins the cluster form's cluster size (honoured when
- * it divides the split count and such clusters fit); 0: the model's size.
+ * Test hook: the Flash Decode form.  form 1 = split + merge kernels, 2 = persistent split
+ * kernel + merge kernel, 3 = the single-kernel cluster form (each when it can run); anything
+ * else: the analytic model's choice (default).  cluster in 1..16 pins the cluster form's
+ * cluster size (honoured when it divides the split count and such clusters fit); 0: the
+ * model's size.
  */
-void loom_debug_decode_cluster(int mode, int cluster);
+void loom_debug_decode_form(int form, int cluster);
 
 #ifdef __cplusplus
 }

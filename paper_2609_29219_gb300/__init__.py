@@ -28,7 +28,8 @@ __all__ = [
     "loom_model_fwd_plan_variant", "loom_model_heg_pipe", "loom_model_fwd_time_us_design",
     "loom_attn_decode_paged", "loom_attn_fwd_varlen", "loom_gemm_bf16", "loom_gemm_bf16_bt", "loom_gemm_tile_n", "loom_gemm_splits", "loom_gemm_cta_pair", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
     "loom_debug_gemm_splits", "loom_debug_gemm_cta_pair", "loom_model_decode_cluster_time_us",
-    "loom_attn_decode_cluster_form", "loom_decode_max_clusters", "loom_debug_decode_cluster",
+    "loom_attn_decode_form", "loom_decode_max_clusters", "loom_decode_persistent_slots", "loom_debug_decode_form",
+    "loom_model_decode_persistent_time_us", "DECODE_SPLIT_MERGE", "DECODE_PERSISTENT", "DECODE_CLUSTER",
     "loom_debug_prefill_slots", "loom_debug_decode_stage_plan", "loom_debug_gemm_stages",
 ]
 
@@ -134,12 +135,16 @@ def capi() -> ctypes.CDLL:
             lib.loom_model_decode_time_us.restype = ctypes.c_double
             lib.loom_model_decode_cluster_time_us.argtypes = [i32] * 8
             lib.loom_model_decode_cluster_time_us.restype = ctypes.c_double
-            lib.loom_attn_decode_cluster_form.argtypes = [i32] * 7
-            lib.loom_attn_decode_cluster_form.restype = i32
+            lib.loom_model_decode_persistent_time_us.argtypes = [i32] * 7
+            lib.loom_model_decode_persistent_time_us.restype = ctypes.c_double
+            lib.loom_attn_decode_form.argtypes = [i32] * 7 + [ctypes.POINTER(i32)]
+            lib.loom_attn_decode_form.restype = i32
             lib.loom_decode_max_clusters.argtypes = [i32, i32, i32]
             lib.loom_decode_max_clusters.restype = i32
-            lib.loom_debug_decode_cluster.argtypes = [i32, i32]
-            lib.loom_debug_decode_cluster.restype = None
+            lib.loom_decode_persistent_slots.argtypes = [i32, i32]
+            lib.loom_decode_persistent_slots.restype = i32
+            lib.loom_debug_decode_form.argtypes = [i32, i32]
+            lib.loom_debug_decode_form.restype = None
             lib.loom_debug_prefill_slots.argtypes = [i32, i32]
             lib.loom_debug_prefill_slots.restype = i32
             lib.loom_debug_decode_stage_plan.argtypes = [i32, i32, i32]
@@ -497,18 +502,33 @@ def loom_model_decode_cluster_time_us(splits, cluster, B, Hq, Hkv, Skv, D, clust
     return float(capi().loom_model_decode_cluster_time_us(splits, cluster, B, Hq, Hkv, Skv, D, clusters))
 
 
-def loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, num_splits=0, paged=False) -> int:
-    """The cluster size if a decode call with these sizes runs the single-kernel cluster
-    form, 0 if the split + merge kernels, -1 on invalid sizes."""
-    return int(capi().loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, num_splits, int(bool(paged))))
+DECODE_SPLIT_MERGE, DECODE_PERSISTENT, DECODE_CLUSTER = 1, 2, 3
+
+
+def loom_attn_decode_form(B, Hq, Hkv, Skv, D, num_splits=0, paged=False):
+    """(form, cluster size) a decode call with these sizes runs: DECODE_SPLIT_MERGE,
+    DECODE_PERSISTENT or DECODE_CLUSTER (with its cluster size; 0 otherwise); form -1 on
+    invalid sizes."""
+    cs = ctypes.c_int(0)
+    f = int(capi().loom_attn_decode_form(B, Hq, Hkv, Skv, D, num_splits, int(bool(paged)), ctypes.byref(cs)))
+    return f, int(cs.value)
+
+
+def loom_model_decode_persistent_time_us(splits, B, Hq, Hkv, Skv, D, ctas) -> float:
+    return float(capi().loom_model_decode_persistent_time_us(splits, B, Hq, Hkv, Skv, D, ctas))
+
+
+def loom_decode_persistent_slots(D, G) -> int:
+    return int(capi().loom_decode_persistent_slots(D, G))
 
 
 def loom_decode_max_clusters(D, G, cluster) -> int:
     return int(capi().loom_decode_max_clusters(D, G, cluster))
 
 
-def loom_debug_decode_cluster(mode: int, cluster: int = 0) -> None:
-    capi().loom_debug_decode_cluster(int(mode), int(cluster))
+def loom_debug_decode_form(form: int, cluster: int = 0) -> None:
+    """Pin the Flash Decode form (DECODE_*; 0: the model's) and the cluster size (0: the model's)."""
+    capi().loom_debug_decode_form(int(form), int(cluster))
 
 
 def loom_debug_prefill_slots(D: int, slots: int) -> bool:

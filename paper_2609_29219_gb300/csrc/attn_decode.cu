@@ -23,7 +23,7 @@
 //   It is launched with programmatic dependent launch so its launch overlaps the
 //   split kernel's tail.
 //
-// Single-kernel (cluster) form, decode_cluster_kernel -- persistent clusters of CS CTAs
+// Single-kernel (cluster) form, decode_persistent_kernel<.., true> -- persistent clusters of CS CTAs
 // (CS divides the split count, CS <= 16).  A unit is one (batch, kv head, head group);
 // each cluster walks its units (dealt in a snake order over the units sorted by
 // sequence length), and for every unit CTA r of the cluster streams the unit's splits
@@ -511,9 +511,20 @@ __global__ void __launch_bounds__(C::THREADS, C::CTAS_PER_SM)
                      });
 }
 
-// ---------------------------------------------------------------- single-kernel form
+// ---------------------------------------------------------------- persistent forms
+// Two persistent kernels share one body (decode_persistent_kernel):
+//   CLUSTER = true: the single-kernel form.  Clusters of cs CTAs walk units (batch, kv
+//     head, head group); CTA r of a cluster takes splits r, r + cs, ... of each unit and the
+//     cluster merges its partials over distributed shared memory.
+//   CLUSTER = false: the persistent split kernel of the split + merge form.  Each CTA walks
+//     items (unit, split) and writes each item's partial (O_i, lse_i) to the workspace for
+//     the merge kernel, exactly as decode_split_kernel does, but without a CTA launch, a
+//     pipeline fill and a tail per item: the loader streams the next item's q and K/V
+//     while the compute warps finish the current one.
+// Both deal their work in a snake order over the sequences sorted by length (longest
+// first), which evens out the work per cluster or CTA when lengths differ.
 template <int D, int GT>
-struct ClusterSmem {
+struct PersistSmem {
   using C = DecodeCfg<D>;
   static constexpr int kMaxSortedB = 256;  // sequences sorted by length for the dealing
   // ring first (16-byte aligned bulk-copy destinations), then the small arrays
@@ -521,8 +532,8 @@ struct ClusterSmem {
   static constexpr uint32_t ALPHA_OFF = P_OFF + C::NCW * C::TW * GT * 4;  // [NCW][GT] f32
   static constexpr uint32_t WM_OFF = ALPHA_OFF + C::NCW * GT * 4;         // [NCW][GT] f32
   static constexpr uint32_t WL_OFF = WM_OFF + C::NCW * GT * 4;            // [NCW][GT] f32
-  static constexpr uint32_t Q_OFF = (WL_OFF + C::NCW * GT * 4 + 15) / 16 * 16;  // [GT][D] bf16, q of a unit
-  static constexpr uint32_t PO_OFF = Q_OFF + GT * D * 2;                 // [GT][D] f32, this CTA's partial O
+  static constexpr uint32_t Q_OFF = (WL_OFF + C::NCW * GT * 4 + 15) / 16 * 16;  // [GT][D] bf16, q of an item
+  static constexpr uint32_t PO_OFF = Q_OFF + GT * D * 2;                 // [GT][D] f32, the CTA's partial O
   static constexpr uint32_t PL_OFF = PO_OFF + GT * D * 4;                // [GT] f32, its log-sum-exps
   static constexpr uint32_t ORDER_OFF = (PL_OFF + GT * 4 + 15) / 16 * 16;  // [kMaxSortedB] int32
   static constexpr uint32_t BAR_OFF = ORDER_OFF + kMaxSortedB * 4;
@@ -533,42 +544,46 @@ struct ClusterSmem {
   static_assert(C::CTAS_PER_SM * (BYTES + 1024) <= 228 * 1024, "CTAs per SM of the stage plan");
 };
 
-// The k-th unit of cluster `cid` of n_clusters: units sorted by sequence length (longest
-// first), dealt in a snake order (even rounds left to right, odd rounds right to left);
-// -1 past the last.
-__device__ __forceinline__ int cluster_unit(int kk, int cid, int n_clusters, int n_units) {
-  const long long i = static_cast<long long>(kk) * n_clusters + ((kk & 1) ? n_clusters - 1 - cid : cid);
-  return i < n_units ? static_cast<int>(i) : -1;
+// The k-th work index of worker `w` of n_workers: a snake order over the sorted work
+// (even rounds left to right, odd rounds right to left); -1 past the last.
+__device__ __forceinline__ int snake_index(int kk, int w, int n_workers, int n_work) {
+  const long long i = static_cast<long long>(kk) * n_workers + ((kk & 1) ? n_workers - 1 - w : w);
+  return i < n_work ? static_cast<int>(i) : -1;
 }
 
-template <int D, int GT, bool PAGED>
+template <int D, int GT, bool PAGED, bool CLUSTER>
 __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_SM)
-    decode_cluster_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
-                          const __nv_bfloat16* __restrict__ v, const int32_t* __restrict__ seqlens,
-                          __nv_bfloat16* __restrict__ o, float* __restrict__ lse, int B, int Hq, int Hkv, int Skv,
-                          int splits, int n_groups, float c, KernelCtl ctl,
-                          const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
-                          PagedView pv) {
+    decode_persistent_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
+                             const __nv_bfloat16* __restrict__ v, const int32_t* __restrict__ seqlens,
+                             __nv_bfloat16* __restrict__ o, float* __restrict__ lse, float* __restrict__ o_part,
+                             float* __restrict__ lse_part, int B, int Hq, int Hkv, int Skv, int splits,
+                             int n_groups, float c, KernelCtl ctl, const __grid_constant__ CUtensorMap tm_k,
+                             const __grid_constant__ CUtensorMap tm_v, PagedView pv) {
   using C = DecodeCfg<D>;
-  using L = ClusterSmem<D, GT>;
+  using L = PersistSmem<D, GT>;
   extern __shared__ __align__(128) uint8_t smem[];
+  // split + merge form: let the merge grid launch as soon as every CTA is resident
+  if constexpr (!CLUSTER) asm volatile("griddepcontrol.launch_dependents;");
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int cs = static_cast<int>(cluster_nctarank());
-  const int rank = static_cast<int>(cluster_ctarank());
-  const int cid = static_cast<int>(blockIdx.x) / cs;
-  const int n_clusters = static_cast<int>(gridDim.x) / cs;
+  const int cs = CLUSTER ? static_cast<int>(cluster_nctarank()) : 1;
+  const int rank = CLUSTER ? static_cast<int>(cluster_ctarank()) : 0;
+  const int worker = static_cast<int>(blockIdx.x) / cs;         // cluster (or CTA) index
+  const int n_workers = static_cast<int>(gridDim.x) / cs;
   const int G = Hq / Hkv;
   const int upb = Hkv * n_groups;  // units per sequence
-  const int n_units = B * upb;
-  const int per_cta = splits / cs;  // splits r, r + cs, ... of every unit belong to CTA r
+  // work: units (cluster form; CTA r takes splits r, r + cs, ...) or (unit, split) items
+  // ordered sequence (by length), then split, then unit
+  const int per_seq = CLUSTER ? upb : upb * splits;
+  const int n_work = B * per_seq;
+  const int per_cta = CLUSTER ? splits / cs : 1;  // splits of a work piece this CTA streams
 
   const uint32_t s_base = smem_u32(smem);
   const uint32_t bar_full = s_base + L::BAR_OFF;
   const uint32_t bar_empty = bar_full + C::NSTAGE * 8;
   const uint32_t bar_qf = bar_empty + C::NSTAGE * 8;
   const uint32_t bar_qe = bar_qf + 8;
-  const uint32_t bar_ready = bar_qe + 8;     // every CTA's partial of the current unit is written
-  const uint32_t bar_consumed = bar_ready + 8;  // every CTA has read this CTA's partial
+  const uint32_t bar_ready = bar_qe + 8;        // cluster form: every CTA's partial of the unit is written
+  const uint32_t bar_consumed = bar_ready + 8;  // cluster form: every CTA has read this CTA's partial
   Abort ab{reinterpret_cast<volatile int*>(smem + L::ABORT_OFF)};
 
   // the sequences in order of decreasing length (ties by index): the dealing order
@@ -599,16 +614,18 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
     fence_barrier_init();
   }
   __syncthreads();
-  cluster_sync_all();  // every CTA's barriers exist before a peer arrives on them
+  if constexpr (CLUSTER) cluster_sync_all();  // every CTA's barriers exist before a peer arrives on them
 
-  // unit i (sorted order) -> sequence, kv head, head group, and the sequence's chunk length
-  struct Unit {
-    int b, hk, grp, h0, nh, len, chunk;
+  // work index i -> sequence, kv head, head group, first split, and the sequence's chunk
+  struct Work {
+    int b, hk, grp, h0, nh, len, chunk, split0;
   };
-  auto unit = [&](int i) {
-    Unit u;
-    const int br = i / upb, j = i % upb;
+  auto work = [&](int i) {
+    Work u;
+    const int br = i / per_seq, rem = i % per_seq;
+    const int j = CLUSTER ? rem : rem % upb;
     u.b = sorted ? order[br] : br;
+    u.split0 = CLUSTER ? rank : rem / upb;
     u.hk = j / n_groups;
     u.grp = j % n_groups;
     u.h0 = u.hk * G + u.grp * GT;
@@ -618,9 +635,9 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
     u.chunk = (ch + kDecodeChunkAlign - 1) / kDecodeChunkAlign * kDecodeChunkAlign;
     return u;
   };
-  // keys [*t0, *t1) of this CTA's jj-th split of unit u
-  auto split_range = [&](const Unit& u, int jj, int* t0, int* t1) {
-    const int s = rank + jj * cs;
+  // keys [*t0, *t1) of this CTA's jj-th split of work u
+  auto split_range = [&](const Work& u, int jj, int* t0, int* t1) {
+    const int s = u.split0 + jj * cs;
     *t0 = min(s * u.chunk, u.len);
     *t1 = min(*t0 + u.chunk, u.len);
   };
@@ -630,9 +647,9 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
     PagedLoader pl;
     int pos = 0, skipped = -1, q_loads = 0;
     bool ok = true;
-    for (int kk = 0, ui; ok && (ui = cluster_unit(kk, cid, n_clusters, n_units)) >= 0; ++kk) {
-      const Unit u = unit(ui);
-      // the unit's q rows (one bulk copy), once the compute warps have read the previous unit's
+    for (int kk = 0, wi; ok && (wi = snake_index(kk, worker, n_workers, n_work)) >= 0; ++kk) {
+      const Work u = work(wi);
+      // the work's q rows (one bulk copy), once the compute warps have read the previous ones
       if (kk > 0 && !(ok = mbar_wait_warp(bar_qe, (kk - 1) & 1, ctl, ab))) break;
       if (lane == 0) {
         const uint32_t qbytes = static_cast<uint32_t>(u.nh) * D * 2;
@@ -683,11 +700,11 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
     float* part_o = reinterpret_cast<float*>(smem + L::PO_OFF);
     float* part_l = reinterpret_cast<float*>(smem + L::PL_OFF);
     int pos = 0;
-    // A failed (timed-out) wait is made known to all compute warps at the unit's next
+    // A failed (timed-out) wait is made known to all compute warps at the work piece's next
     // common point (a barrier reduction), so that they leave together and none is left
     // waiting at a barrier of the merge.
-    for (int kk = 0, ui; (ui = cluster_unit(kk, cid, n_clusters, n_units)) >= 0; ++kk) {
-      const Unit u = unit(ui);
+    for (int kk = 0, wi; (wi = snake_index(kk, worker, n_workers, n_work)) >= 0; ++kk) {
+      const Work u = work(wi);
       bool ok = mbar_wait_warp(bar_qf, kk & 1, ctl, ab);
       float qf[GT][8];
       load_q<D, GT>(reinterpret_cast<const __nv_bfloat16*>(smem + L::Q_OFF), u.nh, lr.kl, c, qf);
@@ -701,7 +718,7 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
 #pragma unroll
         for (int d = 0; d < C::VD; ++d) acc_o[h][d] = 0.f;
 
-      int n_st = 0;  // this CTA's stages of the unit
+      int n_st = 0;  // this CTA's stages of the work piece
       for (int jj = 0; jj < per_cta; ++jj) {
         int t0, t1;
         split_range(u, jj, &t0, &t1);
@@ -718,28 +735,49 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
           decode_stage<C, GT>(ks, ks + C::TILE_BYTES, min(C::T, t1 - tok0), warp, lane, lr, qf, m_run, l_run, acc_o,
                               ps, alpha_s);
           __syncwarp();
-          // the unit's last slot stays held: it is the scratch of the merge below
+          // the last slot of the work piece stays held: it is the scratch of the merge below
           if (st + 1 < n_st && lane == 0) mbar_arrive(bar_empty + 8 * slot);
         }
       }
-      // this CTA's partial of the unit, once every CTA has read its previous one
-      if (ok && kk > 0) ok = mbar_wait_cluster_warp(bar_consumed, (kk - 1) & 1, ctl, ab);
+      // cluster form: this CTA's partial, once every CTA has read its previous one
+      if (CLUSTER && ok && kk > 0) ok = mbar_wait_cluster_warp(bar_consumed, (kk - 1) & 1, ctl, ab);
       if (named_bar_any(1, C::NCW * 32, !ok)) break;
+      const size_t part_row0 = (static_cast<size_t>(u.b) * Hq + u.h0) * splits + u.split0;  // split form
       if (n_st > 0) {
         const int last = (pos - 1) % C::NSTAGE;
         merge_warps<D, GT>(reinterpret_cast<float*>(smem + last * C::STAGE_BYTES),
                            reinterpret_cast<float*>(smem + L::WM_OFF), reinterpret_cast<float*>(smem + L::WL_OFF),
                            u.nh, warp, lane, lr, m_run, l_run, acc_o, [&](int idx, int h, int d, float ov, float lv) {
-                             part_o[idx] = ov;
-                             if (d == 0) part_l[h] = lv;
+                             if constexpr (CLUSTER) {
+                               part_o[idx] = ov;
+                               if (d == 0) part_l[h] = lv;
+                             } else {
+                               const size_t row = part_row0 + static_cast<size_t>(h) * splits;
+                               o_part[row * D + d] = ov;
+                               if (d == 0) lse_part[row] = lv;
+                             }
                            });
         asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");  // partial written, slot read
         if (lane == 0) mbar_arrive(bar_empty + 8 * last);
-      } else {  // no key of the unit falls to this CTA
-        for (int idx = threadIdx.x; idx < u.nh * D; idx += C::NCW * 32) part_o[idx] = 0.f;
-        if (threadIdx.x < u.nh) part_l[threadIdx.x] = -INFINITY;
-        asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");
+      } else {  // no key of the work piece falls to this CTA
+        for (int idx = threadIdx.x; idx < u.nh * D; idx += C::NCW * 32) {
+          if constexpr (CLUSTER) {
+            part_o[idx] = 0.f;
+          } else {
+            o_part[(part_row0 + static_cast<size_t>(idx / D) * splits) * D + idx % D] = 0.f;
+          }
+        }
+        if (threadIdx.x < u.nh) {
+          if constexpr (CLUSTER) {
+            part_l[threadIdx.x] = -INFINITY;
+          } else {
+            lse_part[part_row0 + static_cast<size_t>(threadIdx.x) * splits] = -INFINITY;
+          }
+        }
+        if constexpr (CLUSTER) asm volatile("bar.sync 1, %0;" ::"n"(C::NCW * 32) : "memory");
       }
+      if constexpr (!CLUSTER) continue;
+
       if (static_cast<int>(threadIdx.x) < cs) mbar_arrive_cluster(map_shared_rank(bar_ready, threadIdx.x));
       ok = mbar_wait_cluster_warp(bar_ready, kk & 1, ctl, ab);
       if (named_bar_any(1, C::NCW * 32, !ok)) break;
@@ -777,9 +815,9 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, DecodeCfg<D>::CTAS_PER_
       if (static_cast<int>(threadIdx.x) < cs) mbar_arrive_cluster(map_shared_rank(bar_consumed, threadIdx.x));
     }
   }
-  // Leave together: no CTA exits while a peer may still read its partial or arrive on its
-  // barriers.
-  cluster_sync_all();
+  // Cluster form: leave together -- no CTA exits while a peer may still read its partial or
+  // arrive on its barriers.
+  if constexpr (CLUSTER) cluster_sync_all();
 }
 
 // One CTA (D threads) per (batch, query head).  The split log-sum-exps are read in
@@ -896,10 +934,10 @@ bool prepare_split() {
   return prepare_kernel(decode_split_kernel<D, GT, PAGED, Cfg>, DecodeSmem<Cfg, GT>::BYTES, false, once);
 }
 
-template <int D, int GT, bool PAGED>
-bool prepare_cluster() {
+template <int D, int GT, bool PAGED, bool CLUSTER>
+bool prepare_persistent() {
   static PerDeviceOnce once;
-  return prepare_kernel(decode_cluster_kernel<D, GT, PAGED>, ClusterSmem<D, GT>::BYTES, true, once);
+  return prepare_kernel(decode_persistent_kernel<D, GT, PAGED, CLUSTER>, PersistSmem<D, GT>::BYTES, CLUSTER, once);
 }
 
 cudaLaunchConfig_t launch_config(dim3 grid, uint32_t smem, int cluster, cudaStream_t stream, cudaLaunchAttribute* attr) {
@@ -934,16 +972,40 @@ int max_clusters(int cs) {
     if (c != 0) return c - 1;
   }
   int clusters = 0;
-  if (prepare_cluster<D, GT, PAGED>()) {
+  if (prepare_persistent<D, GT, PAGED, true>()) {
     cudaLaunchAttribute attr[1];
-    const cudaLaunchConfig_t cfg = launch_config(dim3(cs * 64), ClusterSmem<D, GT>::BYTES, cs, nullptr, attr);
-    if (cudaOccupancyMaxActiveClusters(&clusters, decode_cluster_kernel<D, GT, PAGED>, &cfg) != cudaSuccess) {
+    const cudaLaunchConfig_t cfg = launch_config(dim3(cs * 64), PersistSmem<D, GT>::BYTES, cs, nullptr, attr);
+    if (cudaOccupancyMaxActiveClusters(&clusters, decode_persistent_kernel<D, GT, PAGED, true>, &cfg) !=
+        cudaSuccess) {
       cudaGetLastError();
       clusters = 0;
     }
   }
   if (dev < 64) cache[dev][cs].store(clusters + 1, std::memory_order_relaxed);
   return clusters;
+}
+
+// CTAs of the persistent split kernel resident on the current device at once (blocks per
+// SM x SMs); 0 if the device cannot be asked.  Cached per device.
+template <int D, int GT, bool PAGED>
+int persistent_slots() {
+  static std::atomic<int> cache[64];  // value + 1 once known
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 0;
+  if (dev < 64) {
+    const int c = cache[dev].load(std::memory_order_relaxed);
+    if (c != 0) return c - 1;
+  }
+  int per_sm = 0, sms = 0;
+  if (!prepare_persistent<D, GT, PAGED, false>() ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_persistent_kernel<D, GT, PAGED, false>,
+                                                    DecodeCfg<D>::THREADS, PersistSmem<D, GT>::BYTES) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+    cudaGetLastError();
+    per_sm = sms = 0;
+  }
+  if (dev < 64) cache[dev].store(per_sm * sms + 1, std::memory_order_relaxed);
+  return per_sm * sms;
 }
 
 // Views of the K and V caches for the split kernels' loaders: paged caches as TMA tensors,
@@ -980,27 +1042,49 @@ cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl
   return cudaGetLastError();
 }
 
+template <int D, int GT, bool PAGED, bool CLUSTER>
+cudaError_t launch_persistent_kernel(const DecodeArgs& a, dim3 grid, int cs, const PagedKV* pk, const KernelCtl& ctl,
+                                     cudaStream_t stream) {
+  if (!prepare_persistent<D, GT, PAGED, CLUSTER>()) return cudaErrorInvalidConfiguration;
+  CUtensorMap tk, tv;
+  PagedView view;
+  if (!kv_views<D, PAGED>(a, pk, &tk, &tv, &view)) return cudaErrorInvalidValue;
+  const int G = a.Hq / a.Hkv;
+  const int n_groups = (G + GT - 1) / GT;
+  cudaLaunchAttribute attr[1];
+  const cudaLaunchConfig_t cfg = launch_config(grid, PersistSmem<D, GT>::BYTES, CLUSTER ? cs : 0, stream, attr);
+  return cudaLaunchKernelEx(&cfg, decode_persistent_kernel<D, GT, PAGED, CLUSTER>,
+                            static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.k),
+                            static_cast<const __nv_bfloat16*>(a.v), a.seqlens, static_cast<__nv_bfloat16*>(a.o),
+                            a.lse, a.o_part, a.lse_part, a.B, a.Hq, a.Hkv, a.Skv, a.splits, n_groups,
+                            a.scale * kLog2e, ctl, tk, tv, view);
+}
+
 // The cluster kernel with clusters of cs CTAs: as many clusters as fit at once, at most one
 // per unit.
 template <int D, int GT, bool PAGED>
 cudaError_t launch_cluster(const DecodeArgs& a, int cs, const PagedKV* pk, const KernelCtl& ctl,
                            cudaStream_t stream) {
   const int fit = max_clusters<D, GT, PAGED>(cs);
-  if (fit < 1 || !prepare_cluster<D, GT, PAGED>()) return cudaErrorInvalidConfiguration;
-  CUtensorMap tk, tv;
-  PagedView view;
-  if (!kv_views<D, PAGED>(a, pk, &tk, &tv, &view)) return cudaErrorInvalidValue;
+  if (fit < 1) return cudaErrorInvalidConfiguration;
   const int G = a.Hq / a.Hkv;
-  const int n_groups = (G + GT - 1) / GT;
-  const long long units = static_cast<long long>(a.B) * a.Hkv * n_groups;
+  const long long units = static_cast<long long>(a.B) * a.Hkv * ((G + GT - 1) / GT);
   const long long n_clusters = units < fit ? units : fit;
-  cudaLaunchAttribute attr[1];
-  const cudaLaunchConfig_t cfg =
-      launch_config(dim3(static_cast<unsigned>(n_clusters * cs)), ClusterSmem<D, GT>::BYTES, cs, stream, attr);
-  return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<D, GT, PAGED>, static_cast<const __nv_bfloat16*>(a.q),
-                            static_cast<const __nv_bfloat16*>(a.k), static_cast<const __nv_bfloat16*>(a.v),
-                            a.seqlens, static_cast<__nv_bfloat16*>(a.o), a.lse, a.B, a.Hq, a.Hkv, a.Skv, a.splits,
-                            n_groups, a.scale * kLog2e, ctl, tk, tv, view);
+  return launch_persistent_kernel<D, GT, PAGED, true>(a, dim3(static_cast<unsigned>(n_clusters * cs)), cs, pk, ctl,
+                                                      stream);
+}
+
+// The persistent split kernel: as many CTAs as fit at once, evened out so that every CTA
+// walks the same number of (unit, split) items (the last round is the only short one).
+template <int D, int GT, bool PAGED>
+cudaError_t launch_persist(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
+  const int slots = persistent_slots<D, GT, PAGED>();
+  if (slots < 1) return cudaErrorInvalidConfiguration;
+  const int G = a.Hq / a.Hkv;
+  const long long items = static_cast<long long>(a.B) * a.Hkv * ((G + GT - 1) / GT) * a.splits;
+  const long long per = (items + slots - 1) / slots;
+  const long long ctas = (items + per - 1) / per;
+  return launch_persistent_kernel<D, GT, PAGED, false>(a, dim3(static_cast<unsigned>(ctas)), 1, pk, ctl, stream);
 }
 
 template <int D>
@@ -1020,23 +1104,41 @@ cudaError_t launch_merge(const DecodeArgs& a, cudaStream_t stream) {
                             static_cast<__nv_bfloat16*>(a.o), a.lse, a.splits);
 }
 
-// The Flash Decode form of a launch: 0 = split + merge kernels, cs > 0 = the cluster kernel
-// with clusters of cs CTAs.  a.fused = -1 forbids the cluster form; a.fused = 1 takes it
-// with the model's cluster size whenever some cluster size runs; a.fused = 0 lets the model
-// decide (Eq. 9 over both forms at the call's split count); a.cluster > 0 pins the size
-// (when it divides the split count and such clusters fit).
+// The Flash Decode form of a launch (Eq. 9 over the forms at the call's split count):
+// kDecodeSplitMerge, kDecodePersistent (both with the merge kernel) or kDecodeCluster with
+// *cs CTAs per cluster.  a.form pins a form (0: the model's choice); a pinned form that
+// cannot run falls back to the model's.  a.cluster pins the cluster size (when it divides
+// the split count and such clusters fit).
 template <int D, int GT, bool PAGED>
-int decode_form(const DecodeArgs& a) {
-  if (a.fused < 0) return 0;
+int decode_form(const DecodeArgs& a, int* cs_out) {
+  *cs_out = 0;
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
                                                 cudaSuccess)
-    return 0;
+    return kDecodeSplitMerge;
+  const int slots = persistent_slots<D, GT, PAGED>();
   const model::DecodeClusterChoice ch = model::choose_decode_cluster(
       a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, [](int cs) { return max_clusters<D, GT, PAGED>(cs); }, a.cluster);
-  if (ch.cs == 0) return 0;
-  if (a.fused == 1) return ch.cs;
-  return ch.t_us < model::decode_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms) * (1.0 - 1e-9) ? ch.cs : 0;
+  if (a.form == kDecodeSplitMerge) return kDecodeSplitMerge;
+  if (a.form == kDecodePersistent && slots > 0) return kDecodePersistent;
+  if (a.form == kDecodeCluster && ch.cs > 0) {
+    *cs_out = ch.cs;
+    return kDecodeCluster;
+  }
+  const double t_split = model::decode_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms);
+  const double t_persist =
+      slots > 0 ? model::decode_persistent_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, slots) : 1e300;
+  int form = kDecodeSplitMerge;
+  double best = t_split;
+  if (t_persist < best * (1.0 - 1e-9)) {
+    form = kDecodePersistent;
+    best = t_persist;
+  }
+  if (ch.cs > 0 && ch.t_us < best * (1.0 - 1e-9)) {
+    form = kDecodeCluster;
+    *cs_out = ch.cs;
+  }
+  return form;
 }
 
 // Stage plans compiled beside the model's for the block-size ablation (contiguous cache,
@@ -1069,9 +1171,11 @@ cudaError_t launch_ablation(const DecodeArgs& a, const KernelCtl& ctl, cudaStrea
 template <int D, int GT, bool PAGED>
 cudaError_t launch_form(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
   if (D == 128 && GT == 4 && !PAGED && a.stage_plan > 0) return launch_ablation(a, ctl, stream);
-  const int cs = decode_form<D, GT, PAGED>(a);
-  if (cs > 0) return launch_cluster<D, GT, PAGED>(a, cs, pk, ctl, stream);
-  const cudaError_t e = launch_split<D, GT, PAGED>(a, pk, ctl, stream);
+  int cs = 0;
+  const int form = decode_form<D, GT, PAGED>(a, &cs);
+  if (form == kDecodeCluster) return launch_cluster<D, GT, PAGED>(a, cs, pk, ctl, stream);
+  const cudaError_t e = form == kDecodePersistent ? launch_persist<D, GT, PAGED>(a, pk, ctl, stream)
+                                                  : launch_split<D, GT, PAGED>(a, pk, ctl, stream);
   if (e != cudaSuccess) return e;
   return launch_merge<D>(a, stream);
 }
@@ -1086,12 +1190,20 @@ cudaError_t launch_decode_d(const DecodeArgs& a, const PagedKV* pk, const Kernel
 }
 
 template <int D, bool PAGED>
-int decode_form_d(const DecodeArgs& a) {
+int decode_form_d(const DecodeArgs& a, int* cs) {
   const int G = a.Hq / a.Hkv;
-  if (G >= 8) return decode_form<D, 8, PAGED>(a);
-  if (G >= 4) return decode_form<D, 4, PAGED>(a);
-  if (G >= 2) return decode_form<D, 2, PAGED>(a);
-  return decode_form<D, 1, PAGED>(a);
+  if (G >= 8) return decode_form<D, 8, PAGED>(a, cs);
+  if (G >= 4) return decode_form<D, 4, PAGED>(a, cs);
+  if (G >= 2) return decode_form<D, 2, PAGED>(a, cs);
+  return decode_form<D, 1, PAGED>(a, cs);
+}
+
+template <int D>
+int persistent_slots_d(int G) {
+  if (G >= 8) return persistent_slots<D, 8, false>();
+  if (G >= 4) return persistent_slots<D, 4, false>();
+  if (G >= 2) return persistent_slots<D, 2, false>();
+  return persistent_slots<D, 1, false>();
 }
 
 template <int D>
@@ -1117,10 +1229,12 @@ cudaError_t launch_decode_paged(const DecodeArgs& a, const PagedKV& pk, const Ke
   return launch_decode_d<64, true>(a, &pk, ctl, stream);
 }
 
-int decode_cluster_form(const DecodeArgs& a, bool paged) {
-  if (a.D == 128) return paged ? decode_form_d<128, true>(a) : decode_form_d<128, false>(a);
-  return paged ? decode_form_d<64, true>(a) : decode_form_d<64, false>(a);
+int decode_form_of(const DecodeArgs& a, bool paged, int* cs) {
+  if (a.D == 128) return paged ? decode_form_d<128, true>(a, cs) : decode_form_d<128, false>(a, cs);
+  return paged ? decode_form_d<64, true>(a, cs) : decode_form_d<64, false>(a, cs);
 }
+
+int decode_persistent_slots(int D, int G) { return D == 128 ? persistent_slots_d<128>(G) : persistent_slots_d<64>(G); }
 
 int decode_max_clusters(int D, int G, int cs) { return D == 128 ? max_clusters_d<128>(G, cs) : max_clusters_d<64>(G, cs); }
 

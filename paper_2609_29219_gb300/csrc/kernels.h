@@ -46,7 +46,7 @@ struct DecodeArgs {
   float* lse_part;          // [B, Hq, splits] fp32 (workspace)
   int B, Hq, Hkv, Skv, D, splits;
   float scale;
-  int fused;    // 0: the model's form; 1: the cluster form wherever it can run; -1: split + merge kernels
+  int form;     // 0: the model's form; else a kDecode* form (when it can run)
   int cluster;  // cluster form: 0 = the model's cluster size, else this size (if it divides splits and fits)
   int stage_plan;  // 0: the model's stage plan; i > 0: the i-th compiled ablation plan (split + merge form)
 };
@@ -84,9 +84,15 @@ int decode_check_args(const void* q, const void* k_cache, const void* v_cache, c
                       int num_splits, int* splits);
 
 cudaError_t launch_decode(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream);
-// The form a decode launch with these arguments runs: 0 = split + merge kernels, cs > 0 =
-// the single-kernel cluster form with clusters of cs CTAs.
-int decode_cluster_form(const DecodeArgs& a, bool paged);
+// Flash Decode forms: a split kernel of one CTA per (split, unit) + the merge kernel; a
+// persistent split kernel walking (unit, split) items + the merge kernel; one persistent
+// kernel whose clusters merge over distributed shared memory.
+constexpr int kDecodeSplitMerge = 1, kDecodePersistent = 2, kDecodeCluster = 3;
+// The form a decode launch with these arguments runs (and, for the cluster form, its
+// cluster size in *cs).
+int decode_form_of(const DecodeArgs& a, bool paged, int* cs);
+// CTAs of the persistent split kernel resident at once on the current device (0: unknown).
+int decode_persistent_slots(int D, int G);
 // Clusters of cs cluster-decode CTAs (G query heads per kv head) resident at once on the
 // current device; 0 if none fit or the device cannot be asked.
 int decode_max_clusters(int D, int G, int cs);

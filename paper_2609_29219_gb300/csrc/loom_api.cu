@@ -30,7 +30,7 @@ int g_gemm_tile_n = 0;  // test hook: forced GEMM tile width (0: the model's cho
 int g_gemm_splits = 0;  // test hook: forced GEMM split count (0: the model's choice)
 int g_gemm_pair = 0;    // test hook: 1 forces CTA-pair tiles, -1 forbids them, 0: the model's choice
 int g_gemm_stages = 0;  // test hook: GEMM ring depth (0: the model's; a compiled neighbour otherwise)
-int g_decode_fused = 0;    // test hook: 1 forces the cluster decode form, -1 forbids it, 0: the model's choice
+int g_decode_form = 0;     // test hook: the Flash Decode form (0: the model's; kDecode* otherwise)
 int g_decode_cluster = 0;  // test hook: the cluster decode form's cluster size (0: the model's)
 int g_decode_stage_plan = 0;  // test hook: a compiled ablation stage plan of the decode split kernel
 
@@ -134,9 +134,14 @@ int loom_attn_decode_num_splits(int B, int Hq, int Hkv, int Skv, int D) {
   // device, or from the GB300 estimate when no device answers.
   const bool device = current_sm_count() > 0;
   const int G = Hq / Hkv;
-  const int splits = model::choose_decode_plan(B, Hq, Hkv, Skv, D, sms, [&](int cs) {
-                       return device ? decode_max_clusters(D, G, cs) : model::decode_default_clusters(sms, cs, D);
-                     }).splits;
+  const int slots = device ? decode_persistent_slots(D, G) : sms * model::decode_stage(D).ctas_per_sm;
+  const int splits = model::choose_decode_plan(
+                         B, Hq, Hkv, Skv, D, sms,
+                         [&](int cs) {
+                           return device ? decode_max_clusters(D, G, cs) : model::decode_default_clusters(sms, cs, D);
+                         },
+                         slots)
+                         .splits;
   std::lock_guard<std::mutex> lock(g_split_mutex);
   if (g_split_cache.size() >= 256) g_split_cache.erase(g_split_cache.begin());
   g_split_cache.emplace_back(key, splits);
@@ -199,7 +204,7 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D,
-               num_splits, scale, g_decode_fused, g_decode_cluster, g_decode_stage_plan};
+               num_splits, scale, g_decode_form, g_decode_cluster, g_decode_stage_plan};
   return launch_decode(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                  : LOOM_ERR_CUDA;
 }
@@ -269,7 +274,7 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D, num_splits, scale,
-               g_decode_fused, g_decode_cluster, 0};
+               g_decode_form, g_decode_cluster, 0};
   PagedKV pk{block_table, num_pages, page_size, max_pages, kv_layout};
   return launch_decode_paged(a, pk, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                           : LOOM_ERR_CUDA;
@@ -419,7 +424,8 @@ double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, in
   return model::decode_time_us(splits, B, Hq, Hkv, Skv, D, num_sms);
 }
 
-int loom_attn_decode_cluster_form(int B, int Hq, int Hkv, int Skv, int D, int num_splits, int paged) {
+int loom_attn_decode_form(int B, int Hq, int Hkv, int Skv, int D, int num_splits, int paged, int* cluster) {
+  if (cluster) *cluster = 0;
   if (B <= 0 || Hq <= 0 || Hkv <= 0 || Skv <= 0 || Hq % Hkv != 0 || (D != 64 && D != 128) || num_splits < 0 ||
       num_splits > kMaxDecodeSplits)
     return -1;
@@ -432,11 +438,13 @@ int loom_attn_decode_cluster_form(int B, int Hq, int Hkv, int Skv, int D, int nu
   a.Skv = Skv;
   a.D = D;
   a.splits = num_splits;
-  a.fused = g_decode_fused;
+  a.form = g_decode_form;
   a.cluster = g_decode_cluster;
-  const int cs = decode_cluster_form(a, paged != 0);
+  int cs = 0;
+  const int form = decode_form_of(a, paged != 0, &cs);
   cudaGetLastError();
-  return cs;
+  if (cluster) *cluster = cs;
+  return form;
 }
 
 double loom_model_decode_cluster_time_us(int splits, int cluster, int B, int Hq, int Hkv, int Skv, int D,
@@ -448,6 +456,12 @@ double loom_model_decode_cluster_time_us(int splits, int cluster, int B, int Hq,
   return t > 1e299 ? -1.0 : t;
 }
 
+double loom_model_decode_persistent_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int ctas) {
+  if (splits <= 0 || B <= 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv || Skv <= 0 || ctas <= 0 || (D != 64 && D != 128))
+    return -1.0;
+  return model::decode_persistent_time_us(splits, B, Hq, Hkv, Skv, D, ctas);
+}
+
 int loom_decode_max_clusters(int D, int G, int cluster) {
   if ((D != 64 && D != 128) || G <= 0 || cluster <= 0 || cluster > model::kMaxClusterSize) return 0;
   const int sms = current_sm_count();
@@ -457,8 +471,17 @@ int loom_decode_max_clusters(int D, int G, int cluster) {
   return n;
 }
 
-void loom_debug_decode_cluster(int mode, int cluster) {
-  g_decode_fused = (mode == 1 || mode == -1) ? mode : 0;
+int loom_decode_persistent_slots(int D, int G) {
+  if ((D != 64 && D != 128) || G <= 0) return 0;
+  const int sms = current_sm_count();
+  if (sms <= 0) return model::kGb300.num_sms * model::decode_stage(D).ctas_per_sm;
+  const int n = decode_persistent_slots(D, G);
+  cudaGetLastError();
+  return n;
+}
+
+void loom_debug_decode_form(int form, int cluster) {
+  g_decode_form = (form == kDecodeSplitMerge || form == kDecodePersistent || form == kDecodeCluster) ? form : 0;
   g_decode_cluster = (cluster >= 1 && cluster <= model::kMaxClusterSize) ? cluster : 0;
 }
 

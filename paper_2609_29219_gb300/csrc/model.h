@@ -48,6 +48,8 @@ struct ArchDesc {
   double item_boundary_ns;  // prefill: between two work items of a CTA, the last P.V, the O
                             // read-out and the next item's first S (in-kernel clock trace:
                             // ~2400 clk at the 1.447 GHz reference clock)
+  double decode_item_ns;    // persistent decode: per (unit, split) item, the warps' merge and
+                            // the partial write (assumed)
   double softmax_triple_clk_per_key;  // three tiles' softmax running together (design 4, 96-key
                                       // tiles, 14 warps at 128 registers), clocks per key of a
                                       // round (measured: 876 TFLOP/s on B1 H64 S8192 D64 causal)
@@ -60,7 +62,7 @@ struct ArchDesc {
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 1660.0, 28.4, 300.0,
+    129.0e6, 1.07, 1660.0, 300.0, 28.4, 300.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -407,6 +409,29 @@ constexpr double decode_cluster_time_us(int splits, int cs, int B, int Hq, int H
   return heg_seq(a.cta_start_ns, heg_for(static_cast<double>(cdiv(units, clusters)), per_unit)) * 1e-3;
 }
 
+// Eq. 5 for the persistent split kernel + merge: ctas persistent CTAs walk the units x
+// splits items (ceil(items / ctas) each, as evened out by the launch), each CTA streaming
+// its items back to back at min(its share of HBM, the rate one CTA sustains); the start-up
+// once, a per-item cost for the warps' merge and the partial write (item_ns), then the
+// merge launch of the split + merge form.
+constexpr double decode_persistent_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int slots,
+                                           const ArchDesc& a = kGb300) {
+  if (splits < 1 || slots < 1) return 1e300;
+  const int G = Hq / Hkv;
+  const long long items = 1LL * B * Hkv * cdiv(G, decode_group_tile(G)) * splits;
+  const long long per = cdiv(items, slots);
+  const double ctas = static_cast<double>(cdiv(items, per));
+  const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
+  const double chunk_bytes = 2.0 * chunk * D * 2;
+  double rate = a.hbm_gbs / ctas;
+  if (rate > a.decode_cta_gbs) rate = a.decode_cta_gbs;
+  const double t_split = heg_seq(a.cta_start_ns, heg_for(static_cast<double>(per),
+                                                         heg_seq(chunk_bytes / rate, a.decode_item_ns)));
+  const double part_bytes = 1.0 * B * Hq * splits * (D + 1) * 4;
+  const double t_merge = a.launch_ns * 0.2 + 2.0 * part_bytes / a.hbm_gbs;
+  return heg_seq(t_split, t_merge) * 1e-3;
+}
+
 // Clusters of cs decode CTAs in one GPC-sized group when no device can be asked: whole
 // clusters in 8 equal groups of SMs at the stage plan's CTAs per SM.
 constexpr int decode_default_clusters(int num_sms, int cs, int D) {
@@ -437,16 +462,22 @@ constexpr DecodeClusterChoice choose_decode_cluster(int splits, int B, int Hq, i
   return best;
 }
 
-// Eq. 9 over both Flash Decode forms and every split count; fit(cs) as above (always 0:
-// the split + merge form alone).  Ties keep the split + merge form and fewer splits.
+// Eq. 9 over the Flash Decode forms and every split count: the split + merge form, the
+// persistent split + merge form on `slots` CTAs (0: not considered) and the cluster form
+// with fit(cs) clusters of cs CTAs (always 0: not considered).  Ties keep the earlier form
+// and fewer splits.  DecodeSplitPlan::cluster: 0 split + merge, -1 persistent, cs cluster.
 template <class Fit>
 constexpr DecodeSplitPlan choose_decode_plan(int B, int Hq, int Hkv, int Skv, int D, int num_sms, Fit fit,
-                                             const ArchDesc& a = kGb300) {
+                                             int slots = 0, const ArchDesc& a = kGb300) {
   DecodeSplitPlan best{1, 1e300, 0};
   const long long max_splits = cdiv(Skv, 64) < 1024 ? cdiv(Skv, 64) : 1024;
   for (int s = 1; s <= max_splits; ++s) {
     const double t = decode_time_us(s, B, Hq, Hkv, Skv, D, num_sms, a);
     if (t < best.t_us * (1.0 - 1e-9)) best = {s, t, 0};
+  }
+  for (int s = 1; slots > 0 && s <= max_splits; ++s) {
+    const double t = decode_persistent_time_us(s, B, Hq, Hkv, Skv, D, slots, a);
+    if (t < best.t_us * (1.0 - 1e-9)) best = {s, t, -1};
   }
   for (int s = 1; s <= max_splits; ++s) {
     const DecodeClusterChoice c = choose_decode_cluster(s, B, Hq, Hkv, Skv, D, fit, 0, a);
@@ -458,7 +489,7 @@ constexpr DecodeSplitPlan choose_decode_plan(int B, int Hq, int Hkv, int Skv, in
 // The split + merge form alone (Eq. 9 over its split counts).
 constexpr DecodeSplitPlan choose_decode_splits(int B, int Hq, int Hkv, int Skv, int D, int num_sms,
                                                const ArchDesc& a = kGb300) {
-  return choose_decode_plan(B, Hq, Hkv, Skv, D, num_sms, [](int) { return 0; }, a);
+  return choose_decode_plan(B, Hq, Hkv, Skv, D, num_sms, [](int) { return 0; }, 0, a);
 }
 
 }  // namespace model

@@ -22,22 +22,23 @@ def loom():
     return m
 
 
-@pytest.fixture(autouse=True, params=[0, 1, -1], ids=["model_form", "cluster_form", "split_merge"])
+@pytest.fixture(autouse=True, params=[0, 1, 2, 3], ids=["model_form", "split_merge", "persistent", "cluster"])
 def form(request, loom):
-    """Every test runs with the model's choice of form, with the cluster form forced (the
-    model's cluster size), and with split + merge kernels forced."""
-    loom.loom_debug_decode_cluster(request.param)
+    """Every test runs with the model's choice of form and with each form forced: split
+    kernel + merge, persistent split kernel + merge, and the single-kernel cluster form (at
+    the model's cluster size)."""
+    loom.loom_debug_decode_form(request.param)
     yield request.param
-    loom.loom_debug_decode_cluster(0)
+    loom.loom_debug_decode_form(0)
 
 
 def _expect_form(loom, form, B, Hq, Hkv, Skv, D, splits):
-    used = loom.loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, splits)
-    if form == -1:
-        assert used == 0
-    elif form == 1:
+    used, cs = loom.loom_attn_decode_form(B, Hq, Hkv, Skv, D, splits)
+    if form:
+        assert used == form
+    if used == loom.DECODE_CLUSTER:
         s = splits or loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
-        assert used >= 1 and s % used == 0
+        assert cs >= 1 and s % cs == 0
 
 
 def _inputs(seed, B, Hq, Hkv, Skv, D):
@@ -84,22 +85,23 @@ def test_every_cluster_size(loom, form, splits, clusters):
     """The cluster form with each cluster size pinned (CTA r takes splits r, r + cs, ...):
     sequences of 0 .. Skv keys over a batch that leaves clusters several units each."""
     import torch
-    if form != 1:
+    if form != 3:
         pytest.skip("cluster sizes are pinned under the forced cluster form")
     B, Hq, Hkv, Skv, D = 9, 16, 4, 4000, 128
     q, k, v = _inputs(splits, B, Hq, Hkv, Skv, D)
     lens = np.array([4000, 0, 1, 63, 65, 1000, 3999, 2048, 777], np.int32)
     o_ref, lse_ref = oracle.attention(q, k, v, seqlens_k=lens)
     for cs in clusters:
-        loom.loom_debug_decode_cluster(1, cs)
-        used = loom.loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, splits)
+        loom.loom_debug_decode_form(3, cs)
+        used, got = loom.loom_attn_decode_form(B, Hq, Hkv, Skv, D, splits)
+        assert used == loom.DECODE_CLUSTER
         if splits % cs == 0 and cs <= 16:
-            assert used == cs
+            assert got == cs
         else:
-            assert used != cs
+            assert got != cs
         o, lse = _run(loom, q, k, v, lens, splits)
         assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"splits={splits} cluster={cs}")
-    loom.loom_debug_decode_cluster(1, 0)
+    loom.loom_debug_decode_form(3, 0)
 
 
 @pytest.mark.parametrize("D", [64, 128])
@@ -131,7 +133,7 @@ def test_partials_match_oracle_split_form(loom, form):
     """The workspace holds the per-split partial (O_i, lse_i) of the Flash Decode form
     (split + merge kernels; the cluster form keeps its partials in shared memory)."""
     import torch
-    loom.loom_debug_decode_cluster(-1)
+    loom.loom_debug_decode_form(1)
     B, Hq, Hkv, Skv, D, S = 2, 8, 2, 1000, 128, 5
     q, k, v = _inputs(9, B, Hq, Hkv, Skv, D)
     lens = np.array([1000, 333], np.int32)

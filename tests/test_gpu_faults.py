@@ -64,6 +64,35 @@ def test_decode_skipped_stage_times_out_and_context_survives(loom):
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "decode after timeout")
 
 
+@pytest.mark.parametrize("lens,splits", [(2048, 2), (160, 5)], ids=["all_items_abort", "one_item_aborts"])
+def test_persistent_decode_skipped_stage_times_out_and_context_survives(loom, lens, splits):
+    """The persistent split kernel: the CTA whose second stage is never filled gives up on
+    it and unwinds; the next call on the same context is correct."""
+    import torch
+    B, Hq, Hkv, Skv, D = 1, 4, 1, 2048, 128
+    q = synth.bf16_normal(38, synth.STREAM_Q, (B, Hq, 1, D))
+    k = synth.bf16_normal(38, synth.STREAM_K, (B, Hkv, Skv, D))
+    v = synth.bf16_normal(38, synth.STREAM_V, (B, Hkv, Skv, D))
+    qd, kd, vd = to_dev(q), to_dev(k), to_dev(v)
+    sl_h = np.array([lens], np.int32)
+    sl = torch.from_numpy(sl_h).cuda()
+    loom.loom_debug_decode_form(2)
+    try:
+        assert loom.loom_attn_decode_form(B, Hq, Hkv, Skv, D, splits)[0] == 2
+
+        def bad():
+            loom.loom_debug_inject(1)
+            loom.loom_attn_decode(qd, kd, vd, sl, num_splits=splits)
+
+        _expect_timeout(loom, bad)
+        o, lse = loom.loom_attn_decode(qd, kd, vd, sl, num_splits=splits, return_lse=True)
+        loom.loom_attn_check_error()
+    finally:
+        loom.loom_debug_decode_form(0)
+    o_ref, lse_ref = oracle.attention(q, k, v, seqlens_k=sl_h)
+    assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "persistent decode after timeout")
+
+
 @pytest.mark.parametrize("lens,splits", [(2048, 2), (160, 2), (2048, 16)], ids=["both_abort", "one_aborts", "c16"])
 def test_cluster_decode_skipped_stage_times_out_and_context_survives(loom, lens, splits):
     """The single-kernel cluster form (one cluster of `splits` CTAs): every CTA with a
@@ -78,9 +107,9 @@ def test_cluster_decode_skipped_stage_times_out_and_context_survives(loom, lens,
     qd, kd, vd = to_dev(q), to_dev(k), to_dev(v)
     sl_h = np.array([lens], np.int32)
     sl = torch.from_numpy(sl_h).cuda()
-    loom.loom_debug_decode_cluster(1, splits)
+    loom.loom_debug_decode_form(3, splits)
     try:
-        assert loom.loom_attn_decode_cluster_form(B, Hq, Hkv, Skv, D, splits) == splits
+        assert loom.loom_attn_decode_form(B, Hq, Hkv, Skv, D, splits) == (3, splits)
 
         def bad():
             loom.loom_debug_inject(1)
@@ -90,7 +119,7 @@ def test_cluster_decode_skipped_stage_times_out_and_context_survives(loom, lens,
         o, lse = loom.loom_attn_decode(qd, kd, vd, sl, num_splits=splits, return_lse=True)
         loom.loom_attn_check_error()
     finally:
-        loom.loom_debug_decode_cluster(0)
+        loom.loom_debug_decode_form(0)
     o_ref, lse_ref = oracle.attention(q, k, v, seqlens_k=sl_h)
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "cluster decode after timeout")
 

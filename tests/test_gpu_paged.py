@@ -26,13 +26,13 @@ def loom():
     m.loom_debug_set_timeout_ns(0)
 
 
-@pytest.fixture(autouse=True, params=[1, -1], ids=["cluster_form", "split_merge"])
+@pytest.fixture(autouse=True, params=[1, 2, 3], ids=["split_merge", "persistent", "cluster"])
 def form(request, loom):
-    """Every test runs with the single-kernel cluster form forced (the model's cluster size)
-    and with split + merge kernels forced."""
-    loom.loom_debug_decode_cluster(request.param)
+    """Every test runs with each Flash Decode form forced: split kernel + merge, persistent
+    split kernel + merge, and the single-kernel cluster form (the model's cluster size)."""
+    loom.loom_debug_decode_form(request.param)
     yield request.param
-    loom.loom_debug_decode_cluster(0)
+    loom.loom_debug_decode_form(0)
 
 
 def paged_case(seed, B, Hq, Hkv, P, lens, D, spare=5, poison=True, shuffle=True):
@@ -146,8 +146,7 @@ def test_batched_serving_shape(loom, form, P, layout):
     lens = synth.decode_lengths(0, B, 4096, 8192)
     q, kc, vc, table, sl = paged_case(0, B, Hq, Hkv, P, lens, D, spare=0, poison=False)
     o, lse = run_paged(loom, q, kc, vc, table, sl, 16, layout)
-    assert (loom.loom_attn_decode_cluster_form(B, Hq, Hkv, table.shape[1] * P, D, 16, paged=True) > 0) == \
-        (form == 1)
+    assert loom.loom_attn_decode_form(B, Hq, Hkv, table.shape[1] * P, D, 16, paged=True)[0] == form
     o_ref, lse_ref = oracle.decode_paged(q, kc, vc, table, sl, page_size=P)
     assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"batched paged P={P} {layout}")
 

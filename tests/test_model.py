@@ -110,19 +110,22 @@ DECODE_SHAPES = [(16, 32, 8, 8192, 128), (1, 32, 8, 131072, 128), (1, 8, 8, 4096
 
 
 def _decode_candidates(loom, B, Hq, Hkv, Skv, D):
-    """Modeled time of every (form, split count) candidate: the two-kernel form for every
-    split count, the cluster form for every split count and cluster size dividing it, with
-    the clusters it is priced at."""
+    """Modeled time of every (form, split count) candidate: the split + merge form and the
+    persistent split + merge form for every split count, the cluster form for every split
+    count and cluster size dividing it, with the CTAs and clusters they are priced at.
+    Form order for ties: split + merge (0), persistent (1), cluster (2)."""
     cands = []
     G = Hq // Hkv
+    slots = loom.loom_decode_persistent_slots(D, G)
     for s in range(1, min(1024, math.ceil(Skv / 64)) + 1):
         cands.append((loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS), 0, s))
+        cands.append((loom.loom_model_decode_persistent_time_us(s, B, Hq, Hkv, Skv, D, slots), 1, s))
         for cs in range(1, min(16, s) + 1):
             if s % cs:
                 continue
             t = loom.loom_model_decode_cluster_time_us(s, cs, B, Hq, Hkv, Skv, D, loom.loom_decode_max_clusters(D, G, cs))
             if t > 0:
-                cands.append((t, cs, s))
+                cands.append((t, 2, s))
     return cands
 
 
@@ -132,8 +135,8 @@ def test_decode_split_is_brute_force_argmin(loom, B, Hq, Hkv, Skv, D):
     chosen = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
     cands = _decode_candidates(loom, B, Hq, Hkv, Skv, D)
     best = min(t for t, _, _ in cands)
-    winners = [(f > 0, s, f) for t, f, s in cands if t <= best * (1 + 1e-9)]
-    assert min(winners)[1] == chosen              # ties: the two-kernel form, then the fewest splits
+    winners = sorted((f, s) for t, f, s in cands if t <= best * (1 + 1e-9))
+    assert winners[0][1] == chosen                # ties: the earlier form, then the fewest splits
 
 
 def test_cluster_form_limits(loom):
