@@ -352,7 +352,9 @@ constexpr int decode_group_tile(int G) { return G >= 8 ? 8 : G >= 4 ? 4 : G >= 2
 // The split loop of Flash Decode (Eq. 6-7 with an open load boundary), evaluated on the
 // busiest SM: it runs ceil(CTAs / SMs) split CTAs in rounds of at most CTAs-per-SM at a
 // time; a round of k CTAs streams at min(the SM's share of HBM / k, the rate one CTA
-// sustains), and each round pays the CTA start-up (launch and first copies).
+// sustains).  The first round pays the CTA start-up (launch and first copies); a later
+// round's start-ups overlap the streaming of the CTAs still running on the SM (the
+// hardware launches a CTA as soon as one leaves), so they cost nothing more.
 constexpr double decode_split_loop_ns(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms,
                                       const ArchDesc& a) {
   const DecodeStagePlan& sp = decode_stage(D);
@@ -366,14 +368,27 @@ constexpr double decode_split_loop_ns(int splits, int B, int Hq, int Hkv, int Sk
   const double active_sms = static_cast<double>(ctas < num_sms ? ctas : num_sms);
   const double share = a.hbm_gbs / active_sms;  // bytes/ns for one SM
   double t_split = 0.0;
+  bool first = true;
   for (long long left = per_sm; left > 0;) {
     const long long k = left < sp.ctas_per_sm ? left : sp.ctas_per_sm;
     left -= k;
     double bw = share / static_cast<double>(k);
     if (bw > a.decode_cta_gbs) bw = a.decode_cta_gbs;
-    t_split += heg_seq(a.cta_start_ns, chunk_bytes / bw);
+    t_split += heg_seq(first ? a.cta_start_ns : 0.0, chunk_bytes / bw);
+    first = false;
   }
   return t_split;
+}
+
+// Stream rate (bytes/ns) of one of `ctas` CTAs resident at once: the busiest SM holds
+// ceil(ctas / SMs) of them and they share its part of HBM, up to the rate one CTA sustains.
+constexpr double decode_cta_rate(double ctas, int num_sms, const ArchDesc& a) {
+  const double active = ctas < num_sms ? ctas : static_cast<double>(num_sms);
+  long long k = static_cast<long long>(ctas / num_sms);
+  if (static_cast<double>(k) * num_sms < ctas) ++k;
+  if (k < 1) k = 1;
+  const double rate = a.hbm_gbs / active / static_cast<double>(k);
+  return rate < a.decode_cta_gbs ? rate : a.decode_cta_gbs;
 }
 
 // Eq. 5 for Flash Decode in the split + merge form: T = T_split-loop ; T_merge (gather +
@@ -403,8 +418,7 @@ constexpr double decode_cluster_time_us(int splits, int cs, int B, int Hq, int H
   const double ctas = static_cast<double>(clusters * cs);
   const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
   const double cta_unit_bytes = static_cast<double>(splits / cs) * 2.0 * chunk * D * 2;
-  double rate = a.hbm_gbs / ctas;
-  if (rate > a.decode_cta_gbs) rate = a.decode_cta_gbs;
+  const double rate = decode_cta_rate(ctas, a.num_sms, a);
   const double per_unit = heg_seq(cta_unit_bytes / rate, a.cluster_merge_ns * cs);
   return heg_seq(a.cta_start_ns, heg_for(static_cast<double>(cdiv(units, clusters)), per_unit)) * 1e-3;
 }
@@ -423,8 +437,7 @@ constexpr double decode_persistent_time_us(int splits, int B, int Hq, int Hkv, i
   const double ctas = static_cast<double>(cdiv(items, per));
   const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
   const double chunk_bytes = 2.0 * chunk * D * 2;
-  double rate = a.hbm_gbs / ctas;
-  if (rate > a.decode_cta_gbs) rate = a.decode_cta_gbs;
+  const double rate = decode_cta_rate(ctas, a.num_sms, a);
   const double t_split = heg_seq(a.cta_start_ns, heg_for(static_cast<double>(per),
                                                          heg_seq(chunk_bytes / rate, a.decode_item_ns)));
   const double part_bytes = 1.0 * B * Hq * splits * (D + 1) * 4;
