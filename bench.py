@@ -807,93 +807,41 @@ def run_model_sweep(torch, loom, dev, stream, args, peaks):
         torch.cuda.empty_cache()
     decode = [(1, 32, 8, 131072, 128), (1, 32, 8, 32768, 128), (4, 32, 8, 16384, 128), (16, 32, 8, 8192, 128),
               (64, 32, 8, 2048, 128), (1, 64, 16, 65536, 64)]
+    names = {1: "split+merge", 2: "persistent+merge", 3: "cluster"}
     for B, Hq, Hkv, Skv, D in decode:
         wl = Decode("sweep", B, Hq, Hkv, Skv, D, splits=0)
         wl.setup(torch, dev, loom)
+        G = Hq // Hkv
+        slots = loom.loom_decode_persistent_slots(D, G)
+        fits = {cs: loom.loom_decode_max_clusters(D, G, cs) for cs in range(1, 17)}
         n = min(1024, (Skv + 63) // 64)
-        modeled = sorted((loom.loom_model_decode_time_us(sp, B, Hq, Hkv, Skv, D, sms), sp) for sp in range(1, n + 1))
-        for rank, (model_us, sp) in enumerate(modeled[:5]):
+        cands = []  # (modeled us, form, splits, cluster size): Eq. 9's candidates over forms and split counts
+        for sp in range(1, n + 1):
+            cands.append((loom.loom_model_decode_time_us(sp, B, Hq, Hkv, Skv, D, sms), 1, sp, 0))
+            if slots > 0:
+                cands.append((loom.loom_model_decode_persistent_time_us(sp, B, Hq, Hkv, Skv, D, slots), 2, sp, 0))
+            for cs in range(1, min(16, sp) + 1):
+                if sp % cs == 0 and fits[cs] > 0:
+                    t = loom.loom_model_decode_cluster_time_us(sp, cs, B, Hq, Hkv, Skv, D, fits[cs])
+                    if t > 0:
+                        cands.append((t, 3, sp, cs))
+        cands.sort()
+        chosen_splits = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
+        chosen_form = loom.loom_attn_decode_form(B, Hq, Hkv, Skv, D, 0)
+        for rank, (model_us, form, sp, cs) in enumerate(cands[:5]):
             wl.splits = sp
             nbytes = loom.loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, sp)
             wl.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+            loom.loom_debug_decode_form(form, cs)
             r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks)
             loom.loom_attn_check_error(stream)
             print(json.dumps({"sweep": "model", "kind": "decode", "workload": wl.describe(), "splits": sp,
-                              "model_rank": rank + 1, "measured_us": round(r["ms_per_step"] * 1e3, 2),
+                              "form": names[form] + (str(cs) if cs else ""), "model_rank": rank + 1,
+                              "library_choice": sp == chosen_splits and (form, cs) == chosen_form,
+                              "measured_us": round(r["ms_per_step"] * 1e3, 2),
                               "model_us": round(model_us, 2), "measured_gbs": r["value"],
                               "model_gbs": round(wl.bytes / (model_us * 1e-6) / 1e9, 1)}), flush=True)
-        wl.inp = None
-        torch.cuda.empty_cache()
-
-
-def run_ablation_sweep(torch, loom, dev, stream, args, peaks):
-    """The paper's block-size ablation restated for this path: around each constant the
-    analytic model fixes (the prefill K/V ring depth, the decode stage plan, the GEMM ring
-    depth), every neighbour that is compiled is timed on the benchmark workloads beside the
-    model's choice (is the model's point locally best?)."""
-    steps = max(10, args.steps // 4)
-
-    def line(kind, wl, param, model, r):
-        print(json.dumps({"sweep": "ablation", "kind": kind, "workload": wl.describe(), "param": param,
-                          "model_choice": model, "measured_ms": round(r["ms_per_step"], 5), "value": r["value"],
-                          "unit": r["unit"], "frac": r["roofline"]["frac"]}), flush=True)
-
-    # prefill: ring depth of the two-tile design (BN = 128 keys is fixed by the softmax layout)
-    lens = synth.decode_lengths(0, 16, 4096, 8192)
-    prefill = [(Prefill("prefill", 4, 32, 32, 2048, 128, causal=False), (2, 3)),
-               (Prefill("prefill_causal", 4, 32, 32, 2048, 128, causal=True), (2, 3)),
-               (Prefill("long_prefill_d128", 1, 32, 8, 8192, 128, causal=True), (2, 3)),
-               (Prefill("long_prefill_d64", 1, 64, 16, 8192, 64, causal=True), (3, 6, 9, 10)),
-               (Prefill("prefill_d64", 4, 32, 32, 2048, 64, causal=False), (3, 6, 9, 10))]
-    for wl, depths in prefill:
-        wl.setup(torch, dev, loom)
-        model_depth = loom.loom_model_fwd_plan_variant(wl.D, 2)["kv_slots"]
-        for d in depths:
-            assert loom.loom_debug_prefill_slots(wl.D, d)
-            r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks)
-            loom.loom_attn_check_error(stream)
-            line("prefill_ring_depth", wl, {"kv_slots": d}, d == model_depth, r)
-        loom.loom_debug_prefill_slots(wl.D, 0)
-        wl.inp = None
-        torch.cuda.empty_cache()
-
-    # decode: keys per stage x ring stages x CTAs per SM of the split kernel (split + merge form)
-    plans = [(64, 3, 2), (32, 2, 2), (32, 3, 2), (32, 4, 2), (64, 2, 2), (64, 4, 1), (128, 2, 1), (128, 3, 1)]
-    loom.loom_debug_decode_form(1)
-    for wl in (Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
-               Decode("long_decode", 1, 32, 8, 131072, 128, splits=0)):
-        wl.setup(torch, dev, loom)
-        for i, (t, st, c) in enumerate(plans):
-            assert loom.loom_debug_decode_stage_plan(t, st, c)
-            r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks)
-            loom.loom_attn_check_error(stream)
-            line("decode_stage_plan", wl, {"tokens": t, "stages": st, "ctas_per_sm": c}, i == 0, r)
-        loom.loom_debug_decode_stage_plan(0)
-        wl.inp = None
-        torch.cuda.empty_cache()
-    loom.loom_debug_decode_form(0)
-
-    # GEMM: K-stage ring depth of the kernel the model picks (deeper rings do not fit)
-    for (M, N, K), kernel, depths in [((8192, 8192, 8192), "pair", (5, 6)), ((16384, 16384, 16384), "pair", (5, 6)),
-                                      ((4096, 4096, 4096), 256, (3, 4)), ((2048, 2048, 16384), 128, (5, 6))]:
-        wl = Gemm("ablation", M, N, K)
-        wl.setup(torch, dev, loom)
-        if kernel == "pair":
-            loom.loom_debug_gemm_cta_pair(1)
-        else:
-            loom.loom_debug_gemm_cta_pair(-1)
-            loom.loom_debug_gemm_tile_n(kernel)
-            loom.loom_debug_gemm_splits(1)
-        for d in depths:
-            loom.loom_debug_gemm_stages(d if d != max(depths) else 0)
-            r = measure(torch, wl, max(10, min(steps, 200)), args.warmup, stream, lambda: None, 1, float, peaks,
-                        warm_s=0.25)
-            loom.loom_attn_check_error(stream)
-            line("gemm_ring_depth", wl, {"kernel": kernel, "stages": d}, d == max(depths), r)
-        loom.loom_debug_gemm_stages(0)
-        loom.loom_debug_gemm_cta_pair(0)
-        loom.loom_debug_gemm_tile_n(0)
-        loom.loom_debug_gemm_splits(0)
+        loom.loom_debug_decode_form(0)
         wl.inp = None
         torch.cuda.empty_cache()
 

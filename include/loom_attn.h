@@ -130,6 +130,8 @@ size_t loom_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int Skv, int D, 
  *      merge their partials over distributed shared memory; it leaves the workspace
  *      untouched, but the call checks and requires it all the same.
  * All three follow the split rule above and give the same result up to rounding order.
+ * With num_splits = 0 the model picks the split count and the form together (Eq. 9 over
+ * both); a split count the caller fixes runs form 1 (loom_debug_decode_form pins another).
  * Errors: INVALID_ARG, UNSUPPORTED, MISALIGNED, WORKSPACE, CUDA.
  */
 loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_cache,

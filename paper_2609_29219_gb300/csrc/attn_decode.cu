@@ -1104,14 +1104,16 @@ cudaError_t launch_merge(const DecodeArgs& a, cudaStream_t stream) {
                             static_cast<__nv_bfloat16*>(a.o), a.lse, a.splits);
 }
 
-// The Flash Decode form of a launch (Eq. 9 over the forms at the call's split count):
-// kDecodeSplitMerge, kDecodePersistent (both with the merge kernel) or kDecodeCluster with
-// *cs CTAs per cluster.  a.form pins a form (0: the model's choice); a pinned form that
-// cannot run falls back to the model's.  a.cluster pins the cluster size (when it divides
-// the split count and such clusters fit).
+// The Flash Decode form of a launch: kDecodeSplitMerge, kDecodePersistent (both with the
+// merge kernel) or kDecodeCluster with *cs CTAs per cluster.  A split count the caller fixed
+// runs the split + merge form; a split count the model chose comes with the model's form
+// (Eq. 9 over the forms at that count, which is the form of the joint argmin).  a.form
+// pins a form (a pinned form that cannot run falls back to the rule above); a.cluster pins
+// the cluster size (when it divides the split count and such clusters fit).
 template <int D, int GT, bool PAGED>
 int decode_form(const DecodeArgs& a, int* cs_out) {
   *cs_out = 0;
+  if (a.form == 0 && !a.by_model) return kDecodeSplitMerge;
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
                                                 cudaSuccess)

@@ -49,6 +49,7 @@ struct DecodeArgs {
   int form;     // 0: the model's form; else a kDecode* form (when it can run)
   int cluster;  // cluster form: 0 = the model's cluster size, else this size (if it divides splits and fits)
   int stage_plan;  // 0: the model's stage plan; i > 0: the i-th compiled ablation plan (split + merge form)
+  int by_model;    // 1: the split count is the model's (num_splits = 0), which then also picks the form
 };
 
 struct FwdArgs {

@@ -191,6 +191,7 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
                              const int32_t* seqlens_k, void* o, float* lse, void* workspace,
                              size_t workspace_bytes, int B, int Hq, int Hkv, int Skv, int D,
                              float scale, int num_splits, void* stream) {
+  const int by_model = num_splits == 0 ? 1 : 0;
   const int st = decode_check_args(q, k_cache, v_cache, seqlens_k, o, lse, B, Hq, Hkv, Skv, D, scale, num_splits,
                                    &num_splits);
   if (st != LOOM_OK) return static_cast<loom_status>(st);
@@ -204,7 +205,7 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D,
-               num_splits, scale, g_decode_form, g_decode_cluster, g_decode_stage_plan};
+               num_splits, scale, g_decode_form, g_decode_cluster, g_decode_stage_plan, by_model};
   return launch_decode(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                  : LOOM_ERR_CUDA;
 }
@@ -262,6 +263,7 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
       (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
     return LOOM_ERR_MISALIGNED;
   const int Skv = max_pages * page_size;
+  const int by_model = num_splits == 0 ? 1 : 0;
   if (num_splits == 0) num_splits = loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D);
   if (num_splits <= 0) return LOOM_ERR_INVALID_ARG;
   const size_t need = decode_workspace_bytes(B, Hq, D, num_splits);
@@ -274,7 +276,7 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D, num_splits, scale,
-               g_decode_form, g_decode_cluster, 0};
+               g_decode_form, g_decode_cluster, 0, by_model};
   PagedKV pk{block_table, num_pages, page_size, max_pages, kv_layout};
   return launch_decode_paged(a, pk, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                           : LOOM_ERR_CUDA;
@@ -429,9 +431,11 @@ int loom_attn_decode_form(int B, int Hq, int Hkv, int Skv, int D, int num_splits
   if (B <= 0 || Hq <= 0 || Hkv <= 0 || Skv <= 0 || Hq % Hkv != 0 || (D != 64 && D != 128) || num_splits < 0 ||
       num_splits > kMaxDecodeSplits)
     return -1;
+  const int by_model = num_splits == 0 ? 1 : 0;
   if (num_splits == 0) num_splits = loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D);
   if (num_splits <= 0) return -1;
   DecodeArgs a{};
+  a.by_model = by_model;
   a.B = B;
   a.Hq = Hq;
   a.Hkv = Hkv;

@@ -66,5 +66,5 @@ extern "C" loom_status loom_attn_decode_noalloc(const void* q, const void* k_cac
   void* scratch = loom::scratch_ptr();
   if (!scratch) return LOOM_ERR_CUDA;
   return loom_attn_decode(q, k_cache, v_cache, seqlens_k, o, lse, scratch, loom::kNoallocScratchBytes,
-                          B, Hq, Hkv, Skv, D, scale, splits, stream);
+                          B, Hq, Hkv, Skv, D, scale, num_splits, stream);
 }

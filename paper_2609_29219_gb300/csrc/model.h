@@ -352,9 +352,7 @@ constexpr int decode_group_tile(int G) { return G >= 8 ? 8 : G >= 4 ? 4 : G >= 2
 // The split loop of Flash Decode (Eq. 6-7 with an open load boundary), evaluated on the
 // busiest SM: it runs ceil(CTAs / SMs) split CTAs in rounds of at most CTAs-per-SM at a
 // time; a round of k CTAs streams at min(the SM's share of HBM / k, the rate one CTA
-// sustains).  The first round pays the CTA start-up (launch and first copies); a later
-// round's start-ups overlap the streaming of the CTAs still running on the SM (the
-// hardware launches a CTA as soon as one leaves), so they cost nothing more.
+// sustains), and each round pays the CTA start-up (launch and first copies).
 constexpr double decode_split_loop_ns(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms,
                                       const ArchDesc& a) {
   const DecodeStagePlan& sp = decode_stage(D);
@@ -368,14 +366,12 @@ constexpr double decode_split_loop_ns(int splits, int B, int Hq, int Hkv, int Sk
   const double active_sms = static_cast<double>(ctas < num_sms ? ctas : num_sms);
   const double share = a.hbm_gbs / active_sms;  // bytes/ns for one SM
   double t_split = 0.0;
-  bool first = true;
   for (long long left = per_sm; left > 0;) {
     const long long k = left < sp.ctas_per_sm ? left : sp.ctas_per_sm;
     left -= k;
     double bw = share / static_cast<double>(k);
     if (bw > a.decode_cta_gbs) bw = a.decode_cta_gbs;
-    t_split += heg_seq(first ? a.cta_start_ns : 0.0, chunk_bytes / bw);
-    first = false;
+    t_split += heg_seq(a.cta_start_ns, chunk_bytes / bw);
   }
   return t_split;
 }

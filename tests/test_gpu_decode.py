@@ -36,6 +36,8 @@ def _expect_form(loom, form, B, Hq, Hkv, Skv, D, splits):
     used, cs = loom.loom_attn_decode_form(B, Hq, Hkv, Skv, D, splits)
     if form:
         assert used == form
+    elif splits:  # a split count the caller fixes runs the split + merge form
+        assert used == loom.DECODE_SPLIT_MERGE
     if used == loom.DECODE_CLUSTER:
         s = splits or loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
         assert cs >= 1 and s % cs == 0
