@@ -48,21 +48,23 @@ struct ArchDesc {
   double item_boundary_ns;  // prefill: between two work items of a CTA, the last P.V, the O
                             // read-out and the next item's first S (in-kernel clock trace:
                             // ~2400 clk at the 1.447 GHz reference clock)
-  double decode_item_ns;    // persistent decode: per (unit, split) item, the warps' merge and
-                            // the partial write (assumed)
+  double decode_item_ns;    // persistent decode: per (unit, split) item, the warps' merge with
+                            // the item's last ring slot held, the partial write and the next
+                            // item's q (fitted: B4 H32/8 S16384 measured 56 / 60 us with one / two
+                            // items per CTA)
   double softmax_triple_clk_per_key;  // three tiles' softmax running together (design 4, 96-key
                                       // tiles, 14 warps at 128 registers), clocks per key of a
                                       // round (measured: 876 TFLOP/s on B1 H64 S8192 D64 causal)
-  double cluster_merge_ns;          // per unit and CTA of a cluster-decode cluster: the warps'
-                                    // merge, the handshakes waiting on the slowest CTA and the
-                                    // DSMEM gather (fitted: 147 / 103 / 93 us measured with
-                                    // clusters of 16 / 8 / 2 on the batched decode)
+  double cluster_merge_ns;          // per unit and CTA of a cluster-decode cluster: the
+                                    // handshakes waiting on the slowest CTA and the DSMEM gather
+                                    // (fitted: 147 us measured with clusters of 16 on the batched
+                                    // decode, 123 us with clusters of 4 on B64 S2048)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 1660.0, 300.0, 28.4, 300.0,
+    129.0e6, 1.07, 1660.0, 3000.0, 28.4, 150.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -401,10 +403,10 @@ constexpr double decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int
 // Eq. 5 for the single-kernel form: persistent clusters of cs CTAs (cs divides the split
 // count); the min(fit_clusters, units) clusters each walk ceil(units / clusters) units, and
 // a CTA streams splits / cs chunks of every unit at min(its share of HBM, the rate one CTA
-// sustains), without a break between units.  Per unit it pays the gather + global softmax +
-// scaling over DSMEM and the handshakes, which wait for the slowest of the cluster's CTAs
-// (cluster_merge_ns per CTA of the cluster); the start-up once.  No merge launch, no
-// workspace.
+// sustains), without a break between units.  Per unit it pays what the persistent split
+// kernel pays per item (decode_item_ns) and the gather + global softmax + scaling over DSMEM
+// with its handshakes, which wait for the slowest of the cluster's CTAs (cluster_merge_ns
+// per CTA of the cluster); the start-up once.  No merge launch, no workspace.
 constexpr double decode_cluster_time_us(int splits, int cs, int B, int Hq, int Hkv, int Skv, int D,
                                         int fit_clusters, const ArchDesc& a = kGb300) {
   if (cs < 1 || cs > kMaxClusterSize || splits < cs || splits % cs != 0 || fit_clusters < 1) return 1e300;
@@ -415,7 +417,7 @@ constexpr double decode_cluster_time_us(int splits, int cs, int B, int Hq, int H
   const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
   const double cta_unit_bytes = static_cast<double>(splits / cs) * 2.0 * chunk * D * 2;
   const double rate = decode_cta_rate(ctas, a.num_sms, a);
-  const double per_unit = heg_seq(cta_unit_bytes / rate, a.cluster_merge_ns * cs);
+  const double per_unit = heg_seq(cta_unit_bytes / rate, heg_seq(a.decode_item_ns, a.cluster_merge_ns * cs));
   return heg_seq(a.cta_start_ns, heg_for(static_cast<double>(cdiv(units, clusters)), per_unit)) * 1e-3;
 }
 
