@@ -342,10 +342,18 @@ void loom_debug_prefill_design(int design);
  * loom_debug_gemm_stages: the GEMM's K-stage ring depth ([K, N] B): the CTA pair with 5
  *   (model: 6), 256-wide persistent tiles with 3 (model: 4), 128-wide with 5 (model: 6);
  *   other values or kernels run the model's depth.  0 restores the model's.
+ * loom_debug_gemm_order: the GEMM's tile order.  group_rows (1..1024; 0: the default, 12
+ *   for CTA-pair tiles and 8 otherwise) tile rows form one group, walked column by column,
+ *   so tiles in flight together share rows of A and columns of B in L2.  The CTA-pair
+ *   kernel walks K from its end in every other round of tiles, so a round starts on the K
+ *   slices the previous round touched last (still in L2); k_alternate = -1 turns that off
+ *   (0 or 1: on).  Either changes only which CTA computes which tile when, and the order of
+ *   the fp32 sum over K blocks.
  */
 int loom_debug_prefill_slots(int D, int slots);
 int loom_debug_decode_stage_plan(int tokens, int stages, int ctas_per_sm);
 void loom_debug_gemm_stages(int stages);
+void loom_debug_gemm_order(int group_rows, int k_alternate);
 
 /*
  * Test hook: the Flash Decode form.  form 1 = split + merge kernels, 2 = persistent split

@@ -65,16 +65,20 @@ struct GemmParams {
   int M, N, K;
   int tiles_m, tiles_n, k_iters;
   int splits;  // split-K kernel: CTAs per cluster (= per tile)
+  int group;   // tile rows per group of the tile order
+  int k_alt;   // CTA-pair kernel: 1 walks K backwards in every other round of tiles
+  int b_blocks;  // B [K, N]: 1 when tm_b views B as 64-column blocks (a stage's B in one box)
   KernelCtl ctl;
 };
 
-// Tile t -> (tm, tn): groups of 8 tile rows, column-major inside a group.
+// Tile t -> (tm, tn): groups of p.group tile rows, column-major inside a group (CTAs
+// working at the same time share A rows and B columns in L2).
 __device__ __forceinline__ void tile_coords(const GemmParams& p, int t, int& tm, int& tn) {
-  constexpr int kGroup = 8;
-  const int per_group = kGroup * p.tiles_n;
+  const int group = p.group;
+  const int per_group = group * p.tiles_n;
   const int g = t / per_group;
-  const int first = g * kGroup;
-  const int rows = min(kGroup, p.tiles_m - first);
+  const int first = g * group;
+  const int rows = min(group, p.tiles_m - first);
   const int in = t - g * per_group;
   tm = first + in % rows;
   tn = in / rows;
@@ -203,6 +207,8 @@ __global__ void __launch_bounds__(GemmCfg<BN, NS>::THREADS, 1)
           tma_load_3d(dst, &tm_a, ks * C::BK, tm * C::BM, 0, bar_full + 8 * s);
           if constexpr (BK_MAJOR) {  // BN rows of B [N, K], 64 K-columns: one box
             tma_load_3d(dst + C::A_BYTES, &tm_b, ks * C::BK, tn * BN, 0, bar_full + 8 * s);
+          } else if (p.b_blocks) {  // the tile's NB 64-column blocks of B [K, N]: one box
+            tma_load_3d(dst + C::A_BYTES, &tm_b, 0, ks * C::BK, tn * C::NB, bar_full + 8 * s);
           } else {
 #pragma unroll
             for (int x = 0; x < C::NB; ++x)
@@ -354,6 +360,8 @@ __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
         tma_load_3d(dst, &tm_a, ks * C::BK, tm * C::BM, 0, bar_full + 8 * s);
         if constexpr (BK_MAJOR) {
           tma_load_3d(dst + C::A_BYTES, &tm_b, ks * C::BK, tn * BN, 0, bar_full + 8 * s);
+        } else if (p.b_blocks) {
+          tma_load_3d(dst + C::A_BYTES, &tm_b, 0, ks * C::BK, tn * C::NB, bar_full + 8 * s);
         } else {
 #pragma unroll
           for (int x = 0; x < C::NB; ++x)
@@ -578,12 +586,14 @@ __global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
     if (lane == 0) {
       prefetch_tensormap(&tm_a);
       prefetch_tensormap(&tm_b);
-      int it = 0, issued = 0, skipped = -1;
+      int it = 0, issued = 0, skipped = -1, lt = 0;
       bool ok = true;
-      for (int t = pair; ok && t < tiles; t += n_pairs) {
+      for (int t = pair; ok && t < tiles; t += n_pairs, ++lt) {
         int tm, tn;
         tile_coords(p, t, tm, tn);
-        for (int ks = 0; ks < p.k_iters; ++ks, ++it) {
+        const bool back = p.k_alt && (lt & 1);
+        for (int kq = 0; kq < p.k_iters; ++kq, ++it) {
+          const int ks = back ? p.k_iters - 1 - kq : kq;
           const int s = it % C::NSTAGE;
           if (!(ok = mbar_wait(bar_empty + 8 * s, ((it / C::NSTAGE) & 1) ^ 1, p.ctl, ab))) break;
           issued = it + 1;
@@ -597,6 +607,8 @@ __global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
           tma_load_3d_pair(dst, &tm_a, ks * C::BK, tm * 256 + static_cast<int>(rank) * C::BM, 0, full0);
           if constexpr (BK_MAJOR) {  // this CTA's 128 rows of B [N, K], 64 K-columns: one box
             tma_load_3d_pair(dst + C::A_BYTES, &tm_b, ks * C::BK, tn * C::BN + static_cast<int>(rank) * 128, 0, full0);
+          } else if (p.b_blocks) {  // both 64-column blocks of this CTA's half in one box
+            tma_load_3d_pair(dst + C::A_BYTES, &tm_b, 0, ks * C::BK, tn * 4 + static_cast<int>(rank) * 2, full0);
           } else {
 #pragma unroll
             for (int x = 0; x < C::NBH; ++x)
@@ -717,6 +729,21 @@ bool set_smem_attr(const void* fn, PerDeviceOnce& done, int dev) {
   });
 }
 
+// B [K, N] with N % 64 == 0 as a 3-D tensor of 64-column blocks: (column in block, K row,
+// block), strides 2 B, 2N B and 128 B; a box of `blocks` blocks x 64 K-rows lands in shared
+// memory as `blocks` consecutive 8 KB (64 x 64, 128B-swizzled) blocks.
+bool b_blocks_map(CUtensorMap* map, const void* base, int K, int N, int blocks) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc || N % 64 != 0) return false;
+  cuuint64_t dims[3] = {64, static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(N / 64)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(N) * 2, 128};
+  cuuint32_t box[3] = {64, 64, static_cast<cuuint32_t>(blocks)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // B's box: 64 columns x 64 K-rows of B [K, N], or 64 K-columns x b_rows rows of B [N, K].
 bool make_maps(const GemmArgs& a, int bm, int b_rows, CUtensorMap* ma, CUtensorMap* mb, CUtensorMap* mc) {
   const bool b_ok = a.b_kmajor ? matrix_map(mb, a.b, a.N, a.K, 64, b_rows) : matrix_map(mb, a.b, a.K, a.N, 64, 64);
@@ -733,8 +760,22 @@ GemmParams make_params(const GemmArgs& a, const KernelCtl& ctl, int bn, int spli
   p.tiles_n = (a.N + bn - 1) / bn;
   p.k_iters = (a.K + 63) / 64;
   p.splits = splits;
+  p.group = a.group > 0 ? a.group : 8;
+  p.k_alt = 0;
+  p.b_blocks = 0;
   p.ctl = ctl;
   return p;
+}
+
+// B [K, N] with N % 64 == 0: one TMA box per stage for all of a stage's 64-column blocks of
+// B instead of one box per block.  Measured on GB300 (CTA pair, 8192^3): 1699 against 1550
+// TFLOP/s with two boxes, level with B given [N, K] (1690), whose stage is one box too.
+void use_b_blocks(const GemmArgs& a, int blocks, CUtensorMap* mb, GemmParams* p) {
+  CUtensorMap m;
+  if (!a.b_kmajor && b_blocks_map(&m, a.b, a.K, a.N, blocks)) {
+    *mb = m;
+    p->b_blocks = 1;
+  }
 }
 
 template <int BN, bool BKM, int NS = 0>
@@ -745,7 +786,8 @@ cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stre
     return cudaErrorInvalidValue;
   CUtensorMap ma, mb, mc;
   if (!make_maps(a, C::BM, BN, &ma, &mb, &mc)) return cudaErrorInvalidValue;
-  const GemmParams p = make_params(a, ctl, BN, 1);
+  GemmParams p = make_params(a, ctl, BN, 1);
+  use_b_blocks(a, C::NB, &mb, &p);
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   const int grid = static_cast<int>(tiles < sms ? tiles : sms);
@@ -819,7 +861,8 @@ cudaError_t launch_splitk(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t 
   if (!prepare_splitk<BN, BKM>(dev)) return cudaErrorInvalidValue;
   CUtensorMap ma, mb;
   if (!make_maps(a, GemmCfg<BN>::BM, BN, &ma, &mb, nullptr)) return cudaErrorInvalidValue;
-  const GemmParams p = make_params(a, ctl, BN, S);
+  GemmParams p = make_params(a, ctl, BN, S);
+  use_b_blocks(a, GemmCfg<BN>::NB, &mb, &p);
   const long long ctas = static_cast<long long>(p.tiles_m) * p.tiles_n * S;
   if (ctas > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   cudaLaunchAttribute attr[1];
@@ -883,6 +926,13 @@ cudaError_t launch_pair(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t st
   if (!make_maps(a, GemmPairCfg::BM, 128, &ma, &mb, &mc)) return cudaErrorInvalidValue;
   GemmParams p = make_params(a, ctl, GemmPairCfg::BN, 1);
   p.tiles_m = (a.M + 255) / 256;  // 256-row tiles of the pair
+  // 76 pairs in flight cover 12 tile rows x 6-7 tile columns; with every other round
+  // walking K backwards, a round starts on the K slices of A the previous round (same rows)
+  // read last.  GB300, 8192^3: 812 MB read from DRAM against 1064 MB in groups of 8 rows
+  // walked forwards (A + B: 268 MB; cuBLAS 1005-1020 MB), time within 1 %.
+  if (a.group <= 0) p.group = 12;
+  p.k_alt = a.k_alt >= 0 ? 1 : 0;
+  use_b_blocks(a, GemmPairCfg::NBH, &mb, &p);
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x3fffffffLL) return cudaErrorInvalidConfiguration;
   const long long pairs = tiles < slots / 2 ? tiles : slots / 2;

@@ -17,6 +17,8 @@ struct GemmArgs {
   int pair;       // 0: the model's choice, 1: CTA-pair 256 x 256 tiles, -1: never CTA pairs
   int b_kmajor;   // 1: b is [N, K] row-major and C = A B^T
   int stages;     // 0: the model's ring depth; a compiled neighbour of it otherwise (block-size ablation)
+  int group;      // tile rows per group of the tile order (0: 12 for CTA-pair tiles, 8 otherwise)
+  int k_alt;      // CTA-pair kernel: K walked backwards in every other round of tiles (0, 1: yes; -1: no)
 };
 
 struct GemmChoice {

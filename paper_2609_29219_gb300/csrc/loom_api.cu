@@ -30,6 +30,8 @@ int g_gemm_tile_n = 0;  // test hook: forced GEMM tile width (0: the model's cho
 int g_gemm_splits = 0;  // test hook: forced GEMM split count (0: the model's choice)
 int g_gemm_pair = 0;    // test hook: 1 forces CTA-pair tiles, -1 forbids them, 0: the model's choice
 int g_gemm_stages = 0;  // test hook: GEMM ring depth (0: the model's; a compiled neighbour otherwise)
+int g_gemm_group = 0;   // test hook: tile rows per group of the GEMM tile order (0: the default)
+int g_gemm_k_alt = 0;   // test hook: -1 stops the CTA-pair GEMM walking K backwards every other round
 int g_decode_form = 0;     // test hook: the Flash Decode form (0: the model's; kDecode* otherwise)
 int g_decode_cluster = 0;  // test hook: the cluster decode form's cluster size (0: the model's)
 int g_decode_stage_plan = 0;  // test hook: a compiled ablation stage plan of the decode split kernel
@@ -290,7 +292,7 @@ loom_status gemm_call(const void* a, const void* b, void* c, int M, int N, int K
   if (K % 8 != 0 || N % 8 != 0) return LOOM_ERR_UNSUPPORTED;  // 16-byte row strides for TMA
   KernelCtl ctl;
   if (!make_ctl(&ctl)) return LOOM_ERR_CUDA;
-  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n, g_gemm_splits, g_gemm_pair, b_kmajor, g_gemm_stages};
+  GemmArgs g{a, b, c, M, N, K, g_gemm_tile_n, g_gemm_splits, g_gemm_pair, b_kmajor, g_gemm_stages, g_gemm_group, g_gemm_k_alt};
   return launch_gemm(g, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK : LOOM_ERR_CUDA;
 }
 }  // namespace
@@ -354,6 +356,11 @@ void loom_debug_gemm_splits(int splits) { g_gemm_splits = model::gemm_split_supp
 void loom_debug_gemm_cta_pair(int mode) { g_gemm_pair = (mode == 1 || mode == -1) ? mode : 0; }
 
 void loom_debug_gemm_stages(int stages) { g_gemm_stages = stages > 0 ? stages : 0; }
+
+void loom_debug_gemm_order(int group_rows, int k_alternate) {
+  g_gemm_group = (group_rows >= 1 && group_rows <= 1024) ? group_rows : 0;
+  g_gemm_k_alt = k_alternate < 0 ? -1 : 0;
+}
 
 loom_status loom_attn_check_error(void* stream) {
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return LOOM_ERR_CUDA;

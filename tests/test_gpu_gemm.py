@@ -76,7 +76,8 @@ def _run(loom, a, b):
 # ---------------------------------------------------------------- persistent tiles (S = 1)
 @pytest.mark.parametrize("tile_n", [0, *TILE_WIDTHS, "pair"], ids=["model", *[f"bn{b}" for b in TILE_WIDTHS], "pair"])
 @pytest.mark.parametrize("M,K,N", [(128, 64, 256), (1, 8, 8), (200, 136, 304), (130, 72, 264), (255, 1000, 520),
-                                   (1000, 1000, 1000), (64, 4096, 64), (2048, 256, 256), (384, 320, 768)])
+                                   (1000, 1000, 1000), (64, 4096, 64), (2048, 256, 256), (384, 320, 768),
+                                   (200, 136, 320), (1000, 1000, 960)])
 def test_full_parity(loom, forced, tile_n, M, K, N):
     if tile_n == "pair":
         forced(0, 0, 1)
@@ -112,7 +113,8 @@ def test_large_full(loom, forced, tile_n, M, K, N):
 # ---------------------------------------------------------------- split-K clusters
 @pytest.mark.parametrize("splits", SPLITS, ids=[f"s{s}" for s in SPLITS])
 @pytest.mark.parametrize("tile_n", TILE_WIDTHS, ids=[f"bn{b}" for b in TILE_WIDTHS])
-@pytest.mark.parametrize("M,K,N", [(128, 1024, 256), (200, 1000, 304), (130, 4096, 520), (384, 2048, 1000)])
+@pytest.mark.parametrize("M,K,N", [(128, 1024, 256), (200, 1000, 304), (130, 4096, 520), (384, 2048, 1000),
+                                   (200, 1000, 320)])
 def test_split_parity(loom, forced, tile_n, splits, M, K, N):
     forced(tile_n, splits)
     a, b = _inputs(3 * M + K + N, M, K, N)
@@ -223,3 +225,21 @@ def test_transposed_b_matches_plain_layout_bitwise(loom, forced):
     c2 = loom.loom_gemm_bf16(a, b.t().contiguous(), b_transposed=True)
     loom.loom_attn_check_error()
     assert torch.equal(c1.view(torch.int16), c2.view(torch.int16))
+
+
+@pytest.mark.parametrize("group,k_alt", [(16, 1), (1, 1), (3, -1), (8, -1)])
+@pytest.mark.parametrize("tile_n", [256, "pair"])
+def test_tile_orders(loom, forced, group, k_alt, tile_n):
+    """Other tile orders (rows per group, K walked backwards every other round) compute the
+    same product: several rounds of tiles per CTA, a ragged K tail and ragged edges."""
+    if tile_n == "pair":
+        forced(0, 0, 1)
+    else:
+        forced(tile_n, 1)
+    loom.loom_debug_gemm_order(group, k_alt)
+    try:
+        for M, K, N in [(4000, 328, 4096), (1000, 200, 2040)]:
+            a, b = _inputs(M + group, M, K, N)
+            _check(_run(loom, a, b), oracle.gemm(a, b), K, f"{M}x{K}x{N} group={group} k_alt={k_alt} {tile_n}")
+    finally:
+        loom.loom_debug_gemm_order(0, 0)
