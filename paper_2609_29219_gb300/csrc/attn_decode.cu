@@ -191,19 +191,18 @@ __device__ __forceinline__ void decode_stage(const uint8_t* ks, const uint8_t* v
     const int tl = warp * C::TW + r * C::TPR + lr.tg;
     const uint4 raw = *reinterpret_cast<const uint4*>(ks + tl * (D * 2) + lr.kl * 16);
     const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
-    float kf[8];
+    float2 kf[4];  // dims (2i, 2i + 1) of this lane's 8
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      kf[2 * i] = bf16lo(w[i]);
-      kf[2 * i + 1] = bf16hi(w[i]);
-    }
+    for (int i = 0; i < 4; ++i) kf[i] = make_float2(bf16lo(w[i]), bf16hi(w[i]));
+    // two-wide fp32 FMAs (one instruction per pair of dims): even and odd dims summed
+    // apart, then added
     float acc[GT];
 #pragma unroll
     for (int h = 0; h < GT; ++h) {
-      float s = 0.f;
+      float2 s = __fmul2_rn(make_float2(qf[h][0], qf[h][1]), kf[0]);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) s = fmaf(qf[h][i], kf[i], s);
-      acc[h] = s;
+      for (int i = 1; i < 4; ++i) s = __ffma2_rn(make_float2(qf[h][2 * i], qf[h][2 * i + 1]), kf[i], s);
+      acc[h] = s.x + s.y;
     }
     const float s = transpose_reduce<C::KL, GT>(acc, lane);
     sc[r] = (tl < ntok) ? s : -INFINITY;
@@ -235,9 +234,13 @@ __device__ __forceinline__ void decode_stage(const uint8_t* ks, const uint8_t* v
   if (__any_sync(0xffffffffu, need)) {
 #pragma unroll
     for (int h = 0; h < GT; ++h) {
-      const float a = alpha_s[h];
+      const float2 a = make_float2(alpha_s[h], alpha_s[h]);
 #pragma unroll
-      for (int d = 0; d < C::VD; ++d) acc_o[h][d] *= a;
+      for (int d = 0; d < C::VD; d += 2) {
+        const float2 r = __fmul2_rn(make_float2(acc_o[h][d], acc_o[h][d + 1]), a);
+        acc_o[h][d] = r.x;
+        acc_o[h][d + 1] = r.y;
+      }
     }
   }
 
@@ -246,17 +249,14 @@ __device__ __forceinline__ void decode_stage(const uint8_t* ks, const uint8_t* v
 #pragma unroll 4
   for (int tt = 0; tt < nmine; ++tt) {
     const int tl = warp * C::TW + tt;
-    float vf[C::VD];
+    float2 vf[C::VD / 2];  // dims (2j, 2j + 1) of this lane's VD
     if constexpr (C::VD == 4) {
       const uint2 raw = *reinterpret_cast<const uint2*>(vs + tl * (D * 2) + lane * 8);
-      vf[0] = bf16lo(raw.x);
-      vf[1] = bf16hi(raw.x);
-      vf[2] = bf16lo(raw.y);
-      vf[3] = bf16hi(raw.y);
+      vf[0] = make_float2(bf16lo(raw.x), bf16hi(raw.x));
+      vf[1] = make_float2(bf16lo(raw.y), bf16hi(raw.y));
     } else {
       const uint32_t raw = *reinterpret_cast<const uint32_t*>(vs + tl * (D * 2) + lane * 4);
-      vf[0] = bf16lo(raw);
-      vf[1] = bf16hi(raw);
+      vf[0] = make_float2(bf16lo(raw), bf16hi(raw));
     }
     float pv[GT];
     if constexpr (GT % 4 == 0) {
@@ -273,9 +273,15 @@ __device__ __forceinline__ void decode_stage(const uint8_t* ks, const uint8_t* v
       for (int h = 0; h < GT; ++h) pv[h] = ps[tt * GT + h];
     }
 #pragma unroll
-    for (int h = 0; h < GT; ++h)
+    for (int h = 0; h < GT; ++h) {
+      const float2 p2 = make_float2(pv[h], pv[h]);
 #pragma unroll
-      for (int d = 0; d < C::VD; ++d) acc_o[h][d] = fmaf(pv[h], vf[d], acc_o[h][d]);
+      for (int j = 0; j < C::VD / 2; ++j) {
+        const float2 r = __ffma2_rn(p2, vf[j], make_float2(acc_o[h][2 * j], acc_o[h][2 * j + 1]));
+        acc_o[h][2 * j] = r.x;
+        acc_o[h][2 * j + 1] = r.y;
+      }
+    }
   }
 }
 
