@@ -45,9 +45,11 @@ struct ArchDesc {
   double mma_issue_busy_factor;     // MMA stream slowdown while high-ILP warps share the SM with
                                     // the MMA warp issuing warp-wide (measured: 546 vs 512 clk
                                     // per 128^3 GEMM; 1338 when a lone lane issues)
-  double item_boundary_ns;  // prefill: between two work items of a CTA, the last P.V, the O
-                            // read-out and the next item's first S (in-kernel clock trace:
-                            // ~2400 clk at the 1.447 GHz reference clock)
+  double item_boundary_ns;  // prefill: per work item of a CTA, the part that does not overlap
+                            // the previous item: its first S -> softmax -> P.V chain, the causal
+                            // diagonal steps and the last P.V with the O read-out (in-kernel
+                            // clock trace of causal B4 H32 S2048: ~6300 clk per item at ~1.9 GHz;
+                            // with fwd_launch_ns fitted to B1 S1024 and B16 S512 non-causal)
   double decode_item_ns;    // persistent decode: per (unit, split) item, the warps' merge with
                             // the item's last ring slot held, the partial write and the next
                             // item's q (fitted: B4 H32/8 S16384 measured 56 / 60 us with one / two
@@ -59,12 +61,16 @@ struct ArchDesc {
                                     // handshakes waiting on the slowest CTA and the DSMEM gather
                                     // (fitted: 147 us measured with clusters of 16 on the batched
                                     // decode, 123 us with clusters of 4 on B64 S2048)
+  double fwd_launch_ns;             // prefill: once per launch, the launch itself, the first Q
+                                    // and K/V loads from HBM and the last item's epilogue
+                                    // (fitted with item_boundary_ns: B1 H32 S1024 measured 23.2 us,
+                                    // B16 H16 S512 45.5 us, one and four items per CTA)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 1660.0, 3000.0, 28.4, 150.0,
+    129.0e6, 1.07, 3400.0, 3000.0, 28.4, 150.0, 7800.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -249,12 +255,12 @@ constexpr int causal_block_layout(int planes, int group, int Skv, int D, int ite
 }
 
 // Modeled time (us) of a whole prefill launch under a plan (Eq. 5-7 over the CTA's
-// items: item boundary ; for(KV tiles, pipe), in waves over the SMs).  The query tiles of
+// items: launch ; for(items, item boundary ; for(KV tiles, pipe))).  The query tiles of
 // an item take turns on the tensor pipe, so a KV-tile step costs a full round of
 // q_tiles iterations even when some tile (causal: the item's upper tiles) has no work left
-// in it: an item costs its slowest tile's KV tiles x q_tiles x t_iter.  The boundary
-// between items (the last P.V, the O read-out and the next item's first S: ~2400 clk in an
-// in-kernel clock trace) is item_boundary_ns.
+// in it: an item costs its slowest tile's KV tiles x q_tiles x t_iter, plus the part of
+// the item that overlaps nothing (item_boundary_ns: its first S -> softmax -> P.V chain,
+// the diagonal steps, the last P.V and the O read-out), and a launch adds fwd_launch_ns.
 constexpr double fwd_time_us(const FwdPlan& p, int B, int Hq, int Sq, int Skv, int D, int causal,
                              const ArchDesc& a = kGb300) {
   (void)D;
@@ -279,9 +285,12 @@ constexpr double fwd_time_us(const FwdPlan& p, int B, int Hq, int Sq, int Skv, i
   }
   item_tiles /= static_cast<double>(groups);
   const double t_item = heg_seq(a.item_boundary_ns, heg_for(item_tiles * p.q_tiles, p.t_iter_ns));
-  const double waves = static_cast<double>(items) / a.num_sms;  // persistent CTAs
-  const double w = waves < 1.0 ? 1.0 : waves;
-  return w * t_item * 1e-3;
+  // Persistent CTAs take whole items.  Equal items (non-causal): the busiest CTA runs
+  // ceil(items / SMs) of them.  Causal items differ in length and the snake dealing evens
+  // the work per CTA out, so the average share is priced (at least one item).
+  const double share = static_cast<double>(items) / a.num_sms;
+  const double w = causal ? (share < 1.0 ? 1.0 : share) : static_cast<double>(cdiv(items, a.num_sms));
+  return heg_seq(a.fwd_launch_ns, w * t_item) * 1e-3;
 }
 
 // ------------------------------------------------------------------ decode
