@@ -68,6 +68,8 @@ struct GemmParams {
   int group;   // tile rows per group of the tile order
   int k_alt;   // CTA-pair kernel: 1 walks K backwards in every other round of tiles
   int b_blocks;  // B [K, N]: 1 when tm_b views B as 64-column blocks (a stage's B in one box)
+  int narrow_from;  // CTA-pair kernel: units from here on are 256 x 128 halves of the last tiles
+  int n_units;      // CTA-pair kernel: work units (whole tiles, then the narrow halves)
   KernelCtl ctl;
 };
 
@@ -538,10 +540,36 @@ __device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
       : "memory");
 }
 
+// Work unit u of the pair kernel: a whole 256 x 256 tile, or (u >= p.narrow_from) one
+// 256 x 128 half of one of the tiles of the last, thinly filled round.  Its tiles are then
+// halved along N, so twice as many pairs take them and the round takes about half as long
+// (no partial sums to combine: the halves are different columns of C).
+struct PairUnit {
+  int tm, col0;  // 256-row tile index, first column of C
+  bool narrow;
+};
+__device__ __forceinline__ PairUnit pair_unit(const GemmParams& p, int u) {
+  PairUnit w;
+  int t = u, half = 0;
+  w.narrow = u >= p.narrow_from;
+  if (w.narrow) {
+    const int v = u - p.narrow_from;
+    t = p.narrow_from + (v >> 1);
+    half = v & 1;
+  }
+  int tn;
+  tile_coords(p, t, w.tm, tn);
+  w.col0 = tn * 256 + half * 128;
+  return w;
+}
+
+// tm_bn: B for a narrow unit's stage, this CTA's 64 columns (K-major: 64 rows of B [N, K];
+// B [K, N] as 64-column blocks: one block; otherwise tm_b's own 64 x 64 box).
 template <bool BK_MAJOR, int NS = 6>
 __global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
-                     const __grid_constant__ CUtensorMap tm_c, const GemmParams p) {
+                     const __grid_constant__ CUtensorMap tm_c, const __grid_constant__ CUtensorMap tm_bn,
+                     const GemmParams p) {
   using C = GemmPairCfgT<NS>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_base = smem_u32(smem_raw);
@@ -558,7 +586,7 @@ __global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
   const uint32_t bar_drain = bar_acce + 16;
   uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::TMEM_PTR_OFF);
   Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
-  const int tiles = p.tiles_m * p.tiles_n;  // 256 x 256 tiles
+  const int units = p.n_units;  // whole tiles, then narrow halves
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::NSTAGE; ++s) {
@@ -586,11 +614,13 @@ __global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
     if (lane == 0) {
       prefetch_tensormap(&tm_a);
       prefetch_tensormap(&tm_b);
+      prefetch_tensormap(&tm_bn);
       int it = 0, issued = 0, skipped = -1, lt = 0;
       bool ok = true;
-      for (int t = pair; ok && t < tiles; t += n_pairs, ++lt) {
-        int tm, tn;
-        tile_coords(p, t, tm, tn);
+      for (int t = pair; ok && t < units; t += n_pairs, ++lt) {
+        const PairUnit w = pair_unit(p, t);
+        const int tm = w.tm;
+        const int bcol = w.col0 + static_cast<int>(rank) * (w.narrow ? 64 : 128);  // this CTA's B columns
         const bool back = p.k_alt && (lt & 1);
         for (int kq = 0; kq < p.k_iters; ++kq, ++it) {
           const int ks = back ? p.k_iters - 1 - kq : kq;
@@ -602,18 +632,26 @@ __global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
             continue;
           }
           const uint32_t full0 = map_shared_rank(bar_full + 8 * s, 0);  // the even CTA's barrier
-          if (rank == 0) mbar_expect_tx(bar_full + 8 * s, 2 * C::STAGE_BYTES);
+          if (rank == 0)
+            mbar_expect_tx(bar_full + 8 * s, 2 * (w.narrow ? C::A_BYTES + C::B_BOX_BYTES : C::STAGE_BYTES));
           const uint32_t dst = sbase + s * C::STAGE_BYTES;
           tma_load_3d_pair(dst, &tm_a, ks * C::BK, tm * 256 + static_cast<int>(rank) * C::BM, 0, full0);
-          if constexpr (BK_MAJOR) {  // this CTA's 128 rows of B [N, K], 64 K-columns: one box
-            tma_load_3d_pair(dst + C::A_BYTES, &tm_b, ks * C::BK, tn * C::BN + static_cast<int>(rank) * 128, 0, full0);
+          if (w.narrow) {  // this CTA's 64 columns of B: one box
+            if constexpr (BK_MAJOR) {
+              tma_load_3d_pair(dst + C::A_BYTES, &tm_bn, ks * C::BK, bcol, 0, full0);
+            } else if (p.b_blocks) {
+              tma_load_3d_pair(dst + C::A_BYTES, &tm_bn, 0, ks * C::BK, bcol / 64, full0);
+            } else {
+              tma_load_3d_pair(dst + C::A_BYTES, &tm_bn, bcol, ks * C::BK, 0, full0);
+            }
+          } else if constexpr (BK_MAJOR) {  // this CTA's 128 rows of B [N, K], 64 K-columns: one box
+            tma_load_3d_pair(dst + C::A_BYTES, &tm_b, ks * C::BK, bcol, 0, full0);
           } else if (p.b_blocks) {  // both 64-column blocks of this CTA's half in one box
-            tma_load_3d_pair(dst + C::A_BYTES, &tm_b, 0, ks * C::BK, tn * 4 + static_cast<int>(rank) * 2, full0);
+            tma_load_3d_pair(dst + C::A_BYTES, &tm_b, 0, ks * C::BK, bcol / 64, full0);
           } else {
 #pragma unroll
             for (int x = 0; x < C::NBH; ++x)
-              tma_load_3d_pair(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b,
-                               tn * C::BN + static_cast<int>(rank) * 128 + x * 64, ks * C::BK, 0, full0);
+              tma_load_3d_pair(dst + C::A_BYTES + x * C::B_BOX_BYTES, &tm_b, bcol + x * 64, ks * C::BK, 0, full0);
           }
         }
       }
@@ -627,14 +665,16 @@ __global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
     // ------------------------------------------------------------------ MMA issuer (even CTA)
     if (rank == 0) {  // the whole warp; one elected lane issues
       constexpr uint32_t idesc = idesc_bf16(256, C::BN, 0, BK_MAJOR ? 0 : 1);
+      constexpr uint32_t idesc_n = idesc_bf16(256, C::BN / 2, 0, BK_MAJOR ? 0 : 1);  // narrow units
       constexpr uint32_t kstep_b = BK_MAJOR ? 2u : 128u;
       const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
       const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, BK_MAJOR ? 16u : C::B_BOX_BYTES, 1024);
       constexpr uint32_t kStage16 = C::STAGE_BYTES >> 4;
       int it = 0, lt = 0;
       bool ok = true;
-      for (int t = pair; ok && t < tiles; t += n_pairs, ++lt) {
+      for (int t = pair; ok && t < units; t += n_pairs, ++lt) {
         const int b = lt & 1, use = lt >> 1;
+        const uint32_t id = t >= p.narrow_from ? idesc_n : idesc;
         if (lt >= 2 && !(ok = mbar_wait_cluster_warp(bar_acce + 8 * b, (use - 1) & 1, p.ctl, ab))) break;
         tc_fence_after();
         const uint32_t d = tmem + static_cast<uint32_t>(b * C::BN);
@@ -645,7 +685,7 @@ __global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
           const uint64_t da = da0 + s * kStage16, db = db0 + s * kStage16;
 #pragma unroll
           for (int kk = 0; kk < C::BK / 16; ++kk)
-            mma_ss_pair(d, da + kk * 2, db + kk * kstep_b, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
+            mma_ss_pair(d, da + kk * 2, db + kk * kstep_b, id, (ks > 0 || kk > 0) ? 1u : 0u);
           tc_commit_pair_both(bar_empty + 8 * s);
         }
         if (!ok) break;
@@ -662,15 +702,18 @@ __global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
     const uint32_t stg = sbase + C::STG_OFF + static_cast<uint32_t>(warp) * C::STG_WARP;
     int lt = 0;
     bool ok = true;
-    for (int t = pair; ok && t < tiles; t += n_pairs, ++lt) {
-      int tm, tn;
-      tile_coords(p, t, tm, tn);
+    for (int t = pair; ok && t < units; t += n_pairs, ++lt) {
+      const PairUnit w = pair_unit(p, t);
       const int b = lt & 1, use = lt >> 1;
       if (!(ok = mbar_wait_warp(bar_acc + 8 * b, use & 1, p.ctl, ab))) break;
       tc_fence_after();
-      epilogue_warp<C::BN / 64>(&tm_c, tmem + lane_addr + static_cast<uint32_t>(b * C::BN), stg, half, tn * C::BN,
-                                tm * 256 + static_cast<int>(rank) * C::BM + quarter * 32, p.M, p.N,
-                                map_shared_rank(bar_acce + 8 * b, 0), true);
+      const uint32_t acc = tmem + lane_addr + static_cast<uint32_t>(b * C::BN);
+      const int row0 = w.tm * 256 + static_cast<int>(rank) * C::BM + quarter * 32;
+      const uint32_t release = map_shared_rank(bar_acce + 8 * b, 0);
+      if (w.narrow)
+        epilogue_warp<C::BN / 128>(&tm_c, acc, stg, half, w.col0, row0, p.M, p.N, release, true);
+      else
+        epilogue_warp<C::BN / 64>(&tm_c, acc, stg, half, w.col0, row0, p.M, p.N, release, true);
     }
     if (lane == 0) bulk_wait_group0();
   }
@@ -763,6 +806,8 @@ GemmParams make_params(const GemmArgs& a, const KernelCtl& ctl, int bn, int spli
   p.group = a.group > 0 ? a.group : 8;
   p.k_alt = 0;
   p.b_blocks = 0;
+  p.narrow_from = 0x7fffffff;
+  p.n_units = 0;
   p.ctl = ctl;
   return p;
 }
@@ -935,10 +980,29 @@ cudaError_t launch_pair(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t st
   use_b_blocks(a, GemmPairCfg::NBH, &mb, &p);
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x3fffffffLL) return cudaErrorInvalidConfiguration;
-  const long long pairs = tiles < slots / 2 ? tiles : slots / 2;
+  // The last round's tiles become two 256 x 128 units each when that round would keep at
+  // most a quarter of the pairs busy.  GB300, same-box A/B: 2304^2 x 8192 (5 of 76 pairs in
+  // the last round) 941 -> 1066-1081 TFLOP/s; with a third or more of the pairs busy the
+  // halves lost 1-3 % (4096^3: 28 pairs, 8192^3: 36): a wide tile in a thinly filled round
+  // runs faster than in a full one.
+  const long long avail = slots / 2;
+  const long long rest = tiles % avail;
+  p.narrow_from = static_cast<int>(tiles);
+  p.n_units = static_cast<int>(tiles);
+  CUtensorMap mbn = mb;  // narrow units' B: one 64-column box per CTA
+  if (rest > 0 && 4 * rest <= avail) {
+    bool ok = true;
+    if (BKM) ok = matrix_map(&mbn, a.b, a.N, a.K, 64, 64);
+    else if (p.b_blocks) ok = b_blocks_map(&mbn, a.b, a.K, a.N, 1);
+    if (ok) {
+      p.narrow_from = static_cast<int>(tiles - rest);
+      p.n_units = static_cast<int>(tiles + rest);
+    }
+  }
+  const long long pairs = p.n_units < avail ? p.n_units : avail;
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = pair_config<NS>(static_cast<int>(2 * pairs), stream, attr);
-  return cudaLaunchKernelEx(&cfg, gemm_pair_kernel<BKM, NS>, ma, mb, mc, p);
+  return cudaLaunchKernelEx(&cfg, gemm_pair_kernel<BKM, NS>, ma, mb, mc, mbn, p);
 }
 
 // Ring depths compiled beside the model's for the block-size ablation ([K, N] B only): the

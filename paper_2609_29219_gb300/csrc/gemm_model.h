@@ -159,14 +159,22 @@ constexpr GemmPlan gemm_pair_plan(const ArchDesc& a = kGb300) {
   return p;
 }
 
-// `pair_ctas` CTAs (whole pairs) fit on the GPU at once.
+// `pair_ctas` CTAs (whole pairs) fit on the GPU at once.  A last round that would keep at
+// most a quarter of the pairs busy runs its tiles as two 256 x 128 halves each (N = 128
+// pair MMAs, each SM loading 64 columns of B: 24 KB per stage), about half a round.
 constexpr double gemm_pair_time_us(long long M, long long N, long long K, int pair_ctas, const ArchDesc& a = kGb300) {
   const GemmPlan p = gemm_pair_plan(a);
   const long long tiles = cdiv(M, 256) * cdiv(N, 256);
   const long long pairs = pair_ctas / 2 > 0 ? pair_ctas / 2 : 1;
-  const long long per_pair = cdiv(tiles, pairs);
-  const double t_tile = dmax(heg_for(cdiv(K, p.bk), p.t_iter_ns), p.t_epi_tile_ns);
-  const double t = heg_seq(heg_seq(p.t_load_ns, heg_for(per_pair, t_tile)), p.t_epi_ns);
+  const long long full = tiles / pairs, rest = tiles % pairs;
+  const long long k_iters = cdiv(K, p.bk);
+  const double t_tile = dmax(heg_for(k_iters, p.t_iter_ns), p.t_epi_tile_ns);
+  const double t_load_n = (128 + 64) * p.bk * 2.0 / a.l2_smem_gbs_sm;
+  const double t_mma_n = (p.bk / 16.0) * dmax(a.mma_clk_per_n * 128, a.mma_min_clk) / a.sm_ghz;
+  const double t_tile_n = dmax(heg_for(k_iters, heg_pipe(t_load_n, t_mma_n, 0.0, 1, 0)),
+                               (kGemmEpiTileNs + 2 * kGemmEpiChunkNs) * kGemmPairEpiFactor);
+  const double last = rest == 0 ? 0.0 : (4 * rest <= pairs ? t_tile_n : t_tile);
+  const double t = heg_seq(heg_seq(p.t_load_ns, heg_seq(heg_for(full, t_tile), last)), p.t_epi_ns);
   return (t + a.launch_ns * 0.2) * 1e-3;
 }
 

@@ -243,3 +243,16 @@ def test_tile_orders(loom, forced, group, k_alt, tile_n):
             _check(_run(loom, a, b), oracle.gemm(a, b), K, f"{M}x{K}x{N} group={group} k_alt={k_alt} {tile_n}")
     finally:
         loom.loom_debug_gemm_order(0, 0)
+
+
+@pytest.mark.parametrize("M,K,N", [(2304, 200, 2304), (2300, 136, 2296), (520, 1000, 264)])
+def test_pair_last_round_in_halves(loom, forced, M, K, N):
+    """CTA pairs whose last round of tiles is thinly filled take those tiles as two 256 x 128
+    halves (81 tiles on 76 pairs; few tiles): full tiles, then halves, ragged edges."""
+    forced(0, 0, 1)
+    a, b = _inputs(M + K, M, K, N)
+    _check(_run(loom, a, b), oracle.gemm(a, b), K, f"{M}x{K}x{N} pair, halved last round")
+    bt = np.ascontiguousarray(b.T)
+    c = loom.loom_gemm_bf16(to_dev(a), to_dev(bt), b_transposed=True)
+    loom.loom_attn_check_error()
+    _check(c.float().cpu().numpy().astype(np.float64), oracle.gemm(a, b), K, f"{M}x{K}x{N} pair B^T")
