@@ -285,6 +285,7 @@ __global__ void __launch_bounds__(320, 1) mix_kernel(long long* out, const uint8
 //   3: scalar FMA and ex2 only (no pack, no sum): MUFU-bound reference
 //   4: variant 0 with every other pair's exponentials on the FMA pipe (exp2_poly)
 //   5: variant 0 with one pair in four on the FMA pipe
+//   6, 7, 8: variant 0 with one pair in 8, 4 or 16 on the FMA pipe in packed form (exp2_poly2)
 template <int V, int CAP_THREADS = 256>
 __global__ void __launch_bounds__(CAP_THREADS, 1) softmax_row_kernel(long long* cyc, float* sink, int iters) {
   if (threadIdx.x >= 256) return;  // extra threads only lower the register cap
@@ -308,15 +309,23 @@ __global__ void __launch_bounds__(CAP_THREADS, 1) softmax_row_kernel(long long* 
     for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], s[120 + g]);
     const float mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
     const float nm = -mx * c;
-    if constexpr (V == 0 || V == 4 || V == 5) {
+    if constexpr (V == 0 || V == 4 || V == 5 || V >= 6) {
       const uint64_t nms2 = f2(nm, nm);
       uint64_t acc[4] = {0, 0, 0, 0};
 #pragma unroll
       for (int i = 0; i < 64; ++i) {
         const uint64_t x = fma2(f2(s[2 * i], s[2 * i + 1]), c2, nms2);
         const bool poly = (V == 4 && (i & 1)) || (V == 5 && (i & 3) == 3);
-        const float p0 = poly ? exp2_poly(f2lo(x)) : ex2(f2lo(x));
-        const float p1 = poly ? exp2_poly(f2hi(x)) : ex2(f2hi(x));
+        const bool poly2 = (V == 6 && (i & 7) == 7) || (V == 7 && (i & 3) == 3) || (V == 8 && (i & 15) == 15);
+        float p0, p1;
+        if (poly2) {
+          const uint64_t pp = exp2_poly2(x);
+          p0 = f2lo(pp);
+          p1 = f2hi(pp);
+        } else {
+          p0 = poly ? exp2_poly(f2lo(x)) : ex2(f2lo(x));
+          p1 = poly ? exp2_poly(f2hi(x)) : ex2(f2hi(x));
+        }
         acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
         keep ^= pack_bf16x2(p0, p1);
       }
@@ -402,7 +411,7 @@ int main() {
   // softmax row step variants: 4 warps (one per SM sub-partition) and 8 warps (two each)
   {
     const int iters = 2000;
-    for (int v = 0; v < 6; ++v)
+    for (int v = 0; v < 9; ++v)
       for (int warps : {4, 8}) {
         auto launch = [&] {
           if (v == 0) softmax_row_kernel<0><<<sms, warps * 32>>>(d, out, iters);
@@ -411,6 +420,9 @@ int main() {
           if (v == 3) softmax_row_kernel<3><<<sms, warps * 32>>>(d, out, iters);
           if (v == 4) softmax_row_kernel<4><<<sms, warps * 32>>>(d, out, iters);
           if (v == 5) softmax_row_kernel<5><<<sms, warps * 32>>>(d, out, iters);
+          if (v == 6) softmax_row_kernel<6><<<sms, warps * 32>>>(d, out, iters);
+          if (v == 7) softmax_row_kernel<7><<<sms, warps * 32>>>(d, out, iters);
+          if (v == 8) softmax_row_kernel<8><<<sms, warps * 32>>>(d, out, iters);
         };
         const double cyc = avg_cycles(launch, d, h, sms);
         if (cyc <= 0) { printf(", \"error\": \"softmax probe failed\"}\n"); return 1; }
@@ -426,6 +438,10 @@ int main() {
       const double cyc = avg_cycles(launch, d, h, sms);
       if (cyc <= 0) { printf(", \"error\": \"softmax probe failed\"}\n"); return 1; }
       printf(", \"softmax_row128_v0_clk_8warps_168regs\": %.1f", cyc / iters);
+      auto launch6 = [&] { softmax_row_kernel<6, 320><<<sms, 320>>>(d, out, iters); };
+      const double cyc6 = avg_cycles(launch6, d, h, sms);
+      if (cyc6 <= 0) { printf(", \"error\": \"softmax probe failed\"}\n"); return 1; }
+      printf(", \"softmax_row128_v6_clk_8warps_168regs\": %.1f", cyc6 / iters);
       break;
     }
   }

@@ -407,6 +407,13 @@ __device__ __forceinline__ float exp2_poly(float x) {
   return __int_as_float(__float_as_int(p) + (__float_as_int(t) << 23));
 }
 
+// The same 2^x for a pair of floats with packed f32x2 arithmetic (one instruction per
+// step for both): about six instructions per exponential instead of a dozen.  x = n + f
+// by rounding through 1.5*2^23 (t), f = x - n by one packed FMA, the cubic by three, and
+// n added to each exponent field from t's low mantissa bits.  Valid for x <= 64; inputs
+// below -125 (and -inf) give 2^-125.
+__device__ __forceinline__ uint64_t exp2_poly2(uint64_t x2);
+
 // Two floats -> bf16x2 (round to nearest even); `lo` lands in the low half.
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   uint32_t r;
@@ -443,6 +450,18 @@ __device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
   uint64_t d;
   asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
+}
+__device__ __forceinline__ uint64_t exp2_poly2(uint64_t x2) {
+  const uint64_t x = f2(fmaxf(f2lo(x2), -125.f), fmaxf(f2hi(x2), -125.f));
+  const uint64_t t = add2(x, f2(12582912.f, 12582912.f));  // 1.5 * 2^23
+  const uint64_t n = add2(t, f2(-12582912.f, -12582912.f));
+  const uint64_t f = fma2(n, f2(-1.f, -1.f), x);
+  uint64_t p = fma2(f2(0.055088684f, 0.055088684f), f, f2(0.24260405f, 0.24260405f));
+  p = fma2(p, f, f2(0.6932762f, 0.6932762f));
+  p = fma2(p, f, f2(0.99992895f, 0.99992895f));
+  const uint32_t lo = __float_as_uint(f2lo(p)) + (__float_as_uint(f2lo(t)) << 23);
+  const uint32_t hi = __float_as_uint(f2hi(p)) + (__float_as_uint(f2hi(t)) << 23);
+  return f2(__uint_as_float(lo), __uint_as_float(hi));
 }
 // max(a, b, c) in one instruction (three-input form, sm_100+).
 __device__ __forceinline__ float max3(float a, float b, float c) {
