@@ -582,6 +582,7 @@ def main():
                          "paged_decode_hnd_p16, "
                          "long_decode, "
                          "gemm_4096, gemm_16k_256_16k, gemm_256_256_16k, gemm_8192, cublas_8192 (torch.matmul), "
+                         "batched_decode_persistent, batched_decode_cluster4, "
                          "varlen_prefill_small), run --steps "
                          "launches, print nothing")
     args = ap.parse_args()
@@ -846,6 +847,78 @@ def run_model_sweep(torch, loom, dev, stream, args, peaks):
         torch.cuda.empty_cache()
 
 
+def run_ablation_sweep(torch, loom, dev, stream, args, peaks):
+    """The paper's block-size ablation restated for this path: around each constant the
+    analytic model fixes (the prefill K/V ring depth, the decode stage plan, the GEMM ring
+    depth), every neighbour that is compiled is timed on the benchmark workloads beside the
+    model's choice (is the model's point locally best?)."""
+    steps = max(10, args.steps // 4)
+
+    def line(kind, wl, param, model, r):
+        print(json.dumps({"sweep": "ablation", "kind": kind, "workload": wl.describe(), "param": param,
+                          "model_choice": model, "measured_ms": round(r["ms_per_step"], 5), "value": r["value"],
+                          "unit": r["unit"], "frac": r["roofline"]["frac"]}), flush=True)
+
+    # prefill: ring depth of the two-tile design (BN = 128 keys is fixed by the softmax layout)
+    lens = synth.decode_lengths(0, 16, 4096, 8192)
+    prefill = [(Prefill("prefill", 4, 32, 32, 2048, 128, causal=False), (2, 3)),
+               (Prefill("prefill_causal", 4, 32, 32, 2048, 128, causal=True), (2, 3)),
+               (Prefill("long_prefill_d128", 1, 32, 8, 8192, 128, causal=True), (2, 3)),
+               (Prefill("long_prefill_d64", 1, 64, 16, 8192, 64, causal=True), (3, 6, 9, 10)),
+               (Prefill("prefill_d64", 4, 32, 32, 2048, 64, causal=False), (3, 6, 9, 10))]
+    for wl, depths in prefill:
+        wl.setup(torch, dev, loom)
+        model_depth = loom.loom_model_fwd_plan_variant(wl.D, 2)["kv_slots"]
+        for d in depths:
+            assert loom.loom_debug_prefill_slots(wl.D, d)
+            r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks)
+            loom.loom_attn_check_error(stream)
+            line("prefill_ring_depth", wl, {"kv_slots": d}, d == model_depth, r)
+        loom.loom_debug_prefill_slots(wl.D, 0)
+        wl.inp = None
+        torch.cuda.empty_cache()
+
+    # decode: keys per stage x ring stages x CTAs per SM of the split kernel (split + merge form)
+    plans = [(64, 3, 2), (32, 2, 2), (32, 3, 2), (32, 4, 2), (64, 2, 2), (64, 4, 1), (128, 2, 1), (128, 3, 1)]
+    loom.loom_debug_decode_form(1)  # the split + merge form, whose split kernel the plans change
+    for wl in (Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16, lengths=lens),
+               Decode("long_decode", 1, 32, 8, 131072, 128, splits=0)):
+        wl.setup(torch, dev, loom)
+        for i, (t, st, c) in enumerate(plans):
+            assert loom.loom_debug_decode_stage_plan(t, st, c)
+            r = measure(torch, wl, steps, args.warmup, stream, lambda: None, 1, float, peaks)
+            loom.loom_attn_check_error(stream)
+            line("decode_stage_plan", wl, {"tokens": t, "stages": st, "ctas_per_sm": c}, i == 0, r)
+        loom.loom_debug_decode_stage_plan(0)
+        wl.inp = None
+        torch.cuda.empty_cache()
+    loom.loom_debug_decode_form(0)
+
+    # GEMM: K-stage ring depth of the kernel the model picks (deeper rings do not fit)
+    for (M, N, K), kernel, depths in [((8192, 8192, 8192), "pair", (5, 6)), ((16384, 16384, 16384), "pair", (5, 6)),
+                                      ((4096, 4096, 4096), 256, (3, 4)), ((2048, 2048, 16384), 128, (5, 6))]:
+        wl = Gemm("ablation", M, N, K)
+        wl.setup(torch, dev, loom)
+        if kernel == "pair":
+            loom.loom_debug_gemm_cta_pair(1)
+        else:
+            loom.loom_debug_gemm_cta_pair(-1)
+            loom.loom_debug_gemm_tile_n(kernel)
+            loom.loom_debug_gemm_splits(1)
+        for d in depths:
+            loom.loom_debug_gemm_stages(d if d != max(depths) else 0)
+            r = measure(torch, wl, max(10, min(steps, 200)), args.warmup, stream, lambda: None, 1, float, peaks,
+                        warm_s=0.25)
+            loom.loom_attn_check_error(stream)
+            line("gemm_ring_depth", wl, {"kernel": kernel, "stages": d}, d == max(depths), r)
+        loom.loom_debug_gemm_stages(0)
+        loom.loom_debug_gemm_cta_pair(0)
+        loom.loom_debug_gemm_tile_n(0)
+        loom.loom_debug_gemm_splits(0)
+        wl.inp = None
+        torch.cuda.empty_cache()
+
+
 GEMM_DIMS = (256, 2048, 16384)
 
 
@@ -939,11 +1012,15 @@ def run_ncu_case(torch, loom, dev, stream, args):
     cases["prefill_d64_small"] = Prefill("prefill_d64_small", 1, 16, 4, 8192, 64, causal=True)
     cases["batched_decode_persistent"] = Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16,
                                              lengths=synth.decode_lengths(0, 16, 4096, 8192))
+    cases["batched_decode_cluster4"] = Decode("batched_decode", 16, 32, 8, 8192, 128, splits=16,
+                                           lengths=synth.decode_lengths(0, 16, 4096, 8192))
     wl = cases[args.ncu_case]
     if args.prefill_design:
         loom.loom_debug_prefill_design(args.prefill_design)
     if args.ncu_case == "batched_decode_persistent":
         loom.loom_debug_decode_form(2)
+    if args.ncu_case == "batched_decode_cluster4":
+        loom.loom_debug_decode_form(3, 4)  # the single-kernel form, clusters of 4 CTAs
     wl.sets = 1  # one input set: the smallest device footprint for a capture
     wl.setup(torch, dev, loom)
     with torch.cuda.stream(stream):
