@@ -5,8 +5,8 @@
  *
  *     O = softmax(scale * Q K^T [+ causal mask]) V,   LSE = ln sum_j exp(scale * q . k_j)
  *
- * in the two forms the Loom paper evaluates: Flash Attention prefill (Sec. 3.2.2:
- * "matrix multiplication, softmax, and value aggregation" fused in one kernel) and
+ * in the two forms the Loom paper evaluates: Flash Attention prefill (Sec. 3.2.2: the
+ * score product, the softmax and the weighted sum of values fused in one kernel) and
  * Flash Decode (Sec. 2.6 Flash Decode example and Sec. 3.2.3: the sequence axis is
  * split across cores, each split runs a local softmax loop, and the partial results
  * are gathered, globally softmaxed and finally scaled).

@@ -5,7 +5,7 @@
 // It shares no code, header or constant with the CUDA library.
 //
 // What it computes (the paper never prints the formula; the evaluation describes Flash
-// Attention as "matrix multiplication, softmax, and value aggregation" (Sec. 3.2.2) and
+// Attention as the fusion of the two matrix products with the softmax between them (Sec. 3.2.2) and
 // Flash Decode as a local softmax loop followed by gathering partial results, a global
 // softmax and a final scaling (Sec. 2.6, Flash Decode example; Sec. 3.2.3)):
 //

@@ -1,8 +1,8 @@
 // Flash Attention prefill for GB300 (sm_103a): TMA + mbarrier ring, tcgen05 MMAs with
 // TMEM accumulators, warp-specialised loader / MMA / softmax roles.
 //
-// Paper: Sec. 3.2.2 evaluates Flash Attention as fused "matrix multiplication, softmax,
-// and value aggregation"; the pipelining of its load, compute and store stages through
+// Paper: Sec. 3.2.2 evaluates Flash Attention as one fused kernel for the score product,
+// the softmax and the weighted sum of values; the pipelining of its load, compute and store stages through
 // counted circular buffers is the virtual-buffer protocol of Sec. 2.3, and the tile and
 // stage constants come from the latency model of Sec. 2.6 (Eq. 6-9, in model.h).
 //
