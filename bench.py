@@ -292,17 +292,22 @@ class PagedDecode(Decode):
     pages are dealt in a seeded shuffled order across the cache (a cache that has served
     many requests), so consecutive logical pages are scattered in HBM."""
 
-    def __init__(self, name, B, Hq, Hkv, Skv, D, splits, page_size, lengths, seed=0, sets=2, layout="nhd"):
+    def __init__(self, name, B, Hq, Hkv, Skv, D, splits, page_size, lengths, seed=0, sets=2, layout="nhd",
+                 in_order=False):
         super().__init__(name, B, Hq, Hkv, Skv, D, splits, lengths=lengths, seed=seed, sets=sets)
-        self.P, self.layout = page_size, layout
+        self.P, self.layout, self.in_order = page_size, layout, in_order
 
     def describe(self):
-        return super().describe().replace("decode ", f"paged decode ({self.layout}) page_size={self.P} ", 1)
+        pages = "pages in order" if self.in_order else "pages shuffled"
+        return super().describe().replace("decode ", f"paged decode ({self.layout}, {pages}) page_size={self.P} ", 1)
 
     def paged(self, k, v, s):
         B, Hkv, S, D, P = self.B, self.Hkv, self.Skv, self.D, self.P
         npg = S // P
-        order = np.random.default_rng(self.seed + s).permutation(B * npg).astype(np.int32)
+        if self.in_order:  # page p of sequence b is cache page b * npg + p
+            order = np.arange(B * npg, dtype=np.int32)
+        else:
+            order = np.random.default_rng(self.seed + s).permutation(B * npg).astype(np.int32)
         kc = np.empty((B * npg, P, Hkv, D), np.uint16)
         vc = np.empty_like(kc)
         kc[order] = k.reshape(B, Hkv, npg, P, D).transpose(0, 2, 3, 1, 4).reshape(B * npg, P, Hkv, D)
@@ -567,7 +572,7 @@ def main():
     ap.add_argument("--only", default=None,
                     help="comma-separated subset (and order) of the extra workloads to run")
     ap.add_argument("--oracle-seconds", type=float, default=12.0)
-    ap.add_argument("--sweep", choices=["decode", "model", "gemm", "ablation"], default=None,
+    ap.add_argument("--sweep", choices=["decode", "model", "gemm", "ablation", "paged"], default=None,
                     help="decode: model-vs-measured sweep of the decode split count; model: the analytic "
                          "model's ranking and accuracy over prefill designs and shapes and decode split "
                          "counts and shapes; gemm: the BF16 GEMM over the shape grid {256, 2048, 16384}^3 "
@@ -618,6 +623,8 @@ def main():
         return run_gemm_sweep(torch, loom, dev, stream, args, peaks)
     if args.sweep == "ablation":
         return run_ablation_sweep(torch, loom, dev, stream, args, peaks)
+    if args.sweep == "paged":
+        return run_paged_sweep(torch, loom, dev, stream, args)
 
     # headline: prefill non-causal, with clocks sampled during the timed loop
     headline.setup(torch, dev, loom)
@@ -917,6 +924,48 @@ def run_ablation_sweep(torch, loom, dev, stream, args, peaks):
         loom.loom_debug_gemm_splits(0)
         wl.inp = None
         torch.cuda.empty_cache()
+
+
+def run_paged_sweep(torch, loom, dev, stream, args):
+    """Paged decode against page placement: the batched decode over the contiguous cache
+    and over paged caches (token- and head-major, page sizes 16 to 256) with each
+    sequence's pages shuffled across the cache or in order, timed interleaved in shuffled
+    rounds on one box (GB/s of the same algorithmic bytes)."""
+    import random
+    lens = synth.decode_lengths(0, 16, 4096, 8192)
+    shape = (16, 32, 8, 8192, 128)
+    wls = {"contiguous": Decode("batched_decode", *shape, splits=16, lengths=lens)}
+    for layout, P in (("nhd", 16), ("hnd", 16), ("nhd", 64), ("hnd", 256)):
+        for in_order in (False, True):
+            key = f"{layout}_p{P}_{'in_order' if in_order else 'shuffled'}"
+            wls[key] = PagedDecode("paged", *shape, splits=16, page_size=P, lengths=lens, layout=layout,
+                                   in_order=in_order)
+    for wl in wls.values():
+        wl.sets = 1
+        wl.setup(torch, dev, loom)
+    nbytes = wls["contiguous"].bytes
+    steps = max(20, min(args.steps, 200))
+    res = {k: [] for k in wls}
+    rng = random.Random(9)
+    with torch.cuda.stream(stream):
+        for _ in range(8):
+            order = list(wls)
+            rng.shuffle(order)
+            for key in order:
+                wl = wls[key]
+                for i in range(max(3, args.warmup)):
+                    wl.step(i, stream)
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                for i in range(steps):
+                    wl.step(i, stream)
+                e1.record(stream)
+                e1.synchronize()
+                res[key].append(nbytes * steps / (e0.elapsed_time(e1) * 1e-3) / 1e9)
+    loom.loom_attn_check_error(stream)
+    for key, v in res.items():
+        print(json.dumps({"sweep": "paged", "cache": key, "workload": wls[key].describe(),
+                          "gbs_median": round(statistics.median(v), 1), "rounds": len(v)}), flush=True)
 
 
 GEMM_DIMS = (256, 2048, 16384)
