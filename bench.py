@@ -140,6 +140,14 @@ def profiled_traffic():
     return PROFILED_TRAFFIC_BYTES if h.hexdigest() == PROFILED_SOURCES_SHA256 else None
 
 
+def headline_config(wl, world):
+    """The `config` of the headline workload, the same object on both arms' lines."""
+    return {"workload": wl.describe(), "B": 4, "Hq": 32, "Hkv": 32, "Sq": 2048, "Skv": 2048, "D": 128,
+            "causal": False, "global_batch": 4 * world, "seq_len": 2048,
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+            "l2": "inputs larger than L2 (268 MB per step), 2 rotating input sets"}
+
+
 def prefill_flops(B, Hq, Sq, Skv, D, causal):
     """Algorithmic FLOPs: 4*D per visible (query, key) pair (QK^T and PV, 2 FLOP per MAC)."""
     if not causal:
@@ -700,10 +708,7 @@ def main():
             "vs_baseline": None,
             "dtype": "bf16",
             "data": "synthetic (seeded splitmix64/Box-Muller N(0,1) rounded to bf16)",
-            "config": {"workload": headline.describe(), "B": 4, "Hq": 32, "Hkv": 32, "Sq": 2048, "Skv": 2048,
-                       "D": 128, "causal": False, "global_batch": 4 * world, "seq_len": 2048,
-                       "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                       "l2": "inputs larger than L2 (268 MB per step), 2 rotating input sets"},
+            "config": headline_config(headline, world),
             "roofline": roof,
             "cpu_baseline": cpu,
             "e2e": e2e,
@@ -1112,8 +1117,7 @@ def run_reference(args, wl, world, rank):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded splitmix64/Box-Muller N(0,1) rounded to bf16)",
-        "config": {"workload": wl.describe(), "B": 4, "Hq": 32, "Hkv": 32, "Sq": 2048, "Skv": 2048, "D": 128,
-                   "causal": False},
+        "config": headline_config(wl, world),
         "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
                          "sample": f"{rows_per_step} query rows of one (b,h) head per step (fp64 oracle, "
                                    f"{cores} threads)"},
