@@ -356,6 +356,17 @@ void loom_debug_gemm_stages(int stages);
 void loom_debug_gemm_order(int group_rows, int k_alternate);
 
 /*
+ * loom_debug_decode_tensor_cores: 1 (the default) lets the split + merge form run its
+ * split kernel on the tensor cores for a contiguous cache (D 64 or 128, at most 32 query
+ * heads per kv head): per 64-key stage, S = Q K^T and O += P V as tcgen05 MMAs with the
+ * query heads as rows of a TMEM tile, the softmax on one warp; 0 runs the CUDA-core split
+ * kernel instead (the paged cache and the persistent forms always use the CUDA-core
+ * stage).  P is rounded to bf16 before P V on the tensor cores, as in the prefill; the
+ * CUDA-core stage keeps it in fp32.
+ */
+void loom_debug_decode_tensor_cores(int on);
+
+/*
  * Test hook: the Flash Decode form.  form 1 = split + merge kernels, 2 = persistent split
  * kernel + merge kernel, 3 = the single-kernel cluster form (each when it can run); anything
  * else: the analytic model's choice (default).  cluster in 1..16 pins the cluster form's

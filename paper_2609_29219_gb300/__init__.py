@@ -31,7 +31,7 @@ __all__ = [
     "loom_attn_decode_form", "loom_decode_max_clusters", "loom_decode_persistent_slots", "loom_debug_decode_form",
     "loom_model_decode_persistent_time_us", "DECODE_SPLIT_MERGE", "DECODE_PERSISTENT", "DECODE_CLUSTER",
     "loom_debug_prefill_slots", "loom_debug_decode_stage_plan", "loom_debug_gemm_stages",
-    "loom_debug_gemm_order",
+    "loom_debug_gemm_order", "loom_debug_decode_tensor_cores",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -154,6 +154,8 @@ def capi() -> ctypes.CDLL:
             lib.loom_debug_gemm_stages.restype = None
             lib.loom_debug_gemm_order.argtypes = [i32, i32]
             lib.loom_debug_gemm_order.restype = None
+            lib.loom_debug_decode_tensor_cores.argtypes = [i32]
+            lib.loom_debug_decode_tensor_cores.restype = None
             _lib = lib
     return _lib
 
@@ -547,6 +549,11 @@ def loom_debug_decode_stage_plan(tokens: int, stages: int = 0, ctas_per_sm: int 
 def loom_debug_gemm_stages(stages: int) -> None:
     """Pin the GEMM's K-stage ring depth where a neighbour is compiled (0: the model's)."""
     capi().loom_debug_gemm_stages(int(stages))
+
+
+def loom_debug_decode_tensor_cores(on: bool) -> None:
+    """Let the split + merge decode run its split kernel on the tensor cores (default), or not."""
+    capi().loom_debug_decode_tensor_cores(1 if on else 0)
 
 
 def loom_debug_gemm_order(group_rows: int = 0, k_alternate: int = 0) -> None:

@@ -517,6 +517,328 @@ __global__ void __launch_bounds__(C::THREADS, C::CTAS_PER_SM)
                      });
 }
 
+// ---------------------------------------------------------------- tensor-core split kernel
+// The split kernel of the split + merge form for a contiguous cache with the dot products
+// on the tensor cores (Sec. 2.6 Flash Decode HEG, local softmax loop).  The query heads
+// of one kv head are the rows of a 128-row tile held in TMEM (rows 0..G-1; the rest are
+// zero and their results unused): per 64-key stage S = Q K^T is one M = 128 MMA with A in
+// TMEM and the 128B-swizzled K tile as B, one warp (lane = query head) turns S into P =
+// 2^(S c - m) in place as bf16, and O += P V is a second MMA with P in TMEM and V as an
+// MN-major B.  The padded rows cost nothing that matters here -- the stage's MMAs take a
+// fraction of the time its bytes take to arrive -- while the CUDA cores are left with 64
+// exponentials per head and stage instead of every product of the dot products.
+//   warps: 0 query rows (Q into TMEM, softmax, epilogue; TMEM lanes 0-31), 1 loader
+//   (TMA, lane 0), 2 MMA issuer (whole warp, one elected lane)
+//   TMEM: [0, D/2) Q as bf16 pairs | [64, 128) S, then P over its first 32 columns |
+//         [128, 128 + D) O
+template <int D>
+struct DecodeTcCfg {
+  static constexpr int T = 64;  // keys per stage
+  // ring depth: about 96 KB of shared memory at either D, so that exactly two CTAs share
+  // an SM (their 2 x 256 TMEM columns are the SM's 512)
+  static constexpr int NSTAGE = D == 64 ? 6 : 3;
+  static constexpr int NBOX = D / 64;                     // 128-byte swizzle atoms along D
+  static constexpr uint32_t BOX_BYTES = T * 128;          // 64 keys x 64 dims
+  static constexpr uint32_t TILE_BYTES = NBOX * BOX_BYTES;  // one K or V tile
+  static constexpr uint32_t STAGE_BYTES = 2 * TILE_BYTES;   // K, then V
+  static constexpr uint32_t BAR_OFF = NSTAGE * STAGE_BYTES;
+  // barriers: full[NSTAGE], empty[NSTAGE], q, s, p, o, drain
+  static constexpr int NBAR = 2 * NSTAGE + 5;
+  static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
+  static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
+  static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;  // + 1024-byte alignment slack
+  static constexpr uint32_t Q_COL = 0;
+  static constexpr uint32_t S_COL = 64;
+  static constexpr uint32_t O_COL = 128;
+  static constexpr uint32_t TMEM_COLS = 256;  // a power of two: 2 CTAs per SM
+  static constexpr int THREADS = 96;
+  static constexpr int MAX_G = 32;            // query heads per kv head: TMEM lanes of warp 0
+  static_assert(O_COL + D <= TMEM_COLS, "TMEM budget");
+  static_assert(Q_COL + D / 2 <= S_COL && S_COL + T <= O_COL, "TMEM regions");
+  static_assert(2 * (BYTES + 1024) <= 228 * 1024 && 3 * (BYTES + 1024) > 228 * 1024, "exactly two CTAs per SM");
+};
+
+// Warp 0 of decode_tc_split_kernel: lane h is query head h0 + h (lanes >= G carry zero rows).
+// Q goes into TMEM as bf16 pairs (its memory order); per stage the lane reads its 64
+// scores, masks keys past the split's end, moves the running max lazily (O rescaled in
+// TMEM after the previous P.V when it moved by more than kRescaleThreshold), writes P over
+// S and arrives on bar_p; at the end O / l and the log-sum-exp go to the split's partial.
+template <int D>
+__device__ __forceinline__ void decode_tc_rows(const __nv_bfloat16* __restrict__ q, float* __restrict__ o_part,
+                                               float* __restrict__ lse_part, uint32_t tmem, int b, int h0, int G,
+                                               int Hq, int splits, size_t row0, int t_begin, int t_end, int n_st,
+                                               float c, uint8_t* smem, uint32_t bar_full, uint32_t bar_q,
+                                               uint32_t bar_s, uint32_t bar_p, uint32_t bar_o, const KernelCtl& ctl,
+                                               const Abort& ab) {
+  using C = DecodeTcCfg<D>;
+  const int lane = threadIdx.x & 31;
+  const bool real = lane < G;
+  {
+    uint32_t w[32];
+    const uint4* src = reinterpret_cast<const uint4*>(q + (static_cast<size_t>(b) * Hq + h0 + (real ? lane : 0)) * D);
+#pragma unroll
+    for (int half = 0; half < D / 64; ++half) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const uint4 v = real ? src[half * 8 + i] : make_uint4(0u, 0u, 0u, 0u);
+        w[4 * i] = v.x;
+        w[4 * i + 1] = v.y;
+        w[4 * i + 2] = v.z;
+        w[4 * i + 3] = v.w;
+      }
+      tmem_st32(tmem + C::Q_COL + half * 32, w);
+    }
+    tmem_wait_st();
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar_q);
+  }
+  const uint64_t c2 = f2(c, c);
+  float m_run = -INFINITY, l_run = 0.f;
+  bool ok = true;
+  for (int it = 0; it < n_st; ++it) {
+    if (!(ok = mbar_wait_warp(bar_s, it & 1, ctl, ab))) break;
+    tc_fence_after();
+    uint32_t s[C::T];
+    tmem_ld32(tmem + C::S_COL, s);
+    tmem_ld32(tmem + C::S_COL + 32, s + 32);
+    tmem_wait_ld();
+    reg_fence32(s);
+    reg_fence32(s + 32);
+    const int ntok = min(C::T, t_end - (t_begin + it * C::T));
+    if (ntok < C::T) {
+#pragma unroll
+      for (int i = 0; i < C::T; ++i)
+        if (i >= ntok) s[i] = __float_as_uint(-INFINITY);
+    }
+    float mm[8];
+#pragma unroll
+    for (int g = 0; g < 8; ++g) mm[g] = __uint_as_float(s[g]);
+#pragma unroll
+    for (int i = 8; i + 16 <= C::T; i += 16)
+#pragma unroll
+      for (int g = 0; g < 8; ++g) mm[g] = max3(mm[g], __uint_as_float(s[i + g]), __uint_as_float(s[i + 8 + g]));
+#pragma unroll
+    for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], __uint_as_float(s[C::T - 8 + g]));
+    const float mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
+    const float m_new = fmaxf(m_run, mx * c);
+    const bool need = m_new > m_run + kRescaleThreshold;
+    const float alpha = need ? ex2(m_run - m_new) : 1.f;
+    if (need) m_run = m_new;
+    const float ms = (m_run == -INFINITY) ? 0.f : m_run;
+    const uint64_t nms2 = f2(-ms, -ms);
+    uint64_t acc[4] = {0, 0, 0, 0};
+    uint32_t pk[C::T / 2];
+#pragma unroll
+    for (int i = 0; i < C::T / 2; ++i) {
+      const uint64_t x = fma2(f2(__uint_as_float(s[2 * i]), __uint_as_float(s[2 * i + 1])), c2, nms2);
+      const float p0 = ex2(f2lo(x));
+      const float p1 = ex2(f2hi(x));
+      acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
+      pk[i] = pack_bf16x2(p0, p1);
+    }
+    tmem_st32(tmem + C::S_COL, pk);
+    tmem_wait_st();
+    if (ntok < C::T) {
+      // V rows past the split's end may hold anything (a cache past a sequence's length
+      // is never written): zero them so that their P = 0 adds exactly nothing to P.V
+      const int slot = it % C::NSTAGE;
+      if (!(ok = mbar_wait_warp(bar_full + 8 * slot, (it / C::NSTAGE) & 1, ctl, ab))) break;
+      uint4* vt = reinterpret_cast<uint4*>(smem + slot * C::STAGE_BYTES + C::TILE_BYTES);
+#pragma unroll
+      for (int x = 0; x < C::NBOX; ++x)
+        for (int i = lane; i < (C::T - ntok) * 8; i += 32)
+          vt[x * (C::BOX_BYTES / 16) + ntok * 8 + i] = make_uint4(0u, 0u, 0u, 0u);
+      fence_proxy_async_smem();
+    }
+    // O must hold the previous P.V before it is rescaled (it has: S of this stage was
+    // committed after it), and be rescaled before this stage's P.V
+    if (it > 0 && __any_sync(0xffffffffu, need)) {
+      if (!(ok = mbar_wait_warp(bar_o, (it - 1) & 1, ctl, ab))) break;
+      tc_fence_after();
+      const uint64_t a2 = f2(alpha, alpha);
+#pragma unroll 1
+      for (int ch = 0; ch < D / 32; ++ch) {
+        uint32_t rr[32];
+        tmem_ld32(tmem + C::O_COL + ch * 32, rr);
+        tmem_wait_ld();
+        reg_fence32(rr);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const uint64_t x = mul2(f2(__uint_as_float(rr[2 * i]), __uint_as_float(rr[2 * i + 1])), a2);
+          rr[2 * i] = __float_as_uint(f2lo(x));
+          rr[2 * i + 1] = __float_as_uint(f2hi(x));
+        }
+        tmem_st32(tmem + C::O_COL + ch * 32, rr);
+      }
+      tmem_wait_st();
+    }
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar_p);
+    const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+    l_run = l_run * alpha + (f2lo(a01) + f2hi(a01));
+  }
+  if (!ok) return;
+  // epilogue: the last P.V, then O / l and the log-sum-exp of each real row
+  if (!mbar_wait_warp(bar_o, (n_st - 1) & 1, ctl, ab)) return;
+  tc_fence_after();
+  const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
+  float* dst = o_part + (row0 + static_cast<size_t>(real ? lane : 0) * splits) * D;
+#pragma unroll 1
+  for (int ch = 0; ch < D / 32; ++ch) {
+    uint32_t rr[32];
+    tmem_ld32(tmem + C::O_COL + ch * 32, rr);
+    tmem_wait_ld();
+    reg_fence32(rr);
+    if (real) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        reinterpret_cast<float4*>(dst + ch * 32)[i] =
+            make_float4(__uint_as_float(rr[4 * i]) * inv_l, __uint_as_float(rr[4 * i + 1]) * inv_l,
+                        __uint_as_float(rr[4 * i + 2]) * inv_l, __uint_as_float(rr[4 * i + 3]) * inv_l);
+    }
+  }
+  if (real) lse_part[row0 + static_cast<size_t>(lane) * splits] = l_run > 0.f ? (m_run + log2f(l_run)) * kLn2 : -INFINITY;
+}
+
+template <int D>
+__global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
+    decode_tc_split_kernel(const __nv_bfloat16* __restrict__ q, const int32_t* __restrict__ seqlens,
+                           float* __restrict__ o_part, float* __restrict__ lse_part, int Hq, int Hkv, int Skv,
+                           int splits, float c, KernelCtl ctl, const __grid_constant__ CUtensorMap tm_k,
+                           const __grid_constant__ CUtensorMap tm_v) {
+  using C = DecodeTcCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  // Let the merge grid launch as soon as every split CTA is resident.
+  asm volatile("griddepcontrol.launch_dependents;");
+  const uint32_t raw_base = smem_u32(smem_raw);
+  const uint32_t sbase = (raw_base + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (sbase - raw_base);
+  const int split = blockIdx.x, hk = blockIdx.y, b = blockIdx.z;
+  const int G = Hq / Hkv, h0 = hk * G;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  int len = seqlens ? seqlens[b] : Skv;
+  len = max(0, min(len, Skv));
+  int chunk = (len + splits - 1) / splits;
+  chunk = (chunk + kDecodeChunkAlign - 1) / kDecodeChunkAlign * kDecodeChunkAlign;
+  const int t_begin = min(split * chunk, len);
+  const int t_end = min(t_begin + chunk, len);
+  const size_t row0 = (static_cast<size_t>(b) * Hq + h0) * splits + split;  // head h0's partial
+  if (t_begin >= t_end) {  // empty split: contributes nothing to the merge
+    for (int i = threadIdx.x; i < G * D; i += blockDim.x)
+      o_part[(row0 + static_cast<size_t>(i / D) * splits) * D + i % D] = 0.f;
+    if (static_cast<int>(threadIdx.x) < G) lse_part[row0 + static_cast<size_t>(threadIdx.x) * splits] = -INFINITY;
+    return;
+  }
+  const int n_st = (t_end - t_begin + C::T - 1) / C::T;
+  const int kv_z = b * Hkv + hk;
+
+  const uint32_t bar_full = sbase + C::BAR_OFF;
+  const uint32_t bar_empty = bar_full + 8 * C::NSTAGE;
+  const uint32_t bar_q = bar_empty + 8 * C::NSTAGE;  // Q is in TMEM
+  const uint32_t bar_s = bar_q + 8;                  // S of the stage is in TMEM
+  const uint32_t bar_p = bar_s + 8;                  // P of the stage is in TMEM (O rescaled)
+  const uint32_t bar_o = bar_p + 8;                  // the stage's P.V is done
+  const uint32_t bar_drain = bar_o + 8;
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::TMEM_PTR_OFF);
+  Abort ab{reinterpret_cast<volatile int*>(smem + C::ABORT_OFF)};
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSTAGE; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, 1);
+    }
+    mbar_init(bar_q, 1);
+    mbar_init(bar_s, 1);
+    mbar_init(bar_p, 1);
+    mbar_init(bar_o, 1);
+    mbar_init(bar_drain, 1);
+    *ab.flag = 0;
+    *(ab.flag + 1) = 0;
+    fence_barrier_init();
+  }
+  if (warp == 2) tmem_alloc(smem_u32(tmem_ptr), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_ptr;
+
+  if (warp == 1) {
+    // ------------------------------------------------------------ loader (lane 0)
+    if (lane == 0) {
+      prefetch_tensormap(&tm_k);
+      prefetch_tensormap(&tm_v);
+      int issued = 0, skipped = -1;
+      for (int it = 0; it < n_st; ++it) {
+        const int s = it % C::NSTAGE;
+        if (!mbar_wait(bar_empty + 8 * s, ((it / C::NSTAGE) & 1) ^ 1, ctl, ab)) break;
+        issued = it + 1;
+        if (ctl.inject == 1 && it == 1) {  // test hook: never fill this stage
+          skipped = it;
+          continue;
+        }
+        // keys [tok0, tok0 + 64) of this kv head; rows past Skv read as zeros and every
+        // key past the split's end is masked by the softmax
+        const int tok0 = t_begin + it * C::T;
+        const uint32_t dst = sbase + s * C::STAGE_BYTES;
+        mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
+#pragma unroll
+        for (int x = 0; x < C::NBOX; ++x) {
+          tma_load_3d(dst + x * C::BOX_BYTES, &tm_k, x * 64, tok0, kv_z, bar_full + 8 * s);
+          tma_load_3d(dst + C::TILE_BYTES + x * C::BOX_BYTES, &tm_v, x * 64, tok0, kv_z, bar_full + 8 * s);
+        }
+      }
+      // Drain: never leave the CTA with copies still landing in its shared memory.
+      Abort no_abort{ab.flag + 1};
+      for (int i = max(0, issued - C::NSTAGE); i < issued; ++i)
+        if (i != skipped) mbar_wait(bar_full + 8 * (i % C::NSTAGE), (i / C::NSTAGE) & 1, ctl, no_abort);
+    }
+  } else if (warp == 2) {
+    // ------------------------------------------------------------ MMA issuer
+    constexpr uint32_t idesc_s = idesc_bf16(128, C::T, 0, 0);  // Q (TMEM) x K^T (K-major)
+    constexpr uint32_t idesc_pv = idesc_bf16(128, D, 0, 1);    // P (TMEM) x V (MN-major)
+    bool ok = mbar_wait_warp(bar_q, 0, ctl, ab);
+    tc_fence_after();
+    for (int it = 0; ok && it < n_st; ++it) {
+      const int s = it % C::NSTAGE;
+      if (!(ok = mbar_wait_warp(bar_full + 8 * s, (it / C::NSTAGE) & 1, ctl, ab))) break;
+      tc_fence_after();
+      const uint32_t kslot = sbase + s * C::STAGE_BYTES;
+      // S = Q K^T over D in 64-wide boxes (the previous stage's P.V, issued before, has
+      // read the P these columns held: the MMAs of a CTA run in issue order)
+#pragma unroll
+      for (int x = 0; x < C::NBOX; ++x)
+        mma_ts_kmaj_k64_el(tmem + C::S_COL, tmem + C::Q_COL + x * 32,
+                           sdesc_sw128(kslot + x * C::BOX_BYTES, 16, 1024), idesc_s, x > 0 ? 1u : 0u);
+      tc_commit_el(bar_s);
+      if (!(ok = mbar_wait_warp(bar_p, it & 1, ctl, ab))) break;
+      tc_fence_after();
+      // O += P V over the stage's 64 keys
+      mma_ts_k64_el(tmem + C::O_COL, tmem + C::S_COL, sdesc_sw128(kslot + C::TILE_BYTES, C::BOX_BYTES, 1024),
+                    idesc_pv, it > 0 ? 1u : 0u);
+      tc_commit_el(bar_o);
+      tc_commit_el(bar_empty + 8 * s);
+    }
+    // every MMA issued above is done before TMEM is released
+    Abort no_abort{ab.flag + 1};
+    tc_commit_el(bar_drain);
+    mbar_wait_warp(bar_drain, 0, ctl, no_abort);
+  } else {
+    // ------------------------------------------------------------ query rows (warp 0)
+    decode_tc_rows<D>(q, o_part, lse_part, tmem, b, h0, G, Hq, splits, row0, t_begin, t_end, n_st, c, smem, bar_full,
+                      bar_q, bar_s, bar_p, bar_o, ctl, ab);
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
 // ---------------------------------------------------------------- persistent forms
 // Two persistent kernels share one body (decode_persistent_kernel):
 //   CLUSTER = true: the single-kernel form.  Clusters of cs CTAs walk units (batch, kv
@@ -1048,6 +1370,43 @@ cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl
   return cudaGetLastError();
 }
 
+// The contiguous cache [B, Hkv, Skv, D] as a 3-D tensor (dim, key, kv head of a sequence)
+// in 64-dim x 64-key boxes, 128-byte swizzled: the tensor-core split kernel's K and V tiles.
+bool kv_map_sw128(CUtensorMap* map, const void* cache, int B, int Hkv, int Skv, int D) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(Skv),
+                        static_cast<cuuint64_t>(B) * Hkv};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(Skv) * D * 2};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(DecodeTcCfg<128>::T), 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(cache), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Whether the tensor-core split kernel takes this decode: a contiguous cache, at most 32
+// query heads per kv head, the model's stage plan.
+bool decode_tc_eligible(const DecodeArgs& a) {
+  const int G = a.Hq / a.Hkv;
+  return a.tc && a.stage_plan == 0 && G <= DecodeTcCfg<128>::MAX_G && (a.D == 64 || a.D == 128);
+}
+
+template <int D>
+cudaError_t launch_tc_split(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  using C = DecodeTcCfg<D>;
+  static PerDeviceOnce once;
+  if (!prepare_kernel(decode_tc_split_kernel<D>, C::BYTES, false, once)) return cudaErrorInvalidValue;
+  CUtensorMap tk, tv;
+  if (!kv_map_sw128(&tk, a.k, a.B, a.Hkv, a.Skv, D) || !kv_map_sw128(&tv, a.v, a.B, a.Hkv, a.Skv, D))
+    return cudaErrorInvalidValue;
+  dim3 grid(a.splits, a.Hkv, a.B);
+  decode_tc_split_kernel<D><<<grid, C::THREADS, C::BYTES, stream>>>(
+      static_cast<const __nv_bfloat16*>(a.q), a.seqlens, a.o_part, a.lse_part, a.Hq, a.Hkv, a.Skv, a.splits,
+      a.scale * kLog2e, ctl, tk, tv);
+  return cudaGetLastError();
+}
+
 template <int D, int GT, bool PAGED, bool CLUSTER>
 cudaError_t launch_persistent_kernel(const DecodeArgs& a, dim3 grid, int cs, const PagedKV* pk, const KernelCtl& ctl,
                                      cudaStream_t stream) {
@@ -1182,8 +1541,13 @@ cudaError_t launch_form(const DecodeArgs& a, const PagedKV* pk, const KernelCtl&
   int cs = 0;
   const int form = decode_form<D, GT, PAGED>(a, &cs);
   if (form == kDecodeCluster) return launch_cluster<D, GT, PAGED>(a, cs, pk, ctl, stream);
-  const cudaError_t e = form == kDecodePersistent ? launch_persist<D, GT, PAGED>(a, pk, ctl, stream)
-                                                  : launch_split<D, GT, PAGED>(a, pk, ctl, stream);
+  cudaError_t e;
+  if (form == kDecodePersistent)
+    e = launch_persist<D, GT, PAGED>(a, pk, ctl, stream);
+  else if (!PAGED && decode_tc_eligible(a))
+    e = launch_tc_split<D>(a, ctl, stream);
+  else
+    e = launch_split<D, GT, PAGED>(a, pk, ctl, stream);
   if (e != cudaSuccess) return e;
   return launch_merge<D>(a, stream);
 }

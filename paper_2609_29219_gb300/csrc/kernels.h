@@ -50,6 +50,7 @@ struct DecodeArgs {
   int cluster;  // cluster form: 0 = the model's cluster size, else this size (if it divides splits and fits)
   int stage_plan;  // 0: the model's stage plan; i > 0: the i-th compiled ablation plan (split + merge form)
   int by_model;    // 1: the split count is the model's (num_splits = 0), which then also picks the form
+  int tc;          // 1: the split + merge form's split kernel may run on the tensor cores (contiguous cache)
 };
 
 struct FwdArgs {

@@ -35,6 +35,7 @@ int g_gemm_k_alt = 0;   // test hook: -1 stops the CTA-pair GEMM walking K backw
 int g_decode_form = 0;     // test hook: the Flash Decode form (0: the model's; kDecode* otherwise)
 int g_decode_cluster = 0;  // test hook: the cluster decode form's cluster size (0: the model's)
 int g_decode_stage_plan = 0;  // test hook: a compiled ablation stage plan of the decode split kernel
+int g_decode_tc = 1;  // test hook: 0 runs the split + merge form's CUDA-core split kernel on a contiguous cache
 
 constexpr int kMaxDevices = 64;
 uint32_t* g_err_ptr[kMaxDevices] = {};
@@ -207,7 +208,7 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D,
-               num_splits, scale, g_decode_form, g_decode_cluster, g_decode_stage_plan, by_model};
+               num_splits, scale, g_decode_form, g_decode_cluster, g_decode_stage_plan, by_model, g_decode_tc};
   return launch_decode(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                  : LOOM_ERR_CUDA;
 }
@@ -278,7 +279,7 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D, num_splits, scale,
-               g_decode_form, g_decode_cluster, 0, by_model};
+               g_decode_form, g_decode_cluster, 0, by_model, 0};
   PagedKV pk{block_table, num_pages, page_size, max_pages, kv_layout};
   return launch_decode_paged(a, pk, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                           : LOOM_ERR_CUDA;
@@ -356,6 +357,8 @@ void loom_debug_gemm_splits(int splits) { g_gemm_splits = model::gemm_split_supp
 void loom_debug_gemm_cta_pair(int mode) { g_gemm_pair = (mode == 1 || mode == -1) ? mode : 0; }
 
 void loom_debug_gemm_stages(int stages) { g_gemm_stages = stages > 0 ? stages : 0; }
+
+void loom_debug_decode_tensor_cores(int on) { g_decode_tc = on ? 1 : 0; }
 
 void loom_debug_gemm_order(int group_rows, int k_alternate) {
   g_gemm_group = (group_rows >= 1 && group_rows <= 1024) ? group_rows : 0;

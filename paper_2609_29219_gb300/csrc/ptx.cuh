@@ -308,6 +308,25 @@ __device__ __forceinline__ void mma_ts_k64_el(uint32_t d_tmem, uint32_t a_tmem, 
       "r"(a_tmem), "l"(b), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// Four K-steps with A in TMEM (8 columns per step) and a 128-byte-swizzled K-major B
+// (32 bytes = 2 units per step within a 64-element swizzle row).
+__device__ __forceinline__ void mma_ts_kmaj_k64_el(uint32_t d_tmem, uint32_t a_tmem, uint64_t b,
+                                                   uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p, q, e;\n\t.reg .b64 b1, b2, b3;\n\t.reg .b32 t1, t2, t3;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "setp.eq.b32 q, %3, %3;\n\t"
+      "add.s32 t1, %1, 8;\n\tadd.s64 b1, %2, 2;\n\t"
+      "add.s32 t2, %1, 16;\n\tadd.s64 b2, %2, 4;\n\t"
+      "add.s32 t3, %1, 24;\n\tadd.s64 b3, %2, 6;\n\t"
+      "elect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [t1], b1, %3, q;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [t2], b2, %3, q;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [t3], b3, %3, q;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 // One K=16 step, both operands in shared memory.
 __device__ __forceinline__ void mma_ss_el(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                           uint32_t accumulate) {

@@ -22,14 +22,19 @@ def loom():
     return m
 
 
-@pytest.fixture(autouse=True, params=[0, 1, 2, 3], ids=["model_form", "split_merge", "persistent", "cluster"])
+@pytest.fixture(autouse=True, params=[(0, True), (1, True), (1, False), (2, True), (3, True)],
+                ids=["model_form", "split_merge", "split_merge_cuda_core", "persistent", "cluster"])
 def form(request, loom):
     """Every test runs with the model's choice of form and with each form forced: split
-    kernel + merge, persistent split kernel + merge, and the single-kernel cluster form (at
+    kernel + merge (its split kernel on the tensor cores where it takes the shape, and on
+    the CUDA cores), persistent split kernel + merge, and the single-kernel cluster form (at
     the model's cluster size)."""
-    loom.loom_debug_decode_form(request.param)
-    yield request.param
+    f, tc = request.param
+    loom.loom_debug_decode_form(f)
+    loom.loom_debug_decode_tensor_cores(tc)
+    yield f
     loom.loom_debug_decode_form(0)
+    loom.loom_debug_decode_tensor_cores(True)
 
 
 def _expect_form(loom, form, B, Hq, Hkv, Skv, D, splits):
@@ -120,7 +125,25 @@ def test_edge_lengths(loom, form, D):
         assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"D={D} splits={splits}")
 
 
-@pytest.mark.parametrize("Hq,Hkv", [(1, 1), (3, 1), (8, 8), (16, 2), (32, 1), (12, 4)])
+@pytest.mark.parametrize("D", [64, 128])
+def test_cache_past_length_is_never_used(loom, form, D):
+    """Keys and values past a sequence's length may hold anything (NaN here): the output
+    equals the oracle's on a finite cache, in every form (the tensor-core split kernel
+    zeroes the V rows of a ragged last stage before P.V)."""
+    B, Hq, Hkv, Skv = 3, 16, 4, 400
+    q, k, v = _inputs(21, B, Hq, Hkv, Skv, D)
+    lens = np.array([1, 257, 390], np.int32)
+    kp, vp = k.copy(), v.copy()
+    for b, n in enumerate(lens):
+        kp[b, :, n:] = 0x7FC0  # bf16 quiet NaN
+        vp[b, :, n:] = 0x7FC0
+    o_ref, lse_ref = oracle.attention(q, k, v, seqlens_k=lens)
+    for splits in (1, 3, 7):
+        o, lse = _run(loom, q, kp, vp, lens, splits)
+        assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"D={D} splits={splits}")
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(1, 1), (3, 1), (8, 8), (16, 2), (32, 1), (12, 4), (64, 2)])
 def test_group_sizes(loom, form, Hq, Hkv):
     B, Skv, D = 2, 777, 128
     q, k, v = _inputs(Hq + Hkv, B, Hq, Hkv, Skv, D)

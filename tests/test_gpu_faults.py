@@ -46,7 +46,11 @@ def _expect_timeout(loom, call):
     loom.loom_attn_check_error()  # the word was cleared
 
 
-def test_decode_skipped_stage_times_out_and_context_survives(loom):
+@pytest.mark.parametrize("tensor_cores", [True, False], ids=["tc", "cuda_core"])
+def test_decode_skipped_stage_times_out_and_context_survives(loom, tensor_cores):
+    """The split kernel on the tensor cores and on the CUDA cores: a stage whose copy is
+    never issued times out, the kernel returns (its MMAs drained, TMEM released) and the
+    next call is correct."""
     B, Hq, Hkv, Skv, D = 1, 4, 1, 2048, 128  # one split of 32 stages, one CTA
     q = synth.bf16_normal(31, synth.STREAM_Q, (B, Hq, 1, D))
     k = synth.bf16_normal(31, synth.STREAM_K, (B, Hkv, Skv, D))
@@ -57,9 +61,13 @@ def test_decode_skipped_stage_times_out_and_context_survives(loom):
         loom.loom_debug_inject(1)
         loom.loom_attn_decode(qd, kd, vd, None, num_splits=1)
 
-    _expect_timeout(loom, bad)
-    o, lse = loom.loom_attn_decode(qd, kd, vd, None, num_splits=1, return_lse=True)
-    loom.loom_attn_check_error()
+    loom.loom_debug_decode_tensor_cores(tensor_cores)
+    try:
+        _expect_timeout(loom, bad)
+        o, lse = loom.loom_attn_decode(qd, kd, vd, None, num_splits=1, return_lse=True)
+        loom.loom_attn_check_error()
+    finally:
+        loom.loom_debug_decode_tensor_cores(True)
     o_ref, lse_ref = oracle.attention(q, k, v)
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "decode after timeout")
 
