@@ -99,8 +99,9 @@ int loom_attn_decode_num_splits(int B, int Hq, int Hkv, int Skv, int D);
 
 /*
  * Device workspace (bytes) that loom_attn_decode needs: the per-split partial outputs
- * O_i [B, Hq, splits, D] fp32 and log-sum-exps lse_i [B, Hq, splits] fp32.  num_splits
- * = 0 means the model's choice.  Returns 0 on invalid sizes.
+ * O_i [B, Hq, splits, D] fp32 and log-sum-exps lse_i [B, Hq, splits] fp32 (each from a
+ * 256-byte boundary), then 256 bytes holding the persistent split kernel's item counter.
+ * num_splits = 0 means the model's choice.  Returns 0 on invalid sizes.
  */
 size_t loom_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int Skv, int D, int num_splits);
 
@@ -114,7 +115,9 @@ size_t loom_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int Skv, int D, 
  *   o          [B, Hq, 1, D]      bf16, written
  *   lse        [B, Hq]            fp32, written; may be NULL
  *   workspace  device scratch of at least loom_attn_decode_workspace_bytes(...) bytes;
- *              its contents on entry do not matter and are overwritten.
+ *              its contents on entry do not matter and are overwritten (the item
+ *              counter in its last 256 bytes is left armed for the next call; a
+ *              workspace serves one call at a time).
  *   num_splits 0 = analytic model, otherwise 1..1024 splits of each sequence.
  * Split i of sequence b covers keys [i*C, min((i+1)*C, len_b)), C = ceil(len_b/splits)
  * rounded up to a multiple of 64; empty splits contribute nothing.  A sequence of
@@ -236,6 +239,14 @@ double loom_model_decode_cluster_time_us(int splits, int cluster, int B, int Hq,
  * resident CTAs; < 0 on bad sizes. */
 double loom_model_decode_persistent_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int ctas);
 
+/* Modeled time (us) of the split + merge form with its split kernel on the tensor cores
+ * (persistent CTAs, two per SM of `num_sms`, taking the items on demand): the start-up
+ * once, the items in rounds of at most 2 * num_sms, each streaming its chunk and paying a
+ * fixed boundary cost, then the merge.  The split count with num_splits = 0 and the form
+ * of a contiguous-cache call use it where that kernel takes the shape (at most 32 query
+ * heads per kv head); < 0 on bad sizes or more heads per kv head. */
+double loom_model_decode_tc_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms);
+
 /*
  * Which Flash Decode form a call with these sizes runs on the current device: 1 = split
  * kernel + merge kernel, 2 = persistent split kernel + merge kernel, 3 = the single-kernel
@@ -356,15 +367,21 @@ void loom_debug_gemm_stages(int stages);
 void loom_debug_gemm_order(int group_rows, int k_alternate);
 
 /*
- * loom_debug_decode_tensor_cores: 1 (the default) lets the split + merge form run its
- * split kernel on the tensor cores for a contiguous cache (D 64 or 128, at most 32 query
- * heads per kv head): per 64-key stage, S = Q K^T and O += P V as tcgen05 MMAs with the
- * query heads as rows of a TMEM tile, the softmax on one warp; 0 runs the CUDA-core split
- * kernel instead (the paged cache and the persistent forms always use the CUDA-core
- * stage).  P is rounded to bf16 before P V on the tensor cores, as in the prefill; the
- * CUDA-core stage keeps it in fp32.
+ * loom_debug_decode_tensor_cores: which split kernel the split + merge form runs on a
+ * contiguous cache (D 64 or 128, at most 32 query heads per kv head; the paged cache and
+ * the other forms always use the CUDA-core stage).
+ *   1 (the default): tensor cores, persistent.  Two CTAs per SM take (sequence, kv head,
+ *     split) items, longest sequence first, from a counter in the workspace's last 256
+ *     bytes until none is left, and stream the next item's q and K/V without a break; per
+ *     64-key stage S = Q K^T and O += P V are tcgen05 MMAs with the query heads as rows
+ *     of a TMEM tile and the softmax on one warp.  The merge kernel re-arms the counter;
+ *     a workspace whose counter was never armed (its first call) is dealt statically.
+ *   2: the same stage on the tensor cores, one CTA per (split, kv head, sequence).
+ *   0: the CUDA-core split kernel.
+ * Other values select 1.  On the tensor cores P is rounded to bf16 before P V, as in
+ * the prefill; the CUDA-core stage keeps it in fp32.
  */
-void loom_debug_decode_tensor_cores(int on);
+void loom_debug_decode_tensor_cores(int mode);
 
 /*
  * Test hook: the Flash Decode form.  form 1 = split + merge kernels, 2 = persistent split

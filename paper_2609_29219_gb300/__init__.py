@@ -29,7 +29,7 @@ __all__ = [
     "loom_attn_decode_paged", "loom_attn_fwd_varlen", "loom_gemm_bf16", "loom_gemm_bf16_bt", "loom_gemm_tile_n", "loom_gemm_splits", "loom_gemm_cta_pair", "loom_model_gemm_time_us", "loom_debug_gemm_tile_n",
     "loom_debug_gemm_splits", "loom_debug_gemm_cta_pair", "loom_model_decode_cluster_time_us",
     "loom_attn_decode_form", "loom_decode_max_clusters", "loom_decode_persistent_slots", "loom_debug_decode_form",
-    "loom_model_decode_persistent_time_us", "DECODE_SPLIT_MERGE", "DECODE_PERSISTENT", "DECODE_CLUSTER",
+    "loom_model_decode_persistent_time_us", "loom_model_decode_tc_time_us", "DECODE_SPLIT_MERGE", "DECODE_PERSISTENT", "DECODE_CLUSTER",
     "loom_debug_prefill_slots", "loom_debug_decode_stage_plan", "loom_debug_gemm_stages",
     "loom_debug_gemm_order", "loom_debug_decode_tensor_cores",
 ]
@@ -138,6 +138,8 @@ def capi() -> ctypes.CDLL:
             lib.loom_model_decode_cluster_time_us.restype = ctypes.c_double
             lib.loom_model_decode_persistent_time_us.argtypes = [i32] * 7
             lib.loom_model_decode_persistent_time_us.restype = ctypes.c_double
+            lib.loom_model_decode_tc_time_us.argtypes = [i32] * 7
+            lib.loom_model_decode_tc_time_us.restype = ctypes.c_double
             lib.loom_attn_decode_form.argtypes = [i32] * 7 + [ctypes.POINTER(i32)]
             lib.loom_attn_decode_form.restype = i32
             lib.loom_decode_max_clusters.argtypes = [i32, i32, i32]
@@ -523,6 +525,10 @@ def loom_model_decode_persistent_time_us(splits, B, Hq, Hkv, Skv, D, ctas) -> fl
     return float(capi().loom_model_decode_persistent_time_us(splits, B, Hq, Hkv, Skv, D, ctas))
 
 
+def loom_model_decode_tc_time_us(splits, B, Hq, Hkv, Skv, D, num_sms) -> float:
+    return float(capi().loom_model_decode_tc_time_us(splits, B, Hq, Hkv, Skv, D, num_sms))
+
+
 def loom_decode_persistent_slots(D, G) -> int:
     return int(capi().loom_decode_persistent_slots(D, G))
 
@@ -551,9 +557,10 @@ def loom_debug_gemm_stages(stages: int) -> None:
     capi().loom_debug_gemm_stages(int(stages))
 
 
-def loom_debug_decode_tensor_cores(on: bool) -> None:
-    """Let the split + merge decode run its split kernel on the tensor cores (default), or not."""
-    capi().loom_debug_decode_tensor_cores(1 if on else 0)
+def loom_debug_decode_tensor_cores(mode) -> None:
+    """Split kernel of the split + merge decode on a contiguous cache: 1 / True (default)
+    tensor cores, persistent; 2 tensor cores, one CTA per split; 0 / False CUDA cores."""
+    capi().loom_debug_decode_tensor_cores(int(mode))
 
 
 def loom_debug_gemm_order(group_rows: int = 0, k_alternate: int = 0) -> None:

@@ -552,7 +552,7 @@ struct DecodeTcCfg {
   static constexpr uint32_t O_COL = 128;
   static constexpr uint32_t TMEM_COLS = 256;  // a power of two: 2 CTAs per SM
   static constexpr int THREADS = 96;
-  static constexpr int MAX_G = 32;            // query heads per kv head: TMEM lanes of warp 0
+  static constexpr int MAX_G = kDecodeTcMaxGroup;  // query heads per kv head: TMEM lanes of warp 0
   static_assert(O_COL + D <= TMEM_COLS, "TMEM budget");
   static_assert(Q_COL + D / 2 <= S_COL && S_COL + T <= O_COL, "TMEM regions");
   static_assert(2 * (BYTES + 1024) <= 228 * 1024 && 3 * (BYTES + 1024) > 228 * 1024, "exactly two CTAs per SM");
@@ -828,6 +828,404 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
     // ------------------------------------------------------------ query rows (warp 0)
     decode_tc_rows<D>(q, o_part, lse_part, tmem, b, h0, G, Hq, splits, row0, t_begin, t_end, n_st, c, smem, bar_full,
                       bar_q, bar_s, bar_p, bar_o, ctl, ab);
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------- tensor-core persistent split kernel
+// decode_tc_persist_kernel: the tensor-core split kernel as persistent CTAs (two per SM,
+// the TMEM and shared memory of DecodeTcCfg).  The loader takes (sequence, kv head, split)
+// items from the workspace counter (one atomic per item; the sequences sorted by length,
+// longest first) and streams each item's q (TMA, 128-byte swizzled, 64 dims per box) and
+// K/V stages into the ring without a break between items.  With every stage it records in
+// the slot which item and which stage of it the slot holds; the MMA warp and the softmax
+// warp walk the ring and learn the item boundaries from those records, so neither needs
+// the counter.  A final record with b = -1 ends both.
+template <int D>
+struct DecodeTcPersistCfg {
+  using C = DecodeTcCfg<D>;
+  static constexpr int kMaxSortedB = 256;                 // sequences sorted by length
+  static constexpr uint32_t Q_BOX_BYTES = C::MAX_G * 128;  // up to 32 heads x 64 dims
+  static constexpr uint32_t Q_OFF = C::NSTAGE * C::STAGE_BYTES;
+  static constexpr uint32_t META_OFF = Q_OFF + C::NBOX * Q_BOX_BYTES;  // [NSTAGE] x 8 int32
+  static constexpr uint32_t ORDER_OFF = META_OFF + C::NSTAGE * 32;     // [kMaxSortedB] int32
+  static constexpr uint32_t LENS_OFF = ORDER_OFF + kMaxSortedB * 4;     // [kMaxSortedB] int32
+  static constexpr uint32_t BAR_OFF = LENS_OFF + kMaxSortedB * 4;
+  // barriers: full[NSTAGE], empty[NSTAGE], q_full, q_empty, q, s, p, o, drain
+  static constexpr int NBAR = 2 * C::NSTAGE + 7;
+  static constexpr uint32_t TMEM_PTR_OFF = BAR_OFF + NBAR * 8;
+  static constexpr uint32_t ABORT_OFF = TMEM_PTR_OFF + 8;
+  static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;  // + 1024-byte alignment slack
+  static_assert(Q_OFF % 1024 == 0 && Q_BOX_BYTES % 1024 == 0, "q boxes start on the swizzle period");
+  static_assert(2 * (BYTES + 1024) <= 228 * 1024 && 3 * (BYTES + 1024) > 228 * 1024, "exactly two CTAs per SM");
+};
+
+// Warp 0 of decode_tc_persist_kernel: the softmax of decode_tc_rows over the ring's
+// records.  At an item's first stage it moves the item's q rows from the swizzled boxes
+// into TMEM (lane h reads head h, its 16-byte chunks in swizzled order: no bank conflicts)
+// and starts a fresh running state; at its last stage it writes the item's partial.
+template <int D>
+__device__ __forceinline__ void decode_tc_persist_rows(const uint8_t* smem, float* __restrict__ o_part,
+                                                       float* __restrict__ lse_part, uint32_t tmem, int G, int Hq,
+                                                       int splits, float c, uint32_t bar_full, uint32_t bar_qf,
+                                                       uint32_t bar_qe, uint32_t bar_q, uint32_t bar_s, uint32_t bar_p,
+                                                       uint32_t bar_o, const KernelCtl& ctl, const Abort& ab) {
+  using C = DecodeTcCfg<D>;
+  using L = DecodeTcPersistCfg<D>;
+  const int lane = threadIdx.x & 31;
+  const bool real = lane < G;
+  const uint64_t c2 = f2(c, c);
+  float m_run = -INFINITY, l_run = 0.f;
+  int nq = 0;
+  for (int st = 0;; ++st) {
+    const int slot = st % C::NSTAGE;
+    if (!mbar_wait_warp(bar_full + 8 * slot, (st / C::NSTAGE) & 1, ctl, ab)) return;
+    const volatile int* rec = reinterpret_cast<const volatile int*>(smem + L::META_OFF + slot * 32);
+    const int b = rec[0];
+    if (b < 0) return;  // no more items
+    const int hk = rec[1], split = rec[2], j = rec[3], n_st = rec[4], ntok = rec[6];
+    if (j == 0) {
+      if (!mbar_wait_warp(bar_qf, nq & 1, ctl, ab)) return;
+#pragma unroll
+      for (int x = 0; x < C::NBOX; ++x) {
+        uint32_t w[32];
+        const uint8_t* row = smem + L::Q_OFF + x * L::Q_BOX_BYTES + (real ? lane : 0) * 128;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const uint4 v = real ? *reinterpret_cast<const uint4*>(row + ((i ^ (lane & 7)) << 4))
+                               : make_uint4(0u, 0u, 0u, 0u);
+          w[4 * i] = v.x;
+          w[4 * i + 1] = v.y;
+          w[4 * i + 2] = v.z;
+          w[4 * i + 3] = v.w;
+        }
+        tmem_st32(tmem + C::Q_COL + x * 32, w);
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(bar_qe);  // the q boxes may take the next item's rows
+        mbar_arrive(bar_q);   // q is in TMEM
+      }
+      ++nq;
+      m_run = -INFINITY;
+      l_run = 0.f;
+    }
+    if (!mbar_wait_warp(bar_s, st & 1, ctl, ab)) return;
+    tc_fence_after();
+    uint32_t s[C::T];
+    tmem_ld32(tmem + C::S_COL, s);
+    tmem_ld32(tmem + C::S_COL + 32, s + 32);
+    tmem_wait_ld();
+    reg_fence32(s);
+    reg_fence32(s + 32);
+    if (ntok < C::T) {
+#pragma unroll
+      for (int i = 0; i < C::T; ++i)
+        if (i >= ntok) s[i] = __float_as_uint(-INFINITY);
+    }
+    float mm[8];
+#pragma unroll
+    for (int g = 0; g < 8; ++g) mm[g] = __uint_as_float(s[g]);
+#pragma unroll
+    for (int i = 8; i + 16 <= C::T; i += 16)
+#pragma unroll
+      for (int g = 0; g < 8; ++g) mm[g] = max3(mm[g], __uint_as_float(s[i + g]), __uint_as_float(s[i + 8 + g]));
+#pragma unroll
+    for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], __uint_as_float(s[C::T - 8 + g]));
+    const float mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
+    const float m_new = fmaxf(m_run, mx * c);
+    const bool need = m_new > m_run + kRescaleThreshold;
+    const float alpha = need ? ex2(m_run - m_new) : 1.f;
+    if (need) m_run = m_new;
+    const float ms = (m_run == -INFINITY) ? 0.f : m_run;
+    const uint64_t nms2 = f2(-ms, -ms);
+    uint64_t acc[4] = {0, 0, 0, 0};
+    uint32_t pk[C::T / 2];
+#pragma unroll
+    for (int i = 0; i < C::T / 2; ++i) {
+      const uint64_t x = fma2(f2(__uint_as_float(s[2 * i]), __uint_as_float(s[2 * i + 1])), c2, nms2);
+      const float p0 = ex2(f2lo(x));
+      const float p1 = ex2(f2hi(x));
+      acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
+      pk[i] = pack_bf16x2(p0, p1);
+    }
+    tmem_st32(tmem + C::S_COL, pk);
+    tmem_wait_st();
+    if (ntok < C::T) {
+      // V rows past the split's end may hold anything: zero them (P = 0 meets 0)
+      uint4* vt = reinterpret_cast<uint4*>(const_cast<uint8_t*>(smem) + slot * C::STAGE_BYTES + C::TILE_BYTES);
+#pragma unroll
+      for (int x = 0; x < C::NBOX; ++x)
+        for (int i = lane; i < (C::T - ntok) * 8; i += 32)
+          vt[x * (C::BOX_BYTES / 16) + ntok * 8 + i] = make_uint4(0u, 0u, 0u, 0u);
+      fence_proxy_async_smem();
+    }
+    // O holds the previous stage's P.V (committed before this stage's S) when rescaled
+    if (j > 0 && __any_sync(0xffffffffu, need)) {
+      if (!mbar_wait_warp(bar_o, (st - 1) & 1, ctl, ab)) return;
+      tc_fence_after();
+      const uint64_t a2 = f2(alpha, alpha);
+#pragma unroll 1
+      for (int ch = 0; ch < D / 32; ++ch) {
+        uint32_t rr[32];
+        tmem_ld32(tmem + C::O_COL + ch * 32, rr);
+        tmem_wait_ld();
+        reg_fence32(rr);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const uint64_t x = mul2(f2(__uint_as_float(rr[2 * i]), __uint_as_float(rr[2 * i + 1])), a2);
+          rr[2 * i] = __float_as_uint(f2lo(x));
+          rr[2 * i + 1] = __float_as_uint(f2hi(x));
+        }
+        tmem_st32(tmem + C::O_COL + ch * 32, rr);
+      }
+      tmem_wait_st();
+    }
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar_p);
+    const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+    l_run = l_run * alpha + (f2lo(a01) + f2hi(a01));
+    if (j == n_st - 1) {
+      // the item's last P.V, then O / l and the log-sum-exp of each real row
+      if (!mbar_wait_warp(bar_o, st & 1, ctl, ab)) return;
+      tc_fence_after();
+      const size_t row0 = (static_cast<size_t>(b) * Hq + static_cast<size_t>(hk) * G) * splits + split;
+      const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
+      float* dst = o_part + (row0 + static_cast<size_t>(real ? lane : 0) * splits) * D;
+#pragma unroll 1
+      for (int ch = 0; ch < D / 32; ++ch) {
+        uint32_t rr[32];
+        tmem_ld32(tmem + C::O_COL + ch * 32, rr);
+        tmem_wait_ld();
+        reg_fence32(rr);
+        if (real) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            reinterpret_cast<float4*>(dst + ch * 32)[i] =
+                make_float4(__uint_as_float(rr[4 * i]) * inv_l, __uint_as_float(rr[4 * i + 1]) * inv_l,
+                            __uint_as_float(rr[4 * i + 2]) * inv_l, __uint_as_float(rr[4 * i + 3]) * inv_l);
+        }
+      }
+      if (real)
+        lse_part[row0 + static_cast<size_t>(lane) * splits] = l_run > 0.f ? (m_run + log2f(l_run)) * kLn2 : -INFINITY;
+    }
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
+    decode_tc_persist_kernel(const int32_t* __restrict__ seqlens, float* __restrict__ o_part,
+                             float* __restrict__ lse_part, unsigned long long* __restrict__ sched, int B, int Hq,
+                             int Hkv, int Skv, int splits, float c, KernelCtl ctl, const __grid_constant__ CUtensorMap tm_q,
+                             const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v) {
+  using C = DecodeTcCfg<D>;
+  using L = DecodeTcPersistCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  // Let the merge grid launch as soon as every CTA is resident.
+  asm volatile("griddepcontrol.launch_dependents;");
+  const uint32_t raw_base = smem_u32(smem_raw);
+  const uint32_t sbase = (raw_base + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (sbase - raw_base);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = Hq / Hkv;
+  const long long per_seq = static_cast<long long>(Hkv) * splits;
+  const long long n_items = B * per_seq;
+
+  // the sequences in order of decreasing length (ties by index): items are taken in it
+  int* order = reinterpret_cast<int*>(smem + L::ORDER_OFF);
+  const bool sorted = seqlens != nullptr && B <= L::kMaxSortedB;
+  if (sorted) {
+    int* lens = reinterpret_cast<int*>(smem + L::LENS_OFF);
+    for (int bb = threadIdx.x; bb < B; bb += blockDim.x) lens[bb] = seqlens[bb];
+    __syncthreads();
+    for (int bb = threadIdx.x; bb < B; bb += blockDim.x) {
+      const int lb = lens[bb];
+      int r = 0;
+      for (int x = 0; x < B; ++x) {
+        const int lx = lens[x];
+        r += (lx > lb) || (lx == lb && x < bb);
+      }
+      order[r] = bb;
+    }
+  }
+  const uint32_t bar_full = sbase + L::BAR_OFF;
+  const uint32_t bar_empty = bar_full + 8 * C::NSTAGE;
+  const uint32_t bar_qf = bar_empty + 8 * C::NSTAGE;  // an item's q rows are in the boxes
+  const uint32_t bar_qe = bar_qf + 8;                 // the boxes were read
+  const uint32_t bar_q = bar_qe + 8;                  // q is in TMEM
+  const uint32_t bar_s = bar_q + 8;                   // S of the stage is in TMEM
+  const uint32_t bar_p = bar_s + 8;                   // P of the stage is in TMEM (O rescaled)
+  const uint32_t bar_o = bar_p + 8;                   // the stage's P.V is done
+  const uint32_t bar_drain = bar_o + 8;
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + L::TMEM_PTR_OFF);
+  Abort ab{reinterpret_cast<volatile int*>(smem + L::ABORT_OFF)};
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSTAGE; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, 1);
+    }
+    mbar_init(bar_qf, 1);
+    mbar_init(bar_qe, 1);
+    mbar_init(bar_q, 1);
+    mbar_init(bar_s, 1);
+    mbar_init(bar_p, 1);
+    mbar_init(bar_o, 1);
+    mbar_init(bar_drain, 1);
+    *ab.flag = 0;
+    *(ab.flag + 1) = 0;
+    fence_barrier_init();
+  }
+  if (warp == 2) tmem_alloc(smem_u32(tmem_ptr), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_ptr;
+
+  if (warp == 1) {
+    // ------------------------------------------------------------ loader (lane 0)
+    if (lane == 0) {
+      prefetch_tensormap(&tm_q);
+      prefetch_tensormap(&tm_k);
+      prefetch_tensormap(&tm_v);
+      // Item blockIdx.x first.  An armed counter deals the items past the first gridDim.x
+      // on demand, one ticket fetched an item ahead so that its latency is hidden; a
+      // workspace never armed (its first call) deals them statically, item blockIdx.x +
+      // k * gridDim.x (every CTA reads the same unarmed tag: all take the same branch).
+      unsigned long long ticket = atomicAdd(sched, 1ull);
+      int dynamic = -1;  // read from the first ticket once the first item is under way
+      long long item = blockIdx.x;
+      int st = 0, nq = 0, skipped = -1;
+      bool ok = true;
+      for (long long kk = 1; ok && item < n_items; ++kk) {
+        const int rb = static_cast<int>(item / per_seq);
+        const int rem = static_cast<int>(item - rb * per_seq);
+        const int b = sorted ? order[rb] : rb;
+        const int split = rem / Hkv, hk = rem - split * Hkv;
+        int len = seqlens ? seqlens[b] : Skv;
+        len = max(0, min(len, Skv));
+        int chunk = (len + splits - 1) / splits;
+        chunk = (chunk + kDecodeChunkAlign - 1) / kDecodeChunkAlign * kDecodeChunkAlign;
+        const int t_begin = min(split * chunk, len);
+        const int t_end = min(t_begin + chunk, len);
+        if (t_begin >= t_end) {
+          // empty split: contributes nothing to the merge
+          const size_t row0 = (static_cast<size_t>(b) * Hq + static_cast<size_t>(hk) * G) * splits + split;
+          for (int r = 0; r < G; ++r) {
+            float4* dst = reinterpret_cast<float4*>(o_part + (row0 + static_cast<size_t>(r) * splits) * D);
+            for (int i = 0; i < D / 4; ++i) dst[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+            lse_part[row0 + static_cast<size_t>(r) * splits] = -INFINITY;
+          }
+        } else {
+          // the item's q rows, once the softmax warp has moved the previous ones to TMEM
+          if (!(ok = mbar_wait(bar_qe, (nq & 1) ^ 1, ctl, ab))) break;
+          mbar_expect_tx(bar_qf, static_cast<uint32_t>(C::NBOX * G * 128));
+#pragma unroll
+          for (int x = 0; x < C::NBOX; ++x)
+            tma_load_3d(sbase + L::Q_OFF + x * L::Q_BOX_BYTES, &tm_q, x * 64, b * Hq + hk * G, 0, bar_qf);
+          ++nq;
+          const int n_st = (t_end - t_begin + C::T - 1) / C::T;
+          const int kv_z = b * Hkv + hk;
+          for (int j = 0; j < n_st; ++j, ++st) {
+            const int s = st % C::NSTAGE;
+            if (!(ok = mbar_wait(bar_empty + 8 * s, ((st / C::NSTAGE) & 1) ^ 1, ctl, ab))) break;
+            if (ctl.inject == 1 && st == 1) {  // test hook: never fill this stage
+              skipped = st;
+              continue;
+            }
+            const int tok0 = t_begin + j * C::T;
+            volatile int* rec = reinterpret_cast<volatile int*>(smem + L::META_OFF + s * 32);
+            rec[0] = b;
+            rec[1] = hk;
+            rec[2] = split;
+            rec[3] = j;
+            rec[4] = n_st;
+            rec[5] = tok0;
+            rec[6] = min(C::T, t_end - tok0);
+            const uint32_t dst = sbase + s * C::STAGE_BYTES;
+            mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
+#pragma unroll
+            for (int x = 0; x < C::NBOX; ++x) {
+              tma_load_3d(dst + x * C::BOX_BYTES, &tm_k, x * 64, tok0, kv_z, bar_full + 8 * s);
+              tma_load_3d(dst + C::TILE_BYTES + x * C::BOX_BYTES, &tm_v, x * 64, tok0, kv_z, bar_full + 8 * s);
+            }
+          }
+        }
+        if (!ok) break;
+        if (dynamic < 0) dynamic = static_cast<uint32_t>(ticket >> 32) == kDecodeSchedTag ? 1 : 0;
+        if (dynamic) {
+          item = static_cast<long long>(gridDim.x) + static_cast<uint32_t>(ticket);
+          if (item < n_items) ticket = atomicAdd(sched, 1ull);
+        } else {
+          item = blockIdx.x + kk * static_cast<long long>(gridDim.x);
+        }
+      }
+      // the end record
+      bool ended = false;
+      if (ok) {
+        const int s = st % C::NSTAGE;
+        if (mbar_wait(bar_empty + 8 * s, ((st / C::NSTAGE) & 1) ^ 1, ctl, ab)) {
+          *reinterpret_cast<volatile int*>(smem + L::META_OFF + s * 32) = -1;
+          mbar_arrive(bar_full + 8 * s);
+          ended = true;
+        }
+      }
+      // Drain: never leave the CTA with copies still landing in its shared memory (after
+      // the end record the stage it replaced has been consumed).
+      Abort no_abort{ab.flag + 1};
+      for (int i = max(0, st - C::NSTAGE + (ended ? 1 : 0)); i < st; ++i)
+        if (i != skipped) mbar_wait(bar_full + 8 * (i % C::NSTAGE), (i / C::NSTAGE) & 1, ctl, no_abort);
+      if (nq > 0) mbar_wait(bar_qf, (nq - 1) & 1, ctl, no_abort);
+    }
+  } else if (warp == 2) {
+    // ------------------------------------------------------------ MMA issuer
+    constexpr uint32_t idesc_s = idesc_bf16(128, C::T, 0, 0);  // Q (TMEM) x K^T (K-major)
+    constexpr uint32_t idesc_pv = idesc_bf16(128, D, 0, 1);    // P (TMEM) x V (MN-major)
+    int nq = 0;
+    for (int st = 0;; ++st) {
+      const int s = st % C::NSTAGE;
+      if (!mbar_wait_warp(bar_full + 8 * s, (st / C::NSTAGE) & 1, ctl, ab)) break;
+      tc_fence_after();
+      const volatile int* rec = reinterpret_cast<const volatile int*>(smem + L::META_OFF + s * 32);
+      if (rec[0] < 0) break;  // no more items
+      const int j = rec[3];
+      if (j == 0) {  // an item's first stage: its q must be in TMEM
+        if (!mbar_wait_warp(bar_q, nq & 1, ctl, ab)) break;
+        tc_fence_after();
+        ++nq;
+      }
+      const uint32_t kslot = sbase + s * C::STAGE_BYTES;
+      // S = Q K^T (the previous stage's P.V, issued before, has read the P these columns
+      // held: the MMAs of a CTA run in issue order)
+#pragma unroll
+      for (int x = 0; x < C::NBOX; ++x)
+        mma_ts_kmaj_k64_el(tmem + C::S_COL, tmem + C::Q_COL + x * 32,
+                           sdesc_sw128(kslot + x * C::BOX_BYTES, 16, 1024), idesc_s, x > 0 ? 1u : 0u);
+      tc_commit_el(bar_s);
+      if (!mbar_wait_warp(bar_p, st & 1, ctl, ab)) break;
+      tc_fence_after();
+      mma_ts_k64_el(tmem + C::O_COL, tmem + C::S_COL, sdesc_sw128(kslot + C::TILE_BYTES, C::BOX_BYTES, 1024),
+                    idesc_pv, j > 0 ? 1u : 0u);
+      tc_commit_el(bar_o);
+      tc_commit_el(bar_empty + 8 * s);
+    }
+    // every MMA issued above is done before TMEM is released
+    Abort no_abort{ab.flag + 1};
+    tc_commit_el(bar_drain);
+    mbar_wait_warp(bar_drain, 0, ctl, no_abort);
+  } else {
+    // ------------------------------------------------------------ softmax (warp 0)
+    decode_tc_persist_rows<D>(smem, o_part, lse_part, tmem, G, Hq, splits, c, bar_full, bar_qf, bar_qe, bar_q, bar_s,
+                              bar_p, bar_o, ctl, ab);
   }
 
   __syncwarp();
@@ -1155,12 +1553,16 @@ template <int D>
 __global__ void __launch_bounds__(D) decode_merge_kernel(const float* __restrict__ o_part,
                                                          const float* __restrict__ lse_part,
                                                          __nv_bfloat16* __restrict__ o,
-                                                         float* __restrict__ lse, int splits) {
+                                                         float* __restrict__ lse, int splits,
+                                                         unsigned long long* __restrict__ sched) {
   constexpr int NW = D / 32;
   __shared__ float w_s[kMaxDecodeSplits];
   __shared__ float red[NW];
   // Wait until the split kernel's partials are complete and visible.
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  // The split kernel has taken its last item: arm the workspace's item counter for the next call.
+  if (sched != nullptr && blockIdx.x == 0 && threadIdx.x == 0)
+    *sched = static_cast<unsigned long long>(kDecodeSchedTag) << 32;
   const int bh = blockIdx.x, d = threadIdx.x, lane = d & 31, wid = d >> 5;
   const float* lp = lse_part + static_cast<size_t>(bh) * splits;
 
@@ -1389,7 +1791,7 @@ bool kv_map_sw128(CUtensorMap* map, const void* cache, int B, int Hkv, int Skv, 
 // query heads per kv head, the model's stage plan.
 bool decode_tc_eligible(const DecodeArgs& a) {
   const int G = a.Hq / a.Hkv;
-  return a.tc && a.stage_plan == 0 && G <= DecodeTcCfg<128>::MAX_G && (a.D == 64 || a.D == 128);
+  return a.tc != 0 && a.stage_plan == 0 && G <= DecodeTcCfg<128>::MAX_G && (a.D == 64 || a.D == 128);
 }
 
 template <int D>
@@ -1404,6 +1806,44 @@ cudaError_t launch_tc_split(const DecodeArgs& a, const KernelCtl& ctl, cudaStrea
   decode_tc_split_kernel<D><<<grid, C::THREADS, C::BYTES, stream>>>(
       static_cast<const __nv_bfloat16*>(a.q), a.seqlens, a.o_part, a.lse_part, a.Hq, a.Hkv, a.Skv, a.splits,
       a.scale * kLog2e, ctl, tk, tv);
+  return cudaGetLastError();
+}
+
+// The queries [B * Hq rows, D] as a 3-D tensor (dim, row, 1) in 64-dim x G-row boxes,
+// 128-byte swizzled: an item's q rows for the persistent tensor-core split kernel.
+bool q_map_sw128(CUtensorMap* map, const void* q, int rows, int D, int G) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(rows), 1};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(rows) * D * 2};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(G), 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// The persistent tensor-core split kernel: two CTAs per SM (or one per item when fewer).
+template <int D>
+cudaError_t launch_tc_persist(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+  using L = DecodeTcPersistCfg<D>;
+  if (a.sched == nullptr) return cudaErrorInvalidValue;
+  static PerDeviceOnce once;
+  if (!prepare_kernel(decode_tc_persist_kernel<D>, L::BYTES, false, once)) return cudaErrorInvalidValue;
+  const int G = a.Hq / a.Hkv;
+  CUtensorMap tq, tk, tv;
+  if (!q_map_sw128(&tq, a.q, a.B * a.Hq, D, G) || !kv_map_sw128(&tk, a.k, a.B, a.Hkv, a.Skv, D) ||
+      !kv_map_sw128(&tv, a.v, a.B, a.Hkv, a.Skv, D))
+    return cudaErrorInvalidValue;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
+                                                cudaSuccess)
+    return cudaErrorInvalidValue;
+  const long long items = static_cast<long long>(a.B) * a.Hkv * a.splits;
+  const long long ctas = items < 2LL * sms ? items : 2LL * sms;
+  decode_tc_persist_kernel<D><<<static_cast<unsigned>(ctas), DecodeTcCfg<D>::THREADS, L::BYTES, stream>>>(
+      a.seqlens, a.o_part, a.lse_part, a.sched, a.B, a.Hq, a.Hkv, a.Skv, a.splits, a.scale * kLog2e, ctl, tq, tk,
+      tv);
   return cudaGetLastError();
 }
 
@@ -1466,7 +1906,7 @@ cudaError_t launch_merge(const DecodeArgs& a, cudaStream_t stream) {
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, decode_merge_kernel<D>, static_cast<const float*>(a.o_part),
                             static_cast<const float*>(a.lse_part),
-                            static_cast<__nv_bfloat16*>(a.o), a.lse, a.splits);
+                            static_cast<__nv_bfloat16*>(a.o), a.lse, a.splits, a.sched);
 }
 
 // The Flash Decode form of a launch: kDecodeSplitMerge, kDecodePersistent (both with the
@@ -1492,7 +1932,9 @@ int decode_form(const DecodeArgs& a, int* cs_out) {
     *cs_out = ch.cs;
     return kDecodeCluster;
   }
-  const double t_split = model::decode_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms);
+  const double t_split = (!PAGED && decode_tc_eligible(a))
+                             ? model::decode_tc_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms)
+                             : model::decode_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms);
   const double t_persist =
       slots > 0 ? model::decode_persistent_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, slots) : 1e300;
   int form = kDecodeSplitMerge;
@@ -1545,7 +1987,7 @@ cudaError_t launch_form(const DecodeArgs& a, const PagedKV* pk, const KernelCtl&
   if (form == kDecodePersistent)
     e = launch_persist<D, GT, PAGED>(a, pk, ctl, stream);
   else if (!PAGED && decode_tc_eligible(a))
-    e = launch_tc_split<D>(a, ctl, stream);
+    e = a.tc == 2 ? launch_tc_split<D>(a, ctl, stream) : launch_tc_persist<D>(a, ctl, stream);
   else
     e = launch_split<D, GT, PAGED>(a, pk, ctl, stream);
   if (e != cudaSuccess) return e;

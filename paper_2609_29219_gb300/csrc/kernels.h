@@ -50,8 +50,17 @@ struct DecodeArgs {
   int cluster;  // cluster form: 0 = the model's cluster size, else this size (if it divides splits and fits)
   int stage_plan;  // 0: the model's stage plan; i > 0: the i-th compiled ablation plan (split + merge form)
   int by_model;    // 1: the split count is the model's (num_splits = 0), which then also picks the form
-  int tc;          // 1: the split + merge form's split kernel may run on the tensor cores (contiguous cache)
+  int tc;          // split + merge form's split kernel on a contiguous cache: 0 CUDA cores; tensor
+                   // cores, 1 persistent CTAs taking items from the workspace counter, 2 one CTA per split
+  unsigned long long* sched;  // the workspace's item counter (tag kDecodeSchedTag in the high word)
 };
+
+// High word of an armed item counter: a signalling-NaN pattern that no float the decode
+// path writes to the workspace carries, so that a workspace never used before is told
+// apart (its first call deals items statically; the merge kernel then arms the counter).
+constexpr uint32_t kDecodeSchedTag = 0x7FBADC0Du;
+// Query heads per kv head that the tensor-core split kernels take (the lanes of one warp).
+constexpr int kDecodeTcMaxGroup = 32;
 
 struct FwdArgs {
   const void* q;  // [B, Hq, Sq, D] bf16
@@ -76,7 +85,13 @@ inline size_t decode_workspace_bytes(int B, int Hq, int D, int splits) {
   const size_t rows = static_cast<size_t>(B) * Hq * splits;
   const size_t opart = rows * D * sizeof(float);
   const size_t lpart = rows * sizeof(float);
-  return ((opart + 255) / 256) * 256 + ((lpart + 255) / 256) * 256;
+  return ((opart + 255) / 256) * 256 + ((lpart + 255) / 256) * 256 + 256;  // + the item counter
+}
+
+// The item counter's place in a decode workspace (after the partial O and LSE).
+inline unsigned long long* decode_sched_word(void* workspace, int B, int Hq, int D, int splits) {
+  return reinterpret_cast<unsigned long long*>(static_cast<char*>(workspace) + decode_workspace_bytes(B, Hq, D, splits) -
+                                               256);
 }
 
 // Argument checks of the contiguous decode entry points, in their order, up to (not

@@ -35,7 +35,8 @@ int g_gemm_k_alt = 0;   // test hook: -1 stops the CTA-pair GEMM walking K backw
 int g_decode_form = 0;     // test hook: the Flash Decode form (0: the model's; kDecode* otherwise)
 int g_decode_cluster = 0;  // test hook: the cluster decode form's cluster size (0: the model's)
 int g_decode_stage_plan = 0;  // test hook: a compiled ablation stage plan of the decode split kernel
-int g_decode_tc = 1;  // test hook: 0 runs the split + merge form's CUDA-core split kernel on a contiguous cache
+// test hook: the split + merge form's split kernel on a contiguous cache (DecodeArgs::tc)
+int g_decode_tc = 1;
 
 constexpr int kMaxDevices = 64;
 uint32_t* g_err_ptr[kMaxDevices] = {};
@@ -64,9 +65,9 @@ int current_sm_count() {
 }
 
 struct SplitKey {
-  int B, Hq, Hkv, Skv, D, sms;
+  int B, Hq, Hkv, Skv, D, sms, tc;
   bool operator==(const SplitKey& o) const {
-    return B == o.B && Hq == o.Hq && Hkv == o.Hkv && Skv == o.Skv && D == o.D && sms == o.sms;
+    return B == o.B && Hq == o.Hq && Hkv == o.Hkv && Skv == o.Skv && D == o.D && sms == o.sms && tc == o.tc;
   }
 };
 std::vector<std::pair<SplitKey, int>> g_split_cache;
@@ -127,7 +128,10 @@ int loom_attn_decode_num_splits(int B, int Hq, int Hkv, int Skv, int D) {
   int sms = current_sm_count();
   if (sms <= 0) sms = model::kGb300.num_sms;
   // The enumeration costs ~0.1 ms of host time: remember the answer per problem shape.
-  const SplitKey key{B, Hq, Hkv, Skv, D, sms};
+  // the split + merge form's split kernel runs on the tensor cores for a contiguous cache
+  // (a paged cache takes the same split count, with the CUDA-core kernel)
+  const int tc = (g_decode_tc != 0 && Hq / Hkv <= kDecodeTcMaxGroup) ? 1 : 0;
+  const SplitKey key{B, Hq, Hkv, Skv, D, sms, tc};
   {
     std::lock_guard<std::mutex> lock(g_split_mutex);
     for (const auto& e : g_split_cache)
@@ -143,7 +147,7 @@ int loom_attn_decode_num_splits(int B, int Hq, int Hkv, int Skv, int D) {
                          [&](int cs) {
                            return device ? decode_max_clusters(D, G, cs) : model::decode_default_clusters(sms, cs, D);
                          },
-                         slots)
+                         slots, model::kGb300, tc != 0)
                          .splits;
   std::lock_guard<std::mutex> lock(g_split_mutex);
   if (g_split_cache.size() >= 256) g_split_cache.erase(g_split_cache.begin());
@@ -208,7 +212,8 @@ loom_status loom_attn_decode(const void* q, const void* k_cache, const void* v_c
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D,
-               num_splits, scale, g_decode_form, g_decode_cluster, g_decode_stage_plan, by_model, g_decode_tc};
+               num_splits, scale, g_decode_form, g_decode_cluster, g_decode_stage_plan, by_model, g_decode_tc,
+               decode_sched_word(workspace, B, Hq, D, num_splits)};
   return launch_decode(a, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                  : LOOM_ERR_CUDA;
 }
@@ -279,7 +284,7 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D, num_splits, scale,
-               g_decode_form, g_decode_cluster, 0, by_model, 0};
+               g_decode_form, g_decode_cluster, 0, by_model, 0, decode_sched_word(workspace, B, Hq, D, num_splits)};
   PagedKV pk{block_table, num_pages, page_size, max_pages, kv_layout};
   return launch_decode_paged(a, pk, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                           : LOOM_ERR_CUDA;
@@ -358,7 +363,7 @@ void loom_debug_gemm_cta_pair(int mode) { g_gemm_pair = (mode == 1 || mode == -1
 
 void loom_debug_gemm_stages(int stages) { g_gemm_stages = stages > 0 ? stages : 0; }
 
-void loom_debug_decode_tensor_cores(int on) { g_decode_tc = on ? 1 : 0; }
+void loom_debug_decode_tensor_cores(int mode) { g_decode_tc = (mode >= 0 && mode <= 2) ? mode : 1; }
 
 void loom_debug_gemm_order(int group_rows, int k_alternate) {
   g_gemm_group = (group_rows >= 1 && group_rows <= 1024) ? group_rows : 0;
@@ -436,6 +441,13 @@ double loom_model_decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, in
   return model::decode_time_us(splits, B, Hq, Hkv, Skv, D, num_sms);
 }
 
+double loom_model_decode_tc_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms) {
+  if (splits <= 0 || B <= 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv || Skv <= 0 || num_sms <= 0 ||
+      (D != 64 && D != 128) || Hq / Hkv > kDecodeTcMaxGroup)
+    return -1.0;
+  return model::decode_tc_time_us(splits, B, Hq, Hkv, Skv, D, num_sms);
+}
+
 int loom_attn_decode_form(int B, int Hq, int Hkv, int Skv, int D, int num_splits, int paged, int* cluster) {
   if (cluster) *cluster = 0;
   if (B <= 0 || Hq <= 0 || Hkv <= 0 || Skv <= 0 || Hq % Hkv != 0 || (D != 64 && D != 128) || num_splits < 0 ||
@@ -454,6 +466,7 @@ int loom_attn_decode_form(int B, int Hq, int Hkv, int Skv, int D, int num_splits
   a.splits = num_splits;
   a.form = g_decode_form;
   a.cluster = g_decode_cluster;
+  a.tc = g_decode_tc;
   int cs = 0;
   const int form = decode_form_of(a, paged != 0, &cs);
   cudaGetLastError();

@@ -65,12 +65,17 @@ struct ArchDesc {
                                     // and K/V loads from HBM and the last item's epilogue
                                     // (fitted with item_boundary_ns: B1 H32 S1024 measured 23.2 us,
                                     // B16 H16 S512 45.5 us, one and four items per CTA)
+  double decode_tc_item_ns;         // persistent tensor-core decode: per (sequence, kv head, split)
+                                    // item, the stall of the S -> softmax -> P.V chain at the item's
+                                    // boundary (O read-out, next q into TMEM) that the full ring does
+                                    // not hide (fitted: batched B16 H32/8 lengths U[4096, 8192], 16 vs
+                                    // 32 splits, 70.9 vs 74.2 us, less the merge's extra partials)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 3400.0, 3000.0, 28.4, 150.0, 7800.0,
+    129.0e6, 1.07, 3400.0, 3000.0, 28.4, 150.0, 7800.0, 300.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -452,6 +457,29 @@ constexpr double decode_persistent_time_us(int splits, int B, int Hq, int Hkv, i
   return heg_seq(t_split, t_merge) * 1e-3;
 }
 
+// Eq. 5 for the split + merge form whose split kernel runs on the tensor cores as
+// persistent CTAs (two per SM) taking the items on demand: the start-up once; the items,
+// all of one length, go in rounds of at most `ctas` (the last round may be partial, its
+// CTAs then sharing HBM among fewer); each item streams its chunk at the CTA's rate and
+// pays decode_tc_item_ns at its boundary; then the merge launch.
+constexpr double decode_tc_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms,
+                                   const ArchDesc& a = kGb300) {
+  if (splits < 1 || num_sms < 1) return 1e300;
+  const long long items = 1LL * B * Hkv * splits;
+  const long long slots = 2LL * num_sms;
+  const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
+  const double chunk_bytes = 2.0 * chunk * D * 2;
+  double t_split = a.cta_start_ns;
+  for (long long left = items; left > 0;) {
+    const long long active = left < slots ? left : slots;
+    left -= active;
+    t_split += chunk_bytes / decode_cta_rate(static_cast<double>(active), num_sms, a) + a.decode_tc_item_ns;
+  }
+  const double part_bytes = 1.0 * B * Hq * splits * (D + 1) * 4;
+  const double t_merge = a.launch_ns * 0.2 + 2.0 * part_bytes / a.hbm_gbs;
+  return heg_seq(t_split, t_merge) * 1e-3;
+}
+
 // Clusters of cs decode CTAs in one GPC-sized group when no device can be asked: whole
 // clusters in 8 equal groups of SMs at the stage plan's CTAs per SM.
 constexpr int decode_default_clusters(int num_sms, int cs, int D) {
@@ -482,17 +510,19 @@ constexpr DecodeClusterChoice choose_decode_cluster(int splits, int B, int Hq, i
   return best;
 }
 
-// Eq. 9 over the Flash Decode forms and every split count: the split + merge form, the
-// persistent split + merge form on `slots` CTAs (0: not considered) and the cluster form
-// with fit(cs) clusters of cs CTAs (always 0: not considered).  Ties keep the earlier form
-// and fewer splits.  DecodeSplitPlan::cluster: 0 split + merge, -1 persistent, cs cluster.
+// Eq. 9 over the Flash Decode forms and every split count: the split + merge form (its
+// split kernel on the tensor cores when `tc`), the persistent split + merge form on
+// `slots` CTAs (0: not considered) and the cluster form with fit(cs) clusters of cs CTAs
+// (always 0: not considered).  Ties keep the earlier form and fewer splits.
+// DecodeSplitPlan::cluster: 0 split + merge, -1 persistent, cs cluster.
 template <class Fit>
 constexpr DecodeSplitPlan choose_decode_plan(int B, int Hq, int Hkv, int Skv, int D, int num_sms, Fit fit,
-                                             int slots = 0, const ArchDesc& a = kGb300) {
+                                             int slots = 0, const ArchDesc& a = kGb300, bool tc = false) {
   DecodeSplitPlan best{1, 1e300, 0};
   const long long max_splits = cdiv(Skv, 64) < 1024 ? cdiv(Skv, 64) : 1024;
   for (int s = 1; s <= max_splits; ++s) {
-    const double t = decode_time_us(s, B, Hq, Hkv, Skv, D, num_sms, a);
+    const double t = tc ? decode_tc_time_us(s, B, Hq, Hkv, Skv, D, num_sms, a)
+                        : decode_time_us(s, B, Hq, Hkv, Skv, D, num_sms, a);
     if (t < best.t_us * (1.0 - 1e-9)) best = {s, t, 0};
   }
   for (int s = 1; slots > 0 && s <= max_splits; ++s) {

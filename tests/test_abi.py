@@ -85,10 +85,11 @@ def test_decode_rejects_bad_arguments(lib):
 
 
 def test_workspace_size_formula(lib):
-    # O_i [B,Hq,S,D] fp32 + lse_i [B,Hq,S] fp32, each padded to 256 bytes
+    # O_i [B,Hq,S,D] fp32 + lse_i [B,Hq,S] fp32, each padded to 256 bytes, + 256 bytes
+    # for the persistent split kernel's item counter
     B, Hq, D, S = 3, 8, 128, 7
     rows = B * Hq * S
-    expect = (rows * D * 4 + 255) // 256 * 256 + (rows * 4 + 255) // 256 * 256
+    expect = (rows * D * 4 + 255) // 256 * 256 + (rows * 4 + 255) // 256 * 256 + 256
     assert lib.loom_attn_decode_workspace_bytes(B, Hq, 2, 4096, D, S) == expect
     assert lib.loom_attn_decode_workspace_bytes(B, Hq, 2, 4096, 96, S) == 0
     assert lib.loom_attn_decode_workspace_bytes(B, Hq, 2, 4096, D, 2000) == 0

@@ -22,19 +22,20 @@ def loom():
     return m
 
 
-@pytest.fixture(autouse=True, params=[(0, True), (1, True), (1, False), (2, True), (3, True)],
-                ids=["model_form", "split_merge", "split_merge_cuda_core", "persistent", "cluster"])
+@pytest.fixture(autouse=True, params=[(0, 1), (1, 1), (1, 2), (1, 0), (2, 1), (3, 1)],
+                ids=["model_form", "split_merge", "split_merge_tc_per_split", "split_merge_cuda_core",
+                     "persistent", "cluster"])
 def form(request, loom):
     """Every test runs with the model's choice of form and with each form forced: split
-    kernel + merge (its split kernel on the tensor cores where it takes the shape, and on
-    the CUDA cores), persistent split kernel + merge, and the single-kernel cluster form (at
-    the model's cluster size)."""
+    kernel + merge (its split kernel on the tensor cores where it takes the shape --
+    persistent CTAs, or one CTA per split -- and on the CUDA cores), persistent split
+    kernel + merge, and the single-kernel cluster form (at the model's cluster size)."""
     f, tc = request.param
     loom.loom_debug_decode_form(f)
     loom.loom_debug_decode_tensor_cores(tc)
     yield f
     loom.loom_debug_decode_form(0)
-    loom.loom_debug_decode_tensor_cores(True)
+    loom.loom_debug_decode_tensor_cores(1)
 
 
 def _expect_form(loom, form, B, Hq, Hkv, Skv, D, splits):
@@ -171,6 +172,43 @@ def test_partials_match_oracle_split_form(loom, form):
     off = (n * D * 4 + 255) // 256 * 256
     lpart = ws[off: off + n * 4].view(torch.float32).cpu().numpy().astype(np.float64).reshape(B, Hq, S)
     assert_parity(opart, o_part_ref, lpart, lse_part_ref, "partials")
+
+
+def test_item_counter_first_call_static_then_armed(loom, form):
+    """The persistent tensor-core split kernel takes items from a counter in the
+    workspace's last 256 bytes.  A workspace never used (all bytes 0xFF) is dealt
+    statically; the merge kernel then arms the counter, and the next call, dealt on
+    demand, gives the same bits (each item's arithmetic does not depend on its CTA)."""
+    import torch
+    B, Hq, Hkv, Skv, D, S = 4, 32, 8, 3000, 128, 7
+    q, k, v = (to_dev(x) for x in _inputs(17, B, Hq, Hkv, Skv, D))
+    sl = torch.tensor([3000, 1, 2047, 700], dtype=torch.int32, device="cuda")
+    nbytes = loom.loom_attn_decode_workspace_bytes(B, Hq, Hkv, Skv, D, S)
+    ws = torch.full((nbytes,), 0xFF, dtype=torch.uint8, device="cuda")
+    o1, l1 = loom.loom_attn_decode(q, k, v, sl, num_splits=S, workspace=ws, return_lse=True)
+    loom.loom_attn_check_error()
+    word = int(ws[nbytes - 256: nbytes - 248].cpu().view(torch.int64)[0]) & 0xFFFFFFFFFFFFFFFF
+    if form in (0, 1):  # the split + merge form's merge kernel arms the counter
+        assert word == 0x7FBADC0D << 32
+    o2, l2 = loom.loom_attn_decode(q, k, v, sl, num_splits=S, workspace=ws, return_lse=True)
+    loom.loom_attn_check_error()
+    assert torch.equal(o1.view(torch.int16), o2.view(torch.int16))
+    assert torch.equal(l1, l2)
+    o_ref, lse_ref = oracle.attention(*(_inputs(17, B, Hq, Hkv, Skv, D)), seqlens_k=sl.cpu().numpy())
+    assert_parity(o_to_f64(o2), o_ref, l2.cpu().numpy(), lse_ref, "armed counter")
+
+
+def test_more_sequences_than_the_length_sort_takes(loom, form):
+    """Above 256 sequences the persistent kernels take the sequences in index order instead
+    of sorting them by length; lengths 0..200 with empty sequences and empty splits."""
+    B, Hq, Hkv, Skv, D = 300, 4, 1, 200, 64
+    q, k, v = _inputs(23, B, Hq, Hkv, Skv, D)
+    lens = np.random.default_rng(23).integers(0, Skv + 1, size=B).astype(np.int32)
+    lens[:3] = [0, 200, 1]
+    o_ref, lse_ref = oracle.attention(q, k, v, seqlens_k=lens)
+    for splits in (1, 3):
+        o, lse = _run(loom, q, k, v, lens, splits)
+        assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, f"B=300 splits={splits}")
 
 
 def test_workspace_and_argument_errors(loom):

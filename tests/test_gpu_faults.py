@@ -46,11 +46,11 @@ def _expect_timeout(loom, call):
     loom.loom_attn_check_error()  # the word was cleared
 
 
-@pytest.mark.parametrize("tensor_cores", [True, False], ids=["tc", "cuda_core"])
+@pytest.mark.parametrize("tensor_cores", [1, 2, 0], ids=["tc_persistent", "tc_per_split", "cuda_core"])
 def test_decode_skipped_stage_times_out_and_context_survives(loom, tensor_cores):
-    """The split kernel on the tensor cores and on the CUDA cores: a stage whose copy is
-    never issued times out, the kernel returns (its MMAs drained, TMEM released) and the
-    next call is correct."""
+    """The split kernel on the tensor cores (persistent, or one CTA per split) and on the
+    CUDA cores: a stage whose copy is never issued times out, the kernel returns (its
+    copies and MMAs drained, TMEM released) and the next call is correct."""
     B, Hq, Hkv, Skv, D = 1, 4, 1, 2048, 128  # one split of 32 stages, one CTA
     q = synth.bf16_normal(31, synth.STREAM_Q, (B, Hq, 1, D))
     k = synth.bf16_normal(31, synth.STREAM_K, (B, Hkv, Skv, D))
@@ -67,7 +67,7 @@ def test_decode_skipped_stage_times_out_and_context_survives(loom, tensor_cores)
         o, lse = loom.loom_attn_decode(qd, kd, vd, None, num_splits=1, return_lse=True)
         loom.loom_attn_check_error()
     finally:
-        loom.loom_debug_decode_tensor_cores(True)
+        loom.loom_debug_decode_tensor_cores(1)
     o_ref, lse_ref = oracle.attention(q, k, v)
     assert_parity(o_to_f64(o), o_ref, lse.cpu().numpy(), lse_ref, "decode after timeout")
 

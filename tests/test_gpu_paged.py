@@ -131,13 +131,13 @@ def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P, layout):
     lens = np.array([S, 777, 64], dtype=np.int32)
     for splits in (1, 5):
         o1, l1 = run_paged(loom, q, kc, vc, table, lens, splits, layout)
-        loom.loom_debug_decode_tensor_cores(False)
+        loom.loom_debug_decode_tensor_cores(0)
         try:
             o2, l2 = loom.loom_attn_decode(to_dev(q), to_dev(k), to_dev(v), torch.from_numpy(lens).cuda(),
                                            num_splits=splits, return_lse=True)
             loom.loom_attn_check_error()
         finally:
-            loom.loom_debug_decode_tensor_cores(True)
+            loom.loom_debug_decode_tensor_cores(1)
         assert torch.equal(o1.view(torch.int16), o2.view(torch.int16))
         assert torch.equal(l1, l2)
 

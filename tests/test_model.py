@@ -110,15 +110,18 @@ DECODE_SHAPES = [(16, 32, 8, 8192, 128), (1, 32, 8, 131072, 128), (1, 8, 8, 4096
 
 
 def _decode_candidates(loom, B, Hq, Hkv, Skv, D):
-    """Modeled time of every (form, split count) candidate: the split + merge form and the
-    persistent split + merge form for every split count, the cluster form for every split
-    count and cluster size dividing it, with the CTAs and clusters they are priced at.
-    Form order for ties: split + merge (0), persistent (1), cluster (2)."""
+    """Modeled time of every (form, split count) candidate: the split + merge form (its
+    split kernel on the tensor cores where that kernel takes the shape, at most 32 query
+    heads per kv head) and the persistent split + merge form for every split count, the
+    cluster form for every split count and cluster size dividing it, with the CTAs and
+    clusters they are priced at.  Form order for ties: split + merge (0), persistent (1),
+    cluster (2)."""
     cands = []
     G = Hq // Hkv
     slots = loom.loom_decode_persistent_slots(D, G)
+    split_merge = loom.loom_model_decode_tc_time_us if G <= 32 else loom.loom_model_decode_time_us
     for s in range(1, min(1024, math.ceil(Skv / 64)) + 1):
-        cands.append((loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS), 0, s))
+        cands.append((split_merge(s, B, Hq, Hkv, Skv, D, NUM_SMS), 0, s))
         cands.append((loom.loom_model_decode_persistent_time_us(s, B, Hq, Hkv, Skv, D, slots), 1, s))
         for cs in range(1, min(16, s) + 1):
             if s % cs:
@@ -167,11 +170,37 @@ def test_decode_time_not_below_hbm_roofline(loom, B, Hq, Hkv, Skv, D):
 
 
 def test_decode_more_splits_than_needed_cost_more(loom):
-    # beyond the argmin, extra splits only add merge work and CTA start-up
+    # beyond the argmin, extra splits only add merge work and item boundaries
     B, Hq, Hkv, Skv, D = 16, 32, 8, 8192, 128
     s = loom.loom_attn_decode_num_splits(B, Hq, Hkv, Skv, D)
-    t = lambda n: loom.loom_model_decode_time_us(n, B, Hq, Hkv, Skv, D, NUM_SMS)
+    t = lambda n: loom.loom_model_decode_tc_time_us(n, B, Hq, Hkv, Skv, D, NUM_SMS)
     assert t(min(128, 8 * s)) > t(s)
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,Skv,D", DECODE_SHAPES)
+def test_tc_decode_pays_the_start_up_once(loom, B, Hq, Hkv, Skv, D):
+    # the persistent tensor-core split kernel starts once and streams its items back to
+    # back, where the one-CTA-per-split kernel pays the start-up in every round of CTAs:
+    # with more than one round it is faster; in one round they differ by an item boundary
+    for s in range(1, min(64, math.ceil(Skv / 64)) + 1):
+        t_tc = loom.loom_model_decode_tc_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS)
+        t_cc = loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS)
+        if B * Hkv * s > 2 * NUM_SMS:
+            assert 0 < t_tc < t_cc, (s, t_tc, t_cc)
+        else:
+            assert abs(t_tc - t_cc) < 1.0, (s, t_tc, t_cc)
+        assert t_tc * 1e-6 >= 2.0 * B * Hkv * Skv * D * 2 / (PEAK_GBS * 1e9) * 0.999
+
+
+def test_tc_decode_rounds_and_limits(loom):
+    t = lambda s, Hq=32, Hkv=8: loom.loom_model_decode_tc_time_us(s, 1, Hq, Hkv, 131072, 128, NUM_SMS)
+    assert t(8, Hq=512, Hkv=8) < 0          # 64 query heads per kv head: not this kernel
+    assert t(0) < 0
+    # 38 splits x 8 kv heads = 304 items: one round on two CTAs per SM; one more split
+    # leaves 8 items to a second round, streamed by 8 CTAs at the rate one CTA sustains
+    assert 8 * 38 == 2 * NUM_SMS
+    assert t(39) > t(38) * 1.3
+    assert loom.loom_attn_decode_num_splits(1, 32, 8, 131072, 128) == 38
 
 
 @pytest.mark.parametrize("D", [64, 128])
