@@ -367,16 +367,19 @@ void loom_debug_gemm_stages(int stages);
 void loom_debug_gemm_order(int group_rows, int k_alternate);
 
 /*
- * loom_debug_decode_tensor_cores: which split kernel the split + merge form runs on a
- * contiguous cache (D 64 or 128, at most 32 query heads per kv head; the paged cache and
- * the other forms always use the CUDA-core stage).
- *   1 (the default): tensor cores, persistent.  Two CTAs per SM take (sequence, kv head,
- *     split) items, longest sequence first, from a counter in the workspace's last 256
- *     bytes until none is left, and stream the next item's q and K/V without a break; per
+ * loom_debug_decode_tensor_cores: which split kernel the split + merge form runs (D 64
+ * or 128, at most 32 query heads per kv head; the other forms always use the CUDA-core
+ * stage).
+ *   1 (the default): tensor cores, persistent, contiguous cache or paged cache with
+ *     pages of at least 32 keys (smaller pages take the CUDA-core kernel).  Two CTAs per
+ *     SM take (sequence, kv head, split) items, longest sequence first, from a counter in
+ *     the workspace's last 256 bytes until none is left, and stream the next item's q and
+ *     K/V without a break (a paged cache: each 64-key stage copied page by page); per
  *     64-key stage S = Q K^T and O += P V are tcgen05 MMAs with the query heads as rows
  *     of a TMEM tile and the softmax on one warp.  The merge kernel re-arms the counter;
  *     a workspace whose counter was never armed (its first call) is dealt statically.
- *   2: the same stage on the tensor cores, one CTA per (split, kv head, sequence).
+ *   2: the same stage on the tensor cores, one CTA per (split, kv head, sequence), for a
+ *     contiguous cache (a paged cache takes the CUDA-core kernel).
  *   0: the CUDA-core split kernel.
  * Other values select 1.  On the tensor cores P is rounded to bf16 before P V, as in
  * the prefill; the CUDA-core stage keeps it in fp32.

@@ -1022,12 +1022,19 @@ __device__ __forceinline__ void decode_tc_persist_rows(const uint8_t* smem, floa
   }
 }
 
-template <int D>
+// PAGED: K/V from a paged cache.  A 64-key stage is then copied in pieces of min(page
+// size, 64) keys, one per page it touches (each page looked up in the block table), into
+// the same 128-byte-swizzled tile: a piece of r rows starts r x 128 bytes into its box,
+// a multiple of 1024 (page sizes 8, 16, 32 or multiples of 64), so the swizzle pattern is
+// the one a single 64-row box leaves.  Pieces past the split's end are not copied (their
+// keys are masked and their V rows zeroed).
+template <int D, bool PAGED>
 __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
     decode_tc_persist_kernel(const int32_t* __restrict__ seqlens, float* __restrict__ o_part,
                              float* __restrict__ lse_part, unsigned long long* __restrict__ sched, int B, int Hq,
                              int Hkv, int Skv, int splits, float c, KernelCtl ctl, const __grid_constant__ CUtensorMap tm_q,
-                             const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v) {
+                             const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                             PagedView pv) {
   using C = DecodeTcCfg<D>;
   using L = DecodeTcPersistCfg<D>;
   extern __shared__ uint8_t smem_raw[];
@@ -1143,6 +1150,7 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
               continue;
             }
             const int tok0 = t_begin + j * C::T;
+            const int ntok = min(C::T, t_end - tok0);
             volatile int* rec = reinterpret_cast<volatile int*>(smem + L::META_OFF + s * 32);
             rec[0] = b;
             rec[1] = hk;
@@ -1150,13 +1158,44 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
             rec[3] = j;
             rec[4] = n_st;
             rec[5] = tok0;
-            rec[6] = min(C::T, t_end - tok0);
+            rec[6] = ntok;
             const uint32_t dst = sbase + s * C::STAGE_BYTES;
-            mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
+            if constexpr (PAGED) {
+              const int P = pv.page_size;
+              const int rows = P < C::T ? P : C::T;
+              const int npiece = (ntok + rows - 1) / rows;
+              const int32_t* tbl = pv.block_table + static_cast<size_t>(b) * pv.max_pages;
+              int page[C::T / 8];
 #pragma unroll
-            for (int x = 0; x < C::NBOX; ++x) {
-              tma_load_3d(dst + x * C::BOX_BYTES, &tm_k, x * 64, tok0, kv_z, bar_full + 8 * s);
-              tma_load_3d(dst + C::TILE_BYTES + x * C::BOX_BYTES, &tm_v, x * 64, tok0, kv_z, bar_full + 8 * s);
+              for (int i = 0; i < C::T / 8; ++i)
+                page[i] = i < npiece ? tbl[(tok0 + i * rows) / P] : 0;
+              mbar_expect_tx(bar_full + 8 * s, 2u * C::NBOX * npiece * rows * 128);
+#pragma unroll
+              for (int i = 0; i < C::T / 8; ++i) {
+                if (i >= npiece) break;
+                // An out-of-range page (a caller error) is sent past the end of the cache,
+                // where the copy engine reads zeros.  HND view [pages x Hkv, page_size, D]:
+                // (dim, row in page, page x Hkv + hk); NHD view [keys of all pages, Hkv, D]:
+                // (dim, hk, key).
+                const int t = tok0 + i * rows;
+                const bool bad = page[i] < 0 || page[i] >= pv.num_pages;
+                const int y = pv.hnd ? t % P : hk;
+                const int z = pv.hnd ? (bad ? pv.num_pages * Hkv : page[i] * Hkv + hk)
+                                     : (bad ? pv.num_pages * P : page[i] * P + t % P);
+#pragma unroll
+                for (int x = 0; x < C::NBOX; ++x) {
+                  const uint32_t off = x * C::BOX_BYTES + i * rows * 128;
+                  tma_load_3d(dst + off, &tm_k, x * 64, y, z, bar_full + 8 * s);
+                  tma_load_3d(dst + C::TILE_BYTES + off, &tm_v, x * 64, y, z, bar_full + 8 * s);
+                }
+              }
+            } else {
+              mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
+#pragma unroll
+              for (int x = 0; x < C::NBOX; ++x) {
+                tma_load_3d(dst + x * C::BOX_BYTES, &tm_k, x * 64, tok0, kv_z, bar_full + 8 * s);
+                tma_load_3d(dst + C::TILE_BYTES + x * C::BOX_BYTES, &tm_v, x * 64, tok0, kv_z, bar_full + 8 * s);
+              }
             }
           }
         }
@@ -1565,6 +1604,17 @@ __global__ void __launch_bounds__(D) decode_merge_kernel(const float* __restrict
     *sched = static_cast<unsigned long long>(kDecodeSchedTag) << 32;
   const int bh = blockIdx.x, d = threadIdx.x, lane = d & 31, wid = d >> 5;
   const float* lp = lse_part + static_cast<size_t>(bh) * splits;
+  const float* op = o_part + static_cast<size_t>(bh) * splits * D + d;
+  // Up to kMergeRegSplits splits, every partial of this thread's dimension is requested
+  // before the weights are known, so the merge waits for one round trip to memory
+  // instead of one per reduction step and per batch of partials.
+  constexpr int kMergeRegSplits = 64;
+  const bool in_regs = splits <= kMergeRegSplits;
+  float pre[kMergeRegSplits];
+  if (in_regs) {
+#pragma unroll
+    for (int i = 0; i < kMergeRegSplits; ++i) pre[i] = i < splits ? op[static_cast<size_t>(i) * D] : 0.f;
+  }
 
   float m = -INFINITY;
   for (int i = d; i < splits; i += D) m = fmaxf(m, lp[i]);
@@ -1591,14 +1641,26 @@ __global__ void __launch_bounds__(D) decode_merge_kernel(const float* __restrict
 #pragma unroll
   for (int w = 0; w < NW; ++w) W += red[w];
 
-  const float* op = o_part + static_cast<size_t>(bh) * splits * D + d;
+  // the same order of additions either way: eight running sums over whole groups of
+  // eight splits, the remainder into the first
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-  int i = 0;
-  for (; i + 8 <= splits; i += 8) {
+  if (in_regs) {
+    const int full = splits & ~7;
 #pragma unroll
-    for (int u = 0; u < 8; ++u) acc[u] = fmaf(w_s[i + u], op[static_cast<size_t>(i + u) * D], acc[u]);
+    for (int i = 0; i < kMergeRegSplits; ++i) {
+      if (i < full)
+        acc[i & 7] = fmaf(w_s[i], pre[i], acc[i & 7]);
+      else if (i < splits)
+        acc[0] = fmaf(w_s[i], pre[i], acc[0]);
+    }
+  } else {
+    int i = 0;
+    for (; i + 8 <= splits; i += 8) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u) acc[u] = fmaf(w_s[i + u], op[static_cast<size_t>(i + u) * D], acc[u]);
+    }
+    for (; i < splits; ++i) acc[0] = fmaf(w_s[i], op[static_cast<size_t>(i) * D], acc[0]);
   }
-  for (; i < splits; ++i) acc[0] = fmaf(w_s[i], op[static_cast<size_t>(i) * D], acc[0]);
   const float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
   const bool any = W > 0.f;
   o[static_cast<size_t>(bh) * D + d] = __float2bfloat16_rn(any ? sum / W : 0.f);
@@ -1823,27 +1885,51 @@ bool q_map_sw128(CUtensorMap* map, const void* q, int rows, int D, int G) {
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// A paged cache as the paged loader's 3-D view (paged_map) in 64-dim boxes of `rows`
+// keys, 128-byte swizzled: the persistent tensor-core split kernel's K/V pieces.
+bool paged_map_sw128(CUtensorMap* map, const void* cache, const PagedKV& pk, int Hkv, int D, int rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  const bool hnd = pk.layout == kPagedHND;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(hnd ? pk.page_size : Hkv),
+                        static_cast<cuuint64_t>(pk.num_pages) * (hnd ? Hkv : pk.page_size)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(hnd ? pk.page_size : Hkv) * D * 2};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(hnd ? rows : 1), static_cast<cuuint32_t>(hnd ? 1 : rows)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(cache), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // The persistent tensor-core split kernel: two CTAs per SM (or one per item when fewer).
-template <int D>
-cudaError_t launch_tc_persist(const DecodeArgs& a, const KernelCtl& ctl, cudaStream_t stream) {
+template <int D, bool PAGED>
+cudaError_t launch_tc_persist(const DecodeArgs& a, const PagedKV* pk, const KernelCtl& ctl, cudaStream_t stream) {
   using L = DecodeTcPersistCfg<D>;
   if (a.sched == nullptr) return cudaErrorInvalidValue;
   static PerDeviceOnce once;
-  if (!prepare_kernel(decode_tc_persist_kernel<D>, L::BYTES, false, once)) return cudaErrorInvalidValue;
+  if (!prepare_kernel(decode_tc_persist_kernel<D, PAGED>, L::BYTES, false, once)) return cudaErrorInvalidValue;
   const int G = a.Hq / a.Hkv;
   CUtensorMap tq, tk, tv;
-  if (!q_map_sw128(&tq, a.q, a.B * a.Hq, D, G) || !kv_map_sw128(&tk, a.k, a.B, a.Hkv, a.Skv, D) ||
-      !kv_map_sw128(&tv, a.v, a.B, a.Hkv, a.Skv, D))
-    return cudaErrorInvalidValue;
+  PagedView view{nullptr, 0, 0, 0, 0};
+  if (!q_map_sw128(&tq, a.q, a.B * a.Hq, D, G)) return cudaErrorInvalidValue;
+  if constexpr (PAGED) {
+    const int rows = pk->page_size < DecodeTcCfg<D>::T ? pk->page_size : DecodeTcCfg<D>::T;
+    if (!paged_map_sw128(&tk, a.k, *pk, a.Hkv, D, rows) || !paged_map_sw128(&tv, a.v, *pk, a.Hkv, D, rows))
+      return cudaErrorInvalidValue;
+    view = PagedView{pk->block_table, pk->page_size, pk->max_pages, pk->num_pages, pk->layout == kPagedHND ? 1 : 0};
+  } else {
+    if (!kv_map_sw128(&tk, a.k, a.B, a.Hkv, a.Skv, D) || !kv_map_sw128(&tv, a.v, a.B, a.Hkv, a.Skv, D))
+      return cudaErrorInvalidValue;
+  }
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
                                                 cudaSuccess)
     return cudaErrorInvalidValue;
   const long long items = static_cast<long long>(a.B) * a.Hkv * a.splits;
   const long long ctas = items < 2LL * sms ? items : 2LL * sms;
-  decode_tc_persist_kernel<D><<<static_cast<unsigned>(ctas), DecodeTcCfg<D>::THREADS, L::BYTES, stream>>>(
+  decode_tc_persist_kernel<D, PAGED><<<static_cast<unsigned>(ctas), DecodeTcCfg<D>::THREADS, L::BYTES, stream>>>(
       a.seqlens, a.o_part, a.lse_part, a.sched, a.B, a.Hq, a.Hkv, a.Skv, a.splits, a.scale * kLog2e, ctl, tq, tk,
-      tv);
+      tv, view);
   return cudaGetLastError();
 }
 
@@ -1932,6 +2018,8 @@ int decode_form(const DecodeArgs& a, int* cs_out) {
     *cs_out = ch.cs;
     return kDecodeCluster;
   }
+  // (a paged call is priced with the CUDA-core kernel whatever its page size, so that the
+  // form does not depend on the page size, which the form query does not know)
   const double t_split = (!PAGED && decode_tc_eligible(a))
                              ? model::decode_tc_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms)
                              : model::decode_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms);
@@ -1986,8 +2074,8 @@ cudaError_t launch_form(const DecodeArgs& a, const PagedKV* pk, const KernelCtl&
   cudaError_t e;
   if (form == kDecodePersistent)
     e = launch_persist<D, GT, PAGED>(a, pk, ctl, stream);
-  else if (!PAGED && decode_tc_eligible(a))
-    e = a.tc == 2 ? launch_tc_split<D>(a, ctl, stream) : launch_tc_persist<D>(a, ctl, stream);
+  else if (decode_tc_eligible(a) && (!PAGED || (a.tc == 1 && pk->page_size >= kDecodeTcMinPage)))
+    e = a.tc == 2 ? launch_tc_split<D>(a, ctl, stream) : launch_tc_persist<D, PAGED>(a, pk, ctl, stream);
   else
     e = launch_split<D, GT, PAGED>(a, pk, ctl, stream);
   if (e != cudaSuccess) return e;

@@ -284,7 +284,8 @@ loom_status loom_attn_decode_paged(const void* q, const void* k_cache, const voi
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              (rows * D * sizeof(float) + 255) / 256 * 256);
   DecodeArgs a{q, k_cache, v_cache, seqlens_k, o, lse, o_part, lse_part, B, Hq, Hkv, Skv, D, num_splits, scale,
-               g_decode_form, g_decode_cluster, 0, by_model, 0, decode_sched_word(workspace, B, Hq, D, num_splits)};
+               g_decode_form, g_decode_cluster, 0, by_model, g_decode_tc,
+               decode_sched_word(workspace, B, Hq, D, num_splits)};
   PagedKV pk{block_table, num_pages, page_size, max_pages, kv_layout};
   return launch_decode_paged(a, pk, ctl, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LOOM_OK
                                                                                           : LOOM_ERR_CUDA;

@@ -168,3 +168,37 @@ def test_no_false_timeouts_under_default_limit(loom):
     for causal in (False, True):
         loom.loom_attn_fwd(q, q, q, causal=causal)
     loom.loom_attn_check_error()
+
+
+@pytest.mark.parametrize("tensor_cores", [1, 0], ids=["tc_persistent", "cuda_core"])
+def test_paged_decode_skipped_stage_times_out_and_context_survives(loom, tensor_cores):
+    """The split kernel over a paged cache (64-key pages, in a shuffled order): a stage
+    whose copies are never issued times out, the kernel unwinds, and the next call on the
+    same context matches the oracle."""
+    import torch
+    B, Hq, Hkv, P, D = 2, 8, 2, 64, 128
+    lens = np.array([1000, 333], np.int32)
+    npg = [(int(n) + P - 1) // P for n in lens]
+    max_pages = max(npg)
+    kc = synth.bf16_normal(41, synth.STREAM_K, (sum(npg), P, Hkv, D))
+    vc = synth.bf16_normal(41, synth.STREAM_V, (sum(npg), P, Hkv, D))
+    q = synth.bf16_normal(41, synth.STREAM_Q, (B, Hq, 1, D))
+    order = np.random.default_rng(41).permutation(sum(npg)).astype(np.int32)
+    table = np.full((B, max_pages), -1, np.int32)
+    table[0, :npg[0]] = order[:npg[0]]
+    table[1, :npg[1]] = order[npg[0]:]
+    qd, kd, vd = to_dev(q), to_dev(kc), to_dev(vc)
+    td, sl = torch.from_numpy(table).cuda(), torch.from_numpy(lens).cuda()
+    loom.loom_debug_decode_tensor_cores(tensor_cores)
+    try:
+        def bad():
+            loom.loom_debug_inject(1)
+            loom.loom_attn_decode_paged(qd, kd, vd, td, sl, num_splits=2)
+
+        _expect_timeout(loom, bad)
+        o, lse = loom.loom_attn_decode_paged(qd, kd, vd, td, sl, num_splits=2, return_lse=True)
+        loom.loom_attn_check_error()
+    finally:
+        loom.loom_debug_decode_tensor_cores(1)
+    o_ref, lse_ref = oracle.decode_paged(q, kc, vc, table, lens, page_size=P)
+    assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, "paged decode after timeout")

@@ -1,5 +1,5 @@
 """GPU parity of Flash Decode over a paged KV cache (through the C ABI) against the fp64
-oracle (``oracle.decode_paged``), plus bit equality with the contiguous kernel when the
+oracle (``oracle.decode_paged``), plus bit equality with the contiguous kernels when the
 pages are laid out in order (the two load the same rows into the same places)."""
 import numpy as np
 import pytest
@@ -26,13 +26,19 @@ def loom():
     m.loom_debug_set_timeout_ns(0)
 
 
-@pytest.fixture(autouse=True, params=[1, 2, 3], ids=["split_merge", "persistent", "cluster"])
+@pytest.fixture(autouse=True, params=[(1, 1), (1, 0), (2, 1), (3, 1)],
+                ids=["split_merge", "split_merge_cuda_core", "persistent", "cluster"])
 def form(request, loom):
-    """Every test runs with each Flash Decode form forced: split kernel + merge, persistent
-    split kernel + merge, and the single-kernel cluster form (the model's cluster size)."""
-    loom.loom_debug_decode_form(request.param)
-    yield request.param
+    """Every test runs with each Flash Decode form forced: split kernel + merge (the split
+    kernel on the tensor cores -- persistent CTAs copying each stage page by page -- and
+    on the CUDA cores), persistent split kernel + merge, and the single-kernel cluster
+    form (the model's cluster size)."""
+    f, tc = request.param
+    loom.loom_debug_decode_form(f)
+    loom.loom_debug_decode_tensor_cores(tc)
+    yield f
     loom.loom_debug_decode_form(0)
+    loom.loom_debug_decode_tensor_cores(1)
 
 
 def paged_case(seed, B, Hq, Hkv, P, lens, D, spare=5, poison=True, shuffle=True):
@@ -117,8 +123,8 @@ def test_edge_lengths_and_empty(loom, layout):
 @pytest.mark.parametrize("P", [16, 64])
 def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P, layout):
     """With page j of sequence b at physical index b * pages + j, the paged and the
-    contiguous CUDA-core kernels copy identical rows to identical places: outputs are equal
-    bit for bit (the contiguous tensor-core split kernel rounds P to bf16, so it is off here)."""
+    contiguous kernels of each form (and of either split kernel) copy identical rows to
+    identical places: outputs are equal bit for bit."""
     import torch
     B, Hq, Hkv, S, D = 3, 16, 4, 1024, 128
     k = synth.bf16_normal(8, synth.STREAM_K, (B, Hkv, S, D))
@@ -131,13 +137,9 @@ def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P, layout):
     lens = np.array([S, 777, 64], dtype=np.int32)
     for splits in (1, 5):
         o1, l1 = run_paged(loom, q, kc, vc, table, lens, splits, layout)
-        loom.loom_debug_decode_tensor_cores(0)
-        try:
-            o2, l2 = loom.loom_attn_decode(to_dev(q), to_dev(k), to_dev(v), torch.from_numpy(lens).cuda(),
-                                           num_splits=splits, return_lse=True)
-            loom.loom_attn_check_error()
-        finally:
-            loom.loom_debug_decode_tensor_cores(1)
+        o2, l2 = loom.loom_attn_decode(to_dev(q), to_dev(k), to_dev(v), torch.from_numpy(lens).cuda(),
+                                       num_splits=splits, return_lse=True)
+        loom.loom_attn_check_error()
         assert torch.equal(o1.view(torch.int16), o2.view(torch.int16))
         assert torch.equal(l1, l2)
 
