@@ -1048,23 +1048,6 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
   const long long per_seq = static_cast<long long>(Hkv) * splits;
   const long long n_items = B * per_seq;
 
-  // the sequences in order of decreasing length (ties by index): items are taken in it
-  int* order = reinterpret_cast<int*>(smem + L::ORDER_OFF);
-  const bool sorted = seqlens != nullptr && B <= L::kMaxSortedB;
-  if (sorted) {
-    int* lens = reinterpret_cast<int*>(smem + L::LENS_OFF);
-    for (int bb = threadIdx.x; bb < B; bb += blockDim.x) lens[bb] = seqlens[bb];
-    __syncthreads();
-    for (int bb = threadIdx.x; bb < B; bb += blockDim.x) {
-      const int lb = lens[bb];
-      int r = 0;
-      for (int x = 0; x < B; ++x) {
-        const int lx = lens[x];
-        r += (lx > lb) || (lx == lb && x < bb);
-      }
-      order[r] = bb;
-    }
-  }
   const uint32_t bar_full = sbase + L::BAR_OFF;
   const uint32_t bar_empty = bar_full + 8 * C::NSTAGE;
   const uint32_t bar_qf = bar_empty + 8 * C::NSTAGE;  // an item's q rows are in the boxes
@@ -1097,6 +1080,29 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_ptr;
+  // Launched as a dependent of the previous kernel in the stream (the previous call's
+  // merge lets it start early): everything above touches no global memory; from here on
+  // the previous kernel's writes must be complete and visible.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+
+  // the sequences in order of decreasing length (ties by index): items are taken in it
+  int* order = reinterpret_cast<int*>(smem + L::ORDER_OFF);
+  const bool sorted = seqlens != nullptr && B <= L::kMaxSortedB;
+  if (sorted) {
+    int* lens = reinterpret_cast<int*>(smem + L::LENS_OFF);
+    for (int bb = threadIdx.x; bb < B; bb += blockDim.x) lens[bb] = seqlens[bb];
+    __syncthreads();
+    for (int bb = threadIdx.x; bb < B; bb += blockDim.x) {
+      const int lb = lens[bb];
+      int r = 0;
+      for (int x = 0; x < B; ++x) {
+        const int lx = lens[x];
+        r += (lx > lb) || (lx == lb && x < bb);
+      }
+      order[r] = bb;
+    }
+    __syncthreads();
+  }
 
   if (warp == 1) {
     // ------------------------------------------------------------ loader (lane 0)
@@ -1597,6 +1603,9 @@ __global__ void __launch_bounds__(D) decode_merge_kernel(const float* __restrict
   constexpr int NW = D / 32;
   __shared__ float w_s[kMaxDecodeSplits];
   __shared__ float red[NW];
+  // Let the next kernel in the stream (the next call's split kernel) launch early; it
+  // waits for this grid before it touches global memory.
+  asm volatile("griddepcontrol.launch_dependents;");
   // Wait until the split kernel's partials are complete and visible.
   asm volatile("griddepcontrol.wait;" ::: "memory");
   // The split kernel has taken its last item: arm the workspace's item counter for the next call.
@@ -1927,10 +1936,20 @@ cudaError_t launch_tc_persist(const DecodeArgs& a, const PagedKV* pk, const Kern
     return cudaErrorInvalidValue;
   const long long items = static_cast<long long>(a.B) * a.Hkv * a.splits;
   const long long ctas = items < 2LL * sms ? items : 2LL * sms;
-  decode_tc_persist_kernel<D, PAGED><<<static_cast<unsigned>(ctas), DecodeTcCfg<D>::THREADS, L::BYTES, stream>>>(
-      a.seqlens, a.o_part, a.lse_part, a.sched, a.B, a.Hq, a.Hkv, a.Skv, a.splits, a.scale * kLog2e, ctl, tq, tk,
-      tv, view);
-  return cudaGetLastError();
+  // programmatic dependent launch: the CTAs set up their barriers and TMEM while the
+  // previous kernel in the stream finishes (the kernel waits for it before any global access)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(ctas));
+  cfg.blockDim = dim3(DecodeTcCfg<D>::THREADS);
+  cfg.dynamicSmemBytes = L::BYTES;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decode_tc_persist_kernel<D, PAGED>, a.seqlens, a.o_part, a.lse_part, a.sched, a.B,
+                            a.Hq, a.Hkv, a.Skv, a.splits, a.scale * kLog2e, ctl, tq, tk, tv, view);
 }
 
 template <int D, int GT, bool PAGED, bool CLUSTER>
