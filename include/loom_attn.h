@@ -370,8 +370,7 @@ void loom_debug_gemm_order(int group_rows, int k_alternate);
  * loom_debug_decode_tensor_cores: which split kernel the split + merge form runs (D 64
  * or 128, at most 32 query heads per kv head; the other forms always use the CUDA-core
  * stage).
- *   1 (the default): tensor cores, persistent, contiguous cache or paged cache with
- *     pages of at least 32 keys (smaller pages take the CUDA-core kernel).  Two CTAs per
+ *   1 (the default): tensor cores, persistent, contiguous or paged cache.  Two CTAs per
  *     SM take (sequence, kv head, split) items, longest sequence first, from a counter in
  *     the workspace's last 256 bytes until none is left, and stream the next item's q and
  *     K/V without a break (a paged cache: each 64-key stage copied page by page); per

@@ -1023,11 +1023,12 @@ __device__ __forceinline__ void decode_tc_persist_rows(const uint8_t* smem, floa
 }
 
 // PAGED: K/V from a paged cache.  A 64-key stage is then copied in pieces of min(page
-// size, 64) keys, one per page it touches (each page looked up in the block table), into
-// the same 128-byte-swizzled tile: a piece of r rows starts r x 128 bytes into its box,
-// a multiple of 1024 (page sizes 8, 16, 32 or multiples of 64), so the swizzle pattern is
-// the one a single 64-row box leaves.  Pieces past the split's end are not copied (their
-// keys are masked and their V rows zeroed).
+// size, 64) keys, one per page it touches (each page looked up in the block table, each
+// piece looked up and copied by its own loader lane), into the same 128-byte-swizzled
+// tile: a piece of r rows starts r x 128 bytes into its box, a multiple of 1024 (page
+// sizes 8, 16, 32 or multiples of 64), so the swizzle pattern is the one a single 64-row
+// box leaves.  Pieces past the split's end are not copied (their keys are masked and
+// their V rows zeroed).
 template <int D, bool PAGED>
 __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
     decode_tc_persist_kernel(const int32_t* __restrict__ seqlens, float* __restrict__ o_part,
@@ -1105,58 +1106,67 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
   }
 
   if (warp == 1) {
-    // ------------------------------------------------------------ loader (lane 0)
+    // ------------------------------------------------------------ loader (whole warp)
+    // Lane 0 takes the tickets, waits on the ring and writes the records; a paged stage's
+    // pieces are looked up and copied by one lane each, so that the copies of a stage go
+    // out together.
     if (lane == 0) {
       prefetch_tensormap(&tm_q);
       prefetch_tensormap(&tm_k);
       prefetch_tensormap(&tm_v);
-      // Item blockIdx.x first.  An armed counter deals the items past the first gridDim.x
-      // on demand, one ticket fetched an item ahead so that its latency is hidden; a
-      // workspace never armed (its first call) deals them statically, item blockIdx.x +
-      // k * gridDim.x (every CTA reads the same unarmed tag: all take the same branch).
-      unsigned long long ticket = atomicAdd(sched, 1ull);
-      int dynamic = -1;  // read from the first ticket once the first item is under way
-      long long item = blockIdx.x;
-      int st = 0, nq = 0, skipped = -1;
-      bool ok = true;
-      for (long long kk = 1; ok && item < n_items; ++kk) {
-        const int rb = static_cast<int>(item / per_seq);
-        const int rem = static_cast<int>(item - rb * per_seq);
-        const int b = sorted ? order[rb] : rb;
-        const int split = rem / Hkv, hk = rem - split * Hkv;
-        int len = seqlens ? seqlens[b] : Skv;
-        len = max(0, min(len, Skv));
-        int chunk = (len + splits - 1) / splits;
-        chunk = (chunk + kDecodeChunkAlign - 1) / kDecodeChunkAlign * kDecodeChunkAlign;
-        const int t_begin = min(split * chunk, len);
-        const int t_end = min(t_begin + chunk, len);
-        if (t_begin >= t_end) {
-          // empty split: contributes nothing to the merge
-          const size_t row0 = (static_cast<size_t>(b) * Hq + static_cast<size_t>(hk) * G) * splits + split;
-          for (int r = 0; r < G; ++r) {
-            float4* dst = reinterpret_cast<float4*>(o_part + (row0 + static_cast<size_t>(r) * splits) * D);
-            for (int i = 0; i < D / 4; ++i) dst[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-            lse_part[row0 + static_cast<size_t>(r) * splits] = -INFINITY;
-          }
-        } else {
-          // the item's q rows, once the softmax warp has moved the previous ones to TMEM
-          if (!(ok = mbar_wait(bar_qe, (nq & 1) ^ 1, ctl, ab))) break;
+    }
+    // Item blockIdx.x first.  An armed counter deals the items past the first gridDim.x
+    // on demand, one ticket fetched an item ahead so that its latency is hidden; a
+    // workspace never armed (its first call) deals them statically, item blockIdx.x +
+    // k * gridDim.x (every CTA reads the same unarmed tag: all take the same branch).
+    unsigned long long ticket = lane == 0 ? atomicAdd(sched, 1ull) : 0ull;
+    int dynamic = -1;  // read from the first ticket once the first item is under way
+    long long item = blockIdx.x;
+    int st = 0, nq = 0, skipped = -1;
+    bool ok = true;
+    for (long long kk = 1; ok && item < n_items; ++kk) {
+      const int rb = static_cast<int>(item / per_seq);
+      const int rem = static_cast<int>(item - rb * per_seq);
+      const int b = sorted ? order[rb] : rb;
+      const int split = rem / Hkv, hk = rem - split * Hkv;
+      int len = seqlens ? seqlens[b] : Skv;
+      len = max(0, min(len, Skv));
+      int chunk = (len + splits - 1) / splits;
+      chunk = (chunk + kDecodeChunkAlign - 1) / kDecodeChunkAlign * kDecodeChunkAlign;
+      const int t_begin = min(split * chunk, len);
+      const int t_end = min(t_begin + chunk, len);
+      if (t_begin >= t_end) {
+        // empty split: contributes nothing to the merge
+        const size_t row0 = (static_cast<size_t>(b) * Hq + static_cast<size_t>(hk) * G) * splits + split;
+        for (int i = lane; i < G * (D / 4); i += 32) {
+          const int r = i / (D / 4);
+          reinterpret_cast<float4*>(o_part + (row0 + static_cast<size_t>(r) * splits) * D)[i % (D / 4)] =
+              make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        for (int r = lane; r < G; r += 32) lse_part[row0 + static_cast<size_t>(r) * splits] = -INFINITY;
+      } else {
+        // the item's q rows, once the softmax warp has moved the previous ones to TMEM
+        if (!(ok = mbar_wait_warp(bar_qe, (nq & 1) ^ 1, ctl, ab))) break;
+        if (lane == 0) {
           mbar_expect_tx(bar_qf, static_cast<uint32_t>(C::NBOX * G * 128));
 #pragma unroll
           for (int x = 0; x < C::NBOX; ++x)
             tma_load_3d(sbase + L::Q_OFF + x * L::Q_BOX_BYTES, &tm_q, x * 64, b * Hq + hk * G, 0, bar_qf);
-          ++nq;
-          const int n_st = (t_end - t_begin + C::T - 1) / C::T;
-          const int kv_z = b * Hkv + hk;
-          for (int j = 0; j < n_st; ++j, ++st) {
-            const int s = st % C::NSTAGE;
-            if (!(ok = mbar_wait(bar_empty + 8 * s, ((st / C::NSTAGE) & 1) ^ 1, ctl, ab))) break;
-            if (ctl.inject == 1 && st == 1) {  // test hook: never fill this stage
-              skipped = st;
-              continue;
-            }
-            const int tok0 = t_begin + j * C::T;
-            const int ntok = min(C::T, t_end - tok0);
+        }
+        ++nq;
+        const int n_st = (t_end - t_begin + C::T - 1) / C::T;
+        const int kv_z = b * Hkv + hk;
+        for (int j = 0; j < n_st; ++j, ++st) {
+          const int s = st % C::NSTAGE;
+          if (!(ok = mbar_wait_warp(bar_empty + 8 * s, ((st / C::NSTAGE) & 1) ^ 1, ctl, ab))) break;
+          if (ctl.inject == 1 && st == 1) {  // test hook: never fill this stage
+            skipped = st;
+            continue;
+          }
+          const int tok0 = t_begin + j * C::T;
+          const int ntok = min(C::T, t_end - tok0);
+          const uint32_t dst = sbase + s * C::STAGE_BYTES;
+          if (lane == 0) {
             volatile int* rec = reinterpret_cast<volatile int*>(smem + L::META_OFF + s * 32);
             rec[0] = b;
             rec[1] = hk;
@@ -1165,37 +1175,33 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
             rec[4] = n_st;
             rec[5] = tok0;
             rec[6] = ntok;
-            const uint32_t dst = sbase + s * C::STAGE_BYTES;
-            if constexpr (PAGED) {
-              const int P = pv.page_size;
-              const int rows = P < C::T ? P : C::T;
-              const int npiece = (ntok + rows - 1) / rows;
-              const int32_t* tbl = pv.block_table + static_cast<size_t>(b) * pv.max_pages;
-              int page[C::T / 8];
+          }
+          if constexpr (PAGED) {
+            const int P = pv.page_size;
+            const int rows = P < C::T ? P : C::T;
+            const int npiece = (ntok + rows - 1) / rows;  // at most 8 (pages of 8 keys or more)
+            if (lane == 0) mbar_expect_tx(bar_full + 8 * s, 2u * C::NBOX * npiece * rows * 128);
+            __syncwarp();
+            if (lane < npiece) {
+              // An out-of-range page (a caller error) is sent past the end of the cache,
+              // where the copy engine reads zeros.  HND view [pages x Hkv, page_size, D]:
+              // (dim, row in page, page x Hkv + hk); NHD view [keys of all pages, Hkv, D]:
+              // (dim, hk, key).
+              const int t = tok0 + lane * rows;
+              const int page = pv.block_table[static_cast<size_t>(b) * pv.max_pages + t / P];
+              const bool bad = page < 0 || page >= pv.num_pages;
+              const int y = pv.hnd ? t % P : hk;
+              const int z = pv.hnd ? (bad ? pv.num_pages * Hkv : page * Hkv + hk)
+                                   : (bad ? pv.num_pages * P : page * P + t % P);
 #pragma unroll
-              for (int i = 0; i < C::T / 8; ++i)
-                page[i] = i < npiece ? tbl[(tok0 + i * rows) / P] : 0;
-              mbar_expect_tx(bar_full + 8 * s, 2u * C::NBOX * npiece * rows * 128);
-#pragma unroll
-              for (int i = 0; i < C::T / 8; ++i) {
-                if (i >= npiece) break;
-                // An out-of-range page (a caller error) is sent past the end of the cache,
-                // where the copy engine reads zeros.  HND view [pages x Hkv, page_size, D]:
-                // (dim, row in page, page x Hkv + hk); NHD view [keys of all pages, Hkv, D]:
-                // (dim, hk, key).
-                const int t = tok0 + i * rows;
-                const bool bad = page[i] < 0 || page[i] >= pv.num_pages;
-                const int y = pv.hnd ? t % P : hk;
-                const int z = pv.hnd ? (bad ? pv.num_pages * Hkv : page[i] * Hkv + hk)
-                                     : (bad ? pv.num_pages * P : page[i] * P + t % P);
-#pragma unroll
-                for (int x = 0; x < C::NBOX; ++x) {
-                  const uint32_t off = x * C::BOX_BYTES + i * rows * 128;
-                  tma_load_3d(dst + off, &tm_k, x * 64, y, z, bar_full + 8 * s);
-                  tma_load_3d(dst + C::TILE_BYTES + off, &tm_v, x * 64, y, z, bar_full + 8 * s);
-                }
+              for (int x = 0; x < C::NBOX; ++x) {
+                const uint32_t off = x * C::BOX_BYTES + lane * rows * 128;
+                tma_load_3d(dst + off, &tm_k, x * 64, y, z, bar_full + 8 * s);
+                tma_load_3d(dst + C::TILE_BYTES + off, &tm_v, x * 64, y, z, bar_full + 8 * s);
               }
-            } else {
+            }
+          } else {
+            if (lane == 0) {
               mbar_expect_tx(bar_full + 8 * s, C::STAGE_BYTES);
 #pragma unroll
               for (int x = 0; x < C::NBOX; ++x) {
@@ -1204,8 +1210,11 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
               }
             }
           }
+          __syncwarp();
         }
-        if (!ok) break;
+      }
+      if (!ok) break;
+      if (lane == 0) {
         if (dynamic < 0) dynamic = static_cast<uint32_t>(ticket >> 32) == kDecodeSchedTag ? 1 : 0;
         if (dynamic) {
           item = static_cast<long long>(gridDim.x) + static_cast<uint32_t>(ticket);
@@ -1214,18 +1223,23 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
           item = blockIdx.x + kk * static_cast<long long>(gridDim.x);
         }
       }
-      // the end record
-      bool ended = false;
-      if (ok) {
-        const int s = st % C::NSTAGE;
-        if (mbar_wait(bar_empty + 8 * s, ((st / C::NSTAGE) & 1) ^ 1, ctl, ab)) {
+      item = __shfl_sync(0xffffffffu, item, 0);
+    }
+    // the end record
+    bool ended = false;
+    if (ok) {
+      const int s = st % C::NSTAGE;
+      if (mbar_wait_warp(bar_empty + 8 * s, ((st / C::NSTAGE) & 1) ^ 1, ctl, ab)) {
+        if (lane == 0) {
           *reinterpret_cast<volatile int*>(smem + L::META_OFF + s * 32) = -1;
           mbar_arrive(bar_full + 8 * s);
-          ended = true;
         }
+        ended = true;
       }
-      // Drain: never leave the CTA with copies still landing in its shared memory (after
-      // the end record the stage it replaced has been consumed).
+    }
+    // Drain: never leave the CTA with copies still landing in its shared memory (after
+    // the end record the stage it replaced has been consumed).
+    if (lane == 0) {
       Abort no_abort{ab.flag + 1};
       for (int i = max(0, st - C::NSTAGE + (ended ? 1 : 0)); i < st; ++i)
         if (i != skipped) mbar_wait(bar_full + 8 * (i % C::NSTAGE), (i / C::NSTAGE) & 1, ctl, no_abort);
@@ -2093,7 +2107,7 @@ cudaError_t launch_form(const DecodeArgs& a, const PagedKV* pk, const KernelCtl&
   cudaError_t e;
   if (form == kDecodePersistent)
     e = launch_persist<D, GT, PAGED>(a, pk, ctl, stream);
-  else if (decode_tc_eligible(a) && (!PAGED || (a.tc == 1 && pk->page_size >= kDecodeTcMinPage)))
+  else if (decode_tc_eligible(a) && !(PAGED && a.tc == 2))
     e = a.tc == 2 ? launch_tc_split<D>(a, ctl, stream) : launch_tc_persist<D, PAGED>(a, pk, ctl, stream);
   else
     e = launch_split<D, GT, PAGED>(a, pk, ctl, stream);

@@ -61,11 +61,6 @@ struct DecodeArgs {
 constexpr uint32_t kDecodeSchedTag = 0x7FBADC0Du;
 // Query heads per kv head that the tensor-core split kernels take (the lanes of one warp).
 constexpr int kDecodeTcMaxGroup = 32;
-// Smallest page size of a paged cache that the tensor-core split kernel takes.  It copies
-// a stage page by page in 64-dim boxes (rows x 128 bytes each); below 32-key pages the
-// copies are too small to keep HBM busy (measured on the batched paged decode against the
-// CUDA-core kernel: 8-key pages 0.52x, 16 0.82x, 32 1.15x, 64 and more 1.21x).
-constexpr int kDecodeTcMinPage = 32;
 
 struct FwdArgs {
   const void* q;  // [B, Hq, Sq, D] bf16

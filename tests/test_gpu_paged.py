@@ -121,14 +121,11 @@ def test_edge_lengths_and_empty(loom, layout):
 
 @LAYOUTS
 @pytest.mark.parametrize("P", [16, 64])
-def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P, layout, request):
+def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P, layout):
     """With page j of sequence b at physical index b * pages + j, the paged and the
     contiguous kernels of each form (and of either split kernel) copy identical rows to
-    identical places: outputs are equal bit for bit.  Pages below 32 keys take the
-    CUDA-core split kernel, so the contiguous call takes it too."""
+    identical places: outputs are equal bit for bit."""
     import torch
-    _, tc = request.node.callspec.params["form"]
-    contiguous_tc = tc if P >= 32 else 0
     B, Hq, Hkv, S, D = 3, 16, 4, 1024, 128
     k = synth.bf16_normal(8, synth.STREAM_K, (B, Hkv, S, D))
     v = synth.bf16_normal(8, synth.STREAM_V, (B, Hkv, S, D))
@@ -140,13 +137,9 @@ def test_in_order_pages_match_contiguous_kernel_bitwise(loom, P, layout, request
     lens = np.array([S, 777, 64], dtype=np.int32)
     for splits in (1, 5):
         o1, l1 = run_paged(loom, q, kc, vc, table, lens, splits, layout)
-        loom.loom_debug_decode_tensor_cores(contiguous_tc)
-        try:
-            o2, l2 = loom.loom_attn_decode(to_dev(q), to_dev(k), to_dev(v), torch.from_numpy(lens).cuda(),
-                                           num_splits=splits, return_lse=True)
-            loom.loom_attn_check_error()
-        finally:
-            loom.loom_debug_decode_tensor_cores(tc)
+        o2, l2 = loom.loom_attn_decode(to_dev(q), to_dev(k), to_dev(v), torch.from_numpy(lens).cuda(),
+                                       num_splits=splits, return_lse=True)
+        loom.loom_attn_check_error()
         assert torch.equal(o1.view(torch.int16), o2.view(torch.int16))
         assert torch.equal(l1, l2)
 
