@@ -2051,9 +2051,7 @@ int decode_form(const DecodeArgs& a, int* cs_out) {
     *cs_out = ch.cs;
     return kDecodeCluster;
   }
-  // (a paged call is priced with the CUDA-core kernel whatever its page size, so that the
-  // form does not depend on the page size, which the form query does not know)
-  const double t_split = (!PAGED && decode_tc_eligible(a))
+  const double t_split = (decode_tc_eligible(a) && !(PAGED && a.tc == 2))
                              ? model::decode_tc_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms)
                              : model::decode_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms);
   const double t_persist =
