@@ -762,24 +762,30 @@ def run_decode_sweep(torch, loom, dev, stream, args, peaks):
             wl.splits = sp
             nbytes = loom.loom_attn_decode_workspace_bytes(wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sp)
             wl.ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
-            # split + merge, the persistent split kernel + merge, then the cluster form with
-            # every power-of-two cluster size dividing sp
-            for form, cs in [(1, 0), (2, 0)] + [(3, c) for c in (2, 4, 8, 16) if sp % c == 0]:
+            # split + merge (its split kernel on the tensor cores, then on the CUDA cores), the
+            # persistent CUDA-core split kernel + merge, then the cluster form with every
+            # power-of-two cluster size dividing sp
+            for form, cs, tc in [(1, 0, 1), (1, 0, 0), (2, 0, 1)] + [(3, c, 1) for c in (2, 4, 8, 16) if sp % c == 0]:
                 n_fit = loom.loom_decode_max_clusters(wl.D, G, cs) if cs else 0
                 if cs and n_fit < 1:
                     continue
                 loom.loom_debug_decode_form(form, cs)
+                loom.loom_debug_decode_tensor_cores(tc)
                 r = measure(torch, wl, max(10, args.steps // 4), args.warmup, stream, lambda: None, 1, float, peaks)
                 loom.loom_attn_check_error(stream)
+                loom.loom_debug_decode_tensor_cores(1)
                 if form == 3:
                     model_us = loom.loom_model_decode_cluster_time_us(sp, cs, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, n_fit)
                 elif form == 2:
                     model_us = loom.loom_model_decode_persistent_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, slots)
+                elif tc:
+                    model_us = loom.loom_model_decode_tc_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sms)
                 else:
                     model_us = loom.loom_model_decode_time_us(sp, wl.B, wl.Hq, wl.Hkv, wl.Skv, wl.D, sms)
-                name = {1: "split+merge", 2: "persistent+merge", 3: f"cluster{cs}"}[form]
+                name = {1: "split+merge" if tc else "split+merge (CUDA cores)", 2: "persistent+merge",
+                        3: f"cluster{cs}"}[form]
                 print(json.dumps({"sweep": "decode", "workload": wl.describe(), "splits": sp, "form": name,
-                                  "model_choice": sp == chosen and (form, cs if form == 3 else 0) == chosen_form,
+                                  "model_choice": sp == chosen and tc == 1 and (form, cs if form == 3 else 0) == chosen_form,
                                   "measured_us": round(r["ms_per_step"] * 1e3, 2),
                                   "model_us": round(model_us, 2), "GB/s": r["value"],
                                   "frac": r["roofline"]["frac"]}), flush=True)
