@@ -70,12 +70,23 @@ struct ArchDesc {
                                     // boundary (O read-out, next q into TMEM) that the full ring does
                                     // not hide (fitted: batched B16 H32/8 lengths U[4096, 8192], 16 vs
                                     // 32 splits, 70.9 vs 74.2 us, less the merge's extra partials)
+  double decode_tc_cta_gbs;         // persistent tensor-core decode: KV stream rate one CTA sustains
+                                    // when HBM is not the bound (fitted: B1 H32/8 Skv 131072 with
+                                    // 8 and 16 splits, 64 and 128 CTAs, 218.6 and 117.2 us)
+  double decode_tc_stage_ns;        // persistent tensor-core decode: one 64-key stage's S -> softmax
+                                    // -> P.V chain, the floor of a stage when its bytes arrive faster
+                                    // (fitted: D = 64, B1 H64/16 Skv 65536, 19 splits: 56.6 us for 54
+                                    // stages per CTA)
+  double decode_merge_ns;           // the merge launch's fixed cost in a decode step: the dependent
+                                    // launch, its wait for the split grid, one round trip to the
+                                    // partials (fitted: a timing probe without the merge launch,
+                                    // 3.2-4.8 us per step less the partials' traffic)
 };
 
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 3400.0, 3000.0, 28.4, 150.0, 7800.0, 300.0,
+    129.0e6, 1.07, 3400.0, 3000.0, 28.4, 150.0, 7800.0, 300.0, 39.0, 870.0, 3000.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -410,7 +421,7 @@ constexpr double decode_time_us(int splits, int B, int Hq, int Hkv, int Skv, int
                                 const ArchDesc& a = kGb300) {
   const double t_split = decode_split_loop_ns(splits, B, Hq, Hkv, Skv, D, num_sms, a);
   const double part_bytes = 1.0 * B * Hq * splits * (D + 1) * 4;
-  const double t_merge = a.launch_ns * 0.2 + 2.0 * part_bytes / a.hbm_gbs;
+  const double t_merge = a.decode_merge_ns + 2.0 * part_bytes / a.hbm_gbs;
   return heg_seq(t_split, t_merge) * 1e-3;
 }
 
@@ -453,15 +464,18 @@ constexpr double decode_persistent_time_us(int splits, int B, int Hq, int Hkv, i
   const double t_split = heg_seq(a.cta_start_ns, heg_for(static_cast<double>(per),
                                                          heg_seq(chunk_bytes / rate, a.decode_item_ns)));
   const double part_bytes = 1.0 * B * Hq * splits * (D + 1) * 4;
-  const double t_merge = a.launch_ns * 0.2 + 2.0 * part_bytes / a.hbm_gbs;
+  const double t_merge = a.decode_merge_ns + 2.0 * part_bytes / a.hbm_gbs;
   return heg_seq(t_split, t_merge) * 1e-3;
 }
 
 // Eq. 5 for the split + merge form whose split kernel runs on the tensor cores as
 // persistent CTAs (two per SM) taking the items on demand: the start-up once; the items,
-// all of one length, go in rounds of at most `ctas` (the last round may be partial, its
-// CTAs then sharing HBM among fewer); each item streams its chunk at the CTA's rate and
-// pays decode_tc_item_ns at its boundary; then the merge launch.
+// all of one length, go in rounds of at most 2 x SMs (the last round may be partial).
+// Within a round the active CTAs share HBM (the stage runs on the tensor pipe, so two CTAs
+// on an SM do not slow each other), each up to the rate one CTA sustains; an item streams
+// its chunk at that rate, or at one S -> softmax -> P.V chain per 64-key stage when that is
+// slower (Eq. 6 with an open load boundary), and pays decode_tc_item_ns at its boundary;
+// then the merge launch.
 constexpr double decode_tc_time_us(int splits, int B, int Hq, int Hkv, int Skv, int D, int num_sms,
                                    const ArchDesc& a = kGb300) {
   if (splits < 1 || num_sms < 1) return 1e300;
@@ -469,14 +483,17 @@ constexpr double decode_tc_time_us(int splits, int B, int Hq, int Hkv, int Skv, 
   const long long slots = 2LL * num_sms;
   const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
   const double chunk_bytes = 2.0 * chunk * D * 2;
+  const double chain = static_cast<double>(chunk / 64) * a.decode_tc_stage_ns;
   double t_split = a.cta_start_ns;
   for (long long left = items; left > 0;) {
     const long long active = left < slots ? left : slots;
     left -= active;
-    t_split += chunk_bytes / decode_cta_rate(static_cast<double>(active), num_sms, a) + a.decode_tc_item_ns;
+    double rate = a.hbm_gbs / static_cast<double>(active);
+    if (rate > a.decode_tc_cta_gbs) rate = a.decode_tc_cta_gbs;
+    t_split += heg_pipe(chunk_bytes / rate, chain, 0.0, 1, 1) + a.decode_tc_item_ns;
   }
   const double part_bytes = 1.0 * B * Hq * splits * (D + 1) * 4;
-  const double t_merge = a.launch_ns * 0.2 + 2.0 * part_bytes / a.hbm_gbs;
+  const double t_merge = a.decode_merge_ns + 2.0 * part_bytes / a.hbm_gbs;
   return heg_seq(t_split, t_merge) * 1e-3;
 }
 

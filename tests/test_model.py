@@ -181,14 +181,12 @@ def test_decode_more_splits_than_needed_cost_more(loom):
 def test_tc_decode_pays_the_start_up_once(loom, B, Hq, Hkv, Skv, D):
     # the persistent tensor-core split kernel starts once and streams its items back to
     # back, where the one-CTA-per-split kernel pays the start-up in every round of CTAs:
-    # with more than one round it is faster; in one round they differ by an item boundary
+    # with more than one round it is faster; no count beats the HBM roofline
     for s in range(1, min(64, math.ceil(Skv / 64)) + 1):
         t_tc = loom.loom_model_decode_tc_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS)
         t_cc = loom.loom_model_decode_time_us(s, B, Hq, Hkv, Skv, D, NUM_SMS)
         if B * Hkv * s > 2 * NUM_SMS:
             assert 0 < t_tc < t_cc, (s, t_tc, t_cc)
-        else:
-            assert abs(t_tc - t_cc) < 1.0, (s, t_tc, t_cc)
         assert t_tc * 1e-6 >= 2.0 * B * Hkv * Skv * D * 2 / (PEAK_GBS * 1e9) * 0.999
 
 
@@ -200,7 +198,19 @@ def test_tc_decode_rounds_and_limits(loom):
     # leaves 8 items to a second round, streamed by 8 CTAs at the rate one CTA sustains
     assert 8 * 38 == 2 * NUM_SMS
     assert t(39) > t(38) * 1.3
-    assert loom.loom_attn_decode_num_splits(1, 32, 8, 131072, 128) == 38
+    # the long decode's count fills the SMs once, two CTAs on some of them (32 splits x 8
+    # kv heads = 256 CTAs: the sweep's measured best)
+    s = loom.loom_attn_decode_num_splits(1, 32, 8, 131072, 128)
+    assert NUM_SMS < 8 * s <= 2 * NUM_SMS
+
+
+def test_tc_decode_stage_chain_floor(loom):
+    # at D = 64 a 64-key stage carries half the bytes for the same S -> softmax -> P.V
+    # chain: with every SM busy the chain, not HBM, bounds the stage, so the modeled time
+    # exceeds the byte time by the chain's share
+    t64 = loom.loom_model_decode_tc_time_us(19, 1, 64, 16, 65536, 64, NUM_SMS)
+    bytes_time = 2.0 * 16 * 65536 * 64 * 2 / (PEAK_GBS * 1e3)  # us
+    assert t64 > bytes_time * 1.2
 
 
 @pytest.mark.parametrize("D", [64, 128])
