@@ -837,10 +837,11 @@ def run_model_sweep(torch, loom, dev, stream, args, peaks):
         cands = []  # (modeled us, form, splits, cluster size): Eq. 9's candidates over forms and split counts
         # the split + merge form's split kernel runs on the tensor cores for up to 32 query
         # heads per kv head
-        split_merge = loom.loom_model_decode_tc_time_us if G <= 32 else loom.loom_model_decode_time_us
+        tc = G <= 32
+        split_merge = loom.loom_model_decode_tc_time_us if tc else loom.loom_model_decode_time_us
         for sp in range(1, n + 1):
             cands.append((split_merge(sp, B, Hq, Hkv, Skv, D, sms), 1, sp, 0))
-            if slots > 0:
+            if slots > 0 and not tc:  # the CUDA-core persistent kernel, where the tensor-core one does not run
                 cands.append((loom.loom_model_decode_persistent_time_us(sp, B, Hq, Hkv, Skv, D, slots), 2, sp, 0))
             for cs in range(1, min(16, sp) + 1):
                 if sp % cs == 0 and fits[cs] > 0:

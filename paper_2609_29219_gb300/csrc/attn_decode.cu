@@ -2051,11 +2051,14 @@ int decode_form(const DecodeArgs& a, int* cs_out) {
     *cs_out = ch.cs;
     return kDecodeCluster;
   }
-  const double t_split = (decode_tc_eligible(a) && !(PAGED && a.tc == 2))
-                             ? model::decode_tc_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms)
-                             : model::decode_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms);
+  // Where the split + merge form's split kernel runs on the tensor cores it is priced as
+  // such, and the CUDA-core persistent split kernel (the same schedule with a slower
+  // stage, measured slower or equal on every shape) is not a candidate.
+  const bool tc = decode_tc_eligible(a) && !(PAGED && a.tc == 2);
+  const double t_split = tc ? model::decode_tc_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms)
+                            : model::decode_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, sms);
   const double t_persist =
-      slots > 0 ? model::decode_persistent_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, slots) : 1e300;
+      (slots > 0 && !tc) ? model::decode_persistent_time_us(a.splits, a.B, a.Hq, a.Hkv, a.Skv, D, slots) : 1e300;
   int form = kDecodeSplitMerge;
   double best = t_split;
   if (t_persist < best * (1.0 - 1e-9)) {

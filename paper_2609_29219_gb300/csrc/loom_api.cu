@@ -141,7 +141,9 @@ int loom_attn_decode_num_splits(int B, int Hq, int Hkv, int Skv, int D) {
   // device, or from the GB300 estimate when no device answers.
   const bool device = current_sm_count() > 0;
   const int G = Hq / Hkv;
-  const int slots = device ? decode_persistent_slots(D, G) : sms * model::decode_stage(D).ctas_per_sm;
+  // (the CUDA-core persistent split kernel is a candidate only where the tensor-core one
+  // does not run)
+  const int slots = tc ? 0 : device ? decode_persistent_slots(D, G) : sms * model::decode_stage(D).ctas_per_sm;
   const int splits = model::choose_decode_plan(
                          B, Hq, Hkv, Skv, D, sms,
                          [&](int cs) {

@@ -112,17 +112,20 @@ DECODE_SHAPES = [(16, 32, 8, 8192, 128), (1, 32, 8, 131072, 128), (1, 8, 8, 4096
 def _decode_candidates(loom, B, Hq, Hkv, Skv, D):
     """Modeled time of every (form, split count) candidate: the split + merge form (its
     split kernel on the tensor cores where that kernel takes the shape, at most 32 query
-    heads per kv head) and the persistent split + merge form for every split count, the
+    heads per kv head; elsewhere also the CUDA-core persistent split + merge form) for
+    every split count, the
     cluster form for every split count and cluster size dividing it, with the CTAs and
     clusters they are priced at.  Form order for ties: split + merge (0), persistent (1),
     cluster (2)."""
     cands = []
     G = Hq // Hkv
     slots = loom.loom_decode_persistent_slots(D, G)
-    split_merge = loom.loom_model_decode_tc_time_us if G <= 32 else loom.loom_model_decode_time_us
+    tc = G <= 32
+    split_merge = loom.loom_model_decode_tc_time_us if tc else loom.loom_model_decode_time_us
     for s in range(1, min(1024, math.ceil(Skv / 64)) + 1):
         cands.append((split_merge(s, B, Hq, Hkv, Skv, D, NUM_SMS), 0, s))
-        cands.append((loom.loom_model_decode_persistent_time_us(s, B, Hq, Hkv, Skv, D, slots), 1, s))
+        if not tc:  # the CUDA-core persistent split kernel, where the tensor-core one does not run
+            cands.append((loom.loom_model_decode_persistent_time_us(s, B, Hq, Hkv, Skv, D, slots), 1, s))
         for cs in range(1, min(16, s) + 1):
             if s % cs:
                 continue
