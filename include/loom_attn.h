@@ -123,11 +123,16 @@ size_t loom_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int Skv, int D, 
  * rounded up to a multiple of 64; empty splits contribute nothing.  A sequence of
  * length 0 yields O = 0 and LSE = -inf.
  * Three forms compute it, chosen by the analytic model (see loom_attn_decode_form):
- *   1  a split kernel of one CTA per (split, batch, kv head) writing the partials (O_i,
- *      lse_i) into the workspace, then a merge kernel (the gather, global softmax and
- *      final scaling of the Flash Decode HEG);
- *   2  the same partials and merge kernel, with a persistent split kernel whose CTAs walk
- *      the (split, batch, kv head) items, streaming K/V across item boundaries;
+ *   1  a split kernel writing the partials (O_i, lse_i) into the workspace, then a merge
+ *      kernel (the gather, global softmax and final scaling of the Flash Decode HEG).
+ *      The split kernel runs on the tensor cores (D 64 or 128, at most 32 query heads
+ *      per kv head): persistent CTAs take the (sequence, kv head, split) items from a
+ *      counter in the workspace (loom_debug_decode_tensor_cores); otherwise it is a
+ *      CUDA-core kernel of one CTA per (split, batch, kv head);
+ *   2  the same partials and merge kernel, with a persistent CUDA-core split kernel whose
+ *      CTAs walk the (split, batch, kv head) items in a fixed order, streaming K/V across
+ *      item boundaries (the model considers it only where the tensor-core kernel does not
+ *      run);
  *   3  one persistent kernel in which clusters of cs CTAs (cs divides num_splits, cs <= 16)
  *      walk the (batch, kv head) pairs, CTA r taking splits r, r + cs, ... of each, and
  *      merge their partials over distributed shared memory; it leaves the workspace
