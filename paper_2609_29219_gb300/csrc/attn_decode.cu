@@ -529,14 +529,16 @@ __global__ void __launch_bounds__(C::THREADS, C::CTAS_PER_SM)
 // exponentials per head and stage instead of every product of the dot products.
 //   warps: 0 query rows (Q into TMEM, softmax, epilogue; TMEM lanes 0-31), 1 loader
 //   (TMA, lane 0), 2 MMA issuer (whole warp, one elected lane)
-//   TMEM: [0, D/2) Q as bf16 pairs | [64, 128) S, then P over its first 32 columns |
-//         [128, 128 + D) O
+//   TMEM: [0, D/2) Q as bf16 pairs | [64, 64 + T) S, then P over its first T/2 columns |
+//         [64 + T, 64 + T + D) O
 template <int D>
 struct DecodeTcCfg {
-  static constexpr int T = 64;  // keys per stage
-  // ring depth: about 96 KB of shared memory at either D, so that exactly two CTAs share
-  // an SM (their 2 x 256 TMEM columns are the SM's 512)
-  static constexpr int NSTAGE = D == 64 ? 6 : 3;
+  // keys per stage: 64 at D = 128; 128 at D = 64, where a 64-key stage's bytes arrive
+  // faster than its S -> softmax -> P.V chain runs and the TMEM columns allow the wider S
+  static constexpr int T = model::decode_tc_stage_keys(D);
+  // ring depth: 3 stages of 32 KB, so that exactly two CTAs share an SM (their 2 x 256
+  // TMEM columns are the SM's 512)
+  static constexpr int NSTAGE = 3;
   static constexpr int NBOX = D / 64;                     // 128-byte swizzle atoms along D
   static constexpr uint32_t BOX_BYTES = T * 128;          // 64 keys x 64 dims
   static constexpr uint32_t TILE_BYTES = NBOX * BOX_BYTES;  // one K or V tile
@@ -549,14 +551,99 @@ struct DecodeTcCfg {
   static constexpr uint32_t BYTES = ABORT_OFF + 16 + 1024;  // + 1024-byte alignment slack
   static constexpr uint32_t Q_COL = 0;
   static constexpr uint32_t S_COL = 64;
-  static constexpr uint32_t O_COL = 128;
+  static constexpr uint32_t O_COL = S_COL + T;
   static constexpr uint32_t TMEM_COLS = 256;  // a power of two: 2 CTAs per SM
   static constexpr int THREADS = 96;
   static constexpr int MAX_G = kDecodeTcMaxGroup;  // query heads per kv head: TMEM lanes of warp 0
   static_assert(O_COL + D <= TMEM_COLS, "TMEM budget");
-  static_assert(Q_COL + D / 2 <= S_COL && S_COL + T <= O_COL, "TMEM regions");
+  static_assert(Q_COL + D / 2 <= S_COL && S_COL + T <= O_COL && O_COL + D <= TMEM_COLS, "TMEM regions");
+  static_assert(T % 64 == 0 && T % kDecodeChunkAlign == 0, "stages of whole 64-key score halves");
   static_assert(2 * (BYTES + 1024) <= 228 * 1024 && 3 * (BYTES + 1024) > 228 * 1024, "exactly two CTAs per SM");
 };
+
+// 64 scores of this lane's row from TMEM column `taddr` on, keys at or past `nvalid` (of
+// these 64) masked to -inf.
+__device__ __forceinline__ void decode_tc_scores64(uint32_t taddr, uint32_t* s, int nvalid) {
+  tmem_ld32(taddr, s);
+  tmem_ld32(taddr + 32, s + 32);
+  tmem_wait_ld();
+  reg_fence32(s);
+  reg_fence32(s + 32);
+  if (nvalid < 64) {
+#pragma unroll
+    for (int i = 0; i < 64; ++i)
+      if (i >= nvalid) s[i] = __float_as_uint(-INFINITY);
+  }
+}
+
+__device__ __forceinline__ float decode_tc_max64(const uint32_t* s) {
+  float mm[8];
+#pragma unroll
+  for (int g = 0; g < 8; ++g) mm[g] = __uint_as_float(s[g]);
+#pragma unroll
+  for (int i = 8; i + 16 <= 64; i += 16)
+#pragma unroll
+    for (int g = 0; g < 8; ++g) mm[g] = max3(mm[g], __uint_as_float(s[i + g]), __uint_as_float(s[i + 8 + g]));
+#pragma unroll
+  for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], __uint_as_float(s[56 + g]));
+  return fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
+}
+
+// One stage's softmax on warp 0 of a tensor-core split kernel (lane = a query head's row):
+// the stage's T scores are read from TMEM in 64-key halves (twice when T = 128: once for
+// the maximum, once for the exponentials, so that 64 scores are live at a time), keys at
+// or past ntok are masked, the running maximum (base 2, scaled by c) moves only when it
+// grows by more than kRescaleThreshold, and P goes back over S as bf16 pairs (a half's 64
+// keys in 32 columns).  Returns the row sum of P; *alpha is the factor O needs, *need
+// whether the maximum moved.
+template <class C>
+__device__ __forceinline__ float decode_tc_softmax(uint32_t tmem, int ntok, float c, float* m_run, float* alpha,
+                                                   bool* need) {
+  constexpr int NH = C::T / 64;
+  uint32_t s[64];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int h = 0; h < NH; ++h) {
+    decode_tc_scores64(tmem + C::S_COL + 64 * h, s, ntok - 64 * h);
+    mx = fmaxf(mx, decode_tc_max64(s));
+  }
+  const float m_new = fmaxf(*m_run, mx * c);
+  *need = m_new > *m_run + kRescaleThreshold;
+  *alpha = *need ? ex2(*m_run - m_new) : 1.f;
+  if (*need) *m_run = m_new;
+  const float ms = (*m_run == -INFINITY) ? 0.f : *m_run;
+  const uint64_t c2 = f2(c, c);
+  const uint64_t nms2 = f2(-ms, -ms);
+  uint64_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+  for (int h = 0; h < NH; ++h) {
+    if (NH > 1) decode_tc_scores64(tmem + C::S_COL + 64 * h, s, ntok - 64 * h);  // (one half: still in s)
+    uint32_t pk[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const uint64_t x = fma2(f2(__uint_as_float(s[2 * i]), __uint_as_float(s[2 * i + 1])), c2, nms2);
+      const float p0 = ex2(f2lo(x));
+      const float p1 = ex2(f2hi(x));
+      acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
+      pk[i] = pack_bf16x2(p0, p1);
+    }
+    // P of keys [64h, 64h + 64) over S columns [32h, 32h + 32): S of those columns was read
+    tmem_st32(tmem + C::S_COL + 32 * h, pk);
+  }
+  tmem_wait_st();
+  const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+  return f2lo(a01) + f2hi(a01);
+}
+
+// O += P V over one stage: P (bf16, TMEM, T/2 columns) x the stage's V tile (MN-major), in
+// groups of 64 keys (four K = 16 steps each).
+template <class C>
+__device__ __forceinline__ void decode_tc_issue_pv(uint32_t tmem, uint32_t vtile, uint32_t idesc_pv, bool accumulate) {
+#pragma unroll
+  for (int g = 0; g < C::T / 64; ++g)
+    mma_ts_k64_el(tmem + C::O_COL, tmem + C::S_COL + 32 * g, sdesc_sw128(vtile + g * 64 * 128, C::BOX_BYTES, 1024),
+                  idesc_pv, (accumulate || g > 0) ? 1u : 0u);
+}
 
 // Warp 0 of decode_tc_split_kernel: lane h is query head h0 + h (lanes >= G carry zero rows).
 // Q goes into TMEM as bf16 pairs (its memory order); per stage the lane reads its 64
@@ -593,52 +680,15 @@ __device__ __forceinline__ void decode_tc_rows(const __nv_bfloat16* __restrict__
     __syncwarp();
     if (lane == 0) mbar_arrive(bar_q);
   }
-  const uint64_t c2 = f2(c, c);
   float m_run = -INFINITY, l_run = 0.f;
   bool ok = true;
   for (int it = 0; it < n_st; ++it) {
     if (!(ok = mbar_wait_warp(bar_s, it & 1, ctl, ab))) break;
     tc_fence_after();
-    uint32_t s[C::T];
-    tmem_ld32(tmem + C::S_COL, s);
-    tmem_ld32(tmem + C::S_COL + 32, s + 32);
-    tmem_wait_ld();
-    reg_fence32(s);
-    reg_fence32(s + 32);
     const int ntok = min(C::T, t_end - (t_begin + it * C::T));
-    if (ntok < C::T) {
-#pragma unroll
-      for (int i = 0; i < C::T; ++i)
-        if (i >= ntok) s[i] = __float_as_uint(-INFINITY);
-    }
-    float mm[8];
-#pragma unroll
-    for (int g = 0; g < 8; ++g) mm[g] = __uint_as_float(s[g]);
-#pragma unroll
-    for (int i = 8; i + 16 <= C::T; i += 16)
-#pragma unroll
-      for (int g = 0; g < 8; ++g) mm[g] = max3(mm[g], __uint_as_float(s[i + g]), __uint_as_float(s[i + 8 + g]));
-#pragma unroll
-    for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], __uint_as_float(s[C::T - 8 + g]));
-    const float mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
-    const float m_new = fmaxf(m_run, mx * c);
-    const bool need = m_new > m_run + kRescaleThreshold;
-    const float alpha = need ? ex2(m_run - m_new) : 1.f;
-    if (need) m_run = m_new;
-    const float ms = (m_run == -INFINITY) ? 0.f : m_run;
-    const uint64_t nms2 = f2(-ms, -ms);
-    uint64_t acc[4] = {0, 0, 0, 0};
-    uint32_t pk[C::T / 2];
-#pragma unroll
-    for (int i = 0; i < C::T / 2; ++i) {
-      const uint64_t x = fma2(f2(__uint_as_float(s[2 * i]), __uint_as_float(s[2 * i + 1])), c2, nms2);
-      const float p0 = ex2(f2lo(x));
-      const float p1 = ex2(f2hi(x));
-      acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
-      pk[i] = pack_bf16x2(p0, p1);
-    }
-    tmem_st32(tmem + C::S_COL, pk);
-    tmem_wait_st();
+    float alpha;
+    bool need;
+    const float psum = decode_tc_softmax<C>(tmem, ntok, c, &m_run, &alpha, &need);
     if (ntok < C::T) {
       // V rows past the split's end may hold anything (a cache past a sequence's length
       // is never written): zero them so that their P = 0 adds exactly nothing to P.V
@@ -676,8 +726,7 @@ __device__ __forceinline__ void decode_tc_rows(const __nv_bfloat16* __restrict__
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(bar_p);
-    const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
-    l_run = l_run * alpha + (f2lo(a01) + f2hi(a01));
+    l_run = l_run * alpha + psum;
   }
   if (!ok) return;
   // epilogue: the last P.V, then O / l and the log-sum-exp of each real row
@@ -815,8 +864,7 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
       if (!(ok = mbar_wait_warp(bar_p, it & 1, ctl, ab))) break;
       tc_fence_after();
       // O += P V over the stage's 64 keys
-      mma_ts_k64_el(tmem + C::O_COL, tmem + C::S_COL, sdesc_sw128(kslot + C::TILE_BYTES, C::BOX_BYTES, 1024),
-                    idesc_pv, it > 0 ? 1u : 0u);
+      decode_tc_issue_pv<C>(tmem, kslot + C::TILE_BYTES, idesc_pv, it > 0);
       tc_commit_el(bar_o);
       tc_commit_el(bar_empty + 8 * s);
     }
@@ -881,7 +929,6 @@ __device__ __forceinline__ void decode_tc_persist_rows(const uint8_t* smem, floa
   using L = DecodeTcPersistCfg<D>;
   const int lane = threadIdx.x & 31;
   const bool real = lane < G;
-  const uint64_t c2 = f2(c, c);
   float m_run = -INFINITY, l_run = 0.f;
   int nq = 0;
   for (int st = 0;; ++st) {
@@ -921,45 +968,9 @@ __device__ __forceinline__ void decode_tc_persist_rows(const uint8_t* smem, floa
     }
     if (!mbar_wait_warp(bar_s, st & 1, ctl, ab)) return;
     tc_fence_after();
-    uint32_t s[C::T];
-    tmem_ld32(tmem + C::S_COL, s);
-    tmem_ld32(tmem + C::S_COL + 32, s + 32);
-    tmem_wait_ld();
-    reg_fence32(s);
-    reg_fence32(s + 32);
-    if (ntok < C::T) {
-#pragma unroll
-      for (int i = 0; i < C::T; ++i)
-        if (i >= ntok) s[i] = __float_as_uint(-INFINITY);
-    }
-    float mm[8];
-#pragma unroll
-    for (int g = 0; g < 8; ++g) mm[g] = __uint_as_float(s[g]);
-#pragma unroll
-    for (int i = 8; i + 16 <= C::T; i += 16)
-#pragma unroll
-      for (int g = 0; g < 8; ++g) mm[g] = max3(mm[g], __uint_as_float(s[i + g]), __uint_as_float(s[i + 8 + g]));
-#pragma unroll
-    for (int g = 0; g < 8; ++g) mm[g] = fmaxf(mm[g], __uint_as_float(s[C::T - 8 + g]));
-    const float mx = fmaxf(max3(mm[0], mm[1], mm[2]), max3(max3(mm[3], mm[4], mm[5]), mm[6], mm[7]));
-    const float m_new = fmaxf(m_run, mx * c);
-    const bool need = m_new > m_run + kRescaleThreshold;
-    const float alpha = need ? ex2(m_run - m_new) : 1.f;
-    if (need) m_run = m_new;
-    const float ms = (m_run == -INFINITY) ? 0.f : m_run;
-    const uint64_t nms2 = f2(-ms, -ms);
-    uint64_t acc[4] = {0, 0, 0, 0};
-    uint32_t pk[C::T / 2];
-#pragma unroll
-    for (int i = 0; i < C::T / 2; ++i) {
-      const uint64_t x = fma2(f2(__uint_as_float(s[2 * i]), __uint_as_float(s[2 * i + 1])), c2, nms2);
-      const float p0 = ex2(f2lo(x));
-      const float p1 = ex2(f2hi(x));
-      acc[i & 3] = add2(acc[i & 3], f2(p0, p1));
-      pk[i] = pack_bf16x2(p0, p1);
-    }
-    tmem_st32(tmem + C::S_COL, pk);
-    tmem_wait_st();
+    float alpha;
+    bool need;
+    const float psum = decode_tc_softmax<C>(tmem, ntok, c, &m_run, &alpha, &need);
     if (ntok < C::T) {
       // V rows past the split's end may hold anything: zero them (P = 0 meets 0)
       uint4* vt = reinterpret_cast<uint4*>(const_cast<uint8_t*>(smem) + slot * C::STAGE_BYTES + C::TILE_BYTES);
@@ -993,8 +1004,7 @@ __device__ __forceinline__ void decode_tc_persist_rows(const uint8_t* smem, floa
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(bar_p);
-    const uint64_t a01 = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
-    l_run = l_run * alpha + (f2lo(a01) + f2hi(a01));
+    l_run = l_run * alpha + psum;
     if (j == n_st - 1) {
       // the item's last P.V, then O / l and the log-sum-exp of each real row
       if (!mbar_wait_warp(bar_o, st & 1, ctl, ab)) return;
@@ -1179,7 +1189,7 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
           if constexpr (PAGED) {
             const int P = pv.page_size;
             const int rows = P < C::T ? P : C::T;
-            const int npiece = (ntok + rows - 1) / rows;  // at most 8 (pages of 8 keys or more)
+            const int npiece = (ntok + rows - 1) / rows;  // at most T / 8 <= 16 (pages of 8 keys or more)
             if (lane == 0) mbar_expect_tx(bar_full + 8 * s, 2u * C::NBOX * npiece * rows * 128);
             __syncwarp();
             if (lane < npiece) {
@@ -1272,8 +1282,7 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
       tc_commit_el(bar_s);
       if (!mbar_wait_warp(bar_p, st & 1, ctl, ab)) break;
       tc_fence_after();
-      mma_ts_k64_el(tmem + C::O_COL, tmem + C::S_COL, sdesc_sw128(kslot + C::TILE_BYTES, C::BOX_BYTES, 1024),
-                    idesc_pv, j > 0 ? 1u : 0u);
+      decode_tc_issue_pv<C>(tmem, kslot + C::TILE_BYTES, idesc_pv, j > 0);
       tc_commit_el(bar_o);
       tc_commit_el(bar_empty + 8 * s);
     }
@@ -1858,14 +1867,15 @@ cudaError_t launch_split(const DecodeArgs& a, const PagedKV* pk, const KernelCtl
 }
 
 // The contiguous cache [B, Hkv, Skv, D] as a 3-D tensor (dim, key, kv head of a sequence)
-// in 64-dim x 64-key boxes, 128-byte swizzled: the tensor-core split kernel's K and V tiles.
+// in 64-dim x T-key boxes (T: the tensor-core stage's keys at this D), 128-byte swizzled:
+// the tensor-core split kernels' K and V tiles.
 bool kv_map_sw128(CUtensorMap* map, const void* cache, int B, int Hkv, int Skv, int D) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return false;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(Skv),
                         static_cast<cuuint64_t>(B) * Hkv};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(Skv) * D * 2};
-  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(DecodeTcCfg<128>::T), 1};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(model::decode_tc_stage_keys(D)), 1};
   cuuint32_t estr[3] = {1, 1, 1};
   return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(cache), dims, strides, box, estr,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,

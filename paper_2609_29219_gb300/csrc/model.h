@@ -73,10 +73,10 @@ struct ArchDesc {
   double decode_tc_cta_gbs;         // persistent tensor-core decode: KV stream rate one CTA sustains
                                     // when HBM is not the bound (fitted: B1 H32/8 Skv 131072 with
                                     // 8 and 16 splits, 64 and 128 CTAs, 218.6 and 117.2 us)
-  double decode_tc_stage_ns;        // persistent tensor-core decode: one 64-key stage's S -> softmax
-                                    // -> P.V chain, the floor of a stage when its bytes arrive faster
-                                    // (fitted: D = 64, B1 H64/16 Skv 65536, 19 splits: 56.6 us for 54
-                                    // stages per CTA)
+  double decode_tc_stage_ns;        // persistent tensor-core decode: the S -> softmax -> P.V chain
+                                    // per 64 keys of a stage, the floor of a stage when its bytes
+                                    // arrive faster (fitted: D = 64, B1 H64/16 Skv 65536, 19 splits
+                                    // in 128-key stages: 54.4 us for 3456 keys per CTA)
   double decode_merge_ns;           // the merge launch's fixed cost in a decode step: the dependent
                                     // launch, its wait for the split grid, one round trip to the
                                     // partials (fitted: a timing probe without the merge launch,
@@ -86,7 +86,7 @@ struct ArchDesc {
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 3400.0, 3000.0, 28.4, 150.0, 7800.0, 300.0, 39.0, 870.0, 3000.0,
+    129.0e6, 1.07, 3400.0, 3000.0, 28.4, 150.0, 7800.0, 300.0, 39.0, 835.0, 3000.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
@@ -468,6 +468,11 @@ constexpr double decode_persistent_time_us(int splits, int B, int Hq, int Hkv, i
   return heg_seq(t_split, t_merge) * 1e-3;
 }
 
+// Keys per stage of the tensor-core decode split kernels: 64 at D = 128 (TMEM: q 64, S 64
+// and O 128 columns of a CTA's 256); 128 at D = 64 (q 32, S 128, O 64), where a 64-key
+// stage carries too few bytes to cover its S -> softmax -> P.V chain.
+constexpr int decode_tc_stage_keys(int D) { return D == 64 ? 128 : 64; }
+
 // Eq. 5 for the split + merge form whose split kernel runs on the tensor cores as
 // persistent CTAs (two per SM) taking the items on demand: the start-up once; the items,
 // all of one length, go in rounds of at most 2 x SMs (the last round may be partial).
@@ -483,7 +488,7 @@ constexpr double decode_tc_time_us(int splits, int B, int Hq, int Hkv, int Skv, 
   const long long slots = 2LL * num_sms;
   const long long chunk = cdiv(cdiv(Skv, splits), 64) * 64;
   const double chunk_bytes = 2.0 * chunk * D * 2;
-  const double chain = static_cast<double>(chunk / 64) * a.decode_tc_stage_ns;
+  const double chain = static_cast<double>(chunk / 64) * a.decode_tc_stage_ns;  // per 64 keys of the chunk
   double t_split = a.cta_start_ns;
   for (long long left = items; left > 0;) {
     const long long active = left < slots ? left : slots;
