@@ -378,8 +378,8 @@ void loom_debug_gemm_order(int group_rows, int k_alternate);
  *   1 (the default): tensor cores, persistent, contiguous or paged cache.  Two CTAs per
  *     SM take (sequence, kv head, split) items, longest sequence first, from a counter in
  *     the workspace's last 256 bytes until none is left, and stream the next item's q and
- *     K/V without a break (a paged cache: each 64-key stage copied page by page); per
- *     64-key stage S = Q K^T and O += P V are tcgen05 MMAs with the query heads as rows
+ *     K/V without a break (a paged cache: each stage copied page by page); per stage of
+ *     64 keys (128 at D = 64) S = Q K^T and O += P V are tcgen05 MMAs with the query heads as rows
  *     of a TMEM tile and the softmax on one warp.  The merge kernel re-arms the counter;
  *     a workspace whose counter was never armed (its first call) is dealt statically.
  *   2: the same stage on the tensor cores, one CTA per (split, kv head, sequence), for a

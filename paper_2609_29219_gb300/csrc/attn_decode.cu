@@ -518,14 +518,14 @@ __global__ void __launch_bounds__(C::THREADS, C::CTAS_PER_SM)
 }
 
 // ---------------------------------------------------------------- tensor-core split kernel
-// The split kernel of the split + merge form for a contiguous cache with the dot products
-// on the tensor cores (Sec. 2.6 Flash Decode HEG, local softmax loop).  The query heads
-// of one kv head are the rows of a 128-row tile held in TMEM (rows 0..G-1; the rest are
-// zero and their results unused): per 64-key stage S = Q K^T is one M = 128 MMA with A in
+// The split kernel of the split + merge form with the dot products on the tensor cores
+// (Sec. 2.6 Flash Decode HEG, local softmax loop).  The query heads of one kv head are the
+// rows of a 128-row tile held in TMEM (rows 0..G-1; the rest are zero and their results
+// unused): per stage of T keys (64; 128 at D = 64) S = Q K^T is one M = 128 MMA with A in
 // TMEM and the 128B-swizzled K tile as B, one warp (lane = query head) turns S into P =
 // 2^(S c - m) in place as bf16, and O += P V is a second MMA with P in TMEM and V as an
 // MN-major B.  The padded rows cost nothing that matters here -- the stage's MMAs take a
-// fraction of the time its bytes take to arrive -- while the CUDA cores are left with 64
+// fraction of the time its bytes take to arrive -- while the CUDA cores are left with T
 // exponentials per head and stage instead of every product of the dot products.
 //   warps: 0 query rows (Q into TMEM, softmax, epilogue; TMEM lanes 0-31), 1 loader
 //   (TMA, lane 0), 2 MMA issuer (whole warp, one elected lane)
@@ -1032,8 +1032,8 @@ __device__ __forceinline__ void decode_tc_persist_rows(const uint8_t* smem, floa
   }
 }
 
-// PAGED: K/V from a paged cache.  A 64-key stage is then copied in pieces of min(page
-// size, 64) keys, one per page it touches (each page looked up in the block table, each
+// PAGED: K/V from a paged cache.  A stage of T keys is then copied in pieces of min(page
+// size, T) keys, one per page it touches (each page looked up in the block table, each
 // piece looked up and copied by its own loader lane), into the same 128-byte-swizzled
 // tile: a piece of r rows starts r x 128 bytes into its box, a multiple of 1024 (page
 // sizes 8, 16, 32 or multiples of 64), so the swizzle pattern is the one a single 64-row
