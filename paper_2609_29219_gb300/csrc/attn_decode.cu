@@ -1033,7 +1033,7 @@ __device__ __forceinline__ void decode_tc_persist_rows(const uint8_t* smem, floa
 }
 
 // PAGED: K/V from a paged cache.  A stage of T keys is then copied in pieces of min(page
-// size, T) keys, one per page it touches (each page looked up in the block table, each
+// size, 64) keys, one per page it touches (each page looked up in the block table, each
 // piece looked up and copied by its own loader lane), into the same 128-byte-swizzled
 // tile: a piece of r rows starts r x 128 bytes into its box, a multiple of 1024 (page
 // sizes 8, 16, 32 or multiples of 64), so the swizzle pattern is the one a single 64-row
@@ -1187,8 +1187,10 @@ __global__ void __launch_bounds__(DecodeTcCfg<D>::THREADS, 2)
             rec[6] = ntok;
           }
           if constexpr (PAGED) {
+            // pieces of min(page, 64) keys: a stage starts on a multiple of 64, so a piece
+            // never crosses a page even when a stage (128 keys at D = 64) does
             const int P = pv.page_size;
-            const int rows = P < C::T ? P : C::T;
+            const int rows = P < kDecodeChunkAlign ? P : kDecodeChunkAlign;
             const int npiece = (ntok + rows - 1) / rows;  // at most T / 8 <= 16 (pages of 8 keys or more)
             if (lane == 0) mbar_expect_tx(bar_full + 8 * s, 2u * C::NBOX * npiece * rows * 128);
             __syncwarp();
@@ -1946,7 +1948,7 @@ cudaError_t launch_tc_persist(const DecodeArgs& a, const PagedKV* pk, const Kern
   PagedView view{nullptr, 0, 0, 0, 0};
   if (!q_map_sw128(&tq, a.q, a.B * a.Hq, D, G)) return cudaErrorInvalidValue;
   if constexpr (PAGED) {
-    const int rows = pk->page_size < DecodeTcCfg<D>::T ? pk->page_size : DecodeTcCfg<D>::T;
+    const int rows = pk->page_size < kDecodeChunkAlign ? pk->page_size : kDecodeChunkAlign;
     if (!paged_map_sw128(&tk, a.k, *pk, a.Hkv, D, rows) || !paged_map_sw128(&tv, a.v, *pk, a.Hkv, D, rows))
       return cudaErrorInvalidValue;
     view = PagedView{pk->block_table, pk->page_size, pk->max_pages, pk->num_pages, pk->layout == kPagedHND ? 1 : 0};

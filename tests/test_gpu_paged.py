@@ -98,6 +98,22 @@ def test_page_sizes(loom, P, D, layout):
         assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"P={P} D={D} splits={splits}")
 
 
+@LAYOUTS
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("P", [64, 128, 256])
+def test_splits_starting_mid_page(loom, P, D, layout):
+    """Chunks of 192 keys (900 keys in 5 splits): splits start on odd multiples of 64, so
+    a stage (128 keys at D = 64) runs across a page boundary; every copy must stay within
+    its page."""
+    B, Hq, Hkv = 3, 8, 2
+    lens = [900, 2 * P + 192, 191]
+    q, kc, vc, table, sl = paged_case(P + 3 * D, B, Hq, Hkv, P, lens, D)
+    for splits in (5, 3):
+        o, lse = run_paged(loom, q, kc, vc, table, sl, splits, layout)
+        o_ref, lse_ref = oracle.decode_paged(q, kc, vc, table, sl, page_size=P)
+        assert_parity(o_to_f64(o)[:, :, 0], o_ref, lse.cpu().numpy(), lse_ref, f"P={P} D={D} splits={splits}")
+
+
 @pytest.mark.parametrize("G", [1, 2, 4, 8, 16])
 def test_gqa_groups(loom, G):
     B, Hkv, P, D = 2, 2, 16, 128
