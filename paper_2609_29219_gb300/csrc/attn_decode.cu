@@ -646,10 +646,11 @@ __device__ __forceinline__ void decode_tc_issue_pv(uint32_t tmem, uint32_t vtile
 }
 
 // Warp 0 of decode_tc_split_kernel: lane h is query head h0 + h (lanes >= G carry zero rows).
-// Q goes into TMEM as bf16 pairs (its memory order); per stage the lane reads its 64
-// scores, masks keys past the split's end, moves the running max lazily (O rescaled in
-// TMEM after the previous P.V when it moved by more than kRescaleThreshold), writes P over
-// S and arrives on bar_p; at the end O / l and the log-sum-exp go to the split's partial.
+// Q goes into TMEM as bf16 pairs (its memory order); per stage the lane runs
+// decode_tc_softmax over its T scores (keys past the split's end masked, P written over
+// S), rescales O in TMEM after the previous P.V when the running max moved, zeroes the V
+// rows past the split's end, and arrives on bar_p; at the end O / l and the log-sum-exp
+// go to the split's partial.
 template <int D>
 __device__ __forceinline__ void decode_tc_rows(const __nv_bfloat16* __restrict__ q, float* __restrict__ o_part,
                                                float* __restrict__ lse_part, uint32_t tmem, int b, int h0, int G,
