@@ -126,7 +126,7 @@ class ClockSampler:
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one launch of the
 # headline prefill kernel from an ncu capture of it, and the SHA-256 of the kernel
 # sources it was taken from: the number is reported only while the sources are unchanged.
-PROFILED_TRAFFIC_BYTES = 242.8e6
+PROFILED_TRAFFIC_BYTES = 243.0e6
 PROFILED_SOURCES_SHA256 = "8a2a9d5f3176395e3a8c3a6a08c7db05b0f532a5115c45d4ad7a71186654aa59"
 
 
