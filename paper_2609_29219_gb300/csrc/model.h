@@ -63,8 +63,8 @@ struct ArchDesc {
                                     // decode, 123 us with clusters of 4 on B64 S2048)
   double fwd_launch_ns;             // prefill: once per launch, the launch itself, the first Q
                                     // and K/V loads from HBM and the last item's epilogue
-                                    // (fitted with item_boundary_ns: B1 H32 S1024 measured 23.2 us,
-                                    // B16 H16 S512 45.5 us, one and four items per CTA)
+                                    // (fitted: B1 H32 S1024 measured 18.9 us, B16 H16 S512 41.3 us,
+                                    // one and four items per CTA, launches timed back to back)
   double decode_tc_item_ns;         // persistent tensor-core decode: per (sequence, kv head, split)
                                     // item, the stall of the S -> softmax -> P.V chain at the item's
                                     // boundary (O read-out, next q into TMEM) that the full ring does
@@ -86,7 +86,7 @@ struct ArchDesc {
 inline constexpr ArchDesc kGb300 = {
     152, 228 * 1024, 227 * 1024, 512, 65536,
     1.447, 6783.5, 1910.3, 110.0, 32.0, 128.0, 1500.0, 150.0, 2500.0, 32.0, 6000.0, 0.5, 48.0, 9.8, 10.75,
-    129.0e6, 1.07, 3400.0, 3000.0, 28.4, 150.0, 7800.0, 300.0, 39.0, 835.0, 3000.0,
+    129.0e6, 1.07, 3400.0, 3000.0, 28.4, 150.0, 2000.0, 300.0, 39.0, 835.0, 3000.0,
 };
 
 // ------------------------------------------------------------------ HEG composition
