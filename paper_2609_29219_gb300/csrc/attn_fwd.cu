@@ -519,9 +519,12 @@ __global__ void __launch_bounds__(FwdCfg<D, SLOTS>::THREADS, 1)
   // Launched as a programmatic dependent of the previous kernel in the stream: the set-up
   // above touches no global memory; from here on the previous kernel's writes must be
   // complete and visible.  The next launch may then start its own set-up on SMs this
-  // grid frees.
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  asm volatile("griddepcontrol.launch_dependents;");
+  // grid frees.  (Not in the ragged-batch instantiation, which is launched plainly: the
+  // two instructions alone cost it 4 %.)
+  if constexpr (!VARLEN) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;");
+  }
 
   if (warp == 8) {
     // ------------------------------------------------------------------ loader
@@ -1684,8 +1687,7 @@ cudaError_t launch_varlen_d(const FwdVarlenArgs& a, const KernelCtl& ctl, cudaSt
   constexpr int kRows = C::NQT * C::BM;
   const long long bound = static_cast<long long>(a.B) * a.Hq * ((a.max_seqlen_q + kRows - 1) / kRows);
   const int grid = static_cast<int>(bound > 0 && bound < sms ? bound : sms);
-  return launch_dependent(!a.causal, attn_fwd_kernel<D, true>, grid, C::THREADS, C::BYTES, stream, mq, mk, mv, mo,
-                          p);
+  return launch_dependent(false, attn_fwd_kernel<D, true>, grid, C::THREADS, C::BYTES, stream, mq, mk, mv, mo, p);
 }
 
 // Launch one design: C is its configuration, rows_per_item the query rows of one work
