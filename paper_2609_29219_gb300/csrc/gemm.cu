@@ -608,6 +608,11 @@ __global__ void __launch_bounds__(GemmPairCfgT<NS>::THREADS, 1)
   cluster_sync_all();  // both CTAs' barriers initialised, TMEM allocated in both
   tc_fence_after();
   const uint32_t tmem = *tmem_ptr;
+  // Launched as a programmatic dependent of the previous kernel in the stream: the set-up
+  // above touches no global memory; from here on that kernel's writes must be complete
+  // and visible, and the next launch may start its own set-up on SMs this grid frees.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;");
 
   if (warp == 8) {
     // ------------------------------------------------------------------ loader (both CTAs)
@@ -926,7 +931,7 @@ bool prepare_pair(int dev) {
 }
 
 template <int NS = 6>
-cudaLaunchConfig_t pair_config(int grid, cudaStream_t stream, cudaLaunchAttribute* attr) {
+cudaLaunchConfig_t pair_config(int grid, cudaStream_t stream, cudaLaunchAttribute* attr, bool dependent = false) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
   cfg.blockDim = dim3(GemmPairCfgT<NS>::THREADS, 1, 1);
@@ -938,6 +943,11 @@ cudaLaunchConfig_t pair_config(int grid, cudaStream_t stream, cudaLaunchAttribut
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  if (dependent) {  // a programmatic dependent of the previous kernel (attr holds two entries)
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.numAttrs = 2;
+  }
   return cfg;
 }
 
@@ -1000,8 +1010,8 @@ cudaError_t launch_pair(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t st
     }
   }
   const long long pairs = p.n_units < avail ? p.n_units : avail;
-  cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = pair_config<NS>(static_cast<int>(2 * pairs), stream, attr);
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = pair_config<NS>(static_cast<int>(2 * pairs), stream, attr, true);
   return cudaLaunchKernelEx(&cfg, gemm_pair_kernel<BKM, NS>, ma, mb, mc, mbn, p);
 }
 
