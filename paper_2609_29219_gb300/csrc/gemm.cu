@@ -185,6 +185,11 @@ __global__ void __launch_bounds__(GemmCfg<BN, NS>::THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_ptr;
+  // Launched as a programmatic dependent of the previous kernel in the stream: the set-up
+  // above touches no global memory; from here on that kernel's writes must be complete
+  // and visible, and the next launch may start its own set-up on SMs this grid frees.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;");
 
   if (warp == 8) {
     // ------------------------------------------------------------------ loader
@@ -841,8 +846,18 @@ cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stre
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   const int grid = static_cast<int>(tiles < sms ? tiles : sms);
-  gemm_kernel<BN, BKM, NS><<<grid, C::THREADS, C::BYTES, stream>>>(ma, mb, mc, p);
-  return cudaGetLastError();
+  // a programmatic dependent of the previous kernel (the kernel waits for it after its set-up)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(C::THREADS);
+  cfg.dynamicSmemBytes = C::BYTES;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gemm_kernel<BN, BKM, NS>, ma, mb, mc, p);
 }
 
 template <int BN>
