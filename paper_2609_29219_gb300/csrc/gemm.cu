@@ -347,6 +347,11 @@ __global__ void __launch_bounds__(GemmCfg<BN>::SPLIT_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_ptr;
+  // Launched as a programmatic dependent of the previous kernel in the stream: the set-up
+  // above touches no global memory; from here on that kernel's writes must be complete
+  // and visible, and the next launch may start its own set-up.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;");
 
   if (warp == 4) {
     // ------------------------------------------------------------------ loader
@@ -861,7 +866,8 @@ cudaError_t launch_bn(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t stre
 }
 
 template <int BN>
-cudaLaunchConfig_t splitk_config(int grid, int S, cudaStream_t stream, cudaLaunchAttribute* attr) {
+cudaLaunchConfig_t splitk_config(int grid, int S, cudaStream_t stream, cudaLaunchAttribute* attr,
+                                 bool dependent = false) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
   cfg.blockDim = dim3(GemmCfg<BN>::SPLIT_THREADS, 1, 1);
@@ -873,6 +879,11 @@ cudaLaunchConfig_t splitk_config(int grid, int S, cudaStream_t stream, cudaLaunc
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  if (dependent) {  // a programmatic dependent of the previous kernel (attr holds two entries)
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.numAttrs = 2;
+  }
   return cfg;
 }
 
@@ -930,8 +941,8 @@ cudaError_t launch_splitk(const GemmArgs& a, const KernelCtl& ctl, cudaStream_t 
   use_b_blocks(a, GemmCfg<BN>::NB, &mb, &p);
   const long long ctas = static_cast<long long>(p.tiles_m) * p.tiles_n * S;
   if (ctas > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = splitk_config<BN>(static_cast<int>(ctas), S, stream, attr);
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = splitk_config<BN>(static_cast<int>(ctas), S, stream, attr, true);
   return cudaLaunchKernelEx(&cfg, gemm_splitk_kernel<BN, BKM>, ma, mb, p);
 }
 
