@@ -515,6 +515,8 @@ def measure(torch, wl, steps, warmup, stream, barrier, world, reduce_max, peaks,
     total_ms = reduce_max(total_ms)
     ms_per_step = total_ms / steps
     value = job_value(wl.value(ms_per_step * 1e-3), world)
+    # a launch's duration: the timed loop's duration per step (one launch per prefill
+    # step, the split and merge launches per decode step), gaps between launches included
     avg_launch_ms = statistics.mean(launch_ms) if launch_ms else ms_per_step
     if wl.unit == "TFLOP/s":
         achieved = wl.flops / (avg_launch_ms * 1e-3) / 1e12
